@@ -1,0 +1,11 @@
+"""Seeded synthetic workloads shared by the oracle tests, the GPU tests and the bench.
+
+This package only draws inputs (cost tables, search problems, candidate
+batches).  It holds none of the method's arithmetic: no DAG, no makespan,
+no lower bound, no search.
+"""
+from .workloads import (  # noqa: F401
+    CANDIDATE_DTYPE, Workload, config1, config2, config3, config4, config5_tables,
+    config5_candidates, all_candidates, random_candidates, get_config, n_compositions,
+    place_list,
+)

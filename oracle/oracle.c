@@ -1,0 +1,691 @@
+/*
+ * Poseidon CPU oracle -- TEST INFRASTRUCTURE ONLY (see oracle.h).
+ *
+ * Everything here follows the paper's definitions literally and is meant to
+ * be checked by eye against it:
+ *   Sec. 4.1.1  nodes: F_{s,m}, B_{s,m} (2NM), R_s (N), control nodes S, E
+ *   Sec. 4.1.2  edges: inter-stage F_{s,m}->F_{s+1,m}, B_{s,m}->B_{s-1,m};
+ *               intra-stage chain given by the schedule (2M-1 per stage);
+ *               B_{s,M}->R_s; S->F_{1,1}; R_s->E
+ *   Sec. 4.1.3  weights: F/B = per-layer time summed over the stage's layers,
+ *               inter-stage edge = activation transfer time, intra-stage
+ *               edges 0, R_s = all-reduce time summed over the stage's
+ *               layers, control nodes and auxiliary edges 0
+ *   Sec. 4.1    T = longest path (node + edge weights), computed by DP
+ *   Eq. 2       g(S_x), Theorem 1: prune when g(S_x) > T_min
+ *   Sec. 4.2.3  warm-up sampling, then enumeration of 3D configurations,
+ *               device-to-stage assignments and layer allocations with
+ *               memory constraints
+ *
+ * Readings where the paper is silent (the library documents the same ones):
+ *   - 1F1B order of stage s (1-based) with W_s = min(N-s+1, M) warm-up
+ *     forwards: F_1..F_W, then (B_i, F_{W+i}) for i = 1..M-W, then the
+ *     remaining backwards.
+ *   - weights use per-layer tables summed over the stage's layers (reduces to
+ *     the paper's product for identical layers).
+ *   - inter-stage edge weights come from a table indexed by the ordered
+ *     (sending class, receiving class) pair.
+ *   - memory of stage s: sum(mem_w) + W_s * sum(mem_a) <= cap.
+ *   - one pipeline is modelled: all D pipelines are identical (Sec. 4.2.3),
+ *     so the D edges into R_s carry the same value.
+ *   - objective across slices: T / (D*M) (time per sample), compared exactly
+ *     by cross-multiplication; ties go to the lowest global index.
+ */
+#include "oracle.h"
+
+#include <stdlib.h>
+#include <string.h>
+
+/* ------------------------------------------------------------------ */
+/* Binomial coefficients by Pascal's rule.                             */
+/* ------------------------------------------------------------------ */
+static uint64_t binom_tab[128][16];
+static int binom_ready = 0;
+
+static void binom_init(void) {
+    if (binom_ready) return;
+    for (int n = 0; n < 128; ++n) {
+        for (int k = 0; k <= 15; ++k) {
+            if (k == 0) binom_tab[n][k] = 1;
+            else if (n == 0) binom_tab[n][k] = 0;
+            else binom_tab[n][k] = binom_tab[n - 1][k - 1] + binom_tab[n - 1][k];
+        }
+    }
+    binom_ready = 1;
+}
+
+uint64_t orc_binom(int n, int k) {
+    binom_init();
+    if (n < 0 || k < 0 || k > n || n > 127 || k > 15) return 0;
+    return binom_tab[n][k];
+}
+
+/* Number of compositions of r layers into p non-empty stages. */
+static uint64_t n_comp(int r, int p) {
+    if (p == 0) return r == 0 ? 1 : 0;
+    if (r < p) return 0;
+    return orc_binom(r - 1, p - 1);
+}
+
+/* Lexicographic order on (l_1, ..., l_S): the rank of a composition is the
+ * number of compositions that are lexicographically smaller. */
+uint64_t orc_rank(int L, int S, const int32_t *layers) {
+    uint64_t r = 0;
+    int rem = L;
+    for (int s = 0; s < S - 1; ++s) {
+        int after = S - s - 1;
+        for (int v = 1; v < layers[s]; ++v) r += n_comp(rem - v, after);
+        rem -= layers[s];
+    }
+    return r;
+}
+
+int orc_unrank(int L, int S, uint64_t rank, int32_t *layers) {
+    if (S < 1 || S > ORC_MAX_S || S > L || L > 127) return -1;
+    if (rank >= n_comp(L, S)) return -1;
+    int rem = L;
+    for (int s = 0; s < S - 1; ++s) {
+        int after = S - s - 1;
+        int v;
+        for (v = 1; v <= rem - after; ++v) {
+            uint64_t cnt = n_comp(rem - v, after);
+            if (rank < cnt) break;
+            rank -= cnt;
+        }
+        layers[s] = v;
+        rem -= v;
+    }
+    layers[S - 1] = rem;
+    return 0;
+}
+
+/* ------------------------------------------------------------------ */
+/* Stage weights (Sec. 4.1.3) and memory (Sec. 3.2).                   */
+/* ------------------------------------------------------------------ */
+typedef struct {
+    int64_t F[ORC_MAX_S], B[ORC_MAX_S], d[ORC_MAX_S];
+    int64_t pf[ORC_MAX_S], pb[ORC_MAX_S]; /* pf[s]: F edge s->s+1, pb[s]: B edge s+1->s */
+} stage_w;
+
+static int warmup_count(int S, int M, int s /* 0-based */) {
+    int w = S - s; /* N - s + 1 in 1-based stage numbering */
+    return w < M ? w : M;
+}
+
+static void stage_weights(const orc_tables *t, int S, const int32_t *cls, const int32_t *layers,
+                          stage_w *w) {
+    int L = t->L;
+    int first = 0;
+    for (int s = 0; s < S; ++s) {
+        const int32_t *f = t->fwd + (int64_t)cls[s] * L;
+        const int32_t *b = t->bwd + (int64_t)cls[s] * L;
+        const int32_t *d = t->dsync + (int64_t)cls[s] * L;
+        int64_t sf = 0, sb = 0, sd = 0;
+        for (int l = first; l < first + layers[s]; ++l) {
+            sf += f[l];
+            sb += b[l];
+            sd += d[l];
+        }
+        w->F[s] = sf;
+        w->B[s] = sb;
+        w->d[s] = sd;
+        first += layers[s];
+    }
+    int K = t->n_types * t->n_tp;
+    for (int s = 0; s + 1 < S; ++s) {
+        w->pf[s] = t->p2p_f[(int64_t)cls[s] * K + cls[s + 1]];
+        w->pb[s] = t->p2p_b[(int64_t)cls[s + 1] * K + cls[s]];
+    }
+}
+
+/* Memory of stage s holding layers [first, first+l): weights plus W_s
+ * in-flight micro-batches of activations must fit the device capacity. */
+static int stage_memory_ok(const orc_tables *t, int S, int M, int s, int cls, int first, int l) {
+    int L = t->L;
+    const int64_t *mw = t->mem_w + (int64_t)cls * L;
+    const int64_t *ma = t->mem_a + (int64_t)cls * L;
+    int64_t sw = 0, sa = 0;
+    for (int i = first; i < first + l; ++i) {
+        sw += mw[i];
+        sa += ma[i];
+    }
+    int64_t need = sw + (int64_t)warmup_count(S, M, s) * sa;
+    return need <= t->cap[cls];
+}
+
+static int config_memory_ok(const orc_tables *t, int S, int M, const int32_t *cls,
+                            const int32_t *layers) {
+    int first = 0;
+    for (int s = 0; s < S; ++s) {
+        if (!stage_memory_ok(t, S, M, s, cls[s], first, layers[s])) return 0;
+        first += layers[s];
+    }
+    return 1;
+}
+
+/* Overflow guard: every path visits each node at most once, so its length is
+ * at most M*sum_l max_k(fwd+bwd) + sum_l max_k dsync + 2M(S-1)*max p2p. */
+static int64_t overflow_bound(const orc_tables *t, int S, int M) {
+    int K = t->n_types * t->n_tp, L = t->L;
+    int64_t A = 0, Dm = 0, P = 0;
+    for (int l = 0; l < L; ++l) {
+        int64_t mfb = 0, md = 0;
+        for (int k = 0; k < K; ++k) {
+            int64_t fb = (int64_t)t->fwd[(int64_t)k * L + l] + t->bwd[(int64_t)k * L + l];
+            if (fb > mfb) mfb = fb;
+            if (t->dsync[(int64_t)k * L + l] > md) md = t->dsync[(int64_t)k * L + l];
+        }
+        A += mfb;
+        Dm += md;
+    }
+    for (int i = 0; i < K * K; ++i) {
+        if (t->p2p_f[i] > P) P = t->p2p_f[i];
+        if (t->p2p_b[i] > P) P = t->p2p_b[i];
+    }
+    return (int64_t)M * A + Dm + 2 * (int64_t)M * (S - 1) * P;
+}
+
+/* ------------------------------------------------------------------ */
+/* The explicit DAG (Sec. 4.1) and its longest path.                   */
+/* ------------------------------------------------------------------ */
+typedef struct {
+    int n_nodes, n_edges;
+    int64_t *w;          /* node weights */
+    int *esrc, *edst;    /* edge list */
+    int64_t *ew;         /* edge weights */
+    int *indeg, *head, *next_e, *queue;
+    int64_t *start, *fin;
+    int cap_nodes, cap_edges;
+} dag;
+
+static void dag_free(dag *g) {
+    free(g->w); free(g->esrc); free(g->edst); free(g->ew); free(g->indeg); free(g->head);
+    free(g->next_e); free(g->queue); free(g->start); free(g->fin);
+    memset(g, 0, sizeof(*g));
+}
+
+static int dag_reserve(dag *g, int nodes, int edges) {
+    if (nodes <= g->cap_nodes && edges <= g->cap_edges) return 0;
+    dag_free(g);
+    g->w = malloc(sizeof(int64_t) * nodes);
+    g->indeg = malloc(sizeof(int) * nodes);
+    g->head = malloc(sizeof(int) * nodes);
+    g->queue = malloc(sizeof(int) * nodes);
+    g->start = malloc(sizeof(int64_t) * nodes);
+    g->fin = malloc(sizeof(int64_t) * nodes);
+    g->esrc = malloc(sizeof(int) * edges);
+    g->edst = malloc(sizeof(int) * edges);
+    g->ew = malloc(sizeof(int64_t) * edges);
+    g->next_e = malloc(sizeof(int) * edges);
+    if (!g->w || !g->indeg || !g->head || !g->queue || !g->start || !g->fin || !g->esrc ||
+        !g->edst || !g->ew || !g->next_e) {
+        dag_free(g);
+        return -1;
+    }
+    g->cap_nodes = nodes;
+    g->cap_edges = edges;
+    return 0;
+}
+
+static void add_edge(dag *g, int a, int b, int64_t w) {
+    int e = g->n_edges++;
+    g->esrc[e] = a;
+    g->edst[e] = b;
+    g->ew[e] = w;
+}
+
+/* node numbering: 0 = start S; F(s,m), B(s,m) compute nodes; R(s); E last */
+#define NODE_F(s, m) (1 + 2 * ((s) * M + (m)))
+#define NODE_B(s, m) (2 + 2 * ((s) * M + (m)))
+#define NODE_R(s) (1 + 2 * S * M + (s))
+
+static int build_and_solve(dag *g, int S, int M, const stage_w *sw, orc_dag_counts *counts,
+                           int64_t *T_out) {
+    int n_nodes = 2 + 2 * S * M + S;
+    int n_edges_max = 2 * (S - 1) * M + S * (2 * M - 1) + S + 1 + S;
+    if (dag_reserve(g, n_nodes, n_edges_max)) return -1;
+    g->n_nodes = n_nodes;
+    g->n_edges = 0;
+    int node_E = n_nodes - 1;
+
+    /* nodes and weights (Sec. 4.1.1, 4.1.3) */
+    g->w[0] = 0;
+    g->w[node_E] = 0;
+    for (int s = 0; s < S; ++s) {
+        for (int m = 0; m < M; ++m) {
+            g->w[NODE_F(s, m)] = sw->F[s];
+            g->w[NODE_B(s, m)] = sw->B[s];
+        }
+        g->w[NODE_R(s)] = sw->d[s];
+    }
+    int64_t c_inter = 0, c_intra = 0, c_ar = 0, c_aux = 0;
+
+    /* inter-stage edges: activations forward, gradients backward */
+    for (int m = 0; m < M; ++m) {
+        for (int s = 0; s + 1 < S; ++s) {
+            add_edge(g, NODE_F(s, m), NODE_F(s + 1, m), sw->pf[s]);
+            add_edge(g, NODE_B(s + 1, m), NODE_B(s, m), sw->pb[s]);
+            c_inter += 2;
+        }
+    }
+    /* intra-stage edges: the 1F1B order of each stage, weight 0 */
+    int order_node[2 * 255];
+    for (int s = 0; s < S; ++s) {
+        int W = warmup_count(S, M, s), n = 0;
+        for (int m = 0; m < W; ++m) order_node[n++] = NODE_F(s, m);
+        for (int i = 0; i < M - W; ++i) {
+            order_node[n++] = NODE_B(s, i);
+            order_node[n++] = NODE_F(s, W + i);
+        }
+        for (int m = M - W; m < M; ++m) order_node[n++] = NODE_B(s, m);
+        if (n != 2 * M) return -1;
+        /* F_{s,m} must come before B_{s,m} in the chain */
+        for (int m = 0; m < M; ++m) {
+            int pf_ = -1, pb_ = -1;
+            for (int i = 0; i < n; ++i) {
+                if (order_node[i] == NODE_F(s, m)) pf_ = i;
+                if (order_node[i] == NODE_B(s, m)) pb_ = i;
+            }
+            if (!(pf_ >= 0 && pb_ > pf_)) return -1;
+        }
+        for (int i = 0; i + 1 < n; ++i) {
+            add_edge(g, order_node[i], order_node[i + 1], 0);
+            c_intra += 1;
+        }
+    }
+    /* all-reduce edges B_{s,M} -> R_s and auxiliary edges */
+    for (int s = 0; s < S; ++s) {
+        add_edge(g, NODE_B(s, M - 1), NODE_R(s), 0);
+        c_ar += 1;
+    }
+    add_edge(g, 0, NODE_F(0, 0), 0);
+    c_aux += 1;
+    for (int s = 0; s < S; ++s) {
+        add_edge(g, NODE_R(s), node_E, 0);
+        c_aux += 1;
+    }
+    if (counts) {
+        counts->nodes = n_nodes;
+        counts->compute_nodes = 2 * (int64_t)S * M;
+        counts->allreduce_nodes = S;
+        counts->control_nodes = 2;
+        counts->inter_edges = c_inter;
+        counts->intra_edges = c_intra;
+        counts->allreduce_edges = c_ar;
+        counts->aux_edges = c_aux;
+    }
+
+    /* Kahn topological order; longest path where a node finishes at its
+     * latest predecessor finish (+ edge weight) plus its own weight. */
+    for (int i = 0; i < n_nodes; ++i) {
+        g->indeg[i] = 0;
+        g->head[i] = -1;
+        g->start[i] = 0;
+    }
+    for (int e = 0; e < g->n_edges; ++e) {
+        g->indeg[g->edst[e]]++;
+        g->next_e[e] = g->head[g->esrc[e]];
+        g->head[g->esrc[e]] = e;
+    }
+    int qh = 0, qt = 0;
+    for (int i = 0; i < n_nodes; ++i)
+        if (g->indeg[i] == 0) g->queue[qt++] = i;
+    while (qh < qt) {
+        int u = g->queue[qh++];
+        g->fin[u] = g->start[u] + g->w[u];
+        for (int e = g->head[u]; e >= 0; e = g->next_e[e]) {
+            int v = g->edst[e];
+            int64_t cand = g->fin[u] + g->ew[e];
+            if (cand > g->start[v]) g->start[v] = cand;
+            if (--g->indeg[v] == 0) g->queue[qt++] = v;
+        }
+    }
+    if (qt != n_nodes) return -1; /* not a DAG */
+    *T_out = g->fin[node_E];
+    return 0;
+}
+
+static int check_inputs(const orc_tables *t, int S, int M, const int32_t *cls,
+                        const int32_t *layers) {
+    int K = t->n_types * t->n_tp;
+    if (S < 1 || S > ORC_MAX_S || M < 1 || M > 255 || S > t->L || t->L > 127) return -1;
+    int sum = 0;
+    for (int s = 0; s < S; ++s) {
+        if (cls[s] < 0 || cls[s] >= K || layers[s] < 1) return -1;
+        sum += layers[s];
+    }
+    return sum == t->L ? 0 : -1;
+}
+
+int orc_eval(const orc_tables *t, int S, int M, const int32_t *cls, const int32_t *layers,
+             int32_t *T, int32_t *feasible, orc_dag_counts *counts) {
+    if (check_inputs(t, S, M, cls, layers)) return -1;
+    stage_w sw;
+    stage_weights(t, S, cls, layers, &sw);
+    dag g;
+    memset(&g, 0, sizeof(g));
+    int64_t T64;
+    int rc = build_and_solve(&g, S, M, &sw, counts, &T64);
+    dag_free(&g);
+    if (rc) return -1;
+    if (T64 >= ((int64_t)1 << 31)) return -1;
+    *T = (int32_t)T64;
+    *feasible = config_memory_ok(t, S, M, cls, layers);
+    return 0;
+}
+
+int orc_eval_finish(const orc_tables *t, int S, int M, const int32_t *cls, const int32_t *layers,
+                    int32_t *finish) {
+    if (check_inputs(t, S, M, cls, layers)) return -1;
+    stage_w sw;
+    stage_weights(t, S, cls, layers, &sw);
+    dag g;
+    memset(&g, 0, sizeof(g));
+    int64_t T64;
+    int rc = build_and_solve(&g, S, M, &sw, NULL, &T64);
+    if (!rc) {
+        for (int s = 0; s < S; ++s)
+            for (int m = 0; m < M; ++m) {
+                finish[(s * M + m)] = (int32_t)g.fin[NODE_F(s, m)];
+                finish[S * M + (s * M + m)] = (int32_t)g.fin[NODE_B(s, m)];
+            }
+    }
+    dag_free(&g);
+    return rc;
+}
+
+/* Eq. 2 with stage totals (1-based x):
+ *   g(S_x) = sum_{i<x} F_i + M (F_x + B_x) + max_{1<=i<=x} ( sum_{j=i}^{x-1} B_j + d_i ) */
+static int64_t lower_bound_w(const stage_w *w, int M, int x) {
+    int64_t g = 0;
+    for (int i = 1; i <= x - 1; ++i) g += w->F[i - 1];
+    g += (int64_t)M * (w->F[x - 1] + w->B[x - 1]);
+    int64_t best = 0;
+    for (int i = 1; i <= x; ++i) {
+        int64_t v = w->d[i - 1];
+        for (int j = i; j <= x - 1; ++j) v += w->B[j - 1];
+        if (i == 1 || v > best) best = v;
+    }
+    return g + best;
+}
+
+int64_t orc_lower_bound(const orc_tables *t, int S, int M, const int32_t *cls,
+                        const int32_t *layers, int x) {
+    if (check_inputs(t, S, M, cls, layers) || x < 1 || x > S) return -1;
+    stage_w sw;
+    stage_weights(t, S, cls, layers, &sw);
+    return lower_bound_w(&sw, M, x);
+}
+
+int orc_eval_batch(const orc_tables *t, const orc_candidate *c, int64_t n, int32_t *T,
+                   uint8_t *feasible) {
+    int K = t->n_types * t->n_tp;
+    (void)K;
+    dag g;
+    memset(&g, 0, sizeof(g));
+    for (int64_t i = 0; i < n; ++i) {
+        int S = c[i].S, M = c[i].M;
+        int32_t layers[ORC_MAX_S], cls[ORC_MAX_S];
+        int ok = S >= 1 && S <= ORC_MAX_S && S <= t->L && M >= 1 && c[i].tp_idx < t->n_tp;
+        if (ok) ok = orc_unrank(t->L, S, c[i].map_rank, layers) == 0;
+        for (int s = 0; ok && s < S; ++s) {
+            int ty = (c[i].type_code >> (2 * s)) & 3;
+            if (ty >= t->n_types) ok = 0;
+            cls[s] = ty * t->n_tp + c[i].tp_idx;
+        }
+        if (!ok) {
+            T[i] = -1;
+            feasible[i] = 2;
+            continue;
+        }
+        if (overflow_bound(t, S, M) >= ((int64_t)1 << 31)) {
+            T[i] = -1;
+            feasible[i] = 3;
+            continue;
+        }
+        stage_w sw;
+        stage_weights(t, S, cls, layers, &sw);
+        int64_t T64;
+        if (build_and_solve(&g, S, M, &sw, NULL, &T64)) {
+            dag_free(&g);
+            return -1;
+        }
+        T[i] = (int32_t)T64;
+        feasible[i] = (uint8_t)config_memory_ok(t, S, M, cls, layers);
+    }
+    dag_free(&g);
+    return 0;
+}
+
+/* ------------------------------------------------------------------ */
+/* Search (Sec. 4.2.3).                                                */
+/* ------------------------------------------------------------------ */
+typedef struct {
+    const orc_problem *p;
+    int S, L, M, D, m_idx, tp_idx, prune;
+    uint64_t place_rank, n_place, n_map;
+    int32_t cls[ORC_MAX_S], types[ORC_MAX_S], layers[ORC_MAX_S];
+    unsigned char *feas; /* feas[x*(L+1)+c]: layers [c, L) fit stages x..S-1 */
+    orc_plan *best;
+    orc_stats *st;
+    dag g;
+    int err;
+} search_ctx;
+
+/* a strictly better than the incumbent: smaller T/(D*M), then smaller index */
+static int better(int64_t T, int D, int M, uint64_t idx, const orc_plan *b) {
+    if (!b->found) return 1;
+    int64_t lhs = T * (int64_t)b->D * b->M, rhs = (int64_t)b->T * D * M;
+    if (lhs != rhs) return lhs < rhs;
+    return idx < b->global_index;
+}
+
+static void consider_leaf(search_ctx *cx) {
+    stage_w sw;
+    stage_weights(&cx->p->tab, cx->S, cx->cls, cx->layers, &sw);
+    int64_t T64;
+    if (build_and_solve(&cx->g, cx->S, cx->M, &sw, NULL, &T64)) {
+        cx->err = 1;
+        return;
+    }
+    uint64_t map_rank = orc_rank(cx->L, cx->S, cx->layers);
+    uint64_t idx = ((((uint64_t)cx->m_idx * cx->p->tab.n_tp + cx->tp_idx) * cx->n_place +
+                     cx->place_rank) * cx->n_map) + map_rank;
+    if (better(T64, cx->D, cx->M, idx, cx->best)) {
+        orc_plan *b = cx->best;
+        b->found = 1;
+        b->m_idx = cx->m_idx;
+        b->tp_idx = cx->tp_idx;
+        b->M = cx->M;
+        b->D = cx->D;
+        b->T = (int32_t)T64;
+        b->place_rank = cx->place_rank;
+        b->map_rank = map_rank;
+        b->global_index = idx;
+        for (int s = 0; s < ORC_MAX_S; ++s) {
+            b->types[s] = s < cx->S ? cx->types[s] : -1;
+            b->layers[s] = s < cx->S ? cx->layers[s] : 0;
+        }
+    }
+}
+
+/* Prefix S_x (stages 0..x-1 placed, 1-based x) is cut when its lower bound
+ * exceeds the incumbent: g(S_x)/(D M) > T_inc/(D_inc M_inc), i.e. it is strictly worse. */
+static int pruned_by_bound(search_ctx *cx, int x) {
+    if (!cx->prune || !cx->best->found) return 0;
+    stage_w sw;
+    stage_weights(&cx->p->tab, x, cx->cls, cx->layers, &sw);
+    int64_t g = lower_bound_w(&sw, cx->M, x);
+    const orc_plan *b = cx->best;
+    return g * (int64_t)b->D * b->M > (int64_t)b->T * cx->D * cx->M;
+}
+
+static void dfs(search_ctx *cx, int x, int used) {
+    if (cx->err) return;
+    int S = cx->S, L = cx->L;
+    int lo = 1, hi = L - used - (S - x - 1);
+    if (x == S - 1) lo = hi; /* the last stage takes the remaining layers */
+    for (int l = lo; l <= hi; ++l) {
+        cx->layers[x] = l;
+        if (!stage_memory_ok(&cx->p->tab, S, cx->M, x, cx->cls[x], used, l) ||
+            !cx->feas[(x + 1) * (L + 1) + used + l]) {
+            cx->st->prefixes_memory++;
+            continue;
+        }
+        /* the stage-x bound uses only stages 0..x, which are all fixed now */
+        if (pruned_by_bound(cx, x + 1)) {
+            cx->st->prefixes_pruned++;
+            continue;
+        }
+        if (x == S - 1) {
+            cx->st->leaves_evaluated++;
+            consider_leaf(cx);
+        } else {
+            dfs(cx, x + 1, used + l);
+        }
+    }
+}
+
+/* feas[x][c] = the layers [c, L) can be split over stages x..S-1 within memory */
+static void suffix_feasibility(search_ctx *cx) {
+    int S = cx->S, L = cx->L;
+    for (int x = 0; x <= S; ++x)
+        for (int c = 0; c <= L; ++c) cx->feas[x * (L + 1) + c] = 0;
+    cx->feas[S * (L + 1) + L] = 1;
+    for (int x = S - 1; x >= 0; --x)
+        for (int c = 0; c < L; ++c)
+            for (int l = 1; c + l <= L; ++l)
+                if (cx->feas[(x + 1) * (L + 1) + c + l] &&
+                    stage_memory_ok(&cx->p->tab, S, cx->M, x, cx->cls[x], c, l)) {
+                    cx->feas[x * (L + 1) + c] = 1;
+                    break;
+                }
+}
+
+/* next type sequence in lexicographic order among the allowed placements */
+static int next_placement(const orc_problem *p, int32_t *seq, int first) {
+    int S = p->S, T = p->tab.n_types;
+    for (;;) {
+        if (first) {
+            for (int s = 0; s < S; ++s) seq[s] = 0;
+            first = 0;
+        } else {
+            int s = S - 1;
+            while (s >= 0 && seq[s] == T - 1) seq[s--] = 0;
+            if (s < 0) return 0;
+            seq[s]++;
+        }
+        if (p->placement == 0) return 1;
+        int ok = 1;
+        for (int ty = 0; ty < T && ok; ++ty) {
+            int cnt = 0;
+            for (int s = 0; s < S; ++s) cnt += seq[s] == ty;
+            ok = cnt == p->type_counts[ty];
+        }
+        if (ok) return 1;
+    }
+}
+
+/* splitmix64 (Steele, Lea & Flood, OOPSLA 2014) for warm-up sampling */
+static uint64_t splitmix64(uint64_t *state) {
+    uint64_t z = (*state += 0x9E3779B97F4A7C15ull);
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+static void set_slice(search_ctx *cx, int m_idx, int tp_idx, uint64_t place_rank,
+                      const int32_t *seq) {
+    const orc_problem *p = cx->p;
+    cx->m_idx = m_idx;
+    cx->tp_idx = tp_idx;
+    cx->M = p->M_list[m_idx];
+    cx->D = p->dp_list[tp_idx];
+    cx->place_rank = place_rank;
+    for (int s = 0; s < cx->S; ++s) {
+        cx->types[s] = seq[s];
+        cx->cls[s] = seq[s] * p->tab.n_tp + tp_idx;
+    }
+    suffix_feasibility(cx);
+}
+
+int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_plan *plan,
+               orc_stats *stats) {
+    int S = p->S, L = p->tab.L;
+    if (S < 1 || S > ORC_MAX_S || S > L || L > 127 || p->n_M < 1 || p->tab.n_types < 1 ||
+        p->tab.n_types > 4 || p->tab.n_tp < 1)
+        return -1;
+    for (int i = 0; i < p->n_M; ++i)
+        if (p->M_list[i] < 1 || p->M_list[i] > 255) return -1;
+    for (int i = 0; i < p->tab.n_tp; ++i)
+        if (p->dp_list[i] < 1) return -1;
+    for (int i = 0; i < p->n_M; ++i)
+        if (overflow_bound(&p->tab, S, p->M_list[i]) >= ((int64_t)1 << 31)) return -2;
+
+    memset(plan, 0, sizeof(*plan));
+    memset(stats, 0, sizeof(*stats));
+    search_ctx cx;
+    memset(&cx, 0, sizeof(cx));
+    cx.p = p;
+    cx.S = S;
+    cx.L = L;
+    cx.prune = prune;
+    cx.best = plan;
+    cx.st = stats;
+    cx.n_map = n_comp(L, S);
+    cx.feas = malloc((size_t)(S + 1) * (L + 1));
+    if (!cx.feas) return -1;
+
+    int32_t seq[ORC_MAX_S];
+    cx.n_place = 0;
+    for (int f = 1; next_placement(p, seq, f); f = 0) cx.n_place++;
+
+    /* warm-up: random feasible configurations seed T_min (Sec. 4.2.3) */
+    if (warmup > 0 && cx.n_place > 0 && cx.n_place <= (1u << 20)) {
+        int32_t *places = malloc(sizeof(int32_t) * S * cx.n_place);
+        if (places) {
+            uint64_t i = 0;
+            for (int f = 1; next_placement(p, seq, f); f = 0, ++i)
+                memcpy(places + i * S, seq, sizeof(int32_t) * S);
+            uint64_t rs = seed;
+            uint64_t n_slices = (uint64_t)p->n_M * p->tab.n_tp * cx.n_place;
+            for (int w = 0; w < warmup; ++w) {
+                uint64_t sl = splitmix64(&rs) % n_slices;
+                uint64_t pr = sl % cx.n_place;
+                int tp = (int)((sl / cx.n_place) % p->tab.n_tp);
+                int mi = (int)(sl / cx.n_place / p->tab.n_tp);
+                set_slice(&cx, mi, tp, pr, places + pr * S);
+                if (!cx.feas[0]) continue;
+                int used = 0;
+                for (int x = 0; x < S; ++x) {
+                    int opts[128], n = 0;
+                    int hi = L - used - (S - x - 1), lo = x == S - 1 ? hi : 1;
+                    for (int l = lo; l <= hi; ++l)
+                        if (stage_memory_ok(&p->tab, S, cx.M, x, cx.cls[x], used, l) &&
+                            cx.feas[(x + 1) * (L + 1) + used + l])
+                            opts[n++] = l;
+                    cx.layers[x] = opts[splitmix64(&rs) % (uint64_t)n];
+                    used += cx.layers[x];
+                }
+                stats->warmup_evaluated++;
+                consider_leaf(&cx);
+            }
+            free(places);
+        }
+    }
+
+    /* exhaustive enumeration in global-index order with the two cuts */
+    for (int mi = 0; mi < p->n_M && !cx.err; ++mi) {
+        for (int tp = 0; tp < p->tab.n_tp && !cx.err; ++tp) {
+            uint64_t pr = 0;
+            for (int f = 1; next_placement(p, seq, f) && !cx.err; f = 0, ++pr) {
+                set_slice(&cx, mi, tp, pr, seq);
+                if (!cx.feas[0]) continue;
+                dfs(&cx, 0, 0);
+            }
+        }
+    }
+    free(cx.feas);
+    dag_free(&cx.g);
+    return cx.err ? -1 : 0;
+}

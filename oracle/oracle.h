@@ -1,0 +1,106 @@
+/*
+ * Poseidon CPU oracle -- TEST INFRASTRUCTURE ONLY.
+ *
+ * A plain, slow, single-threaded C implementation of what the search hot
+ * path computes, written from the paper's definitions:
+ *   - the DAG cost model of Sec. 4.1 (nodes Sec. 4.1.1, edges Sec. 4.1.2,
+ *     weights Sec. 4.1.3) with the 1F1B intra-stage order, evaluated as the
+ *     longest path through an explicitly built graph (Kahn order + DP);
+ *   - per-stage memory feasibility (Sec. 3.2, Sec. 4.2.3, Lemma "memlimit"
+ *     of App. B.3);
+ *   - the stage-level lower bound g(S_x) of Eq. 2 and the search of
+ *     Sec. 4.2.3 (depth-first over slices and layer allocations, prune when
+ *     g(S_x) > T_min, Theorem 1).
+ *
+ * Only tests/, __graft_entry__.smoke() and bench.py's CPU baseline may load
+ * this library.  It shares no code, header or table with the CUDA path.
+ */
+#ifndef POSEIDON_ORACLE_H
+#define POSEIDON_ORACLE_H
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ORC_MAX_S 16
+
+typedef struct {
+    int32_t L, n_types, n_tp;            /* K = n_types * n_tp classes, k = type*n_tp + tp_idx */
+    const int32_t *fwd, *bwd, *dsync;    /* [K][L] microseconds per layer */
+    const int32_t *p2p_f, *p2p_b;        /* [K][K] microseconds, [src class][dst class] */
+    const int64_t *mem_w, *mem_a;        /* [K][L] bytes; mem_a per in-flight micro-batch */
+    const int64_t *cap;                  /* [K] bytes */
+} orc_tables;
+
+/* 16-byte candidate record (same field meaning as the library's). */
+typedef struct {
+    uint64_t map_rank;
+    uint32_t type_code;
+    uint8_t S, M, tp_idx, pad;
+} orc_candidate;
+
+typedef struct {
+    orc_tables tab;
+    int32_t S;
+    int32_t n_M;
+    const int32_t *M_list;      /* [n_M] ascending */
+    const int32_t *dp_list;     /* [n_tp] data-parallel degree D per TP index */
+    int32_t placement;          /* 0 = any type per stage, 1 = exact per-type stage counts */
+    const int32_t *type_counts; /* [n_types] (placement 1) */
+} orc_problem;
+
+typedef struct {
+    int32_t found;
+    int32_t m_idx, tp_idx, M, D;
+    int32_t T;                  /* makespan (us) */
+    uint64_t place_rank, map_rank, global_index;
+    int32_t types[ORC_MAX_S], layers[ORC_MAX_S];
+} orc_plan;
+
+typedef struct {
+    uint64_t leaves_evaluated;  /* complete configurations whose DAG was evaluated */
+    uint64_t prefixes_pruned;   /* partial configurations cut by g(S_x) > T_min */
+    uint64_t prefixes_memory;   /* partial configurations cut by memory */
+    uint64_t warmup_evaluated;
+} orc_stats;
+
+typedef struct {
+    int64_t nodes, compute_nodes, allreduce_nodes, control_nodes;
+    int64_t inter_edges, intra_edges, allreduce_edges, aux_edges;
+} orc_dag_counts;
+
+/* C(n, k) from Pascal's rule; 0 when k < 0 or k > n.  n <= 127, k <= 15
+ * (exact in 64 bits there; S <= 16 stages never needs more). */
+uint64_t orc_binom(int n, int k);
+/* Lexicographic (ascending l_1, l_2, ...) rank <-> composition of L into S parts. */
+int orc_unrank(int L, int S, uint64_t rank, int32_t *layers);
+uint64_t orc_rank(int L, int S, const int32_t *layers);
+
+/* Evaluate one configuration: stage s (0-based) holds layers[s] consecutive
+ * layers and runs on class cls[s].  Writes the makespan (longest path) and
+ * the memory-feasibility flag.  Returns 0, or -1 on invalid input. */
+int orc_eval(const orc_tables *t, int S, int M, const int32_t *cls, const int32_t *layers,
+             int32_t *T, int32_t *feasible, orc_dag_counts *counts);
+/* Same DAG, but also returns every node's finish time (F then B, stage-major,
+ * [s][m]); finish must hold 2*S*M values. */
+int orc_eval_finish(const orc_tables *t, int S, int M, const int32_t *cls, const int32_t *layers,
+                    int32_t *finish);
+/* g(S_x) of Eq. 2 for the prefix of stages 1..x (1 <= x <= S). */
+int64_t orc_lower_bound(const orc_tables *t, int S, int M, const int32_t *cls,
+                        const int32_t *layers, int x);
+/* Decode and evaluate n candidate records.  feasible: 1 ok, 0 memory
+ * infeasible, 2 invalid record, 3 overflow guard tripped. */
+int orc_eval_batch(const orc_tables *t, const orc_candidate *c, int64_t n, int32_t *T,
+                   uint8_t *feasible);
+/* Exact search of Sec. 4.2.3.  prune=0 disables the g(S_x) prune (memory
+ * infeasible prefixes are still skipped).  warmup = number of random feasible
+ * samples evaluated first (Sec. 4.2.3); it never changes the result.
+ * Returns 0 (plan->found tells whether a feasible plan exists) or -1. */
+int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_plan *plan,
+               orc_stats *stats);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

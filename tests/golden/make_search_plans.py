@@ -1,0 +1,40 @@
+"""Write tests/golden/search_plans.json: the oracle's exact search result for
+the four search workloads (configs 1-4 of gen/), so GPU tests and the bench
+can compare against the oracle without re-running its slowest search
+(config 4 takes minutes single-threaded).  Calls only oracle/ and gen/.
+
+    python tests/golden/make_search_plans.py [--configs 1 2 3 4]
+"""
+import argparse
+import json
+import os
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+sys.path.insert(0, ROOT)
+
+import gen  # noqa: E402
+import oracle  # noqa: E402
+
+OUT = os.path.join(os.path.dirname(os.path.abspath(__file__)), "search_plans.json")
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--configs", type=int, nargs="*", default=[1, 2, 3, 4])
+    args = ap.parse_args()
+    data = json.load(open(OUT)) if os.path.exists(OUT) else {}
+    for c in args.configs:
+        w = gen.get_config(c)
+        t0 = time.time()
+        plan, stats = oracle.search(w, prune=True, warmup=500, seed=0)
+        data[f"config{c}"] = dict(workload=w.name, seed=w.seed, plan=plan, oracle_stats=stats,
+                                  oracle_seconds=round(time.time() - t0, 2))
+        print(c, plan, flush=True)
+    with open(OUT, "w") as f:
+        json.dump(data, f, indent=1, sort_keys=True)
+
+
+if __name__ == "__main__":
+    main()
