@@ -1,0 +1,211 @@
+/*
+ * poseidon.h -- C ABI of libposeidon.so: batched evaluation of Poseidon's
+ * DAG training-time model and the exact parallelism search built on it,
+ * on one GB300 (sm_103a).
+ *
+ * Model (paper Sec. 4.1): for a pipeline of N = S stages and M micro-batches
+ * the DAG has nodes F_{s,m}, B_{s,m} (Sec. 4.1.1), inter-stage edges
+ * F_{s,m} -> F_{s+1,m} and B_{s+1,m} -> B_{s,m}, an intra-stage chain in 1F1B
+ * order, B_{s,M} -> R_s and R_s -> E (Sec. 4.1.2).  Node weights are the
+ * per-layer times summed over the stage's layers, inter-stage edges carry the
+ * activation-transfer time, R_s the gradient all-reduce time (Sec. 4.1.3).
+ * The makespan T is the longest path: T = max_s (finish(B_{s,M}) + d_s).
+ *
+ * Conventions shared by every entry point:
+ *  - every call returns a pos_status; no C++ exception crosses the ABI;
+ *    poseidon_last_error() describes the last failure of the calling thread;
+ *  - the caller owns every buffer it passes; the library copies what it keeps;
+ *  - costs are int32 microseconds, memory int64 bytes; all arithmetic is
+ *    integer, so results are exact and reproducible;
+ *  - class k = type * n_tp + tp_idx indexes every per-class table.
+ */
+#ifndef POSEIDON_H
+#define POSEIDON_H
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t pos_status;
+#define POS_OK 0
+#define POS_EINVAL 1        /* bad argument, table or problem */
+#define POS_EOVERFLOW 2     /* a makespan could exceed int32 (guard below) */
+#define POS_ENOMEM 3        /* device or host allocation failed */
+#define POS_ECUDA 4         /* a CUDA runtime call failed */
+#define POS_ETIMEOUT 5      /* a bounded device loop hit its iteration limit */
+#define POS_EINFEASIBLE 6   /* the search space has no memory-feasible plan */
+#define POS_ENOTIMPL 7
+
+#define POS_SCHED_1F1B 0    /* the only schedule implemented */
+
+#define POS_PLACE_FREE 0    /* any device type on any stage */
+#define POS_PLACE_EXACT 1   /* exactly type_counts[t] stages of type t */
+
+#define POS_MAX_STAGES 16
+#define POS_MAX_LAYERS 127
+#define POS_MAX_TYPES 4
+#define POS_MAX_TP 8
+
+/*
+ * Profiled cost tables (Sec. 3.2 and Sec. 4.1.3), host pointers, row-major:
+ *   fwd, bwd, dsync [K][L]   per-layer forward, backward and DP all-reduce
+ *                            time in us (>= 0);
+ *   p2p_f, p2p_b    [K][K]   activation / gradient transfer time per
+ *                            micro-batch, indexed [sending class][receiving
+ *                            class]; the F edge s->s+1 uses p2p_f[k_s][k_s+1],
+ *                            the B edge s+1->s uses p2p_b[k_s+1][k_s];
+ *   mem_w, mem_a    [K][L]   bytes per layer: resident (weights, optimizer)
+ *                            and activations per in-flight micro-batch (>= 0);
+ *   cap             [K]      device memory per class, bytes.
+ * A stage s (1-based) holding layers [a, b) on class k fits when
+ *   sum mem_w + W_s * sum mem_a <= cap[k],   W_s = min(S - s + 1, M),
+ * W_s being the 1F1B in-flight micro-batches of that stage.
+ * Limits: 1 <= L <= 127, 1 <= n_types <= 4, 1 <= n_tp <= 8, and per class
+ * sum_l (fwd + bwd) and sum_l dsync below 2^31.
+ */
+typedef struct pos_tables {
+    int32_t L, n_types, n_tp;
+    const int32_t *fwd, *bwd, *dsync;
+    const int32_t *p2p_f, *p2p_b;
+    const int64_t *mem_w, *mem_a;
+    const int64_t *cap;
+} pos_tables;
+
+/*
+ * One encoded candidate plan, 16 bytes:
+ *   map_rank   lexicographic rank of the layer composition (l_1..l_S) among
+ *              all C(L-1, S-1) compositions of L into S non-empty stages;
+ *              rank 0 = (1, ..., 1, L-S+1);
+ *   type_code  device type of stage s (0-based) in bits [2s, 2s+2);
+ *   S          stages (1..16), M micro-batches (1..255), tp_idx < n_tp.
+ */
+typedef struct pos_candidate {
+    uint64_t map_rank;
+    uint32_t type_code;
+    uint8_t S, M, tp_idx, pad;
+} pos_candidate;
+
+/* feasible[] codes written by poseidon_eval_batch */
+#define POS_FEAS_NO 0        /* some stage exceeds its memory capacity */
+#define POS_FEAS_YES 1
+#define POS_FEAS_INVALID 2   /* a field is out of range; makespan = -1 */
+#define POS_FEAS_OVERFLOW 3  /* guard U(S,M) >= 2^31; makespan = -1 */
+
+/*
+ * Overflow guard: every DAG path visits each node once, so
+ *   T <= U(S,M) = M * sum_l max_k (fwd + bwd) + sum_l max_k dsync
+ *                 + 2 M (S-1) max_{k,k'} max(p2p_f, p2p_b).
+ * Candidates with U(S,M) >= 2^31 are not evaluated.
+ */
+
+/*
+ * Copy the tables to the current CUDA device and build the per-class
+ * exclusive prefix sums used by every kernel (hot-path step a1, Sec. 4.1.3).
+ * *handle owns the device copies until poseidon_tables_destroy.  schedule
+ * must be POS_SCHED_1F1B.
+ * Errors: POS_EINVAL (null pointer, limits, negative cost or memory),
+ * POS_EOVERFLOW (a class's summed costs reach 2^31), POS_ENOTIMPL (schedule),
+ * POS_ENOMEM, POS_ECUDA.
+ */
+pos_status poseidon_tables_create(const pos_tables *tables, int32_t schedule, void **handle);
+pos_status poseidon_tables_destroy(void *handle);
+
+/*
+ * Evaluate n candidates: makespan (Sec. 4.1) and memory feasibility
+ * (Sec. 3.2).  d_cands (16-byte aligned), d_makespan (int32[n]) and
+ * d_feasible (uint8[n]) are DEVICE pointers on the handle's device; outputs
+ * are in input order; the call is asynchronous on `stream` (a cudaStream_t,
+ * NULL = legacy default stream) and returns after the launches.  Infeasible
+ * plans still get their makespan.  No global scratch memory is used.
+ * Errors: POS_EINVAL (null handle or pointers, n < 0, misaligned
+ * candidates), POS_ECUDA (launch failure).
+ */
+pos_status poseidon_eval_batch(void *handle, const pos_candidate *d_cands, int64_t n,
+                               int32_t *d_makespan, uint8_t *d_feasible, void *stream);
+
+/*
+ * Same as poseidon_eval_batch but with HOST buffers: copies the candidates
+ * to the device, evaluates, copies the results back and synchronises.
+ * Allocates n*21 bytes of device memory for the duration of the call.
+ */
+pos_status poseidon_eval_batch_host(void *handle, const pos_candidate *cands, int64_t n,
+                                    int32_t *makespan, uint8_t *feasible);
+
+/*
+ * Deterministic argmin over eval_batch outputs (hot-path step a9): the
+ * smallest makespan among entries with feasible == 1, ties broken to the
+ * lowest index.  Device pointers; *d_out (int64, device) receives the index
+ * or -1 when no entry is feasible.  Asynchronous on `stream`; uses a
+ * stream-ordered scratch allocation of at most 16 bytes per SM * 4.
+ */
+pos_status poseidon_argmin(const int32_t *d_makespan, const uint8_t *d_feasible, int64_t n,
+                           int64_t *d_out, void *stream);
+
+/*
+ * Search problem (Sec. 4.2.3): choose M from M_list, a TP index, a
+ * device-type-to-stage placement and a layer composition for S stages.
+ * Slices are (m_idx, tp_idx, placement) in this nesting order; placements
+ * are the allowed type sequences in lexicographic order.  Global index of a
+ * plan = (((m_idx*n_tp + tp_idx)*n_place + place_rank)*n_map + map_rank),
+ * n_map = C(L-1, S-1).  Objective: time per sample T/(D*M), compared exactly;
+ * ties go to the lowest global index.
+ */
+typedef struct pos_problem {
+    pos_tables tables;
+    int32_t S;
+    int32_t n_M;
+    const int32_t *M_list;      /* [n_M], 1..255 */
+    const int32_t *tp_list;     /* [n_tp] TP degree of each TP index (reported) */
+    const int32_t *dp_list;     /* [n_tp] data-parallel degree D of each TP index */
+    int32_t placement;          /* POS_PLACE_FREE or POS_PLACE_EXACT */
+    const int32_t *type_counts; /* [n_types] stages per type (POS_PLACE_EXACT) */
+    int32_t warmup;             /* random feasible samples seeding T_min (paper: 500) */
+    int32_t prune;              /* 1: stage-level prune g(S_x) > T_min (Eq. 2); 0: exhaustive */
+    uint64_t seed;              /* warm-up sampling seed */
+    int32_t schedule;           /* POS_SCHED_1F1B */
+    int64_t frontier_cap;       /* entries per frontier buffer; 0 = default */
+} pos_problem;
+
+typedef struct pos_plan {
+    int32_t found;
+    int32_t m_idx, tp_idx, M, tp, D, S;
+    int32_t makespan;           /* T in us */
+    int32_t type[POS_MAX_STAGES];
+    int32_t layers[POS_MAX_STAGES];
+    uint64_t place_rank, map_rank, global_index;
+} pos_plan;
+
+typedef struct pos_search_stats {
+    uint64_t evaluated;         /* complete plans whose makespan was computed */
+    uint64_t warmup_evaluated;  /* of which in the warm-up */
+    uint64_t prefixes;          /* partial plans generated (all depths) */
+    uint64_t pruned_bound;      /* children cut by g(S_x) > T_min */
+    uint64_t pruned_memory;     /* children cut by memory feasibility */
+    uint64_t relaxations;       /* DAG node relaxations (2*S*M per evaluation) */
+    uint64_t slices, slices_feasible;
+    uint64_t launches;          /* kernel launches */
+    double ms_setup, ms_warmup, ms_search, ms_total;
+} pos_search_stats;
+
+/*
+ * Exact search (Sec. 4.2.3) on the current CUDA device: warm-up sampling,
+ * then enumeration of every slice's layer compositions with the memory cut
+ * and, if prune != 0, the stage-level prune of Eq. 2 / Theorem 1; the result
+ * equals the exhaustive optimum.  Host pointers in, host plan out;
+ * synchronous.  stats may be NULL.
+ * Errors: POS_EINVAL, POS_EOVERFLOW (guard fails for some M), POS_ENOMEM,
+ * POS_ECUDA, POS_ETIMEOUT, POS_EINFEASIBLE (no memory-feasible plan; *out
+ * has found = 0).
+ * Limits: at most 65535 slices with a feasible root per M value; the global
+ * index must fit in 64 bits; lcm of all D*M below 2^32.
+ */
+pos_status poseidon_search(const pos_problem *problem, pos_plan *out, pos_search_stats *stats);
+
+/* Message describing the last error of the calling thread ("" if none). */
+const char *poseidon_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* POSEIDON_H */

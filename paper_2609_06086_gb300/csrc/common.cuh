@@ -1,0 +1,355 @@
+// Shared internals of libposeidon: error state, the device table blob and
+// the per-candidate device routines (composition unranking/ranking, stage
+// weights, memory feasibility, the 1F1B makespan wavefront).
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+
+#include "../../include/poseidon.h"
+
+namespace pos {
+
+// ---------------------------------------------------------------------------
+// Error state (per host thread)
+// ---------------------------------------------------------------------------
+void set_error(const std::string &msg);
+pos_status fail(pos_status st, const std::string &msg);
+pos_status cuda_fail(cudaError_t e, const char *what);
+
+#define POS_CUDA(call)                                           \
+    do {                                                         \
+        cudaError_t e_ = (call);                                 \
+        if (e_ != cudaSuccess) return pos::cuda_fail(e_, #call); \
+    } while (0)
+
+// ---------------------------------------------------------------------------
+// Table blob: one contiguous device buffer, staged whole into shared memory
+// by every kernel.  Offsets are bytes from the blob start, 16-byte aligned.
+//   binom  u64 [128][16]        C(n, k), k <= 15
+//   Pw, Pa i64 [K][L+1] each    exclusive prefix sums of mem_w, mem_a
+//   cap    i64 [K]
+//   Pf, Pb, Pd i32 [K][L+1]     exclusive prefix sums of fwd, bwd, dsync
+//   p2f, p2b   i32 [K][K]       transfer times [src class][dst class]
+// ---------------------------------------------------------------------------
+constexpr int kBinomN = 128;
+constexpr int kBinomK = 16;
+
+struct BlobLayout {
+    int L, K, n_types, n_tp;
+    int off_binom, off_Pw, off_Pa, off_cap, off_Pf, off_Pb, off_Pd, off_p2f, off_p2b;
+    int bytes;  // multiple of 16
+};
+
+BlobLayout make_layout(int L, int n_types, int n_tp);
+
+struct Handle {
+    int device;
+    BlobLayout lay;
+    void *d_blob;  // device copy of the blob
+    // overflow guard terms: sum_l max_k(fwd+bwd), sum_l max_k dsync, max p2p
+    int64_t guard_A, guard_D, guard_P;
+};
+
+pos_status validate_tables(const pos_tables *t);
+pos_status create_handle(const pos_tables *t, Handle **out);
+void destroy_handle(Handle *h);
+int sm_count();
+
+// View of the blob staged in shared memory.  It keeps the shared-memory
+// base and a pointer to the layout in kernel parameter space; every access
+// adds an offset read from there, so no table pointer occupies a register.
+struct Tab {
+    const unsigned char *base;  // the staged blob (dynamic shared memory)
+    const BlobLayout *ly;       // points into kernel parameter space
+    __device__ __forceinline__ int L() const { return ly->L; }
+    __device__ __forceinline__ int Lp1() const { return ly->L + 1; }
+    __device__ __forceinline__ int K() const { return ly->K; }
+    __device__ __forceinline__ int n_tp() const { return ly->n_tp; }
+    __device__ __forceinline__ int n_types() const { return ly->n_types; }
+};
+
+__device__ __forceinline__ int32_t ld32(const unsigned char *base, uint32_t off) {
+    return *reinterpret_cast<const int32_t *>(base + off);
+}
+__device__ __forceinline__ int64_t ld64(const unsigned char *base, uint32_t off) {
+    return *reinterpret_cast<const int64_t *>(base + off);
+}
+
+__device__ __forceinline__ Tab tab_at(const unsigned char *base, const BlobLayout &ly) {
+    Tab t;
+    t.base = base;
+    t.ly = &ly;
+    return t;
+}
+
+__device__ __forceinline__ int32_t Pf(const Tab &t, int k, int c) {
+    return ld32(t.base, t.ly->off_Pf + 4u * (uint32_t)(k * (t.ly->L + 1) + c));
+}
+__device__ __forceinline__ int32_t Pb(const Tab &t, int k, int c) {
+    return ld32(t.base, t.ly->off_Pb + 4u * (uint32_t)(k * (t.ly->L + 1) + c));
+}
+__device__ __forceinline__ int32_t Pd(const Tab &t, int k, int c) {
+    return ld32(t.base, t.ly->off_Pd + 4u * (uint32_t)(k * (t.ly->L + 1) + c));
+}
+__device__ __forceinline__ int64_t Pw(const Tab &t, int k, int c) {
+    return ld64(t.base, t.ly->off_Pw + 8u * (uint32_t)(k * (t.ly->L + 1) + c));
+}
+__device__ __forceinline__ int64_t Pa(const Tab &t, int k, int c) {
+    return ld64(t.base, t.ly->off_Pa + 8u * (uint32_t)(k * (t.ly->L + 1) + c));
+}
+__device__ __forceinline__ int64_t cap_of(const Tab &t, int k) {
+    return ld64(t.base, t.ly->off_cap + 8u * (uint32_t)k);
+}
+__device__ __forceinline__ int32_t p2f(const Tab &t, int a, int b) {
+    return ld32(t.base, t.ly->off_p2f + 4u * (uint32_t)(a * t.ly->K + b));
+}
+__device__ __forceinline__ int32_t p2b(const Tab &t, int a, int b) {
+    return ld32(t.base, t.ly->off_p2b + 4u * (uint32_t)(a * t.ly->K + b));
+}
+__device__ __forceinline__ uint64_t binom(const Tab &t, int n, int k) {
+    return (uint64_t)ld64(t.base, t.ly->off_binom + 8u * (uint32_t)(n * kBinomK + k));
+}
+
+// Cooperative 16-byte copy of the blob into shared memory.
+__device__ __forceinline__ void stage_blob(unsigned char *dst, const void *src, int bytes) {
+    const uint4 *s = reinterpret_cast<const uint4 *>(src);
+    uint4 *d = reinterpret_cast<uint4 *>(dst);
+    for (int i = threadIdx.x; i < bytes / 16; i += blockDim.x) d[i] = __ldg(s + i);
+}
+
+// ---------------------------------------------------------------------------
+// Composition <-> lexicographic rank (combinatorial number system).
+// With p stages left and rem layers left, the compositions whose current
+// stage takes fewer than v layers number C(rem-1, p-1) - C(rem-v, p-1)
+// (hockey-stick sum of C(rem-u-1, p-2) over u < v).
+// cut[0] = 0, cut[s+1] = layers of stages 0..s, cut[S] = L.
+// ---------------------------------------------------------------------------
+template <int S>
+__device__ __forceinline__ void unrank_cuts(const Tab &t, uint64_t rank, int (&cut)[S + 1]) {
+    const int L = t.L();
+    cut[0] = 0;
+#pragma unroll
+    for (int s = 0; s < S - 1; ++s) {
+        const int rem = L - cut[s];
+        const int k = S - s - 1;  // p - 1 with p = S - s stages left
+        // Y = C(rem-1, k) - rank >= 1; the stage takes v = rem - j layers for
+        // the smallest j in [k, rem-1] with C(j, k) >= Y.
+        const uint64_t Y = binom(t, rem - 1, k) - rank;
+        int lo = k, hi = rem - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (binom(t, mid, k) >= Y) hi = mid;
+            else lo = mid + 1;
+        }
+        rank = binom(t, lo, k) - Y;
+        cut[s + 1] = cut[s] + (rem - lo);
+    }
+    cut[S] = L;
+}
+
+// Rank of the composition given by cut[0..S] (same numbering as above).
+template <int S>
+__device__ __forceinline__ uint64_t rank_cuts(const Tab &t, const int (&cut)[S + 1]) {
+    uint64_t r = 0;
+#pragma unroll
+    for (int s = 0; s < S - 1; ++s) {
+        const int rem = t.L() - cut[s];
+        const int l = cut[s + 1] - cut[s];
+        const int k = S - s - 1;
+        r += binom(t, rem - 1, k) - binom(t, rem - l, k);
+    }
+    return r;
+}
+
+// ---------------------------------------------------------------------------
+// Stage weights (Sec. 4.1.3) from prefix-sum differences; memory (Sec. 3.2).
+// ---------------------------------------------------------------------------
+template <int S>
+struct StageW {
+    int32_t F[S], B[S], d[S];
+    int32_t pf[S], pb[S];  // pf[s]: F edge s->s+1; pb[s]: B edge s+1->s
+};
+
+// In-flight micro-batches of 0-based stage s under 1F1B: min(S - s, M).
+__device__ __forceinline__ int inflight(int S, int M, int s) { return min(S - s, M); }
+
+// Does 0-based stage s of an S-stage pipeline on class k fit layers [a, b)?
+__device__ __forceinline__ bool stage_fits(const Tab &t, int S, int M, int s, int k, int a,
+                                           int b) {
+    const int64_t need = (Pw(t, k, b) - Pw(t, k, a)) +
+                         (int64_t)inflight(S, M, s) * (Pa(t, k, b) - Pa(t, k, a));
+    return need <= cap_of(t, k);
+}
+
+template <int S>
+__device__ __forceinline__ void stage_weights(const Tab &t, const int (&cut)[S + 1],
+                                              const int (&cls)[S], StageW<S> &w) {
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+        w.F[s] = Pf(t, cls[s], cut[s + 1]) - Pf(t, cls[s], cut[s]);
+        w.B[s] = Pb(t, cls[s], cut[s + 1]) - Pb(t, cls[s], cut[s]);
+        w.d[s] = Pd(t, cls[s], cut[s + 1]) - Pd(t, cls[s], cut[s]);
+    }
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+        w.pf[s] = (s + 1 < S) ? p2f(t, cls[s], cls[s + 1 < S ? s + 1 : s]) : 0;
+        w.pb[s] = (s + 1 < S) ? p2b(t, cls[s + 1 < S ? s + 1 : s], cls[s]) : 0;
+    }
+}
+
+template <int S>
+__device__ __forceinline__ bool plan_fits(const Tab &t, int M, const int (&cut)[S + 1],
+                                          const int (&cls)[S]) {
+    bool ok = true;
+#pragma unroll
+    for (int s = 0; s < S; ++s) ok &= stage_fits(t, S, M, s, cls[s], cut[s], cut[s + 1]);
+    return ok;
+}
+
+// ---------------------------------------------------------------------------
+// 1F1B makespan as a max-plus wavefront (Sec. 4.1, longest path by DP).
+//
+// Stage s (1-based) runs W_s = min(S-s+1, M) forwards, then (B_i, F_{W+i})
+// pairs, then the remaining backwards.  Every op is one relaxation
+//     finish = max(finish of the stage's previous op,
+//                  finish of the inter-stage predecessor + edge) + weight.
+// The ops are visited in the level order of the unit-weight schedule,
+//     F_{s,m}: m + s - 1 (m <= W_s), 2m + s - 2 (m > W_s);
+//     B_{s,m}: 2S - s + 2m - 1,
+// a topological order with at most one op per stage per level in which,
+// visiting the stages of a level in descending order, the inter-stage
+// predecessor of an op is always the latest op of that kind on the
+// neighbouring stage.  So per stage only the finish of its last forward (Fo)
+// and last backward (Bo) are kept, in registers.  For M >= S the levels
+// split into a ramp-up (levels 1..2S-1), M-S steady two-level steps in which
+// every stage does one F and one B, and a ramp-down (levels 2M..2M+2S-2);
+// the ramps depend on S only and are fully unrolled.  M < S takes a
+// predicated level loop (a separate instantiation, kPathGeneric).
+// ---------------------------------------------------------------------------
+enum { kPathFast = 0, kPathGeneric = 1 };
+
+// Op of 1-based stage s1 at ramp-up level t (1 <= t <= 2S-1) and at
+// ramp-down level 2M + tau (0 <= tau <= 2S-2), for M >= S: 0 none, 1 F, 2 B.
+__host__ __device__ constexpr int ramp_up_op(int S, int s1, int t) {
+    return (t >= s1 && t <= S) ? 1
+           : ((t >= 2 * S - s1 + 2) && ((t + s1) & 1) == 0) ? 1
+           : ((t >= 2 * S - s1 + 1) && ((t + s1) & 1) == 1) ? 2
+                                                              : 0;
+}
+__host__ __device__ constexpr int ramp_down_op(int S, int s1, int tau) {
+    return ((tau <= s1 - 2) && ((tau + s1) & 1) == 0) ? 1
+           : ((tau <= 2 * S - s1 - 1) && ((tau + s1) & 1) == 1) ? 2
+                                                                : 0;
+}
+// Was the last op of stage s1 before ramp-up level t a backward?  (No op
+// yet counts as a forward: Fo starts at 0, the finish time of node S.)
+__host__ __device__ constexpr bool up_last_is_b(int S, int s1, int t) {
+    for (int u = t - 1; u >= 1; --u)
+        if (ramp_up_op(S, s1, u)) return ramp_up_op(S, s1, u) == 2;
+    return false;
+}
+// Same before ramp-down level 2M + tau; at the end of the steady state odd
+// stages (1-based) last ran F and even stages B.
+__host__ __device__ constexpr bool down_last_is_b(int S, int s1, int tau) {
+    for (int u = tau - 1; u >= 0; --u)
+        if (ramp_down_op(S, s1, u)) return ramp_down_op(S, s1, u) == 2;
+    return (s1 & 1) == 0;
+}
+
+#define POS_RELAX_F(s, clock)                                                           \
+    do {                                                                                \
+        int32_t in_ = (s) > 0 ? Fo[(s) > 0 ? (s)-1 : 0] + w.pf[(s) > 0 ? (s)-1 : 0] : 0; \
+        Fo[s] = max((clock), in_) + w.F[s];                                             \
+    } while (0)
+
+#define POS_RELAX_B(s, clock)                                                     \
+    do {                                                                          \
+        int32_t in_ = (s) + 1 < S ? Bo[(s) + 1 < S ? (s) + 1 : 0] + w.pb[s] : 0; \
+        Bo[s] = max((clock), in_) + w.B[s];                                       \
+    } while (0)
+
+template <int S, int PATH>
+__device__ __forceinline__ int32_t makespan_1f1b(const StageW<S> &w, int M) {
+    int32_t Fo[S], Bo[S];
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+        Fo[s] = 0;
+        Bo[s] = 0;
+    }
+    if (PATH == kPathFast) {
+        // ramp-up: levels t = 1 .. 2S-1, stages in descending order
+#pragma unroll
+        for (int t = 1; t <= 2 * S - 1; ++t) {
+#pragma unroll
+            for (int s1 = S; s1 >= 1; --s1) {
+                const int s = s1 - 1;
+                const int op = ramp_up_op(S, s1, t);
+                const int32_t clk = up_last_is_b(S, s1, t) ? Bo[s] : Fo[s];
+                if (op == 1) POS_RELAX_F(s, clk);
+                else if (op == 2) POS_RELAX_B(s, clk);
+            }
+        }
+        // steady state: each step is two levels; at an even level even
+        // stages (1-based) run F and odd stages B, at an odd level the
+        // reverse.  An F follows the stage's B and vice versa.
+        for (int j = 0; j < M - S; ++j) {
+#pragma unroll
+            for (int s1 = S; s1 >= 1; --s1) {
+                const int s = s1 - 1;
+                if ((s1 & 1) == 0) POS_RELAX_F(s, Bo[s]);
+                else POS_RELAX_B(s, Fo[s]);
+            }
+#pragma unroll
+            for (int s1 = S; s1 >= 1; --s1) {
+                const int s = s1 - 1;
+                if ((s1 & 1) == 1) POS_RELAX_F(s, Bo[s]);
+                else POS_RELAX_B(s, Fo[s]);
+            }
+        }
+        // ramp-down: levels 2M + tau, tau = 0 .. 2S-2
+#pragma unroll
+        for (int tau = 0; tau <= 2 * S - 2; ++tau) {
+#pragma unroll
+            for (int s1 = S; s1 >= 1; --s1) {
+                const int s = s1 - 1;
+                const int op = ramp_down_op(S, s1, tau);
+                const int32_t clk = down_last_is_b(S, s1, tau) ? Bo[s] : Fo[s];
+                if (op == 1) POS_RELAX_F(s, clk);
+                else if (op == 2) POS_RELAX_B(s, clk);
+            }
+        }
+    } else {
+        // every level visits every stage with predicates.  A stage's ops
+        // are chained, so its last finish is max(Fo, Bo).
+        const int levels = 2 * (M + S - 1);
+        for (int t = 1; t <= levels; ++t) {
+#pragma unroll
+            for (int s1 = S; s1 >= 1; --s1) {
+                const int s = s1 - 1;
+                const int ws = min(S - s1 + 1, M);
+                const bool odd = ((t + s1) & 1) != 0;
+                const bool fwd = (t >= s1 && t <= s1 + ws - 1) ||
+                                 (!odd && t >= 2 * ws + s1 && t <= 2 * M + s1 - 2);
+                const bool bwd = odd && t >= 2 * S - s1 + 1 && t <= 2 * S - s1 + 2 * M - 1;
+                const int32_t clk = max(Fo[s], Bo[s]);
+                if (fwd) POS_RELAX_F(s, clk);
+                else if (bwd) POS_RELAX_B(s, clk);
+            }
+        }
+    }
+    int32_t T = 0;
+#pragma unroll
+    for (int s = 0; s < S; ++s) T = max(T, Bo[s] + w.d[s]);
+    return T;
+}
+
+// Overflow guard U(S, M) >= 2^31 ?
+__host__ __device__ __forceinline__ bool guard_trips(int64_t A, int64_t D, int64_t P, int S,
+                                                     int M) {
+    const int64_t U = (int64_t)M * A + D + 2 * (int64_t)M * (S - 1) * P;
+    return U >= ((int64_t)1 << 31);
+}
+
+}  // namespace pos

@@ -1,0 +1,844 @@
+// poseidon_search: exact parallelism search of Sec. 4.2.3 on the GPU.
+//
+//  1. slices (m_idx, tp_idx, placement) in global-index order; per slice a
+//     suffix-feasibility table feas[x] = bitset of c such that layers [c, L)
+//     can be split over stages x..S-1 within memory (exact memory cut);
+//  2. warm-up (Sec. 4.2.3): random memory-feasible plans seed the incumbent
+//     T_min and give every sampled slice a first objective;
+//  3. slices are taken in batches, most promising first; per batch the
+//     layer compositions are enumerated level by level (stage 1, 2, ...):
+//     every prefix S_x that survives the memory cut and the prune
+//     g(S_x) > T_min (Eq. 2, Theorem 1) is written to the next frontier,
+//     the last two stages are completed in one kernel, and complete plans
+//     are evaluated by the templated leaf kernel, which lowers the incumbent.
+//     Frontiers have a fixed capacity; warps whose children do not fit are
+//     deferred and re-expanded after the part that fit has been finished.
+#include <algorithm>
+#include <chrono>
+#include <cstring>
+#include <numeric>
+#include <vector>
+
+#include "search_kernels.cuh"
+
+namespace pos {
+
+constexpr int kThreads = 256;
+
+// ---------------------------------------------------------------------------
+// suffix feasibility: one block per slice, thread c
+// ---------------------------------------------------------------------------
+__global__ void feas_kernel(const SliceRec *slices, int n_slices, int S, uint4 *feas,
+                            const void *blob, BlobLayout lay) {
+    extern __shared__ __align__(16) unsigned char sm[];
+    __shared__ uint32_t prev[4], cur[4];
+    stage_blob(sm, blob, lay.bytes);
+    __syncthreads();
+    const Tab t = tab_at(sm, lay);
+    const int L = lay.L, c = threadIdx.x;
+    for (int sl = blockIdx.x; sl < n_slices; sl += gridDim.x) {
+        const SliceRec &sr = slices[sl];
+        const int M = sr.M;
+        uint4 *row = feas + (size_t)sr.gid * (S + 1);
+        // x = S: only the empty suffix starting at c = L
+        if (c < 4) prev[c] = (L >> 5) == c ? (1u << (L & 31)) : 0u;
+        __syncthreads();
+        if (c == 0) row[S] = make_uint4(prev[0], prev[1], prev[2], prev[3]);
+        for (int x = S - 1; x >= 0; --x) {
+            bool ok = false;
+            if (c < L) {
+                const int k = sr.cls[x];
+                for (int l = 1; c + l <= L; ++l) {
+                    if (!stage_fits(t, S, M, x, k, c, c + l)) break;
+                    const int e = c + l;
+                    if ((prev[e >> 5] >> (e & 31)) & 1u) {
+                        ok = true;
+                        break;
+                    }
+                }
+            }
+            const unsigned b = __ballot_sync(0xffffffffu, ok);
+            if ((c & 31) == 0) cur[c >> 5] = b;
+            __syncthreads();
+            if (c < 4) prev[c] = cur[c];
+            __syncthreads();
+            if (c == 0) row[x] = make_uint4(prev[0], prev[1], prev[2], prev[3]);
+        }
+        __syncthreads();
+    }
+}
+
+__device__ __forceinline__ bool feas_bit(const uint4 *feas, int S, uint32_t gid, int x, int c) {
+    const uint4 w = __ldg(feas + (size_t)gid * (S + 1) + x);
+    const uint32_t word = (c >> 5) == 0 ? w.x : (c >> 5) == 1 ? w.y : (c >> 5) == 2 ? w.z : w.w;
+    return (word >> (c & 31)) & 1u;
+}
+
+__global__ void root_bits_kernel(const uint4 *feas, int n_slices, int S, uint8_t *out) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n_slices) out[i] = feas_bit(feas, S, i, 0, 0);
+}
+
+// ---------------------------------------------------------------------------
+// warm-up sampler (Sec. 4.2.3): random memory-feasible plans.  splitmix64
+// (Steele, Lea & Flood, 2014) on the counter (seed, sample index).
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint64_t splitmix64_next(uint64_t &s) {
+    uint64_t z = (s += 0x9E3779B97F4A7C15ull);
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    return z ^ (z >> 31);
+}
+
+__global__ void sample_kernel(const SliceRec *slices, const uint32_t *feasible, int n_feasible,
+                              int n_samples, int S, uint64_t seed, const uint4 *feas,
+                              Leaf *out, const void *blob, BlobLayout lay) {
+    extern __shared__ __align__(16) unsigned char sm[];
+    stage_blob(sm, blob, lay.bytes);
+    __syncthreads();
+    const Tab t = tab_at(sm, lay);
+    const int L = lay.L;
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n_samples;
+         i += gridDim.x * blockDim.x) {
+        uint64_t st = seed ^ ((uint64_t)i * 0xD1B54A32D192ED03ull);
+        const uint32_t sl = feasible[splitmix64_next(st) % (uint64_t)n_feasible];
+        const SliceRec &sr = slices[sl];
+        Leaf lf;
+        lf.slice = sl;
+        for (int s = 0; s < 16; ++s) lf.cut[s] = 0;
+        lf.pad[0] = lf.pad[1] = lf.pad[2] = 0;
+        int c = 0;
+        for (int x = 0; x < S - 1; ++x) {
+            const int k = sr.cls[x];
+            int n_ok = 0;
+            for (int l = 1; c + l <= L - (S - x - 1); ++l) {
+                if (!stage_fits(t, S, sr.M, x, k, c, c + l)) break;
+                n_ok += feas_bit(feas, S, sr.gid, x + 1, c + l);
+            }
+            int r = (int)(splitmix64_next(st) % (uint64_t)max(n_ok, 1));
+            int pick = 1;
+            for (int l = 1; c + l <= L - (S - x - 1); ++l) {
+                if (feas_bit(feas, S, sr.gid, x + 1, c + l)) {
+                    if (r == 0) {
+                        pick = l;
+                        break;
+                    }
+                    --r;
+                }
+            }
+            c += pick;
+            lf.cut[x] = (uint8_t)c;
+        }
+        out[i] = lf;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// level expansion and completion (Sec. 4.2.1 prune, Sec. 3.2 memory cut)
+// ---------------------------------------------------------------------------
+struct ExpandParams {
+    const Prefix *in;
+    long long n_in;
+    const uint32_t *groups;  // work list of 32-parent groups, or NULL = all groups
+    long long n_groups;
+    int x;                   // depth of the parents (stages 0..x-1 placed)
+    int S, M;
+    int prune;
+    const SliceRec *slices;
+    const uint4 *feas;
+    Prefix *out;             // expand: children at depth x+1
+    Leaf *leaves;            // complete: full plans
+    unsigned long long *out_count;
+    unsigned long long cap;
+    uint32_t *deferred;
+    unsigned long long *n_deferred;
+    const Key128 *inc;
+    unsigned long long *stats;
+    const void *blob;
+    BlobLayout lay;
+};
+
+// Stage totals of placed stages 0..x-1 give the two carries of Eq. 2:
+//   A  = sum_{i<x} F_i,   Bm = max_{i<x} (sum_{j=i}^{x-1} B_j + d_i)
+// (Bm = -1 when x = 0; every d is >= 0).  For a new stage x with (F, B, d):
+//   g(S_{x+1}) = A + M (F + B) + max(Bm, d).
+__device__ __forceinline__ void carries(const Tab &t, const SliceRec &sr, const uint8_t *cut,
+                                        int x, int64_t &A, int64_t &Bm, int &c) {
+    A = 0;
+    Bm = -1;
+    c = 0;
+    for (int i = 0; i < x; ++i) {
+        const int k = sr.cls[i], c2 = cut[i];
+        A += Pf(t, k, c2) - Pf(t, k, c);
+        Bm = max(Bm, (int64_t)(Pd(t, k, c2) - Pd(t, k, c))) + (Pb(t, k, c2) - Pb(t, k, c));
+        c = c2;
+    }
+}
+
+// Children of one parent at depth x (x <= S-3).  WRITE=false counts them;
+// WRITE=true writes them from out+pos.  Both passes take the same decisions
+// (the incumbent does not change while expansion kernels run).
+template <bool WRITE>
+__device__ int expand_one(const ExpandParams &p, const Tab &t, const Prefix &pr, uint64_t thr,
+                          unsigned long long pos, unsigned long long &cut_bound,
+                          unsigned long long &cut_mem) {
+    if (pr.slice == kPrefixHole) return 0;
+    const SliceRec &sr = p.slices[pr.slice];
+    const int S = p.S, M = p.M, x = p.x, L = t.L();
+    int64_t A, Bm;
+    int c;
+    carries(t, sr, pr.cut, x, A, Bm, c);
+    const int k = sr.cls[x];
+    const uint64_t scale = sr.scale;
+    int n = 0;
+    for (int l = 1; c + l <= L - (S - x - 1); ++l) {
+        const int c2 = c + l;
+        if (!stage_fits(t, S, M, x, k, c, c2)) {
+            ++cut_mem;
+            break;
+        }
+        if (p.prune) {
+            const int64_t F = Pf(t, k, c2) - Pf(t, k, c), B = Pb(t, k, c2) - Pb(t, k, c);
+            const int64_t d = Pd(t, k, c2) - Pd(t, k, c);
+            const int64_t g = A + (int64_t)M * (F + B) + max(Bm, d);
+            if ((uint64_t)g * scale > thr) {
+                ++cut_bound;
+                break;
+            }
+        }
+        if (!feas_bit(p.feas, S, sr.gid, x + 1, c2)) {
+            ++cut_mem;
+            continue;
+        }
+        if (WRITE) {
+            Prefix ch = pr;
+            ch.cut[x] = (uint8_t)c2;
+            p.out[pos + n] = ch;
+        }
+        ++n;
+    }
+    return n;
+}
+
+// Complete plans from one parent at depth S-2: choose l_{S-1}; stage S-1
+// takes the rest.  Checks memory of both stages and g(S_{S-1}), g(S_S).
+template <bool WRITE>
+__device__ int complete_one(const ExpandParams &p, const Tab &t, const Prefix &pr, uint64_t thr,
+                            unsigned long long pos, unsigned long long &cut_bound,
+                            unsigned long long &cut_mem) {
+    if (pr.slice == kPrefixHole) return 0;
+    const SliceRec &sr = p.slices[pr.slice];
+    const int S = p.S, M = p.M, L = t.L(), a = S - 2, b = S - 1;
+    int64_t A, Bm;
+    int c;
+    carries(t, sr, pr.cut, a, A, Bm, c);
+    const int ka = sr.cls[a], kb = sr.cls[b];
+    const uint64_t scale = sr.scale;
+    int n = 0;
+    for (int l = 1; c + l <= L - 1; ++l) {
+        const int c2 = c + l;
+        if (!stage_fits(t, S, M, a, ka, c, c2)) {
+            ++cut_mem;
+            break;
+        }
+        const int64_t Fa = Pf(t, ka, c2) - Pf(t, ka, c), Ba = Pb(t, ka, c2) - Pb(t, ka, c);
+        const int64_t da = Pd(t, ka, c2) - Pd(t, ka, c);
+        if (p.prune && (uint64_t)(A + (int64_t)M * (Fa + Ba) + max(Bm, da)) * scale > thr) {
+            ++cut_bound;
+            break;
+        }
+        if (!stage_fits(t, S, M, b, kb, c2, L)) {
+            ++cut_mem;
+            continue;
+        }
+        if (p.prune) {
+            const int64_t Fb = Pf(t, kb, L) - Pf(t, kb, c2), Bb = Pb(t, kb, L) - Pb(t, kb, c2);
+            const int64_t db = Pd(t, kb, L) - Pd(t, kb, c2);
+            const int64_t g = A + Fa + (int64_t)M * (Fb + Bb) + max(max(Bm, da) + Ba, db);
+            if ((uint64_t)g * scale > thr) {
+                ++cut_bound;
+                continue;
+            }
+        }
+        if (WRITE) {
+            Leaf lf;
+            lf.slice = pr.slice;
+            for (int s = 0; s < 16; ++s) lf.cut[s] = s < 14 ? (s < a ? pr.cut[s] : 0) : 0;
+            lf.cut[a] = (uint8_t)c2;
+            lf.pad[0] = lf.pad[1] = lf.pad[2] = 0;
+            p.leaves[pos + n] = lf;
+        }
+        ++n;
+    }
+    return n;
+}
+
+// One warp per group of 32 consecutive parents: count, reserve output slots
+// with one atomic, write -- or, when the output is full, defer the group.
+template <bool COMPLETE>
+__global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
+    extern __shared__ __align__(16) unsigned char sm[];
+    stage_blob(sm, p.blob, p.lay.bytes);
+    __syncthreads();
+    const Tab t = tab_at(sm, p.lay);
+    const uint64_t thr = p.prune ? __ldcg(&p.inc->obj) : ~0ull;
+    const int lane = threadIdx.x & 31;
+    const long long warp = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
+    const long long n_warps = ((long long)gridDim.x * blockDim.x) >> 5;
+    const long long n_work = p.groups ? p.n_groups : (p.n_in + 31) / 32;
+    unsigned long long emitted = 0, cb = 0, cm = 0;
+    for (long long w = warp; w < n_work; w += n_warps) {
+        const long long g = p.groups ? (long long)p.groups[w] : w;
+        const long long i = g * 32 + lane;
+        Prefix pr;
+        pr.slice = kPrefixHole;
+        if (i < p.n_in) pr = p.in[i];
+        unsigned long long dummy_b = 0, dummy_m = 0;
+        const int n = COMPLETE ? complete_one<false>(p, t, pr, thr, 0, dummy_b, dummy_m)
+                               : expand_one<false>(p, t, pr, thr, 0, dummy_b, dummy_m);
+        int incl = n;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += v;
+        }
+        const int total = __shfl_sync(0xffffffffu, incl, 31);
+        unsigned long long base = 0;
+        if (lane == 0 && total > 0) base = atomicAdd(p.out_count, (unsigned long long)total);
+        base = __shfl_sync(0xffffffffu, base, 0);
+        if (total == 0) continue;
+        const unsigned long long my = base + (unsigned long long)(incl - n);
+        if (base + (unsigned long long)total <= p.cap) {
+            if (COMPLETE) complete_one<true>(p, t, pr, thr, my, cb, cm);
+            else expand_one<true>(p, t, pr, thr, my, cb, cm);
+            emitted += n;
+        } else {
+            // no room: mark this warp's reserved slots below cap as holes
+            for (unsigned long long q = my; q < my + (unsigned long long)n && q < p.cap; ++q) {
+                if (COMPLETE) p.leaves[q].slice = kLeafHole;
+                else p.out[q].slice = kPrefixHole;
+            }
+            if (lane == 0) {
+                const unsigned long long d = atomicAdd(p.n_deferred, 1ull);
+                p.deferred[d] = (uint32_t)g;
+            }
+        }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        emitted += __shfl_xor_sync(0xffffffffu, emitted, o);
+        cb += __shfl_xor_sync(0xffffffffu, cb, o);
+        cm += __shfl_xor_sync(0xffffffffu, cm, o);
+    }
+    if (lane == 0) {
+        if (!COMPLETE && emitted) atomicAdd(p.stats + kStPrefixes, emitted);
+        if (cb) atomicAdd(p.stats + kStPrunedBound, cb);
+        if (cm) atomicAdd(p.stats + kStPrunedMemory, cm);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+static uint64_t gcd64(uint64_t a, uint64_t b) {
+    while (b) {
+        const uint64_t r = a % b;
+        a = b;
+        b = r;
+    }
+    return a;
+}
+
+struct DevBuf {
+    void *p = nullptr;
+    size_t bytes = 0;
+    DevBuf() = default;
+    DevBuf(const DevBuf &) = delete;
+    DevBuf &operator=(const DevBuf &) = delete;
+    ~DevBuf() {
+        if (p) cudaFree(p);
+    }
+    cudaError_t reserve(size_t b) {
+        if (b <= bytes) return cudaSuccess;
+        if (p) cudaFree(p);
+        p = nullptr;
+        bytes = 0;
+        const cudaError_t e = cudaMalloc(&p, b);
+        if (e == cudaSuccess) bytes = b;
+        return e;
+    }
+};
+
+struct Search {
+    const pos_problem *pb = nullptr;
+    Handle *h = nullptr;
+    cudaStream_t stream = nullptr;
+    int S = 0, L = 0, n_tp = 0;
+    uint64_t n_map = 0, n_place = 0;
+    long long cap = 0;
+    int grid_level = 0, grid_leaf = 0;
+    std::vector<std::vector<int>> places;
+    std::vector<SliceRec> slices;
+    DevBuf d_slices, d_feas, d_batch, d_inc, d_ctr, d_best, d_feasible, d_leaves, d_roots;
+    DevBuf d_front[POS_MAX_STAGES + 1];      // per depth: Prefix buffers
+    DevBuf d_defer[2 * (POS_MAX_STAGES + 1)];  // per depth: two deferred group lists
+    unsigned long long *ctr = nullptr;  // [0..15] out counts per depth, [16..31] deferred, [32] leaves
+    unsigned long long *stats = nullptr;
+    uint64_t launches = 0;
+    pos_status err = POS_OK;
+
+    ~Search() {
+        if (stream) cudaStreamDestroy(stream);
+        if (h) destroy_handle(h);
+    }
+};
+
+static pos_status validate_problem(const pos_problem *p) {
+    if (!p) return fail(POS_EINVAL, "problem is NULL");
+    if (p->schedule != POS_SCHED_1F1B) return fail(POS_ENOTIMPL, "only 1F1B is implemented");
+    if (p->S < 1 || p->S > POS_MAX_STAGES) return fail(POS_EINVAL, "S must be in 1..16");
+    if (p->S > p->tables.L) return fail(POS_EINVAL, "S > L");
+    if (p->n_M < 1 || !p->M_list) return fail(POS_EINVAL, "empty M_list");
+    for (int i = 0; i < p->n_M; ++i)
+        if (p->M_list[i] < 1 || p->M_list[i] > 255) return fail(POS_EINVAL, "M out of 1..255");
+    if (!p->dp_list || !p->tp_list) return fail(POS_EINVAL, "tp_list/dp_list is NULL");
+    for (int i = 0; i < p->tables.n_tp; ++i)
+        if (p->dp_list[i] < 1) return fail(POS_EINVAL, "D must be >= 1");
+    if (p->placement != POS_PLACE_FREE && p->placement != POS_PLACE_EXACT)
+        return fail(POS_EINVAL, "unknown placement rule");
+    if (p->placement == POS_PLACE_EXACT) {
+        if (!p->type_counts) return fail(POS_EINVAL, "type_counts is NULL");
+        int sum = 0;
+        for (int i = 0; i < p->tables.n_types; ++i) {
+            if (p->type_counts[i] < 0) return fail(POS_EINVAL, "negative type count");
+            sum += p->type_counts[i];
+        }
+        if (sum != p->S) return fail(POS_EINVAL, "type_counts must sum to S");
+    }
+    if (p->warmup < 0) return fail(POS_EINVAL, "warmup < 0");
+    if (p->frontier_cap < 0) return fail(POS_EINVAL, "frontier_cap < 0");
+    return POS_OK;
+}
+
+// allowed stage-type sequences in lexicographic order
+static pos_status enumerate_places(Search &s) {
+    const pos_problem *p = s.pb;
+    const int S = p->S, T = p->tables.n_types;
+    std::vector<int> seq(S, 0);
+    const uint64_t limit = 1ull << 22;
+    for (;;) {
+        bool ok = true;
+        if (p->placement == POS_PLACE_EXACT) {
+            for (int ty = 0; ty < T && ok; ++ty) {
+                int cnt = 0;
+                for (int x = 0; x < S; ++x) cnt += seq[x] == ty;
+                ok = cnt == p->type_counts[ty];
+            }
+        }
+        if (ok) {
+            s.places.push_back(seq);
+            if (s.places.size() > limit) return fail(POS_EINVAL, "too many placements");
+        }
+        int x = S - 1;
+        while (x >= 0 && seq[x] == T - 1) seq[x--] = 0;
+        if (x < 0) break;
+        seq[x]++;
+    }
+    s.n_place = s.places.size();
+    return POS_OK;
+}
+
+static uint64_t host_binom(int n, int k) {
+    if (k < 0 || k > n) return 0;
+    uint64_t r = 1;
+    for (int i = 1; i <= k; ++i) r = r * (uint64_t)(n - k + i) / (uint64_t)i;
+    return r;
+}
+
+static void host_unrank(int L, int S, uint64_t rank, int32_t *layers) {
+    int rem = L;
+    for (int s = 0; s < S - 1; ++s) {
+        const int after = S - s - 1;
+        int v = 1;
+        for (; v <= rem - after; ++v) {
+            const uint64_t cnt = host_binom(rem - v - 1, after - 1);
+            if (rank < cnt) break;
+            rank -= cnt;
+        }
+        layers[s] = v;
+        rem -= v;
+    }
+    layers[S - 1] = rem;
+}
+
+static pos_status sync_read(Search &s, void *dst, const void *src, size_t bytes) {
+    POS_CUDA(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToHost, s.stream));
+    POS_CUDA(cudaStreamSynchronize(s.stream));
+    return POS_OK;
+}
+
+static pos_status ensure_depth(Search &s, int depth) {
+    POS_CUDA(s.d_front[depth].reserve(sizeof(Prefix) * (size_t)s.cap));
+    return POS_OK;
+}
+
+static pos_status ensure_defer(Search &s, int depth, long long groups) {
+    const size_t b = sizeof(uint32_t) * (size_t)std::max<long long>(groups, 1);
+    POS_CUDA(s.d_defer[2 * depth].reserve(b));
+    POS_CUDA(s.d_defer[2 * depth + 1].reserve(b));
+    return POS_OK;
+}
+
+static ExpandParams base_params(Search &s, const SliceRec *batch, int M) {
+    ExpandParams p;
+    std::memset(&p, 0, sizeof(p));
+    p.S = s.S;
+    p.M = M;
+    p.prune = s.pb->prune ? 1 : 0;
+    p.slices = batch;
+    p.feas = static_cast<const uint4 *>(s.d_feas.p);
+    p.cap = (unsigned long long)s.cap;
+    p.inc = static_cast<const Key128 *>(s.d_inc.p);
+    p.stats = s.stats;
+    p.blob = s.h->d_blob;
+    p.lay = s.h->lay;
+    return p;
+}
+
+static pos_status run_leaves(Search &s, const Leaf *leaves, unsigned long long *count,
+                             const SliceRec *table, int M, unsigned long long *slice_best) {
+    LeafParams lp;
+    lp.leaves = leaves;
+    lp.count = count;
+    lp.cap = (unsigned long long)s.cap;
+    lp.slices = table;
+    lp.M = M;
+    lp.n_map = s.n_map;
+    lp.inc = static_cast<Key128 *>(s.d_inc.p);
+    lp.stats = s.stats;
+    lp.slice_best = slice_best;
+    lp.blob = s.h->d_blob;
+    lp.lay = s.h->lay;
+    s.launches++;
+    return launch_leaf(s.S, M >= s.S, lp, s.grid_leaf, s.stream);
+}
+
+// Enumerate everything below the prefixes in[0..n_in) (depth x).
+static pos_status process(Search &s, const SliceRec *batch, int M, int x, const Prefix *in,
+                          long long n_in) {
+    const int S = s.S;
+    const bool last = (x == S - 2);
+    const long long all_groups = (n_in + 31) / 32;
+    pos_status st = ensure_defer(s, x, all_groups);
+    if (st != POS_OK) return st;
+    if (!last && (st = ensure_depth(s, x + 1)) != POS_OK) return st;
+    unsigned long long *out_count = last ? s.ctr + 32 : s.ctr + (x + 1);
+    unsigned long long *n_def = s.ctr + 16 + x;
+    const uint32_t *work = nullptr;
+    long long n_work = all_groups;
+    int flip = 0;
+    for (;;) {
+        POS_CUDA(cudaMemsetAsync(out_count, 0, sizeof(unsigned long long), s.stream));
+        POS_CUDA(cudaMemsetAsync(n_def, 0, sizeof(unsigned long long), s.stream));
+        ExpandParams p = base_params(s, batch, M);
+        p.in = in;
+        p.n_in = n_in;
+        p.groups = work;
+        p.n_groups = n_work;
+        p.x = x;
+        p.out = last ? nullptr : static_cast<Prefix *>(s.d_front[x + 1].p);
+        p.leaves = last ? static_cast<Leaf *>(s.d_leaves.p) : nullptr;
+        p.out_count = out_count;
+        p.deferred = static_cast<uint32_t *>(s.d_defer[2 * x + flip].p);
+        p.n_deferred = n_def;
+        const int smem = s.h->lay.bytes;
+        const long long blocks_needed = (n_work * 32 + kThreads - 1) / kThreads;
+        const int grid = (int)std::max<long long>(1, std::min<long long>(blocks_needed,
+                                                                         s.grid_level));
+        s.launches++;
+        if (last) {
+            level_kernel<true><<<grid, kThreads, smem, s.stream>>>(p);
+        } else {
+            level_kernel<false><<<grid, kThreads, smem, s.stream>>>(p);
+        }
+        POS_CUDA(cudaGetLastError());
+        if (last) {
+            // evaluate the leaves that fit; the count stays on the device
+            if ((st = run_leaves(s, p.leaves, out_count, batch, M, nullptr)) != POS_OK) return st;
+        }
+        unsigned long long cnt[2];
+        if ((st = sync_read(s, &cnt[0], out_count, 8)) != POS_OK) return st;
+        if ((st = sync_read(s, &cnt[1], n_def, 8)) != POS_OK) return st;
+        if (!last) {
+            const long long n_out = (long long)std::min<unsigned long long>(cnt[0], s.cap);
+            if (n_out > 0) {
+                st = process(s, batch, M, x + 1, static_cast<const Prefix *>(s.d_front[x + 1].p),
+                             n_out);
+                if (st != POS_OK) return st;
+            }
+        }
+        if (cnt[1] == 0) break;
+        work = static_cast<const uint32_t *>(s.d_defer[2 * x + flip].p);
+        n_work = (long long)cnt[1];
+        flip ^= 1;
+    }
+    return POS_OK;
+}
+
+static double ms_since(std::chrono::steady_clock::time_point t0) {
+    return std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0)
+        .count();
+}
+
+static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats) {
+    const auto t_start = std::chrono::steady_clock::now();
+    const pos_problem *p = s.pb;
+    pos_status st = validate_problem(p);
+    if (st != POS_OK) return st;
+    if ((st = create_handle(&p->tables, &s.h)) != POS_OK) return st;
+    POS_CUDA(cudaStreamCreateWithFlags(&s.stream, cudaStreamNonBlocking));
+    s.S = p->S;
+    s.L = p->tables.L;
+    s.n_tp = p->tables.n_tp;
+    s.n_map = host_binom(s.L - 1, s.S - 1);
+    s.cap = p->frontier_cap > 0 ? p->frontier_cap : (1ll << 26);
+    if ((st = enumerate_places(s)) != POS_OK) return st;
+    const uint64_t n_slices64 = (uint64_t)p->n_M * s.n_tp * s.n_place;
+    if (n_slices64 > (1ull << 22)) return fail(POS_EINVAL, "more than 2^22 slices");
+    const int n_slices = (int)n_slices64;
+    if (s.n_map && n_slices64 > ~0ull / s.n_map) return fail(POS_EINVAL, "global index overflows");
+    // overflow guard for every M (Sec. 4.1 path-length bound)
+    for (int i = 0; i < p->n_M; ++i)
+        if (guard_trips(s.h->guard_A, s.h->guard_D, s.h->guard_P, s.S, p->M_list[i]))
+            return fail(POS_EOVERFLOW, "makespan bound reaches 2^31 for some M");
+    // objective scale: Q = lcm(D*M); T*Q/(D*M) orders plans by time per sample
+    uint64_t Q = 1;
+    for (int i = 0; i < p->n_M; ++i)
+        for (int j = 0; j < s.n_tp; ++j) {
+            const uint64_t dm = (uint64_t)p->dp_list[j] * p->M_list[i];
+            Q = Q / gcd64(Q, dm) * dm;
+            if (Q >= (1ull << 32)) return fail(POS_EINVAL, "lcm of D*M reaches 2^32");
+        }
+    s.slices.resize(n_slices);
+    for (int mi = 0; mi < p->n_M; ++mi)
+        for (int tp = 0; tp < s.n_tp; ++tp)
+            for (uint64_t pr = 0; pr < s.n_place; ++pr) {
+                const uint64_t ord = ((uint64_t)mi * s.n_tp + tp) * s.n_place + pr;
+                SliceRec &r = s.slices[ord];
+                std::memset(&r, 0, sizeof(r));
+                r.ordinal = ord;
+                r.M = p->M_list[mi];
+                r.scale = Q / ((uint64_t)p->dp_list[tp] * p->M_list[mi]);
+                r.gid = (uint32_t)ord;
+                for (int x = 0; x < s.S; ++x) r.cls[x] = (uint8_t)(s.places[pr][x] * s.n_tp + tp);
+            }
+    const int smem = s.h->lay.bytes;
+    int per_sm = 0;
+    POS_CUDA(cudaFuncSetAttribute(level_kernel<false>,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    POS_CUDA(cudaFuncSetAttribute(level_kernel<true>,
+                                  cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    POS_CUDA(cudaFuncSetAttribute(feas_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    POS_CUDA(cudaFuncSetAttribute(sample_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  smem));
+    POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, level_kernel<false>, kThreads,
+                                                           smem));
+    s.grid_level = std::max(1, per_sm) * sm_count();
+    s.grid_leaf = 2 * sm_count();
+
+    POS_CUDA(s.d_slices.reserve(sizeof(SliceRec) * n_slices));
+    POS_CUDA(s.d_feas.reserve(sizeof(uint4) * (size_t)n_slices * (s.S + 1)));
+    POS_CUDA(s.d_inc.reserve(sizeof(Key128)));
+    POS_CUDA(s.d_ctr.reserve(sizeof(unsigned long long) * 64));
+    POS_CUDA(s.d_best.reserve(sizeof(unsigned long long) * n_slices));
+    POS_CUDA(s.d_leaves.reserve(sizeof(Leaf) * (size_t)s.cap));
+    s.ctr = static_cast<unsigned long long *>(s.d_ctr.p);
+    s.stats = s.ctr + 40;
+    POS_CUDA(cudaMemcpyAsync(s.d_slices.p, s.slices.data(), sizeof(SliceRec) * n_slices,
+                             cudaMemcpyHostToDevice, s.stream));
+    POS_CUDA(cudaMemsetAsync(s.d_inc.p, 0xff, sizeof(Key128), s.stream));
+    POS_CUDA(cudaMemsetAsync(s.d_ctr.p, 0, sizeof(unsigned long long) * 64, s.stream));
+    POS_CUDA(cudaMemsetAsync(s.d_best.p, 0xff, sizeof(unsigned long long) * n_slices, s.stream));
+    const SliceRec *d_all = static_cast<const SliceRec *>(s.d_slices.p);
+    feas_kernel<<<std::min(n_slices, 16 * sm_count()), 128, smem, s.stream>>>(
+        d_all, n_slices, s.S, static_cast<uint4 *>(s.d_feas.p), s.h->d_blob, s.h->lay);
+    POS_CUDA(cudaGetLastError());
+    s.launches++;
+    DevBuf d_root;
+    POS_CUDA(d_root.reserve(n_slices));
+    root_bits_kernel<<<(n_slices + 255) / 256, 256, 0, s.stream>>>(
+        static_cast<const uint4 *>(s.d_feas.p), n_slices, s.S, static_cast<uint8_t *>(d_root.p));
+    POS_CUDA(cudaGetLastError());
+    s.launches++;
+    std::vector<uint8_t> root(n_slices);
+    if ((st = sync_read(s, root.data(), d_root.p, n_slices)) != POS_OK) return st;
+    // feasible slices, grouped by M index
+    std::vector<std::vector<uint32_t>> feas_by_m(p->n_M);
+    uint64_t n_feasible = 0;
+    for (int i = 0; i < n_slices; ++i)
+        if (root[i]) {
+            feas_by_m[i / (s.n_tp * s.n_place)].push_back((uint32_t)i);
+            ++n_feasible;
+        }
+    const double ms_setup = ms_since(t_start);
+
+    // warm-up, split over the M values in proportion to their feasible slices
+    const auto t_warm = std::chrono::steady_clock::now();
+    uint64_t warm_evals = 0;
+    if (p->warmup > 0 && n_feasible > 0) {
+        POS_CUDA(s.d_feasible.reserve(sizeof(uint32_t) * n_feasible));
+        for (int mi = 0; mi < p->n_M; ++mi) {
+            const auto &fl = feas_by_m[mi];
+            if (fl.empty()) continue;
+            const long long n_s = std::min<long long>(
+                s.cap, std::max<long long>(1, (long long)p->warmup * (long long)fl.size() /
+                                                  (long long)n_feasible));
+            POS_CUDA(cudaMemcpyAsync(s.d_feasible.p, fl.data(), sizeof(uint32_t) * fl.size(),
+                                     cudaMemcpyHostToDevice, s.stream));
+            sample_kernel<<<(int)std::min<long long>((n_s + 255) / 256, 4 * sm_count()), 256,
+                            smem, s.stream>>>(
+                d_all, static_cast<const uint32_t *>(s.d_feasible.p), (int)fl.size(), (int)n_s,
+                s.S, p->seed + 0x632BE59BD9B4E019ull * (uint64_t)mi,
+                static_cast<const uint4 *>(s.d_feas.p), static_cast<Leaf *>(s.d_leaves.p),
+                s.h->d_blob, s.h->lay);
+            POS_CUDA(cudaGetLastError());
+            s.launches++;
+            unsigned long long cnt = (unsigned long long)n_s;
+            POS_CUDA(cudaMemcpyAsync(s.ctr + 33, &cnt, 8, cudaMemcpyHostToDevice, s.stream));
+            if ((st = run_leaves(s, static_cast<const Leaf *>(s.d_leaves.p), s.ctr + 33, d_all,
+                                 p->M_list[mi], static_cast<unsigned long long *>(s.d_best.p))) !=
+                POS_OK)
+                return st;
+            warm_evals += (uint64_t)n_s;
+        }
+    }
+    std::vector<unsigned long long> best(n_slices);
+    if ((st = sync_read(s, best.data(), s.d_best.p, sizeof(unsigned long long) * n_slices)) !=
+        POS_OK)
+        return st;
+    const double ms_warm = ms_since(t_warm);
+
+    // batches of slices, most promising first
+    const auto t_search = std::chrono::steady_clock::now();
+    struct Group {
+        int mi;
+        unsigned long long best;
+    };
+    std::vector<Group> groups;
+    for (int mi = 0; mi < p->n_M; ++mi) {
+        if (feas_by_m[mi].empty()) continue;
+        auto &fl = feas_by_m[mi];
+        std::stable_sort(fl.begin(), fl.end(),
+                         [&](uint32_t a, uint32_t b) { return best[a] < best[b]; });
+        groups.push_back({mi, best[fl[0]]});
+    }
+    std::stable_sort(groups.begin(), groups.end(),
+                     [](const Group &a, const Group &b) { return a.best < b.best; });
+    POS_CUDA(s.d_batch.reserve(sizeof(SliceRec) * 65535));
+    POS_CUDA(s.d_roots.reserve(sizeof(Prefix) * 65535));
+    for (const Group &g : groups) {
+        const auto &fl = feas_by_m[g.mi];
+        const int M = p->M_list[g.mi];
+        const size_t bsz = std::min<size_t>(
+            65535, std::max<size_t>(32, (fl.size() + 7) / 8));
+        for (size_t b0 = 0; b0 < fl.size(); b0 += bsz) {
+            const size_t nb = std::min(bsz, fl.size() - b0);
+            std::vector<SliceRec> batch(nb);
+            for (size_t j = 0; j < nb; ++j) batch[j] = s.slices[fl[b0 + j]];
+            POS_CUDA(cudaMemcpyAsync(s.d_batch.p, batch.data(), sizeof(SliceRec) * nb,
+                                     cudaMemcpyHostToDevice, s.stream));
+            const SliceRec *d_batch = static_cast<const SliceRec *>(s.d_batch.p);
+            if (s.S == 1) {
+                // the single stage takes every layer: each feasible slice is one plan
+                std::vector<Leaf> lv(nb);
+                for (size_t j = 0; j < nb; ++j) {
+                    std::memset(&lv[j], 0, sizeof(Leaf));
+                    lv[j].slice = (uint32_t)j;
+                }
+                POS_CUDA(cudaMemcpyAsync(s.d_leaves.p, lv.data(), sizeof(Leaf) * nb,
+                                         cudaMemcpyHostToDevice, s.stream));
+                unsigned long long cnt = nb;
+                POS_CUDA(cudaMemcpyAsync(s.ctr + 33, &cnt, 8, cudaMemcpyHostToDevice, s.stream));
+                if ((st = run_leaves(s, static_cast<const Leaf *>(s.d_leaves.p), s.ctr + 33,
+                                     d_batch, M, nullptr)) != POS_OK)
+                    return st;
+                POS_CUDA(cudaStreamSynchronize(s.stream));
+                continue;
+            }
+            std::vector<Prefix> roots(nb);
+            for (size_t j = 0; j < nb; ++j) {
+                std::memset(&roots[j], 0, sizeof(Prefix));
+                roots[j].slice = (uint16_t)j;
+            }
+            POS_CUDA(cudaMemcpyAsync(s.d_roots.p, roots.data(), sizeof(Prefix) * nb,
+                                     cudaMemcpyHostToDevice, s.stream));
+            st = process(s, d_batch, M, 0, static_cast<const Prefix *>(s.d_roots.p),
+                         (long long)nb);
+            if (st != POS_OK) return st;
+        }
+    }
+    POS_CUDA(cudaStreamSynchronize(s.stream));
+    const double ms_search = ms_since(t_search);
+
+    Key128 inc;
+    if ((st = sync_read(s, &inc, s.d_inc.p, sizeof(inc))) != POS_OK) return st;
+    unsigned long long hs[kStCount];
+    if ((st = sync_read(s, hs, s.stats, sizeof(hs))) != POS_OK) return st;
+    if (hs[kStTimeout]) return fail(POS_ETIMEOUT, "incumbent update hit its iteration limit");
+
+    std::memset(out, 0, sizeof(*out));
+    if (stats) {
+        std::memset(stats, 0, sizeof(*stats));
+        stats->evaluated = hs[kStEvaluated];
+        stats->warmup_evaluated = warm_evals;
+        stats->prefixes = hs[kStPrefixes];
+        stats->pruned_bound = hs[kStPrunedBound];
+        stats->pruned_memory = hs[kStPrunedMemory];
+        stats->relaxations = hs[kStRelaxations];
+        stats->slices = (uint64_t)n_slices;
+        stats->slices_feasible = n_feasible;
+        stats->launches = s.launches;
+        stats->ms_setup = ms_setup;
+        stats->ms_warmup = ms_warm;
+        stats->ms_search = ms_search;
+    }
+    if (inc.obj == ~0ull) {
+        if (stats) stats->ms_total = ms_since(t_start);
+        return fail(POS_EINFEASIBLE, "no memory-feasible plan");
+    }
+    const uint64_t ord = inc.idx / s.n_map;
+    const SliceRec &sr = s.slices[ord];
+    out->found = 1;
+    out->map_rank = inc.idx % s.n_map;
+    out->place_rank = ord % s.n_place;
+    out->tp_idx = (int32_t)((ord / s.n_place) % s.n_tp);
+    out->m_idx = (int32_t)(ord / s.n_place / s.n_tp);
+    out->M = p->M_list[out->m_idx];
+    out->tp = p->tp_list[out->tp_idx];
+    out->D = p->dp_list[out->tp_idx];
+    out->S = s.S;
+    out->makespan = (int32_t)(inc.obj / sr.scale);
+    out->global_index = inc.idx;
+    for (int x = 0; x < POS_MAX_STAGES; ++x) {
+        out->type[x] = x < s.S ? s.places[out->place_rank][x] : -1;
+        out->layers[x] = 0;
+    }
+    host_unrank(s.L, s.S, out->map_rank, out->layers);
+    if (stats) stats->ms_total = ms_since(t_start);
+    return POS_OK;
+}
+
+}  // namespace pos
+
+extern "C" pos_status poseidon_search(const pos_problem *problem, pos_plan *out,
+                                      pos_search_stats *stats) {
+    if (!out) return pos::fail(POS_EINVAL, "plan out-pointer is NULL");
+    pos::Search s;
+    s.pb = problem;
+    pos::set_error("");
+    try {
+        return pos::search_impl(s, out, stats);
+    } catch (...) {
+        return pos::fail(POS_ENOMEM, "host exception (allocation failure)");
+    }
+}

@@ -1,0 +1,181 @@
+// Device side of poseidon_search (hot-path steps a2-a8): shared types, the
+// incumbent, and the leaf-evaluation kernel templated on the stage count.
+#pragma once
+#include "common.cuh"
+
+namespace pos {
+
+// Packed incumbent: compared as (obj, idx) -- the scaled objective
+// T * Q/(D*M) first, then the global index -- and updated with a 128-bit
+// compare-and-swap, so concurrent updates always keep the true minimum.
+struct __align__(16) Key128 {
+    unsigned long long idx;
+    unsigned long long obj;
+};
+
+// One slice = (M, TP index, stage-type placement).
+struct SliceRec {
+    uint64_t ordinal;  // (m_idx*n_tp + tp_idx)*n_place + place_rank
+    uint64_t scale;    // Q / (D*M): T * scale orders plans by T/(D*M)
+    uint8_t cls[16];   // class of each stage
+    int32_t M;
+    uint32_t gid;      // row of this slice in the feasibility table
+    uint32_t pad[2];
+};
+static_assert(sizeof(SliceRec) == 48, "SliceRec layout");
+
+// Partial plan at depth x: stages 0..x-1 placed; cut[i] = layers of stages
+// 0..i.  slice indexes the current batch's slice table; 0xffff = hole.
+struct Prefix {
+    uint16_t slice;
+    uint8_t cut[14];
+};
+static_assert(sizeof(Prefix) == 16, "Prefix layout");
+
+// Complete plan: cut[0..S-2]; slice indexes the slice table of the launch.
+struct Leaf {
+    uint32_t slice;
+    uint8_t cut[16];
+    uint32_t pad[3];
+};
+static_assert(sizeof(Leaf) == 32, "Leaf layout");
+
+constexpr uint32_t kLeafHole = 0xffffffffu;
+constexpr uint16_t kPrefixHole = 0xffff;
+
+// device counters / statistics (uint64 each)
+enum {
+    kStPrefixes = 0,
+    kStPrunedBound,
+    kStPrunedMemory,
+    kStEvaluated,
+    kStTimeout,
+    kStRelaxations,
+    kStCount
+};
+
+constexpr int kCasLimit = 1 << 20;
+
+__device__ __forceinline__ bool key_less(unsigned long long ao, unsigned long long ai,
+                                         unsigned long long bo, unsigned long long bi) {
+    return ao < bo || (ao == bo && ai < bi);
+}
+
+// Lower the incumbent to (obj, idx) if that is smaller.  Bounded loop: every
+// failed CAS means another thread lowered the key; after kCasLimit rounds
+// the timeout counter is raised and the update is abandoned.
+__device__ __forceinline__ void incumbent_update(Key128 *inc, unsigned long long obj,
+                                                 unsigned long long idx,
+                                                 unsigned long long *stats) {
+    Key128 cur;
+    cur.obj = __ldcg(&inc->obj);
+    cur.idx = __ldcg(&inc->idx);
+    for (int it = 0; it < kCasLimit; ++it) {
+        if (!key_less(obj, idx, cur.obj, cur.idx)) return;
+        Key128 want;
+        want.obj = obj;
+        want.idx = idx;
+        const Key128 prev = atomicCAS(inc, cur, want);
+        if (prev.obj == cur.obj && prev.idx == cur.idx) return;
+        cur = prev;
+    }
+    atomicAdd(stats + kStTimeout, 1ull);
+}
+
+struct LeafParams {
+    const Leaf *leaves;
+    const unsigned long long *count;  // device count of written leaf slots
+    unsigned long long cap;
+    const SliceRec *slices;
+    int M;
+    uint64_t n_map;
+    Key128 *inc;
+    unsigned long long *stats;
+    unsigned long long *slice_best;  // optional per-slice minimum objective
+    const void *blob;
+    BlobLayout lay;
+};
+
+template <int S, int PATH>
+__global__ void __launch_bounds__(256, (S <= 4 ? 4 : (S <= 8 ? 3 : 2)))
+leaf_kernel(LeafParams p) {
+    extern __shared__ __align__(16) unsigned char sm[];
+    stage_blob(sm, p.blob, p.lay.bytes);
+    __syncthreads();
+    const Tab t = tab_at(sm, p.lay);
+    const unsigned long long c0 = __ldcg(p.count);
+    const unsigned long long n = c0 < p.cap ? c0 : p.cap;
+    const int L = p.lay.L;
+    unsigned long long evaluated = 0;
+    const unsigned long long stride = (unsigned long long)gridDim.x * blockDim.x;
+    // all lanes of a warp iterate together (the warp minimum uses shuffles)
+    const unsigned long long n_round = (n + 31) & ~31ull;
+    for (unsigned long long i = blockIdx.x * (unsigned long long)blockDim.x + threadIdx.x;
+         i < n_round; i += stride) {
+        unsigned long long obj = ~0ull, idx = ~0ull;
+        uint32_t sl = kLeafHole;
+        if (i < n) sl = __ldg(&p.leaves[i].slice);
+        if (sl != kLeafHole) {
+            const SliceRec &sr = p.slices[sl];
+            int cut[S + 1], cls[S];
+            cut[0] = 0;
+#pragma unroll
+            for (int s = 0; s < S - 1; ++s) cut[s + 1] = __ldg(&p.leaves[i].cut[s]);
+            cut[S] = L;
+#pragma unroll
+            for (int s = 0; s < S; ++s) cls[s] = __ldg(&sr.cls[s]);
+            const uint64_t scale = __ldg(&sr.scale);
+            const uint64_t ord = __ldg(&sr.ordinal);
+            const uint64_t rank = rank_cuts<S>(t, cut);
+            StageW<S> w;
+            stage_weights<S>(t, cut, cls, w);
+            const int32_t T = makespan_1f1b<S, PATH>(w, p.M);
+            obj = (unsigned long long)T * scale;
+            idx = ord * p.n_map + rank;
+            ++evaluated;
+            if (p.slice_best) atomicMin(p.slice_best + sl, obj);
+        }
+        // warp minimum, then one CAS attempt per warp
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const unsigned long long oo = __shfl_xor_sync(0xffffffffu, obj, o);
+            const unsigned long long oi = __shfl_xor_sync(0xffffffffu, idx, o);
+            if (key_less(oo, oi, obj, idx)) {
+                obj = oo;
+                idx = oi;
+            }
+        }
+        if ((threadIdx.x & 31) == 0 && obj != ~0ull) incumbent_update(p.inc, obj, idx, p.stats);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) evaluated += __shfl_xor_sync(0xffffffffu, evaluated, o);
+    if ((threadIdx.x & 31) == 0 && evaluated) {
+        atomicAdd(p.stats + kStEvaluated, evaluated);
+        atomicAdd(p.stats + kStRelaxations, evaluated * 2ull * S * (unsigned long long)p.M);
+    }
+}
+
+template <int S, int PATH>
+pos_status launch_leaf_t(const LeafParams &p, int grid, cudaStream_t s) {
+    auto kern = leaf_kernel<S, PATH>;
+    const int smem = p.lay.bytes;
+    POS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    kern<<<grid, 256, smem, s>>>(p);
+    POS_CUDA(cudaGetLastError());
+    return POS_OK;
+}
+
+// per-unit dispatchers (search_leaf_*.cu): S in the unit's range
+pos_status launch_leaf_1_6(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_7_10(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_11_13(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_14_16(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
+
+inline pos_status launch_leaf(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s) {
+    if (S <= 6) return launch_leaf_1_6(S, fast, p, grid, s);
+    if (S <= 10) return launch_leaf_7_10(S, fast, p, grid, s);
+    if (S <= 13) return launch_leaf_11_13(S, fast, p, grid, s);
+    return launch_leaf_14_16(S, fast, p, grid, s);
+}
+
+}  // namespace pos

@@ -1,0 +1,22 @@
+// Instantiation unit of the search leaf kernel (see search_kernels.cuh).
+#include "search_kernels.cuh"
+
+namespace pos {
+
+pos_status launch_leaf_11_13(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s) {
+    switch (S) {
+        case 11:
+            return fast ? launch_leaf_t<11, kPathFast>(p, grid, s)
+                        : launch_leaf_t<11, kPathGeneric>(p, grid, s);
+        case 12:
+            return fast ? launch_leaf_t<12, kPathFast>(p, grid, s)
+                        : launch_leaf_t<12, kPathGeneric>(p, grid, s);
+        case 13:
+            return fast ? launch_leaf_t<13, kPathFast>(p, grid, s)
+                        : launch_leaf_t<13, kPathGeneric>(p, grid, s);
+        default:
+            return fail(POS_EINVAL, "stage count outside this unit");
+    }
+}
+
+}  // namespace pos

@@ -1,0 +1,232 @@
+// Handle life cycle, error state and the cost-table kernel (hot-path step
+// a1: per-class exclusive prefix sums of the Sec. 4.1.3 weights and the
+// Sec. 3.2 memory footprints).
+#include <algorithm>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+
+namespace pos {
+
+static thread_local std::string g_last_error;
+
+void set_error(const std::string &msg) { g_last_error = msg; }
+
+pos_status fail(pos_status st, const std::string &msg) {
+    g_last_error = msg;
+    return st;
+}
+
+pos_status cuda_fail(cudaError_t e, const char *what) {
+    g_last_error = std::string("CUDA error in ") + what + ": " + cudaGetErrorString(e);
+    return e == cudaErrorMemoryAllocation ? POS_ENOMEM : POS_ECUDA;
+}
+
+const char *last_error() { return g_last_error.c_str(); }
+
+int sm_count() {
+    int dev = 0, n = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    return n > 0 ? n : 1;
+}
+
+static int align16(int x) { return (x + 15) & ~15; }
+
+BlobLayout make_layout(int L, int n_types, int n_tp) {
+    BlobLayout ly;
+    ly.L = L;
+    ly.n_types = n_types;
+    ly.n_tp = n_tp;
+    ly.K = n_types * n_tp;
+    const int K = ly.K, Lp1 = L + 1;
+    int off = 0;
+    ly.off_binom = off;
+    off = align16(off + kBinomN * kBinomK * 8);
+    ly.off_Pw = off;
+    off = align16(off + K * Lp1 * 8);
+    ly.off_Pa = off;
+    off = align16(off + K * Lp1 * 8);
+    ly.off_cap = off;
+    off = align16(off + K * 8);
+    ly.off_Pf = off;
+    off = align16(off + K * Lp1 * 4);
+    ly.off_Pb = off;
+    off = align16(off + K * Lp1 * 4);
+    ly.off_Pd = off;
+    off = align16(off + K * Lp1 * 4);
+    ly.off_p2f = off;
+    off = align16(off + K * K * 4);
+    ly.off_p2b = off;
+    off = align16(off + K * K * 4);
+    ly.bytes = off;
+    return ly;
+}
+
+// One thread per (table, class) row: the raw per-layer row sits at entries
+// 1..L of the row; turn it into an exclusive prefix sum with P[0] = 0.
+__global__ void prefix_rows_kernel(unsigned char *blob, BlobLayout ly) {
+    const int K = ly.K, Lp1 = ly.L + 1;
+    const int row = blockIdx.x * blockDim.x + threadIdx.x;
+    if (row >= 5 * K) return;
+    const int table = row / K, k = row % K;
+    if (table < 2) {
+        int64_t *P = reinterpret_cast<int64_t *>(blob + (table == 0 ? ly.off_Pw : ly.off_Pa)) +
+                     (int64_t)k * Lp1;
+        int64_t acc = 0;
+        P[0] = 0;
+        for (int l = 1; l <= ly.L; ++l) {
+            acc += P[l];
+            P[l] = acc;
+        }
+    } else {
+        const int off = table == 2 ? ly.off_Pf : (table == 3 ? ly.off_Pb : ly.off_Pd);
+        int32_t *P = reinterpret_cast<int32_t *>(blob + off) + (int64_t)k * Lp1;
+        int32_t acc = 0;
+        P[0] = 0;
+        for (int l = 1; l <= ly.L; ++l) {
+            acc += P[l];
+            P[l] = acc;
+        }
+    }
+}
+
+pos_status validate_tables(const pos_tables *t) {
+    if (!t) return fail(POS_EINVAL, "tables is NULL");
+    if (t->L < 1 || t->L > POS_MAX_LAYERS) return fail(POS_EINVAL, "L must be in 1..127");
+    if (t->n_types < 1 || t->n_types > POS_MAX_TYPES)
+        return fail(POS_EINVAL, "n_types must be in 1..4");
+    if (t->n_tp < 1 || t->n_tp > POS_MAX_TP) return fail(POS_EINVAL, "n_tp must be in 1..8");
+    if (!t->fwd || !t->bwd || !t->dsync || !t->p2p_f || !t->p2p_b || !t->mem_w || !t->mem_a ||
+        !t->cap)
+        return fail(POS_EINVAL, "a table pointer is NULL");
+    const int K = t->n_types * t->n_tp, L = t->L;
+    for (int k = 0; k < K; ++k) {
+        int64_t sfb = 0, sd = 0, smw = 0, sma = 0;
+        for (int l = 0; l < L; ++l) {
+            const int64_t i = (int64_t)k * L + l;
+            if (t->fwd[i] < 0 || t->bwd[i] < 0 || t->dsync[i] < 0 || t->mem_w[i] < 0 ||
+                t->mem_a[i] < 0)
+                return fail(POS_EINVAL, "negative cost or memory entry");
+            sfb += (int64_t)t->fwd[i] + t->bwd[i];
+            sd += t->dsync[i];
+            smw += t->mem_w[i];
+            sma += t->mem_a[i];
+            if (smw > ((int64_t)1 << 52) || sma > ((int64_t)1 << 52))
+                return fail(POS_EOVERFLOW, "per-class summed memory above 2^52 bytes");
+        }
+        if (sfb >= ((int64_t)1 << 31) || sd >= ((int64_t)1 << 31))
+            return fail(POS_EOVERFLOW, "per-class summed costs reach 2^31");
+        if (t->cap[k] < 0) return fail(POS_EINVAL, "negative capacity");
+    }
+    for (int i = 0; i < K * K; ++i)
+        if (t->p2p_f[i] < 0 || t->p2p_b[i] < 0) return fail(POS_EINVAL, "negative transfer time");
+    return POS_OK;
+}
+
+pos_status create_handle(const pos_tables *t, Handle **out) {
+    pos_status st = validate_tables(t);
+    if (st != POS_OK) return st;
+    const int L = t->L, K = t->n_types * t->n_tp, Lp1 = L + 1;
+    const BlobLayout ly = make_layout(L, t->n_types, t->n_tp);
+    std::vector<unsigned char> host(ly.bytes, 0);
+    // binomials by Pascal's rule (k <= 15 is exact in 64 bits for n <= 127)
+    uint64_t *bn = reinterpret_cast<uint64_t *>(host.data() + ly.off_binom);
+    for (int n = 0; n < kBinomN; ++n)
+        for (int k = 0; k < kBinomK; ++k)
+            bn[n * kBinomK + k] =
+                k == 0 ? 1 : (n == 0 ? 0 : bn[(n - 1) * kBinomK + k - 1] + bn[(n - 1) * kBinomK + k]);
+    // raw rows at entries 1..L; the prefix kernel turns them into sums
+    int64_t *Pw_ = reinterpret_cast<int64_t *>(host.data() + ly.off_Pw);
+    int64_t *Pa_ = reinterpret_cast<int64_t *>(host.data() + ly.off_Pa);
+    int32_t *Pf_ = reinterpret_cast<int32_t *>(host.data() + ly.off_Pf);
+    int32_t *Pb_ = reinterpret_cast<int32_t *>(host.data() + ly.off_Pb);
+    int32_t *Pd_ = reinterpret_cast<int32_t *>(host.data() + ly.off_Pd);
+    for (int k = 0; k < K; ++k)
+        for (int l = 0; l < L; ++l) {
+            const int64_t src = (int64_t)k * L + l, dst = (int64_t)k * Lp1 + l + 1;
+            Pw_[dst] = t->mem_w[src];
+            Pa_[dst] = t->mem_a[src];
+            Pf_[dst] = t->fwd[src];
+            Pb_[dst] = t->bwd[src];
+            Pd_[dst] = t->dsync[src];
+        }
+    std::memcpy(host.data() + ly.off_cap, t->cap, sizeof(int64_t) * K);
+    std::memcpy(host.data() + ly.off_p2f, t->p2p_f, sizeof(int32_t) * K * K);
+    std::memcpy(host.data() + ly.off_p2b, t->p2p_b, sizeof(int32_t) * K * K);
+
+    Handle *h = new (std::nothrow) Handle();
+    if (!h) return fail(POS_ENOMEM, "host allocation failed");
+    h->lay = ly;
+    h->d_blob = nullptr;
+    cudaError_t e = cudaGetDevice(&h->device);
+    if (e == cudaSuccess) e = cudaMalloc(&h->d_blob, ly.bytes);
+    if (e == cudaSuccess) e = cudaMemcpy(h->d_blob, host.data(), ly.bytes, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) {
+        const int rows = 5 * K;
+        prefix_rows_kernel<<<(rows + 127) / 128, 128>>>(static_cast<unsigned char *>(h->d_blob),
+                                                          ly);
+        e = cudaGetLastError();
+    }
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) {
+        if (h->d_blob) cudaFree(h->d_blob);
+        delete h;
+        return cuda_fail(e, "tables upload");
+    }
+    int64_t A = 0, D = 0, P = 0;
+    for (int l = 0; l < L; ++l) {
+        int64_t mfb = 0, md = 0;
+        for (int k = 0; k < K; ++k) {
+            const int64_t i = (int64_t)k * L + l;
+            mfb = std::max<int64_t>(mfb, (int64_t)t->fwd[i] + t->bwd[i]);
+            md = std::max<int64_t>(md, t->dsync[i]);
+        }
+        A += mfb;
+        D += md;
+    }
+    for (int i = 0; i < K * K; ++i)
+        P = std::max<int64_t>(P, std::max(t->p2p_f[i], t->p2p_b[i]));
+    h->guard_A = A;
+    h->guard_D = D;
+    h->guard_P = P;
+    *out = h;
+    return POS_OK;
+}
+
+void destroy_handle(Handle *h) {
+    if (!h) return;
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (cur != h->device) cudaSetDevice(h->device);
+    cudaFree(h->d_blob);
+    if (cur != h->device && cur >= 0) cudaSetDevice(cur);
+    delete h;
+}
+
+}  // namespace pos
+
+extern "C" {
+
+pos_status poseidon_tables_create(const pos_tables *tables, int32_t schedule, void **handle) {
+    if (!handle) return pos::fail(POS_EINVAL, "handle out-pointer is NULL");
+    *handle = nullptr;
+    if (schedule != POS_SCHED_1F1B) return pos::fail(POS_ENOTIMPL, "only 1F1B is implemented");
+    pos::Handle *h = nullptr;
+    const pos_status st = pos::create_handle(tables, &h);
+    if (st == POS_OK) *handle = h;
+    return st;
+}
+
+pos_status poseidon_tables_destroy(void *handle) {
+    if (!handle) return pos::fail(POS_EINVAL, "handle is NULL");
+    pos::destroy_handle(static_cast<pos::Handle *>(handle));
+    return POS_OK;
+}
+
+const char *poseidon_last_error(void) { return pos::last_error(); }
+
+}  // extern "C"
