@@ -1,0 +1,257 @@
+"""Benchmark: the exact parallelism search on the 70B-like heterogeneous
+workload (L=80 layers, S=8 stages, M=32, 3 device types, TP in {1,2,4,8}),
+one poseidon_search call per step through the C ABI.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line.  `value` = DAG makespan evaluations per second of
+search (device time, CUDA events around each step, L2 flushed between
+steps); `time_to_plan_s` = mean step time.  `--impl reference` times the
+CPU oracle on a bounded sample of the same workload instead.
+With torchrun (N > 1) every rank runs an independent replica of the search
+(weak scaling); the step time is the maximum over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import gen  # noqa: E402
+
+WORKLOAD = ("70B-like search: L=80, S=8, M=32, 3 device types (312/125/65 TFLOPS, "
+            "80/32/16 GB, 32/32/64 devices), TP in {1,2,4,8}, D=16/t, stage-type counts "
+            "(2,2,4): 1680 slices, 4.87e12 plans")
+METRIC = "DAG makespan evals/sec (time-to-optimal plan at L=80, S=8)"
+WARMUP_SAMPLES = 65536
+SM_LANES = 128  # INT32 lanes per SM (4 partitions x 32)
+
+
+def dist_env():
+    return int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")), \
+        int(os.environ.get("LOCAL_RANK", "0"))
+
+
+class Clocks:
+    """nvidia-smi sampling during the timed region."""
+
+    def __init__(self, index):
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+        os.makedirs(os.path.dirname(self.path), exist_ok=True)
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(index), f"--query-gpu={q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return None
+        self.proc.terminate()
+        self.proc.wait()
+        self.f.close()
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            p = [x.strip() for x in line.split(",")]
+            if len(p) < 9:
+                continue
+            try:
+                sm.append(float(p[1]))
+                mx = max(mx, float(p[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, p[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def oracle_sample_rate(seconds: float, seed: int = 0):
+    """The CPU oracle (single thread, as it stands) evaluating config-4-shaped
+    plans (S=8, M=32, TP index 3) until `seconds` have elapsed."""
+    import oracle
+    w = gen.config4()
+    tab = oracle.OracleTables.from_workload(w)
+    c = gen.random_candidates(4096, L=w.L, n_types=3, S_range=(8, 8), M_range=(32, 32),
+                              seed=seed)
+    c["tp_idx"] = 3
+    n, t0 = 0, time.perf_counter()
+    while time.perf_counter() - t0 < seconds:
+        oracle.eval_batch(tab, c[:512])
+        n += 512
+    dt = time.perf_counter() - t0
+    return n / dt, n, dt
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return
+    per_step = 2.0
+    for _ in range(args.warmup):
+        oracle_sample_rate(0.2)
+    rates, total_n, total_t = [], 0, 0.0
+    for k in range(args.steps):
+        r, n, dt = oracle_sample_rate(per_step, seed=k)
+        rates.append(r)
+        total_n += n
+        total_t += dt
+    value = total_n / total_t
+    sample = (f"{total_n} config-4 plan evaluations (S=8, M=32, L=80) by the single-threaded "
+              f"CPU oracle, {per_step:.0f} s per step")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "evals/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * total_t / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "int32", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "sample": sample},
+        "cpu_baseline": {"value": value, "unit": "evals/s", "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "evals/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    import paper_2609_06086_gb300 as P
+
+    torch.cuda.set_device(local_rank)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if args.backend == "nccl" else "gloo")
+    w = gen.config4()
+    prob, keep = P.make_problem(w, warmup=WARMUP_SAMPLES, prune=True, seed=0)
+    tab_bytes = sum(a.nbytes for a in keep[0].arrays.values()) + sum(a.nbytes for a in keep[1:])
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.int32, device="cuda")
+
+    for _ in range(args.warmup):
+        P.poseidon_search(prob)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clocks = Clocks(torch.cuda.current_device()) if rank == 0 else None
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    dev_ms, wall_ms, plans = [], [], []
+    agg = dict(evaluated=0, relaxations=0, launches=0, ms_expand=0.0, ms_complete=0.0,
+               ms_leaf=0.0, expand_launches=0, complete_launches=0, leaf_launches=0)
+    for _ in range(args.steps):
+        flush.zero_()  # evict L2 (129 MB) between steps
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        ev0.record()
+        plan, st = P.poseidon_search(prob)
+        ev1.record()
+        torch.cuda.synchronize()
+        wall_ms.append(1e3 * (time.perf_counter() - t0))
+        dev_ms.append(ev0.elapsed_time(ev1))
+        plans.append(plan)
+        for k in agg:
+            agg[k] += st[k]
+    clk = clocks.stop() if clocks else None
+    t_dev = sum(dev_ms)
+    if dist:
+        tt = torch.tensor([t_dev], dtype=torch.float64,
+                          device="cuda" if args.backend == "nccl" else "cpu")
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        t_dev = float(tt.item())
+        dist.barrier()
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        return
+    import json as _json
+    ref = _json.load(open(os.path.join(ROOT, "tests", "golden", "search_plans.json")))["config4"]
+    parity = all(p["global_index"] == ref["plan"]["global_index"] and p["T"] == ref["plan"]["T"]
+                 for p in plans)
+    evals = agg["evaluated"] * world
+    value = evals / (t_dev / 1e3)
+    e2e = evals / (sum(wall_ms) / 1e3)
+    props = torch.cuda.get_device_properties(torch.cuda.current_device())
+    n_sm = props.multi_processor_count
+    # roofline of the dominant kernel kind (device time from events on the
+    # library's stream, accumulated over the timed steps)
+    kinds = {"leaf": agg["ms_leaf"], "expand": agg["ms_expand"], "complete": agg["ms_complete"]}
+    dom = max(kinds, key=kinds.get)
+    mhz = (clk or {}).get("sm_mhz") or 2070.0
+    peak_alu = n_sm * SM_LANES * mhz * 1e6 / 1e12  # Tops/s at the measured SM clock
+    S, M = w.S, w.M_list[0]
+    leaf_ops = 3 * agg["relaxations"] + 9 * S * agg["evaluated"]
+    roof = {"bound": "alu", "kernel": dom, "unit": "Tops/s",
+            "peak": round(peak_alu, 3),
+            "peak_note": f"{n_sm} SMs x {SM_LANES} int32 lanes x {mhz:.0f} MHz (median SM clock "
+                         "under load); derived from unit counts and clocks",
+            "traffic": None}
+    if dom == "leaf":
+        ach = leaf_ops / (agg["ms_leaf"] / 1e3) / 1e12
+        roof.update(achieved=round(ach, 4), frac=round(ach / peak_alu, 4),
+                    ops_per_launch=leaf_ops / max(1, agg["leaf_launches"]))
+    else:
+        roof.update(achieved=None, frac=None)
+    cpu_rate, cpu_n, cpu_t = oracle_sample_rate(args.cpu_seconds)
+    line = {
+        "metric": METRIC, "value": value, "unit": "evals/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": t_dev / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32",
+        "data": "synthetic",
+        "config": {"workload": WORKLOAD, "warmup_samples": WARMUP_SAMPLES,
+                   "prune": "stage-level, Eq. 2", "l2": "flushed (256 MB write) between steps",
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "time_to_plan_s": t_dev / args.steps / 1e3,
+        "relaxations_per_s": agg["relaxations"] * world / (t_dev / 1e3),
+        "evaluations_per_step": agg["evaluated"] / args.steps,
+        "plan": {"T_us": plans[-1]["T"], "global_index": plans[-1]["global_index"],
+                 "tp": plans[-1]["tp"], "D": plans[-1]["D"], "layers": plans[-1]["layers"],
+                 "types": plans[-1]["types"], "matches_oracle": parity},
+        "kernel_ms": {k: round(v / args.steps, 4) for k, v in kinds.items()},
+        "roofline": roof,
+        "cpu_baseline": {"value": cpu_rate, "unit": "evals/s", "cores": 1, "kind": "oracle",
+                         "sample": f"{cpu_n} config-4 plan evaluations (S=8, M=32, L=80) in "
+                                   f"{cpu_t:.1f} s, single-threaded oracle"},
+        "e2e": {"value": e2e, "unit": "evals/s", "h2d_bytes_per_step": int(tab_bytes),
+                "d2h_bytes_per_step": int(P.binding.C.sizeof(P.binding.pos_plan))},
+        "gpu_launches": int(agg["launches"]),
+        "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--backend", choices=["nccl", "gloo"], default="nccl")
+    args = ap.parse_args()
+    rank, world, local_rank = dist_env()
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+    else:
+        run_ours(args, rank, world, local_rank)
+
+
+if __name__ == "__main__":
+    main()

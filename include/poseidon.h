@@ -185,7 +185,10 @@ typedef struct pos_search_stats {
     uint64_t relaxations;       /* DAG node relaxations (2*S*M per evaluation) */
     uint64_t slices, slices_feasible;
     uint64_t launches;          /* kernel launches */
-    double ms_setup, ms_warmup, ms_search, ms_total;
+    double ms_setup, ms_warmup, ms_search, ms_total;  /* host wall clock */
+    /* device time per kernel kind, CUDA events on the search's stream */
+    double ms_expand, ms_complete, ms_leaf;
+    uint64_t expand_launches, complete_launches, leaf_launches;
 } pos_search_stats;
 
 /*

@@ -56,7 +56,10 @@ class pos_search_stats(C.Structure):
     _fields_ = [(n, C.c_uint64) for n in ("evaluated", "warmup_evaluated", "prefixes",
                                           "pruned_bound", "pruned_memory", "relaxations",
                                           "slices", "slices_feasible", "launches")] + \
-               [(n, C.c_double) for n in ("ms_setup", "ms_warmup", "ms_search", "ms_total")]
+               [(n, C.c_double) for n in ("ms_setup", "ms_warmup", "ms_search", "ms_total",
+                                          "ms_expand", "ms_complete", "ms_leaf")] + \
+               [(n, C.c_uint64) for n in ("expand_launches", "complete_launches",
+                                          "leaf_launches")]
 
 
 class PoseidonError(RuntimeError):

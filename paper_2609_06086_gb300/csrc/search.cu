@@ -386,8 +386,14 @@ struct Search {
     unsigned long long *stats = nullptr;
     uint64_t launches = 0;
     pos_status err = POS_OK;
+    // device time per kernel kind (events on `stream`)
+    cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
+    double ms_expand = 0, ms_complete = 0, ms_leaf = 0;
+    uint64_t n_expand = 0, n_complete = 0, n_leaf = 0;
 
     ~Search() {
+        for (cudaEvent_t e : ev)
+            if (e) cudaEventDestroy(e);
         if (stream) cudaStreamDestroy(stream);
         if (h) destroy_handle(h);
     }
@@ -556,19 +562,35 @@ static pos_status process(Search &s, const SliceRec *batch, int M, int x, const 
         const int grid = (int)std::max<long long>(1, std::min<long long>(blocks_needed,
                                                                          s.grid_level));
         s.launches++;
+        POS_CUDA(cudaEventRecord(s.ev[0], s.stream));
         if (last) {
             level_kernel<true><<<grid, kThreads, smem, s.stream>>>(p);
         } else {
             level_kernel<false><<<grid, kThreads, smem, s.stream>>>(p);
         }
         POS_CUDA(cudaGetLastError());
+        POS_CUDA(cudaEventRecord(s.ev[1], s.stream));
         if (last) {
             // evaluate the leaves that fit; the count stays on the device
             if ((st = run_leaves(s, p.leaves, out_count, batch, M, nullptr)) != POS_OK) return st;
+            POS_CUDA(cudaEventRecord(s.ev[2], s.stream));
         }
         unsigned long long cnt[2];
         if ((st = sync_read(s, &cnt[0], out_count, 8)) != POS_OK) return st;
         if ((st = sync_read(s, &cnt[1], n_def, 8)) != POS_OK) return st;
+        float ms_k = 0;
+        POS_CUDA(cudaEventElapsedTime(&ms_k, s.ev[0], s.ev[1]));
+        if (last) {
+            s.ms_complete += ms_k;
+            s.n_complete++;
+            float ms_l = 0;
+            POS_CUDA(cudaEventElapsedTime(&ms_l, s.ev[1], s.ev[2]));
+            s.ms_leaf += ms_l;
+            s.n_leaf++;
+        } else {
+            s.ms_expand += ms_k;
+            s.n_expand++;
+        }
         if (!last) {
             const long long n_out = (long long)std::min<unsigned long long>(cnt[0], s.cap);
             if (n_out > 0) {
@@ -597,6 +619,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     if (st != POS_OK) return st;
     if ((st = create_handle(&p->tables, &s.h)) != POS_OK) return st;
     POS_CUDA(cudaStreamCreateWithFlags(&s.stream, cudaStreamNonBlocking));
+    for (cudaEvent_t &e : s.ev) POS_CUDA(cudaEventCreate(&e));
     s.S = p->S;
     s.L = p->tables.L;
     s.n_tp = p->tables.n_tp;
@@ -801,6 +824,12 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         stats->ms_setup = ms_setup;
         stats->ms_warmup = ms_warm;
         stats->ms_search = ms_search;
+        stats->ms_expand = s.ms_expand;
+        stats->ms_complete = s.ms_complete;
+        stats->ms_leaf = s.ms_leaf;
+        stats->expand_launches = s.n_expand;
+        stats->complete_launches = s.n_complete;
+        stats->leaf_launches = s.n_leaf;
     }
     if (inc.obj == ~0ull) {
         if (stats) stats->ms_total = ms_since(t_start);

@@ -1,0 +1,119 @@
+"""The C ABI without a GPU: the library loads, exports every entry point
+that include/poseidon.h declares, the ctypes structs match the C layout, and
+argument validation rejects bad input before touching the device."""
+import ctypes as C
+import os
+import re
+import subprocess
+import sys
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "poseidon.h")
+
+
+@pytest.fixture(scope="module")
+def P():
+    from paper_2609_06086_gb300 import build
+    build.build()
+    import paper_2609_06086_gb300 as P
+    P.lib()
+    return P
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:pos_status|const char \*)\s*(poseidon_\w+)\(", text,
+                                 re.M)))
+
+
+def test_header_declares_the_binding(P):
+    assert declared_functions() == sorted(P.EXPORTS)
+
+
+def test_every_declared_symbol_is_exported(P):
+    out = subprocess.run(["nm", "-D", "--defined-only", P.binding.LIB_PATH], capture_output=True,
+                         text=True, check=True).stdout
+    syms = set(re.findall(r"\bT (\w+)", out))
+    for f in declared_functions():
+        assert f in syms, f
+
+
+def test_struct_layouts_match_the_header(P, tmp_path):
+    prog = tmp_path / "layout.c"
+    fields = {
+        "pos_tables": [f[0] for f in P.binding.pos_tables._fields_],
+        "pos_candidate": ["map_rank", "type_code", "S", "M", "tp_idx", "pad"],
+        "pos_problem": [f[0] for f in P.binding.pos_problem._fields_],
+        "pos_plan": [f[0] for f in P.binding.pos_plan._fields_],
+        "pos_search_stats": [f[0] for f in P.binding.pos_search_stats._fields_],
+    }
+    lines = ['#include <stdio.h>', '#include <stddef.h>', f'#include "{HEADER}"',
+             "int main(void) {"]
+    for st, fs in fields.items():
+        lines.append(f'printf("{st} %zu\\n", sizeof({st}));')
+        for f in fs:
+            lines.append(f'printf("{st}.{f} %zu\\n", offsetof({st}, {f}));')
+    lines += ["return 0;", "}"]
+    prog.write_text("\n".join(lines))
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-std=c99", "-o", str(exe), str(prog)], check=True)
+    got = dict(l.split() for l in subprocess.run([str(exe)], capture_output=True, text=True,
+                                                  check=True).stdout.splitlines())
+    import gen
+    py = {"pos_tables": P.binding.pos_tables, "pos_problem": P.binding.pos_problem,
+          "pos_plan": P.binding.pos_plan, "pos_search_stats": P.binding.pos_search_stats}
+    for st, cls in py.items():
+        assert int(got[st]) == C.sizeof(cls), st
+        for f in fields[st]:
+            assert int(got[f"{st}.{f}"]) == getattr(cls, f).offset, (st, f)
+    assert int(got["pos_candidate"]) == gen.CANDIDATE_DTYPE.itemsize
+    for f in fields["pos_candidate"]:
+        assert int(got[f"pos_candidate.{f}"]) == gen.CANDIDATE_DTYPE.fields[f][1], f
+
+
+def test_invalid_arguments_rejected_before_the_device(P):
+    L = P.lib()
+    h = C.c_void_p()
+    assert L.poseidon_tables_create(None, 0, C.byref(h)) == P.binding.POS_EINVAL
+    assert b"NULL" in L.poseidon_last_error()
+    import gen
+    w = gen.config1()
+    t = P.Tables.from_workload(w)
+    assert L.poseidon_tables_create(C.byref(t.c), 1, C.byref(h)) == P.binding.POS_ENOTIMPL
+    bad = P.Tables.from_workload(w)
+    bad.arrays["fwd"][0, 0] = -5
+    assert L.poseidon_tables_create(C.byref(bad.c), 0, C.byref(h)) == P.binding.POS_EINVAL
+    big = P.Tables(L=2, n_types=1, n_tp=1, fwd=[[2 ** 30, 2 ** 30]], bwd=[[1, 1]], dsync=[[0, 0]],
+                   p2p_f=[[0]], p2p_b=[[0]], mem_w=[[0, 0]], mem_a=[[0, 0]], cap=[1])
+    assert L.poseidon_tables_create(C.byref(big.c), 0, C.byref(h)) == P.binding.POS_EOVERFLOW
+    assert L.poseidon_eval_batch(None, None, 0, None, None, None) == P.binding.POS_EINVAL
+    plan = P.binding.pos_plan()
+    assert L.poseidon_search(None, C.byref(plan), None) == P.binding.POS_EINVAL
+    prob, keep = P.make_problem(w)
+    prob.S = 17
+    assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
+    prob.S = 2
+    prob.warmup = -1
+    assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
+    with pytest.raises(P.PoseidonError):
+        P.Handle(bad)
+
+
+def test_binding_refuses_to_run_without_the_library(tmp_path, monkeypatch):
+    import paper_2609_06086_gb300.binding as b
+    monkeypatch.setattr(b, "LIB_PATH", str(tmp_path / "missing.so"))
+    monkeypatch.setattr(b, "_lib", None)
+    with pytest.raises(ImportError):
+        b.lib()
+
+
+def test_product_path_does_not_import_the_oracle():
+    src = os.path.join(ROOT, "paper_2609_06086_gb300")
+    for dirpath, _, files in os.walk(src):
+        for f in files:
+            if f.endswith((".py", ".cu", ".cuh", ".h")):
+                text = open(os.path.join(dirpath, f)).read()
+                assert "oracle" not in text.lower(), f

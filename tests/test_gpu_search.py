@@ -1,0 +1,114 @@
+"""poseidon_search on the GPU against the oracle's exact search.  The plan
+(global index, makespan, placement, layers) must be identical."""
+import json
+import os
+import random
+
+import numpy as np
+import pytest
+
+import gen
+from tests.test_oracle import _random_problem
+
+pytestmark = pytest.mark.gpu
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "search_plans.json")
+
+
+@pytest.fixture(scope="module")
+def P():
+    import torch
+    assert torch.cuda.is_available()
+    import paper_2609_06086_gb300 as P
+    P.lib()
+    return P
+
+
+def gpu_search(P, w, **kw):
+    prob, keep = P.make_problem(w, **kw)
+    return P.poseidon_search(prob)
+
+
+def same_plan(a, b):
+    keys = ("global_index", "T", "m_idx", "tp_idx", "M", "D", "place_rank", "map_rank",
+            "types", "layers")
+    return all(a[k] == b[k] for k in keys)
+
+
+@pytest.mark.parametrize("cfg", [1, 2, 3])
+@pytest.mark.parametrize("prune", [True, False])
+def test_configs_match_oracle(P, orc, cfg, prune):
+    w = gen.get_config(cfg)
+    ref, _ = orc.search(w, prune=True, warmup=0)
+    plan, st = gpu_search(P, w, prune=prune, warmup=500, seed=cfg)
+    assert same_plan(plan, ref), (plan, ref)
+    assert st["evaluated"] >= 1
+
+
+def test_config4_matches_stored_oracle_plan(P):
+    """The bench's workload and launch configuration (prune on, warm-up
+    65536 samples); expected plan written by tests/golden/make_search_plans.py."""
+    ref = json.load(open(GOLDEN))["config4"]["plan"]
+    plan, st = gpu_search(P, gen.config4(), prune=True, warmup=65536, seed=0)
+    assert same_plan(plan, ref), (plan, ref)
+    assert st["slices_feasible"] == 420
+
+
+@pytest.mark.parametrize("warmup", [0, 1, 500, 100_000])
+def test_warmup_never_changes_the_plan(P, orc, warmup):
+    w = gen.config2()
+    ref, _ = orc.search(w, prune=False)
+    plan, _ = gpu_search(P, w, prune=True, warmup=warmup, seed=warmup)
+    assert same_plan(plan, ref)
+
+
+@pytest.mark.parametrize("cap", [32, 100, 1000])
+def test_tiny_frontiers_defer_and_still_match(P, orc, cap):
+    for cfg in (2, 3):
+        w = gen.get_config(cfg)
+        ref, _ = orc.search(w, prune=True, warmup=0)
+        plan, _ = gpu_search(P, w, prune=True, warmup=50, frontier_cap=cap)
+        assert same_plan(plan, ref), (cfg, cap)
+
+
+def test_random_small_problems(P, orc):
+    rng = random.Random(23)
+    n_found = 0
+    for seed in range(120):
+        w = _random_problem(rng, seed)
+        ref, _ = orc.search(w, prune=False)
+        try:
+            plan, _ = gpu_search(P, w, prune=bool(seed % 2), warmup=seed % 7, seed=seed)
+        except P.PoseidonError as e:
+            assert e.status == P.binding.POS_EINFEASIBLE and not ref["found"], (seed, e)
+            continue
+        assert ref["found"]
+        assert same_plan(plan, ref), (seed, plan, ref)
+        n_found += 1
+    assert n_found > 60
+
+
+def test_single_stage_and_two_stage(P, orc):
+    w = gen.config1()
+    for S, counts in ((1, None), (2, [1, 1])):
+        w.S = S
+        w.placement = gen.workloads.PLACE_FREE if counts is None else gen.workloads.PLACE_EXACT
+        w.type_counts = counts or []
+        ref, _ = orc.search(w, prune=False)
+        plan, _ = gpu_search(P, w, prune=True, warmup=3)
+        assert same_plan(plan, ref), S
+
+
+def test_infeasible_and_overflow(P):
+    w = gen.config1()
+    w.cap = np.array([1, 1], np.int64)
+    with pytest.raises(P.PoseidonError) as e:
+        gpu_search(P, w)
+    assert e.value.status == P.binding.POS_EINFEASIBLE
+    w = gen.config1()
+    w.M_list = [255]
+    w.fwd = np.full_like(w.fwd, 600_000)
+    w.bwd = np.full_like(w.bwd, 600_000)
+    with pytest.raises(P.PoseidonError) as e:
+        gpu_search(P, w)
+    assert e.value.status == P.binding.POS_EOVERFLOW
