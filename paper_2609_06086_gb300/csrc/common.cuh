@@ -6,6 +6,7 @@
 #include <stdint.h>
 
 #include <string>
+#include <utility>
 
 #include "../../include/poseidon.h"
 
@@ -258,17 +259,54 @@ __host__ __device__ constexpr bool down_last_is_b(int S, int s1, int tau) {
     return (s1 & 1) == 0;
 }
 
-#define POS_RELAX_F(s, clock)                                                           \
-    do {                                                                                \
-        int32_t in_ = (s) > 0 ? Fo[(s) > 0 ? (s)-1 : 0] + w.pf[(s) > 0 ? (s)-1 : 0] : 0; \
-        Fo[s] = max((clock), in_) + w.F[s];                                             \
-    } while (0)
+// One relaxation of stage s (0-based) on the forward or backward side.
+template <int S, int s>
+__device__ __forceinline__ void relax_f(int32_t (&Fo)[S], const StageW<S> &w, int32_t clock) {
+    int32_t in = 0;
+    if constexpr (s > 0) in = Fo[s - 1] + w.pf[s - 1];
+    Fo[s] = max(clock, in) + w.F[s];
+}
+template <int S, int s>
+__device__ __forceinline__ void relax_b(int32_t (&Bo)[S], const StageW<S> &w, int32_t clock) {
+    int32_t in = 0;
+    if constexpr (s + 1 < S) in = Bo[s + 1] + w.pb[s];
+    Bo[s] = max(clock, in) + w.B[s];
+}
 
-#define POS_RELAX_B(s, clock)                                                     \
-    do {                                                                          \
-        int32_t in_ = (s) + 1 < S ? Bo[(s) + 1 < S ? (s) + 1 : 0] + w.pb[s] : 0; \
-        Bo[s] = max((clock), in_) + w.B[s];                                       \
-    } while (0)
+// Ramp op of 1-based stage s1 at level t (UP) or at level 2M + t (DOWN);
+// the clock is the finish of the stage's last op, known at compile time.
+template <int S, bool UP, int t, int s1>
+__device__ __forceinline__ void ramp_op(int32_t (&Fo)[S], int32_t (&Bo)[S], const StageW<S> &w) {
+    constexpr int op = UP ? ramp_up_op(S, s1, t) : ramp_down_op(S, s1, t);
+    constexpr bool last_b = UP ? up_last_is_b(S, s1, t) : down_last_is_b(S, s1, t);
+    constexpr int s = s1 - 1;
+    if constexpr (op == 1) relax_f<S, s>(Fo, w, last_b ? Bo[s] : Fo[s]);
+    else if constexpr (op == 2) relax_b<S, s>(Bo, w, last_b ? Bo[s] : Fo[s]);
+}
+// one level, stages in descending order (i = 0 is stage S)
+template <int S, bool UP, int t, int... i>
+__device__ __forceinline__ void ramp_level(int32_t (&Fo)[S], int32_t (&Bo)[S], const StageW<S> &w,
+                                           std::integer_sequence<int, i...>) {
+    (ramp_op<S, UP, t, S - i>(Fo, Bo, w), ...);
+}
+template <int S, bool UP, int T0, int... t>
+__device__ __forceinline__ void ramp(int32_t (&Fo)[S], int32_t (&Bo)[S], const StageW<S> &w,
+                                     std::integer_sequence<int, t...>) {
+    (ramp_level<S, UP, T0 + t>(Fo, Bo, w, std::make_integer_sequence<int, S>{}), ...);
+}
+// steady level: at level parity P (0 even) stage s1 runs F when s1 has the
+// same parity, B otherwise; an F follows the stage's B and vice versa
+template <int S, int P, int i>
+__device__ __forceinline__ void steady_op(int32_t (&Fo)[S], int32_t (&Bo)[S], const StageW<S> &w) {
+    constexpr int s1 = S - i, s = s1 - 1;
+    if constexpr ((s1 & 1) == P) relax_f<S, s>(Fo, w, Bo[s]);
+    else relax_b<S, s>(Bo, w, Fo[s]);
+}
+template <int S, int P, int... i>
+__device__ __forceinline__ void steady_level(int32_t (&Fo)[S], int32_t (&Bo)[S], const StageW<S> &w,
+                                             std::integer_sequence<int, i...>) {
+    (steady_op<S, P, i>(Fo, Bo, w), ...);
+}
 
 template <int S, int PATH>
 __device__ __forceinline__ int32_t makespan_1f1b(const StageW<S> &w, int M) {
@@ -278,48 +316,16 @@ __device__ __forceinline__ int32_t makespan_1f1b(const StageW<S> &w, int M) {
         Fo[s] = 0;
         Bo[s] = 0;
     }
-    if (PATH == kPathFast) {
-        // ramp-up: levels t = 1 .. 2S-1, stages in descending order
-#pragma unroll
-        for (int t = 1; t <= 2 * S - 1; ++t) {
-#pragma unroll
-            for (int s1 = S; s1 >= 1; --s1) {
-                const int s = s1 - 1;
-                const int op = ramp_up_op(S, s1, t);
-                const int32_t clk = up_last_is_b(S, s1, t) ? Bo[s] : Fo[s];
-                if (op == 1) POS_RELAX_F(s, clk);
-                else if (op == 2) POS_RELAX_B(s, clk);
-            }
-        }
-        // steady state: each step is two levels; at an even level even
-        // stages (1-based) run F and odd stages B, at an odd level the
-        // reverse.  An F follows the stage's B and vice versa.
+    if constexpr (PATH == kPathFast) {
+        // ramp-up: levels 1 .. 2S-1
+        ramp<S, true, 1>(Fo, Bo, w, std::make_integer_sequence<int, 2 * S - 1>{});
+        // steady state: M - S steps of two levels (even, then odd)
         for (int j = 0; j < M - S; ++j) {
-#pragma unroll
-            for (int s1 = S; s1 >= 1; --s1) {
-                const int s = s1 - 1;
-                if ((s1 & 1) == 0) POS_RELAX_F(s, Bo[s]);
-                else POS_RELAX_B(s, Fo[s]);
-            }
-#pragma unroll
-            for (int s1 = S; s1 >= 1; --s1) {
-                const int s = s1 - 1;
-                if ((s1 & 1) == 1) POS_RELAX_F(s, Bo[s]);
-                else POS_RELAX_B(s, Fo[s]);
-            }
+            steady_level<S, 0>(Fo, Bo, w, std::make_integer_sequence<int, S>{});
+            steady_level<S, 1>(Fo, Bo, w, std::make_integer_sequence<int, S>{});
         }
         // ramp-down: levels 2M + tau, tau = 0 .. 2S-2
-#pragma unroll
-        for (int tau = 0; tau <= 2 * S - 2; ++tau) {
-#pragma unroll
-            for (int s1 = S; s1 >= 1; --s1) {
-                const int s = s1 - 1;
-                const int op = ramp_down_op(S, s1, tau);
-                const int32_t clk = down_last_is_b(S, s1, tau) ? Bo[s] : Fo[s];
-                if (op == 1) POS_RELAX_F(s, clk);
-                else if (op == 2) POS_RELAX_B(s, clk);
-            }
-        }
+        ramp<S, false, 0>(Fo, Bo, w, std::make_integer_sequence<int, 2 * S - 1>{});
     } else {
         // every level visits every stage with predicates.  A stage's ops
         // are chained, so its last finish is max(Fo, Bo).
@@ -334,8 +340,10 @@ __device__ __forceinline__ int32_t makespan_1f1b(const StageW<S> &w, int M) {
                                  (!odd && t >= 2 * ws + s1 && t <= 2 * M + s1 - 2);
                 const bool bwd = odd && t >= 2 * S - s1 + 1 && t <= 2 * S - s1 + 2 * M - 1;
                 const int32_t clk = max(Fo[s], Bo[s]);
-                if (fwd) POS_RELAX_F(s, clk);
-                else if (bwd) POS_RELAX_B(s, clk);
+                const int32_t in_f = s > 0 ? Fo[s > 0 ? s - 1 : 0] + w.pf[s > 0 ? s - 1 : 0] : 0;
+                const int32_t in_b = s + 1 < S ? Bo[s + 1 < S ? s + 1 : 0] + w.pb[s] : 0;
+                if (fwd) Fo[s] = max(clk, in_f) + w.F[s];
+                else if (bwd) Bo[s] = max(clk, in_b) + w.B[s];
             }
         }
     }
