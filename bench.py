@@ -34,6 +34,11 @@ WORKLOAD = ("70B-like search: L=80, S=8, M=32, 3 device types (312/125/65 TFLOPS
 METRIC = "DAG makespan evals/sec (time-to-optimal plan at L=80, S=8)"
 WARMUP_SAMPLES = 65536
 SM_LANES = 128  # INT32 lanes per SM (4 partitions x 32)
+# integer ops of one child test in the level kernels: memory check 5 (2 sub,
+# mul, add, cmp), bound 10 (3 sub, add, mul, max, 2 add, mul, cmp),
+# feasibility bit 2; completion checks two stages (5 + 10 + 5 + 12)
+OPS_PER_EXPAND_TEST = 17
+OPS_PER_COMPLETE_TEST = 32
 
 
 def dist_env():
@@ -140,7 +145,8 @@ def run_ours(args, rank, world, local_rank):
         import torch.distributed as dist
         dist.init_process_group("nccl" if args.backend == "nccl" else "gloo")
     w = gen.config4()
-    prob, keep = P.make_problem(w, warmup=WARMUP_SAMPLES, prune=True, seed=0)
+    prob, keep = P.make_problem(w, warmup=WARMUP_SAMPLES, prune=True, seed=0,
+                                frontier_cap=args.frontier_cap)
     tab_bytes = sum(a.nbytes for a in keep[0].arrays.values()) + sum(a.nbytes for a in keep[1:])
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.int32, device="cuda")
 
@@ -153,7 +159,8 @@ def run_ours(args, rank, world, local_rank):
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     dev_ms, wall_ms, plans = [], [], []
     agg = dict(evaluated=0, relaxations=0, launches=0, ms_expand=0.0, ms_complete=0.0,
-               ms_leaf=0.0, expand_launches=0, complete_launches=0, leaf_launches=0)
+               ms_leaf=0.0, expand_launches=0, complete_launches=0, leaf_launches=0,
+               tests_expand=0, tests_complete=0)
     for _ in range(args.steps):
         flush.zero_()  # evict L2 (129 MB) between steps
         torch.cuda.synchronize()
@@ -194,19 +201,24 @@ def run_ours(args, rank, world, local_rank):
     dom = max(kinds, key=kinds.get)
     mhz = (clk or {}).get("sm_mhz") or 2070.0
     peak_alu = n_sm * SM_LANES * mhz * 1e6 / 1e12  # Tops/s at the measured SM clock
-    S, M = w.S, w.M_list[0]
-    leaf_ops = 3 * agg["relaxations"] + 9 * S * agg["evaluated"]
+    S = w.S
+    # algorithmic int32 ops per unit (roofline section)
+    ops = {"leaf": 3 * agg["relaxations"] + 9 * S * agg["evaluated"],
+           "expand": OPS_PER_EXPAND_TEST * agg["tests_expand"],
+           "complete": OPS_PER_COMPLETE_TEST * agg["tests_complete"]}
+    launches = {"leaf": agg["leaf_launches"], "expand": agg["expand_launches"],
+                "complete": agg["complete_launches"]}
     roof = {"bound": "alu", "kernel": dom, "unit": "Tops/s",
             "peak": round(peak_alu, 3),
             "peak_note": f"{n_sm} SMs x {SM_LANES} int32 lanes x {mhz:.0f} MHz (median SM clock "
                          "under load); derived from unit counts and clocks",
             "traffic": None}
-    if dom == "leaf":
-        ach = leaf_ops / (agg["ms_leaf"] / 1e3) / 1e12
-        roof.update(achieved=round(ach, 4), frac=round(ach / peak_alu, 4),
-                    ops_per_launch=leaf_ops / max(1, agg["leaf_launches"]))
-    else:
-        roof.update(achieved=None, frac=None)
+    ach = ops[dom] / (kinds[dom] / 1e3) / 1e12
+    roof.update(achieved=round(ach, 4), frac=round(ach / peak_alu, 5),
+                ops_per_launch=ops[dom] / max(1, launches[dom]))
+    per_kind = {k: {"ms_per_step": round(kinds[k] / args.steps, 4),
+                    "launches_per_step": launches[k] / args.steps,
+                    "tops": round(ops[k] / max(kinds[k], 1e-9) / 1e9, 4)} for k in kinds}
     cpu_rate, cpu_n, cpu_t = oracle_sample_rate(args.cpu_seconds)
     line = {
         "metric": METRIC, "value": value, "unit": "evals/s", "n_gpus": world,
@@ -222,7 +234,7 @@ def run_ours(args, rank, world, local_rank):
         "plan": {"T_us": plans[-1]["T"], "global_index": plans[-1]["global_index"],
                  "tp": plans[-1]["tp"], "D": plans[-1]["D"], "layers": plans[-1]["layers"],
                  "types": plans[-1]["types"], "matches_oracle": parity},
-        "kernel_ms": {k: round(v / args.steps, 4) for k, v in kinds.items()},
+        "kernels": per_kind,
         "roofline": roof,
         "cpu_baseline": {"value": cpu_rate, "unit": "evals/s", "cores": 1, "kind": "oracle",
                          "sample": f"{cpu_n} config-4 plan evaluations (S=8, M=32, L=80) in "
@@ -245,6 +257,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--backend", choices=["nccl", "gloo"], default="nccl")
+    ap.add_argument("--frontier-cap", type=int, default=0,
+                    help="frontier entries per depth (0 = library default)")
     args = ap.parse_args()
     rank, world, local_rank = dist_env()
     if args.impl == "reference":

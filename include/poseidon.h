@@ -164,7 +164,8 @@ typedef struct pos_problem {
     int32_t prune;              /* 1: stage-level prune g(S_x) > T_min (Eq. 2); 0: exhaustive */
     uint64_t seed;              /* warm-up sampling seed */
     int32_t schedule;           /* POS_SCHED_1F1B */
-    int64_t frontier_cap;       /* entries per frontier buffer; 0 = default */
+    int64_t frontier_cap;       /* entries per frontier buffer; 0 = default 2^26;
+                                   raised to at least 32*L */
 } pos_problem;
 
 typedef struct pos_plan {
@@ -189,6 +190,8 @@ typedef struct pos_search_stats {
     /* device time per kernel kind, CUDA events on the search's stream */
     double ms_expand, ms_complete, ms_leaf;
     uint64_t expand_launches, complete_launches, leaf_launches;
+    /* child tests (memory + bound + feasibility checks) per kernel kind */
+    uint64_t tests_expand, tests_complete;
 } pos_search_stats;
 
 /*

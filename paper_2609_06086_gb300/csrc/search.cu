@@ -332,6 +332,8 @@ __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
     }
     if (lane == 0) {
         if (!COMPLETE && emitted) atomicAdd(p.stats + kStPrefixes, emitted);
+        if (emitted + cb + cm)
+            atomicAdd(p.stats + (COMPLETE ? kStTestsComplete : kStTestsExpand), emitted + cb + cm);
         if (cb) atomicAdd(p.stats + kStPrunedBound, cb);
         if (cm) atomicAdd(p.stats + kStPrunedMemory, cm);
     }
@@ -600,6 +602,8 @@ static pos_status process(Search &s, const SliceRec *batch, int M, int x, const 
             }
         }
         if (cnt[1] == 0) break;
+        if ((long long)cnt[1] >= n_work)
+            return fail(POS_ENOMEM, "frontier capacity too small to make progress");
         work = static_cast<const uint32_t *>(s.d_defer[2 * x + flip].p);
         n_work = (long long)cnt[1];
         flip ^= 1;
@@ -624,7 +628,11 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     s.L = p->tables.L;
     s.n_tp = p->tables.n_tp;
     s.n_map = host_binom(s.L - 1, s.S - 1);
+    // a warp group of 32 parents has at most 32*L children, so a buffer of
+    // at least that size always accepts the first group of a pass: every
+    // deferral pass makes progress
     s.cap = p->frontier_cap > 0 ? p->frontier_cap : (1ll << 26);
+    s.cap = std::max<long long>(s.cap, 32LL * s.L);
     if ((st = enumerate_places(s)) != POS_OK) return st;
     const uint64_t n_slices64 = (uint64_t)p->n_M * s.n_tp * s.n_place;
     if (n_slices64 > (1ull << 22)) return fail(POS_EINVAL, "more than 2^22 slices");
@@ -830,6 +838,8 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         stats->expand_launches = s.n_expand;
         stats->complete_launches = s.n_complete;
         stats->leaf_launches = s.n_leaf;
+        stats->tests_expand = hs[kStTestsExpand];
+        stats->tests_complete = hs[kStTestsComplete];
     }
     if (inc.obj == ~0ull) {
         if (stats) stats->ms_total = ms_since(t_start);

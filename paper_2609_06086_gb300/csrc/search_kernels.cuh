@@ -51,6 +51,8 @@ enum {
     kStEvaluated,
     kStTimeout,
     kStRelaxations,
+    kStTestsExpand,
+    kStTestsComplete,
     kStCount
 };
 

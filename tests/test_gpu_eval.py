@@ -99,7 +99,8 @@ def test_overflow_guard_flagged(P, orc):
     T, F = eval_device(P, h, c)
     Tr, Fr = orc.eval_batch(orc.OracleTables(**big), c)
     assert np.array_equal(T, Tr) and np.array_equal(F, Fr)
-    assert F.tolist() == [1, 3, 3, 3]
+    # U(2, M) = M * 2^29: evaluable up to M = 3, flagged from M = 4
+    assert F.tolist() == [1, 1, 3, 3]
 
 
 def test_nondefault_stream_and_host_variant(P, orc):
