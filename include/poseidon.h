@@ -143,6 +143,28 @@ pos_status poseidon_argmin(const int32_t *d_makespan, const uint8_t *d_feasible,
                            int64_t *d_out, void *stream);
 
 /*
+ * poseidon_argmin_noalloc: same inputs, output and result as poseidon_argmin,
+ * for callers that cannot allocate device memory during a call -- a process
+ * whose device memory belongs to another allocator (a framework's caching
+ * allocator holding the free memory, or a service that reserves everything
+ * at start-up and forbids allocation afterwards).  The paper has no
+ * counterpart; this is a library convenience.
+ * It allocates nothing: its per-block partial results live in a fixed
+ * 64 KB array of device global memory (4096 partial results) that every GPU
+ * loading the library holds until the process exits.  The first call on a
+ * device looks up that array's device address (cudaGetSymbolAddress) with
+ * the device current; make that first call before any stream capture.
+ * All calls on a device share the array and it keeps the last call's
+ * contents (every slot a call reads is written earlier in the same call, so
+ * nothing needs clearing); calls that overlap on the GPU, e.g. on two
+ * streams at once, race on it.  Errors: POS_EINVAL for bad arguments or
+ * when the GPU would need more than 4096 partial results (more than 1024
+ * SMs), POS_ECUDA for a failed address lookup or launch.
+ */
+pos_status poseidon_argmin_noalloc(const int32_t *d_makespan, const uint8_t *d_feasible,
+                                   int64_t n, int64_t *d_out, void *stream);
+
+/*
  * Search problem (Sec. 4.2.3): choose M from M_list, a TP index, a
  * device-type-to-stage placement and a layer composition for S stages.
  * Slices are (m_idx, tp_idx, placement) in this nesting order; placements

@@ -25,8 +25,8 @@ MAX_STAGES = 16
 
 # the exported entry points, as declared in include/poseidon.h
 EXPORTS = ["poseidon_tables_create", "poseidon_tables_destroy", "poseidon_eval_batch",
-           "poseidon_eval_batch_host", "poseidon_argmin", "poseidon_search",
-           "poseidon_last_error"]
+           "poseidon_eval_batch_host", "poseidon_argmin", "poseidon_argmin_noalloc",
+           "poseidon_search", "poseidon_last_error"]
 
 
 class pos_tables(C.Structure):
@@ -84,6 +84,7 @@ def lib():
         L.poseidon_eval_batch.argtypes = [vp, vp, i64, vp, vp, vp]
         L.poseidon_eval_batch_host.argtypes = [vp, vp, i64, vp, vp]
         L.poseidon_argmin.argtypes = [vp, vp, i64, vp, vp]
+        L.poseidon_argmin_noalloc.argtypes = [vp, vp, i64, vp, vp]
         L.poseidon_search.argtypes = [C.POINTER(pos_problem), C.POINTER(pos_plan),
                                       C.POINTER(pos_search_stats)]
         L.poseidon_last_error.restype = C.c_char_p
@@ -160,6 +161,12 @@ def poseidon_eval_batch_host(handle: Handle, cands: np.ndarray):
 
 def poseidon_argmin(d_makespan: int, d_feasible: int, n: int, d_out: int, stream: int = 0):
     _check(lib().poseidon_argmin(d_makespan, d_feasible, n, d_out, stream))
+
+
+def poseidon_argmin_noalloc(d_makespan: int, d_feasible: int, n: int, d_out: int,
+                            stream: int = 0):
+    """poseidon_argmin without device allocation (fixed scratch in the library)."""
+    _check(lib().poseidon_argmin_noalloc(d_makespan, d_feasible, n, d_out, stream))
 
 
 def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0):
