@@ -160,7 +160,7 @@ def run_ours(args, rank, world, local_rank):
     dev_ms, wall_ms, plans = [], [], []
     agg = dict(evaluated=0, relaxations=0, launches=0, ms_expand=0.0, ms_complete=0.0,
                ms_leaf=0.0, expand_launches=0, complete_launches=0, leaf_launches=0,
-               tests_expand=0, tests_complete=0)
+               tests_expand=0, tests_complete=0, ms_setup=0.0, ms_warmup=0.0, ms_search=0.0)
     for _ in range(args.steps):
         flush.zero_()  # evict L2 (129 MB) between steps
         torch.cuda.synchronize()
@@ -235,6 +235,8 @@ def run_ours(args, rank, world, local_rank):
                  "tp": plans[-1]["tp"], "D": plans[-1]["D"], "layers": plans[-1]["layers"],
                  "types": plans[-1]["types"], "matches_oracle": parity},
         "kernels": per_kind,
+        "host_ms_per_step": {k: round(agg[k] / args.steps, 3)
+                             for k in ("ms_setup", "ms_warmup", "ms_search")},
         "roofline": roof,
         "cpu_baseline": {"value": cpu_rate, "unit": "evals/s", "cores": 1, "kind": "oracle",
                          "sample": f"{cpu_n} config-4 plan evaluations (S=8, M=32, L=80) in "

@@ -175,14 +175,47 @@ __device__ __forceinline__ void carries(const Tab &t, const SliceRec &sr, const 
     }
 }
 
-// Children of one parent at depth x (x <= S-3).  WRITE=false counts them;
-// WRITE=true writes them from out+pos.  Both passes take the same decisions
-// (the incumbent does not change while expansion kernels run).
-template <bool WRITE>
-__device__ int expand_one(const ExpandParams &p, const Tab &t, const Prefix &pr, uint64_t thr,
-                          unsigned long long pos, unsigned long long &cut_bound,
-                          unsigned long long &cut_mem) {
-    if (pr.slice == kPrefixHole) return 0;
+// 128-bit set of cut positions 0..127.
+struct Bits128 {
+    uint32_t w[4];
+};
+
+__device__ __forceinline__ Bits128 range_bits(int lo, int hi) {  // positions lo..hi
+    Bits128 r;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int a = max(lo - 32 * i, 0), b = min(hi - 32 * i, 31);
+        r.w[i] = (a > b) ? 0u : ((b == 31 ? 0xffffffffu : ((1u << (b + 1)) - 1u)) & ~((1u << a) - 1u));
+    }
+    return r;
+}
+
+__device__ __forceinline__ int popc128(const Bits128 &b) {
+    return __popc(b.w[0]) + __popc(b.w[1]) + __popc(b.w[2]) + __popc(b.w[3]);
+}
+
+// Largest l in [0, hi] with pred(l), for pred true up to some l and false
+// after (pred(0) is taken as true).
+template <class Pred>
+__device__ __forceinline__ int last_true(int hi, Pred pred) {
+    int lo = 0;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (pred(mid)) lo = mid;
+        else hi = mid - 1;
+    }
+    return lo;
+}
+
+// Children of one parent, as the set of new cut positions c2 = c + l.
+// Expansion (parent depth x <= S-3): stage x takes l layers.  Its memory
+// need and g(S_{x+1}) both grow with l, so the admissible l form a prefix
+// [1, hi] found by binary search; the children are the positions in
+// (c, c+hi] from which the remaining layers still fit the remaining stages
+// (feasibility bits).
+__device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, const Prefix &pr,
+                                          uint64_t thr, Bits128 &acc, unsigned long long &cut_b,
+                                          unsigned long long &cut_m) {
     const SliceRec &sr = p.slices[pr.slice];
     const int S = p.S, M = p.M, x = p.x, L = t.L();
     int64_t A, Bm;
@@ -190,43 +223,35 @@ __device__ int expand_one(const ExpandParams &p, const Tab &t, const Prefix &pr,
     carries(t, sr, pr.cut, x, A, Bm, c);
     const int k = sr.cls[x];
     const uint64_t scale = sr.scale;
-    int n = 0;
-    for (int l = 1; c + l <= L - (S - x - 1); ++l) {
-        const int c2 = c + l;
-        if (!stage_fits(t, S, M, x, k, c, c2)) {
-            ++cut_mem;
-            break;
-        }
-        if (p.prune) {
+    const int lmax = L - c - (S - x - 1);
+    const int hi_mem = last_true(lmax, [&](int l) { return stage_fits(t, S, M, x, k, c, c + l); });
+    int hi = hi_mem;
+    if (p.prune)
+        hi = last_true(hi_mem, [&](int l) {
+            const int c2 = c + l;
             const int64_t F = Pf(t, k, c2) - Pf(t, k, c), B = Pb(t, k, c2) - Pb(t, k, c);
             const int64_t d = Pd(t, k, c2) - Pd(t, k, c);
-            const int64_t g = A + (int64_t)M * (F + B) + max(Bm, d);
-            if ((uint64_t)g * scale > thr) {
-                ++cut_bound;
-                break;
-            }
-        }
-        if (!feas_bit(p.feas, S, sr.gid, x + 1, c2)) {
-            ++cut_mem;
-            continue;
-        }
-        if (WRITE) {
-            Prefix ch = pr;
-            ch.cut[x] = (uint8_t)c2;
-            p.out[pos + n] = ch;
-        }
-        ++n;
-    }
+            return (uint64_t)(A + (int64_t)M * (F + B) + max(Bm, d)) * scale <= thr;
+        });
+    const uint4 f = __ldg(p.feas + (size_t)sr.gid * (S + 1) + x + 1);
+    const Bits128 win = range_bits(c + 1, c + hi);
+    acc.w[0] = f.x & win.w[0];
+    acc.w[1] = f.y & win.w[1];
+    acc.w[2] = f.z & win.w[2];
+    acc.w[3] = f.w & win.w[3];
+    const int n = popc128(acc);
+    cut_m += (unsigned long long)(lmax - hi_mem) + (unsigned long long)(hi - n);
+    cut_b += (unsigned long long)(hi_mem - hi);
     return n;
 }
 
-// Complete plans from one parent at depth S-2: choose l_{S-1}; stage S-1
-// takes the rest.  Checks memory of both stages and g(S_{S-1}), g(S_S).
-template <bool WRITE>
-__device__ int complete_one(const ExpandParams &p, const Tab &t, const Prefix &pr, uint64_t thr,
-                            unsigned long long pos, unsigned long long &cut_bound,
-                            unsigned long long &cut_mem) {
-    if (pr.slice == kPrefixHole) return 0;
+// Completion (parent depth S-2): stage a = S-2 takes l layers, stage
+// b = S-1 the rest.  Stage a's memory and g(S_{S-1}) bound l from above,
+// stage b's memory from below (fewer layers as l grows); inside that window
+// each l is checked against g(S_S).
+__device__ __forceinline__ int complete_set(const ExpandParams &p, const Tab &t, const Prefix &pr,
+                                            uint64_t thr, Bits128 &acc, unsigned long long &cut_b,
+                                            unsigned long long &cut_m) {
     const SliceRec &sr = p.slices[pr.slice];
     const int S = p.S, M = p.M, L = t.L(), a = S - 2, b = S - 1;
     int64_t A, Bm;
@@ -234,47 +259,47 @@ __device__ int complete_one(const ExpandParams &p, const Tab &t, const Prefix &p
     carries(t, sr, pr.cut, a, A, Bm, c);
     const int ka = sr.cls[a], kb = sr.cls[b];
     const uint64_t scale = sr.scale;
+    const int lmax = L - c - 1;
+    const int hi_mem = last_true(lmax, [&](int l) { return stage_fits(t, S, M, a, ka, c, c + l); });
+    int hi = hi_mem;
+    if (p.prune)
+        hi = last_true(hi_mem, [&](int l) {
+            const int c2 = c + l;
+            const int64_t F = Pf(t, ka, c2) - Pf(t, ka, c), B = Pb(t, ka, c2) - Pb(t, ka, c);
+            const int64_t d = Pd(t, ka, c2) - Pd(t, ka, c);
+            return (uint64_t)(A + (int64_t)M * (F + B) + max(Bm, d)) * scale <= thr;
+        });
+    // smallest l in [1, hi] whose remainder fits stage b (hi + 1 if none)
+    const int lo = 1 + last_true(hi, [&](int l) {
+                       return l == 0 ? true : !stage_fits(t, S, M, b, kb, c + l, L);
+                   });
+    for (int i = 0; i < 4; ++i) acc.w[i] = 0;
     int n = 0;
-    for (int l = 1; c + l <= L - 1; ++l) {
+    for (int l = lo; l <= hi; ++l) {
         const int c2 = c + l;
-        if (!stage_fits(t, S, M, a, ka, c, c2)) {
-            ++cut_mem;
-            break;
-        }
-        const int64_t Fa = Pf(t, ka, c2) - Pf(t, ka, c), Ba = Pb(t, ka, c2) - Pb(t, ka, c);
-        const int64_t da = Pd(t, ka, c2) - Pd(t, ka, c);
-        if (p.prune && (uint64_t)(A + (int64_t)M * (Fa + Ba) + max(Bm, da)) * scale > thr) {
-            ++cut_bound;
-            break;
-        }
-        if (!stage_fits(t, S, M, b, kb, c2, L)) {
-            ++cut_mem;
-            continue;
-        }
         if (p.prune) {
+            const int64_t Fa = Pf(t, ka, c2) - Pf(t, ka, c), Ba = Pb(t, ka, c2) - Pb(t, ka, c);
+            const int64_t da = Pd(t, ka, c2) - Pd(t, ka, c);
             const int64_t Fb = Pf(t, kb, L) - Pf(t, kb, c2), Bb = Pb(t, kb, L) - Pb(t, kb, c2);
             const int64_t db = Pd(t, kb, L) - Pd(t, kb, c2);
             const int64_t g = A + Fa + (int64_t)M * (Fb + Bb) + max(max(Bm, da) + Ba, db);
             if ((uint64_t)g * scale > thr) {
-                ++cut_bound;
+                ++cut_b;
                 continue;
             }
         }
-        if (WRITE) {
-            Leaf lf;
-            lf.slice = pr.slice;
-            for (int s = 0; s < 16; ++s) lf.cut[s] = s < 14 ? (s < a ? pr.cut[s] : 0) : 0;
-            lf.cut[a] = (uint8_t)c2;
-            lf.pad[0] = lf.pad[1] = lf.pad[2] = 0;
-            p.leaves[pos + n] = lf;
-        }
+        acc.w[c2 >> 5] |= 1u << (c2 & 31);
         ++n;
     }
+    cut_m += (unsigned long long)(lmax - hi_mem) + (unsigned long long)(lo - 1 < hi ? lo - 1 : hi);
+    cut_b += (unsigned long long)(hi_mem - hi);
     return n;
 }
 
-// One warp per group of 32 consecutive parents: count, reserve output slots
-// with one atomic, write -- or, when the output is full, defer the group.
+// One warp per group of 32 consecutive parents: each lane finds its
+// parent's children (a 128-bit set of cut positions), the warp reserves
+// output slots with one atomic and writes them -- or, when the output is
+// full, marks its reserved slots as holes and defers the group.
 template <bool COMPLETE>
 __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
@@ -293,9 +318,12 @@ __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
         Prefix pr;
         pr.slice = kPrefixHole;
         if (i < p.n_in) pr = p.in[i];
-        unsigned long long dummy_b = 0, dummy_m = 0;
-        const int n = COMPLETE ? complete_one<false>(p, t, pr, thr, 0, dummy_b, dummy_m)
-                               : expand_one<false>(p, t, pr, thr, 0, dummy_b, dummy_m);
+        Bits128 acc = {{0u, 0u, 0u, 0u}};
+        unsigned long long lb = 0, lm = 0;
+        int n = 0;
+        if (pr.slice != kPrefixHole)
+            n = COMPLETE ? complete_set(p, t, pr, thr, acc, lb, lm)
+                         : expand_set(p, t, pr, thr, acc, lb, lm);
         int incl = n;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -306,17 +334,42 @@ __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
         unsigned long long base = 0;
         if (lane == 0 && total > 0) base = atomicAdd(p.out_count, (unsigned long long)total);
         base = __shfl_sync(0xffffffffu, base, 0);
-        if (total == 0) continue;
-        const unsigned long long my = base + (unsigned long long)(incl - n);
+        if (total == 0) {
+            cb += lb;
+            cm += lm;
+            continue;
+        }
+        unsigned long long q = base + (unsigned long long)(incl - n);
         if (base + (unsigned long long)total <= p.cap) {
-            if (COMPLETE) complete_one<true>(p, t, pr, thr, my, cb, cm);
-            else expand_one<true>(p, t, pr, thr, my, cb, cm);
+#pragma unroll
+            for (int wd = 0; wd < 4; ++wd) {
+                uint32_t m = acc.w[wd];
+                while (m) {
+                    const int c2 = 32 * wd + __ffs(m) - 1;
+                    m &= m - 1;
+                    if (COMPLETE) {
+                        Leaf lf;
+                        lf.slice = pr.slice;
+#pragma unroll
+                        for (int s2 = 0; s2 < 16; ++s2) lf.cut[s2] = s2 < 14 ? pr.cut[s2 < 14 ? s2 : 0] : 0;
+                        lf.cut[p.S - 2] = (uint8_t)c2;
+                        lf.pad[0] = lf.pad[1] = lf.pad[2] = 0;
+                        p.leaves[q++] = lf;
+                    } else {
+                        Prefix ch = pr;
+                        ch.cut[p.x] = (uint8_t)c2;
+                        p.out[q++] = ch;
+                    }
+                }
+            }
             emitted += n;
+            cb += lb;
+            cm += lm;
         } else {
             // no room: mark this warp's reserved slots below cap as holes
-            for (unsigned long long q = my; q < my + (unsigned long long)n && q < p.cap; ++q) {
-                if (COMPLETE) p.leaves[q].slice = kLeafHole;
-                else p.out[q].slice = kPrefixHole;
+            for (unsigned long long e = q; e < q + (unsigned long long)n && e < p.cap; ++e) {
+                if (COMPLETE) p.leaves[e].slice = kLeafHole;
+                else p.out[e].slice = kPrefixHole;
             }
             if (lane == 0) {
                 const unsigned long long d = atomicAdd(p.n_deferred, 1ull);
@@ -332,10 +385,10 @@ __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
     }
     if (lane == 0) {
         if (!COMPLETE && emitted) atomicAdd(p.stats + kStPrefixes, emitted);
-        if (emitted + cb + cm)
-            atomicAdd(p.stats + (COMPLETE ? kStTestsComplete : kStTestsExpand), emitted + cb + cm);
         if (cb) atomicAdd(p.stats + kStPrunedBound, cb);
         if (cm) atomicAdd(p.stats + kStPrunedMemory, cm);
+        if (emitted + cb + cm)
+            atomicAdd(p.stats + (COMPLETE ? kStTestsComplete : kStTestsExpand), emitted + cb + cm);
     }
 }
 
@@ -540,14 +593,14 @@ static pos_status process(Search &s, const SliceRec *batch, int M, int x, const 
     pos_status st = ensure_defer(s, x, all_groups);
     if (st != POS_OK) return st;
     if (!last && (st = ensure_depth(s, x + 1)) != POS_OK) return st;
-    unsigned long long *out_count = last ? s.ctr + 32 : s.ctr + (x + 1);
-    unsigned long long *n_def = s.ctr + 16 + x;
+    // (children count, deferred groups) of this depth, adjacent: one read
+    unsigned long long *out_count = s.ctr + 2 * x;
+    unsigned long long *n_def = out_count + 1;
     const uint32_t *work = nullptr;
     long long n_work = all_groups;
     int flip = 0;
     for (;;) {
-        POS_CUDA(cudaMemsetAsync(out_count, 0, sizeof(unsigned long long), s.stream));
-        POS_CUDA(cudaMemsetAsync(n_def, 0, sizeof(unsigned long long), s.stream));
+        POS_CUDA(cudaMemsetAsync(out_count, 0, 2 * sizeof(unsigned long long), s.stream));
         ExpandParams p = base_params(s, batch, M);
         p.in = in;
         p.n_in = n_in;
@@ -578,8 +631,7 @@ static pos_status process(Search &s, const SliceRec *batch, int M, int x, const 
             POS_CUDA(cudaEventRecord(s.ev[2], s.stream));
         }
         unsigned long long cnt[2];
-        if ((st = sync_read(s, &cnt[0], out_count, 8)) != POS_OK) return st;
-        if ((st = sync_read(s, &cnt[1], n_def, 8)) != POS_OK) return st;
+        if ((st = sync_read(s, cnt, out_count, sizeof(cnt))) != POS_OK) return st;
         float ms_k = 0;
         POS_CUDA(cudaEventElapsedTime(&ms_k, s.ev[0], s.ev[1]));
         if (last) {
@@ -684,7 +736,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     POS_CUDA(s.d_best.reserve(sizeof(unsigned long long) * n_slices));
     POS_CUDA(s.d_leaves.reserve(sizeof(Leaf) * (size_t)s.cap));
     s.ctr = static_cast<unsigned long long *>(s.d_ctr.p);
-    s.stats = s.ctr + 40;
+    s.stats = s.ctr + 40;  // ctr[0..33]: per-depth counters, ctr[36]: leaf count
     POS_CUDA(cudaMemcpyAsync(s.d_slices.p, s.slices.data(), sizeof(SliceRec) * n_slices,
                              cudaMemcpyHostToDevice, s.stream));
     POS_CUDA(cudaMemsetAsync(s.d_inc.p, 0xff, sizeof(Key128), s.stream));
@@ -735,8 +787,8 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
             POS_CUDA(cudaGetLastError());
             s.launches++;
             unsigned long long cnt = (unsigned long long)n_s;
-            POS_CUDA(cudaMemcpyAsync(s.ctr + 33, &cnt, 8, cudaMemcpyHostToDevice, s.stream));
-            if ((st = run_leaves(s, static_cast<const Leaf *>(s.d_leaves.p), s.ctr + 33, d_all,
+            POS_CUDA(cudaMemcpyAsync(s.ctr + 36, &cnt, 8, cudaMemcpyHostToDevice, s.stream));
+            if ((st = run_leaves(s, static_cast<const Leaf *>(s.d_leaves.p), s.ctr + 36, d_all,
                                  p->M_list[mi], static_cast<unsigned long long *>(s.d_best.p))) !=
                 POS_OK)
                 return st;
@@ -789,8 +841,8 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
                 POS_CUDA(cudaMemcpyAsync(s.d_leaves.p, lv.data(), sizeof(Leaf) * nb,
                                          cudaMemcpyHostToDevice, s.stream));
                 unsigned long long cnt = nb;
-                POS_CUDA(cudaMemcpyAsync(s.ctr + 33, &cnt, 8, cudaMemcpyHostToDevice, s.stream));
-                if ((st = run_leaves(s, static_cast<const Leaf *>(s.d_leaves.p), s.ctr + 33,
+                POS_CUDA(cudaMemcpyAsync(s.ctr + 36, &cnt, 8, cudaMemcpyHostToDevice, s.stream));
+                if ((st = run_leaves(s, static_cast<const Leaf *>(s.d_leaves.p), s.ctr + 36,
                                      d_batch, M, nullptr)) != POS_OK)
                     return st;
                 POS_CUDA(cudaStreamSynchronize(s.stream));
