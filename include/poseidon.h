@@ -186,7 +186,7 @@ typedef struct pos_problem {
     int32_t prune;              /* 1: stage-level prune g(S_x) > T_min (Eq. 2); 0: exhaustive */
     uint64_t seed;              /* warm-up sampling seed */
     int32_t schedule;           /* POS_SCHED_1F1B */
-    int64_t frontier_cap;       /* entries per frontier buffer; 0 = default 2^26;
+    int64_t frontier_cap;       /* entries per frontier buffer; 0 = default 2^24;
                                    raised to at least 32*L */
 } pos_problem;
 
@@ -227,6 +227,11 @@ typedef struct pos_search_stats {
  * has found = 0).
  * Limits: at most 65535 slices with a feasible root per M value; the global
  * index must fit in 64 bits; lcm of all D*M below 2^32.
+ * Memory: the work buffers (one frontier of frontier_cap 32-byte entries per
+ * depth, a leaf buffer of the same length, slice and feasibility tables),
+ * a stream and pinned counters are kept per device between calls, grown on
+ * demand and released at process exit; concurrent searches on one device
+ * are serialised.
  */
 pos_status poseidon_search(const pos_problem *problem, pos_plan *out, pos_search_stats *stats);
 

@@ -7,6 +7,7 @@
 
 #include <string>
 #include <utility>
+#include <vector>
 
 #include "../../include/poseidon.h"
 
@@ -55,6 +56,11 @@ struct Handle {
 
 pos_status validate_tables(const pos_tables *t);
 pos_status create_handle(const pos_tables *t, Handle **out);
+// host part of create_handle: validated blob with raw rows, plus guard terms
+pos_status build_blob(const pos_tables *t, std::vector<unsigned char> &host, BlobLayout &ly,
+                      int64_t &guard_A, int64_t &guard_D, int64_t &guard_P);
+// device part: per-class prefix sums in place, asynchronous on `stream`
+pos_status launch_prefix_rows(void *d_blob, const BlobLayout &ly, cudaStream_t stream);
 void destroy_handle(Handle *h);
 int sm_count();
 

@@ -15,6 +15,8 @@
 //     deferred and re-expanded after the part that fit has been finished.
 #include <algorithm>
 #include <chrono>
+#include <mutex>
+#include <new>
 #include <cstring>
 #include <numeric>
 #include <vector>
@@ -158,23 +160,6 @@ struct ExpandParams {
     BlobLayout lay;
 };
 
-// Stage totals of placed stages 0..x-1 give the two carries of Eq. 2:
-//   A  = sum_{i<x} F_i,   Bm = max_{i<x} (sum_{j=i}^{x-1} B_j + d_i)
-// (Bm = -1 when x = 0; every d is >= 0).  For a new stage x with (F, B, d):
-//   g(S_{x+1}) = A + M (F + B) + max(Bm, d).
-__device__ __forceinline__ void carries(const Tab &t, const SliceRec &sr, const uint8_t *cut,
-                                        int x, int64_t &A, int64_t &Bm, int &c) {
-    A = 0;
-    Bm = -1;
-    c = 0;
-    for (int i = 0; i < x; ++i) {
-        const int k = sr.cls[i], c2 = cut[i];
-        A += Pf(t, k, c2) - Pf(t, k, c);
-        Bm = max(Bm, (int64_t)(Pd(t, k, c2) - Pd(t, k, c))) + (Pb(t, k, c2) - Pb(t, k, c));
-        c = c2;
-    }
-}
-
 // 128-bit set of cut positions 0..127.
 struct Bits128 {
     uint32_t w[4];
@@ -218,9 +203,8 @@ __device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, c
                                           unsigned long long &cut_m) {
     const SliceRec &sr = p.slices[pr.slice];
     const int S = p.S, M = p.M, x = p.x, L = t.L();
-    int64_t A, Bm;
-    int c;
-    carries(t, sr, pr.cut, x, A, Bm, c);
+    const int64_t A = pr.A, Bm = pr.Bm;
+    const int c = x > 0 ? pr.cut[x > 0 ? x - 1 : 0] : 0;
     const int k = sr.cls[x];
     const uint64_t scale = sr.scale;
     const int lmax = L - c - (S - x - 1);
@@ -254,9 +238,8 @@ __device__ __forceinline__ int complete_set(const ExpandParams &p, const Tab &t,
                                             unsigned long long &cut_m) {
     const SliceRec &sr = p.slices[pr.slice];
     const int S = p.S, M = p.M, L = t.L(), a = S - 2, b = S - 1;
-    int64_t A, Bm;
-    int c;
-    carries(t, sr, pr.cut, a, A, Bm, c);
+    const int64_t A = pr.A, Bm = pr.Bm;
+    const int c = a > 0 ? pr.cut[a > 0 ? a - 1 : 0] : 0;
     const int ka = sr.cls[a], kb = sr.cls[b];
     const uint64_t scale = sr.scale;
     const int lmax = L - c - 1;
@@ -356,8 +339,14 @@ __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
                         lf.pad[0] = lf.pad[1] = lf.pad[2] = 0;
                         p.leaves[q++] = lf;
                     } else {
+                        // parent cut c and class k of the new stage x
+                        const int x = p.x;
+                        const int c = x > 0 ? pr.cut[x > 0 ? x - 1 : 0] : 0;
+                        const int k = p.slices[pr.slice].cls[x];
                         Prefix ch = pr;
-                        ch.cut[p.x] = (uint8_t)c2;
+                        ch.cut[x] = (uint8_t)c2;
+                        ch.A = pr.A + (Pf(t, k, c2) - Pf(t, k, c));
+                        ch.Bm = max(pr.Bm, Pd(t, k, c2) - Pd(t, k, c)) + (Pb(t, k, c2) - Pb(t, k, c));
                         p.out[q++] = ch;
                     }
                 }
@@ -424,34 +413,71 @@ struct DevBuf {
     }
 };
 
-struct Search {
-    const pos_problem *pb = nullptr;
-    Handle *h = nullptr;
+// Device work buffers, stream and events of one GPU, kept between calls
+// (grown on demand) so that a search allocates and frees nothing in the
+// steady state.  Searches on the same device are serialised by `mu`.
+struct Workspace {
+    std::mutex mu;
     cudaStream_t stream = nullptr;
+    cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
+    DevBuf blob, d_slices, d_feas, d_batch, d_inc, d_ctr, d_best, d_feasible, d_leaves, d_roots,
+        d_root;
+    DevBuf d_front[POS_MAX_STAGES + 1];        // per depth: Prefix buffers
+    DevBuf d_defer[2 * (POS_MAX_STAGES + 1)];  // per depth: two deferred group lists
+    unsigned long long *h_cnt = nullptr;       // pinned host counters
+};
+
+constexpr int kMaxDevices = 64;
+static std::mutex g_ws_mutex;
+static Workspace *g_ws[kMaxDevices];
+
+static pos_status get_workspace(Workspace **out) {
+    int dev = 0;
+    POS_CUDA(cudaGetDevice(&dev));
+    if (dev < 0 || dev >= kMaxDevices) return fail(POS_EINVAL, "device index above 63");
+    std::lock_guard<std::mutex> lock(g_ws_mutex);
+    if (!g_ws[dev]) {
+        Workspace *w = new (std::nothrow) Workspace();
+        if (!w) return fail(POS_ENOMEM, "host allocation failed");
+        cudaError_t e = cudaStreamCreateWithFlags(&w->stream, cudaStreamNonBlocking);
+        for (int i = 0; i < 3 && e == cudaSuccess; ++i) e = cudaEventCreate(&w->ev[i]);
+        if (e == cudaSuccess) e = cudaMallocHost(&w->h_cnt, 64 * sizeof(unsigned long long));
+        if (e != cudaSuccess) {
+            delete w;
+            return cuda_fail(e, "search workspace");
+        }
+        g_ws[dev] = w;
+    }
+    *out = g_ws[dev];
+    return POS_OK;
+}
+
+struct Search {
+    Workspace &ws;
+    explicit Search(Workspace &w) : ws(w), stream(w.stream), ev(w.ev), d_slices(w.d_slices),
+        d_feas(w.d_feas), d_batch(w.d_batch), d_inc(w.d_inc), d_ctr(w.d_ctr), d_best(w.d_best),
+        d_feasible(w.d_feasible), d_leaves(w.d_leaves), d_roots(w.d_roots), d_root(w.d_root),
+        d_front(w.d_front), d_defer(w.d_defer) {}
+    const pos_problem *pb = nullptr;
+    Handle hd{};
+    Handle *h = &hd;
+    cudaStream_t stream;
+    cudaEvent_t (&ev)[3];
     int S = 0, L = 0, n_tp = 0;
     uint64_t n_map = 0, n_place = 0;
     long long cap = 0;
     int grid_level = 0, grid_leaf = 0;
     std::vector<std::vector<int>> places;
     std::vector<SliceRec> slices;
-    DevBuf d_slices, d_feas, d_batch, d_inc, d_ctr, d_best, d_feasible, d_leaves, d_roots;
-    DevBuf d_front[POS_MAX_STAGES + 1];      // per depth: Prefix buffers
-    DevBuf d_defer[2 * (POS_MAX_STAGES + 1)];  // per depth: two deferred group lists
-    unsigned long long *ctr = nullptr;  // [0..15] out counts per depth, [16..31] deferred, [32] leaves
+    DevBuf &d_slices, &d_feas, &d_batch, &d_inc, &d_ctr, &d_best, &d_feasible, &d_leaves,
+        &d_roots, &d_root;
+    DevBuf (&d_front)[POS_MAX_STAGES + 1];
+    DevBuf (&d_defer)[2 * (POS_MAX_STAGES + 1)];
+    unsigned long long *ctr = nullptr;  // device counters, see search_impl
     unsigned long long *stats = nullptr;
     uint64_t launches = 0;
-    pos_status err = POS_OK;
-    // device time per kernel kind (events on `stream`)
-    cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
     double ms_expand = 0, ms_complete = 0, ms_leaf = 0;
     uint64_t n_expand = 0, n_complete = 0, n_leaf = 0;
-
-    ~Search() {
-        for (cudaEvent_t e : ev)
-            if (e) cudaEventDestroy(e);
-        if (stream) cudaStreamDestroy(stream);
-        if (h) destroy_handle(h);
-    }
 };
 
 static pos_status validate_problem(const pos_problem *p) {
@@ -533,6 +559,12 @@ static void host_unrank(int L, int S, uint64_t rank, int32_t *layers) {
 }
 
 static pos_status sync_read(Search &s, void *dst, const void *src, size_t bytes) {
+    if (bytes <= 64 * sizeof(unsigned long long)) {  // small reads through pinned memory
+        POS_CUDA(cudaMemcpyAsync(s.ws.h_cnt, src, bytes, cudaMemcpyDeviceToHost, s.stream));
+        POS_CUDA(cudaStreamSynchronize(s.stream));
+        std::memcpy(dst, s.ws.h_cnt, bytes);
+        return POS_OK;
+    }
     POS_CUDA(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToHost, s.stream));
     POS_CUDA(cudaStreamSynchronize(s.stream));
     return POS_OK;
@@ -673,9 +705,17 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     const pos_problem *p = s.pb;
     pos_status st = validate_problem(p);
     if (st != POS_OK) return st;
-    if ((st = create_handle(&p->tables, &s.h)) != POS_OK) return st;
-    POS_CUDA(cudaStreamCreateWithFlags(&s.stream, cudaStreamNonBlocking));
-    for (cudaEvent_t &e : s.ev) POS_CUDA(cudaEventCreate(&e));
+    {
+        std::vector<unsigned char> host;
+        st = build_blob(&p->tables, host, s.hd.lay, s.hd.guard_A, s.hd.guard_D, s.hd.guard_P);
+        if (st != POS_OK) return st;
+        POS_CUDA(cudaGetDevice(&s.hd.device));
+        POS_CUDA(s.ws.blob.reserve(s.hd.lay.bytes));
+        s.hd.d_blob = s.ws.blob.p;
+        POS_CUDA(cudaMemcpyAsync(s.hd.d_blob, host.data(), s.hd.lay.bytes, cudaMemcpyHostToDevice,
+                                 s.stream));
+        if ((st = launch_prefix_rows(s.hd.d_blob, s.hd.lay, s.stream)) != POS_OK) return st;
+    }
     s.S = p->S;
     s.L = p->tables.L;
     s.n_tp = p->tables.n_tp;
@@ -683,7 +723,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     // a warp group of 32 parents has at most 32*L children, so a buffer of
     // at least that size always accepts the first group of a pass: every
     // deferral pass makes progress
-    s.cap = p->frontier_cap > 0 ? p->frontier_cap : (1ll << 26);
+    s.cap = p->frontier_cap > 0 ? p->frontier_cap : (1ll << 24);
     s.cap = std::max<long long>(s.cap, 32LL * s.L);
     if ((st = enumerate_places(s)) != POS_OK) return st;
     const uint64_t n_slices64 = (uint64_t)p->n_M * s.n_tp * s.n_place;
@@ -747,7 +787,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         d_all, n_slices, s.S, static_cast<uint4 *>(s.d_feas.p), s.h->d_blob, s.h->lay);
     POS_CUDA(cudaGetLastError());
     s.launches++;
-    DevBuf d_root;
+    DevBuf &d_root = s.d_root;
     POS_CUDA(d_root.reserve(n_slices));
     root_bits_kernel<<<(n_slices + 255) / 256, 256, 0, s.stream>>>(
         static_cast<const uint4 *>(s.d_feas.p), n_slices, s.S, static_cast<uint8_t *>(d_root.p));
@@ -852,6 +892,8 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
             for (size_t j = 0; j < nb; ++j) {
                 std::memset(&roots[j], 0, sizeof(Prefix));
                 roots[j].slice = (uint16_t)j;
+                roots[j].A = 0;
+                roots[j].Bm = -1;  // no stage placed yet
             }
             POS_CUDA(cudaMemcpyAsync(s.d_roots.p, roots.data(), sizeof(Prefix) * nb,
                                      cudaMemcpyHostToDevice, s.stream));
@@ -924,10 +966,17 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
 extern "C" pos_status poseidon_search(const pos_problem *problem, pos_plan *out,
                                       pos_search_stats *stats) {
     if (!out) return pos::fail(POS_EINVAL, "plan out-pointer is NULL");
-    pos::Search s;
-    s.pb = problem;
     pos::set_error("");
+    pos_status st = pos::validate_problem(problem);  // before touching the device
+    if (st == POS_OK) st = pos::validate_tables(&problem->tables);
+    if (st != POS_OK) return st;
+    pos::Workspace *ws = nullptr;
+    st = pos::get_workspace(&ws);
+    if (st != POS_OK) return st;
+    std::lock_guard<std::mutex> lock(ws->mu);
     try {
+        pos::Search s(*ws);
+        s.pb = problem;
         return pos::search_impl(s, out, stats);
     } catch (...) {
         return pos::fail(POS_ENOMEM, "host exception (allocation failure)");

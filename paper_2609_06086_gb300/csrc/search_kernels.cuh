@@ -26,11 +26,17 @@ static_assert(sizeof(SliceRec) == 48, "SliceRec layout");
 
 // Partial plan at depth x: stages 0..x-1 placed; cut[i] = layers of stages
 // 0..i.  slice indexes the current batch's slice table; 0xffff = hole.
+// A and Bm are the two partial sums of Eq. 2 over the placed stages,
+//   A = sum_{i<x} F_i,   Bm = max_{i<x} (sum_{j=i}^{x-1} B_j + d_i)
+// (Bm = -1 at depth 0; every d is >= 0), so that for a new stage x with
+// totals (F, B, d):  g(S_{x+1}) = A + M (F + B) + max(Bm, d).
 struct Prefix {
     uint16_t slice;
     uint8_t cut[14];
+    int32_t A, Bm;
+    uint32_t pad[2];
 };
-static_assert(sizeof(Prefix) == 16, "Prefix layout");
+static_assert(sizeof(Prefix) == 32, "Prefix layout");
 
 // Complete plan: cut[0..S-2]; slice indexes the slice table of the launch.
 struct Leaf {

@@ -127,19 +127,20 @@ pos_status validate_tables(const pos_tables *t) {
     return POS_OK;
 }
 
-pos_status create_handle(const pos_tables *t, Handle **out) {
+pos_status build_blob(const pos_tables *t, std::vector<unsigned char> &host, BlobLayout &ly,
+                      int64_t &guard_A, int64_t &guard_D, int64_t &guard_P) {
     pos_status st = validate_tables(t);
     if (st != POS_OK) return st;
     const int L = t->L, K = t->n_types * t->n_tp, Lp1 = L + 1;
-    const BlobLayout ly = make_layout(L, t->n_types, t->n_tp);
-    std::vector<unsigned char> host(ly.bytes, 0);
+    ly = make_layout(L, t->n_types, t->n_tp);
+    host.assign(ly.bytes, 0);
     // binomials by Pascal's rule (k <= 15 is exact in 64 bits for n <= 127)
     uint64_t *bn = reinterpret_cast<uint64_t *>(host.data() + ly.off_binom);
     for (int n = 0; n < kBinomN; ++n)
         for (int k = 0; k < kBinomK; ++k)
             bn[n * kBinomK + k] =
                 k == 0 ? 1 : (n == 0 ? 0 : bn[(n - 1) * kBinomK + k - 1] + bn[(n - 1) * kBinomK + k]);
-    // raw rows at entries 1..L; the prefix kernel turns them into sums
+    // raw rows at entries 1..L; prefix_rows_kernel turns them into sums
     int64_t *Pw_ = reinterpret_cast<int64_t *>(host.data() + ly.off_Pw);
     int64_t *Pa_ = reinterpret_cast<int64_t *>(host.data() + ly.off_Pa);
     int32_t *Pf_ = reinterpret_cast<int32_t *>(host.data() + ly.off_Pf);
@@ -157,26 +158,6 @@ pos_status create_handle(const pos_tables *t, Handle **out) {
     std::memcpy(host.data() + ly.off_cap, t->cap, sizeof(int64_t) * K);
     std::memcpy(host.data() + ly.off_p2f, t->p2p_f, sizeof(int32_t) * K * K);
     std::memcpy(host.data() + ly.off_p2b, t->p2p_b, sizeof(int32_t) * K * K);
-
-    Handle *h = new (std::nothrow) Handle();
-    if (!h) return fail(POS_ENOMEM, "host allocation failed");
-    h->lay = ly;
-    h->d_blob = nullptr;
-    cudaError_t e = cudaGetDevice(&h->device);
-    if (e == cudaSuccess) e = cudaMalloc(&h->d_blob, ly.bytes);
-    if (e == cudaSuccess) e = cudaMemcpy(h->d_blob, host.data(), ly.bytes, cudaMemcpyHostToDevice);
-    if (e == cudaSuccess) {
-        const int rows = 5 * K;
-        prefix_rows_kernel<<<(rows + 127) / 128, 128>>>(static_cast<unsigned char *>(h->d_blob),
-                                                          ly);
-        e = cudaGetLastError();
-    }
-    if (e == cudaSuccess) e = cudaDeviceSynchronize();
-    if (e != cudaSuccess) {
-        if (h->d_blob) cudaFree(h->d_blob);
-        delete h;
-        return cuda_fail(e, "tables upload");
-    }
     int64_t A = 0, D = 0, P = 0;
     for (int l = 0; l < L; ++l) {
         int64_t mfb = 0, md = 0;
@@ -190,9 +171,43 @@ pos_status create_handle(const pos_tables *t, Handle **out) {
     }
     for (int i = 0; i < K * K; ++i)
         P = std::max<int64_t>(P, std::max(t->p2p_f[i], t->p2p_b[i]));
+    guard_A = A;
+    guard_D = D;
+    guard_P = P;
+    return POS_OK;
+}
+
+pos_status launch_prefix_rows(void *d_blob, const BlobLayout &ly, cudaStream_t stream) {
+    const int rows = 5 * ly.K;
+    prefix_rows_kernel<<<(rows + 127) / 128, 128, 0, stream>>>(
+        static_cast<unsigned char *>(d_blob), ly);
+    POS_CUDA(cudaGetLastError());
+    return POS_OK;
+}
+
+pos_status create_handle(const pos_tables *t, Handle **out) {
+    std::vector<unsigned char> host;
+    BlobLayout ly;
+    int64_t A, D, P;
+    pos_status st = build_blob(t, host, ly, A, D, P);
+    if (st != POS_OK) return st;
+    Handle *h = new (std::nothrow) Handle();
+    if (!h) return fail(POS_ENOMEM, "host allocation failed");
+    h->lay = ly;
+    h->d_blob = nullptr;
     h->guard_A = A;
     h->guard_D = D;
     h->guard_P = P;
+    cudaError_t e = cudaGetDevice(&h->device);
+    if (e == cudaSuccess) e = cudaMalloc(&h->d_blob, ly.bytes);
+    if (e == cudaSuccess) e = cudaMemcpy(h->d_blob, host.data(), ly.bytes, cudaMemcpyHostToDevice);
+    if (e == cudaSuccess && launch_prefix_rows(h->d_blob, ly, 0) != POS_OK) e = cudaErrorLaunchFailure;
+    if (e == cudaSuccess) e = cudaStreamSynchronize(0);
+    if (e != cudaSuccess) {
+        if (h->d_blob) cudaFree(h->d_blob);
+        delete h;
+        return cuda_fail(e, "tables upload");
+    }
     *out = h;
     return POS_OK;
 }
