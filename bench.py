@@ -34,11 +34,15 @@ WORKLOAD = ("70B-like search: L=80, S=8, M=32, 3 device types (312/125/65 TFLOPS
 METRIC = "DAG makespan evals/sec (time-to-optimal plan at L=80, S=8)"
 WARMUP_SAMPLES = 65536
 SM_LANES = 128  # INT32 lanes per SM (4 partitions x 32)
-# integer ops of one child test in the level kernels: memory check 5 (2 sub,
-# mul, add, cmp), bound 10 (3 sub, add, mul, max, 2 add, mul, cmp),
-# feasibility bit 2; completion checks two stages (5 + 10 + 5 + 12)
-OPS_PER_EXPAND_TEST = 17
-OPS_PER_COMPLETE_TEST = 32
+ENTRY_BYTES = 32  # one frontier entry / one complete plan
+
+
+def measured_hbm():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        return float(json.load(open(path))["hbm_gbs"]), "measured copy bandwidth (MEASURED_PEAKS.json)"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback 6.8 TB/s (MEASURED_PEAKS.json absent)"
 
 
 def dist_env():
@@ -160,7 +164,8 @@ def run_ours(args, rank, world, local_rank):
     dev_ms, wall_ms, plans = [], [], []
     agg = dict(evaluated=0, relaxations=0, launches=0, ms_expand=0.0, ms_complete=0.0,
                ms_leaf=0.0, expand_launches=0, complete_launches=0, leaf_launches=0,
-               tests_expand=0, tests_complete=0, ms_setup=0.0, ms_warmup=0.0, ms_search=0.0)
+               parents_expand=0, parents_complete=0, leaves=0, prefixes=0,
+               ms_setup=0.0, ms_warmup=0.0, ms_search=0.0)
     for _ in range(args.steps):
         flush.zero_()  # evict L2 (129 MB) between steps
         torch.cuda.synchronize()
@@ -201,24 +206,33 @@ def run_ours(args, rank, world, local_rank):
     dom = max(kinds, key=kinds.get)
     mhz = (clk or {}).get("sm_mhz") or 2070.0
     peak_alu = n_sm * SM_LANES * mhz * 1e6 / 1e12  # Tops/s at the measured SM clock
+    peak_hbm, hbm_src = measured_hbm()
     S = w.S
-    # algorithmic int32 ops per unit (roofline section)
-    ops = {"leaf": 3 * agg["relaxations"] + 9 * S * agg["evaluated"],
-           "expand": OPS_PER_EXPAND_TEST * agg["tests_expand"],
-           "complete": OPS_PER_COMPLETE_TEST * agg["tests_complete"]}
     launches = {"leaf": agg["leaf_launches"], "expand": agg["expand_launches"],
                 "complete": agg["complete_launches"]}
-    roof = {"bound": "alu", "kernel": dom, "unit": "Tops/s",
-            "peak": round(peak_alu, 3),
-            "peak_note": f"{n_sm} SMs x {SM_LANES} int32 lanes x {mhz:.0f} MHz (median SM clock "
-                         "under load); derived from unit counts and clocks",
-            "traffic": None}
-    ach = ops[dom] / (kinds[dom] / 1e3) / 1e12
-    roof.update(achieved=round(ach, 4), frac=round(ach / peak_alu, 5),
-                ops_per_launch=ops[dom] / max(1, launches[dom]))
-    per_kind = {k: {"ms_per_step": round(kinds[k] / args.steps, 4),
-                    "launches_per_step": launches[k] / args.steps,
-                    "tops": round(ops[k] / max(kinds[k], 1e-9) / 1e9, 4)} for k in kinds}
+    # algorithmic work per kind (roofline section):
+    #  leaf     : int32 ops, 3 per DAG node relaxation + 9 per stage
+    #  expand   : bytes, a 32-byte frontier entry read per parent and written per child
+    #  complete : bytes, a 32-byte entry read per parent and a 32-byte plan written per leaf
+    work = {"leaf": 3 * agg["relaxations"] + 9 * S * agg["evaluated"],
+            "expand": ENTRY_BYTES * (agg["parents_expand"] + agg["prefixes"]),
+            "complete": ENTRY_BYTES * (agg["parents_complete"] + agg["leaves"])}
+    bound = {"leaf": ("alu", "Tops/s", peak_alu, 1e12),
+             "expand": ("hbm", "GB/s", peak_hbm, 1e9),
+             "complete": ("hbm", "GB/s", peak_hbm, 1e9)}
+    per_kind = {}
+    for k in kinds:
+        b, unit, peak, scale = bound[k]
+        ach = work[k] / max(kinds[k] / 1e3, 1e-12) / scale
+        per_kind[k] = {"ms_per_step": round(kinds[k] / args.steps, 4),
+                       "launches_per_step": launches[k] / args.steps, "bound": b,
+                       "achieved": round(ach, 3), "unit": unit, "frac": round(ach / peak, 4)}
+    b, unit, peak, scale = bound[dom]
+    roof = {"bound": b, "kernel": dom, "unit": unit, "peak": round(peak, 3),
+            "achieved": per_kind[dom]["achieved"], "frac": per_kind[dom]["frac"],
+            "work_per_launch": work[dom] / max(1, launches[dom]), "traffic": None,
+            "peak_note": (f"{n_sm} SMs x {SM_LANES} int32 lanes x {mhz:.0f} MHz (median SM "
+                          "clock under load)" if b == "alu" else hbm_src)}
     cpu_rate, cpu_n, cpu_t = oracle_sample_rate(args.cpu_seconds)
     line = {
         "metric": METRIC, "value": value, "unit": "evals/s", "n_gpus": world,
@@ -231,6 +245,7 @@ def run_ours(args, rank, world, local_rank):
         "time_to_plan_s": t_dev / args.steps / 1e3,
         "relaxations_per_s": agg["relaxations"] * world / (t_dev / 1e3),
         "evaluations_per_step": agg["evaluated"] / args.steps,
+        "frontier_entries_per_step": agg["prefixes"] / args.steps,
         "plan": {"T_us": plans[-1]["T"], "global_index": plans[-1]["global_index"],
                  "tp": plans[-1]["tp"], "D": plans[-1]["D"], "layers": plans[-1]["layers"],
                  "types": plans[-1]["types"], "matches_oracle": parity},

@@ -212,8 +212,9 @@ typedef struct pos_search_stats {
     /* device time per kernel kind, CUDA events on the search's stream */
     double ms_expand, ms_complete, ms_leaf;
     uint64_t expand_launches, complete_launches, leaf_launches;
-    /* child tests (memory + bound + feasibility checks) per kernel kind */
-    uint64_t tests_expand, tests_complete;
+    /* frontier entries read by the expansion / completion kernels, and
+       complete plans written by the completion kernel */
+    uint64_t parents_expand, parents_complete, leaves;
 } pos_search_stats;
 
 /*

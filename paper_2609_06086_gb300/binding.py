@@ -59,7 +59,8 @@ class pos_search_stats(C.Structure):
                [(n, C.c_double) for n in ("ms_setup", "ms_warmup", "ms_search", "ms_total",
                                           "ms_expand", "ms_complete", "ms_leaf")] + \
                [(n, C.c_uint64) for n in ("expand_launches", "complete_launches",
-                                          "leaf_launches", "tests_expand", "tests_complete")]
+                                          "leaf_launches", "parents_expand", "parents_complete",
+                                          "leaves")]
 
 
 class PoseidonError(RuntimeError):

@@ -192,6 +192,44 @@ __device__ __forceinline__ int last_true(int hi, Pred pred) {
     return lo;
 }
 
+// Per-parent quantities shared by the search for children and the writes:
+// parent cut c, class k of the new stage, prefix sums at c.
+struct ParentCtx {
+    int c, k;
+    int32_t f0, b0, d0;
+};
+
+__device__ __forceinline__ ParentCtx parent_ctx(const Tab &t, int k, int c) {
+    ParentCtx q;
+    q.c = c;
+    q.k = k;
+    q.f0 = Pf(t, k, c);
+    q.b0 = Pb(t, k, c);
+    q.d0 = Pd(t, k, c);
+    return q;
+}
+
+// largest l in [0, lmax] with stage s (class k) fitting layers [c, c+l)
+__device__ __forceinline__ int mem_limit(const Tab &t, int S, int M, int s, int k, int c,
+                                         int lmax) {
+    const int64_t w0 = Pw(t, k, c), a0 = Pa(t, k, c), cap = cap_of(t, k);
+    const int64_t fl = inflight(S, M, s);
+    return last_true(lmax, [&](int l) {
+        return (Pw(t, k, c + l) - w0) + fl * (Pa(t, k, c + l) - a0) <= cap;
+    });
+}
+
+// largest l in [0, hi] with g = A + M (F + B) + max(Bm, d) <= thr / scale
+__device__ __forceinline__ int bound_limit(const Tab &t, const ParentCtx &q, int M, int64_t A,
+                                           int64_t Bm, uint64_t scale, uint64_t thr, int hi) {
+    return last_true(hi, [&](int l) {
+        const int c2 = q.c + l;
+        const int64_t F = Pf(t, q.k, c2) - q.f0, B = Pb(t, q.k, c2) - q.b0;
+        const int64_t d = Pd(t, q.k, c2) - q.d0;
+        return (uint64_t)(A + (int64_t)M * (F + B) + max(Bm, d)) * scale <= thr;
+    });
+}
+
 // Children of one parent, as the set of new cut positions c2 = c + l.
 // Expansion (parent depth x <= S-3): stage x takes l layers.  Its memory
 // need and g(S_{x+1}) both grow with l, so the admissible l form a prefix
@@ -199,26 +237,15 @@ __device__ __forceinline__ int last_true(int hi, Pred pred) {
 // (c, c+hi] from which the remaining layers still fit the remaining stages
 // (feasibility bits).
 __device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, const Prefix &pr,
+                                          const ParentCtx &q, uint32_t gid, uint64_t scale,
                                           uint64_t thr, Bits128 &acc, unsigned long long &cut_b,
                                           unsigned long long &cut_m) {
-    const SliceRec &sr = p.slices[pr.slice];
     const int S = p.S, M = p.M, x = p.x, L = t.L();
-    const int64_t A = pr.A, Bm = pr.Bm;
-    const int c = x > 0 ? pr.cut[x > 0 ? x - 1 : 0] : 0;
-    const int k = sr.cls[x];
-    const uint64_t scale = sr.scale;
-    const int lmax = L - c - (S - x - 1);
-    const int hi_mem = last_true(lmax, [&](int l) { return stage_fits(t, S, M, x, k, c, c + l); });
-    int hi = hi_mem;
-    if (p.prune)
-        hi = last_true(hi_mem, [&](int l) {
-            const int c2 = c + l;
-            const int64_t F = Pf(t, k, c2) - Pf(t, k, c), B = Pb(t, k, c2) - Pb(t, k, c);
-            const int64_t d = Pd(t, k, c2) - Pd(t, k, c);
-            return (uint64_t)(A + (int64_t)M * (F + B) + max(Bm, d)) * scale <= thr;
-        });
-    const uint4 f = __ldg(p.feas + (size_t)sr.gid * (S + 1) + x + 1);
-    const Bits128 win = range_bits(c + 1, c + hi);
+    const int lmax = L - q.c - (S - x - 1);
+    const int hi_mem = mem_limit(t, S, M, x, q.k, q.c, lmax);
+    const int hi = p.prune ? bound_limit(t, q, M, pr.A, pr.Bm, scale, thr, hi_mem) : hi_mem;
+    const uint4 f = __ldg(p.feas + (size_t)gid * (S + 1) + x + 1);
+    const Bits128 win = range_bits(q.c + 1, q.c + hi);
     acc.w[0] = f.x & win.w[0];
     acc.w[1] = f.y & win.w[1];
     acc.w[2] = f.z & win.w[2];
@@ -234,44 +261,39 @@ __device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, c
 // stage b's memory from below (fewer layers as l grows); inside that window
 // each l is checked against g(S_S).
 __device__ __forceinline__ int complete_set(const ExpandParams &p, const Tab &t, const Prefix &pr,
+                                            const ParentCtx &q, int kb, uint64_t scale,
                                             uint64_t thr, Bits128 &acc, unsigned long long &cut_b,
                                             unsigned long long &cut_m) {
-    const SliceRec &sr = p.slices[pr.slice];
     const int S = p.S, M = p.M, L = t.L(), a = S - 2, b = S - 1;
     const int64_t A = pr.A, Bm = pr.Bm;
-    const int c = a > 0 ? pr.cut[a > 0 ? a - 1 : 0] : 0;
-    const int ka = sr.cls[a], kb = sr.cls[b];
-    const uint64_t scale = sr.scale;
+    const int c = q.c;
     const int lmax = L - c - 1;
-    const int hi_mem = last_true(lmax, [&](int l) { return stage_fits(t, S, M, a, ka, c, c + l); });
-    int hi = hi_mem;
-    if (p.prune)
-        hi = last_true(hi_mem, [&](int l) {
-            const int c2 = c + l;
-            const int64_t F = Pf(t, ka, c2) - Pf(t, ka, c), B = Pb(t, ka, c2) - Pb(t, ka, c);
-            const int64_t d = Pd(t, ka, c2) - Pd(t, ka, c);
-            return (uint64_t)(A + (int64_t)M * (F + B) + max(Bm, d)) * scale <= thr;
-        });
+    const int hi_mem = mem_limit(t, S, M, a, q.k, c, lmax);
+    const int hi = p.prune ? bound_limit(t, q, M, A, Bm, scale, thr, hi_mem) : hi_mem;
     // smallest l in [1, hi] whose remainder fits stage b (hi + 1 if none)
+    const int64_t wL = Pw(t, kb, L), aL = Pa(t, kb, L), capb = cap_of(t, kb);
+    const int64_t flb = inflight(S, M, b);
     const int lo = 1 + last_true(hi, [&](int l) {
-                       return l == 0 ? true : !stage_fits(t, S, M, b, kb, c + l, L);
+                       return (wL - Pw(t, kb, c + l)) + flb * (aL - Pa(t, kb, c + l)) > capb;
                    });
     for (int i = 0; i < 4; ++i) acc.w[i] = 0;
     int n = 0;
+    const int32_t fbL = Pf(t, kb, L), bbL = Pb(t, kb, L), dbL = Pd(t, kb, L);
     for (int l = lo; l <= hi; ++l) {
         const int c2 = c + l;
         if (p.prune) {
-            const int64_t Fa = Pf(t, ka, c2) - Pf(t, ka, c), Ba = Pb(t, ka, c2) - Pb(t, ka, c);
-            const int64_t da = Pd(t, ka, c2) - Pd(t, ka, c);
-            const int64_t Fb = Pf(t, kb, L) - Pf(t, kb, c2), Bb = Pb(t, kb, L) - Pb(t, kb, c2);
-            const int64_t db = Pd(t, kb, L) - Pd(t, kb, c2);
+            const int64_t Fa = Pf(t, q.k, c2) - q.f0, Ba = Pb(t, q.k, c2) - q.b0;
+            const int64_t da = Pd(t, q.k, c2) - q.d0;
+            const int64_t Fb = fbL - Pf(t, kb, c2), Bb = bbL - Pb(t, kb, c2);
+            const int64_t db = dbL - Pd(t, kb, c2);
             const int64_t g = A + Fa + (int64_t)M * (Fb + Bb) + max(max(Bm, da) + Ba, db);
             if ((uint64_t)g * scale > thr) {
                 ++cut_b;
                 continue;
             }
         }
-        acc.w[c2 >> 5] |= 1u << (c2 & 31);
+#pragma unroll
+        for (int wd = 0; wd < 4; ++wd) acc.w[wd] |= (c2 >> 5) == wd ? 1u << (c2 & 31) : 0u;
         ++n;
     }
     cut_m += (unsigned long long)(lmax - hi_mem) + (unsigned long long)(lo - 1 < hi ? lo - 1 : hi);
@@ -283,7 +305,7 @@ __device__ __forceinline__ int complete_set(const ExpandParams &p, const Tab &t,
 // parent's children (a 128-bit set of cut positions), the warp reserves
 // output slots with one atomic and writes them -- or, when the output is
 // full, marks its reserved slots as holes and defers the group.
-template <bool COMPLETE>
+template <bool COMPLETE, int X>
 __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
     stage_blob(sm, p.blob, p.lay.bytes);
@@ -294,7 +316,7 @@ __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
     const long long warp = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
     const long long n_warps = ((long long)gridDim.x * blockDim.x) >> 5;
     const long long n_work = p.groups ? p.n_groups : (p.n_in + 31) / 32;
-    unsigned long long emitted = 0, cb = 0, cm = 0;
+    unsigned long long emitted = 0, cb = 0, cm = 0, parents = 0, written_parents = 0;
     for (long long w = warp; w < n_work; w += n_warps) {
         const long long g = p.groups ? (long long)p.groups[w] : w;
         const long long i = g * 32 + lane;
@@ -304,9 +326,17 @@ __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
         Bits128 acc = {{0u, 0u, 0u, 0u}};
         unsigned long long lb = 0, lm = 0;
         int n = 0;
-        if (pr.slice != kPrefixHole)
-            n = COMPLETE ? complete_set(p, t, pr, thr, acc, lb, lm)
-                         : expand_set(p, t, pr, thr, acc, lb, lm);
+        ParentCtx q = {0, 0, 0, 0, 0};
+        if (pr.slice != kPrefixHole) {
+            const SliceRec &sr = p.slices[pr.slice];
+            // X = depth of the parents = index of the stage placed here
+            const int c = X > 0 ? pr.cut[X > 0 ? X - 1 : 0] : 0;
+            q = parent_ctx(t, sr.cls[X], c);
+            const uint64_t scale = sr.scale;
+            ++parents;
+            n = COMPLETE ? complete_set(p, t, pr, q, sr.cls[X + 1], scale, thr, acc, lb, lm)
+                         : expand_set(p, t, pr, q, sr.gid, scale, thr, acc, lb, lm);
+        }
         int incl = n;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
@@ -320,9 +350,10 @@ __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
         if (total == 0) {
             cb += lb;
             cm += lm;
+            written_parents += (pr.slice != kPrefixHole);
             continue;
         }
-        unsigned long long q = base + (unsigned long long)(incl - n);
+        unsigned long long pos = base + (unsigned long long)(incl - n);
         if (base + (unsigned long long)total <= p.cap) {
 #pragma unroll
             for (int wd = 0; wd < 4; ++wd) {
@@ -334,29 +365,26 @@ __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
                         Leaf lf;
                         lf.slice = pr.slice;
 #pragma unroll
-                        for (int s2 = 0; s2 < 16; ++s2) lf.cut[s2] = s2 < 14 ? pr.cut[s2 < 14 ? s2 : 0] : 0;
-                        lf.cut[p.S - 2] = (uint8_t)c2;
+                        for (int s2 = 0; s2 < 16; ++s2) lf.cut[s2] = s2 < X ? pr.cut[s2 < X ? s2 : 0] : 0;
+                        lf.cut[X] = (uint8_t)c2;
                         lf.pad[0] = lf.pad[1] = lf.pad[2] = 0;
-                        p.leaves[q++] = lf;
+                        p.leaves[pos++] = lf;
                     } else {
-                        // parent cut c and class k of the new stage x
-                        const int x = p.x;
-                        const int c = x > 0 ? pr.cut[x > 0 ? x - 1 : 0] : 0;
-                        const int k = p.slices[pr.slice].cls[x];
                         Prefix ch = pr;
-                        ch.cut[x] = (uint8_t)c2;
-                        ch.A = pr.A + (Pf(t, k, c2) - Pf(t, k, c));
-                        ch.Bm = max(pr.Bm, Pd(t, k, c2) - Pd(t, k, c)) + (Pb(t, k, c2) - Pb(t, k, c));
-                        p.out[q++] = ch;
+                        ch.cut[X < 14 ? X : 0] = (uint8_t)c2;
+                        ch.A = pr.A + (Pf(t, q.k, c2) - q.f0);
+                        ch.Bm = max(pr.Bm, Pd(t, q.k, c2) - q.d0) + (Pb(t, q.k, c2) - q.b0);
+                        p.out[pos++] = ch;
                     }
                 }
             }
             emitted += n;
             cb += lb;
             cm += lm;
+            written_parents += (pr.slice != kPrefixHole);
         } else {
             // no room: mark this warp's reserved slots below cap as holes
-            for (unsigned long long e = q; e < q + (unsigned long long)n && e < p.cap; ++e) {
+            for (unsigned long long e = pos; e < pos + (unsigned long long)n && e < p.cap; ++e) {
                 if (COMPLETE) p.leaves[e].slice = kLeafHole;
                 else p.out[e].slice = kPrefixHole;
             }
@@ -366,18 +394,20 @@ __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
             }
         }
     }
+    (void)parents;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         emitted += __shfl_xor_sync(0xffffffffu, emitted, o);
         cb += __shfl_xor_sync(0xffffffffu, cb, o);
         cm += __shfl_xor_sync(0xffffffffu, cm, o);
+        written_parents += __shfl_xor_sync(0xffffffffu, written_parents, o);
     }
     if (lane == 0) {
-        if (!COMPLETE && emitted) atomicAdd(p.stats + kStPrefixes, emitted);
+        if (emitted) atomicAdd(p.stats + (COMPLETE ? kStLeaves : kStPrefixes), emitted);
         if (cb) atomicAdd(p.stats + kStPrunedBound, cb);
         if (cm) atomicAdd(p.stats + kStPrunedMemory, cm);
-        if (emitted + cb + cm)
-            atomicAdd(p.stats + (COMPLETE ? kStTestsComplete : kStTestsExpand), emitted + cb + cm);
+        if (written_parents)
+            atomicAdd(p.stats + (COMPLETE ? kStParentsComplete : kStParentsExpand), written_parents);
     }
 }
 
@@ -616,6 +646,33 @@ static pos_status run_leaves(Search &s, const Leaf *leaves, unsigned long long *
     return launch_leaf(s.S, M >= s.S, lp, s.grid_leaf, s.stream);
 }
 
+template <bool COMPLETE, int X>
+static pos_status launch_level_t(const ExpandParams &p, int grid, int smem, cudaStream_t st) {
+    auto kern = level_kernel<COMPLETE, X>;
+    POS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    kern<<<grid, kThreads, smem, st>>>(p);
+    POS_CUDA(cudaGetLastError());
+    return POS_OK;
+}
+
+template <int... X>
+static pos_status launch_level_x(bool complete, int x, const ExpandParams &p, int grid, int smem,
+                                 cudaStream_t st, std::integer_sequence<int, X...>) {
+    pos_status r = fail(POS_EINVAL, "depth out of range");
+    ((x == X ? (r = complete ? launch_level_t<true, X>(p, grid, smem, st)
+                             : launch_level_t<false, X>(p, grid, smem, st),
+                0)
+             : 0),
+     ...);
+    return r;
+}
+
+// parents at depth x = 0..14 (completion: x = S-2)
+static pos_status launch_level(bool complete, int x, const ExpandParams &p, int grid, int smem,
+                               cudaStream_t st) {
+    return launch_level_x(complete, x, p, grid, smem, st, std::make_integer_sequence<int, 15>{});
+}
+
 // Enumerate everything below the prefixes in[0..n_in) (depth x).
 static pos_status process(Search &s, const SliceRec *batch, int M, int x, const Prefix *in,
                           long long n_in) {
@@ -650,12 +707,7 @@ static pos_status process(Search &s, const SliceRec *batch, int M, int x, const 
                                                                          s.grid_level));
         s.launches++;
         POS_CUDA(cudaEventRecord(s.ev[0], s.stream));
-        if (last) {
-            level_kernel<true><<<grid, kThreads, smem, s.stream>>>(p);
-        } else {
-            level_kernel<false><<<grid, kThreads, smem, s.stream>>>(p);
-        }
-        POS_CUDA(cudaGetLastError());
+        if ((st = launch_level(last, x, p, grid, smem, s.stream)) != POS_OK) return st;
         POS_CUDA(cudaEventRecord(s.ev[1], s.stream));
         if (last) {
             // evaluate the leaves that fit; the count stays on the device
@@ -757,15 +809,13 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
             }
     const int smem = s.h->lay.bytes;
     int per_sm = 0;
-    POS_CUDA(cudaFuncSetAttribute(level_kernel<false>,
-                                  cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-    POS_CUDA(cudaFuncSetAttribute(level_kernel<true>,
+    POS_CUDA(cudaFuncSetAttribute(level_kernel<false, 0>,
                                   cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
     POS_CUDA(cudaFuncSetAttribute(feas_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
     POS_CUDA(cudaFuncSetAttribute(sample_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   smem));
-    POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, level_kernel<false>, kThreads,
-                                                           smem));
+    POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, level_kernel<false, 0>,
+                                                           kThreads, smem));
     s.grid_level = std::max(1, per_sm) * sm_count();
     s.grid_leaf = 2 * sm_count();
 
@@ -932,8 +982,9 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         stats->expand_launches = s.n_expand;
         stats->complete_launches = s.n_complete;
         stats->leaf_launches = s.n_leaf;
-        stats->tests_expand = hs[kStTestsExpand];
-        stats->tests_complete = hs[kStTestsComplete];
+        stats->parents_expand = hs[kStParentsExpand];
+        stats->parents_complete = hs[kStParentsComplete];
+        stats->leaves = hs[kStLeaves];
     }
     if (inc.obj == ~0ull) {
         if (stats) stats->ms_total = ms_since(t_start);

@@ -57,8 +57,9 @@ enum {
     kStEvaluated,
     kStTimeout,
     kStRelaxations,
-    kStTestsExpand,
-    kStTestsComplete,
+    kStParentsExpand,
+    kStParentsComplete,
+    kStLeaves,
     kStCount
 };
 
