@@ -209,41 +209,42 @@ __device__ __forceinline__ ParentCtx parent_ctx(const Tab &t, int k, int c) {
     return q;
 }
 
-// largest l in [0, lmax] with stage s (class k) fitting layers [c, c+l)
-__device__ __forceinline__ int mem_limit(const Tab &t, int S, int M, int s, int k, int c,
-                                         int lmax) {
-    const int64_t w0 = Pw(t, k, c), a0 = Pa(t, k, c), cap = cap_of(t, k);
-    const int64_t fl = inflight(S, M, s);
-    return last_true(lmax, [&](int l) {
-        return (Pw(t, k, c + l) - w0) + fl * (Pa(t, k, c + l) - a0) <= cap;
-    });
-}
-
-// largest l in [0, hi] with g = A + M (F + B) + max(Bm, d) <= thr / scale
-__device__ __forceinline__ int bound_limit(const Tab &t, const ParentCtx &q, int M, int64_t A,
-                                           int64_t Bm, uint64_t scale, uint64_t thr, int hi) {
-    return last_true(hi, [&](int l) {
-        const int c2 = q.c + l;
-        const int64_t F = Pf(t, q.k, c2) - q.f0, B = Pb(t, q.k, c2) - q.b0;
-        const int64_t d = Pd(t, q.k, c2) - q.d0;
-        return (uint64_t)(A + (int64_t)M * (F + B) + max(Bm, d)) * scale <= thr;
-    });
-}
-
 // Children of one parent, as the set of new cut positions c2 = c + l.
 // Expansion (parent depth x <= S-3): stage x takes l layers.  Its memory
 // need and g(S_{x+1}) both grow with l, so the admissible l form a prefix
 // [1, hi] found by binary search; the children are the positions in
 // (c, c+hi] from which the remaining layers still fit the remaining stages
 // (feasibility bits).
-__device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, const Prefix &pr,
-                                          const ParentCtx &q, uint32_t gid, uint64_t scale,
+__device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, int64_t A,
+                                          int64_t Bm, const ParentCtx &q, uint32_t gid,
+                                          uint64_t scale,
                                           uint64_t thr, Bits128 &acc, unsigned long long &cut_b,
                                           unsigned long long &cut_m) {
     const int S = p.S, M = p.M, x = p.x, L = t.L();
     const int lmax = L - q.c - (S - x - 1);
-    const int hi_mem = mem_limit(t, S, M, x, q.k, q.c, lmax);
-    const int hi = p.prune ? bound_limit(t, q, M, pr.A, pr.Bm, scale, thr, hi_mem) : hi_mem;
+    // two independent binary searches over [0, lmax], interleaved so that
+    // their shared-memory loads overlap; both predicates are monotone
+    const int64_t w0 = Pw(t, q.k, q.c), a0 = Pa(t, q.k, q.c), cap = cap_of(t, q.k);
+    const int64_t fl = inflight(S, M, x);
+    int mlo = 0, mhi = lmax, blo = 0, bhi = p.prune ? lmax : 0;
+    while (mlo < mhi || blo < bhi) {
+        const int mm = (mlo + mhi + 1) >> 1, bm = (blo + bhi + 1) >> 1;
+        const int cm = q.c + mm, cb2 = q.c + bm;
+        const bool fit = (Pw(t, q.k, cm) - w0) + fl * (Pa(t, q.k, cm) - a0) <= cap;
+        const int64_t F = Pf(t, q.k, cb2) - q.f0, B = Pb(t, q.k, cb2) - q.b0;
+        const int64_t d = Pd(t, q.k, cb2) - q.d0;
+        const bool ok = (uint64_t)(A + (int64_t)M * (F + B) + max(Bm, d)) * scale <= thr;
+        if (mlo < mhi) {
+            if (fit) mlo = mm;
+            else mhi = mm - 1;
+        }
+        if (blo < bhi) {
+            if (ok) blo = bm;
+            else bhi = bm - 1;
+        }
+    }
+    const int hi_mem = mlo;
+    const int hi = p.prune ? min(mlo, blo) : mlo;
     const uint4 f = __ldg(p.feas + (size_t)gid * (S + 1) + x + 1);
     const Bits128 win = range_bits(q.c + 1, q.c + hi);
     acc.w[0] = f.x & win.w[0];
@@ -260,22 +261,47 @@ __device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, c
 // b = S-1 the rest.  Stage a's memory and g(S_{S-1}) bound l from above,
 // stage b's memory from below (fewer layers as l grows); inside that window
 // each l is checked against g(S_S).
-__device__ __forceinline__ int complete_set(const ExpandParams &p, const Tab &t, const Prefix &pr,
-                                            const ParentCtx &q, int kb, uint64_t scale,
+__device__ __forceinline__ int complete_set(const ExpandParams &p, const Tab &t, int64_t A,
+                                            int64_t Bm, const ParentCtx &q, int kb,
+                                            uint64_t scale,
                                             uint64_t thr, Bits128 &acc, unsigned long long &cut_b,
                                             unsigned long long &cut_m) {
     const int S = p.S, M = p.M, L = t.L(), a = S - 2, b = S - 1;
-    const int64_t A = pr.A, Bm = pr.Bm;
     const int c = q.c;
     const int lmax = L - c - 1;
-    const int hi_mem = mem_limit(t, S, M, a, q.k, c, lmax);
-    const int hi = p.prune ? bound_limit(t, q, M, A, Bm, scale, thr, hi_mem) : hi_mem;
-    // smallest l in [1, hi] whose remainder fits stage b (hi + 1 if none)
+    // three independent binary searches over [0, lmax], interleaved: stage
+    // a's memory limit, the bound g(S_{S-1}) <= T_min (both true up to some
+    // l), and the last l whose remainder does NOT fit stage b
+    const int64_t w0 = Pw(t, q.k, c), a0 = Pa(t, q.k, c), capa = cap_of(t, q.k);
+    const int64_t fla = inflight(S, M, a);
     const int64_t wL = Pw(t, kb, L), aL = Pa(t, kb, L), capb = cap_of(t, kb);
     const int64_t flb = inflight(S, M, b);
-    const int lo = 1 + last_true(hi, [&](int l) {
-                       return (wL - Pw(t, kb, c + l)) + flb * (aL - Pa(t, kb, c + l)) > capb;
-                   });
+    int mlo = 0, mhi = lmax, blo = 0, bhi = p.prune ? lmax : 0, rlo = 0, rhi = lmax;
+    while (mlo < mhi || blo < bhi || rlo < rhi) {
+        const int mm = (mlo + mhi + 1) >> 1, bm = (blo + bhi + 1) >> 1, rm = (rlo + rhi + 1) >> 1;
+        const int cm = c + mm, cbm = c + bm, crm = c + rm;
+        const bool fit = (Pw(t, q.k, cm) - w0) + fla * (Pa(t, q.k, cm) - a0) <= capa;
+        const int64_t F = Pf(t, q.k, cbm) - q.f0, B = Pb(t, q.k, cbm) - q.b0;
+        const int64_t d = Pd(t, q.k, cbm) - q.d0;
+        const bool ok = (uint64_t)(A + (int64_t)M * (F + B) + max(Bm, d)) * scale <= thr;
+        const bool nofit_b = (wL - Pw(t, kb, crm)) + flb * (aL - Pa(t, kb, crm)) > capb;
+        if (mlo < mhi) {
+            if (fit) mlo = mm;
+            else mhi = mm - 1;
+        }
+        if (blo < bhi) {
+            if (ok) blo = bm;
+            else bhi = bm - 1;
+        }
+        if (rlo < rhi) {
+            if (nofit_b) rlo = rm;
+            else rhi = rm - 1;
+        }
+    }
+    const int hi_mem = mlo;
+    const int hi = p.prune ? min(mlo, blo) : mlo;
+    // smallest l in [1, hi] whose remainder fits stage b (hi + 1 if none)
+    const int lo = 1 + min(rlo, hi);
     for (int i = 0; i < 4; ++i) acc.w[i] = 0;
     int n = 0;
     const int32_t fbL = Pf(t, kb, L), bbL = Pb(t, kb, L), dbL = Pd(t, kb, L);
@@ -306,7 +332,7 @@ __device__ __forceinline__ int complete_set(const ExpandParams &p, const Tab &t,
 // output slots with one atomic and writes them -- or, when the output is
 // full, marks its reserved slots as holes and defers the group.
 template <bool COMPLETE, int X>
-__global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
+__global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(ExpandParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
     stage_blob(sm, p.blob, p.lay.bytes);
     __syncthreads();
@@ -320,22 +346,24 @@ __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
     for (long long w = warp; w < n_work; w += n_warps) {
         const long long g = p.groups ? (long long)p.groups[w] : w;
         const long long i = g * 32 + lane;
-        Prefix pr;
-        pr.slice = kPrefixHole;
-        if (i < p.n_in) pr = p.in[i];
+        Vec32 pv = {make_uint4(kPrefixHole, 0, 0, 0), make_uint4(0, 0, 0, 0)};
+        if (i < p.n_in) pv = load32(p.in + i);
+        const uint32_t slice = pv.a.x & 0xffffu;
+        const bool live = slice != kPrefixHole;
         Bits128 acc = {{0u, 0u, 0u, 0u}};
         unsigned long long lb = 0, lm = 0;
         int n = 0;
         ParentCtx q = {0, 0, 0, 0, 0};
-        if (pr.slice != kPrefixHole) {
-            const SliceRec &sr = p.slices[pr.slice];
-            // X = depth of the parents = index of the stage placed here
-            const int c = X > 0 ? pr.cut[X > 0 ? X - 1 : 0] : 0;
+        if (live) {
+            const SliceRec &sr = p.slices[slice];
+            // X = depth of the parents = index of the stage placed here;
+            // parent byte 2+i holds cut[i]
+            const int c = X > 0 ? (int)get_byte<(X > 0 ? X + 1 : 2)>(pv) : 0;
             q = parent_ctx(t, sr.cls[X], c);
             const uint64_t scale = sr.scale;
-            ++parents;
-            n = COMPLETE ? complete_set(p, t, pr, q, sr.cls[X + 1], scale, thr, acc, lb, lm)
-                         : expand_set(p, t, pr, q, sr.gid, scale, thr, acc, lb, lm);
+            const int64_t A = (int32_t)pv.b.x, Bm = (int32_t)pv.b.y;
+            n = COMPLETE ? complete_set(p, t, A, Bm, q, sr.cls[X + 1], scale, thr, acc, lb, lm)
+                         : expand_set(p, t, A, Bm, q, sr.gid, scale, thr, acc, lb, lm);
         }
         int incl = n;
 #pragma unroll
@@ -350,7 +378,7 @@ __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
         if (total == 0) {
             cb += lb;
             cm += lm;
-            written_parents += (pr.slice != kPrefixHole);
+            written_parents += live;
             continue;
         }
         unsigned long long pos = base + (unsigned long long)(incl - n);
@@ -362,31 +390,37 @@ __global__ void __launch_bounds__(kThreads) level_kernel(ExpandParams p) {
                     const int c2 = 32 * wd + __ffs(m) - 1;
                     m &= m - 1;
                     if (COMPLETE) {
-                        Leaf lf;
-                        lf.slice = pr.slice;
-#pragma unroll
-                        for (int s2 = 0; s2 < 16; ++s2) lf.cut[s2] = s2 < X ? pr.cut[s2 < X ? s2 : 0] : 0;
-                        lf.cut[X] = (uint8_t)c2;
-                        lf.pad[0] = lf.pad[1] = lf.pad[2] = 0;
-                        p.leaves[pos++] = lf;
+                        // leaf: slice in bytes 0-3, cut[i] in byte 4+i; the
+                        // parent's cuts (bytes 2..15) move up two bytes
+                        Vec32 lf;
+                        lf.a.x = slice;
+                        lf.a.y = __funnelshift_r(pv.a.x, pv.a.y, 16);
+                        lf.a.z = __funnelshift_r(pv.a.y, pv.a.z, 16);
+                        lf.a.w = __funnelshift_r(pv.a.z, pv.a.w, 16);
+                        lf.b = make_uint4(pv.a.w >> 16, 0u, 0u, 0u);
+                        set_byte<4 + X>(lf, (uint32_t)c2);
+                        store32(p.leaves + pos++, lf);
                     } else {
-                        Prefix ch = pr;
-                        ch.cut[X < 14 ? X : 0] = (uint8_t)c2;
-                        ch.A = pr.A + (Pf(t, q.k, c2) - q.f0);
-                        ch.Bm = max(pr.Bm, Pd(t, q.k, c2) - q.d0) + (Pb(t, q.k, c2) - q.b0);
-                        p.out[pos++] = ch;
+                        Vec32 ch = pv;
+                        set_byte<2 + (X < 14 ? X : 0)>(ch, (uint32_t)c2);
+                        ch.b.x = (uint32_t)((int32_t)pv.b.x + (Pf(t, q.k, c2) - q.f0));
+                        ch.b.y = (uint32_t)(max((int32_t)pv.b.y, Pd(t, q.k, c2) - q.d0) +
+                                            (Pb(t, q.k, c2) - q.b0));
+                        store32(p.out + pos++, ch);
                     }
                 }
             }
             emitted += n;
             cb += lb;
             cm += lm;
-            written_parents += (pr.slice != kPrefixHole);
+            written_parents += live;
         } else {
             // no room: mark this warp's reserved slots below cap as holes
+            const Vec32 hole = {make_uint4(COMPLETE ? kLeafHole : kPrefixHole, 0, 0, 0),
+                                make_uint4(0, 0, 0, 0)};
             for (unsigned long long e = pos; e < pos + (unsigned long long)n && e < p.cap; ++e) {
-                if (COMPLETE) p.leaves[e].slice = kLeafHole;
-                else p.out[e].slice = kPrefixHole;
+                if (COMPLETE) store32(p.leaves + e, hole);
+                else store32(p.out + e, hole);
             }
             if (lane == 0) {
                 const unsigned long long d = atomicAdd(p.n_deferred, 1ull);

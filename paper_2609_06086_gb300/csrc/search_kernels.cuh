@@ -46,6 +46,41 @@ struct Leaf {
 };
 static_assert(sizeof(Leaf) == 32, "Leaf layout");
 
+// 32-byte entries move as two 16-byte vectors; byte I of an entry is
+// addressed at compile time (word I/4, shift 8*(I%4)).
+struct Vec32 {
+    uint4 a, b;
+};
+
+__device__ __forceinline__ Vec32 load32(const void *ptr) {
+    const uint4 *q = static_cast<const uint4 *>(ptr);
+    Vec32 v;
+    v.a = __ldg(q);
+    v.b = __ldg(q + 1);
+    return v;
+}
+__device__ __forceinline__ void store32(void *ptr, const Vec32 &v) {
+    uint4 *q = static_cast<uint4 *>(ptr);
+    q[0] = v.a;
+    q[1] = v.b;
+}
+__device__ __forceinline__ uint32_t &word_of(Vec32 &v, int w) {
+    return w == 0 ? v.a.x : w == 1 ? v.a.y : w == 2 ? v.a.z : w == 3 ? v.a.w
+         : w == 4 ? v.b.x : w == 5 ? v.b.y : w == 6 ? v.b.z : v.b.w;
+}
+template <int I>
+__device__ __forceinline__ uint32_t get_byte(const Vec32 &v) {
+    const uint32_t w = (I / 4) == 0 ? v.a.x : (I / 4) == 1 ? v.a.y : (I / 4) == 2 ? v.a.z
+                     : (I / 4) == 3 ? v.a.w : (I / 4) == 4 ? v.b.x : (I / 4) == 5 ? v.b.y
+                     : (I / 4) == 6 ? v.b.z : v.b.w;
+    return (w >> (8 * (I % 4))) & 0xffu;
+}
+template <int I>
+__device__ __forceinline__ void set_byte(Vec32 &v, uint32_t b) {
+    uint32_t &w = word_of(v, I / 4);
+    w = (w & ~(0xffu << (8 * (I % 4)))) | ((b & 0xffu) << (8 * (I % 4)));
+}
+
 constexpr uint32_t kLeafHole = 0xffffffffu;
 constexpr uint16_t kPrefixHole = 0xffff;
 
@@ -105,6 +140,17 @@ struct LeafParams {
     BlobLayout lay;
 };
 
+// leaf byte 4+s holds cut[s+1] (layers of stages 0..s)
+template <int S, int... s>
+__device__ __forceinline__ void leaf_cuts_i(const Vec32 &v, int (&cut)[S + 1],
+                                            std::integer_sequence<int, s...>) {
+    ((cut[s + 1] = (int)get_byte<4 + s>(v)), ...);
+}
+template <int S>
+__device__ __forceinline__ void leaf_cuts(const Vec32 &v, int (&cut)[S + 1]) {
+    leaf_cuts_i<S>(v, cut, std::make_integer_sequence<int, S - 1>{});
+}
+
 template <int S, int PATH>
 __global__ void __launch_bounds__(256, (S <= 4 ? 4 : (S <= 8 ? 3 : 2)))
 leaf_kernel(LeafParams p) {
@@ -123,13 +169,16 @@ leaf_kernel(LeafParams p) {
          i < n_round; i += stride) {
         unsigned long long obj = ~0ull, idx = ~0ull;
         uint32_t sl = kLeafHole;
-        if (i < n) sl = __ldg(&p.leaves[i].slice);
+        Vec32 lv = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};
+        if (i < n) {
+            lv = load32(p.leaves + i);
+            sl = lv.a.x;
+        }
         if (sl != kLeafHole) {
             const SliceRec &sr = p.slices[sl];
             int cut[S + 1], cls[S];
             cut[0] = 0;
-#pragma unroll
-            for (int s = 0; s < S - 1; ++s) cut[s + 1] = __ldg(&p.leaves[i].cut[s]);
+            leaf_cuts<S>(lv, cut);
             cut[S] = L;
 #pragma unroll
             for (int s = 0; s < S; ++s) cls[s] = __ldg(&sr.cls[s]);
