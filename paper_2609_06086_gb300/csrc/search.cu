@@ -30,8 +30,10 @@ constexpr int kThreads = 256;
 // ---------------------------------------------------------------------------
 // suffix feasibility: one block per slice, thread c
 // ---------------------------------------------------------------------------
+// Also fills lim[(gid*S + x)*128 + c] = the largest l such that stage x
+// holds layers [c, c+l) within memory (0 if none), capped at L - c.
 __global__ void feas_kernel(const SliceRec *slices, int n_slices, int S, uint4 *feas,
-                            const void *blob, BlobLayout lay) {
+                            uint8_t *lim, const void *blob, BlobLayout lay) {
     extern __shared__ __align__(16) unsigned char sm[];
     __shared__ uint32_t prev[4], cur[4];
     stage_blob(sm, blob, lay.bytes);
@@ -48,17 +50,17 @@ __global__ void feas_kernel(const SliceRec *slices, int n_slices, int S, uint4 *
         if (c == 0) row[S] = make_uint4(prev[0], prev[1], prev[2], prev[3]);
         for (int x = S - 1; x >= 0; --x) {
             bool ok = false;
+            int most = 0;
             if (c < L) {
                 const int k = sr.cls[x];
                 for (int l = 1; c + l <= L; ++l) {
                     if (!stage_fits(t, S, M, x, k, c, c + l)) break;
+                    most = l;
                     const int e = c + l;
-                    if ((prev[e >> 5] >> (e & 31)) & 1u) {
-                        ok = true;
-                        break;
-                    }
+                    if ((prev[e >> 5] >> (e & 31)) & 1u) ok = true;
                 }
             }
+            if (c < 128) lim[((size_t)sr.gid * S + x) * 128 + c] = (uint8_t)most;
             const unsigned b = __ballot_sync(0xffffffffu, ok);
             if ((c & 31) == 0) cur[c >> 5] = b;
             __syncthreads();
@@ -148,6 +150,7 @@ struct ExpandParams {
     int prune;
     const SliceRec *slices;
     const uint4 *feas;
+    const uint8_t *lim;      // per (slice, stage, start) memory limit, see feas_kernel
     Prefix *out;             // expand: children at depth x+1
     Leaf *leaves;            // complete: full plans
     unsigned long long *out_count;
@@ -222,29 +225,18 @@ __device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, i
                                           unsigned long long &cut_m) {
     const int S = p.S, M = p.M, x = p.x, L = t.L();
     const int lmax = L - q.c - (S - x - 1);
-    // two independent binary searches over [0, lmax], interleaved so that
-    // their shared-memory loads overlap; both predicates are monotone
-    const int64_t w0 = Pw(t, q.k, q.c), a0 = Pa(t, q.k, q.c), cap = cap_of(t, q.k);
-    const int64_t fl = inflight(S, M, x);
-    int mlo = 0, mhi = lmax, blo = 0, bhi = p.prune ? lmax : 0;
-    while (mlo < mhi || blo < bhi) {
-        const int mm = (mlo + mhi + 1) >> 1, bm = (blo + bhi + 1) >> 1;
-        const int cm = q.c + mm, cb2 = q.c + bm;
-        const bool fit = (Pw(t, q.k, cm) - w0) + fl * (Pa(t, q.k, cm) - a0) <= cap;
-        const int64_t F = Pf(t, q.k, cb2) - q.f0, B = Pb(t, q.k, cb2) - q.b0;
-        const int64_t d = Pd(t, q.k, cb2) - q.d0;
-        const bool ok = (uint64_t)(A + (int64_t)M * (F + B) + max(Bm, d)) * scale <= thr;
-        if (mlo < mhi) {
-            if (fit) mlo = mm;
-            else mhi = mm - 1;
-        }
-        if (blo < bhi) {
-            if (ok) blo = bm;
-            else bhi = bm - 1;
+    const int hi_mem = min(lmax, (int)__ldg(p.lim + ((size_t)gid * S + x) * 128 + q.c));
+    int hi = hi_mem;
+    if (p.prune) {  // g(S_{x+1}) grows with l: binary search for the last l within the bound
+        int lo = 0;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1, c2 = q.c + mid;
+            const int64_t F = Pf(t, q.k, c2) - q.f0, B = Pb(t, q.k, c2) - q.b0;
+            const int64_t d = Pd(t, q.k, c2) - q.d0;
+            if ((uint64_t)(A + (int64_t)M * (F + B) + max(Bm, d)) * scale <= thr) lo = mid;
+            else hi = mid - 1;
         }
     }
-    const int hi_mem = mlo;
-    const int hi = p.prune ? min(mlo, blo) : mlo;
     const uint4 f = __ldg(p.feas + (size_t)gid * (S + 1) + x + 1);
     const Bits128 win = range_bits(q.c + 1, q.c + hi);
     acc.w[0] = f.x & win.w[0];
@@ -262,46 +254,34 @@ __device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, i
 // stage b's memory from below (fewer layers as l grows); inside that window
 // each l is checked against g(S_S).
 __device__ __forceinline__ int complete_set(const ExpandParams &p, const Tab &t, int64_t A,
-                                            int64_t Bm, const ParentCtx &q, int kb,
+                                            int64_t Bm, const ParentCtx &q, int kb, uint32_t gid,
                                             uint64_t scale,
                                             uint64_t thr, Bits128 &acc, unsigned long long &cut_b,
                                             unsigned long long &cut_m) {
     const int S = p.S, M = p.M, L = t.L(), a = S - 2, b = S - 1;
     const int c = q.c;
     const int lmax = L - c - 1;
-    // three independent binary searches over [0, lmax], interleaved: stage
-    // a's memory limit, the bound g(S_{S-1}) <= T_min (both true up to some
-    // l), and the last l whose remainder does NOT fit stage b
-    const int64_t w0 = Pw(t, q.k, c), a0 = Pa(t, q.k, c), capa = cap_of(t, q.k);
-    const int64_t fla = inflight(S, M, a);
-    const int64_t wL = Pw(t, kb, L), aL = Pa(t, kb, L), capb = cap_of(t, kb);
-    const int64_t flb = inflight(S, M, b);
-    int mlo = 0, mhi = lmax, blo = 0, bhi = p.prune ? lmax : 0, rlo = 0, rhi = lmax;
-    while (mlo < mhi || blo < bhi || rlo < rhi) {
-        const int mm = (mlo + mhi + 1) >> 1, bm = (blo + bhi + 1) >> 1, rm = (rlo + rhi + 1) >> 1;
-        const int cm = c + mm, cbm = c + bm, crm = c + rm;
-        const bool fit = (Pw(t, q.k, cm) - w0) + fla * (Pa(t, q.k, cm) - a0) <= capa;
-        const int64_t F = Pf(t, q.k, cbm) - q.f0, B = Pb(t, q.k, cbm) - q.b0;
-        const int64_t d = Pd(t, q.k, cbm) - q.d0;
-        const bool ok = (uint64_t)(A + (int64_t)M * (F + B) + max(Bm, d)) * scale <= thr;
-        const bool nofit_b = (wL - Pw(t, kb, crm)) + flb * (aL - Pa(t, kb, crm)) > capb;
-        if (mlo < mhi) {
-            if (fit) mlo = mm;
-            else mhi = mm - 1;
-        }
-        if (blo < bhi) {
-            if (ok) blo = bm;
-            else bhi = bm - 1;
-        }
-        if (rlo < rhi) {
-            if (nofit_b) rlo = rm;
-            else rhi = rm - 1;
+    const int hi_mem = min(lmax, (int)__ldg(p.lim + ((size_t)gid * S + a) * 128 + c));
+    int hi = hi_mem;
+    if (p.prune) {  // g(S_{S-1}) grows with l
+        int lo = 0;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1, c2 = c + mid;
+            const int64_t F = Pf(t, q.k, c2) - q.f0, B = Pb(t, q.k, c2) - q.b0;
+            const int64_t d = Pd(t, q.k, c2) - q.d0;
+            if ((uint64_t)(A + (int64_t)M * (F + B) + max(Bm, d)) * scale <= thr) lo = mid;
+            else hi = mid - 1;
         }
     }
-    const int hi_mem = mlo;
-    const int hi = p.prune ? min(mlo, blo) : mlo;
-    // smallest l in [1, hi] whose remainder fits stage b (hi + 1 if none)
-    const int lo = 1 + min(rlo, hi);
+    // stage b fits [c2, L) exactly for the set feasibility bits of depth b,
+    // a suffix of positions: the smallest l is the first set bit above c
+    const uint4 fb = __ldg(p.feas + (size_t)gid * (S + 1) + b);
+    const Bits128 above = range_bits(c + 1, L - 1);
+    const uint32_t m0 = fb.x & above.w[0], m1 = fb.y & above.w[1], m2 = fb.z & above.w[2],
+                   m3 = fb.w & above.w[3];
+    const int first = m0 ? __ffs(m0) - 1 : m1 ? 31 + __ffs(m1) : m2 ? 63 + __ffs(m2)
+                    : m3 ? 95 + __ffs(m3) : 128;
+    const int lo = first - c;
     for (int i = 0; i < 4; ++i) acc.w[i] = 0;
     int n = 0;
     const int32_t fbL = Pf(t, kb, L), bbL = Pb(t, kb, L), dbL = Pd(t, kb, L);
@@ -362,7 +342,8 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
             q = parent_ctx(t, sr.cls[X], c);
             const uint64_t scale = sr.scale;
             const int64_t A = (int32_t)pv.b.x, Bm = (int32_t)pv.b.y;
-            n = COMPLETE ? complete_set(p, t, A, Bm, q, sr.cls[X + 1], scale, thr, acc, lb, lm)
+            n = COMPLETE ? complete_set(p, t, A, Bm, q, sr.cls[X + 1], sr.gid, scale, thr, acc, lb,
+                                        lm)
                          : expand_set(p, t, A, Bm, q, sr.gid, scale, thr, acc, lb, lm);
         }
         int incl = n;
@@ -484,7 +465,7 @@ struct Workspace {
     std::mutex mu;
     cudaStream_t stream = nullptr;
     cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
-    DevBuf blob, d_slices, d_feas, d_batch, d_inc, d_ctr, d_best, d_feasible, d_leaves, d_roots,
+    DevBuf blob, d_lim, d_slices, d_feas, d_batch, d_inc, d_ctr, d_best, d_feasible, d_leaves, d_roots,
         d_root;
     DevBuf d_front[POS_MAX_STAGES + 1];        // per depth: Prefix buffers
     DevBuf d_defer[2 * (POS_MAX_STAGES + 1)];  // per depth: two deferred group lists
@@ -654,6 +635,7 @@ static ExpandParams base_params(Search &s, const SliceRec *batch, int M) {
     p.prune = s.pb->prune ? 1 : 0;
     p.slices = batch;
     p.feas = static_cast<const uint4 *>(s.d_feas.p);
+    p.lim = static_cast<const uint8_t *>(s.ws.d_lim.p);
     p.cap = (unsigned long long)s.cap;
     p.inc = static_cast<const Key128 *>(s.d_inc.p);
     p.stats = s.stats;
@@ -855,6 +837,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
 
     POS_CUDA(s.d_slices.reserve(sizeof(SliceRec) * n_slices));
     POS_CUDA(s.d_feas.reserve(sizeof(uint4) * (size_t)n_slices * (s.S + 1)));
+    POS_CUDA(s.ws.d_lim.reserve((size_t)n_slices * s.S * 128));
     POS_CUDA(s.d_inc.reserve(sizeof(Key128)));
     POS_CUDA(s.d_ctr.reserve(sizeof(unsigned long long) * 64));
     POS_CUDA(s.d_best.reserve(sizeof(unsigned long long) * n_slices));
@@ -868,7 +851,8 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     POS_CUDA(cudaMemsetAsync(s.d_best.p, 0xff, sizeof(unsigned long long) * n_slices, s.stream));
     const SliceRec *d_all = static_cast<const SliceRec *>(s.d_slices.p);
     feas_kernel<<<std::min(n_slices, 16 * sm_count()), 128, smem, s.stream>>>(
-        d_all, n_slices, s.S, static_cast<uint4 *>(s.d_feas.p), s.h->d_blob, s.h->lay);
+        d_all, n_slices, s.S, static_cast<uint4 *>(s.d_feas.p),
+        static_cast<uint8_t *>(s.ws.d_lim.p), s.h->d_blob, s.h->lay);
     POS_CUDA(cudaGetLastError());
     s.launches++;
     DevBuf &d_root = s.d_root;
