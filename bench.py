@@ -111,6 +111,44 @@ def oracle_sample_rate(seconds: float, seed: int = 0):
     return n / dt, n, dt
 
 
+def eval_throughput(P, torch, n, reps, peak_alu):
+    """poseidon_eval_batch on n config-5 candidates (L=64, S ~ U{2..16},
+    M ~ U{8..128}, 2 device types), device-resident, timed with CUDA events
+    on the launching stream; inputs (16 B x n) exceed L2 for n >= 1e7."""
+    w = gen.config5_tables()
+    c = gen.config5_candidates(n, seed=0)
+    S = c["S"].astype(np.int64)
+    M = c["M"].astype(np.int64)
+    relax = int((2 * S * M).sum())
+    ops = 3 * relax + 11 * int(S.sum())  # 6SM + 11S integer ops per candidate
+    h = P.Handle(P.Tables.from_workload(w))
+    d_c = torch.from_numpy(c.view(np.uint8)).cuda()
+    del c
+    d_T = torch.empty(n, dtype=torch.int32, device="cuda")
+    d_F = torch.empty(n, dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+    for _ in range(2):
+        P.poseidon_eval_batch(h, d_c.data_ptr(), n, d_T.data_ptr(), d_F.data_ptr(),
+                              stream.cuda_stream)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    ms = 0.0
+    for _ in range(reps):
+        ev0.record(stream)
+        P.poseidon_eval_batch(h, d_c.data_ptr(), n, d_T.data_ptr(), d_F.data_ptr(),
+                              stream.cuda_stream)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        ms += ev0.elapsed_time(ev1)
+    sec = ms / 1e3 / reps
+    h.close()
+    ach = ops / sec / 1e12
+    return {"workload": "config 5: L=64, S~U{2..16}, M~U{8..128}, 2 device types",
+            "batch": n, "ms_per_call": round(sec * 1e3, 4), "evals_per_s": n / sec,
+            "relaxations_per_s": relax / sec, "bound": "alu", "achieved": round(ach, 3),
+            "unit": "Tops/s", "peak": round(peak_alu, 3), "frac": round(ach / peak_alu, 4)}
+
+
 def run_reference(args, rank, world):
     if rank != 0:
         return
@@ -233,6 +271,7 @@ def run_ours(args, rank, world, local_rank):
             "work_per_launch": work[dom] / max(1, launches[dom]), "traffic": None,
             "peak_note": (f"{n_sm} SMs x {SM_LANES} int32 lanes x {mhz:.0f} MHz (median SM "
                           "clock under load)" if b == "alu" else hbm_src)}
+    evals = [eval_throughput(P, torch, int(n), 5, peak_alu) for n in args.eval_sizes]
     cpu_rate, cpu_n, cpu_t = oracle_sample_rate(args.cpu_seconds)
     line = {
         "metric": METRIC, "value": value, "unit": "evals/s", "n_gpus": world,
@@ -253,6 +292,7 @@ def run_ours(args, rank, world, local_rank):
         "host_ms_per_step": {k: round(agg[k] / args.steps, 3)
                              for k in ("ms_setup", "ms_warmup", "ms_search")},
         "roofline": roof,
+        "eval_throughput": evals,
         "cpu_baseline": {"value": cpu_rate, "unit": "evals/s", "cores": 1, "kind": "oracle",
                          "sample": f"{cpu_n} config-4 plan evaluations (S=8, M=32, L=80) in "
                                    f"{cpu_t:.1f} s, single-threaded oracle"},
@@ -274,6 +314,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--backend", choices=["nccl", "gloo"], default="nccl")
+    ap.add_argument("--eval-sizes", type=float, nargs="*", default=[1e7],
+                    help="config-5 batch sizes for the evaluator measurement")
     ap.add_argument("--frontier-cap", type=int, default=0,
                     help="frontier entries per depth (0 = library default)")
     args = ap.parse_args()

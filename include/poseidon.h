@@ -117,9 +117,11 @@ pos_status poseidon_tables_destroy(void *handle);
  * d_feasible (uint8[n]) are DEVICE pointers on the handle's device; outputs
  * are in input order; the call is asynchronous on `stream` (a cudaStream_t,
  * NULL = legacy default stream) and returns after the launches.  Infeasible
- * plans still get their makespan.  No global scratch memory is used.
+ * plans still get their makespan.  Scratch: the batch is counting-sorted by
+ * (S, M) into a 4*n + 52 KB stream-ordered allocation from a library-owned
+ * memory pool (per device, kept between calls).
  * Errors: POS_EINVAL (null handle or pointers, n < 0, misaligned
- * candidates), POS_ECUDA (launch failure).
+ * candidates), POS_ENOMEM, POS_ECUDA (launch failure).
  */
 pos_status poseidon_eval_batch(void *handle, const pos_candidate *d_cands, int64_t n,
                                int32_t *d_makespan, uint8_t *d_feasible, void *stream);

@@ -1,6 +1,8 @@
 // poseidon_eval_batch, poseidon_eval_batch_host and poseidon_argmin (hot-path
 // step a9).  The evaluation kernels live in eval_kernel.cuh and the
 // eval_range_*.cu instantiation units.
+#include <mutex>
+
 #include "eval_kernel.cuh"
 
 namespace pos {
@@ -53,27 +55,168 @@ __global__ void argmin_final(const int32_t *part_t, const long long *part_i, int
     *out = bi;
 }
 
+// ---------------------------------------------------------------------------
+// counting sort of the candidates by (S, M) key
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ int eval_key(uint32_t w) {
+    const int S = w & 0xff, M = (w >> 8) & 0xff;
+    if (S < 1 || S > POS_MAX_STAGES || M < 1) return -1;
+    return M >= S ? (S - 1) * 256 + M : 4096 + (S - 1) * 16 + M;
+}
+
+// global key histogram; invalid records are answered right here
+__global__ void sort_hist_kernel(const uint4 *cands, int64_t n, uint32_t *hist, int32_t *T,
+                                 uint8_t *F) {
+    __shared__ uint32_t h[kKeys];
+    for (int i = threadIdx.x; i < kKeys; i += blockDim.x) h[i] = 0;
+    __syncthreads();
+    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
+         i += (int64_t)gridDim.x * blockDim.x) {
+        const int k = eval_key(__ldg(&cands[i].w));
+        if (k >= 0) {
+            atomicAdd(&h[k], 1u);
+        } else {
+            T[i] = -1;
+            F[i] = POS_FEAS_INVALID;
+        }
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < kKeys; i += blockDim.x)
+        if (h[i]) atomicAdd(&hist[i], h[i]);
+}
+
+// exclusive prefix sum of the histogram (one block); cursor = offs copy
+__global__ void sort_scan_kernel(const uint32_t *hist, uint32_t *offs, uint32_t *cursor) {
+    __shared__ uint32_t part[1024];
+    const int per = (kKeys + blockDim.x - 1) / blockDim.x;
+    const int lo = threadIdx.x * per, hi = min(kKeys, lo + per);
+    uint32_t sum = 0;
+    for (int i = lo; i < hi; ++i) sum += hist[i];
+    part[threadIdx.x] = sum;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        uint32_t run = 0;
+        for (int i = 0; i < (int)blockDim.x; ++i) {
+            const uint32_t v = part[i];
+            part[i] = run;
+            run += v;
+        }
+        offs[kKeys] = run;
+    }
+    __syncthreads();
+    uint32_t run = part[threadIdx.x];
+    for (int i = lo; i < hi; ++i) {
+        offs[i] = run;
+        cursor[i] = run;
+        run += hist[i];
+    }
+}
+
+// Each block takes chunks of kChunk candidates: counts their keys, reserves
+// one range per key with a single atomic, then places the indices.
+constexpr int kChunk = 32768;
+
+__global__ void sort_scatter_kernel(const uint4 *cands, int64_t n, uint32_t *cursor,
+                                    uint32_t *perm) {
+    __shared__ uint32_t h[kKeys];
+    for (int64_t c0 = blockIdx.x * (int64_t)kChunk; c0 < n; c0 += (int64_t)gridDim.x * kChunk) {
+        const int64_t c1 = min(n, c0 + kChunk);
+        for (int i = threadIdx.x; i < kKeys; i += blockDim.x) h[i] = 0;
+        __syncthreads();
+        for (int64_t i = c0 + threadIdx.x; i < c1; i += blockDim.x) {
+            const int k = eval_key(__ldg(&cands[i].w));
+            if (k >= 0) atomicAdd(&h[k], 1u);
+        }
+        __syncthreads();
+        for (int i = threadIdx.x; i < kKeys; i += blockDim.x)
+            if (h[i]) h[i] = atomicAdd(&cursor[i], h[i]);
+        __syncthreads();
+        for (int64_t i = c0 + threadIdx.x; i < c1; i += blockDim.x) {
+            const int k = eval_key(__ldg(&cands[i].w));
+            if (k >= 0) perm[atomicAdd(&h[k], 1u)] = (uint32_t)i;
+        }
+        __syncthreads();
+    }
+}
+
+// Stream-ordered scratch comes from a library-owned pool per device that
+// keeps its memory between calls (release threshold: unlimited).
+static std::mutex g_pool_mutex;
+static cudaMemPool_t g_pool[64];
+
+static pos_status scratch_pool(cudaMemPool_t *out) {
+    int dev = 0;
+    POS_CUDA(cudaGetDevice(&dev));
+    if (dev < 0 || dev >= 64) return fail(POS_EINVAL, "device index above 63");
+    std::lock_guard<std::mutex> lock(g_pool_mutex);
+    if (!g_pool[dev]) {
+        cudaMemPoolProps props = {};
+        props.allocType = cudaMemAllocationTypePinned;
+        props.location.type = cudaMemLocationTypeDevice;
+        props.location.id = dev;
+        cudaMemPool_t pool;
+        POS_CUDA(cudaMemPoolCreate(&pool, &props));
+        uint64_t keep = ~0ull;
+        POS_CUDA(cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep));
+        g_pool[dev] = pool;
+    }
+    *out = g_pool[dev];
+    return POS_OK;
+}
+
 pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32_t *d_T,
                        uint8_t *d_F, cudaStream_t stream) {
     if (n == 0) return POS_OK;
-    EvalParams p;
-    p.cands = reinterpret_cast<const uint4 *>(d_cands);
-    p.n = n;
-    p.T = d_T;
-    p.F = d_F;
-    p.blob = h->d_blob;
-    p.lay = h->lay;
-    p.gA = h->guard_A;
-    p.gD = h->guard_D;
-    p.gP = h->guard_P;
-    const int smem = eval_smem_bytes(h->lay);
-    pos_status st;
-    if ((st = eval_fast_1_4(p, smem, stream)) != POS_OK) return st;
-    if ((st = eval_fast_5_8(p, smem, stream)) != POS_OK) return st;
-    if ((st = eval_fast_9_12(p, smem, stream)) != POS_OK) return st;
-    if ((st = eval_fast_13_16(p, smem, stream)) != POS_OK) return st;
-    if ((st = eval_generic_2_8(p, smem, stream)) != POS_OK) return st;
-    return eval_generic_9_16(p, smem, stream);
+    cudaMemPool_t pool;
+    pos_status st = scratch_pool(&pool);
+    if (st != POS_OK) return st;
+    // permutation indices are 32-bit: batches above 2^31 go in chunks
+    const int64_t chunk = (int64_t)1 << 31;
+    for (int64_t base = 0; base < n; base += chunk) {
+        const int64_t m = std::min(chunk, n - base);
+        void *scratch = nullptr;
+        const size_t sbytes = sizeof(uint32_t) * (3 * (size_t)kKeys + 1 + (size_t)m);
+        POS_CUDA(cudaMallocFromPoolAsync(&scratch, sbytes, pool, stream));
+        uint32_t *hist = static_cast<uint32_t *>(scratch);
+        uint32_t *offs = hist + kKeys;
+        uint32_t *cursor = offs + kKeys + 1;
+        uint32_t *perm = cursor + kKeys;
+        EvalParams p;
+        p.cands = reinterpret_cast<const uint4 *>(d_cands) + base;
+        p.n = m;
+        p.T = d_T + base;
+        p.F = d_F + base;
+        p.perm = perm;
+        p.offs = offs;
+        p.blob = h->d_blob;
+        p.lay = h->lay;
+        p.gA = h->guard_A;
+        p.gD = h->guard_D;
+        p.gP = h->guard_P;
+        const int grid = (int)std::max<int64_t>(
+            1, std::min<int64_t>((m + 255) / 256, 4LL * sm_count()));
+        cudaError_t e = cudaMemsetAsync(hist, 0, sizeof(uint32_t) * kKeys, stream);
+        if (e == cudaSuccess) {
+            sort_hist_kernel<<<grid, 256, 0, stream>>>(p.cands, m, hist, p.T, p.F);
+            sort_scan_kernel<<<1, 1024, 0, stream>>>(hist, offs, cursor);
+            const int sgrid = (int)std::max<int64_t>(
+                1, std::min<int64_t>((m + kChunk - 1) / kChunk, 4LL * sm_count()));
+            sort_scatter_kernel<<<sgrid, 256, 0, stream>>>(p.cands, m, cursor, perm);
+            e = cudaGetLastError();
+        }
+        if (e == cudaSuccess) {
+            if ((st = eval_fast_1_4(p, stream)) == POS_OK && (st = eval_fast_5_8(p, stream)) == POS_OK &&
+                (st = eval_fast_9_12(p, stream)) == POS_OK &&
+                (st = eval_fast_13_16(p, stream)) == POS_OK &&
+                (st = eval_generic_2_8(p, stream)) == POS_OK)
+                st = eval_generic_9_16(p, stream);
+        }
+        const cudaError_t e2 = cudaFreeAsync(scratch, stream);
+        if (e != cudaSuccess) return cuda_fail(e, "eval sort launch");
+        if (st != POS_OK) return st;
+        if (e2 != cudaSuccess) return cuda_fail(e2, "eval scratch free");
+    }
+    return POS_OK;
 }
 
 }  // namespace pos

@@ -3,12 +3,12 @@
 
 namespace pos {
 
-pos_status eval_fast_1_4(const EvalParams &p, int smem, cudaStream_t s) {
-    return launch_eval_range<1, 4, kPathFast, 4>(p, smem, s);
+pos_status eval_fast_1_4(const EvalParams &p, cudaStream_t s) {
+    return launch_eval_range<1, 4, kPathFast, 8>(p, s);
 }
 
-pos_status eval_fast_5_8(const EvalParams &p, int smem, cudaStream_t s) {
-    return launch_eval_range<5, 8, kPathFast, 3>(p, smem, s);
+pos_status eval_fast_5_8(const EvalParams &p, cudaStream_t s) {
+    return launch_eval_range<5, 8, kPathFast, 5>(p, s);
 }
 
 }  // namespace pos

@@ -3,8 +3,8 @@
 
 namespace pos {
 
-pos_status eval_fast_9_12(const EvalParams &p, int smem, cudaStream_t s) {
-    return launch_eval_range<9, 12, kPathFast, 2>(p, smem, s);
+pos_status eval_fast_9_12(const EvalParams &p, cudaStream_t s) {
+    return launch_eval_range<9, 12, kPathFast, 4>(p, s);
 }
 
 }  // namespace pos

@@ -3,8 +3,8 @@
 
 namespace pos {
 
-pos_status eval_generic_2_8(const EvalParams &p, int smem, cudaStream_t s) {
-    return launch_eval_range<2, 8, kPathGeneric, 1>(p, smem, s);
+pos_status eval_generic_2_8(const EvalParams &p, cudaStream_t s) {
+    return launch_eval_range<2, 8, kPathGeneric, 2>(p, s);
 }
 
 }  // namespace pos
