@@ -233,7 +233,8 @@ __device__ __forceinline__ bool plan_fits(const Tab &t, int M, const int (&cut)[
 // split into a ramp-up (levels 1..2S-1), M-S steady two-level steps in which
 // every stage does one F and one B, and a ramp-down (levels 2M..2M+2S-2);
 // the ramps depend on S only and are fully unrolled.  M < S takes a
-// predicated level loop (a separate instantiation, kPathGeneric).
+// separate instantiation (kPathGeneric) whose schedule is unrolled for
+// each M in 1..S-1.
 // ---------------------------------------------------------------------------
 enum { kPathFast = 0, kPathGeneric = 1 };
 
@@ -314,6 +315,63 @@ __device__ __forceinline__ void steady_level(int32_t (&Fo)[S], int32_t (&Bo)[S],
     (steady_op<S, P, i>(Fo, Bo, w), ...);
 }
 
+// M < S: the same level order, with W_s = min(S-s1+1, M); every op and the
+// type of each stage's previous op are known at compile time for a given
+// (S, M), so the whole schedule is unrolled (M < S <= 16 keeps it small).
+__host__ __device__ constexpr int short_op(int S, int M, int s1, int t) {
+    const int ws = S - s1 + 1 < M ? S - s1 + 1 : M;
+    const bool odd = ((t + s1) & 1) != 0;
+    if ((t >= s1 && t <= s1 + ws - 1) || (!odd && t >= 2 * ws + s1 && t <= 2 * M + s1 - 2))
+        return 1;
+    if (odd && t >= 2 * S - s1 + 1 && t <= 2 * S - s1 + 2 * M - 1) return 2;
+    return 0;
+}
+__host__ __device__ constexpr bool short_last_is_b(int S, int M, int s1, int t) {
+    for (int u = t - 1; u >= 1; --u)
+        if (short_op(S, M, s1, u)) return short_op(S, M, s1, u) == 2;
+    return false;
+}
+template <int S, int M, int t, int s1>
+__device__ __forceinline__ void short_step(int32_t (&Fo)[S], int32_t (&Bo)[S], const StageW<S> &w) {
+    constexpr int op = short_op(S, M, s1, t);
+    constexpr bool last_b = short_last_is_b(S, M, s1, t);
+    constexpr int s = s1 - 1;
+    if constexpr (op == 1) relax_f<S, s>(Fo, w, last_b ? Bo[s] : Fo[s]);
+    else if constexpr (op == 2) relax_b<S, s>(Bo, w, last_b ? Bo[s] : Fo[s]);
+}
+template <int S, int M, int t, int... i>
+__device__ __forceinline__ void short_level(int32_t (&Fo)[S], int32_t (&Bo)[S], const StageW<S> &w,
+                                            std::integer_sequence<int, i...>) {
+    (short_step<S, M, t, S - i>(Fo, Bo, w), ...);
+}
+template <int S, int M, int... t>
+__device__ __forceinline__ void short_all(int32_t (&Fo)[S], int32_t (&Bo)[S], const StageW<S> &w,
+                                          std::integer_sequence<int, t...>) {
+    (short_level<S, M, t + 1>(Fo, Bo, w, std::make_integer_sequence<int, S>{}), ...);
+}
+template <int S, int M>
+__device__ __forceinline__ int32_t makespan_short(const StageW<S> &w) {
+    int32_t Fo[S], Bo[S];
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+        Fo[s] = 0;
+        Bo[s] = 0;
+    }
+    short_all<S, M>(Fo, Bo, w, std::make_integer_sequence<int, 2 * (M + S - 1)>{});
+    int32_t T = 0;
+#pragma unroll
+    for (int s = 0; s < S; ++s) T = max(T, Bo[s] + w.d[s]);
+    return T;
+}
+// runtime M in 1..S-1 -> its unrolled instance
+template <int S, int... m>
+__device__ __forceinline__ int32_t makespan_short_dispatch(const StageW<S> &w, int M,
+                                                           std::integer_sequence<int, m...>) {
+    int32_t T = -1;
+    ((M == m + 1 ? (T = makespan_short<S, m + 1>(w), 0) : 0), ...);
+    return T;
+}
+
 template <int S, int PATH>
 __device__ __forceinline__ int32_t makespan_1f1b(const StageW<S> &w, int M) {
     int32_t Fo[S], Bo[S];
@@ -333,25 +391,8 @@ __device__ __forceinline__ int32_t makespan_1f1b(const StageW<S> &w, int M) {
         // ramp-down: levels 2M + tau, tau = 0 .. 2S-2
         ramp<S, false, 0>(Fo, Bo, w, std::make_integer_sequence<int, 2 * S - 1>{});
     } else {
-        // every level visits every stage with predicates.  A stage's ops
-        // are chained, so its last finish is max(Fo, Bo).
-        const int levels = 2 * (M + S - 1);
-        for (int t = 1; t <= levels; ++t) {
-#pragma unroll
-            for (int s1 = S; s1 >= 1; --s1) {
-                const int s = s1 - 1;
-                const int ws = min(S - s1 + 1, M);
-                const bool odd = ((t + s1) & 1) != 0;
-                const bool fwd = (t >= s1 && t <= s1 + ws - 1) ||
-                                 (!odd && t >= 2 * ws + s1 && t <= 2 * M + s1 - 2);
-                const bool bwd = odd && t >= 2 * S - s1 + 1 && t <= 2 * S - s1 + 2 * M - 1;
-                const int32_t clk = max(Fo[s], Bo[s]);
-                const int32_t in_f = s > 0 ? Fo[s > 0 ? s - 1 : 0] + w.pf[s > 0 ? s - 1 : 0] : 0;
-                const int32_t in_b = s + 1 < S ? Bo[s + 1 < S ? s + 1 : 0] + w.pb[s] : 0;
-                if (fwd) Fo[s] = max(clk, in_f) + w.F[s];
-                else if (bwd) Bo[s] = max(clk, in_b) + w.B[s];
-            }
-        }
+        // M < S (kPathGeneric): fully unrolled instance for this M
+        if constexpr (S > 1) return makespan_short_dispatch<S>(w, M, std::make_integer_sequence<int, S - 1>{});
     }
     int32_t T = 0;
 #pragma unroll

@@ -208,8 +208,11 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
             if ((st = eval_fast_1_4(p, stream)) == POS_OK && (st = eval_fast_5_8(p, stream)) == POS_OK &&
                 (st = eval_fast_9_12(p, stream)) == POS_OK &&
                 (st = eval_fast_13_16(p, stream)) == POS_OK &&
-                (st = eval_generic_2_8(p, stream)) == POS_OK)
-                st = eval_generic_9_16(p, stream);
+                (st = eval_generic_2_8(p, stream)) == POS_OK &&
+                (st = eval_generic_9_12(p, stream)) == POS_OK &&
+                (st = eval_generic_13_14(p, stream)) == POS_OK &&
+                (st = eval_generic_15_15(p, stream)) == POS_OK)
+                st = eval_generic_16_16(p, stream);
         }
         const cudaError_t e2 = cudaFreeAsync(scratch, stream);
         if (e != cudaSuccess) return cuda_fail(e, "eval sort launch");

@@ -4,8 +4,9 @@
 // integer ops and its live registers grow with S (about 7*S), so the batch
 // is first counting-sorted by exact (S, M) into a permutation (stream-ordered
 // scratch), and then a family of kernels, each owning the candidates of one
-// S range and either M >= S (fully unrolled fast path) or M < S (predicated
-// path), walks its contiguous range of the permutation with launch bounds
+// S range and either M >= S (ramps unrolled, steady loop) or M < S (the
+// whole schedule unrolled per (S, M)), walks its contiguous range of the
+// permutation with launch bounds
 // matched to its register need.  Warps therefore see one (S, M) except at
 // bucket boundaries, and no kernel waits at a block barrier after staging the
 // cost tables.
@@ -152,6 +153,9 @@ pos_status eval_fast_5_8(const EvalParams &p, cudaStream_t s);
 pos_status eval_fast_9_12(const EvalParams &p, cudaStream_t s);
 pos_status eval_fast_13_16(const EvalParams &p, cudaStream_t s);
 pos_status eval_generic_2_8(const EvalParams &p, cudaStream_t s);
-pos_status eval_generic_9_16(const EvalParams &p, cudaStream_t s);
+pos_status eval_generic_9_12(const EvalParams &p, cudaStream_t s);
+pos_status eval_generic_13_14(const EvalParams &p, cudaStream_t s);
+pos_status eval_generic_15_15(const EvalParams &p, cudaStream_t s);
+pos_status eval_generic_16_16(const EvalParams &p, cudaStream_t s);
 
 }  // namespace pos

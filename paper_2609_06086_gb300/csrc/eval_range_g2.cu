@@ -3,8 +3,8 @@
 
 namespace pos {
 
-pos_status eval_generic_9_16(const EvalParams &p, cudaStream_t s) {
-    return launch_eval_range<9, 16, kPathGeneric, 2>(p, s);
+pos_status eval_generic_9_12(const EvalParams &p, cudaStream_t s) {
+    return launch_eval_range<9, 12, kPathGeneric, 2>(p, s);
 }
 
 }  // namespace pos

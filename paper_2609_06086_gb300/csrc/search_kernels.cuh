@@ -226,14 +226,18 @@ pos_status launch_leaf_t(const LeafParams &p, int grid, cudaStream_t s) {
 // per-unit dispatchers (search_leaf_*.cu): S in the unit's range
 pos_status launch_leaf_1_6(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
 pos_status launch_leaf_7_10(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
-pos_status launch_leaf_11_13(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
-pos_status launch_leaf_14_16(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_11_12(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_13_14(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_15_15(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_16_16(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
 
 inline pos_status launch_leaf(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s) {
     if (S <= 6) return launch_leaf_1_6(S, fast, p, grid, s);
     if (S <= 10) return launch_leaf_7_10(S, fast, p, grid, s);
-    if (S <= 13) return launch_leaf_11_13(S, fast, p, grid, s);
-    return launch_leaf_14_16(S, fast, p, grid, s);
+    if (S <= 12) return launch_leaf_11_12(S, fast, p, grid, s);
+    if (S <= 14) return launch_leaf_13_14(S, fast, p, grid, s);
+    if (S == 15) return launch_leaf_15_15(S, fast, p, grid, s);
+    return launch_leaf_16_16(S, fast, p, grid, s);
 }
 
 }  // namespace pos

@@ -3,7 +3,7 @@
 
 namespace pos {
 
-pos_status launch_leaf_11_13(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s) {
+pos_status launch_leaf_11_12(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s) {
     switch (S) {
         case 11:
             return fast ? launch_leaf_t<11, kPathFast>(p, grid, s)
@@ -11,9 +11,6 @@ pos_status launch_leaf_11_13(int S, bool fast, const LeafParams &p, int grid, cu
         case 12:
             return fast ? launch_leaf_t<12, kPathFast>(p, grid, s)
                         : launch_leaf_t<12, kPathGeneric>(p, grid, s);
-        case 13:
-            return fast ? launch_leaf_t<13, kPathFast>(p, grid, s)
-                        : launch_leaf_t<13, kPathGeneric>(p, grid, s);
         default:
             return fail(POS_EINVAL, "stage count outside this unit");
     }

@@ -3,17 +3,14 @@
 
 namespace pos {
 
-pos_status launch_leaf_14_16(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s) {
+pos_status launch_leaf_13_14(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s) {
     switch (S) {
+        case 13:
+            return fast ? launch_leaf_t<13, kPathFast>(p, grid, s)
+                        : launch_leaf_t<13, kPathGeneric>(p, grid, s);
         case 14:
             return fast ? launch_leaf_t<14, kPathFast>(p, grid, s)
                         : launch_leaf_t<14, kPathGeneric>(p, grid, s);
-        case 15:
-            return fast ? launch_leaf_t<15, kPathFast>(p, grid, s)
-                        : launch_leaf_t<15, kPathGeneric>(p, grid, s);
-        case 16:
-            return fast ? launch_leaf_t<16, kPathFast>(p, grid, s)
-                        : launch_leaf_t<16, kPathGeneric>(p, grid, s);
         default:
             return fail(POS_EINVAL, "stage count outside this unit");
     }
