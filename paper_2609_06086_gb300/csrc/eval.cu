@@ -114,7 +114,7 @@ __global__ void sort_scan_kernel(const uint32_t *hist, uint32_t *offs, uint32_t 
 
 // Each block takes chunks of kChunk candidates: counts their keys, reserves
 // one range per key with a single atomic, then places the indices.
-constexpr int kChunk = 32768;
+constexpr int kChunk = 8192;
 
 __global__ void sort_scatter_kernel(const uint4 *cands, int64_t n, uint32_t *cursor,
                                     uint32_t *perm) {
@@ -200,8 +200,8 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
             sort_hist_kernel<<<grid, 256, 0, stream>>>(p.cands, m, hist, p.T, p.F);
             sort_scan_kernel<<<1, 1024, 0, stream>>>(hist, offs, cursor);
             const int sgrid = (int)std::max<int64_t>(
-                1, std::min<int64_t>((m + kChunk - 1) / kChunk, 4LL * sm_count()));
-            sort_scatter_kernel<<<sgrid, 256, 0, stream>>>(p.cands, m, cursor, perm);
+                1, std::min<int64_t>((m + kChunk - 1) / kChunk, 8LL * sm_count()));
+            sort_scatter_kernel<<<sgrid, 512, 0, stream>>>(p.cands, m, cursor, perm);
             e = cudaGetLastError();
         }
         if (e == cudaSuccess) {
