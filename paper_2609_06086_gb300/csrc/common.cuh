@@ -29,7 +29,7 @@ pos_status cuda_fail(cudaError_t e, const char *what);
 // ---------------------------------------------------------------------------
 // Table blob: one contiguous device buffer, staged whole into shared memory
 // by every kernel.  Offsets are bytes from the blob start, 16-byte aligned.
-//   binom  u64 [128][16]        C(n, k), k <= 15
+//   binom  u64 [16][128]        C(n, k) at [k][n], k <= 15
 //   Pw, Pa i64 [K][L+1] each    exclusive prefix sums of mem_w, mem_a
 //   cap    i64 [K]
 //   Pf, Pb, Pd i32 [K][L+1]     exclusive prefix sums of fwd, bwd, dsync
@@ -115,8 +115,10 @@ __device__ __forceinline__ int32_t p2f(const Tab &t, int a, int b) {
 __device__ __forceinline__ int32_t p2b(const Tab &t, int a, int b) {
     return ld32(t.base, t.ly->off_p2b + 4u * (uint32_t)(a * t.ly->K + b));
 }
+// stored k-major ([k][n]) so that a warp reading C(n_lane, k) for one k
+// touches consecutive words (no shared-memory bank conflicts)
 __device__ __forceinline__ uint64_t binom(const Tab &t, int n, int k) {
-    return (uint64_t)ld64(t.base, t.ly->off_binom + 8u * (uint32_t)(n * kBinomK + k));
+    return (uint64_t)ld64(t.base, t.ly->off_binom + 8u * (uint32_t)(k * kBinomN + n));
 }
 
 // Cooperative 16-byte copy of the blob into shared memory.

@@ -2,6 +2,7 @@
 // step a9).  The evaluation kernels live in eval_kernel.cuh and the
 // eval_range_*.cu instantiation units.
 #include <mutex>
+#include <utility>
 
 #include "eval_kernel.cuh"
 
@@ -139,6 +140,41 @@ __global__ void sort_scatter_kernel(const uint4 *cands, int64_t n, uint32_t *cur
     }
 }
 
+// Decode pass over the whole sorted range [0, offs[kKeys]).
+__global__ void __launch_bounds__(256, 4) decode_kernel(EvalParams p) {
+    extern __shared__ __align__(16) unsigned char sm[];
+    stage_blob(sm, p.blob, p.lay.bytes);
+    __syncthreads();
+    const Tab t = tab_at(sm, p.lay);
+    const int64_t total = p.offs[kKeys];
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t span = (total + 31) & ~(int64_t)31;
+    for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < span; j += stride) {
+        const bool active = j < total;
+        uint32_t i = 0;
+        uint4 rec = make_uint4(0, 0, 0, 0);
+        if (active) {
+            i = __ldg(p.perm + j);
+            rec = __ldg(p.cands + i);
+        }
+        uint4 out = make_uint4(0, 0, 0, 1u << 24);
+        if (active) out = decode_one(t, rec, p, i);
+        if (active) p.cuts[j] = out;
+    }
+}
+
+pos_status launch_decode(const EvalParams &p, cudaStream_t stream) {
+    const int smem = p.lay.bytes;
+    POS_CUDA(cudaFuncSetAttribute(decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    int per_sm = 0;
+    POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_kernel, 256, smem));
+    const int64_t blocks = (p.n + 255) / 256;
+    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)std::max(per_sm, 1) * sm_count()));
+    decode_kernel<<<grid, 256, smem, stream>>>(p);
+    POS_CUDA(cudaGetLastError());
+    return POS_OK;
+}
+
 // Stream-ordered scratch comes from a library-owned pool per device that
 // keeps its memory between calls (release threshold: unlimited).
 static std::mutex g_pool_mutex;
@@ -175,9 +211,11 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
     for (int64_t base = 0; base < n; base += chunk) {
         const int64_t m = std::min(chunk, n - base);
         void *scratch = nullptr;
-        const size_t sbytes = sizeof(uint32_t) * (3 * (size_t)kKeys + 1 + (size_t)m);
+        // scratch: packed cuts (16 B per candidate), then the sort arrays
+        const size_t sbytes = 16 * (size_t)m + sizeof(uint32_t) * (3 * (size_t)kKeys + 1 + (size_t)m);
         POS_CUDA(cudaMallocFromPoolAsync(&scratch, sbytes, pool, stream));
-        uint32_t *hist = static_cast<uint32_t *>(scratch);
+        uint4 *cuts = static_cast<uint4 *>(scratch);
+        uint32_t *hist = reinterpret_cast<uint32_t *>(static_cast<char *>(scratch) + 16 * (size_t)m);
         uint32_t *offs = hist + kKeys;
         uint32_t *cursor = offs + kKeys + 1;
         uint32_t *perm = cursor + kKeys;
@@ -188,6 +226,7 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
         p.F = d_F + base;
         p.perm = perm;
         p.offs = offs;
+        p.cuts = cuts;
         p.blob = h->d_blob;
         p.lay = h->lay;
         p.gA = h->guard_A;
@@ -204,7 +243,8 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
             sort_scatter_kernel<<<sgrid, 512, 0, stream>>>(p.cands, m, cursor, perm);
             e = cudaGetLastError();
         }
-        if (e == cudaSuccess) {
+        if (e == cudaSuccess) st = launch_decode(p, stream);
+        if (e == cudaSuccess && st == POS_OK) {
             if ((st = eval_fast_1_4(p, stream)) == POS_OK && (st = eval_fast_5_8(p, stream)) == POS_OK &&
                 (st = eval_fast_9_12(p, stream)) == POS_OK &&
                 (st = eval_fast_13_16(p, stream)) == POS_OK &&

@@ -1,6 +1,10 @@
 // Evaluation kernels of poseidon_eval_batch (hot-path steps a2-a5).
 //
-// One thread evaluates one candidate.  The makespan loop costs ~6*S*M
+// One thread evaluates one candidate, in two passes over the (S, M)-sorted
+// batch: a decode pass (field checks, overflow guard, unranking, memory
+// check; few registers, so the latency of its dependent shared-memory
+// lookups is hidden by many warps) writes the cut positions in sorted order,
+// and the makespan pass reads them coalesced.  The makespan loop costs ~6*S*M
 // integer ops and its live registers grow with S (about 7*S), so the batch
 // is first counting-sorted by exact (S, M) into a permutation (stream-ordered
 // scratch), and then a family of kernels, each owning the candidates of one
@@ -34,43 +38,88 @@ struct EvalParams {
     uint8_t *F;
     const uint32_t *perm;  // sorted candidate indices
     const uint32_t *offs;  // [kKeys + 1] start of every key in perm
+    uint4 *cuts;           // per sorted position: cut[1..S-1] in bytes 0..14,
+                           // byte 15 = 1 when the result is already written
     const void *blob;
     BlobLayout lay;
     int64_t gA, gD, gP;
 };
 
+// Decode pass for one candidate: checks its fields and the overflow guard,
+// unranks the composition stage by stage (the steps of unrank_cuts),
+// checks each stage's memory as soon as its cut is known, and packs the cut
+// positions.  Invalid and overflowing candidates are answered here.  S is a
+// runtime value and the stage loop is not unrolled, which keeps the kernel
+// small enough to run many warps per SM.
+__device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, const EvalParams &p,
+                                            uint32_t i) {
+    uint64_t rank = (uint64_t)rec.x | ((uint64_t)rec.y << 32);
+    const uint32_t tcode = rec.z;
+    const int S = rec.w & 0xff;
+    const int M = (rec.w >> 8) & 0xff;
+    const int tp = (rec.w >> 16) & 0xff;
+    const int L = t.L();
+    bool ok = S >= 1 && S <= POS_MAX_STAGES && M >= 1 && S <= L && tp < t.n_tp() &&
+              rank < binom(t, L - 1, S - 1);
+    for (int s = 0; s < S && ok; ++s) ok = ((tcode >> (2 * s)) & 3) < (uint32_t)t.n_types();
+    const uint4 done = make_uint4(0, 0, 0, 1u << 24);  // byte 15 = 1: answered here
+    if (!ok) {
+        p.T[i] = -1;
+        p.F[i] = POS_FEAS_INVALID;
+        return done;
+    }
+    if (guard_trips(p.gA, p.gD, p.gP, S, M)) {
+        p.T[i] = -1;
+        p.F[i] = POS_FEAS_OVERFLOW;
+        return done;
+    }
+    uint64_t lo8 = 0, hi8 = 0;  // cut bytes 0..7 and 8..14
+    bool fits = true;
+    int c = 0;
+#pragma unroll 1
+    for (int s = 0; s < S; ++s) {
+        int c2 = L;
+        if (s < S - 1) {
+            const int rem = L - c, k = S - s - 1;
+            const uint64_t Y = binom(t, rem - 1, k) - rank;
+            int lo = k, hi = rem - 1;
+            while (lo < hi) {
+                const int mid = (lo + hi) >> 1;
+                if (binom(t, mid, k) >= Y) hi = mid;
+                else lo = mid + 1;
+            }
+            rank = binom(t, lo, k) - Y;
+            c2 = c + (rem - lo);
+            if (s < 8) lo8 |= (uint64_t)c2 << (8 * s);
+            else hi8 |= (uint64_t)c2 << (8 * (s - 8));
+        }
+        const int cls = ((tcode >> (2 * s)) & 3) * t.n_tp() + tp;
+        fits &= stage_fits(t, S, M, s, cls, c, c2);
+        c = c2;
+    }
+    p.F[i] = fits ? POS_FEAS_YES : POS_FEAS_NO;
+    return make_uint4((uint32_t)lo8, (uint32_t)(lo8 >> 32), (uint32_t)hi8,
+                      (uint32_t)(hi8 >> 32) & 0x00ffffffu);
+}
+
 template <int PATH>
 struct EvalWith {
     template <int S>
     struct One {
+        // makespan of a decoded candidate (cuts packed by Decode<S>)
         static __device__ __forceinline__ void run(const Tab &t, const uint4 &rec,
-                                                   const EvalParams &p, int32_t &T, uint8_t &F) {
-            const uint64_t rank = (uint64_t)rec.x | ((uint64_t)rec.y << 32);
+                                                   const uint4 &packed, int32_t &T) {
             const uint32_t tcode = rec.z;
             const int M = (rec.w >> 8) & 0xff;
             const int tp = (rec.w >> 16) & 0xff;
-            bool ok = M >= 1 && S <= t.L() && tp < t.n_tp() && rank < binom(t, t.L() - 1, S - 1);
-            int cls[S];
+            int cls[S], cut[S + 1];
 #pragma unroll
-            for (int s = 0; s < S; ++s) {
-                const int ty = (tcode >> (2 * s)) & 3;
-                ok &= ty < t.n_types();
-                cls[s] = ty * t.n_tp() + tp;
-            }
-            if (!ok) {
-                T = -1;
-                F = POS_FEAS_INVALID;
-                return;
-            }
-            if (guard_trips(p.gA, p.gD, p.gP, S, M)) {
-                T = -1;
-                F = POS_FEAS_OVERFLOW;
-                return;
-            }
-            int cut[S + 1];
-            unrank_cuts<S>(t, rank, cut);
-            // memory first, so that its inputs are dead before the wavefront
-            F = plan_fits<S>(t, M, cut, cls) ? POS_FEAS_YES : POS_FEAS_NO;
+            for (int s = 0; s < S; ++s) cls[s] = ((tcode >> (2 * s)) & 3) * t.n_tp() + tp;
+            const uint32_t pw[4] = {packed.x, packed.y, packed.z, packed.w};
+            cut[0] = 0;
+#pragma unroll
+            for (int s = 0; s < S - 1; ++s) cut[s + 1] = (pw[s / 4] >> (8 * (s % 4))) & 0xff;
+            cut[S] = t.L();
             StageW<S> w;
             stage_weights<S>(t, cut, cls, w);
             T = makespan_1f1b<S, PATH>(w, M);
@@ -80,11 +129,11 @@ struct EvalWith {
 
 template <int SLO, int SHI, int PATH>
 __device__ __forceinline__ void dispatch_range(int S, const Tab &t, const uint4 &rec,
-                                               const EvalParams &p, int32_t &T, uint8_t &F) {
-#define POS_EV(n)                                                                              \
-    if (n >= SLO && n <= SHI && S == n) {                                                      \
-        EvalWith<PATH>::template One<(n >= SLO && n <= SHI) ? n : SLO>::run(t, rec, p, T, F); \
-        return;                                                                                \
+                                               const uint4 &packed, int32_t &T) {
+#define POS_EV(n)                                                                            \
+    if (n >= SLO && n <= SHI && S == n) {                                                    \
+        EvalWith<PATH>::template One<(n >= SLO && n <= SHI) ? n : SLO>::run(t, rec, packed, T); \
+        return;                                                                              \
     }
     POS_EV(1) POS_EV(2) POS_EV(3) POS_EV(4) POS_EV(5) POS_EV(6) POS_EV(7) POS_EV(8)
     POS_EV(9) POS_EV(10) POS_EV(11) POS_EV(12) POS_EV(13) POS_EV(14) POS_EV(15) POS_EV(16)
@@ -106,29 +155,27 @@ __global__ void __launch_bounds__(kEvalThreads, MINB) eval_kernel(EvalParams p) 
     // whole warps iterate together (ballots below)
     const int64_t span = ((end - begin) + 31) & ~(int64_t)31;
     for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < span; j += stride) {
-        const bool active = j < end - begin;
+        bool active = j < end - begin;
         uint32_t i = 0;
-        uint4 rec = make_uint4(0, 0, 0, 0);
+        uint4 rec = make_uint4(0, 0, 0, 0), packed = make_uint4(0, 0, 0, 0);
         if (active) {
             i = __ldg(p.perm + begin + j);
-            rec = __ldg(p.cands + i);
+            packed = __ldg(p.cuts + begin + j);
+            active = (packed.w >> 24) == 0;  // not answered by the decode pass
+            if (active) rec = __ldg(p.cands + i);
         }
         const int S = active ? (int)(rec.w & 0xff) : 0;
         int32_t T = -1;
-        uint8_t F = POS_FEAS_INVALID;
         unsigned pending = __ballot_sync(0xffffffffu, active);
         while (pending) {
             const int leader = __ffs(pending) - 1;
             const int Sg = __shfl_sync(0xffffffffu, S, leader);
             const bool mine = active && S == Sg;
             const unsigned grp = __ballot_sync(0xffffffffu, mine);
-            if (mine) dispatch_range<SLO, SHI, PATH>(Sg, t, rec, p, T, F);
+            if (mine) dispatch_range<SLO, SHI, PATH>(Sg, t, rec, packed, T);
             pending &= ~grp;
         }
-        if (active) {
-            p.T[i] = T;
-            p.F[i] = F;
-        }
+        if (active) p.T[i] = T;
     }
 }
 
@@ -146,6 +193,8 @@ pos_status launch_eval_range(const EvalParams &p, cudaStream_t stream) {
     POS_CUDA(cudaGetLastError());
     return POS_OK;
 }
+
+pos_status launch_decode(const EvalParams &p, cudaStream_t stream);
 
 // one launcher per instantiation unit (eval_range_*.cu)
 pos_status eval_fast_1_4(const EvalParams &p, cudaStream_t s);

@@ -135,11 +135,11 @@ pos_status build_blob(const pos_tables *t, std::vector<unsigned char> &host, Blo
     ly = make_layout(L, t->n_types, t->n_tp);
     host.assign(ly.bytes, 0);
     // binomials by Pascal's rule (k <= 15 is exact in 64 bits for n <= 127)
-    uint64_t *bn = reinterpret_cast<uint64_t *>(host.data() + ly.off_binom);
+    uint64_t *bn = reinterpret_cast<uint64_t *>(host.data() + ly.off_binom);  // [k][n]
     for (int n = 0; n < kBinomN; ++n)
         for (int k = 0; k < kBinomK; ++k)
-            bn[n * kBinomK + k] =
-                k == 0 ? 1 : (n == 0 ? 0 : bn[(n - 1) * kBinomK + k - 1] + bn[(n - 1) * kBinomK + k]);
+            bn[k * kBinomN + n] =
+                k == 0 ? 1 : (n == 0 ? 0 : bn[(k - 1) * kBinomN + n - 1] + bn[k * kBinomN + n - 1]);
     // raw rows at entries 1..L; prefix_rows_kernel turns them into sums
     int64_t *Pw_ = reinterpret_cast<int64_t *>(host.data() + ly.off_Pw);
     int64_t *Pa_ = reinterpret_cast<int64_t *>(host.data() + ly.off_Pa);
