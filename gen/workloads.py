@@ -236,7 +236,7 @@ def random_candidates(n: int, *, L: int, n_types: int, S_range=(2, 16), M_range=
         mask = np.where(S >= 16, np.uint64(0xFFFFFFFF),
                         (np.uint64(1) << (2 * S).astype(np.uint64)) - np.uint64(1)).astype(np.uint32)
         tc = tc & mask
-        rank = rng.integers(0, highs[S].astype(np.int64), size=m).astype(np.uint64)
+        rank = rng.integers(0, highs[S], size=m, dtype=np.uint64)
         o = out[lo:hi]
         o["map_rank"] = rank
         o["type_code"] = tc

@@ -159,3 +159,30 @@ def test_config5_full_size_sampled(P, orc):
     ti = torch.from_numpy(idx).cuda()
     assert np.array_equal(d_T[ti].cpu().numpy(), Tr)
     assert np.array_equal(d_F[ti].cpu().numpy(), Fr)
+
+
+def _max_tables(L, n_types, n_tp, seed):
+    rng = np.random.default_rng(seed)
+    K = n_types * n_tp
+    return dict(L=L, n_types=n_types, n_tp=n_tp,
+                fwd=rng.integers(1, 40_000, (K, L)), bwd=rng.integers(1, 80_000, (K, L)),
+                dsync=rng.integers(0, 500, (K, L)), p2p_f=rng.integers(0, 300, (K, K)),
+                p2p_b=rng.integers(0, 300, (K, K)), mem_w=rng.integers(0, 10 ** 9, (K, L)),
+                mem_a=rng.integers(0, 10 ** 8, (K, L)),
+                cap=rng.integers(10 ** 9, 10 ** 11, K))
+
+
+def test_limits_L127_four_types_eight_tp(P, orc):
+    """The largest tables the ABI accepts: L = 127 (ranks up to C(126, 15) ~ 1.2e19),
+    4 device types x 8 TP degrees, S up to 16 and M up to 255 (guard permitting)."""
+    tab = _max_tables(127, 4, 8, 3)
+    h = P.Handle(P.Tables(**tab))
+    c = gen.random_candidates(40_000, L=127, n_types=4, S_range=(1, 16), M_range=(1, 255),
+                              seed=3)
+    c["tp_idx"] = np.random.default_rng(4).integers(0, 8, len(c))
+    c[:100]["S"] = 16
+    c[:50]["map_rank"] = math.comb(126, 15) - 1 - np.arange(50, dtype=np.uint64)
+    T, F = eval_device(P, h, c)
+    Tr, Fr = orc.eval_batch(orc.OracleTables(**tab), c)
+    assert np.array_equal(T, Tr) and np.array_equal(F, Fr)
+    assert (F == 3).sum() > 0 and (F == 1).sum() > 0

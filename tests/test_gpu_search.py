@@ -114,3 +114,37 @@ def test_infeasible_and_overflow(P):
     with pytest.raises(P.PoseidonError) as e:
         gpu_search(P, w)
     assert e.value.status == P.binding.POS_EOVERFLOW
+
+
+def _limits_problem(seed, S, L, n_types, placement, counts, M_list):
+    rng = np.random.default_rng(seed)
+    K = n_types
+    w = gen.Workload(name="limits", L=L, n_types=n_types, n_tp=1,
+                     fwd=rng.integers(1, 500, (K, L)).astype(np.int32),
+                     bwd=rng.integers(1, 900, (K, L)).astype(np.int32),
+                     dsync=rng.integers(0, 200, (K, L)).astype(np.int32),
+                     p2p_f=rng.integers(0, 100, (K, K)).astype(np.int32),
+                     p2p_b=rng.integers(0, 100, (K, K)).astype(np.int32),
+                     mem_w=rng.integers(0, 4, (K, L)).astype(np.int64),
+                     mem_a=rng.integers(0, 2, (K, L)).astype(np.int64),
+                     cap=(rng.integers(20, 60, K) * L // 10).astype(np.int64),
+                     S=S, M_list=M_list, tp_list=[1], dp_list=[1], placement=placement,
+                     type_counts=counts, seed=seed)
+    return w
+
+
+@pytest.mark.parametrize("S,L,types,placement,counts,M_list", [
+    (16, 19, 1, 0, [], [16, 40]),          # 16 stages, M = S and M > S
+    (16, 18, 2, 1, [8, 8], [5]),           # M < S with 16 stages, exact placement
+    (12, 16, 4, 1, [3, 3, 3, 3], [12]),    # 4 device types
+    (3, 127, 2, 0, [], [255]),             # the longest model, the most micro-batches
+])
+def test_search_at_the_limits(P, orc, S, L, types, placement, counts, M_list):
+    w = _limits_problem(S * 31 + L, S, L, types, placement, counts, M_list)
+    ref, _ = orc.search(w, prune=True, warmup=0)
+    try:
+        plan, _ = gpu_search(P, w, prune=True, warmup=200, seed=1)
+    except P.PoseidonError as e:
+        assert e.status == P.binding.POS_EINFEASIBLE and not ref["found"]
+        return
+    assert same_plan(plan, ref), (plan, ref)
