@@ -35,6 +35,8 @@ METRIC = "DAG makespan evals/sec (time-to-optimal plan at L=80, S=8)"
 WARMUP_SAMPLES = 65536
 SM_LANES = 128  # INT32 lanes per SM (4 partitions x 32)
 ENTRY_BYTES = 32  # one frontier entry / one complete plan
+PRUNE_NAMES = {1: "stage-level, Eq. 2 as printed (Theorem 1)",
+               2: "stage-level, tightened: Eq. 2 with P2P edges + completion bounds"}
 
 
 def measured_hbm():
@@ -187,7 +189,7 @@ def run_ours(args, rank, world, local_rank):
         import torch.distributed as dist
         dist.init_process_group("nccl" if args.backend == "nccl" else "gloo")
     w = gen.config4()
-    prob, keep = P.make_problem(w, warmup=WARMUP_SAMPLES, prune=True, seed=0,
+    prob, keep = P.make_problem(w, warmup=WARMUP_SAMPLES, prune=args.prune, seed=0,
                                 frontier_cap=args.frontier_cap)
     tab_bytes = sum(a.nbytes for a in keep[0].arrays.values()) + sum(a.nbytes for a in keep[1:])
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.int32, device="cuda")
@@ -272,6 +274,26 @@ def run_ours(args, rank, world, local_rank):
             "peak_note": (f"{n_sm} SMs x {SM_LANES} int32 lanes x {mhz:.0f} MHz (median SM "
                           "clock under load)" if b == "alu" else hbm_src)}
     evals = [eval_throughput(P, torch, int(n), 5, peak_alu) for n in args.eval_sizes]
+    # the other stage-level prune, same workload, for comparison (not the headline)
+    other = PRUNE_NAMES[1 if args.prune == 2 else 2]
+    other_mode = 1 if args.prune == 2 else 2
+    prob2, keep2 = P.make_problem(w, warmup=WARMUP_SAMPLES, prune=other_mode, seed=0,
+                                  frontier_cap=args.frontier_cap)
+    P.poseidon_search(prob2)
+    o_ms, o_ev, o_ok = [], 0, True
+    for _ in range(max(3, args.steps // 2)):
+        flush.zero_()
+        torch.cuda.synchronize()
+        ev0.record()
+        plan2, st2 = P.poseidon_search(prob2)
+        ev1.record()
+        torch.cuda.synchronize()
+        o_ms.append(ev0.elapsed_time(ev1))
+        o_ev += st2["evaluated"]
+        o_ok &= plan2["global_index"] == ref["plan"]["global_index"]
+    other_prune = {"prune": other, "time_to_plan_s": sum(o_ms) / len(o_ms) / 1e3,
+                   "evaluations_per_step": o_ev / len(o_ms),
+                   "evals_per_s": o_ev / (sum(o_ms) / 1e3), "matches_oracle": o_ok}
     cpu_rate, cpu_n, cpu_t = oracle_sample_rate(args.cpu_seconds)
     line = {
         "metric": METRIC, "value": value, "unit": "evals/s", "n_gpus": world,
@@ -279,7 +301,7 @@ def run_ours(args, rank, world, local_rank):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int32",
         "data": "synthetic",
         "config": {"workload": WORKLOAD, "warmup_samples": WARMUP_SAMPLES,
-                   "prune": "stage-level, Eq. 2", "l2": "flushed (256 MB write) between steps",
+                   "prune": PRUNE_NAMES[args.prune], "l2": "flushed (256 MB write) between steps",
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "time_to_plan_s": t_dev / args.steps / 1e3,
         "relaxations_per_s": agg["relaxations"] * world / (t_dev / 1e3),
@@ -292,6 +314,7 @@ def run_ours(args, rank, world, local_rank):
         "host_ms_per_step": {k: round(agg[k] / args.steps, 3)
                              for k in ("ms_setup", "ms_warmup", "ms_search")},
         "roofline": roof,
+        "other_prune": other_prune,
         "eval_throughput": evals,
         "cpu_baseline": {"value": cpu_rate, "unit": "evals/s", "cores": 1, "kind": "oracle",
                          "sample": f"{cpu_n} config-4 plan evaluations (S=8, M=32, L=80) in "
@@ -316,6 +339,8 @@ def main():
     ap.add_argument("--backend", choices=["nccl", "gloo"], default="nccl")
     ap.add_argument("--eval-sizes", type=float, nargs="*", default=[1e7],
                     help="config-5 batch sizes for the evaluator measurement")
+    ap.add_argument("--prune", type=int, choices=[1, 2], default=2,
+                    help="stage-level prune: 1 = Eq. 2 as printed, 2 = tightened bound")
     ap.add_argument("--frontier-cap", type=int, default=0,
                     help="frontier entries per depth (0 = library default)")
     args = ap.parse_args()

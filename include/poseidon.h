@@ -175,6 +175,28 @@ pos_status poseidon_argmin_noalloc(const int32_t *d_makespan, const uint8_t *d_f
  * n_map = C(L-1, S-1).  Objective: time per sample T/(D*M), compared exactly;
  * ties go to the lowest global index.
  */
+/* Stage-level pruning (Sec. 4.2.1).  Every mode returns the same plan.
+ *   POS_PRUNE_NONE   exhaustive enumeration (memory cut only).
+ *   POS_PRUNE_EQ2    cut a prefix S_x when g(S_x) > T_min, g of Eq. 2 as
+ *                    printed (Theorem 1).
+ *   POS_PRUNE_TIGHT  a larger valid bound, not in the paper: Eq. 2 with the
+ *                    inter-stage F and B edges on its path added, and the
+ *                    largest of two bounds over the stages not yet placed.
+ *                    For a complete plan and 1-based stages i <= y, the path
+ *                    through the first micro-batch's forwards up to y, stage
+ *                    y's whole chain, the last micro-batch's backwards down
+ *                    to i and R_i has length
+ *                      P(y, i) = sum_{j<y} (F_j + pf_j) + M (F_y + B_y)
+ *                                + sum_{j=i}^{y-1} (B_j + pb_j) + d_i <= T;
+ *                    the prefix bound is max( max_{i<=x} P(x, i),
+ *                    min over memory-feasible completions of max_{y>x} P(y, y),
+ *                    min over them of max_{y>x, i<=x} P(y, i) ), the minima
+ *                    taken from per-slice tables built by a dynamic program
+ *                    over (stage, first layer). */
+#define POS_PRUNE_NONE 0
+#define POS_PRUNE_EQ2 1
+#define POS_PRUNE_TIGHT 2
+
 typedef struct pos_problem {
     pos_tables tables;
     int32_t S;
@@ -185,7 +207,7 @@ typedef struct pos_problem {
     int32_t placement;          /* POS_PLACE_FREE or POS_PLACE_EXACT */
     const int32_t *type_counts; /* [n_types] stages per type (POS_PLACE_EXACT) */
     int32_t warmup;             /* random feasible samples seeding T_min (paper: 500) */
-    int32_t prune;              /* 1: stage-level prune g(S_x) > T_min (Eq. 2); 0: exhaustive */
+    int32_t prune;              /* POS_PRUNE_NONE, POS_PRUNE_EQ2 or POS_PRUNE_TIGHT */
     uint64_t seed;              /* warm-up sampling seed */
     int32_t schedule;           /* POS_SCHED_1F1B */
     int64_t frontier_cap;       /* entries per frontier buffer; 0 = default 2^24;
@@ -217,13 +239,20 @@ typedef struct pos_search_stats {
     /* frontier entries read by the expansion / completion kernels, and
        complete plans written by the completion kernel */
     uint64_t parents_expand, parents_complete, leaves;
+    /* POS_PRUNE_TIGHT: device time and launches of the completion-bound
+       tables (one launch per batch of slices) */
+    double ms_bound;
+    uint64_t bound_launches;
+    /* batches of slices run a second time, host-driven, because a frontier
+       of their pipelined pass overflowed frontier_cap */
+    uint64_t reruns;
 } pos_search_stats;
 
 /*
  * Exact search (Sec. 4.2.3) on the current CUDA device: warm-up sampling,
  * then enumeration of every slice's layer compositions with the memory cut
- * and, if prune != 0, the stage-level prune of Eq. 2 / Theorem 1; the result
- * equals the exhaustive optimum.  Host pointers in, host plan out;
+ * and the stage-level prune chosen by problem->prune (Eq. 2 / Theorem 1, or
+ * the tighter bound); the result equals the exhaustive optimum.  Host pointers in, host plan out;
  * synchronous.  stats may be NULL.
  * Errors: POS_EINVAL, POS_EOVERFLOW (guard fails for some M), POS_ENOMEM,
  * POS_ECUDA, POS_ETIMEOUT, POS_EINFEASIBLE (no memory-feasible plan; *out
@@ -231,7 +260,9 @@ typedef struct pos_search_stats {
  * Limits: at most 65535 slices with a feasible root per M value; the global
  * index must fit in 64 bits; lcm of all D*M below 2^32.
  * Memory: the work buffers (one frontier of frontier_cap 32-byte entries per
- * depth, a leaf buffer of the same length, slice and feasibility tables),
+ * depth, a leaf buffer of the same length, slice and feasibility tables,
+ * and with POS_PRUNE_TIGHT 1 KB of bound tables per stage and slice of a
+ * batch),
  * a stream and pinned counters are kept per device between calls, grown on
  * demand and released at process exit; concurrent searches on one device
  * are serialised.

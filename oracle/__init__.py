@@ -85,6 +85,9 @@ def lib():
         L.orc_lower_bound.restype = C.c_int64
         L.orc_lower_bound.argtypes = [C.POINTER(Tables), C.c_int, C.c_int, C.c_void_p,
                                       C.c_void_p, C.c_int]
+        L.orc_lower_bound_tight.restype = C.c_int64
+        L.orc_lower_bound_tight.argtypes = [C.POINTER(Tables), C.c_int, C.c_int, C.c_void_p,
+                                            C.c_void_p, C.c_int]
         L.orc_eval_batch.restype = C.c_int
         L.orc_eval_batch.argtypes = [C.POINTER(Tables), C.c_void_p, C.c_int64, C.c_void_p,
                                      C.c_void_p]
@@ -166,6 +169,18 @@ def finish_times(tab: OracleTables, S, M, cls, layers):
 def lower_bound(tab: OracleTables, S, M, cls, layers, x):
     c, l = _i32(cls, S), _i32(layers, S)
     g = lib().orc_lower_bound(C.byref(tab.c), S, M, c.ctypes.data, l.ctypes.data, x)
+    if g < 0:
+        raise ValueError("invalid configuration")
+    return int(g)
+
+
+def lower_bound_tight(tab: OracleTables, S, M, cls, layers, x):
+    """Tightened prefix bound (P2P-inclusive Eq. 2 plus the completion
+    terms); None when no memory-feasible completion exists."""
+    c, l = _i32(cls, S), _i32(layers, S)
+    g = lib().orc_lower_bound_tight(C.byref(tab.c), S, M, c.ctypes.data, l.ctypes.data, x)
+    if g == -2:
+        return None
     if g < 0:
         raise ValueError("invalid configuration")
     return int(g)

@@ -33,6 +33,7 @@
  */
 #include "oracle.h"
 
+#include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
 
@@ -415,6 +416,99 @@ int64_t orc_lower_bound(const orc_tables *t, int S, int M, const int32_t *cls,
     stage_w sw;
     stage_weights(t, S, cls, layers, &sw);
     return lower_bound_w(&sw, M, x);
+}
+
+/* ------------------------------------------------------------------ */
+/* Tightened stage-level bound (the P2P-inclusive form of Eq. 2 plus a   */
+/* bound over the unplaced stages).  Not in the paper: a library option. */
+/* ------------------------------------------------------------------ */
+/* Length of one S -> E path of the DAG of a complete configuration, for
+ * 1 <= i <= y <= S (1-based): the first micro-batch's forwards and their
+ * F edges up to stage y, stage y's whole chain (M forwards and M
+ * backwards, first op F_{y,1}, last op B_{y,M}), the last micro-batch's
+ * backwards and B edges from stage y down to stage i, and R_i:
+ *   P(y, i) = sum_{j<y} (F_j + pf_j) + M (F_y + B_y)
+ *             + sum_{j=i}^{y-1} (B_j + pb_j) + d_i.
+ * Every such path exists (Sec. 4.1.2), so P(y, i) <= T. */
+static int64_t path_len(const stage_w *w, int M, int y, int i) {
+    int64_t v = 0;
+    for (int j = 1; j <= y - 1; ++j) v += w->F[j - 1] + w->pf[j - 1];
+    v += (int64_t)M * (w->F[y - 1] + w->B[y - 1]);
+    for (int j = i; j <= y - 1; ++j) v += w->B[j - 1] + w->pb[j - 1];
+    return v + w->d[i - 1];
+}
+
+typedef struct {
+    const orc_tables *t;
+    int S, M, x;
+    const int32_t *cls;
+    int32_t layers[ORC_MAX_S];
+    int64_t best2, best3; /* minima over the completions seen so far */
+    int any;
+} tight_ctx;
+
+/* Every memory-feasible completion of stages x+1..S: the two completion
+ * terms of the bound, each minimised over completions separately. */
+static void tight_completions(tight_ctx *q, int s /* 0-based next stage */, int first) {
+    const int L = q->t->L, S = q->S;
+    if (s == S) {
+        if (first != L) return;
+        stage_w w;
+        stage_weights(q->t, S, q->cls, q->layers, &w);
+        int64_t v2 = INT64_MIN, v3 = INT64_MIN;
+        for (int y = q->x + 1; y <= S; ++y) {
+            const int64_t a = path_len(&w, q->M, y, y);
+            if (a > v2) v2 = a;
+            for (int i = 1; i <= q->x; ++i) {
+                const int64_t b = path_len(&w, q->M, y, i);
+                if (b > v3) v3 = b;
+            }
+        }
+        if (!q->any || v2 < q->best2) q->best2 = v2;
+        if (!q->any || v3 < q->best3) q->best3 = v3;
+        q->any = 1;
+        return;
+    }
+    for (int l = 1; first + l <= L - (S - s - 1); ++l) {
+        if (!stage_memory_ok(q->t, S, q->M, s, q->cls[s], first, l)) continue;
+        q->layers[s] = l;
+        tight_completions(q, s + 1, first + l);
+    }
+}
+
+int64_t orc_lower_bound_tight(const orc_tables *t, int S, int M, const int32_t *cls,
+                              const int32_t *layers, int x) {
+    if (x < 1 || x > S || S > ORC_MAX_S || M < 1) return -1;
+    int first = 0;
+    for (int s = 0; s < x; ++s) {
+        if (layers[s] < 1) return -1;
+        first += layers[s];
+    }
+    if (first > t->L - (S - x)) return -1;
+    tight_ctx q;
+    memset(&q, 0, sizeof(q));
+    q.t = t;
+    q.S = S;
+    q.M = M;
+    q.x = x;
+    q.cls = cls;
+    for (int s = 0; s < x; ++s) q.layers[s] = layers[s];
+    /* term 1: the paths through stage x itself, which the prefix fixes
+       (Eq. 2 with the F and B edges on the path added) */
+    stage_w w;
+    for (int s = x; s < S; ++s) q.layers[s] = 1; /* placeholder: only stages <= x are read */
+    stage_weights(t, S, cls, q.layers, &w);
+    int64_t lb = INT64_MIN;
+    for (int i = 1; i <= x; ++i) {
+        const int64_t v = path_len(&w, M, x, i);
+        if (v > lb) lb = v;
+    }
+    if (x == S) return lb;
+    tight_completions(&q, x, first);
+    if (!q.any) return -2; /* no memory-feasible completion */
+    if (q.best2 > lb) lb = q.best2;
+    if (q.best3 > lb) lb = q.best3;
+    return lb;
 }
 
 int orc_eval_batch(const orc_tables *t, const orc_candidate *c, int64_t n, int32_t *T,

@@ -89,6 +89,19 @@ int orc_eval_finish(const orc_tables *t, int S, int M, const int32_t *cls, const
 /* g(S_x) of Eq. 2 for the prefix of stages 1..x (1 <= x <= S). */
 int64_t orc_lower_bound(const orc_tables *t, int S, int M, const int32_t *cls,
                         const int32_t *layers, int x);
+/* Tightened lower bound for the prefix of stages 1..x (only layers[0..x-1]
+ * are read).  With the path lengths
+ *   P(y, i) = sum_{j<y} (F_j + pf_j) + M (F_y + B_y) + sum_{j=i}^{y-1} (B_j + pb_j) + d_i
+ * of a complete configuration (1 <= i <= y <= S), it is the largest of
+ *   max_{i<=x} P(x, i)                        (Eq. 2 with the P2P edges),
+ *   min over completions of max_{y>x} P(y, y),
+ *   min over completions of max_{y>x, i<=x} P(y, i),
+ * the minima taken over the memory-feasible completions of stages x+1..S,
+ * enumerated one by one.  Each P(y, i) is a path of the DAG, so the bound
+ * never exceeds the makespan of a feasible completion.  Returns -1 on
+ * invalid input and -2 when no completion fits in memory. */
+int64_t orc_lower_bound_tight(const orc_tables *t, int S, int M, const int32_t *cls,
+                              const int32_t *layers, int x);
 /* Decode and evaluate n candidate records.  feasible: 1 ok, 0 memory
  * infeasible, 2 invalid record, 3 overflow guard tripped. */
 int orc_eval_batch(const orc_tables *t, const orc_candidate *c, int64_t n, int32_t *T,

@@ -60,7 +60,8 @@ class pos_search_stats(C.Structure):
                                           "ms_expand", "ms_complete", "ms_leaf")] + \
                [(n, C.c_uint64) for n in ("expand_launches", "complete_launches",
                                           "leaf_launches", "parents_expand", "parents_complete",
-                                          "leaves")]
+                                          "leaves")] + \
+               [("ms_bound", C.c_double), ("bound_launches", C.c_uint64), ("reruns", C.c_uint64)]
 
 
 class PoseidonError(RuntimeError):
@@ -170,6 +171,16 @@ def poseidon_argmin_noalloc(d_makespan: int, d_feasible: int, n: int, d_out: int
     _check(lib().poseidon_argmin_noalloc(d_makespan, d_feasible, n, d_out, stream))
 
 
+POS_PRUNE_NONE, POS_PRUNE_EQ2, POS_PRUNE_TIGHT = 0, 1, 2
+
+
+def _prune_mode(prune):
+    """False/True map to POS_PRUNE_NONE/POS_PRUNE_EQ2; 0, 1, 2 pass through."""
+    if isinstance(prune, bool):
+        return POS_PRUNE_EQ2 if prune else POS_PRUNE_NONE
+    return int(prune)
+
+
 def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0):
     """pos_problem for a gen.Workload search; returns (problem, keep-alive list)."""
     tab = Tables.from_workload(w)
@@ -182,7 +193,7 @@ def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0):
 
     p = pos_problem(tab.c, w.S, len(w.M_list), arr(w.M_list), arr(w.tp_list), arr(w.dp_list),
                     w.placement, arr(w.type_counts if w.type_counts else [0] * w.n_types),
-                    int(warmup), int(bool(prune)), int(seed), POS_SCHED_1F1B, int(frontier_cap))
+                    int(warmup), _prune_mode(prune), int(seed), POS_SCHED_1F1B, int(frontier_cap))
     return p, keep
 
 

@@ -26,6 +26,7 @@
 namespace pos {
 
 constexpr int kThreads = 256;
+constexpr int32_t kNoCompletion = 0x7fffffff;  // completion-bound entry without a completion
 
 // ---------------------------------------------------------------------------
 // suffix feasibility: one block per slice, thread c
@@ -81,6 +82,75 @@ __device__ __forceinline__ bool feas_bit(const uint4 *feas, int S, uint32_t gid,
 __global__ void root_bits_kernel(const uint4 *feas, int n_slices, int S, uint8_t *out) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i < n_slices) out[i] = feas_bit(feas, S, i, 0, 0);
+}
+
+// ---------------------------------------------------------------------------
+// completion bounds (prune mode 2).  For a complete plan and 0-based stages
+// i <= y, the DAG path through the first micro-batch's forwards up to stage
+// y, stage y's whole chain, the last micro-batch's backwards down to stage i
+// and R_i has length
+//   P(y, i) = sum_{j<y} (F_j + pf_j) + M (F_y + B_y) + sum_{j=i}^{y-1} (B_j + pb_j) + d_i,
+// so T >= P(y, i).  Eq. 2 is max_i P(x, i) without the edges.  Over the
+// stages y >= x that a prefix has not placed yet, with A = sum_{j<x}
+// (F_j + pf_j) and Bm = max_{i<x} (sum_{j=i}^{x-1} (B_j + pb_j) + d_i):
+//   max_{y>=x} P(y, y)          = A + V1,
+//   max_{y>=x, i<x} P(y, i)     = A + Bm + V2,
+// where, for the stages x..S-1 covering layers [c, L),
+//   V1 = max_y (sum_{x<=j<y} (F_j + pf_j) + M (F_y + B_y) + d_y),
+//   V2 = max_y (sum_{x<=j<y} (F_j + pf_j + B_j + pb_j) + M (F_y + B_y)).
+// V1[x][c] and V2[x][c] hold their minima over every memory-feasible
+// completion, by the recursion over stage x's layer count l
+//   V1[x][c] = min_l max(M (F + B) + d, F + pf_x + V1[x+1][c+l]),
+//   V2[x][c] = min_l max(M (F + B),     F + pf_x + B + pb_x + V2[x+1][c+l]).
+// A prefix whose A + V1 or A + Bm + V2 exceeds the incumbent has no
+// completion that beats it.  Each finite entry is at most the makespan of
+// a feasible plan, so it fits in int32 under the overflow guard.
+// One block per slot of the batch, thread c; vb[(slot*S + x)*128 + c].
+__global__ void bound_kernel(const SliceRec *batch, int nb, int S, const uint8_t *lim, int2 *vb,
+                             const void *blob, BlobLayout lay) {
+    extern __shared__ __align__(16) unsigned char sm[];
+    __shared__ int2 nxt[128];
+    stage_blob(sm, blob, lay.bytes);
+    __syncthreads();
+    const Tab t = tab_at(sm, lay);
+    const int L = lay.L, c = threadIdx.x;
+    for (int slot = blockIdx.x; slot < nb; slot += gridDim.x) {
+        const SliceRec &sr = batch[slot];
+        const int M = sr.M;
+        for (int x = S - 1; x >= 1; --x) {
+            const int k = sr.cls[x];
+            const int32_t pf = x + 1 < S ? p2f(t, k, sr.cls[x + 1]) : 0;
+            const int32_t pb = x + 1 < S ? p2b(t, sr.cls[x + 1], k) : 0;
+            int64_t v1 = INT64_MAX, v2 = INT64_MAX;
+            if (c < L) {
+                const int most = lim[((size_t)sr.gid * S + x) * 128 + c];
+                const int32_t f0 = Pf(t, k, c), b0 = Pb(t, k, c), d0 = Pd(t, k, c);
+                const int l_lo = x == S - 1 ? L - c : 1;
+                const int l_hi = x == S - 1 ? L - c : min(most, L - c - (S - 1 - x));
+                for (int l = l_lo; l <= l_hi && l <= most; ++l) {
+                    const int c2 = c + l;
+                    const int64_t F = Pf(t, k, c2) - f0, B = Pb(t, k, c2) - b0;
+                    const int64_t d = Pd(t, k, c2) - d0;
+                    const int64_t a = (int64_t)M * (F + B);
+                    if (x == S - 1) {
+                        v1 = a + d;
+                        v2 = a;
+                    } else {
+                        const int2 n = nxt[c2];
+                        if (n.x == kNoCompletion) continue;
+                        v1 = min(v1, max(a + d, F + pf + n.x));
+                        v2 = min(v2, max(a, F + pf + B + pb + n.y));
+                    }
+                }
+            }
+            __syncthreads();  // every thread has read row x+1
+            const int2 out = v1 == INT64_MAX ? make_int2(kNoCompletion, kNoCompletion)
+                                             : make_int2((int32_t)v1, (int32_t)v2);
+            nxt[c] = out;
+            vb[((size_t)slot * S + x) * 128 + c] = out;
+            __syncthreads();
+        }
+    }
 }
 
 // ---------------------------------------------------------------------------
@@ -143,6 +213,7 @@ __global__ void sample_kernel(const SliceRec *slices, const uint32_t *feasible, 
 struct ExpandParams {
     const Prefix *in;
     long long n_in;
+    const unsigned long long *n_in_dev;  // if set: n_in = min(*n_in_dev, cap), read on the device
     const uint32_t *groups;  // work list of 32-parent groups, or NULL = all groups
     long long n_groups;
     int x;                   // depth of the parents (stages 0..x-1 placed)
@@ -151,6 +222,7 @@ struct ExpandParams {
     const SliceRec *slices;
     const uint4 *feas;
     const uint8_t *lim;      // per (slice, stage, start) memory limit, see feas_kernel
+    const int2 *vb;          // prune 2: completion bounds per (batch slot, stage, start)
     Prefix *out;             // expand: children at depth x+1
     Leaf *leaves;            // complete: full plans
     unsigned long long *out_count;
@@ -200,6 +272,7 @@ __device__ __forceinline__ int last_true(int hi, Pred pred) {
 struct ParentCtx {
     int c, k;
     int32_t f0, b0, d0;
+    int32_t pf, pb;  // prune 2: F and B edge between the new stage and the next one
 };
 
 __device__ __forceinline__ ParentCtx parent_ctx(const Tab &t, int k, int c) {
@@ -209,6 +282,8 @@ __device__ __forceinline__ ParentCtx parent_ctx(const Tab &t, int k, int c) {
     q.f0 = Pf(t, k, c);
     q.b0 = Pb(t, k, c);
     q.d0 = Pd(t, k, c);
+    q.pf = 0;
+    q.pb = 0;
     return q;
 }
 
@@ -220,7 +295,7 @@ __device__ __forceinline__ ParentCtx parent_ctx(const Tab &t, int k, int c) {
 // (feasibility bits).
 __device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, int64_t A,
                                           int64_t Bm, const ParentCtx &q, uint32_t gid,
-                                          uint64_t scale,
+                                          int slot, uint64_t scale,
                                           uint64_t thr, Bits128 &acc, unsigned long long &cut_b,
                                           unsigned long long &cut_m) {
     const int S = p.S, M = p.M, x = p.x, L = t.L();
@@ -243,9 +318,45 @@ __device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, i
     acc.w[1] = f.y & win.w[1];
     acc.w[2] = f.z & win.w[2];
     acc.w[3] = f.w & win.w[3];
-    const int n = popc128(acc);
+    int n = popc128(acc);
     cut_m += (unsigned long long)(lmax - hi_mem) + (unsigned long long)(hi - n);
     cut_b += (unsigned long long)(hi_mem - hi);
+    if (p.prune == 2 && n > 0) {
+        // completion terms: the bound is not monotone in l, so every
+        // candidate child is tested on its own
+        const int2 *vrow = p.vb + ((size_t)slot * S + x + 1) * 128;
+#pragma unroll
+        for (int wd = 0; wd < 4; ++wd) {
+            uint32_t m = acc.w[wd];
+            while (m) {
+                // up to four candidates at a time, their table loads in flight together
+                int bb[4];
+                int2 v[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    bb[u] = m ? __ffs(m) - 1 : -1;
+                    m &= m - 1;
+                }
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    if (bb[u] >= 0) v[u] = __ldg(vrow + 32 * wd + bb[u]);
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    if (bb[u] < 0) continue;
+                    const int c2 = 32 * wd + bb[u];
+                    const int64_t F = Pf(t, q.k, c2) - q.f0, B = Pb(t, q.k, c2) - q.b0;
+                    const int64_t d = Pd(t, q.k, c2) - q.d0;
+                    const int64_t A2 = A + F + q.pf, Bm2 = max(Bm, d) + B + q.pb;
+                    if (v[u].x == kNoCompletion || (uint64_t)(A2 + v[u].x) * scale > thr ||
+                        (uint64_t)(A2 + Bm2 + v[u].y) * scale > thr) {
+                        acc.w[wd] &= ~(1u << bb[u]);
+                        --n;
+                        ++cut_b;
+                    }
+                }
+            }
+        }
+    }
     return n;
 }
 
@@ -292,7 +403,8 @@ __device__ __forceinline__ int complete_set(const ExpandParams &p, const Tab &t,
             const int64_t da = Pd(t, q.k, c2) - q.d0;
             const int64_t Fb = fbL - Pf(t, kb, c2), Bb = bbL - Pb(t, kb, c2);
             const int64_t db = dbL - Pd(t, kb, c2);
-            const int64_t g = A + Fa + (int64_t)M * (Fb + Bb) + max(max(Bm, da) + Ba, db);
+            const int64_t g =
+                A + Fa + q.pf + (int64_t)M * (Fb + Bb) + max(max(Bm, da) + Ba + q.pb, db);
             if ((uint64_t)g * scale > thr) {
                 ++cut_b;
                 continue;
@@ -321,13 +433,18 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
     const int lane = threadIdx.x & 31;
     const long long warp = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
     const long long n_warps = ((long long)gridDim.x * blockDim.x) >> 5;
-    const long long n_work = p.groups ? p.n_groups : (p.n_in + 31) / 32;
+    long long n_in = p.n_in;
+    if (p.n_in_dev) {
+        const unsigned long long c0 = __ldcg(p.n_in_dev);
+        n_in = (long long)(c0 < p.cap ? c0 : p.cap);
+    }
+    const long long n_work = p.groups ? p.n_groups : (n_in + 31) / 32;
     unsigned long long emitted = 0, cb = 0, cm = 0, parents = 0, written_parents = 0;
     for (long long w = warp; w < n_work; w += n_warps) {
         const long long g = p.groups ? (long long)p.groups[w] : w;
         const long long i = g * 32 + lane;
         Vec32 pv = {make_uint4(kPrefixHole, 0, 0, 0), make_uint4(0, 0, 0, 0)};
-        if (i < p.n_in) pv = load32(p.in + i);
+        if (i < n_in) pv = load32(p.in + i);
         const uint32_t slice = pv.a.x & 0xffffu;
         const bool live = slice != kPrefixHole;
         Bits128 acc = {{0u, 0u, 0u, 0u}};
@@ -340,11 +457,16 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
             // parent byte 2+i holds cut[i]
             const int c = X > 0 ? (int)get_byte<(X > 0 ? X + 1 : 2)>(pv) : 0;
             q = parent_ctx(t, sr.cls[X], c);
+            if (p.prune == 2) {  // X + 1 <= S - 1: the next stage exists
+                q.pf = p2f(t, sr.cls[X], sr.cls[X + 1]);
+                q.pb = p2b(t, sr.cls[X + 1], sr.cls[X]);
+            }
             const uint64_t scale = sr.scale;
             const int64_t A = (int32_t)pv.b.x, Bm = (int32_t)pv.b.y;
             n = COMPLETE ? complete_set(p, t, A, Bm, q, sr.cls[X + 1], sr.gid, scale, thr, acc, lb,
                                         lm)
-                         : expand_set(p, t, A, Bm, q, sr.gid, scale, thr, acc, lb, lm);
+                         : expand_set(p, t, A, Bm, q, sr.gid, (int)slice, scale, thr, acc,
+                                      lb, lm);
         }
         int incl = n;
 #pragma unroll
@@ -384,9 +506,9 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
                     } else {
                         Vec32 ch = pv;
                         set_byte<2 + (X < 14 ? X : 0)>(ch, (uint32_t)c2);
-                        ch.b.x = (uint32_t)((int32_t)pv.b.x + (Pf(t, q.k, c2) - q.f0));
+                        ch.b.x = (uint32_t)((int32_t)pv.b.x + (Pf(t, q.k, c2) - q.f0) + q.pf);
                         ch.b.y = (uint32_t)(max((int32_t)pv.b.y, Pd(t, q.k, c2) - q.d0) +
-                                            (Pb(t, q.k, c2) - q.b0));
+                                            (Pb(t, q.k, c2) - q.b0) + q.pb);
                         store32(p.out + pos++, ch);
                     }
                 }
@@ -465,11 +587,12 @@ struct Workspace {
     std::mutex mu;
     cudaStream_t stream = nullptr;
     cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
-    DevBuf blob, d_lim, d_slices, d_feas, d_batch, d_inc, d_ctr, d_best, d_feasible, d_leaves, d_roots,
+    DevBuf blob, d_lim, d_vb, d_bctr, d_slices, d_feas, d_batch, d_inc, d_ctr, d_best, d_feasible, d_leaves, d_roots,
         d_root;
     DevBuf d_front[POS_MAX_STAGES + 1];        // per depth: Prefix buffers
     DevBuf d_defer[2 * (POS_MAX_STAGES + 1)];  // per depth: two deferred group lists
     unsigned long long *h_cnt = nullptr;       // pinned host counters
+    std::vector<cudaEvent_t> evs;              // timing events of the batch pipelines
 };
 
 constexpr int kMaxDevices = 64;
@@ -521,8 +644,8 @@ struct Search {
     unsigned long long *ctr = nullptr;  // device counters, see search_impl
     unsigned long long *stats = nullptr;
     uint64_t launches = 0;
-    double ms_expand = 0, ms_complete = 0, ms_leaf = 0;
-    uint64_t n_expand = 0, n_complete = 0, n_leaf = 0;
+    double ms_expand = 0, ms_complete = 0, ms_leaf = 0, ms_bound = 0;
+    uint64_t n_expand = 0, n_complete = 0, n_leaf = 0, n_bound = 0, reruns = 0;
 };
 
 static pos_status validate_problem(const pos_problem *p) {
@@ -548,6 +671,7 @@ static pos_status validate_problem(const pos_problem *p) {
         if (sum != p->S) return fail(POS_EINVAL, "type_counts must sum to S");
     }
     if (p->warmup < 0) return fail(POS_EINVAL, "warmup < 0");
+    if (p->prune < 0 || p->prune > 2) return fail(POS_EINVAL, "prune must be 0, 1 or 2");
     if (p->frontier_cap < 0) return fail(POS_EINVAL, "frontier_cap < 0");
     return POS_OK;
 }
@@ -632,10 +756,11 @@ static ExpandParams base_params(Search &s, const SliceRec *batch, int M) {
     std::memset(&p, 0, sizeof(p));
     p.S = s.S;
     p.M = M;
-    p.prune = s.pb->prune ? 1 : 0;
+    p.prune = s.pb->prune;
     p.slices = batch;
     p.feas = static_cast<const uint4 *>(s.d_feas.p);
     p.lim = static_cast<const uint8_t *>(s.ws.d_lim.p);
+    p.vb = static_cast<const int2 *>(s.ws.d_vb.p);
     p.cap = (unsigned long long)s.cap;
     p.inc = static_cast<const Key128 *>(s.d_inc.p);
     p.stats = s.stats;
@@ -830,6 +955,8 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     POS_CUDA(cudaFuncSetAttribute(feas_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
     POS_CUDA(cudaFuncSetAttribute(sample_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   smem));
+    POS_CUDA(cudaFuncSetAttribute(bound_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  smem));
     POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, level_kernel<false, 0>,
                                                            kThreads, smem));
     s.grid_level = std::max(1, per_sm) * sm_count();
@@ -925,48 +1052,162 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     }
     std::stable_sort(groups.begin(), groups.end(),
                      [](const Group &a, const Group &b) { return a.best < b.best; });
-    POS_CUDA(s.d_batch.reserve(sizeof(SliceRec) * 65535));
-    POS_CUDA(s.d_roots.reserve(sizeof(Prefix) * 65535));
+    // every batch, in processing order, uploaded once
+    struct Batch {
+        int M;
+        size_t off, nb;
+    };
+    std::vector<SliceRec> ordered;
+    std::vector<Batch> batches;
+    size_t max_nb = 1;
     for (const Group &g : groups) {
         const auto &fl = feas_by_m[g.mi];
-        const int M = p->M_list[g.mi];
-        const size_t bsz = std::min<size_t>(
-            65535, std::max<size_t>(32, (fl.size() + 7) / 8));
+        const size_t bsz = std::min<size_t>(65535, std::max<size_t>(32, (fl.size() + 7) / 8));
         for (size_t b0 = 0; b0 < fl.size(); b0 += bsz) {
             const size_t nb = std::min(bsz, fl.size() - b0);
-            std::vector<SliceRec> batch(nb);
-            for (size_t j = 0; j < nb; ++j) batch[j] = s.slices[fl[b0 + j]];
-            POS_CUDA(cudaMemcpyAsync(s.d_batch.p, batch.data(), sizeof(SliceRec) * nb,
+            batches.push_back({p->M_list[g.mi], ordered.size(), nb});
+            for (size_t j = 0; j < nb; ++j) ordered.push_back(s.slices[fl[b0 + j]]);
+            max_nb = std::max(max_nb, nb);
+        }
+    }
+    POS_CUDA(s.d_batch.reserve(sizeof(SliceRec) * std::max<size_t>(1, ordered.size())));
+    if (!ordered.empty())
+        POS_CUDA(cudaMemcpyAsync(s.d_batch.p, ordered.data(), sizeof(SliceRec) * ordered.size(),
+                                 cudaMemcpyHostToDevice, s.stream));
+    // roots: slot j of a batch, no stage placed (the first nb serve a batch of nb)
+    std::vector<Prefix> roots(max_nb);
+    for (size_t j = 0; j < max_nb; ++j) {
+        std::memset(&roots[j], 0, sizeof(Prefix));
+        roots[j].slice = (uint16_t)j;
+        roots[j].A = 0;
+        roots[j].Bm = -1;
+    }
+    POS_CUDA(s.d_roots.reserve(sizeof(Prefix) * max_nb));
+    POS_CUDA(cudaMemcpyAsync(s.d_roots.p, roots.data(), sizeof(Prefix) * max_nb,
+                             cudaMemcpyHostToDevice, s.stream));
+    const SliceRec *d_ordered = static_cast<const SliceRec *>(s.d_batch.p);
+    const Prefix *d_rootp = static_cast<const Prefix *>(s.d_roots.p);
+    if (p->prune == 2) POS_CUDA(s.ws.d_vb.reserve(sizeof(int2) * max_nb * s.S * 128));
+    auto launch_bounds_for = [&](const Batch &b) -> pos_status {
+        if (p->prune != 2) return POS_OK;
+        bound_kernel<<<(int)std::min<size_t>(b.nb, 8 * sm_count()), 128, smem, s.stream>>>(
+            d_ordered + b.off, (int)b.nb, s.S, static_cast<const uint8_t *>(s.ws.d_lim.p),
+            static_cast<int2 *>(s.ws.d_vb.p), s.h->d_blob, s.h->lay);
+        POS_CUDA(cudaGetLastError());
+        s.launches++;
+        s.n_bound++;
+        return POS_OK;
+    };
+
+    if (s.S == 1) {
+        // the single stage takes every layer: each feasible slice is one plan
+        for (const Batch &b : batches) {
+            std::vector<Leaf> lv(b.nb);
+            for (size_t j = 0; j < b.nb; ++j) {
+                std::memset(&lv[j], 0, sizeof(Leaf));
+                lv[j].slice = (uint32_t)j;
+            }
+            POS_CUDA(cudaMemcpyAsync(s.d_leaves.p, lv.data(), sizeof(Leaf) * b.nb,
                                      cudaMemcpyHostToDevice, s.stream));
-            const SliceRec *d_batch = static_cast<const SliceRec *>(s.d_batch.p);
-            if (s.S == 1) {
-                // the single stage takes every layer: each feasible slice is one plan
-                std::vector<Leaf> lv(nb);
-                for (size_t j = 0; j < nb; ++j) {
-                    std::memset(&lv[j], 0, sizeof(Leaf));
-                    lv[j].slice = (uint32_t)j;
+            unsigned long long cnt = b.nb;
+            POS_CUDA(cudaMemcpyAsync(s.ctr + 36, &cnt, 8, cudaMemcpyHostToDevice, s.stream));
+            if ((st = run_leaves(s, static_cast<const Leaf *>(s.d_leaves.p), s.ctr + 36,
+                                 d_ordered + b.off, b.M, nullptr)) != POS_OK)
+                return st;
+            POS_CUDA(cudaStreamSynchronize(s.stream));
+        }
+    } else {
+        // Optimistic pass: every batch runs as one stream-ordered pipeline
+        // (completion bounds, one level kernel per depth, the completion
+        // kernel, the leaf kernel); each kernel reads its input count from
+        // the counter the previous one filled, so the host never waits.
+        // Per batch and depth x: bctr[2x] = entries written (uncapped),
+        // bctr[2x+1] = warp groups that did not fit.
+        const int S = s.S;
+        for (int x = 1; x <= S - 2; ++x)
+            if ((st = ensure_depth(s, x)) != POS_OK) return st;
+        for (int x = 0; x <= S - 2; ++x)
+            if ((st = ensure_defer(s, x, (s.cap + 31) / 32 + 1)) != POS_OK) return st;
+        const size_t n_b = batches.size();
+        POS_CUDA(s.ws.d_bctr.reserve(sizeof(unsigned long long) * 32 * std::max<size_t>(1, n_b)));
+        unsigned long long *bctr = static_cast<unsigned long long *>(s.ws.d_bctr.p);
+        POS_CUDA(cudaMemsetAsync(bctr, 0, sizeof(unsigned long long) * 32 * n_b, s.stream));
+        // timing events, S + 2 per batch: before the bound kernel, before
+        // level 0, after each level kernel, after the leaf kernel
+        const size_t n_ev = n_b * (S + 2);
+        while (s.ws.evs.size() < n_ev) {
+            cudaEvent_t e;
+            POS_CUDA(cudaEventCreate(&e));
+            s.ws.evs.push_back(e);
+        }
+        for (size_t bi = 0; bi < n_b; ++bi) {
+            const Batch &b = batches[bi];
+            cudaEvent_t *ev0 = s.ws.evs.data() + bi * (S + 2);
+            cudaEvent_t *ev = ev0 + 1;
+            POS_CUDA(cudaEventRecord(ev0[0], s.stream));
+            if ((st = launch_bounds_for(b)) != POS_OK) return st;
+            unsigned long long *bc = bctr + 32 * bi;
+            POS_CUDA(cudaEventRecord(ev[0], s.stream));
+            for (int x = 0; x <= S - 2; ++x) {
+                const bool last = x == S - 2;
+                ExpandParams ep = base_params(s, d_ordered + b.off, b.M);
+                ep.in = x == 0 ? d_rootp : static_cast<const Prefix *>(s.d_front[x].p);
+                ep.n_in = x == 0 ? (long long)b.nb : 0;
+                ep.n_in_dev = x == 0 ? nullptr : bc + 2 * (x - 1);
+                ep.x = x;
+                ep.out = last ? nullptr : static_cast<Prefix *>(s.d_front[x + 1].p);
+                ep.leaves = last ? static_cast<Leaf *>(s.d_leaves.p) : nullptr;
+                ep.out_count = bc + 2 * x;
+                ep.deferred = static_cast<uint32_t *>(s.d_defer[2 * x].p);
+                ep.n_deferred = bc + 2 * x + 1;
+                const int grid = x == 0 ? (int)std::max<long long>(
+                                              1, std::min<long long>(((long long)b.nb + 255) / 256,
+                                                                     s.grid_level))
+                                        : s.grid_level;
+                s.launches++;
+                if ((st = launch_level(last, x, ep, grid, smem, s.stream)) != POS_OK) return st;
+                POS_CUDA(cudaEventRecord(ev[x + 1], s.stream));
+            }
+            if ((st = run_leaves(s, static_cast<const Leaf *>(s.d_leaves.p), bc + 2 * (S - 2),
+                                 d_ordered + b.off, b.M, nullptr)) != POS_OK)
+                return st;
+            POS_CUDA(cudaEventRecord(ev[S], s.stream));
+        }
+        std::vector<unsigned long long> hb(32 * n_b);
+        if ((st = sync_read(s, hb.data(), bctr, sizeof(unsigned long long) * hb.size())) != POS_OK)
+            return st;
+        for (size_t bi = 0; bi < n_b; ++bi) {
+            cudaEvent_t *ev0 = s.ws.evs.data() + bi * (S + 2);
+            cudaEvent_t *ev = ev0 + 1;
+            float ms_b = 0;
+            POS_CUDA(cudaEventElapsedTime(&ms_b, ev0[0], ev[0]));
+            s.ms_bound += ms_b;
+            for (int x = 0; x <= S - 1; ++x) {
+                float ms = 0;
+                POS_CUDA(cudaEventElapsedTime(&ms, ev[x], ev[x + 1]));
+                if (x < S - 2) {
+                    s.ms_expand += ms;
+                    s.n_expand++;
+                } else if (x == S - 2) {
+                    s.ms_complete += ms;
+                    s.n_complete++;
+                } else {
+                    s.ms_leaf += ms;
+                    s.n_leaf++;
                 }
-                POS_CUDA(cudaMemcpyAsync(s.d_leaves.p, lv.data(), sizeof(Leaf) * nb,
-                                         cudaMemcpyHostToDevice, s.stream));
-                unsigned long long cnt = nb;
-                POS_CUDA(cudaMemcpyAsync(s.ctr + 36, &cnt, 8, cudaMemcpyHostToDevice, s.stream));
-                if ((st = run_leaves(s, static_cast<const Leaf *>(s.d_leaves.p), s.ctr + 36,
-                                     d_batch, M, nullptr)) != POS_OK)
-                    return st;
-                POS_CUDA(cudaStreamSynchronize(s.stream));
-                continue;
             }
-            std::vector<Prefix> roots(nb);
-            for (size_t j = 0; j < nb; ++j) {
-                std::memset(&roots[j], 0, sizeof(Prefix));
-                roots[j].slice = (uint16_t)j;
-                roots[j].A = 0;
-                roots[j].Bm = -1;  // no stage placed yet
-            }
-            POS_CUDA(cudaMemcpyAsync(s.d_roots.p, roots.data(), sizeof(Prefix) * nb,
-                                     cudaMemcpyHostToDevice, s.stream));
-            st = process(s, d_batch, M, 0, static_cast<const Prefix *>(s.d_roots.p),
-                         (long long)nb);
+        }
+        // A batch in which some frontier overflowed lost the children that
+        // did not fit: run it again with the exact, host-driven deferral.
+        // Plans it evaluated twice do not change the incumbent.
+        for (size_t bi = 0; bi < n_b; ++bi) {
+            bool overflow = false;
+            for (int x = 0; x <= S - 2; ++x) overflow |= hb[32 * bi + 2 * x + 1] != 0;
+            if (!overflow) continue;
+            s.reruns++;
+            const Batch &b = batches[bi];
+            if ((st = launch_bounds_for(b)) != POS_OK) return st;
+            st = process(s, d_ordered + b.off, b.M, 0, d_rootp, (long long)b.nb);
             if (st != POS_OK) return st;
         }
     }
@@ -1003,6 +1244,9 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         stats->parents_expand = hs[kStParentsExpand];
         stats->parents_complete = hs[kStParentsComplete];
         stats->leaves = hs[kStLeaves];
+        stats->ms_bound = s.ms_bound;
+        stats->bound_launches = s.n_bound;
+        stats->reruns = s.reruns;
     }
     if (inc.obj == ~0ull) {
         if (stats) stats->ms_total = ms_since(t_start);

@@ -98,6 +98,11 @@ def test_invalid_arguments_rejected_before_the_device(P):
     prob.S = 2
     prob.warmup = -1
     assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
+    prob.warmup = 0
+    for mode in (-1, 3):
+        prob.prune = mode
+        assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
+        assert b"prune" in L.poseidon_last_error()
     with pytest.raises(P.PoseidonError):
         P.Handle(bad)
 

@@ -36,7 +36,7 @@ def same_plan(a, b):
 
 
 @pytest.mark.parametrize("cfg", [1, 2, 3])
-@pytest.mark.parametrize("prune", [True, False])
+@pytest.mark.parametrize("prune", [0, 1, 2])
 def test_configs_match_oracle(P, orc, cfg, prune):
     w = gen.get_config(cfg)
     ref, _ = orc.search(w, prune=True, warmup=0)
@@ -45,21 +45,34 @@ def test_configs_match_oracle(P, orc, cfg, prune):
     assert st["evaluated"] >= 1
 
 
-def test_config4_matches_stored_oracle_plan(P):
-    """The bench's workload and launch configuration (prune on, warm-up
-    65536 samples); expected plan written by tests/golden/make_search_plans.py."""
+@pytest.mark.parametrize("prune", [1, 2])
+def test_config4_matches_stored_oracle_plan(P, prune):
+    """The bench's workload and launch configuration (warm-up 65536 samples;
+    the bench times both prune modes); expected plan written by
+    tests/golden/make_search_plans.py."""
     ref = json.load(open(GOLDEN))["config4"]["plan"]
-    plan, st = gpu_search(P, gen.config4(), prune=True, warmup=65536, seed=0)
+    plan, st = gpu_search(P, gen.config4(), prune=prune, warmup=65536, seed=0)
     assert same_plan(plan, ref), (plan, ref)
     assert st["slices_feasible"] == 420
+
+
+def test_tight_bound_cuts_more(P):
+    """The tightened bound removes prefixes that Eq. 2 keeps: on config 3
+    it generates fewer prefixes and evaluates no more plans."""
+    w = gen.config3()
+    _, s1 = gpu_search(P, w, prune=1, warmup=500, seed=0)
+    _, s2 = gpu_search(P, w, prune=2, warmup=500, seed=0)
+    assert s2["prefixes"] < s1["prefixes"]
+    assert s2["evaluated"] <= s1["evaluated"]
 
 
 @pytest.mark.parametrize("warmup", [0, 1, 500, 100_000])
 def test_warmup_never_changes_the_plan(P, orc, warmup):
     w = gen.config2()
     ref, _ = orc.search(w, prune=False)
-    plan, _ = gpu_search(P, w, prune=True, warmup=warmup, seed=warmup)
-    assert same_plan(plan, ref)
+    for prune in (1, 2):
+        plan, _ = gpu_search(P, w, prune=prune, warmup=warmup, seed=warmup)
+        assert same_plan(plan, ref), prune
 
 
 @pytest.mark.parametrize("cap", [1, 3000, 20_000])
@@ -69,8 +82,9 @@ def test_tiny_frontiers_defer_and_still_match(P, orc, cap):
     for cfg in (2, 3):
         w = gen.get_config(cfg)
         ref, _ = orc.search(w, prune=True, warmup=0)
-        plan, _ = gpu_search(P, w, prune=True, warmup=50, frontier_cap=cap)
-        assert same_plan(plan, ref), (cfg, cap)
+        for prune in (1, 2):
+            plan, _ = gpu_search(P, w, prune=prune, warmup=50, frontier_cap=cap)
+            assert same_plan(plan, ref), (cfg, cap, prune)
 
 
 def test_random_small_problems(P, orc):
@@ -80,7 +94,7 @@ def test_random_small_problems(P, orc):
         w = _random_problem(rng, seed)
         ref, _ = orc.search(w, prune=False)
         try:
-            plan, _ = gpu_search(P, w, prune=bool(seed % 2), warmup=seed % 7, seed=seed)
+            plan, _ = gpu_search(P, w, prune=seed % 3, warmup=seed % 7, seed=seed)
         except P.PoseidonError as e:
             assert e.status == P.binding.POS_EINFEASIBLE and not ref["found"], (seed, e)
             continue
@@ -97,8 +111,9 @@ def test_single_stage_and_two_stage(P, orc):
         w.placement = gen.workloads.PLACE_FREE if counts is None else gen.workloads.PLACE_EXACT
         w.type_counts = counts or []
         ref, _ = orc.search(w, prune=False)
-        plan, _ = gpu_search(P, w, prune=True, warmup=3)
-        assert same_plan(plan, ref), S
+        for prune in (1, 2):
+            plan, _ = gpu_search(P, w, prune=prune, warmup=3)
+            assert same_plan(plan, ref), (S, prune)
 
 
 def test_infeasible_and_overflow(P):
@@ -142,9 +157,10 @@ def _limits_problem(seed, S, L, n_types, placement, counts, M_list):
 def test_search_at_the_limits(P, orc, S, L, types, placement, counts, M_list):
     w = _limits_problem(S * 31 + L, S, L, types, placement, counts, M_list)
     ref, _ = orc.search(w, prune=True, warmup=0)
-    try:
-        plan, _ = gpu_search(P, w, prune=True, warmup=200, seed=1)
-    except P.PoseidonError as e:
-        assert e.status == P.binding.POS_EINFEASIBLE and not ref["found"]
-        return
-    assert same_plan(plan, ref), (plan, ref)
+    for prune in (1, 2):
+        try:
+            plan, _ = gpu_search(P, w, prune=prune, warmup=200, seed=1)
+        except P.PoseidonError as e:
+            assert e.status == P.binding.POS_EINFEASIBLE and not ref["found"]
+            continue
+        assert same_plan(plan, ref), (prune, plan, ref)

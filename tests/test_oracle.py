@@ -194,6 +194,82 @@ def test_lower_bound_value(orc):
     assert orc.lower_bound(tab, 3, 2, cls, lay, 1) == 0 + 2 * 7 + 10
 
 
+def test_tight_bound_hand_value(orc):
+    """Tightened bound on the same three stages, pf = (1, 2), pb = (3, 1),
+    M = 2 (one layer per stage, so the completion is unique).  Path lengths
+    P(y, i) = sum_{j<y}(F_j+pf_j) + M(F_y+B_y) + sum_{j=i}^{y-1}(B_j+pb_j) + d_i:
+    P(1,1) = 24, P(2,1) = 3+18+8+10 = 39, P(2,2) = 21, P(3,1) = 8+22+15+10 = 55,
+    P(3,2) = 37, P(3,3) = 34.  Every prefix of this plan is bounded by 55,
+    where Eq. 2 gives 24 at x = 1 and 48 at x = 3."""
+    tab, cls, lay = stage_tables(orc, [2, 3, 4], [5, 6, 7], [10, 0, 4], [1, 2], [3, 1])
+    for x in (1, 2, 3):
+        assert orc.lower_bound_tight(tab, 3, 2, cls, lay, x) == 55
+    # a large d_3 makes the completion term P(3,3) the largest
+    tab, cls, lay = stage_tables(orc, [2, 3, 4], [5, 6, 7], [10, 0, 40], [1, 2], [3, 1])
+    assert orc.lower_bound_tight(tab, 3, 2, cls, lay, 1) == 8 + 22 + 40
+    assert orc.lower_bound_tight(tab, 3, 2, cls, lay, 3) == 8 + 22 + 40
+
+
+def test_tight_bound_is_the_makespan_of_a_chain(orc):
+    """M = 1: the DAG is a chain, and max_i P(S, i) is exactly its longest
+    path (the closed form of test_single_microbatch_chain)."""
+    rng = random.Random(31)
+    for _ in range(200):
+        S = rng.randint(1, 9)
+        F, B, d, pf, pb = rand_stages(rng, S)
+        tab, cls, lay = stage_tables(orc, F, B, d, pf, pb)
+        T, _ = orc.evaluate(tab, S, 1, cls, lay)
+        assert orc.lower_bound_tight(tab, S, 1, cls, lay, S) == T
+
+
+def test_tight_bound_valid_and_tighter(orc):
+    """Brute force over every plan of small random problems: for each prefix,
+    the tightened bound never exceeds the best makespan among the prefix's
+    memory-feasible completions (so pruning with it is exact), is at least
+    Eq. 2, and is strictly larger than Eq. 2 for a good share of prefixes."""
+    rng = random.Random(32)
+    n_pref = n_strict = 0
+    for seed in range(60):
+        w = _random_problem(rng, seed)
+        tab = orc.OracleTables.from_workload(w)
+        S, L = w.S, w.L
+        for tp in range(w.n_tp):
+            for seq in gen.workloads.place_list(w)[:6]:
+                cls = [t * w.n_tp + tp for t in seq]
+                for M in w.M_list:
+                    best = {}  # prefix -> min T over feasible completions
+                    for r in range(orc.binom(L - 1, S - 1)):
+                        lay = orc.unrank(L, S, r)
+                        T, feas = orc.evaluate(tab, S, M, cls, lay)
+                        if not feas:
+                            continue
+                        for x in range(1, S + 1):
+                            key = tuple(lay[:x])
+                            if key not in best or T < best[key][0]:
+                                best[key] = (T, lay)
+                    for key, (tmin, lay) in best.items():
+                        x = len(key)
+                        lb = orc.lower_bound_tight(tab, S, M, cls, lay, x)
+                        g = orc.lower_bound(tab, S, M, cls, lay, x)
+                        assert lb is not None and g <= lb <= tmin, (seed, key, g, lb, tmin)
+                        n_pref += 1
+                        n_strict += lb > g
+    assert n_pref > 2000 and n_strict > n_pref // 4, (n_pref, n_strict)
+
+
+def test_tight_bound_without_feasible_completion(orc):
+    """A prefix that leaves no memory-feasible completion has no bound."""
+    tab, cls, lay = stage_tables(orc, [2, 3], [5, 6], [0, 0], [1], [1])
+    # stage 2 holds the only layer of class 1; give it a weight that cannot fit
+    tab2 = orc.OracleTables(L=2, n_types=2, n_tp=1, fwd=np.array([[2, 2], [3, 3]]),
+                            bwd=np.array([[5, 5], [6, 6]]), dsync=np.zeros((2, 2)),
+                            p2p_f=np.zeros((2, 2)), p2p_b=np.zeros((2, 2)),
+                            mem_w=np.array([[0, 0], [9, 9]]), mem_a=np.zeros((2, 2)),
+                            cap=np.array([1, 1]))
+    assert orc.lower_bound_tight(tab2, 2, 1, [0, 1], [1, 1], 1) is None
+    assert orc.lower_bound_tight(tab, 2, 1, [0, 1], [1, 1], 1) is not None
+
+
 def test_monotone_in_weights(orc):
     rng = random.Random(16)
     for _ in range(300):
