@@ -45,6 +45,10 @@ struct BlobLayout {
 };
 
 BlobLayout make_layout(int L, int n_types, int n_tp);
+// The timing part of a blob (Pf, Pb, Pd, p2f, p2b: its last five tables),
+// rebased to start at byte 0, for kernels that read nothing else; the
+// timing part starts at byte ly.off_Pf of the full blob.
+BlobLayout timing_layout(const BlobLayout &ly);
 
 struct Handle {
     int device;
@@ -121,11 +125,76 @@ __device__ __forceinline__ uint64_t binom(const Tab &t, int n, int k) {
     return (uint64_t)ld64(t.base, t.ly->off_binom + 8u * (uint32_t)(k * kBinomN + n));
 }
 
-// Cooperative 16-byte copy of the blob into shared memory.
+// Cooperative 16-byte copy of the blob into shared memory, four loads in
+// flight per thread (a load-store pair per iteration would wait a full
+// memory latency each time).
 __device__ __forceinline__ void stage_blob(unsigned char *dst, const void *src, int bytes) {
     const uint4 *s = reinterpret_cast<const uint4 *>(src);
     uint4 *d = reinterpret_cast<uint4 *>(dst);
-    for (int i = threadIdx.x; i < bytes / 16; i += blockDim.x) d[i] = __ldg(s + i);
+    const int n = bytes / 16, bd = blockDim.x;
+    int i = threadIdx.x;
+    for (; i + 3 * bd < n; i += 4 * bd) {
+        const uint4 a = __ldg(s + i), b = __ldg(s + i + bd), c = __ldg(s + i + 2 * bd),
+                    e = __ldg(s + i + 3 * bd);
+        d[i] = a;
+        d[i + bd] = b;
+        d[i + 2 * bd] = c;
+        d[i + 3 * bd] = e;
+    }
+    for (; i < n; i += bd) d[i] = __ldg(s + i);
+}
+
+// Bulk copies global -> this CTA's shared memory on the TMA engine
+// (cp.async.bulk), completion counted in bytes on one mbarrier.  Thread 0
+// calls bulk_begin with the total byte count, then issues the copies
+// (16-byte aligned addresses, sizes multiples of 16); then every thread of
+// the block calls bulk_wait, which returns the same value in all threads:
+// false if the copies did not complete within kBulkWaitLimit polls.
+constexpr int kBulkWaitLimit = 1 << 24;
+
+__device__ __forceinline__ void bulk_begin(uint64_t *bar, uint32_t total_bytes) {
+    const uint32_t b = (uint32_t)__cvta_generic_to_shared(bar);
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(b) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(b),
+                 "r"(total_bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void bulk_copy(void *dst_smem, const void *src, uint32_t bytes,
+                                          uint64_t *bar) {
+    const uint32_t b = (uint32_t)__cvta_generic_to_shared(bar);
+    const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst_smem);
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+            "r"(d),
+        "l"(src), "r"(bytes), "r"(b)
+        : "memory");
+}
+
+__device__ __forceinline__ bool bulk_wait(uint64_t *bar) {
+    __syncthreads();  // the barrier is initialised before anyone polls it
+    const uint32_t b = (uint32_t)__cvta_generic_to_shared(bar);
+    uint32_t done = 0;
+    for (int it = 0; it < kBulkWaitLimit && !done; ++it) {
+        asm volatile(
+            "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\n"
+            " selp.u32 %0, 1, 0, p;\n}"
+            : "=r"(done)
+            : "r"(b)
+            : "memory");
+    }
+    return __syncthreads_and(done) != 0;
+}
+
+// The whole blob (or a rebased part of it) by one bulk copy.
+__device__ __forceinline__ bool stage_blob_bulk(unsigned char *dst, const void *src, int bytes,
+                                                uint64_t *bar) {
+    if (threadIdx.x == 0) {
+        bulk_begin(bar, (uint32_t)bytes);
+        bulk_copy(dst, src, (uint32_t)bytes, bar);
+    }
+    return bulk_wait(bar);
 }
 
 // ---------------------------------------------------------------------------

@@ -27,6 +27,7 @@ namespace pos {
 
 constexpr int kThreads = 256;
 constexpr int32_t kNoCompletion = 0x7fffffff;  // completion-bound entry without a completion
+constexpr int kVbSlotsSmem = 64;  // batches up to this many slots stage their bound rows
 
 // ---------------------------------------------------------------------------
 // suffix feasibility: one block per slice, thread c
@@ -34,11 +35,15 @@ constexpr int32_t kNoCompletion = 0x7fffffff;  // completion-bound entry without
 // Also fills lim[(gid*S + x)*128 + c] = the largest l such that stage x
 // holds layers [c, c+l) within memory (0 if none), capped at L - c.
 __global__ void feas_kernel(const SliceRec *slices, int n_slices, int S, uint4 *feas,
-                            uint8_t *lim, const void *blob, BlobLayout lay) {
+                            uint8_t *lim, const void *blob, BlobLayout lay,
+                            unsigned long long *stats) {
     extern __shared__ __align__(16) unsigned char sm[];
     __shared__ uint32_t prev[4], cur[4];
-    stage_blob(sm, blob, lay.bytes);
-    __syncthreads();
+    __shared__ uint64_t bar;
+    if (!stage_blob_bulk(sm, blob, lay.bytes, &bar)) {
+        if (threadIdx.x == 0) atomicAdd(stats + kStTimeout, 1ull);
+        return;
+    }
     const Tab t = tab_at(sm, lay);
     const int L = lay.L, c = threadIdx.x;
     for (int sl = blockIdx.x; sl < n_slices; sl += gridDim.x) {
@@ -105,13 +110,17 @@ __global__ void root_bits_kernel(const uint4 *feas, int n_slices, int S, uint8_t
 // A prefix whose A + V1 or A + Bm + V2 exceeds the incumbent has no
 // completion that beats it.  Each finite entry is at most the makespan of
 // a feasible plan, so it fits in int32 under the overflow guard.
-// One block per slot of the batch, thread c; vb[(slot*S + x)*128 + c].
+// One block per slot of the batch, thread c; vb[(x*nb + slot)*128 + c], so
+// that the rows of one depth for every slot are contiguous.
 __global__ void bound_kernel(const SliceRec *batch, int nb, int S, const uint8_t *lim, int2 *vb,
-                             const void *blob, BlobLayout lay) {
+                             const void *blob, BlobLayout lay, unsigned long long *stats) {
     extern __shared__ __align__(16) unsigned char sm[];
     __shared__ int2 nxt[128];
-    stage_blob(sm, blob, lay.bytes);
-    __syncthreads();
+    __shared__ uint64_t bar;
+    if (!stage_blob_bulk(sm, blob, lay.bytes, &bar)) {
+        if (threadIdx.x == 0) atomicAdd(stats + kStTimeout, 1ull);
+        return;
+    }
     const Tab t = tab_at(sm, lay);
     const int L = lay.L, c = threadIdx.x;
     for (int slot = blockIdx.x; slot < nb; slot += gridDim.x) {
@@ -147,7 +156,7 @@ __global__ void bound_kernel(const SliceRec *batch, int nb, int S, const uint8_t
             const int2 out = v1 == INT64_MAX ? make_int2(kNoCompletion, kNoCompletion)
                                              : make_int2((int32_t)v1, (int32_t)v2);
             nxt[c] = out;
-            vb[((size_t)slot * S + x) * 128 + c] = out;
+            vb[((size_t)x * nb + slot) * 128 + c] = out;
             __syncthreads();
         }
     }
@@ -163,77 +172,6 @@ __device__ __forceinline__ uint64_t splitmix64_next(uint64_t &s) {
     z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
     return z ^ (z >> 31);
 }
-
-__global__ void sample_kernel(const SliceRec *slices, const uint32_t *feasible, int n_feasible,
-                              int n_samples, int S, uint64_t seed, const uint4 *feas,
-                              Leaf *out, const void *blob, BlobLayout lay) {
-    extern __shared__ __align__(16) unsigned char sm[];
-    stage_blob(sm, blob, lay.bytes);
-    __syncthreads();
-    const Tab t = tab_at(sm, lay);
-    const int L = lay.L;
-    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n_samples;
-         i += gridDim.x * blockDim.x) {
-        uint64_t st = seed ^ ((uint64_t)i * 0xD1B54A32D192ED03ull);
-        const uint32_t sl = feasible[splitmix64_next(st) % (uint64_t)n_feasible];
-        const SliceRec &sr = slices[sl];
-        Leaf lf;
-        lf.slice = sl;
-        for (int s = 0; s < 16; ++s) lf.cut[s] = 0;
-        lf.pad[0] = lf.pad[1] = lf.pad[2] = 0;
-        int c = 0;
-        for (int x = 0; x < S - 1; ++x) {
-            const int k = sr.cls[x];
-            int n_ok = 0;
-            for (int l = 1; c + l <= L - (S - x - 1); ++l) {
-                if (!stage_fits(t, S, sr.M, x, k, c, c + l)) break;
-                n_ok += feas_bit(feas, S, sr.gid, x + 1, c + l);
-            }
-            int r = (int)(splitmix64_next(st) % (uint64_t)max(n_ok, 1));
-            int pick = 1;
-            for (int l = 1; c + l <= L - (S - x - 1); ++l) {
-                if (feas_bit(feas, S, sr.gid, x + 1, c + l)) {
-                    if (r == 0) {
-                        pick = l;
-                        break;
-                    }
-                    --r;
-                }
-            }
-            c += pick;
-            lf.cut[x] = (uint8_t)c;
-        }
-        out[i] = lf;
-    }
-}
-
-// ---------------------------------------------------------------------------
-// level expansion and completion (Sec. 4.2.1 prune, Sec. 3.2 memory cut)
-// ---------------------------------------------------------------------------
-struct ExpandParams {
-    const Prefix *in;
-    long long n_in;
-    const unsigned long long *n_in_dev;  // if set: n_in = min(*n_in_dev, cap), read on the device
-    const uint32_t *groups;  // work list of 32-parent groups, or NULL = all groups
-    long long n_groups;
-    int x;                   // depth of the parents (stages 0..x-1 placed)
-    int S, M;
-    int prune;
-    const SliceRec *slices;
-    const uint4 *feas;
-    const uint8_t *lim;      // per (slice, stage, start) memory limit, see feas_kernel
-    const int2 *vb;          // prune 2: completion bounds per (batch slot, stage, start)
-    Prefix *out;             // expand: children at depth x+1
-    Leaf *leaves;            // complete: full plans
-    unsigned long long *out_count;
-    unsigned long long cap;
-    uint32_t *deferred;
-    unsigned long long *n_deferred;
-    const Key128 *inc;
-    unsigned long long *stats;
-    const void *blob;
-    BlobLayout lay;
-};
 
 // 128-bit set of cut positions 0..127.
 struct Bits128 {
@@ -253,6 +191,87 @@ __device__ __forceinline__ Bits128 range_bits(int lo, int hi) {  // positions lo
 __device__ __forceinline__ int popc128(const Bits128 &b) {
     return __popc(b.w[0]) + __popc(b.w[1]) + __popc(b.w[2]) + __popc(b.w[3]);
 }
+
+// Position of the r-th (0-based) set bit of a 128-bit set with more than r
+// set bits.
+__device__ __forceinline__ int nth_set(const Bits128 &b, int r) {
+    int base = 0;
+#pragma unroll
+    for (int i = 0; i < 3; ++i) {
+        const int p = __popc(b.w[i]);
+        if (base == 32 * i && r >= p) {
+            r -= p;
+            base = 32 * (i + 1);
+        }
+    }
+    const uint32_t word = base == 0 ? b.w[0] : base == 32 ? b.w[1] : base == 64 ? b.w[2] : b.w[3];
+    return base + (int)__fns(word, 0, r + 1);
+}
+
+// One thread per sample: stage by stage, the layer count is drawn uniformly
+// among the counts l that fit the stage's memory (l <= lim) and leave a
+// memory-feasible suffix (feasibility bit of c + l), i.e. the set bits of
+// one 128-bit window, picked with a popcount and a select.
+__global__ void sample_kernel(const SliceRec *slices, const uint32_t *feasible, int n_feasible,
+                              int n_samples, int S, uint64_t seed, const uint4 *feas,
+                              const uint8_t *lim, Leaf *out, int L) {
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n_samples;
+         i += gridDim.x * blockDim.x) {
+        uint64_t st = seed ^ ((uint64_t)i * 0xD1B54A32D192ED03ull);
+        const uint32_t sl = feasible[splitmix64_next(st) % (uint64_t)n_feasible];
+        const SliceRec &sr = slices[sl];
+        const uint32_t gid = sr.gid;
+        uint32_t cw[4] = {0u, 0u, 0u, 0u};  // cut[0..15], byte x = cut[x]
+        int c = 0;
+        for (int x = 0; x < S - 1; ++x) {
+            const int hi = min((int)__ldg(lim + ((size_t)gid * S + x) * 128 + c),
+                               L - c - (S - x - 1));
+            const uint4 f = __ldg(feas + (size_t)gid * (S + 1) + x + 1);
+            const Bits128 win = range_bits(c + 1, c + hi);
+            const Bits128 ok = {{f.x & win.w[0], f.y & win.w[1], f.z & win.w[2], f.w & win.w[3]}};
+            const int n_ok = popc128(ok);
+            const int r = (int)(splitmix64_next(st) % (uint64_t)max(n_ok, 1));
+            c = n_ok > 0 ? nth_set(ok, r) : c + 1;
+            const uint32_t v = (uint32_t)c << (8 * (x % 4));
+#pragma unroll
+            for (int wi = 0; wi < 4; ++wi) cw[wi] |= (x / 4 == wi) ? v : 0u;
+        }
+        // leaf: slice in bytes 0-3, cut[x] in byte 4 + x
+        const Vec32 lf = {make_uint4(sl, cw[0], cw[1], cw[2]), make_uint4(cw[3], 0u, 0u, 0u)};
+        store32(out + i, lf);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// level expansion and completion (Sec. 4.2.1 prune, Sec. 3.2 memory cut)
+// ---------------------------------------------------------------------------
+struct ExpandParams {
+    const Prefix *in;
+    long long n_in;
+    const unsigned long long *n_in_dev;  // if set: n_in = min(*n_in_dev, cap), read on the device
+    const uint32_t *groups;  // work list of 32-parent groups, or NULL = all groups
+    long long n_groups;
+    int x;                   // depth of the parents (stages 0..x-1 placed)
+    int S, M;
+    int prune;
+    const SliceRec *slices;
+    const uint4 *feas;
+    const uint8_t *lim;      // per (slice, stage, start) memory limit, see feas_kernel
+    const int2 *vb;          // prune 2: completion bounds per (batch slot, stage, start)
+    int vb_smem;             // 1: stage this depth's rows of all nb slots in shared memory
+    int nb;                  // slots in the batch
+    Prefix *out;             // expand: children at depth x+1
+    Leaf *leaves;            // complete: full plans
+    unsigned long long *out_count;
+    unsigned long long cap;
+    uint32_t *deferred;
+    unsigned long long *n_deferred;
+    const Key128 *inc;
+    unsigned long long *stats;
+    const void *blob;
+    BlobLayout lay;
+};
+
 
 // Largest l in [0, hi] with pred(l), for pred true up to some l and false
 // after (pred(0) is taken as true).
@@ -295,7 +314,7 @@ __device__ __forceinline__ ParentCtx parent_ctx(const Tab &t, int k, int c) {
 // (feasibility bits).
 __device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, int64_t A,
                                           int64_t Bm, const ParentCtx &q, uint32_t gid,
-                                          int slot, uint64_t scale,
+                                          const int2 *vrow, uint64_t scale,
                                           uint64_t thr, Bits128 &acc, unsigned long long &cut_b,
                                           unsigned long long &cut_m) {
     const int S = p.S, M = p.M, x = p.x, L = t.L();
@@ -324,7 +343,6 @@ __device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, i
     if (p.prune == 2 && n > 0) {
         // completion terms: the bound is not monotone in l, so every
         // candidate child is tested on its own
-        const int2 *vrow = p.vb + ((size_t)slot * S + x + 1) * 128;
 #pragma unroll
         for (int wd = 0; wd < 4; ++wd) {
             uint32_t m = acc.w[wd];
@@ -339,7 +357,7 @@ __device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, i
                 }
 #pragma unroll
                 for (int u = 0; u < 4; ++u)
-                    if (bb[u] >= 0) v[u] = __ldg(vrow + 32 * wd + bb[u]);
+                    if (bb[u] >= 0) v[u] = vrow[32 * wd + bb[u]];
 #pragma unroll
                 for (int u = 0; u < 4; ++u) {
                     if (bb[u] < 0) continue;
@@ -426,19 +444,37 @@ __device__ __forceinline__ int complete_set(const ExpandParams &p, const Tab &t,
 template <bool COMPLETE, int X>
 __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(ExpandParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
-    stage_blob(sm, p.blob, p.lay.bytes);
-    __syncthreads();
-    const Tab t = tab_at(sm, p.lay);
-    const uint64_t thr = p.prune ? __ldcg(&p.inc->obj) : ~0ull;
-    const int lane = threadIdx.x & 31;
-    const long long warp = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
-    const long long n_warps = ((long long)gridDim.x * blockDim.x) >> 5;
     long long n_in = p.n_in;
     if (p.n_in_dev) {
         const unsigned long long c0 = __ldcg(p.n_in_dev);
         n_in = (long long)(c0 < p.cap ? c0 : p.cap);
     }
     const long long n_work = p.groups ? p.n_groups : (n_in + 31) / 32;
+    // blocks without a group leave before staging anything
+    if ((long long)blockIdx.x * (kThreads / 32) >= n_work) return;
+    // timing tables and, when expanding under prune mode 2, the
+    // completion-bound rows of depth X+1 of every slot (contiguous), by TMA
+    __shared__ uint64_t bar;
+    const bool use_v = !COMPLETE && p.prune == 2;
+    const bool stage_v = use_v && p.vb_smem;
+    const int2 *vrows = use_v ? p.vb + (size_t)(X + 1) * p.nb * 128 : nullptr;
+    if (threadIdx.x == 0) {
+        const uint32_t vbytes = stage_v ? (uint32_t)p.nb * 128u * 8u : 0u;
+        bulk_begin(&bar, (uint32_t)p.lay.bytes + vbytes);
+        bulk_copy(sm, p.blob, (uint32_t)p.lay.bytes, &bar);
+        if (stage_v) bulk_copy(sm + p.lay.bytes, vrows, vbytes, &bar);
+    }
+    if (!bulk_wait(&bar)) {
+        if (threadIdx.x == 0) atomicAdd(p.stats + kStTimeout, 1ull);
+        return;
+    }
+    const int2 *vbase = stage_v ? reinterpret_cast<const int2 *>(sm + p.lay.bytes) : vrows;
+    const size_t vstride = 128;
+    const Tab t = tab_at(sm, p.lay);
+    const uint64_t thr = p.prune ? __ldcg(&p.inc->obj) : ~0ull;
+    const int lane = threadIdx.x & 31;
+    const long long warp = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
+    const long long n_warps = ((long long)gridDim.x * blockDim.x) >> 5;
     unsigned long long emitted = 0, cb = 0, cm = 0, parents = 0, written_parents = 0;
     for (long long w = warp; w < n_work; w += n_warps) {
         const long long g = p.groups ? (long long)p.groups[w] : w;
@@ -465,7 +501,8 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
             const int64_t A = (int32_t)pv.b.x, Bm = (int32_t)pv.b.y;
             n = COMPLETE ? complete_set(p, t, A, Bm, q, sr.cls[X + 1], sr.gid, scale, thr, acc, lb,
                                         lm)
-                         : expand_set(p, t, A, Bm, q, sr.gid, (int)slice, scale, thr, acc,
+                         : expand_set(p, t, A, Bm, q, sr.gid, vbase + slice * vstride, scale,
+                                      thr, acc,
                                       lb, lm);
         }
         int incl = n;
@@ -646,6 +683,7 @@ struct Search {
     uint64_t launches = 0;
     double ms_expand = 0, ms_complete = 0, ms_leaf = 0, ms_bound = 0;
     uint64_t n_expand = 0, n_complete = 0, n_leaf = 0, n_bound = 0, reruns = 0;
+    int cur_nb = 0;  // slots of the batch being enumerated (row stride of the bound tables)
 };
 
 static pos_status validate_problem(const pos_problem *p) {
@@ -761,11 +799,13 @@ static ExpandParams base_params(Search &s, const SliceRec *batch, int M) {
     p.feas = static_cast<const uint4 *>(s.d_feas.p);
     p.lim = static_cast<const uint8_t *>(s.ws.d_lim.p);
     p.vb = static_cast<const int2 *>(s.ws.d_vb.p);
+    p.nb = s.cur_nb;
     p.cap = (unsigned long long)s.cap;
     p.inc = static_cast<const Key128 *>(s.d_inc.p);
     p.stats = s.stats;
-    p.blob = s.h->d_blob;
-    p.lay = s.h->lay;
+    // level kernels read only the timing tables: stage that part alone
+    p.blob = static_cast<const unsigned char *>(s.h->d_blob) + s.h->lay.off_Pf;
+    p.lay = timing_layout(s.h->lay);
     return p;
 }
 
@@ -842,7 +882,7 @@ static pos_status process(Search &s, const SliceRec *batch, int M, int x, const 
         p.out_count = out_count;
         p.deferred = static_cast<uint32_t *>(s.d_defer[2 * x + flip].p);
         p.n_deferred = n_def;
-        const int smem = s.h->lay.bytes;
+        const int smem = p.lay.bytes;
         const long long blocks_needed = (n_work * 32 + kThreads - 1) / kThreads;
         const int grid = (int)std::max<long long>(1, std::min<long long>(blocks_needed,
                                                                          s.grid_level));
@@ -953,12 +993,10 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     POS_CUDA(cudaFuncSetAttribute(level_kernel<false, 0>,
                                   cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
     POS_CUDA(cudaFuncSetAttribute(feas_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-    POS_CUDA(cudaFuncSetAttribute(sample_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  smem));
     POS_CUDA(cudaFuncSetAttribute(bound_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                   smem));
-    POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, level_kernel<false, 0>,
-                                                           kThreads, smem));
+    POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+        &per_sm, level_kernel<false, 0>, kThreads, timing_layout(s.h->lay).bytes));
     s.grid_level = std::max(1, per_sm) * sm_count();
     s.grid_leaf = 2 * sm_count();
 
@@ -979,7 +1017,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     const SliceRec *d_all = static_cast<const SliceRec *>(s.d_slices.p);
     feas_kernel<<<std::min(n_slices, 16 * sm_count()), 128, smem, s.stream>>>(
         d_all, n_slices, s.S, static_cast<uint4 *>(s.d_feas.p),
-        static_cast<uint8_t *>(s.ws.d_lim.p), s.h->d_blob, s.h->lay);
+        static_cast<uint8_t *>(s.ws.d_lim.p), s.h->d_blob, s.h->lay, s.stats);
     POS_CUDA(cudaGetLastError());
     s.launches++;
     DevBuf &d_root = s.d_root;
@@ -1013,12 +1051,12 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
                                                   (long long)n_feasible));
             POS_CUDA(cudaMemcpyAsync(s.d_feasible.p, fl.data(), sizeof(uint32_t) * fl.size(),
                                      cudaMemcpyHostToDevice, s.stream));
-            sample_kernel<<<(int)std::min<long long>((n_s + 255) / 256, 4 * sm_count()), 256,
-                            smem, s.stream>>>(
+            sample_kernel<<<(int)std::min<long long>((n_s + 255) / 256, 4 * sm_count()), 256, 0,
+                            s.stream>>>(
                 d_all, static_cast<const uint32_t *>(s.d_feasible.p), (int)fl.size(), (int)n_s,
                 s.S, p->seed + 0x632BE59BD9B4E019ull * (uint64_t)mi,
-                static_cast<const uint4 *>(s.d_feas.p), static_cast<Leaf *>(s.d_leaves.p),
-                s.h->d_blob, s.h->lay);
+                static_cast<const uint4 *>(s.d_feas.p), static_cast<const uint8_t *>(s.ws.d_lim.p),
+                static_cast<Leaf *>(s.d_leaves.p), s.L);
             POS_CUDA(cudaGetLastError());
             s.launches++;
             unsigned long long cnt = (unsigned long long)n_s;
@@ -1062,7 +1100,8 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     size_t max_nb = 1;
     for (const Group &g : groups) {
         const auto &fl = feas_by_m[g.mi];
-        const size_t bsz = std::min<size_t>(65535, std::max<size_t>(32, (fl.size() + 7) / 8));
+        size_t bsz = std::min<size_t>(65535, std::max<size_t>(32, (fl.size() + 7) / 8));
+        if (p->prune == 2) bsz = std::min<size_t>(bsz, kVbSlotsSmem);
         for (size_t b0 = 0; b0 < fl.size(); b0 += bsz) {
             const size_t nb = std::min(bsz, fl.size() - b0);
             batches.push_back({p->M_list[g.mi], ordered.size(), nb});
@@ -1090,9 +1129,11 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     if (p->prune == 2) POS_CUDA(s.ws.d_vb.reserve(sizeof(int2) * max_nb * s.S * 128));
     auto launch_bounds_for = [&](const Batch &b) -> pos_status {
         if (p->prune != 2) return POS_OK;
-        bound_kernel<<<(int)std::min<size_t>(b.nb, 8 * sm_count()), 128, smem, s.stream>>>(
+        const BlobLayout tl = timing_layout(s.h->lay);
+        bound_kernel<<<(int)std::min<size_t>(b.nb, 8 * sm_count()), 128, tl.bytes, s.stream>>>(
             d_ordered + b.off, (int)b.nb, s.S, static_cast<const uint8_t *>(s.ws.d_lim.p),
-            static_cast<int2 *>(s.ws.d_vb.p), s.h->d_blob, s.h->lay);
+            static_cast<int2 *>(s.ws.d_vb.p),
+            static_cast<const unsigned char *>(s.h->d_blob) + s.h->lay.off_Pf, tl, s.stats);
         POS_CUDA(cudaGetLastError());
         s.launches++;
         s.n_bound++;
@@ -1142,6 +1183,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         }
         for (size_t bi = 0; bi < n_b; ++bi) {
             const Batch &b = batches[bi];
+            s.cur_nb = (int)b.nb;
             cudaEvent_t *ev0 = s.ws.evs.data() + bi * (S + 2);
             cudaEvent_t *ev = ev0 + 1;
             POS_CUDA(cudaEventRecord(ev0[0], s.stream));
@@ -1160,12 +1202,16 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
                 ep.out_count = bc + 2 * x;
                 ep.deferred = static_cast<uint32_t *>(s.d_defer[2 * x].p);
                 ep.n_deferred = bc + 2 * x + 1;
+                ep.nb = (int)b.nb;
+                ep.vb_smem = p->prune == 2 && !last;
+                const int smem_l = ep.lay.bytes + (ep.vb_smem ? (int)b.nb * 128 * 8 : 0);
                 const int grid = x == 0 ? (int)std::max<long long>(
                                               1, std::min<long long>(((long long)b.nb + 255) / 256,
                                                                      s.grid_level))
                                         : s.grid_level;
                 s.launches++;
-                if ((st = launch_level(last, x, ep, grid, smem, s.stream)) != POS_OK) return st;
+                if ((st = launch_level(last, x, ep, grid, smem_l, s.stream)) != POS_OK)
+                    return st;
                 POS_CUDA(cudaEventRecord(ev[x + 1], s.stream));
             }
             if ((st = run_leaves(s, static_cast<const Leaf *>(s.d_leaves.p), bc + 2 * (S - 2),
@@ -1206,6 +1252,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
             if (!overflow) continue;
             s.reruns++;
             const Batch &b = batches[bi];
+            s.cur_nb = (int)b.nb;
             if ((st = launch_bounds_for(b)) != POS_OK) return st;
             st = process(s, d_ordered + b.off, b.M, 0, d_rootp, (long long)b.nb);
             if (st != POS_OK) return st;

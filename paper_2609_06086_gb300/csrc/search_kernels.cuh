@@ -155,11 +155,16 @@ template <int S, int PATH>
 __global__ void __launch_bounds__(256, (S <= 4 ? 4 : (S <= 8 ? 3 : 2)))
 leaf_kernel(LeafParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
-    stage_blob(sm, p.blob, p.lay.bytes);
-    __syncthreads();
-    const Tab t = tab_at(sm, p.lay);
+    __shared__ uint64_t bar;
     const unsigned long long c0 = __ldcg(p.count);
     const unsigned long long n = c0 < p.cap ? c0 : p.cap;
+    // blocks without a plan leave before staging the tables
+    if ((unsigned long long)blockIdx.x * blockDim.x >= n) return;
+    if (!stage_blob_bulk(sm, p.blob, p.lay.bytes, &bar)) {
+        if (threadIdx.x == 0) atomicAdd(p.stats + kStTimeout, 1ull);
+        return;
+    }
+    const Tab t = tab_at(sm, p.lay);
     const int L = p.lay.L;
     unsigned long long evaluated = 0;
     const unsigned long long stride = (unsigned long long)gridDim.x * blockDim.x;

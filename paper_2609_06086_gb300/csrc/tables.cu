@@ -66,6 +66,19 @@ BlobLayout make_layout(int L, int n_types, int n_tp) {
     return ly;
 }
 
+BlobLayout timing_layout(const BlobLayout &ly) {
+    BlobLayout t = ly;
+    const int base = ly.off_Pf;
+    t.off_binom = t.off_Pw = t.off_Pa = t.off_cap = -1;  // not staged
+    t.off_Pf -= base;
+    t.off_Pb -= base;
+    t.off_Pd -= base;
+    t.off_p2f -= base;
+    t.off_p2b -= base;
+    t.bytes = ly.bytes - base;
+    return t;
+}
+
 // One thread per (table, class) row: the raw per-layer row sits at entries
 // 1..L of the row; turn it into an exclusive prefix sum with P[0] = 0.
 __global__ void prefix_rows_kernel(unsigned char *blob, BlobLayout ly) {
