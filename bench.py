@@ -191,6 +191,10 @@ def run_ours(args, rank, world, local_rank):
     w = gen.config4()
     prob, keep = P.make_problem(w, warmup=WARMUP_SAMPLES, prune=args.prune, seed=0,
                                 frontier_cap=args.frontier_cap)
+    # the same search with CUDA events around every kernel, for the per-kernel
+    # breakdown (run after the timed steps; the events cost host time)
+    prob_prof, keep_prof = P.make_problem(w, warmup=WARMUP_SAMPLES, prune=args.prune, seed=0,
+                                          frontier_cap=args.frontier_cap, profile=True)
     tab_bytes = sum(a.nbytes for a in keep[0].arrays.values()) + sum(a.nbytes for a in keep[1:])
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.int32, device="cuda")
 
@@ -220,6 +224,20 @@ def run_ours(args, rank, world, local_rank):
         for k in agg:
             agg[k] += st[k]
     clk = clocks.stop() if clocks else None
+    # per-kernel breakdown: the same number of steps again, with CUDA events
+    # around every launch on the library's stream (profile=1)
+    prof_ms = []
+    kagg = {k: 0 for k in agg}
+    for _ in range(args.steps):
+        flush.zero_()
+        torch.cuda.synchronize()
+        ev0.record()
+        plan_p, st_p = P.poseidon_search(prob_prof)
+        ev1.record()
+        torch.cuda.synchronize()
+        prof_ms.append(ev0.elapsed_time(ev1))
+        for k in kagg:
+            kagg[k] += st_p[k]
     t_dev = sum(dev_ms)
     if dist:
         tt = torch.tensor([t_dev], dtype=torch.float64,
@@ -242,21 +260,22 @@ def run_ours(args, rank, world, local_rank):
     n_sm = props.multi_processor_count
     # roofline of the dominant kernel kind (device time from events on the
     # library's stream, accumulated over the timed steps)
-    kinds = {"leaf": agg["ms_leaf"], "expand": agg["ms_expand"], "complete": agg["ms_complete"]}
+    kinds = {"leaf": kagg["ms_leaf"], "expand": kagg["ms_expand"],
+             "complete": kagg["ms_complete"]}
     dom = max(kinds, key=kinds.get)
     mhz = (clk or {}).get("sm_mhz") or 2070.0
     peak_alu = n_sm * SM_LANES * mhz * 1e6 / 1e12  # Tops/s at the measured SM clock
     peak_hbm, hbm_src = measured_hbm()
     S = w.S
-    launches = {"leaf": agg["leaf_launches"], "expand": agg["expand_launches"],
-                "complete": agg["complete_launches"]}
+    launches = {"leaf": kagg["leaf_launches"], "expand": kagg["expand_launches"],
+                "complete": kagg["complete_launches"]}
     # algorithmic work per kind (roofline section):
     #  leaf     : int32 ops, 3 per DAG node relaxation + 9 per stage
     #  expand   : bytes, a 32-byte frontier entry read per parent and written per child
     #  complete : bytes, a 32-byte entry read per parent and a 32-byte plan written per leaf
-    work = {"leaf": 3 * agg["relaxations"] + 9 * S * agg["evaluated"],
-            "expand": ENTRY_BYTES * (agg["parents_expand"] + agg["prefixes"]),
-            "complete": ENTRY_BYTES * (agg["parents_complete"] + agg["leaves"])}
+    work = {"leaf": 3 * kagg["relaxations"] + 9 * S * kagg["evaluated"],
+            "expand": ENTRY_BYTES * (kagg["parents_expand"] + kagg["prefixes"]),
+            "complete": ENTRY_BYTES * (kagg["parents_complete"] + kagg["leaves"])}
     bound = {"leaf": ("alu", "Tops/s", peak_alu, 1e12),
              "expand": ("hbm", "GB/s", peak_hbm, 1e9),
              "complete": ("hbm", "GB/s", peak_hbm, 1e9)}
@@ -311,6 +330,9 @@ def run_ours(args, rank, world, local_rank):
                  "tp": plans[-1]["tp"], "D": plans[-1]["D"], "layers": plans[-1]["layers"],
                  "types": plans[-1]["types"], "matches_oracle": parity},
         "kernels": per_kind,
+        "kernel_timing": (f"{args.steps} further searches of the same workload with CUDA events "
+                          f"around every launch (profile=1): {sum(prof_ms) / len(prof_ms):.3f} "
+                          "ms per search"),
         "host_ms_per_step": {k: round(agg[k] / args.steps, 3)
                              for k in ("ms_setup", "ms_warmup", "ms_search")},
         "roofline": roof,

@@ -212,6 +212,8 @@ typedef struct pos_problem {
     int32_t schedule;           /* POS_SCHED_1F1B */
     int64_t frontier_cap;       /* entries per frontier buffer; 0 = default 2^24;
                                    raised to at least 32*L */
+    int32_t profile;            /* 1: device time per kernel kind in the stats (CUDA
+                                   events around every launch); 0: those fields are 0 */
 } pos_problem;
 
 typedef struct pos_plan {

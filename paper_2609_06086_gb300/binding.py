@@ -41,7 +41,7 @@ class pos_problem(C.Structure):
                 ("M_list", C.c_void_p), ("tp_list", C.c_void_p), ("dp_list", C.c_void_p),
                 ("placement", C.c_int32), ("type_counts", C.c_void_p), ("warmup", C.c_int32),
                 ("prune", C.c_int32), ("seed", C.c_uint64), ("schedule", C.c_int32),
-                ("frontier_cap", C.c_int64)]
+                ("frontier_cap", C.c_int64), ("profile", C.c_int32)]
 
 
 class pos_plan(C.Structure):
@@ -181,7 +181,7 @@ def _prune_mode(prune):
     return int(prune)
 
 
-def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0):
+def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0, profile=False):
     """pos_problem for a gen.Workload search; returns (problem, keep-alive list)."""
     tab = Tables.from_workload(w)
     keep = [tab]
@@ -193,7 +193,8 @@ def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0):
 
     p = pos_problem(tab.c, w.S, len(w.M_list), arr(w.M_list), arr(w.tp_list), arr(w.dp_list),
                     w.placement, arr(w.type_counts if w.type_counts else [0] * w.n_types),
-                    int(warmup), _prune_mode(prune), int(seed), POS_SCHED_1F1B, int(frontier_cap))
+                    int(warmup), _prune_mode(prune), int(seed), POS_SCHED_1F1B, int(frontier_cap),
+                    int(bool(profile)))
     return p, keep
 
 

@@ -19,11 +19,22 @@ namespace pos {
 void set_error(const std::string &msg);
 pos_status fail(pos_status st, const std::string &msg);
 pos_status cuda_fail(cudaError_t e, const char *what);
+// Raises a kernel's dynamic shared-memory limit to `smem` on the current
+// device unless an earlier call already set at least that much (the
+// attribute call costs host time that a launch-bound pipeline feels).
+pos_status ensure_smem(const void *kernel, int smem);
 
 #define POS_CUDA(call)                                           \
     do {                                                         \
         cudaError_t e_ = (call);                                 \
         if (e_ != cudaSuccess) return pos::cuda_fail(e_, #call); \
+    } while (0)
+
+// Propagate a non-OK pos_status.
+#define POS_TRY(call)                             \
+    do {                                          \
+        const pos_status st_ = (call);            \
+        if (st_ != POS_OK) return st_;            \
     } while (0)
 
 // ---------------------------------------------------------------------------

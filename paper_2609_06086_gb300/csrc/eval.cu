@@ -165,7 +165,7 @@ __global__ void __launch_bounds__(256, 4) decode_kernel(EvalParams p) {
 
 pos_status launch_decode(const EvalParams &p, cudaStream_t stream) {
     const int smem = p.lay.bytes;
-    POS_CUDA(cudaFuncSetAttribute(decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    POS_TRY(ensure_smem(reinterpret_cast<const void *>(decode_kernel), smem));
     int per_sm = 0;
     POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_kernel, 256, smem));
     const int64_t blocks = (p.n + 255) / 256;

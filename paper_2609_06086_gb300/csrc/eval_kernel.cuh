@@ -183,7 +183,7 @@ template <int SLO, int SHI, int PATH, int MINB>
 pos_status launch_eval_range(const EvalParams &p, cudaStream_t stream) {
     auto kern = eval_kernel<SLO, SHI, PATH, MINB>;
     const int smem = p.lay.bytes;
-    POS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    POS_TRY(ensure_smem(reinterpret_cast<const void *>(kern), smem));
     int per_sm = 0;
     POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kEvalThreads, smem));
     if (per_sm < 1) return fail(POS_ECUDA, "eval kernel does not fit on an SM");

@@ -110,55 +110,102 @@ __global__ void root_bits_kernel(const uint4 *feas, int n_slices, int S, uint8_t
 // A prefix whose A + V1 or A + Bm + V2 exceeds the incumbent has no
 // completion that beats it.  Each finite entry is at most the makespan of
 // a feasible plan, so it fits in int32 under the overflow guard.
-// One block per slot of the batch, thread c; vb[(x*nb + slot)*128 + c], so
-// that the rows of one depth for every slot are contiguous.
-__global__ void bound_kernel(const SliceRec *batch, int nb, int S, const uint8_t *lim, int2 *vb,
-                             const void *blob, BlobLayout lay, unsigned long long *stats) {
+// One block per memory-feasible slice, four threads per start c (each
+// takes every fourth layer count, then the four minima are combined by
+// shuffles).  vb[(x*n_rows + vslot)*128 + c]; arg[x][c] (shared memory)
+// keeps the smallest l attaining V1[x][c], and thread 0 follows it from
+// (0, 0) to write the slice's argmin completion as a plan: a memory-feasible
+// plan whose makespan is usually close to the slice's best (warm-up seed).
+constexpr int kBoundThreads = 512;
+
+__global__ void __launch_bounds__(kBoundThreads) bound_kernel(
+    const SliceRec *slices, const uint32_t *rows, int n_rows, int S, const uint8_t *lim,
+    int2 *vb, Leaf *greedy, const void *blob, BlobLayout lay, unsigned long long *stats) {
     extern __shared__ __align__(16) unsigned char sm[];
     __shared__ int2 nxt[128];
+    __shared__ uint8_t arg[POS_MAX_STAGES][128];
     __shared__ uint64_t bar;
     if (!stage_blob_bulk(sm, blob, lay.bytes, &bar)) {
         if (threadIdx.x == 0) atomicAdd(stats + kStTimeout, 1ull);
         return;
     }
     const Tab t = tab_at(sm, lay);
-    const int L = lay.L, c = threadIdx.x;
-    for (int slot = blockIdx.x; slot < nb; slot += gridDim.x) {
-        const SliceRec &sr = batch[slot];
+    const int L = lay.L, c = threadIdx.x >> 2, part = threadIdx.x & 3;
+    for (int r = blockIdx.x; r < n_rows; r += gridDim.x) {
+        const uint32_t sl = rows[r];
+        const SliceRec &sr = slices[sl];
         const int M = sr.M;
-        for (int x = S - 1; x >= 1; --x) {
+        const uint32_t vslot = sr.vslot;
+        for (int x = S - 1; x >= 0; --x) {
             const int k = sr.cls[x];
             const int32_t pf = x + 1 < S ? p2f(t, k, sr.cls[x + 1]) : 0;
             const int32_t pb = x + 1 < S ? p2b(t, sr.cls[x + 1], k) : 0;
             int64_t v1 = INT64_MAX, v2 = INT64_MAX;
+            int best_l = 0;
             if (c < L) {
                 const int most = lim[((size_t)sr.gid * S + x) * 128 + c];
                 const int32_t f0 = Pf(t, k, c), b0 = Pb(t, k, c), d0 = Pd(t, k, c);
                 const int l_lo = x == S - 1 ? L - c : 1;
                 const int l_hi = x == S - 1 ? L - c : min(most, L - c - (S - 1 - x));
-                for (int l = l_lo; l <= l_hi && l <= most; ++l) {
+                for (int l = l_lo + part; l <= l_hi && l <= most; l += 4) {
                     const int c2 = c + l;
                     const int64_t F = Pf(t, k, c2) - f0, B = Pb(t, k, c2) - b0;
                     const int64_t d = Pd(t, k, c2) - d0;
                     const int64_t a = (int64_t)M * (F + B);
+                    int64_t w1, w2;
                     if (x == S - 1) {
-                        v1 = a + d;
-                        v2 = a;
+                        w1 = a + d;
+                        w2 = a;
                     } else {
                         const int2 n = nxt[c2];
                         if (n.x == kNoCompletion) continue;
-                        v1 = min(v1, max(a + d, F + pf + n.x));
-                        v2 = min(v2, max(a, F + pf + B + pb + n.y));
+                        w1 = max(a + d, F + pf + n.x);
+                        w2 = max(a, F + pf + B + pb + n.y);
                     }
+                    if (w1 < v1) {  // l increases: the first strict minimum is the smallest l
+                        v1 = w1;
+                        best_l = l;
+                    }
+                    v2 = min(v2, w2);
                 }
             }
+            // combine the four partial minima of start c (lanes 4c .. 4c+3);
+            // ties in V1 go to the smallest l
+#pragma unroll
+            for (int o = 1; o < 4; o <<= 1) {
+                const int64_t o1 = __shfl_xor_sync(0xffffffffu, v1, o);
+                const int64_t o2 = __shfl_xor_sync(0xffffffffu, v2, o);
+                const int ol = __shfl_xor_sync(0xffffffffu, best_l, o);
+                if (o1 < v1 || (o1 == v1 && ol < best_l)) {
+                    v1 = o1;
+                    best_l = ol;
+                }
+                v2 = min(v2, o2);
+            }
             __syncthreads();  // every thread has read row x+1
-            const int2 out = v1 == INT64_MAX ? make_int2(kNoCompletion, kNoCompletion)
-                                             : make_int2((int32_t)v1, (int32_t)v2);
-            nxt[c] = out;
-            vb[((size_t)x * nb + slot) * 128 + c] = out;
+            if (part == 0) {
+                const int2 out = v1 == INT64_MAX ? make_int2(kNoCompletion, kNoCompletion)
+                                                 : make_int2((int32_t)v1, (int32_t)v2);
+                nxt[c] = out;
+                arg[x][c] = (uint8_t)best_l;
+                vb[((size_t)x * n_rows + vslot) * 128 + c] = out;
+            }
             __syncthreads();
         }
+        if (threadIdx.x == 0) {
+            // the root of a memory-feasible slice always has a completion
+            uint32_t cw[4] = {0u, 0u, 0u, 0u};  // cut[x] in byte x
+            int cc = 0;
+            for (int x = 0; x < S - 1; ++x) {
+                cc += arg[x][cc];
+                const uint32_t v = (uint32_t)cc << (8 * (x % 4));
+#pragma unroll
+                for (int wi = 0; wi < 4; ++wi) cw[wi] |= (x / 4 == wi) ? v : 0u;
+            }
+            const Vec32 lf = {make_uint4(sl, cw[0], cw[1], cw[2]), make_uint4(cw[3], 0u, 0u, 0u)};
+            store32(greedy + r, lf);
+        }
+        __syncthreads();
     }
 }
 
@@ -254,12 +301,14 @@ struct ExpandParams {
     int x;                   // depth of the parents (stages 0..x-1 placed)
     int S, M;
     int prune;
+    int exact;               // 1: host-driven pass (lane-per-parent mode with deferral lists)
     const SliceRec *slices;
     const uint4 *feas;
     const uint8_t *lim;      // per (slice, stage, start) memory limit, see feas_kernel
     const int2 *vb;          // prune 2: completion bounds per (batch slot, stage, start)
     int vb_smem;             // 1: stage this depth's rows of all nb slots in shared memory
     int nb;                  // slots in the batch
+    int n_vrows;             // rows per depth of vb (vb[(x*n_vrows + vslot)*128 + c])
     Prefix *out;             // expand: children at depth x+1
     Leaf *leaves;            // complete: full plans
     unsigned long long *out_count;
@@ -437,6 +486,141 @@ __device__ __forceinline__ int complete_set(const ExpandParams &p, const Tab &t,
     return n;
 }
 
+// Small frontiers: one warp per parent.  Lane j tests the layer counts
+// l = 1 + j + 32 r (r = 0..3) of the new stage X at once: memory (l <= the
+// memory limit row), Eq. 2 for the child, the feasibility bit of c + l and
+// the per-candidate test (completion bounds when expanding under prune
+// mode 2, g(S_S) when completing); four ballots hold the survivors, one
+// atomic reserves their slots.  Only the pipelined pass uses this mode; on
+// overflow it counts the parent as deferred without listing it (the batch
+// is then run again by the host-driven path).  Statistics are kept by
+// lane 0.
+template <bool COMPLETE, int X>
+__device__ __forceinline__ void level_warp_mode(const ExpandParams &p, const Tab &t,
+                                                long long n_in, const int2 *vsm,
+                                                const int2 *vdepth, uint64_t thr,
+                                                unsigned long long &emitted,
+                                                unsigned long long &cb, unsigned long long &cm,
+                                                unsigned long long &written) {
+    const int lane = threadIdx.x & 31;
+    const unsigned lt_mask = (1u << lane) - 1u;
+    const long long warp = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
+    const long long n_warps = ((long long)gridDim.x * blockDim.x) >> 5;
+    const int S = p.S, M = p.M, L = t.L();
+    for (long long i = warp; i < n_in; i += n_warps) {
+        const Vec32 pv = load32(p.in + i);  // one address: a broadcast
+        const uint32_t slice = pv.a.x & 0xffffu;
+        if (slice == kPrefixHole) continue;
+        const SliceRec &sr = p.slices[slice];
+        const int c = X > 0 ? (int)get_byte<(X > 0 ? X + 1 : 2)>(pv) : 0;
+        const ParentCtx q = parent_ctx(t, sr.cls[X], c);
+        const int kb = sr.cls[X + 1];  // X + 1 <= S - 1
+        const int32_t pf = p.prune == 2 ? p2f(t, q.k, kb) : 0;
+        const int32_t pb = p.prune == 2 ? p2b(t, kb, q.k) : 0;
+        const uint64_t scale = sr.scale;
+        const uint32_t gid = sr.gid;
+        const int64_t A = (int32_t)pv.b.x, Bm = (int32_t)pv.b.y;
+        const int lmax = COMPLETE ? L - c - 1 : L - c - (S - X - 1);
+        const int hi_mem = min(lmax, (int)__ldg(p.lim + ((size_t)gid * S + X) * 128 + c));
+        // expansion: the next stage must fit from c + l (row X+1); completion:
+        // stage S-1 must hold [c + l, L) (row S-1)
+        const uint4 f = __ldg(p.feas + (size_t)gid * (S + 1) + (COMPLETE ? S - 1 : X + 1));
+        const int2 *vrow = vsm ? vsm + (size_t)slice * 128
+                               : (vdepth ? vdepth + (size_t)sr.vslot * 128 : nullptr);
+        unsigned pass[4];
+        int n_bound = 0, n_win = 0, n_fail = 0;
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            const int l = 1 + lane + 32 * r;
+            const int c2 = c + l;
+            const bool in_mem = l <= hi_mem;
+            bool g_ok = false, cand = false, ok = false;
+            if (in_mem) {
+                const int64_t F = Pf(t, q.k, c2) - q.f0, B = Pb(t, q.k, c2) - q.b0;
+                const int64_t d = Pd(t, q.k, c2) - q.d0;
+                g_ok = !p.prune ||
+                       (uint64_t)(A + (int64_t)M * (F + B) + max(Bm, d)) * scale <= thr;
+                const uint32_t word2 = (c2 >> 5) == 0 ? f.x : (c2 >> 5) == 1 ? f.y
+                                     : (c2 >> 5) == 2 ? f.z : f.w;
+                cand = g_ok && ((word2 >> (c2 & 31)) & 1u);
+                ok = cand;
+                if (cand) {
+                    const int64_t A2 = A + F + pf, Bm2 = max(Bm, d) + B + pb;
+                    if (COMPLETE) {
+                        if (p.prune) {
+                            const int64_t Fb = Pf(t, kb, L) - Pf(t, kb, c2);
+                            const int64_t Bb = Pb(t, kb, L) - Pb(t, kb, c2);
+                            const int64_t db = Pd(t, kb, L) - Pd(t, kb, c2);
+                            ok = (uint64_t)(A2 + (int64_t)M * (Fb + Bb) + max(Bm2, db)) * scale <=
+                                 thr;
+                        }
+                    } else if (p.prune == 2) {
+                        const int2 v = vrow[c2];
+                        ok = v.x != kNoCompletion && (uint64_t)(A2 + v.x) * scale <= thr &&
+                             (uint64_t)(A2 + Bm2 + v.y) * scale <= thr;
+                    }
+                }
+            }
+            pass[r] = __ballot_sync(0xffffffffu, ok);
+            n_bound += __popc(__ballot_sync(0xffffffffu, in_mem && g_ok));
+            n_win += __popc(__ballot_sync(0xffffffffu, cand));
+            n_fail += __popc(__ballot_sync(0xffffffffu, cand && !ok));
+        }
+        const int total = __popc(pass[0]) + __popc(pass[1]) + __popc(pass[2]) + __popc(pass[3]);
+        if (lane == 0) {
+            cm += (unsigned long long)(lmax - hi_mem) + (unsigned long long)(n_bound - n_win);
+            cb += (unsigned long long)(hi_mem - n_bound) + (unsigned long long)n_fail;
+            written += 1;
+        }
+        if (total == 0) continue;
+        unsigned long long base = 0;
+        if (lane == 0) base = atomicAdd(p.out_count, (unsigned long long)total);
+        base = __shfl_sync(0xffffffffu, base, 0);
+        if (base + (unsigned long long)total > p.cap) {
+            // no room: reserved slots below the capacity become holes
+            const Vec32 hole = {make_uint4(COMPLETE ? kLeafHole : kPrefixHole, 0, 0, 0),
+                                make_uint4(0, 0, 0, 0)};
+            for (unsigned long long e = base + lane; e < base + (unsigned long long)total && e < p.cap;
+                 e += 32) {
+                if (COMPLETE) store32(p.leaves + e, hole);
+                else store32(p.out + e, hole);
+            }
+            if (lane == 0) atomicAdd(p.n_deferred, 1ull);
+            continue;
+        }
+        unsigned long long pos = base;
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+            if ((pass[r] >> lane) & 1u) {
+                const int c2 = c + 1 + lane + 32 * r;
+                const unsigned long long at = pos + (unsigned long long)__popc(pass[r] & lt_mask);
+                Vec32 out;
+                if (COMPLETE) {
+                    // leaf: slice in bytes 0-3, cut[i] in byte 4+i; the
+                    // parent's cuts (bytes 2..15) move up two bytes
+                    out.a.x = slice;
+                    out.a.y = __funnelshift_r(pv.a.x, pv.a.y, 16);
+                    out.a.z = __funnelshift_r(pv.a.y, pv.a.z, 16);
+                    out.a.w = __funnelshift_r(pv.a.z, pv.a.w, 16);
+                    out.b = make_uint4(pv.a.w >> 16, 0u, 0u, 0u);
+                    set_byte<4 + X>(out, (uint32_t)c2);
+                    store32(p.leaves + at, out);
+                } else {
+                    const int32_t F = Pf(t, q.k, c2) - q.f0, B = Pb(t, q.k, c2) - q.b0;
+                    const int32_t d = Pd(t, q.k, c2) - q.d0;
+                    out.a = pv.a;
+                    out.b = make_uint4((uint32_t)((int32_t)pv.b.x + F + pf),
+                                       (uint32_t)(max((int32_t)pv.b.y, d) + B + pb), 0u, 0u);
+                    set_byte<2 + (X < 14 ? X : 0)>(out, (uint32_t)c2);
+                    store32(p.out + at, out);
+                }
+            }
+            pos += (unsigned long long)__popc(pass[r]);
+        }
+        if (lane == 0) emitted += (unsigned long long)total;
+    }
+}
+
 // One warp per group of 32 consecutive parents: each lane finds its
 // parent's children (a 128-bit set of cut positions), the warp reserves
 // output slots with one atomic and writes them -- or, when the output is
@@ -450,33 +634,44 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
         n_in = (long long)(c0 < p.cap ? c0 : p.cap);
     }
     const long long n_work = p.groups ? p.n_groups : (n_in + 31) / 32;
-    // blocks without a group leave before staging anything
-    if ((long long)blockIdx.x * (kThreads / 32) >= n_work) return;
+    const long long n_warps = ((long long)gridDim.x * blockDim.x) >> 5;
+    // small frontier in the pipelined pass: one warp per parent
+    const bool warp_mode = !p.exact && !p.groups && n_in <= n_warps;
+    // blocks without work leave before staging anything
+    if ((long long)blockIdx.x * (kThreads / 32) >= (warp_mode ? n_in : n_work)) return;
     // timing tables and, when expanding under prune mode 2, the
     // completion-bound rows of depth X+1 of every slot (contiguous), by TMA
     __shared__ uint64_t bar;
     const bool use_v = !COMPLETE && p.prune == 2;
     const bool stage_v = use_v && p.vb_smem;
-    const int2 *vrows = use_v ? p.vb + (size_t)(X + 1) * p.nb * 128 : nullptr;
+    // depth X+1 of the bound tables: the row of table row v is vdepth + 128 v
+    const int2 *vdepth = use_v ? p.vb + (size_t)(X + 1) * p.n_vrows * 128 : nullptr;
     if (threadIdx.x == 0) {
         const uint32_t vbytes = stage_v ? (uint32_t)p.nb * 128u * 8u : 0u;
         bulk_begin(&bar, (uint32_t)p.lay.bytes + vbytes);
         bulk_copy(sm, p.blob, (uint32_t)p.lay.bytes, &bar);
-        if (stage_v) bulk_copy(sm + p.lay.bytes, vrows, vbytes, &bar);
+    }
+    if (stage_v) {
+        __syncthreads();  // the barrier is armed before the other copies start
+        if (threadIdx.x < 32)
+            for (int slot = threadIdx.x; slot < p.nb; slot += 32)
+                bulk_copy(sm + p.lay.bytes + (size_t)slot * 1024,
+                          vdepth + (size_t)__ldg(&p.slices[slot].vslot) * 128, 1024u, &bar);
     }
     if (!bulk_wait(&bar)) {
         if (threadIdx.x == 0) atomicAdd(p.stats + kStTimeout, 1ull);
         return;
     }
-    const int2 *vbase = stage_v ? reinterpret_cast<const int2 *>(sm + p.lay.bytes) : vrows;
-    const size_t vstride = 128;
+    const int2 *vsm = stage_v ? reinterpret_cast<const int2 *>(sm + p.lay.bytes) : nullptr;
     const Tab t = tab_at(sm, p.lay);
     const uint64_t thr = p.prune ? __ldcg(&p.inc->obj) : ~0ull;
     const int lane = threadIdx.x & 31;
     const long long warp = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
-    const long long n_warps = ((long long)gridDim.x * blockDim.x) >> 5;
-    unsigned long long emitted = 0, cb = 0, cm = 0, parents = 0, written_parents = 0;
-    for (long long w = warp; w < n_work; w += n_warps) {
+    unsigned long long emitted = 0, cb = 0, cm = 0, written_parents = 0;
+    if (warp_mode)
+        level_warp_mode<COMPLETE, X>(p, t, n_in, vsm, vdepth, thr, emitted, cb, cm,
+                                     written_parents);
+    for (long long w = warp; !warp_mode && w < n_work; w += n_warps) {
         const long long g = p.groups ? (long long)p.groups[w] : w;
         const long long i = g * 32 + lane;
         Vec32 pv = {make_uint4(kPrefixHole, 0, 0, 0), make_uint4(0, 0, 0, 0)};
@@ -501,8 +696,10 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
             const int64_t A = (int32_t)pv.b.x, Bm = (int32_t)pv.b.y;
             n = COMPLETE ? complete_set(p, t, A, Bm, q, sr.cls[X + 1], sr.gid, scale, thr, acc, lb,
                                         lm)
-                         : expand_set(p, t, A, Bm, q, sr.gid, vbase + slice * vstride, scale,
-                                      thr, acc,
+                         : expand_set(p, t, A, Bm, q, sr.gid,
+                                      vsm ? vsm + (size_t)slice * 128
+                                          : (vdepth ? vdepth + (size_t)sr.vslot * 128 : nullptr),
+                                      scale, thr, acc,
                                       lb, lm);
         }
         int incl = n;
@@ -568,7 +765,6 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
             }
         }
     }
-    (void)parents;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         emitted += __shfl_xor_sync(0xffffffffu, emitted, o);
@@ -624,7 +820,7 @@ struct Workspace {
     std::mutex mu;
     cudaStream_t stream = nullptr;
     cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
-    DevBuf blob, d_lim, d_vb, d_bctr, d_slices, d_feas, d_batch, d_inc, d_ctr, d_best, d_feasible, d_leaves, d_roots,
+    DevBuf blob, d_lim, d_vb, d_bctr, d_rows, d_greedy, d_wcnt, d_slices, d_feas, d_batch, d_inc, d_ctr, d_best, d_feasible, d_leaves, d_roots,
         d_root;
     DevBuf d_front[POS_MAX_STAGES + 1];        // per depth: Prefix buffers
     DevBuf d_defer[2 * (POS_MAX_STAGES + 1)];  // per depth: two deferred group lists
@@ -683,7 +879,8 @@ struct Search {
     uint64_t launches = 0;
     double ms_expand = 0, ms_complete = 0, ms_leaf = 0, ms_bound = 0;
     uint64_t n_expand = 0, n_complete = 0, n_leaf = 0, n_bound = 0, reruns = 0;
-    int cur_nb = 0;  // slots of the batch being enumerated (row stride of the bound tables)
+    int cur_nb = 0;    // slots of the batch being enumerated
+    int n_vrows = 0;   // rows of the completion-bound tables (memory-feasible slices)
 };
 
 static pos_status validate_problem(const pos_problem *p) {
@@ -800,6 +997,7 @@ static ExpandParams base_params(Search &s, const SliceRec *batch, int M) {
     p.lim = static_cast<const uint8_t *>(s.ws.d_lim.p);
     p.vb = static_cast<const int2 *>(s.ws.d_vb.p);
     p.nb = s.cur_nb;
+    p.n_vrows = s.n_vrows;
     p.cap = (unsigned long long)s.cap;
     p.inc = static_cast<const Key128 *>(s.d_inc.p);
     p.stats = s.stats;
@@ -830,7 +1028,7 @@ static pos_status run_leaves(Search &s, const Leaf *leaves, unsigned long long *
 template <bool COMPLETE, int X>
 static pos_status launch_level_t(const ExpandParams &p, int grid, int smem, cudaStream_t st) {
     auto kern = level_kernel<COMPLETE, X>;
-    POS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    POS_TRY(ensure_smem(reinterpret_cast<const void *>(kern), smem));
     kern<<<grid, kThreads, smem, st>>>(p);
     POS_CUDA(cudaGetLastError());
     return POS_OK;
@@ -872,6 +1070,7 @@ static pos_status process(Search &s, const SliceRec *batch, int M, int x, const 
     for (;;) {
         POS_CUDA(cudaMemsetAsync(out_count, 0, 2 * sizeof(unsigned long long), s.stream));
         ExpandParams p = base_params(s, batch, M);
+        p.exact = 1;
         p.in = in;
         p.n_in = n_in;
         p.groups = work;
@@ -887,28 +1086,30 @@ static pos_status process(Search &s, const SliceRec *batch, int M, int x, const 
         const int grid = (int)std::max<long long>(1, std::min<long long>(blocks_needed,
                                                                          s.grid_level));
         s.launches++;
-        POS_CUDA(cudaEventRecord(s.ev[0], s.stream));
+        const bool prof = s.pb->profile != 0;
+        if (prof) POS_CUDA(cudaEventRecord(s.ev[0], s.stream));
         if ((st = launch_level(last, x, p, grid, smem, s.stream)) != POS_OK) return st;
-        POS_CUDA(cudaEventRecord(s.ev[1], s.stream));
+        (last ? s.n_complete : s.n_expand)++;
+        if (prof) POS_CUDA(cudaEventRecord(s.ev[1], s.stream));
         if (last) {
             // evaluate the leaves that fit; the count stays on the device
             if ((st = run_leaves(s, p.leaves, out_count, batch, M, nullptr)) != POS_OK) return st;
-            POS_CUDA(cudaEventRecord(s.ev[2], s.stream));
+            s.n_leaf++;
+            if (prof) POS_CUDA(cudaEventRecord(s.ev[2], s.stream));
         }
         unsigned long long cnt[2];
         if ((st = sync_read(s, cnt, out_count, sizeof(cnt))) != POS_OK) return st;
-        float ms_k = 0;
-        POS_CUDA(cudaEventElapsedTime(&ms_k, s.ev[0], s.ev[1]));
-        if (last) {
-            s.ms_complete += ms_k;
-            s.n_complete++;
-            float ms_l = 0;
-            POS_CUDA(cudaEventElapsedTime(&ms_l, s.ev[1], s.ev[2]));
-            s.ms_leaf += ms_l;
-            s.n_leaf++;
-        } else {
-            s.ms_expand += ms_k;
-            s.n_expand++;
+        if (prof) {
+            float ms_k = 0;
+            POS_CUDA(cudaEventElapsedTime(&ms_k, s.ev[0], s.ev[1]));
+            if (last) {
+                s.ms_complete += ms_k;
+                float ms_l = 0;
+                POS_CUDA(cudaEventElapsedTime(&ms_l, s.ev[1], s.ev[2]));
+                s.ms_leaf += ms_l;
+            } else {
+                s.ms_expand += ms_k;
+            }
         }
         if (!last) {
             const long long n_out = (long long)std::min<unsigned long long>(cnt[0], s.cap);
@@ -990,11 +1191,9 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
             }
     const int smem = s.h->lay.bytes;
     int per_sm = 0;
-    POS_CUDA(cudaFuncSetAttribute(level_kernel<false, 0>,
-                                  cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-    POS_CUDA(cudaFuncSetAttribute(feas_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
-    POS_CUDA(cudaFuncSetAttribute(bound_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                  smem));
+    POS_TRY(ensure_smem(reinterpret_cast<const void *>(level_kernel<false, 0>), smem));
+    POS_TRY(ensure_smem(reinterpret_cast<const void *>(feas_kernel), smem));
+    POS_TRY(ensure_smem(reinterpret_cast<const void *>(bound_kernel), smem));
     POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(
         &per_sm, level_kernel<false, 0>, kThreads, timing_layout(s.h->lay).bytes));
     s.grid_level = std::max(1, per_sm) * sm_count();
@@ -1038,9 +1237,59 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         }
     const double ms_setup = ms_since(t_start);
 
-    // warm-up, split over the M values in proportion to their feasible slices
+    // prune mode 2: completion-bound tables of every memory-feasible slice
+    // (one launch), and each slice's argmin completion as a warm-up plan
     const auto t_warm = std::chrono::steady_clock::now();
     uint64_t warm_evals = 0;
+    std::vector<size_t> feas_off(p->n_M + 1, 0);  // first row of each M index
+    for (int mi = 0; mi < p->n_M; ++mi) feas_off[mi + 1] = feas_off[mi] + feas_by_m[mi].size();
+    if (p->prune == 2 && n_feasible > 0) {
+        std::vector<uint32_t> rows;
+        rows.reserve(n_feasible);
+        for (int mi = 0; mi < p->n_M; ++mi)
+            for (uint32_t g : feas_by_m[mi]) {
+                s.slices[g].vslot = (uint32_t)rows.size();
+                rows.push_back(g);
+            }
+        s.n_vrows = (int)rows.size();
+        POS_CUDA(s.ws.d_rows.reserve(sizeof(uint32_t) * rows.size()));
+        POS_CUDA(s.ws.d_vb.reserve(sizeof(int2) * 128 * (size_t)s.S * rows.size()));
+        POS_CUDA(s.ws.d_greedy.reserve(sizeof(Leaf) * rows.size()));
+        POS_CUDA(cudaMemcpyAsync(s.ws.d_rows.p, rows.data(), sizeof(uint32_t) * rows.size(),
+                                 cudaMemcpyHostToDevice, s.stream));
+        POS_CUDA(cudaMemcpyAsync(s.d_slices.p, s.slices.data(), sizeof(SliceRec) * n_slices,
+                                 cudaMemcpyHostToDevice, s.stream));
+        const BlobLayout tl = timing_layout(s.h->lay);
+        POS_TRY(ensure_smem(reinterpret_cast<const void *>(bound_kernel), tl.bytes));
+        if (p->profile) POS_CUDA(cudaEventRecord(s.ev[0], s.stream));
+        bound_kernel<<<(int)std::min<size_t>(rows.size(), 8 * sm_count()), kBoundThreads, tl.bytes,
+                       s.stream>>>(
+            d_all, static_cast<const uint32_t *>(s.ws.d_rows.p), (int)rows.size(), s.S,
+            static_cast<const uint8_t *>(s.ws.d_lim.p), static_cast<int2 *>(s.ws.d_vb.p),
+            static_cast<Leaf *>(s.ws.d_greedy.p),
+            static_cast<const unsigned char *>(s.h->d_blob) + s.h->lay.off_Pf, tl, s.stats);
+        POS_CUDA(cudaGetLastError());
+        if (p->profile) POS_CUDA(cudaEventRecord(s.ev[1], s.stream));
+        s.launches++;
+        s.n_bound++;
+        // counts of the greedy plans per M index, then one leaf launch each
+        std::vector<unsigned long long> gc(p->n_M);
+        for (int mi = 0; mi < p->n_M; ++mi) gc[mi] = feas_by_m[mi].size();
+        POS_CUDA(s.ws.d_wcnt.reserve(sizeof(unsigned long long) * p->n_M));
+        POS_CUDA(cudaMemcpyAsync(s.ws.d_wcnt.p, gc.data(), sizeof(unsigned long long) * p->n_M,
+                                 cudaMemcpyHostToDevice, s.stream));
+        for (int mi = 0; mi < p->n_M; ++mi) {
+            if (gc[mi] == 0) continue;
+            if ((st = run_leaves(s, static_cast<const Leaf *>(s.ws.d_greedy.p) + feas_off[mi],
+                                 static_cast<unsigned long long *>(s.ws.d_wcnt.p) + mi, d_all,
+                                 p->M_list[mi], static_cast<unsigned long long *>(s.d_best.p))) !=
+                POS_OK)
+                return st;
+            warm_evals += gc[mi];
+        }
+    }
+    // warm-up sampling (Sec. 4.2.3), split over the M values in proportion
+    // to their feasible slices
     if (p->warmup > 0 && n_feasible > 0) {
         POS_CUDA(s.d_feasible.reserve(sizeof(uint32_t) * n_feasible));
         for (int mi = 0; mi < p->n_M; ++mi) {
@@ -1072,6 +1321,11 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     if ((st = sync_read(s, best.data(), s.d_best.p, sizeof(unsigned long long) * n_slices)) !=
         POS_OK)
         return st;
+    if (p->profile && s.n_bound) {
+        float ms_b = 0;
+        POS_CUDA(cudaEventElapsedTime(&ms_b, s.ev[0], s.ev[1]));
+        s.ms_bound += ms_b;
+    }
     const double ms_warm = ms_since(t_warm);
 
     // batches of slices, most promising first
@@ -1126,19 +1380,6 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
                              cudaMemcpyHostToDevice, s.stream));
     const SliceRec *d_ordered = static_cast<const SliceRec *>(s.d_batch.p);
     const Prefix *d_rootp = static_cast<const Prefix *>(s.d_roots.p);
-    if (p->prune == 2) POS_CUDA(s.ws.d_vb.reserve(sizeof(int2) * max_nb * s.S * 128));
-    auto launch_bounds_for = [&](const Batch &b) -> pos_status {
-        if (p->prune != 2) return POS_OK;
-        const BlobLayout tl = timing_layout(s.h->lay);
-        bound_kernel<<<(int)std::min<size_t>(b.nb, 8 * sm_count()), 128, tl.bytes, s.stream>>>(
-            d_ordered + b.off, (int)b.nb, s.S, static_cast<const uint8_t *>(s.ws.d_lim.p),
-            static_cast<int2 *>(s.ws.d_vb.p),
-            static_cast<const unsigned char *>(s.h->d_blob) + s.h->lay.off_Pf, tl, s.stats);
-        POS_CUDA(cudaGetLastError());
-        s.launches++;
-        s.n_bound++;
-        return POS_OK;
-    };
 
     if (s.S == 1) {
         // the single stage takes every layer: each feasible slice is one plan
@@ -1173,9 +1414,10 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         POS_CUDA(s.ws.d_bctr.reserve(sizeof(unsigned long long) * 32 * std::max<size_t>(1, n_b)));
         unsigned long long *bctr = static_cast<unsigned long long *>(s.ws.d_bctr.p);
         POS_CUDA(cudaMemsetAsync(bctr, 0, sizeof(unsigned long long) * 32 * n_b, s.stream));
-        // timing events, S + 2 per batch: before the bound kernel, before
-        // level 0, after each level kernel, after the leaf kernel
-        const size_t n_ev = n_b * (S + 2);
+        // timing events (profile only), S + 1 per batch: before level 0,
+        // after each level kernel, after the leaf kernel
+        const bool prof = p->profile != 0;
+        const size_t n_ev = prof ? n_b * (S + 1) : 0;
         while (s.ws.evs.size() < n_ev) {
             cudaEvent_t e;
             POS_CUDA(cudaEventCreate(&e));
@@ -1184,12 +1426,9 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         for (size_t bi = 0; bi < n_b; ++bi) {
             const Batch &b = batches[bi];
             s.cur_nb = (int)b.nb;
-            cudaEvent_t *ev0 = s.ws.evs.data() + bi * (S + 2);
-            cudaEvent_t *ev = ev0 + 1;
-            POS_CUDA(cudaEventRecord(ev0[0], s.stream));
-            if ((st = launch_bounds_for(b)) != POS_OK) return st;
+            cudaEvent_t *ev = prof ? s.ws.evs.data() + bi * (S + 1) : nullptr;
             unsigned long long *bc = bctr + 32 * bi;
-            POS_CUDA(cudaEventRecord(ev[0], s.stream));
+            if (prof) POS_CUDA(cudaEventRecord(ev[0], s.stream));
             for (int x = 0; x <= S - 2; ++x) {
                 const bool last = x == S - 2;
                 ExpandParams ep = base_params(s, d_ordered + b.off, b.M);
@@ -1212,35 +1451,26 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
                 s.launches++;
                 if ((st = launch_level(last, x, ep, grid, smem_l, s.stream)) != POS_OK)
                     return st;
-                POS_CUDA(cudaEventRecord(ev[x + 1], s.stream));
+                (last ? s.n_complete : s.n_expand)++;
+                if (prof) POS_CUDA(cudaEventRecord(ev[x + 1], s.stream));
             }
             if ((st = run_leaves(s, static_cast<const Leaf *>(s.d_leaves.p), bc + 2 * (S - 2),
                                  d_ordered + b.off, b.M, nullptr)) != POS_OK)
                 return st;
-            POS_CUDA(cudaEventRecord(ev[S], s.stream));
+            s.n_leaf++;
+            if (prof) POS_CUDA(cudaEventRecord(ev[S], s.stream));
         }
         std::vector<unsigned long long> hb(32 * n_b);
         if ((st = sync_read(s, hb.data(), bctr, sizeof(unsigned long long) * hb.size())) != POS_OK)
             return st;
-        for (size_t bi = 0; bi < n_b; ++bi) {
-            cudaEvent_t *ev0 = s.ws.evs.data() + bi * (S + 2);
-            cudaEvent_t *ev = ev0 + 1;
-            float ms_b = 0;
-            POS_CUDA(cudaEventElapsedTime(&ms_b, ev0[0], ev[0]));
-            s.ms_bound += ms_b;
+        for (size_t bi = 0; bi < n_b && prof; ++bi) {
+            cudaEvent_t *ev = s.ws.evs.data() + bi * (S + 1);
             for (int x = 0; x <= S - 1; ++x) {
                 float ms = 0;
                 POS_CUDA(cudaEventElapsedTime(&ms, ev[x], ev[x + 1]));
-                if (x < S - 2) {
-                    s.ms_expand += ms;
-                    s.n_expand++;
-                } else if (x == S - 2) {
-                    s.ms_complete += ms;
-                    s.n_complete++;
-                } else {
-                    s.ms_leaf += ms;
-                    s.n_leaf++;
-                }
+                if (x < S - 2) s.ms_expand += ms;
+                else if (x == S - 2) s.ms_complete += ms;
+                else s.ms_leaf += ms;
             }
         }
         // A batch in which some frontier overflowed lost the children that
@@ -1253,7 +1483,6 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
             s.reruns++;
             const Batch &b = batches[bi];
             s.cur_nb = (int)b.nb;
-            if ((st = launch_bounds_for(b)) != POS_OK) return st;
             st = process(s, d_ordered + b.off, b.M, 0, d_rootp, (long long)b.nb);
             if (st != POS_OK) return st;
         }

@@ -20,7 +20,8 @@ struct SliceRec {
     uint8_t cls[16];   // class of each stage
     int32_t M;
     uint32_t gid;      // row of this slice in the feasibility table
-    uint32_t pad[2];
+    uint32_t vslot;    // row of this slice in the completion-bound tables (prune mode 2)
+    uint32_t pad;
 };
 static_assert(sizeof(SliceRec) == 48, "SliceRec layout");
 
@@ -222,7 +223,7 @@ template <int S, int PATH>
 pos_status launch_leaf_t(const LeafParams &p, int grid, cudaStream_t s) {
     auto kern = leaf_kernel<S, PATH>;
     const int smem = p.lay.bytes;
-    POS_CUDA(cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    POS_TRY(ensure_smem(reinterpret_cast<const void *>(kern), smem));
     kern<<<grid, 256, smem, s>>>(p);
     POS_CUDA(cudaGetLastError());
     return POS_OK;

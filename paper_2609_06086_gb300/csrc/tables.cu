@@ -3,6 +3,8 @@
 // Sec. 3.2 memory footprints).
 #include <algorithm>
 #include <cstring>
+#include <map>
+#include <mutex>
 #include <new>
 #include <string>
 #include <vector>
@@ -26,6 +28,19 @@ pos_status cuda_fail(cudaError_t e, const char *what) {
 }
 
 const char *last_error() { return g_last_error.c_str(); }
+
+pos_status ensure_smem(const void *kernel, int smem) {
+    static std::mutex mu;
+    static std::map<std::pair<int, const void *>, int> set;  // (device, kernel) -> limit
+    int dev = 0;
+    POS_CUDA(cudaGetDevice(&dev));
+    std::lock_guard<std::mutex> lock(mu);
+    int &cur = set[{dev, kernel}];
+    if (smem <= cur) return POS_OK;
+    POS_CUDA(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem));
+    cur = smem;
+    return POS_OK;
+}
 
 int sm_count() {
     int dev = 0, n = 0;
