@@ -28,6 +28,7 @@ namespace pos {
 constexpr int kThreads = 256;
 constexpr int32_t kNoCompletion = 0x7fffffff;  // completion-bound entry without a completion
 constexpr int kVbSlotsSmem = 64;  // batches up to this many slots stage their bound rows
+                                  // in shared memory; larger ones read them from L2
 
 // ---------------------------------------------------------------------------
 // suffix feasibility: one block per slice, thread c
@@ -116,11 +117,13 @@ __global__ void root_bits_kernel(const uint4 *feas, int n_slices, int S, uint8_t
 // keeps the smallest l attaining V1[x][c], and thread 0 follows it from
 // (0, 0) to write the slice's argmin completion as a plan: a memory-feasible
 // plan whose makespan is usually close to the slice's best (warm-up seed).
+// root_lb[slice] = V1[0][0] * scale, a lower bound on the slice's objective.
 constexpr int kBoundThreads = 512;
 
 __global__ void __launch_bounds__(kBoundThreads) bound_kernel(
     const SliceRec *slices, const uint32_t *rows, int n_rows, int S, const uint8_t *lim,
-    int2 *vb, Leaf *greedy, const void *blob, BlobLayout lay, unsigned long long *stats) {
+    int2 *vb, Leaf *greedy, unsigned long long *root_lb, const void *blob, BlobLayout lay,
+    unsigned long long *stats) {
     extern __shared__ __align__(16) unsigned char sm[];
     __shared__ int2 nxt[128];
     __shared__ uint8_t arg[POS_MAX_STAGES][128];
@@ -204,6 +207,9 @@ __global__ void __launch_bounds__(kBoundThreads) bound_kernel(
             }
             const Vec32 lf = {make_uint4(sl, cw[0], cw[1], cw[2]), make_uint4(cw[3], 0u, 0u, 0u)};
             store32(greedy + r, lf);
+            // the slice's root bound V1[0][0] = min over plans of max_y P(y, y),
+            // as an objective (orders the slices)
+            root_lb[sl] = (unsigned long long)nxt[0].x * sr.scale;
         }
         __syncthreads();
     }
@@ -820,7 +826,7 @@ struct Workspace {
     std::mutex mu;
     cudaStream_t stream = nullptr;
     cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
-    DevBuf blob, d_lim, d_vb, d_bctr, d_rows, d_greedy, d_wcnt, d_slices, d_feas, d_batch, d_inc, d_ctr, d_best, d_feasible, d_leaves, d_roots,
+    DevBuf blob, d_lim, d_vb, d_bctr, d_rows, d_greedy, d_wcnt, d_lb, d_slices, d_feas, d_batch, d_inc, d_ctr, d_best, d_feasible, d_leaves, d_roots,
         d_root;
     DevBuf d_front[POS_MAX_STAGES + 1];        // per depth: Prefix buffers
     DevBuf d_defer[2 * (POS_MAX_STAGES + 1)];  // per depth: two deferred group lists
@@ -1255,6 +1261,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         POS_CUDA(s.ws.d_rows.reserve(sizeof(uint32_t) * rows.size()));
         POS_CUDA(s.ws.d_vb.reserve(sizeof(int2) * 128 * (size_t)s.S * rows.size()));
         POS_CUDA(s.ws.d_greedy.reserve(sizeof(Leaf) * rows.size()));
+        POS_CUDA(s.ws.d_lb.reserve(sizeof(unsigned long long) * n_slices));
         POS_CUDA(cudaMemcpyAsync(s.ws.d_rows.p, rows.data(), sizeof(uint32_t) * rows.size(),
                                  cudaMemcpyHostToDevice, s.stream));
         POS_CUDA(cudaMemcpyAsync(s.d_slices.p, s.slices.data(), sizeof(SliceRec) * n_slices,
@@ -1266,7 +1273,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
                        s.stream>>>(
             d_all, static_cast<const uint32_t *>(s.ws.d_rows.p), (int)rows.size(), s.S,
             static_cast<const uint8_t *>(s.ws.d_lim.p), static_cast<int2 *>(s.ws.d_vb.p),
-            static_cast<Leaf *>(s.ws.d_greedy.p),
+            static_cast<Leaf *>(s.ws.d_greedy.p), static_cast<unsigned long long *>(s.ws.d_lb.p),
             static_cast<const unsigned char *>(s.h->d_blob) + s.h->lay.off_Pf, tl, s.stats);
         POS_CUDA(cudaGetLastError());
         if (p->profile) POS_CUDA(cudaEventRecord(s.ev[1], s.stream));
@@ -1335,12 +1342,20 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         unsigned long long best;
     };
     std::vector<Group> groups;
+    // slice order: with the completion bounds, by each slice's root lower
+    // bound (the slice most likely to hold the optimum first); otherwise by
+    // the best warm-up plan of the slice
+    std::vector<unsigned long long> key = best;
+    if (p->prune == 2 && n_feasible > 0 &&
+        (st = sync_read(s, key.data(), s.ws.d_lb.p, sizeof(unsigned long long) * n_slices)) !=
+            POS_OK)
+        return st;
     for (int mi = 0; mi < p->n_M; ++mi) {
         if (feas_by_m[mi].empty()) continue;
         auto &fl = feas_by_m[mi];
         std::stable_sort(fl.begin(), fl.end(),
-                         [&](uint32_t a, uint32_t b) { return best[a] < best[b]; });
-        groups.push_back({mi, best[fl[0]]});
+                         [&](uint32_t a, uint32_t b) { return key[a] < key[b]; });
+        groups.push_back({mi, key[fl[0]]});
     }
     std::stable_sort(groups.begin(), groups.end(),
                      [](const Group &a, const Group &b) { return a.best < b.best; });
@@ -1354,13 +1369,22 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     size_t max_nb = 1;
     for (const Group &g : groups) {
         const auto &fl = feas_by_m[g.mi];
-        size_t bsz = std::min<size_t>(65535, std::max<size_t>(32, (fl.size() + 7) / 8));
-        if (p->prune == 2) bsz = std::min<size_t>(bsz, kVbSlotsSmem);
-        for (size_t b0 = 0; b0 < fl.size(); b0 += bsz) {
-            const size_t nb = std::min(bsz, fl.size() - b0);
+        // Eq. 2 alone: eight batches, best first, so that the incumbent
+        // improves between them.  With the completion bounds the warm-up
+        // already holds each slice's argmin completion and every launch
+        // costs more than a little extra pruning saves: a first batch of
+        // the 1/16 of the slices with the smallest root bounds (most likely
+        // to hold the optimum), then the rest in one batch.
+        const size_t bsz = p->prune == 2
+                               ? std::min<size_t>(65535, fl.size())
+                               : std::min<size_t>(65535, std::max<size_t>(32, (fl.size() + 7) / 8));
+        const size_t first = p->prune == 2 ? (fl.size() + 15) / 16 : bsz;
+        for (size_t b0 = 0; b0 < fl.size();) {
+            const size_t nb = std::min(b0 == 0 ? first : bsz, fl.size() - b0);
             batches.push_back({p->M_list[g.mi], ordered.size(), nb});
             for (size_t j = 0; j < nb; ++j) ordered.push_back(s.slices[fl[b0 + j]]);
             max_nb = std::max(max_nb, nb);
+            b0 += nb;
         }
     }
     POS_CUDA(s.d_batch.reserve(sizeof(SliceRec) * std::max<size_t>(1, ordered.size())));
@@ -1442,7 +1466,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
                 ep.deferred = static_cast<uint32_t *>(s.d_defer[2 * x].p);
                 ep.n_deferred = bc + 2 * x + 1;
                 ep.nb = (int)b.nb;
-                ep.vb_smem = p->prune == 2 && !last;
+                ep.vb_smem = p->prune == 2 && !last && b.nb <= kVbSlotsSmem;
                 const int smem_l = ep.lay.bytes + (ep.vb_smem ? (int)b.nb * 128 * 8 : 0);
                 const int grid = x == 0 ? (int)std::max<long long>(
                                               1, std::min<long long>(((long long)b.nb + 255) / 256,
