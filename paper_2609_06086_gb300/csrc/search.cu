@@ -30,6 +30,25 @@ constexpr int32_t kNoCompletion = 0x7fffffff;  // completion-bound entry without
 constexpr int kVbSlotsSmem = 64;  // batches up to this many slots stage their bound rows
                                   // in shared memory; larger ones read them from L2
 
+// 128-bit set of cut positions 0..127.
+struct Bits128 {
+    uint32_t w[4];
+};
+
+__device__ __forceinline__ Bits128 range_bits(int lo, int hi) {  // positions lo..hi
+    Bits128 r;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int a = max(lo - 32 * i, 0), b = min(hi - 32 * i, 31);
+        r.w[i] = (a > b) ? 0u : ((b == 31 ? 0xffffffffu : ((1u << (b + 1)) - 1u)) & ~((1u << a) - 1u));
+    }
+    return r;
+}
+
+__device__ __forceinline__ int popc128(const Bits128 &b) {
+    return __popc(b.w[0]) + __popc(b.w[1]) + __popc(b.w[2]) + __popc(b.w[3]);
+}
+
 // ---------------------------------------------------------------------------
 // suffix feasibility: one block per slice, thread c
 // ---------------------------------------------------------------------------
@@ -59,13 +78,19 @@ __global__ void feas_kernel(const SliceRec *slices, int n_slices, int S, uint4 *
             bool ok = false;
             int most = 0;
             if (c < L) {
+                // memory grows with the layer count: binary search for the
+                // largest l that fits, then any suffix start in (c, c+l]
                 const int k = sr.cls[x];
-                for (int l = 1; c + l <= L; ++l) {
-                    if (!stage_fits(t, S, M, x, k, c, c + l)) break;
-                    most = l;
-                    const int e = c + l;
-                    if ((prev[e >> 5] >> (e & 31)) & 1u) ok = true;
+                int lo = 0, hi = L - c;
+                while (lo < hi) {
+                    const int mid = (lo + hi + 1) >> 1;
+                    if (stage_fits(t, S, M, x, k, c, c + mid)) lo = mid;
+                    else hi = mid - 1;
                 }
+                most = lo;
+                const Bits128 win = range_bits(c + 1, c + most);
+                ok = ((prev[0] & win.w[0]) | (prev[1] & win.w[1]) | (prev[2] & win.w[2]) |
+                      (prev[3] & win.w[3])) != 0u;
             }
             if (c < 128) lim[((size_t)sr.gid * S + x) * 128 + c] = (uint8_t)most;
             const unsigned b = __ballot_sync(0xffffffffu, ok);
@@ -226,24 +251,6 @@ __device__ __forceinline__ uint64_t splitmix64_next(uint64_t &s) {
     return z ^ (z >> 31);
 }
 
-// 128-bit set of cut positions 0..127.
-struct Bits128 {
-    uint32_t w[4];
-};
-
-__device__ __forceinline__ Bits128 range_bits(int lo, int hi) {  // positions lo..hi
-    Bits128 r;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const int a = max(lo - 32 * i, 0), b = min(hi - 32 * i, 31);
-        r.w[i] = (a > b) ? 0u : ((b == 31 ? 0xffffffffu : ((1u << (b + 1)) - 1u)) & ~((1u << a) - 1u));
-    }
-    return r;
-}
-
-__device__ __forceinline__ int popc128(const Bits128 &b) {
-    return __popc(b.w[0]) + __popc(b.w[1]) + __popc(b.w[2]) + __popc(b.w[3]);
-}
 
 // Position of the r-th (0-based) set bit of a 128-bit set with more than r
 // set bits.
@@ -831,6 +838,10 @@ struct Workspace {
     DevBuf d_front[POS_MAX_STAGES + 1];        // per depth: Prefix buffers
     DevBuf d_defer[2 * (POS_MAX_STAGES + 1)];  // per depth: two deferred group lists
     unsigned long long *h_cnt = nullptr;       // pinned host counters
+    unsigned char *h_stage = nullptr;          // pinned staging area for uploads
+    size_t h_stage_cap = 0;
+    unsigned char *h_read = nullptr;           // pinned landing area for reads
+    size_t h_read_cap = 0;
     std::vector<cudaEvent_t> evs;              // timing events of the batch pipelines
 };
 
@@ -874,7 +885,7 @@ struct Search {
     uint64_t n_map = 0, n_place = 0;
     long long cap = 0;
     int grid_level = 0, grid_leaf = 0;
-    std::vector<std::vector<int>> places;
+    std::vector<uint8_t> places;  // n_place x S stage types, placement-rank order
     std::vector<SliceRec> slices;
     DevBuf &d_slices, &d_feas, &d_batch, &d_inc, &d_ctr, &d_best, &d_feasible, &d_leaves,
         &d_roots, &d_root;
@@ -886,6 +897,7 @@ struct Search {
     double ms_expand = 0, ms_complete = 0, ms_leaf = 0, ms_bound = 0;
     uint64_t n_expand = 0, n_complete = 0, n_leaf = 0, n_bound = 0, reruns = 0;
     int cur_nb = 0;    // slots of the batch being enumerated
+    size_t stage_off = 0;  // bytes of the staging area used by this search
     int n_vrows = 0;   // rows of the completion-bound tables (memory-feasible slices)
 };
 
@@ -921,27 +933,30 @@ static pos_status validate_problem(const pos_problem *p) {
 static pos_status enumerate_places(Search &s) {
     const pos_problem *p = s.pb;
     const int S = p->S, T = p->tables.n_types;
-    std::vector<int> seq(S, 0);
     const uint64_t limit = 1ull << 22;
-    for (;;) {
-        bool ok = true;
-        if (p->placement == POS_PLACE_EXACT) {
-            for (int ty = 0; ty < T && ok; ++ty) {
-                int cnt = 0;
-                for (int x = 0; x < S; ++x) cnt += seq[x] == ty;
-                ok = cnt == p->type_counts[ty];
-            }
+    std::vector<uint8_t> seq;
+    if (p->placement == POS_PLACE_EXACT) {
+        // the distinct permutations of the multiset, in lexicographic order
+        for (int ty = 0; ty < T; ++ty) seq.insert(seq.end(), p->type_counts[ty], (uint8_t)ty);
+        do {
+            s.places.insert(s.places.end(), seq.begin(), seq.end());
+            if (s.places.size() > limit * S) return fail(POS_EINVAL, "too many placements");
+        } while (std::next_permutation(seq.begin(), seq.end()));
+    } else {
+        // every sequence in T^S, as an odometer (last stage fastest)
+        double total = 1;
+        for (int x = 0; x < S; ++x) total *= T;
+        if (total > (double)limit) return fail(POS_EINVAL, "too many placements");
+        seq.assign(S, 0);
+        for (;;) {
+            s.places.insert(s.places.end(), seq.begin(), seq.end());
+            int x = S - 1;
+            while (x >= 0 && seq[x] == T - 1) seq[x--] = 0;
+            if (x < 0) break;
+            seq[x]++;
         }
-        if (ok) {
-            s.places.push_back(seq);
-            if (s.places.size() > limit) return fail(POS_EINVAL, "too many placements");
-        }
-        int x = S - 1;
-        while (x >= 0 && seq[x] == T - 1) seq[x--] = 0;
-        if (x < 0) break;
-        seq[x]++;
     }
-    s.n_place = s.places.size();
+    s.n_place = s.places.size() / S;
     return POS_OK;
 }
 
@@ -975,8 +990,44 @@ static pos_status sync_read(Search &s, void *dst, const void *src, size_t bytes)
         std::memcpy(dst, s.ws.h_cnt, bytes);
         return POS_OK;
     }
-    POS_CUDA(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToHost, s.stream));
+    if (bytes > s.ws.h_read_cap) {  // no copy is in flight: the old area can go
+        if (s.ws.h_read) cudaFreeHost(s.ws.h_read);
+        s.ws.h_read = nullptr;
+        s.ws.h_read_cap = 0;
+        POS_CUDA(cudaMallocHost(&s.ws.h_read, bytes + bytes / 2));
+        s.ws.h_read_cap = bytes + bytes / 2;
+    }
+    POS_CUDA(cudaMemcpyAsync(s.ws.h_read, src, bytes, cudaMemcpyDeviceToHost, s.stream));
     POS_CUDA(cudaStreamSynchronize(s.stream));
+    std::memcpy(dst, s.ws.h_read, bytes);
+    return POS_OK;
+}
+
+// Enqueues an upload through the workspace's pinned staging area (an
+// upload straight from pageable memory makes the host wait while the
+// driver stages it).  The area is sized at the start of a search and only
+// reused after that search has synchronised; if it is full the copy goes
+// from pageable memory.
+static pos_status upload(Search &s, void *dst, const void *src, size_t bytes) {
+    const size_t off = (s.stage_off + 255) & ~(size_t)255;
+    if (off + bytes > s.ws.h_stage_cap) {
+        POS_CUDA(cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, s.stream));
+        return POS_OK;
+    }
+    std::memcpy(s.ws.h_stage + off, src, bytes);
+    POS_CUDA(cudaMemcpyAsync(dst, s.ws.h_stage + off, bytes, cudaMemcpyHostToDevice, s.stream));
+    s.stage_off = off + bytes;
+    return POS_OK;
+}
+
+static pos_status reserve_stage(Search &s, size_t bytes) {
+    s.stage_off = 0;
+    if (bytes <= s.ws.h_stage_cap) return POS_OK;
+    if (s.ws.h_stage) cudaFreeHost(s.ws.h_stage);  // the previous search has synchronised
+    s.ws.h_stage = nullptr;
+    s.ws.h_stage_cap = 0;
+    POS_CUDA(cudaMallocHost(&s.ws.h_stage, bytes));
+    s.ws.h_stage_cap = bytes;
     return POS_OK;
 }
 
@@ -1145,17 +1196,6 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     const pos_problem *p = s.pb;
     pos_status st = validate_problem(p);
     if (st != POS_OK) return st;
-    {
-        std::vector<unsigned char> host;
-        st = build_blob(&p->tables, host, s.hd.lay, s.hd.guard_A, s.hd.guard_D, s.hd.guard_P);
-        if (st != POS_OK) return st;
-        POS_CUDA(cudaGetDevice(&s.hd.device));
-        POS_CUDA(s.ws.blob.reserve(s.hd.lay.bytes));
-        s.hd.d_blob = s.ws.blob.p;
-        POS_CUDA(cudaMemcpyAsync(s.hd.d_blob, host.data(), s.hd.lay.bytes, cudaMemcpyHostToDevice,
-                                 s.stream));
-        if ((st = launch_prefix_rows(s.hd.d_blob, s.hd.lay, s.stream)) != POS_OK) return st;
-    }
     s.S = p->S;
     s.L = p->tables.L;
     s.n_tp = p->tables.n_tp;
@@ -1170,6 +1210,20 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     if (n_slices64 > (1ull << 22)) return fail(POS_EINVAL, "more than 2^22 slices");
     const int n_slices = (int)n_slices64;
     if (s.n_map && n_slices64 > ~0ull / s.n_map) return fail(POS_EINVAL, "global index overflows");
+    // pinned staging for this search's uploads (tables, slice records, lists)
+    if ((st = reserve_stage(s, ((size_t)256 << 10) + (size_t)n_slices * 320 +
+                                   (size_t)p->n_M * 16)) != POS_OK)
+        return st;
+    {
+        std::vector<unsigned char> host;
+        st = build_blob(&p->tables, host, s.hd.lay, s.hd.guard_A, s.hd.guard_D, s.hd.guard_P);
+        if (st != POS_OK) return st;
+        POS_CUDA(cudaGetDevice(&s.hd.device));
+        POS_CUDA(s.ws.blob.reserve(s.hd.lay.bytes));
+        s.hd.d_blob = s.ws.blob.p;
+        POS_TRY(upload(s, s.hd.d_blob, host.data(), s.hd.lay.bytes));
+        if ((st = launch_prefix_rows(s.hd.d_blob, s.hd.lay, s.stream)) != POS_OK) return st;
+    }
     // overflow guard for every M (Sec. 4.1 path-length bound)
     for (int i = 0; i < p->n_M; ++i)
         if (guard_trips(s.h->guard_A, s.h->guard_D, s.h->guard_P, s.S, p->M_list[i]))
@@ -1193,7 +1247,8 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
                 r.M = p->M_list[mi];
                 r.scale = Q / ((uint64_t)p->dp_list[tp] * p->M_list[mi]);
                 r.gid = (uint32_t)ord;
-                for (int x = 0; x < s.S; ++x) r.cls[x] = (uint8_t)(s.places[pr][x] * s.n_tp + tp);
+                for (int x = 0; x < s.S; ++x)
+                    r.cls[x] = (uint8_t)(s.places[pr * s.S + x] * s.n_tp + tp);
             }
     const int smem = s.h->lay.bytes;
     int per_sm = 0;
@@ -1214,13 +1269,12 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     POS_CUDA(s.d_leaves.reserve(sizeof(Leaf) * (size_t)s.cap));
     s.ctr = static_cast<unsigned long long *>(s.d_ctr.p);
     s.stats = s.ctr + 40;  // ctr[0..33]: per-depth counters, ctr[36]: leaf count
-    POS_CUDA(cudaMemcpyAsync(s.d_slices.p, s.slices.data(), sizeof(SliceRec) * n_slices,
-                             cudaMemcpyHostToDevice, s.stream));
+    POS_TRY(upload(s, s.d_slices.p, s.slices.data(), sizeof(SliceRec) * n_slices));
     POS_CUDA(cudaMemsetAsync(s.d_inc.p, 0xff, sizeof(Key128), s.stream));
     POS_CUDA(cudaMemsetAsync(s.d_ctr.p, 0, sizeof(unsigned long long) * 64, s.stream));
     POS_CUDA(cudaMemsetAsync(s.d_best.p, 0xff, sizeof(unsigned long long) * n_slices, s.stream));
     const SliceRec *d_all = static_cast<const SliceRec *>(s.d_slices.p);
-    feas_kernel<<<std::min(n_slices, 16 * sm_count()), 128, smem, s.stream>>>(
+    feas_kernel<<<std::min(n_slices, 2 * sm_count()), 128, smem, s.stream>>>(
         d_all, n_slices, s.S, static_cast<uint4 *>(s.d_feas.p),
         static_cast<uint8_t *>(s.ws.d_lim.p), s.h->d_blob, s.h->lay, s.stats);
     POS_CUDA(cudaGetLastError());
@@ -1262,10 +1316,8 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         POS_CUDA(s.ws.d_vb.reserve(sizeof(int2) * 128 * (size_t)s.S * rows.size()));
         POS_CUDA(s.ws.d_greedy.reserve(sizeof(Leaf) * rows.size()));
         POS_CUDA(s.ws.d_lb.reserve(sizeof(unsigned long long) * n_slices));
-        POS_CUDA(cudaMemcpyAsync(s.ws.d_rows.p, rows.data(), sizeof(uint32_t) * rows.size(),
-                                 cudaMemcpyHostToDevice, s.stream));
-        POS_CUDA(cudaMemcpyAsync(s.d_slices.p, s.slices.data(), sizeof(SliceRec) * n_slices,
-                                 cudaMemcpyHostToDevice, s.stream));
+        POS_TRY(upload(s, s.ws.d_rows.p, rows.data(), sizeof(uint32_t) * rows.size()));
+        POS_TRY(upload(s, s.d_slices.p, s.slices.data(), sizeof(SliceRec) * n_slices));
         const BlobLayout tl = timing_layout(s.h->lay);
         POS_TRY(ensure_smem(reinterpret_cast<const void *>(bound_kernel), tl.bytes));
         if (p->profile) POS_CUDA(cudaEventRecord(s.ev[0], s.stream));
@@ -1283,8 +1335,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         std::vector<unsigned long long> gc(p->n_M);
         for (int mi = 0; mi < p->n_M; ++mi) gc[mi] = feas_by_m[mi].size();
         POS_CUDA(s.ws.d_wcnt.reserve(sizeof(unsigned long long) * p->n_M));
-        POS_CUDA(cudaMemcpyAsync(s.ws.d_wcnt.p, gc.data(), sizeof(unsigned long long) * p->n_M,
-                                 cudaMemcpyHostToDevice, s.stream));
+        POS_TRY(upload(s, s.ws.d_wcnt.p, gc.data(), sizeof(unsigned long long) * p->n_M));
         for (int mi = 0; mi < p->n_M; ++mi) {
             if (gc[mi] == 0) continue;
             if ((st = run_leaves(s, static_cast<const Leaf *>(s.ws.d_greedy.p) + feas_off[mi],
@@ -1305,8 +1356,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
             const long long n_s = std::min<long long>(
                 s.cap, std::max<long long>(1, (long long)p->warmup * (long long)fl.size() /
                                                   (long long)n_feasible));
-            POS_CUDA(cudaMemcpyAsync(s.d_feasible.p, fl.data(), sizeof(uint32_t) * fl.size(),
-                                     cudaMemcpyHostToDevice, s.stream));
+            POS_TRY(upload(s, s.d_feasible.p, fl.data(), sizeof(uint32_t) * fl.size()));
             sample_kernel<<<(int)std::min<long long>((n_s + 255) / 256, 4 * sm_count()), 256, 0,
                             s.stream>>>(
                 d_all, static_cast<const uint32_t *>(s.d_feasible.p), (int)fl.size(), (int)n_s,
@@ -1315,8 +1365,8 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
                 static_cast<Leaf *>(s.d_leaves.p), s.L);
             POS_CUDA(cudaGetLastError());
             s.launches++;
-            unsigned long long cnt = (unsigned long long)n_s;
-            POS_CUDA(cudaMemcpyAsync(s.ctr + 36, &cnt, 8, cudaMemcpyHostToDevice, s.stream));
+            const unsigned long long cnt = (unsigned long long)n_s;
+            POS_TRY(upload(s, s.ctr + 36, &cnt, 8));
             if ((st = run_leaves(s, static_cast<const Leaf *>(s.d_leaves.p), s.ctr + 36, d_all,
                                  p->M_list[mi], static_cast<unsigned long long *>(s.d_best.p))) !=
                 POS_OK)
@@ -1389,8 +1439,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     }
     POS_CUDA(s.d_batch.reserve(sizeof(SliceRec) * std::max<size_t>(1, ordered.size())));
     if (!ordered.empty())
-        POS_CUDA(cudaMemcpyAsync(s.d_batch.p, ordered.data(), sizeof(SliceRec) * ordered.size(),
-                                 cudaMemcpyHostToDevice, s.stream));
+        POS_TRY(upload(s, s.d_batch.p, ordered.data(), sizeof(SliceRec) * ordered.size()));
     // roots: slot j of a batch, no stage placed (the first nb serve a batch of nb)
     std::vector<Prefix> roots(max_nb);
     for (size_t j = 0; j < max_nb; ++j) {
@@ -1400,8 +1449,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         roots[j].Bm = -1;
     }
     POS_CUDA(s.d_roots.reserve(sizeof(Prefix) * max_nb));
-    POS_CUDA(cudaMemcpyAsync(s.d_roots.p, roots.data(), sizeof(Prefix) * max_nb,
-                             cudaMemcpyHostToDevice, s.stream));
+    POS_TRY(upload(s, s.d_roots.p, roots.data(), sizeof(Prefix) * max_nb));
     const SliceRec *d_ordered = static_cast<const SliceRec *>(s.d_batch.p);
     const Prefix *d_rootp = static_cast<const Prefix *>(s.d_roots.p);
 
@@ -1413,10 +1461,9 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
                 std::memset(&lv[j], 0, sizeof(Leaf));
                 lv[j].slice = (uint32_t)j;
             }
-            POS_CUDA(cudaMemcpyAsync(s.d_leaves.p, lv.data(), sizeof(Leaf) * b.nb,
-                                     cudaMemcpyHostToDevice, s.stream));
-            unsigned long long cnt = b.nb;
-            POS_CUDA(cudaMemcpyAsync(s.ctr + 36, &cnt, 8, cudaMemcpyHostToDevice, s.stream));
+            POS_TRY(upload(s, s.d_leaves.p, lv.data(), sizeof(Leaf) * b.nb));
+            const unsigned long long cnt = b.nb;
+            POS_TRY(upload(s, s.ctr + 36, &cnt, 8));
             if ((st = run_leaves(s, static_cast<const Leaf *>(s.d_leaves.p), s.ctr + 36,
                                  d_ordered + b.off, b.M, nullptr)) != POS_OK)
                 return st;
@@ -1566,7 +1613,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     out->makespan = (int32_t)(inc.obj / sr.scale);
     out->global_index = inc.idx;
     for (int x = 0; x < POS_MAX_STAGES; ++x) {
-        out->type[x] = x < s.S ? s.places[out->place_rank][x] : -1;
+        out->type[x] = x < s.S ? s.places[out->place_rank * s.S + x] : -1;
         out->layers[x] = 0;
     }
     host_unrank(s.L, s.S, out->map_rank, out->layers);
