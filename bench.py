@@ -35,6 +35,14 @@ METRIC = "DAG makespan evals/sec (time-to-optimal plan at L=80, S=8)"
 WARMUP_SAMPLES = 65536
 SM_LANES = 128  # INT32 lanes per SM (4 partitions x 32)
 ENTRY_BYTES = 32  # one frontier entry / one complete plan
+# DRAM bytes per evaluated plan of leaf_kernel, from one ncu capture of
+# dram__bytes_read.sum + dram__bytes_write.sum over a config-4 search's leaf
+# launches (profiles/leaf_kernel_config4.md), valid while the kernel's
+# sources hash to LEAF_SOURCES_SHA256 (else the traffic is reported as null)
+LEAF_DRAM_BYTES_PER_PLAN = 59685376 / 1925970
+LEAF_SOURCES = ("paper_2609_06086_gb300/csrc/search_kernels.cuh",
+                "paper_2609_06086_gb300/csrc/common.cuh")
+LEAF_SOURCES_SHA256 = "9add3f061939606b"
 PRUNE_NAMES = {1: "stage-level, Eq. 2 as printed (Theorem 1)",
                2: "stage-level, tightened: Eq. 2 with P2P edges + completion bounds"}
 
@@ -45,6 +53,15 @@ def measured_hbm():
         return float(json.load(open(path))["hbm_gbs"]), "measured copy bandwidth (MEASURED_PEAKS.json)"
     except (OSError, KeyError, ValueError):
         return 6800.0, "fallback 6.8 TB/s (MEASURED_PEAKS.json absent)"
+
+
+def leaf_sources_unchanged() -> bool:
+    import hashlib
+    h = hashlib.sha256()
+    for f in LEAF_SOURCES:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16] == LEAF_SOURCES_SHA256
 
 
 def dist_env():
@@ -206,7 +223,7 @@ def run_ours(args, rank, world, local_rank):
     clocks = Clocks(torch.cuda.current_device()) if rank == 0 else None
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     dev_ms, wall_ms, plans = [], [], []
-    agg = dict(evaluated=0, relaxations=0, launches=0, ms_expand=0.0, ms_complete=0.0,
+    agg = dict(evaluated=0, warmup_evaluated=0, relaxations=0, launches=0, ms_expand=0.0, ms_complete=0.0,
                ms_leaf=0.0, expand_launches=0, complete_launches=0, leaf_launches=0,
                parents_expand=0, parents_complete=0, leaves=0, prefixes=0,
                ms_setup=0.0, ms_warmup=0.0, ms_search=0.0)
@@ -228,6 +245,8 @@ def run_ours(args, rank, world, local_rank):
     # around every launch on the library's stream (profile=1)
     prof_ms = []
     kagg = {k: 0 for k in agg}
+    for k in ("ms_depth", "launches_depth", "parents_depth", "children_depth"):
+        kagg[k] = [0] * 16
     for _ in range(args.steps):
         flush.zero_()
         torch.cuda.synchronize()
@@ -237,7 +256,10 @@ def run_ours(args, rank, world, local_rank):
         torch.cuda.synchronize()
         prof_ms.append(ev0.elapsed_time(ev1))
         for k in kagg:
-            kagg[k] += st_p[k]
+            if isinstance(kagg[k], list):
+                kagg[k] = [u + v for u, v in zip(kagg[k], st_p[k])]
+            else:
+                kagg[k] += st_p[k]
     t_dev = sum(dev_ms)
     if dist:
         tt = torch.tensor([t_dev], dtype=torch.float64,
@@ -258,27 +280,32 @@ def run_ours(args, rank, world, local_rank):
     e2e = evals / (sum(wall_ms) / 1e3)
     props = torch.cuda.get_device_properties(torch.cuda.current_device())
     n_sm = props.multi_processor_count
-    # roofline of the dominant kernel kind (device time from events on the
-    # library's stream, accumulated over the timed steps)
-    kinds = {"leaf": kagg["ms_leaf"], "expand": kagg["ms_expand"],
-             "complete": kagg["ms_complete"]}
-    dom = max(kinds, key=kinds.get)
+    # Per kernel (device time from CUDA events around every launch on the
+    # library's stream, profiled steps): the leaf kernel (makespans of the
+    # complete plans) and the level kernel of each parent depth x (x = S-2
+    # completes the last two stages).  Algorithmic work (roofline
+    # section):
+    #  leaf    : int32 ops, 3 per DAG node relaxation + 9 per stage
+    #  level x : bytes, a 32-byte frontier entry read per parent and a 32-byte
+    #            child (or complete plan) written per child
     mhz = (clk or {}).get("sm_mhz") or 2070.0
     peak_alu = n_sm * SM_LANES * mhz * 1e6 / 1e12  # Tops/s at the measured SM clock
     peak_hbm, hbm_src = measured_hbm()
     S = w.S
-    launches = {"leaf": kagg["leaf_launches"], "expand": kagg["expand_launches"],
-                "complete": kagg["complete_launches"]}
-    # algorithmic work per kind (roofline section):
-    #  leaf     : int32 ops, 3 per DAG node relaxation + 9 per stage
-    #  expand   : bytes, a 32-byte frontier entry read per parent and written per child
-    #  complete : bytes, a 32-byte entry read per parent and a 32-byte plan written per leaf
-    work = {"leaf": 3 * kagg["relaxations"] + 9 * S * kagg["evaluated"],
-            "expand": ENTRY_BYTES * (kagg["parents_expand"] + kagg["prefixes"]),
-            "complete": ENTRY_BYTES * (kagg["parents_complete"] + kagg["leaves"])}
-    bound = {"leaf": ("alu", "Tops/s", peak_alu, 1e12),
-             "expand": ("hbm", "GB/s", peak_hbm, 1e9),
-             "complete": ("hbm", "GB/s", peak_hbm, 1e9)}
+    kinds, launches, work, bound = {}, {}, {}, {}
+    kinds["leaf_kernel"] = kagg["ms_leaf"]
+    launches["leaf_kernel"] = kagg["leaf_launches"]
+    # the timed leaf launches are the search's (the warm-up's are not in ms_leaf)
+    leaf_plans = kagg["evaluated"] - kagg["warmup_evaluated"]
+    work["leaf_kernel"] = (3 * 2 * S * w.M_list[0] + 9 * S) * leaf_plans
+    bound["leaf_kernel"] = ("alu", "Tops/s", peak_alu, 1e12)
+    for x in range(S - 1):
+        name = f"level_kernel<{'complete' if x == S - 2 else 'expand'}, depth {x}>"
+        kinds[name] = kagg["ms_depth"][x]
+        launches[name] = kagg["launches_depth"][x]
+        work[name] = ENTRY_BYTES * (kagg["parents_depth"][x] + kagg["children_depth"][x])
+        bound[name] = ("hbm", "GB/s", peak_hbm, 1e9)
+    dom = max(kinds, key=kinds.get)
     per_kind = {}
     for k in kinds:
         b, unit, peak, scale = bound[k]
@@ -287,9 +314,15 @@ def run_ours(args, rank, world, local_rank):
                        "launches_per_step": launches[k] / args.steps, "bound": b,
                        "achieved": round(ach, 3), "unit": unit, "frac": round(ach / peak, 4)}
     b, unit, peak, scale = bound[dom]
+    traffic = None
+    if dom == "leaf_kernel" and leaf_sources_unchanged():
+        traffic = round(LEAF_DRAM_BYTES_PER_PLAN * leaf_plans / max(1, launches[dom]))
     roof = {"bound": b, "kernel": dom, "unit": unit, "peak": round(peak, 3),
             "achieved": per_kind[dom]["achieved"], "frac": per_kind[dom]["frac"],
-            "work_per_launch": work[dom] / max(1, launches[dom]), "traffic": None,
+            "work_per_launch": work[dom] / max(1, launches[dom]), "traffic": traffic,
+            "traffic_note": ("DRAM bytes per launch: ncu dram__bytes_read.sum + "
+                             "dram__bytes_write.sum per plan (profiles/leaf_kernel_config4.md) "
+                             "x plans per launch" if traffic is not None else None),
             "peak_note": (f"{n_sm} SMs x {SM_LANES} int32 lanes x {mhz:.0f} MHz (median SM "
                           "clock under load)" if b == "alu" else hbm_src)}
     evals = [eval_throughput(P, torch, int(n), 5, peak_alu) for n in args.eval_sizes]

@@ -248,6 +248,13 @@ typedef struct pos_search_stats {
     /* batches of slices run a second time, host-driven, because a frontier
        of their pipelined pass overflowed frontier_cap */
     uint64_t reruns;
+    /* per parent depth x (stages 0..x-1 placed; x = S-2 is the completion):
+       device time of its level kernels (profile only), their launches, the
+       frontier entries they read and the children (plans) they wrote */
+    double ms_depth[POS_MAX_STAGES];
+    uint64_t launches_depth[POS_MAX_STAGES];
+    uint64_t parents_depth[POS_MAX_STAGES];
+    uint64_t children_depth[POS_MAX_STAGES];
 } pos_search_stats;
 
 /*

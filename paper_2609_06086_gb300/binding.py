@@ -61,7 +61,9 @@ class pos_search_stats(C.Structure):
                [(n, C.c_uint64) for n in ("expand_launches", "complete_launches",
                                           "leaf_launches", "parents_expand", "parents_complete",
                                           "leaves")] + \
-               [("ms_bound", C.c_double), ("bound_launches", C.c_uint64), ("reruns", C.c_uint64)]
+               [("ms_bound", C.c_double), ("bound_launches", C.c_uint64), ("reruns", C.c_uint64),
+                ("ms_depth", C.c_double * 16), ("launches_depth", C.c_uint64 * 16),
+                ("parents_depth", C.c_uint64 * 16), ("children_depth", C.c_uint64 * 16)]
 
 
 class PoseidonError(RuntimeError):
@@ -208,5 +210,6 @@ def poseidon_search(problem: pos_problem):
                tp=plan.tp, D=plan.D, T=plan.makespan, place_rank=plan.place_rank,
                map_rank=plan.map_rank, global_index=plan.global_index,
                types=list(plan.type)[:S], layers=list(plan.layers)[:S])
-    stats = {n: getattr(st, n) for n, _ in pos_search_stats._fields_}
+    stats = {n: (list(getattr(st, n)) if n.endswith("_depth") else getattr(st, n))
+             for n, _ in pos_search_stats._fields_}
     return out, stats

@@ -60,6 +60,9 @@ BlobLayout make_layout(int L, int n_types, int n_tp);
 // rebased to start at byte 0, for kernels that read nothing else; the
 // timing part starts at byte ly.off_Pf of the full blob.
 BlobLayout timing_layout(const BlobLayout &ly);
+// The memory part (Pw, Pa, cap: the three tables after the binomials),
+// rebased likewise; it starts at byte ly.off_Pw of the full blob.
+BlobLayout memory_layout(const BlobLayout &ly);
 
 struct Handle {
     int device;

@@ -789,8 +789,11 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
         if (emitted) atomicAdd(p.stats + (COMPLETE ? kStLeaves : kStPrefixes), emitted);
         if (cb) atomicAdd(p.stats + kStPrunedBound, cb);
         if (cm) atomicAdd(p.stats + kStPrunedMemory, cm);
-        if (written_parents)
+        if (written_parents) {
             atomicAdd(p.stats + (COMPLETE ? kStParentsComplete : kStParentsExpand), written_parents);
+            atomicAdd(p.stats + kStDepthParents + X, written_parents);
+        }
+        if (emitted) atomicAdd(p.stats + kStDepthChildren + X, emitted);
     }
 }
 
@@ -895,6 +898,8 @@ struct Search {
     unsigned long long *stats = nullptr;
     uint64_t launches = 0;
     double ms_expand = 0, ms_complete = 0, ms_leaf = 0, ms_bound = 0;
+    double ms_depth[POS_MAX_STAGES] = {};
+    uint64_t launches_depth[POS_MAX_STAGES] = {};
     uint64_t n_expand = 0, n_complete = 0, n_leaf = 0, n_bound = 0, reruns = 0;
     int cur_nb = 0;    // slots of the batch being enumerated
     size_t stage_off = 0;  // bytes of the staging area used by this search
@@ -1147,6 +1152,7 @@ static pos_status process(Search &s, const SliceRec *batch, int M, int x, const 
         if (prof) POS_CUDA(cudaEventRecord(s.ev[0], s.stream));
         if ((st = launch_level(last, x, p, grid, smem, s.stream)) != POS_OK) return st;
         (last ? s.n_complete : s.n_expand)++;
+        s.launches_depth[x]++;
         if (prof) POS_CUDA(cudaEventRecord(s.ev[1], s.stream));
         if (last) {
             // evaluate the leaves that fit; the count stays on the device
@@ -1159,6 +1165,7 @@ static pos_status process(Search &s, const SliceRec *batch, int M, int x, const 
         if (prof) {
             float ms_k = 0;
             POS_CUDA(cudaEventElapsedTime(&ms_k, s.ev[0], s.ev[1]));
+            s.ms_depth[x] += ms_k;
             if (last) {
                 s.ms_complete += ms_k;
                 float ms_l = 0;
@@ -1264,19 +1271,26 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     POS_CUDA(s.d_feas.reserve(sizeof(uint4) * (size_t)n_slices * (s.S + 1)));
     POS_CUDA(s.ws.d_lim.reserve((size_t)n_slices * s.S * 128));
     POS_CUDA(s.d_inc.reserve(sizeof(Key128)));
-    POS_CUDA(s.d_ctr.reserve(sizeof(unsigned long long) * 64));
+    POS_CUDA(s.d_ctr.reserve(sizeof(unsigned long long) * 128));
     POS_CUDA(s.d_best.reserve(sizeof(unsigned long long) * n_slices));
     POS_CUDA(s.d_leaves.reserve(sizeof(Leaf) * (size_t)s.cap));
     s.ctr = static_cast<unsigned long long *>(s.d_ctr.p);
     s.stats = s.ctr + 40;  // ctr[0..33]: per-depth counters, ctr[36]: leaf count
+    static_assert(40 + kStCount <= 128, "counter block");
     POS_TRY(upload(s, s.d_slices.p, s.slices.data(), sizeof(SliceRec) * n_slices));
     POS_CUDA(cudaMemsetAsync(s.d_inc.p, 0xff, sizeof(Key128), s.stream));
-    POS_CUDA(cudaMemsetAsync(s.d_ctr.p, 0, sizeof(unsigned long long) * 64, s.stream));
+    POS_CUDA(cudaMemsetAsync(s.d_ctr.p, 0, sizeof(unsigned long long) * 128, s.stream));
     POS_CUDA(cudaMemsetAsync(s.d_best.p, 0xff, sizeof(unsigned long long) * n_slices, s.stream));
     const SliceRec *d_all = static_cast<const SliceRec *>(s.d_slices.p);
-    feas_kernel<<<std::min(n_slices, 2 * sm_count()), 128, smem, s.stream>>>(
-        d_all, n_slices, s.S, static_cast<uint4 *>(s.d_feas.p),
-        static_cast<uint8_t *>(s.ws.d_lim.p), s.h->d_blob, s.h->lay, s.stats);
+    {
+        // the memory tables alone (Pw, Pa, cap) are staged per block
+        const BlobLayout ml = memory_layout(s.h->lay);
+        POS_TRY(ensure_smem(reinterpret_cast<const void *>(feas_kernel), ml.bytes));
+        feas_kernel<<<std::min(n_slices, 16 * sm_count()), 128, ml.bytes, s.stream>>>(
+            d_all, n_slices, s.S, static_cast<uint4 *>(s.d_feas.p),
+            static_cast<uint8_t *>(s.ws.d_lim.p),
+            static_cast<const unsigned char *>(s.h->d_blob) + s.h->lay.off_Pw, ml, s.stats);
+    }
     POS_CUDA(cudaGetLastError());
     s.launches++;
     DevBuf &d_root = s.d_root;
@@ -1523,6 +1537,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
                 if ((st = launch_level(last, x, ep, grid, smem_l, s.stream)) != POS_OK)
                     return st;
                 (last ? s.n_complete : s.n_expand)++;
+                s.launches_depth[x]++;
                 if (prof) POS_CUDA(cudaEventRecord(ev[x + 1], s.stream));
             }
             if ((st = run_leaves(s, static_cast<const Leaf *>(s.d_leaves.p), bc + 2 * (S - 2),
@@ -1539,6 +1554,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
             for (int x = 0; x <= S - 1; ++x) {
                 float ms = 0;
                 POS_CUDA(cudaEventElapsedTime(&ms, ev[x], ev[x + 1]));
+                if (x <= S - 2) s.ms_depth[x] += ms;
                 if (x < S - 2) s.ms_expand += ms;
                 else if (x == S - 2) s.ms_complete += ms;
                 else s.ms_leaf += ms;
@@ -1592,6 +1608,12 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         stats->parents_complete = hs[kStParentsComplete];
         stats->leaves = hs[kStLeaves];
         stats->ms_bound = s.ms_bound;
+        for (int x = 0; x < POS_MAX_STAGES; ++x) {
+            stats->ms_depth[x] = s.ms_depth[x];
+            stats->launches_depth[x] = s.launches_depth[x];
+            stats->parents_depth[x] = hs[kStDepthParents + x];
+            stats->children_depth[x] = hs[kStDepthChildren + x];
+        }
         stats->bound_launches = s.n_bound;
         stats->reruns = s.reruns;
     }

@@ -96,7 +96,9 @@ enum {
     kStParentsExpand,
     kStParentsComplete,
     kStLeaves,
-    kStCount
+    kStDepthParents,                                // + x: parents read at depth x
+    kStDepthChildren = kStDepthParents + POS_MAX_STAGES,  // + x: children (plans) written
+    kStCount = kStDepthChildren + POS_MAX_STAGES
 };
 
 constexpr int kCasLimit = 1 << 20;

@@ -94,6 +94,17 @@ BlobLayout timing_layout(const BlobLayout &ly) {
     return t;
 }
 
+BlobLayout memory_layout(const BlobLayout &ly) {
+    BlobLayout t = ly;
+    const int base = ly.off_Pw;
+    t.off_binom = t.off_Pf = t.off_Pb = t.off_Pd = t.off_p2f = t.off_p2b = -1;  // not staged
+    t.off_Pw -= base;
+    t.off_Pa -= base;
+    t.off_cap -= base;
+    t.bytes = ly.off_Pf - base;
+    return t;
+}
+
 // One thread per (table, class) row: the raw per-layer row sits at entries
 // 1..L of the row; turn it into an exclusive prefix sum with P[0] = 0.
 __global__ void prefix_rows_kernel(unsigned char *blob, BlobLayout ly) {
