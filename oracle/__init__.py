@@ -22,11 +22,15 @@ _lib = None
 MAX_S = 16
 
 
+SCHED_1F1B, SCHED_EAGER_1F1B = 0, 1
+
+
 class Tables(C.Structure):
     _fields_ = [("L", C.c_int32), ("n_types", C.c_int32), ("n_tp", C.c_int32),
                 ("fwd", C.c_void_p), ("bwd", C.c_void_p), ("dsync", C.c_void_p),
                 ("p2p_f", C.c_void_p), ("p2p_b", C.c_void_p),
-                ("mem_w", C.c_void_p), ("mem_a", C.c_void_p), ("cap", C.c_void_p)]
+                ("mem_w", C.c_void_p), ("mem_a", C.c_void_p), ("cap", C.c_void_p),
+                ("schedule", C.c_int32)]
 
 
 class Problem(C.Structure):
@@ -101,22 +105,23 @@ def lib():
 class OracleTables:
     """Holds contiguous copies of a workload's tables and the ctypes struct."""
 
-    def __init__(self, L, n_types, n_tp, fwd, bwd, dsync, p2p_f, p2p_b, mem_w, mem_a, cap):
+    def __init__(self, L, n_types, n_tp, fwd, bwd, dsync, p2p_f, p2p_b, mem_w, mem_a, cap,
+                 schedule=SCHED_1F1B):
         K = n_types * n_tp
         i32 = lambda a, shp: np.ascontiguousarray(np.asarray(a, np.int32).reshape(shp))  # noqa: E731
         i64 = lambda a, shp: np.ascontiguousarray(np.asarray(a, np.int64).reshape(shp))  # noqa: E731
         self.arrays = dict(fwd=i32(fwd, (K, L)), bwd=i32(bwd, (K, L)), dsync=i32(dsync, (K, L)),
                            p2p_f=i32(p2p_f, (K, K)), p2p_b=i32(p2p_b, (K, K)),
                            mem_w=i64(mem_w, (K, L)), mem_a=i64(mem_a, (K, L)), cap=i64(cap, (K,)))
-        self.L, self.n_types, self.n_tp = L, n_types, n_tp
+        self.L, self.n_types, self.n_tp, self.schedule = L, n_types, n_tp, schedule
         a = self.arrays
         self.c = Tables(L, n_types, n_tp, *(a[n].ctypes.data for n in
                                             ("fwd", "bwd", "dsync", "p2p_f", "p2p_b", "mem_w",
-                                             "mem_a", "cap")))
+                                             "mem_a", "cap")), schedule)
 
     @classmethod
-    def from_workload(cls, w):
-        return cls(**w.tables_dict())
+    def from_workload(cls, w, schedule=SCHED_1F1B):
+        return cls(**w.tables_dict(), schedule=schedule)
 
 
 def _i32(x, n=None):
@@ -198,9 +203,10 @@ def eval_batch(tab: OracleTables, cands: np.ndarray):
     return T, F
 
 
-def search(w, prune=True, warmup=0, seed=0, tab: OracleTables | None = None):
+def search(w, prune=True, warmup=0, seed=0, tab: OracleTables | None = None,
+           schedule=SCHED_1F1B):
     """Exact search over a gen.Workload search problem.  Returns (plan dict, stats dict)."""
-    tab = tab or OracleTables.from_workload(w)
+    tab = tab or OracleTables.from_workload(w, schedule)
     M_list = _i32(w.M_list)
     dp = _i32(w.dp_list)
     tc = _i32(w.type_counts if w.type_counts else [0] * w.n_types)

@@ -20,7 +20,8 @@
  * Readings where the paper is silent (the library documents the same ones):
  *   - 1F1B order of stage s (1-based) with W_s = min(N-s+1, M) warm-up
  *     forwards: F_1..F_W, then (B_i, F_{W+i}) for i = 1..M-W, then the
- *     remaining backwards.
+ *     remaining backwards.  Eager 1F1B (App. B): the same with
+ *     W_s = min(2(N-s)+1, M).
  *   - weights use per-layer tables summed over the stage's layers (reduces to
  *     the paper's product for identical layers).
  *   - inter-stage edge weights come from a table indexed by the ordered
@@ -108,8 +109,11 @@ typedef struct {
     int64_t pf[ORC_MAX_S], pb[ORC_MAX_S]; /* pf[s]: F edge s->s+1, pb[s]: B edge s+1->s */
 } stage_w;
 
-static int warmup_count(int S, int M, int s /* 0-based */) {
-    int w = S - s; /* N - s + 1 in 1-based stage numbering */
+/* Forwards before the first backward of stage s (0-based), which is also
+ * the number of micro-batches whose activations the stage holds at once:
+ * N - s + 1 (1F1B) or 2(N - s) + 1 (Eager 1F1B) in 1-based numbering. */
+static int warmup_count(int sched, int S, int M, int s /* 0-based */) {
+    int w = sched == ORC_SCHED_EAGER_1F1B ? 2 * (S - 1 - s) + 1 : S - s;
     return w < M ? w : M;
 }
 
@@ -150,7 +154,7 @@ static int stage_memory_ok(const orc_tables *t, int S, int M, int s, int cls, in
         sw += mw[i];
         sa += ma[i];
     }
-    int64_t need = sw + (int64_t)warmup_count(S, M, s) * sa;
+    int64_t need = sw + (int64_t)warmup_count(t->schedule, S, M, s) * sa;
     return need <= t->cap[cls];
 }
 
@@ -240,8 +244,8 @@ static void add_edge(dag *g, int a, int b, int64_t w) {
 #define NODE_B(s, m) (2 + 2 * ((s) * M + (m)))
 #define NODE_R(s) (1 + 2 * S * M + (s))
 
-static int build_and_solve(dag *g, int S, int M, const stage_w *sw, orc_dag_counts *counts,
-                           int64_t *T_out) {
+static int build_and_solve(dag *g, int sched, int S, int M, const stage_w *sw,
+                           orc_dag_counts *counts, int64_t *T_out) {
     int n_nodes = 2 + 2 * S * M + S;
     int n_edges_max = 2 * (S - 1) * M + S * (2 * M - 1) + S + 1 + S;
     if (dag_reserve(g, n_nodes, n_edges_max)) return -1;
@@ -269,10 +273,10 @@ static int build_and_solve(dag *g, int S, int M, const stage_w *sw, orc_dag_coun
             c_inter += 2;
         }
     }
-    /* intra-stage edges: the 1F1B order of each stage, weight 0 */
+    /* intra-stage edges: the schedule's order of each stage, weight 0 */
     int order_node[2 * 255];
     for (int s = 0; s < S; ++s) {
-        int W = warmup_count(S, M, s), n = 0;
+        int W = warmup_count(sched, S, M, s), n = 0;
         for (int m = 0; m < W; ++m) order_node[n++] = NODE_F(s, m);
         for (int i = 0; i < M - W; ++i) {
             order_node[n++] = NODE_B(s, i);
@@ -366,7 +370,7 @@ int orc_eval(const orc_tables *t, int S, int M, const int32_t *cls, const int32_
     dag g;
     memset(&g, 0, sizeof(g));
     int64_t T64;
-    int rc = build_and_solve(&g, S, M, &sw, counts, &T64);
+    int rc = build_and_solve(&g, t->schedule, S, M, &sw, counts, &T64);
     dag_free(&g);
     if (rc) return -1;
     if (T64 >= ((int64_t)1 << 31)) return -1;
@@ -383,7 +387,7 @@ int orc_eval_finish(const orc_tables *t, int S, int M, const int32_t *cls, const
     dag g;
     memset(&g, 0, sizeof(g));
     int64_t T64;
-    int rc = build_and_solve(&g, S, M, &sw, NULL, &T64);
+    int rc = build_and_solve(&g, t->schedule, S, M, &sw, NULL, &T64);
     if (!rc) {
         for (int s = 0; s < S; ++s)
             for (int m = 0; m < M; ++m) {
@@ -540,7 +544,7 @@ int orc_eval_batch(const orc_tables *t, const orc_candidate *c, int64_t n, int32
         stage_w sw;
         stage_weights(t, S, cls, layers, &sw);
         int64_t T64;
-        if (build_and_solve(&g, S, M, &sw, NULL, &T64)) {
+        if (build_and_solve(&g, t->schedule, S, M, &sw, NULL, &T64)) {
             dag_free(&g);
             return -1;
         }
@@ -578,7 +582,7 @@ static void consider_leaf(search_ctx *cx) {
     stage_w sw;
     stage_weights(&cx->p->tab, cx->S, cx->cls, cx->layers, &sw);
     int64_t T64;
-    if (build_and_solve(&cx->g, cx->S, cx->M, &sw, NULL, &T64)) {
+    if (build_and_solve(&cx->g, cx->p->tab.schedule, cx->S, cx->M, &sw, NULL, &T64)) {
         cx->err = 1;
         return;
     }

@@ -31,7 +31,17 @@ typedef struct {
     const int32_t *p2p_f, *p2p_b;        /* [K][K] microseconds, [src class][dst class] */
     const int64_t *mem_w, *mem_a;        /* [K][L] bytes; mem_a per in-flight micro-batch */
     const int64_t *cap;                  /* [K] bytes */
+    int32_t schedule;                    /* ORC_SCHED_1F1B or ORC_SCHED_EAGER_1F1B */
 } orc_tables;
+
+/* Pipeline schedules: the order of each stage's chain and its in-flight
+ * micro-batches.  Stage s (1-based) of N runs W_s forwards, then
+ * (B_i, F_{W_s+i}) for i = 1..M-W_s, then the remaining backwards, with
+ *   1F1B:        W_s = min(N-s+1, M)
+ *   Eager 1F1B:  W_s = min(2(N-s)+1, M)     (App. B: warm-up of 2(N-i)+1
+ *                forwards, steady B-F groups, cool-down backwards). */
+#define ORC_SCHED_1F1B 0
+#define ORC_SCHED_EAGER_1F1B 1
 
 /* 16-byte candidate record (same field meaning as the library's). */
 typedef struct {

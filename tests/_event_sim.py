@@ -1,9 +1,10 @@
 """An event-driven stage simulator: a second, independent CPU formulation of
-the 1F1B pipeline used only to pin the oracle.
+the 1F1B and Eager-1F1B pipelines used only to pin the oracle.
 
 Instead of building the DAG of Sec. 4.1 and taking its longest path, this
 simulates each stage as a worker with a queue.  A stage keeps at most W_s
-micro-batches in flight (activations held); it runs a forward whenever it has
+micro-batches in flight (activations held): N-s+1 under 1F1B and 2(N-s)+1
+under Eager 1F1B (1-based s, at most M); it runs a forward whenever it has
 room and forwards remain, else a backward.  An op starts when its stage is
 free and its input (activation from stage s-1, gradient from stage s+1) has
 arrived; the gradient all-reduce of stage s starts when its last backward
@@ -11,9 +12,9 @@ ends.  The iteration ends when every all-reduce has ended.
 """
 
 
-def stage_program(S, M, s):
+def stage_program(S, M, s, eager=False):
     """Op sequence of stage s (0-based) from the in-flight rule."""
-    W = min(S - s, M)
+    W = min(2 * (S - 1 - s) + 1 if eager else S - s, M)
     prog, in_flight, nf, nb = [], 0, 0, 0
     while nb < M:
         if nf < M and in_flight < W:
@@ -27,10 +28,10 @@ def stage_program(S, M, s):
     return prog
 
 
-def simulate(S, M, F, B, pf, pb, d):
+def simulate(S, M, F, B, pf, pb, d, eager=False):
     """F, B, d: per-stage times; pf[s]: activation transfer s->s+1;
     pb[s]: gradient transfer s+1->s.  Returns (T, fin_F, fin_B)."""
-    progs = [stage_program(S, M, s) for s in range(S)]
+    progs = [stage_program(S, M, s, eager) for s in range(S)]
     pos = [0] * S
     free = [0] * S
     fin_F = [[None] * M for _ in range(S)]

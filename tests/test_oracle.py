@@ -16,7 +16,7 @@ from tests._event_sim import simulate, stage_program
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "two_stage_1f1b.txt")
 
 
-def stage_tables(orc, F, B, d, pf, pb):
+def stage_tables(orc, F, B, d, pf, pb, schedule=0):
     """Tables where stage s holds layer s of its own class s."""
     S = len(F)
     fwd = np.zeros((S, S), np.int32)
@@ -31,7 +31,7 @@ def stage_tables(orc, F, B, d, pf, pb):
         p2b[s + 1, s] = pb[s]
     tab = orc.OracleTables(L=S, n_types=S, n_tp=1, fwd=fwd, bwd=bwd, dsync=ds, p2p_f=p2f,
                            p2p_b=p2b, mem_w=np.zeros((S, S)), mem_a=np.zeros((S, S)),
-                           cap=np.ones(S))
+                           cap=np.ones(S), schedule=schedule)
     return tab, list(range(S)), [1] * S
 
 
@@ -364,10 +364,10 @@ def test_eval_batch_flags(orc):
 
 # -- search (Sec. 4.2) --------------------------------------------------------------
 
-def _brute_force_plan(orc, w):
+def _brute_force_plan(orc, w, schedule=0):
     """Every candidate through eval_batch; argmin of T/(D M), then global index."""
     cands = gen.all_candidates(w)
-    tab = orc.OracleTables.from_workload(w)
+    tab = orc.OracleTables.from_workload(w, schedule)
     T, F = orc.eval_batch(tab, cands)
     best = None
     n_place = len(gen.place_list(w))
