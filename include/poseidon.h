@@ -37,7 +37,14 @@ typedef int32_t pos_status;
 #define POS_EINFEASIBLE 6   /* the search space has no memory-feasible plan */
 #define POS_ENOTIMPL 7
 
-#define POS_SCHED_1F1B 0    /* the only schedule implemented */
+/* Pipeline schedules (the intra-stage order of Sec. 4.1.2).  Stage s
+ * (1-based) of N runs W_s forwards, then (B_i, F_{W_s+i}) for
+ * i = 1..M-W_s, then the remaining backwards, and holds the activations of
+ * W_s micro-batches at once:
+ *   POS_SCHED_1F1B        W_s = min(N-s+1, M)
+ *   POS_SCHED_EAGER_1F1B  W_s = min(2(N-s)+1, M)   (Eager 1F1B, App. B) */
+#define POS_SCHED_1F1B 0
+#define POS_SCHED_EAGER_1F1B 1
 
 #define POS_PLACE_FREE 0    /* any device type on any stage */
 #define POS_PLACE_EXACT 1   /* exactly type_counts[t] stages of type t */
@@ -103,7 +110,8 @@ typedef struct pos_candidate {
  * Copy the tables to the current CUDA device and build the per-class
  * exclusive prefix sums used by every kernel (hot-path step a1, Sec. 4.1.3).
  * *handle owns the device copies until poseidon_tables_destroy.  schedule
- * must be POS_SCHED_1F1B.
+ * (POS_SCHED_1F1B or POS_SCHED_EAGER_1F1B) applies to every evaluation
+ * through the handle.
  * Errors: POS_EINVAL (null pointer, limits, negative cost or memory),
  * POS_EOVERFLOW (a class's summed costs reach 2^31), POS_ENOTIMPL (schedule),
  * POS_ENOMEM, POS_ECUDA.
@@ -209,7 +217,7 @@ typedef struct pos_problem {
     int32_t warmup;             /* random feasible samples seeding T_min (paper: 500) */
     int32_t prune;              /* POS_PRUNE_NONE, POS_PRUNE_EQ2 or POS_PRUNE_TIGHT */
     uint64_t seed;              /* warm-up sampling seed */
-    int32_t schedule;           /* POS_SCHED_1F1B */
+    int32_t schedule;           /* POS_SCHED_1F1B or POS_SCHED_EAGER_1F1B */
     int64_t frontier_cap;       /* entries per frontier buffer; 0 = default 2^24;
                                    raised to at least 32*L */
     int32_t profile;            /* 1: device time per kernel kind in the stats (CUDA

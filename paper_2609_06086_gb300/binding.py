@@ -20,6 +20,7 @@ POS_OK, POS_EINVAL, POS_EOVERFLOW, POS_ENOMEM, POS_ECUDA, POS_ETIMEOUT, POS_EINF
 STATUS_NAMES = ["POS_OK", "POS_EINVAL", "POS_EOVERFLOW", "POS_ENOMEM", "POS_ECUDA",
                 "POS_ETIMEOUT", "POS_EINFEASIBLE", "POS_ENOTIMPL"]
 POS_SCHED_1F1B = 0
+POS_SCHED_EAGER_1F1B = 1
 POS_PLACE_FREE, POS_PLACE_EXACT = 0, 1
 MAX_STAGES = 16
 
@@ -183,7 +184,8 @@ def _prune_mode(prune):
     return int(prune)
 
 
-def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0, profile=False):
+def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0, profile=False,
+                 schedule=POS_SCHED_1F1B):
     """pos_problem for a gen.Workload search; returns (problem, keep-alive list)."""
     tab = Tables.from_workload(w)
     keep = [tab]
@@ -195,7 +197,7 @@ def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0, profile=Fals
 
     p = pos_problem(tab.c, w.S, len(w.M_list), arr(w.M_list), arr(w.tp_list), arr(w.dp_list),
                     w.placement, arr(w.type_counts if w.type_counts else [0] * w.n_types),
-                    int(warmup), _prune_mode(prune), int(seed), POS_SCHED_1F1B, int(frontier_cap),
+                    int(warmup), _prune_mode(prune), int(seed), int(schedule), int(frontier_cap),
                     int(bool(profile)))
     return p, keep
 

@@ -51,6 +51,7 @@ constexpr int kBinomK = 16;
 
 struct BlobLayout {
     int L, K, n_types, n_tp;
+    int sched;  // POS_SCHED_1F1B or POS_SCHED_EAGER_1F1B (stage chains, in-flight counts)
     int off_binom, off_Pw, off_Pa, off_cap, off_Pf, off_Pb, off_Pd, off_p2f, off_p2b;
     int bytes;  // multiple of 16
 };
@@ -73,10 +74,10 @@ struct Handle {
 };
 
 pos_status validate_tables(const pos_tables *t);
-pos_status create_handle(const pos_tables *t, Handle **out);
+pos_status create_handle(const pos_tables *t, int sched, Handle **out);
 // host part of create_handle: validated blob with raw rows, plus guard terms
-pos_status build_blob(const pos_tables *t, std::vector<unsigned char> &host, BlobLayout &ly,
-                      int64_t &guard_A, int64_t &guard_D, int64_t &guard_P);
+pos_status build_blob(const pos_tables *t, int sched, std::vector<unsigned char> &host,
+                      BlobLayout &ly, int64_t &guard_A, int64_t &guard_D, int64_t &guard_P);
 // device part: per-class prefix sums in place, asynchronous on `stream`
 pos_status launch_prefix_rows(void *d_blob, const BlobLayout &ly, cudaStream_t stream);
 void destroy_handle(Handle *h);
@@ -265,13 +266,18 @@ struct StageW {
 };
 
 // In-flight micro-batches of 0-based stage s under 1F1B: min(S - s, M).
-__device__ __forceinline__ int inflight(int S, int M, int s) { return min(S - s, M); }
+// Micro-batches a 0-based stage s holds at once = its warm-up forwards:
+// N-s+1 (1F1B) or 2(N-s)+1 (Eager 1F1B) in 1-based numbering, at most M.
+__host__ __device__ __forceinline__ int inflight(int sched, int S, int M, int s) {
+    const int w = sched == POS_SCHED_EAGER_1F1B ? 2 * (S - 1 - s) + 1 : S - s;
+    return w < M ? w : M;
+}
 
 // Does 0-based stage s of an S-stage pipeline on class k fit layers [a, b)?
 __device__ __forceinline__ bool stage_fits(const Tab &t, int S, int M, int s, int k, int a,
                                            int b) {
     const int64_t need = (Pw(t, k, b) - Pw(t, k, a)) +
-                         (int64_t)inflight(S, M, s) * (Pa(t, k, b) - Pa(t, k, a));
+                         (int64_t)inflight(t.ly->sched, S, M, s) * (Pa(t, k, b) - Pa(t, k, a));
     return need <= cap_of(t, k);
 }
 
@@ -321,7 +327,10 @@ __device__ __forceinline__ bool plan_fits(const Tab &t, int M, const int (&cut)[
 // separate instantiation (kPathGeneric) whose schedule is unrolled for
 // each M in 1..S-1.
 // ---------------------------------------------------------------------------
-enum { kPathFast = 0, kPathGeneric = 1 };
+// Paths: 1F1B with M >= S (ramps + steady loop), 1F1B with M < S (unrolled
+// per M), Eager 1F1B with M >= 2S-1 (ramps + steady loop), Eager 1F1B with
+// M < 2S-1 (level program).
+enum { kPathFast = 0, kPathGeneric = 1, kPathEager = 2, kPathEagerShort = 3 };
 
 // Op of 1-based stage s1 at ramp-up level t (1 <= t <= 2S-1) and at
 // ramp-down level 2M + tau (0 <= tau <= 2S-2), for M >= S: 0 none, 1 F, 2 B.
@@ -483,6 +492,212 @@ __device__ __forceinline__ int32_t makespan_1f1b(const StageW<S> &w, int M) {
 #pragma unroll
     for (int s = 0; s < S; ++s) T = max(T, Bo[s] + w.d[s]);
     return T;
+}
+
+// ---------------------------------------------------------------------------
+// Eager 1F1B (App. B): stage s (1-based) runs W_s = min(2(S-s)+1, M)
+// forwards, then (B_i, F_{W_s+i}) pairs, then the remaining backwards.  In
+// the unit-weight level order (stages descending within a level)
+//     F_{s,m}: s + m - 1 (m <= W_s), 2m - 2S + 3s - 2 (m > W_s);
+//     B_{s,m}: 2S - s + 2m - 1,
+// each stage runs at most one op per level, but a stage can be two forwards
+// ahead of the next one: the forward predecessor of F_{s,m} is the latest
+// or the previous forward of stage s-1 (its lag, 1 or 2, is known at
+// compile time).  So each stage keeps Fo (last forward), Fp (the one before)
+// and Bo.  For M >= 2S-1 the levels split into a ramp-up (levels 1..2S-1),
+// M-2S+1 steady two-level steps in which every stage alternates B and F
+// (lag 2), and a ramp-down (levels 2M+tau, tau = -2S+2..2S-2).
+// ---------------------------------------------------------------------------
+__host__ __device__ constexpr int eager_up_op(int S, int s1, int t) {
+    return (t >= s1 && t <= 2 * S - s1) ? 1
+           : (t >= 2 * S - s1 + 1 && ((t + s1) & 1) == 1) ? 2
+           : (t >= 2 * S - s1 + 2 && ((t + s1) & 1) == 0) ? 1
+                                                            : 0;
+}
+__host__ __device__ constexpr int eager_down_op(int S, int s1, int tau) {
+    return ((((tau + s1) % 2) + 2) % 2 == 0 && tau <= 3 * s1 - 2 * S - 2) ? 1
+           : ((((tau + s1) % 2) + 2) % 2 == 1 && tau <= 2 * S - s1 - 1) ? 2
+                                                                          : 0;
+}
+__host__ __device__ constexpr bool eager_up_last_is_b(int S, int s1, int t) {
+    for (int u = t - 1; u >= 1; --u)
+        if (eager_up_op(S, s1, u)) return eager_up_op(S, s1, u) == 2;
+    return false;
+}
+// before the ramp-down, the last steady level 2M-2S+1 ran F on odd stages
+__host__ __device__ constexpr bool eager_down_last_is_b(int S, int s1, int tau) {
+    for (int u = tau - 1; u >= -2 * S + 2; --u)
+        if (eager_down_op(S, s1, u)) return eager_down_op(S, s1, u) == 2;
+    return (s1 & 1) == 0;
+}
+// forwards of stage s1 in ramp-up levels < t / ramp-down levels < 2M+tau
+__host__ __device__ constexpr int eager_up_nf(int S, int s1, int t) {
+    int n = 0;
+    for (int u = 1; u < t; ++u) n += eager_up_op(S, s1, u) == 1;
+    return n;
+}
+__host__ __device__ constexpr int eager_down_nf(int S, int s1, int tau) {
+    int n = 0;
+    for (int u = -2 * S + 2; u < tau; ++u) n += eager_down_op(S, s1, u) == 1;
+    return n;
+}
+// forwards stage s1-1 has done beyond stage s1 before this op (1 or 2)
+__host__ __device__ constexpr int eager_up_lag(int S, int s1, int t) {
+    return eager_up_nf(S, s1 - 1, t) - eager_up_nf(S, s1, t);
+}
+__host__ __device__ constexpr int eager_down_lag(int S, int s1, int tau) {
+    return (eager_down_nf(S, s1, 2 * S - 1) - eager_down_nf(S, s1 - 1, 2 * S - 1)) +
+           eager_down_nf(S, s1 - 1, tau) - eager_down_nf(S, s1, tau);
+}
+
+template <int S, int s, int LAG>
+__device__ __forceinline__ void relax_f_lag(int32_t (&Fo)[S], int32_t (&Fp)[S],
+                                            const StageW<S> &w, int32_t clock) {
+    int32_t in = 0;
+    if constexpr (s > 0) {
+        static_assert(LAG == 1 || LAG == 2, "forward lag");
+        in = (LAG == 2 ? Fp[s - 1] : Fo[s - 1]) + w.pf[s - 1];
+    }
+    Fp[s] = Fo[s];
+    Fo[s] = max(clock, in) + w.F[s];
+}
+
+template <int S, bool UP, int t, int s1>
+__device__ __forceinline__ void eager_ramp_op(int32_t (&Fo)[S], int32_t (&Fp)[S], int32_t (&Bo)[S],
+                                              const StageW<S> &w) {
+    constexpr int op = UP ? eager_up_op(S, s1, t) : eager_down_op(S, s1, t);
+    constexpr bool last_b = UP ? eager_up_last_is_b(S, s1, t) : eager_down_last_is_b(S, s1, t);
+    constexpr int s = s1 - 1;
+    if constexpr (op == 1) {
+        constexpr int lag = s1 == 1 ? 1 : (UP ? eager_up_lag(S, s1, t) : eager_down_lag(S, s1, t));
+        relax_f_lag<S, s, lag>(Fo, Fp, w, last_b ? Bo[s] : Fo[s]);
+    } else if constexpr (op == 2) {
+        relax_b<S, s>(Bo, w, last_b ? Bo[s] : Fo[s]);
+    }
+}
+template <int S, bool UP, int t, int... i>
+__device__ __forceinline__ void eager_ramp_level(int32_t (&Fo)[S], int32_t (&Fp)[S],
+                                                 int32_t (&Bo)[S], const StageW<S> &w,
+                                                 std::integer_sequence<int, i...>) {
+    (eager_ramp_op<S, UP, t, S - i>(Fo, Fp, Bo, w), ...);
+}
+template <int S, bool UP, int T0, int... t>
+__device__ __forceinline__ void eager_ramp(int32_t (&Fo)[S], int32_t (&Fp)[S], int32_t (&Bo)[S],
+                                           const StageW<S> &w, std::integer_sequence<int, t...>) {
+    (eager_ramp_level<S, UP, T0 + t>(Fo, Fp, Bo, w, std::make_integer_sequence<int, S>{}), ...);
+}
+// steady level of parity P: stage s1 with the parity of P runs F (after its
+// B, forward lag 2), the others B (after their F)
+template <int S, int P, int i>
+__device__ __forceinline__ void eager_steady_op(int32_t (&Fo)[S], int32_t (&Fp)[S],
+                                                int32_t (&Bo)[S], const StageW<S> &w) {
+    constexpr int s1 = S - i, s = s1 - 1;
+    if constexpr ((s1 & 1) == P) relax_f_lag<S, s, 2>(Fo, Fp, w, Bo[s]);
+    else relax_b<S, s>(Bo, w, Fo[s]);
+}
+template <int S, int P, int... i>
+__device__ __forceinline__ void eager_steady_level(int32_t (&Fo)[S], int32_t (&Fp)[S],
+                                                   int32_t (&Bo)[S], const StageW<S> &w,
+                                                   std::integer_sequence<int, i...>) {
+    (eager_steady_op<S, P, i>(Fo, Fp, Bo, w), ...);
+}
+
+// Eager 1F1B, M >= 2S-1
+template <int S>
+__device__ __forceinline__ int32_t makespan_eager(const StageW<S> &w, int M) {
+    int32_t Fo[S], Fp[S], Bo[S];
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+        Fo[s] = 0;
+        Fp[s] = 0;
+        Bo[s] = 0;
+    }
+    eager_ramp<S, true, 1>(Fo, Fp, Bo, w, std::make_integer_sequence<int, 2 * S - 1>{});
+    for (int j = 0; j < M - 2 * S + 1; ++j) {
+        eager_steady_level<S, 0>(Fo, Fp, Bo, w, std::make_integer_sequence<int, S>{});
+        eager_steady_level<S, 1>(Fo, Fp, Bo, w, std::make_integer_sequence<int, S>{});
+    }
+    eager_ramp<S, false, -2 * S + 2>(Fo, Fp, Bo, w, std::make_integer_sequence<int, 4 * S - 3>{});
+    int32_t T = 0;
+#pragma unroll
+    for (int s = 0; s < S; ++s) T = max(T, Bo[s] + w.d[s]);
+    return T;
+}
+
+// Level program of one (schedule, S, M): per level one 64-bit word, bit s of
+// bits 0-15 = stage s runs a forward, bits 16-31 = a backward, bits 32-47 =
+// that forward's predecessor is the previous forward of stage s-1 (lag 2).
+// Built on the host from the unit-weight ASAP levels of the schedule's
+// chains (schedules.cu); used for Eager 1F1B with M < 2S-1.
+template <int S>
+__device__ __forceinline__ int32_t makespan_program(const StageW<S> &w, const uint64_t *prog,
+                                                    int n_levels) {
+    int32_t Fo[S], Fp[S], Bo[S], clk[S];
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+        Fo[s] = 0;
+        Fp[s] = 0;
+        Bo[s] = 0;
+        clk[s] = 0;
+    }
+#pragma unroll 1
+    for (int l = 0; l < n_levels; ++l) {
+        const uint64_t word = __ldg(prog + l);
+        const uint32_t fm = (uint32_t)word & 0xffffu, bm = (uint32_t)(word >> 16) & 0xffffu;
+        const uint32_t lm = (uint32_t)(word >> 32) & 0xffffu;
+#pragma unroll
+        for (int s = S - 1; s >= 0; --s) {
+            if ((fm >> s) & 1u) {
+                int32_t in = 0;
+                if (s > 0) in = (((lm >> s) & 1u) ? Fp[s - 1] : Fo[s - 1]) + w.pf[s > 0 ? s - 1 : 0];
+                Fp[s] = Fo[s];
+                Fo[s] = max(clk[s], in) + w.F[s];
+                clk[s] = Fo[s];
+            } else if ((bm >> s) & 1u) {
+                int32_t in = 0;
+                if (s + 1 < S) in = Bo[s + 1 < S ? s + 1 : s] + w.pb[s];
+                Bo[s] = max(clk[s], in) + w.B[s];
+                clk[s] = Bo[s];
+            }
+        }
+    }
+    int32_t T = 0;
+#pragma unroll
+    for (int s = 0; s < S; ++s) T = max(T, Bo[s] + w.d[s]);
+    return T;
+}
+
+// Level programs on the device: index[(S-1)*32 + M] = (first word, levels)
+// for the (S, M) pairs a schedule's short path covers.
+struct Programs {
+    const uint64_t *words;
+    const uint2 *index;
+};
+// Programs of a schedule on the current device (built and uploaded on first
+// use, kept for the process); words = index = NULL for 1F1B.
+pos_status schedule_programs(int sched, Programs *out);
+
+// Makespan of one decoded plan on path PATH.
+template <int S, int PATH>
+__device__ __forceinline__ int32_t makespan_path(const StageW<S> &w, int M, const Programs &pg) {
+    if constexpr (PATH == kPathEager) {
+        return makespan_eager<S>(w, M);
+    } else if constexpr (PATH == kPathEagerShort) {
+        const uint2 ix = __ldg(pg.index + (S - 1) * 32 + M);
+        return makespan_program<S>(w, pg.words + ix.x, (int)ix.y);
+    } else {
+        return makespan_1f1b<S, PATH>(w, M);
+    }
+}
+
+// Path of (schedule, S, M) and the first M of the fast path.
+__host__ __device__ __forceinline__ int fast_min_m(int sched, int S) {
+    return sched == POS_SCHED_EAGER_1F1B ? 2 * S - 1 : S;
+}
+__host__ __device__ __forceinline__ int path_of(int sched, int S, int M) {
+    const bool fast = M >= fast_min_m(sched, S);
+    return sched == POS_SCHED_EAGER_1F1B ? (fast ? kPathEager : kPathEagerShort)
+                                         : (fast ? kPathFast : kPathGeneric);
 }
 
 // Overflow guard U(S, M) >= 2^31 ?

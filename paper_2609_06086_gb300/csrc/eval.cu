@@ -59,21 +59,22 @@ __global__ void argmin_final(const int32_t *part_t, const long long *part_i, int
 // ---------------------------------------------------------------------------
 // counting sort of the candidates by (S, M) key
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ int eval_key(uint32_t w) {
+__device__ __forceinline__ int eval_key(int sched, uint32_t w) {
     const int S = w & 0xff, M = (w >> 8) & 0xff;
     if (S < 1 || S > POS_MAX_STAGES || M < 1) return -1;
-    return M >= S ? (S - 1) * 256 + M : 4096 + (S - 1) * 16 + M;
+    return M >= fast_min_m(sched, S) ? fast_key_begin(S) + M : generic_key_begin(S) + M;
 }
 
 // global key histogram; invalid records are answered right here
-__global__ void sort_hist_kernel(const uint4 *cands, int64_t n, uint32_t *hist, int32_t *T,
+__global__ void sort_hist_kernel(int sched, const uint4 *cands, int64_t n, uint32_t *hist,
+                                 int32_t *T,
                                  uint8_t *F) {
     __shared__ uint32_t h[kKeys];
     for (int i = threadIdx.x; i < kKeys; i += blockDim.x) h[i] = 0;
     __syncthreads();
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
-        const int k = eval_key(__ldg(&cands[i].w));
+        const int k = eval_key(sched, __ldg(&cands[i].w));
         if (k >= 0) {
             atomicAdd(&h[k], 1u);
         } else {
@@ -117,7 +118,7 @@ __global__ void sort_scan_kernel(const uint32_t *hist, uint32_t *offs, uint32_t 
 // one range per key with a single atomic, then places the indices.
 constexpr int kChunk = 8192;
 
-__global__ void sort_scatter_kernel(const uint4 *cands, int64_t n, uint32_t *cursor,
+__global__ void sort_scatter_kernel(int sched, const uint4 *cands, int64_t n, uint32_t *cursor,
                                     uint32_t *perm) {
     __shared__ uint32_t h[kKeys];
     for (int64_t c0 = blockIdx.x * (int64_t)kChunk; c0 < n; c0 += (int64_t)gridDim.x * kChunk) {
@@ -125,7 +126,7 @@ __global__ void sort_scatter_kernel(const uint4 *cands, int64_t n, uint32_t *cur
         for (int i = threadIdx.x; i < kKeys; i += blockDim.x) h[i] = 0;
         __syncthreads();
         for (int64_t i = c0 + threadIdx.x; i < c1; i += blockDim.x) {
-            const int k = eval_key(__ldg(&cands[i].w));
+            const int k = eval_key(sched, __ldg(&cands[i].w));
             if (k >= 0) atomicAdd(&h[k], 1u);
         }
         __syncthreads();
@@ -133,7 +134,7 @@ __global__ void sort_scatter_kernel(const uint4 *cands, int64_t n, uint32_t *cur
             if (h[i]) h[i] = atomicAdd(&cursor[i], h[i]);
         __syncthreads();
         for (int64_t i = c0 + threadIdx.x; i < c1; i += blockDim.x) {
-            const int k = eval_key(__ldg(&cands[i].w));
+            const int k = eval_key(sched, __ldg(&cands[i].w));
             if (k >= 0) perm[atomicAdd(&h[k], 1u)] = (uint32_t)i;
         }
         __syncthreads();
@@ -206,6 +207,8 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
     cudaMemPool_t pool;
     pos_status st = scratch_pool(&pool);
     if (st != POS_OK) return st;
+    Programs pg;  // the schedule's level programs (Eager 1F1B, few micro-batches)
+    if ((st = schedule_programs(h->lay.sched, &pg)) != POS_OK) return st;
     // permutation indices are 32-bit: batches above 2^31 go in chunks
     const int64_t chunk = (int64_t)1 << 31;
     for (int64_t base = 0; base < n; base += chunk) {
@@ -232,27 +235,38 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
         p.gA = h->guard_A;
         p.gD = h->guard_D;
         p.gP = h->guard_P;
+        p.pg = pg;
         const int grid = (int)std::max<int64_t>(
             1, std::min<int64_t>((m + 255) / 256, 4LL * sm_count()));
         cudaError_t e = cudaMemsetAsync(hist, 0, sizeof(uint32_t) * kKeys, stream);
         if (e == cudaSuccess) {
-            sort_hist_kernel<<<grid, 256, 0, stream>>>(p.cands, m, hist, p.T, p.F);
+            sort_hist_kernel<<<grid, 256, 0, stream>>>(p.lay.sched, p.cands, m, hist, p.T, p.F);
             sort_scan_kernel<<<1, 1024, 0, stream>>>(hist, offs, cursor);
             const int sgrid = (int)std::max<int64_t>(
                 1, std::min<int64_t>((m + kChunk - 1) / kChunk, 8LL * sm_count()));
-            sort_scatter_kernel<<<sgrid, 512, 0, stream>>>(p.cands, m, cursor, perm);
+            sort_scatter_kernel<<<sgrid, 512, 0, stream>>>(p.lay.sched, p.cands, m, cursor, perm);
             e = cudaGetLastError();
         }
         if (e == cudaSuccess) st = launch_decode(p, stream);
         if (e == cudaSuccess && st == POS_OK) {
-            if ((st = eval_fast_1_4(p, stream)) == POS_OK && (st = eval_fast_5_8(p, stream)) == POS_OK &&
-                (st = eval_fast_9_12(p, stream)) == POS_OK &&
-                (st = eval_fast_13_16(p, stream)) == POS_OK &&
-                (st = eval_generic_2_8(p, stream)) == POS_OK &&
-                (st = eval_generic_9_12(p, stream)) == POS_OK &&
-                (st = eval_generic_13_14(p, stream)) == POS_OK &&
-                (st = eval_generic_15_15(p, stream)) == POS_OK)
+            if (p.lay.sched == POS_SCHED_EAGER_1F1B) {
+                if ((st = eval_eager_1_6(p, stream)) == POS_OK &&
+                    (st = eval_eager_7_10(p, stream)) == POS_OK &&
+                    (st = eval_eager_11_13(p, stream)) == POS_OK &&
+                    (st = eval_eager_14_16(p, stream)) == POS_OK &&
+                    (st = eval_eager_short_2_8(p, stream)) == POS_OK &&
+                    (st = eval_eager_short_9_12(p, stream)) == POS_OK)
+                    st = eval_eager_short_13_16(p, stream);
+            } else if ((st = eval_fast_1_4(p, stream)) == POS_OK &&
+                       (st = eval_fast_5_8(p, stream)) == POS_OK &&
+                       (st = eval_fast_9_12(p, stream)) == POS_OK &&
+                       (st = eval_fast_13_16(p, stream)) == POS_OK &&
+                       (st = eval_generic_2_8(p, stream)) == POS_OK &&
+                       (st = eval_generic_9_12(p, stream)) == POS_OK &&
+                       (st = eval_generic_13_14(p, stream)) == POS_OK &&
+                       (st = eval_generic_15_15(p, stream)) == POS_OK) {
                 st = eval_generic_16_16(p, stream);
+            }
         }
         const cudaError_t e2 = cudaFreeAsync(scratch, stream);
         if (e != cudaSuccess) return cuda_fail(e, "eval sort launch");

@@ -15,9 +15,10 @@
 // bucket boundaries, and no kernel waits at a block barrier after staging the
 // cost tables.
 //
-// Sort keys: M >= S -> (S-1)*256 + M (the M < S slots of each S stay empty),
-// M < S -> 4096 + (S-1)*16 + M; records with S outside 1..16 or M = 0 are
-// flagged invalid by the sort pass and get no key.
+// Sort keys: fast path (M >= S for 1F1B, M >= 2S-1 for Eager 1F1B) ->
+// (S-1)*256 + M (the other slots of each S stay empty); short path ->
+// 4096 + (S-1)*32 + M; records with S outside 1..16 or M = 0 are flagged
+// invalid by the sort pass and get no key.
 #pragma once
 #include <algorithm>
 
@@ -25,11 +26,11 @@
 
 namespace pos {
 
-constexpr int kKeys = 4096 + 256;   // fast keys, then M < S keys
+constexpr int kKeys = 4096 + 16 * 32;  // fast keys, then short-path keys
 constexpr int kEvalThreads = 128;
 
 __host__ __device__ inline int fast_key_begin(int S) { return (S - 1) * 256; }
-__host__ __device__ inline int generic_key_begin(int S) { return 4096 + (S - 1) * 16; }
+__host__ __device__ inline int generic_key_begin(int S) { return 4096 + (S - 1) * 32; }
 
 struct EvalParams {
     const uint4 *cands;
@@ -43,6 +44,7 @@ struct EvalParams {
     const void *blob;
     BlobLayout lay;
     int64_t gA, gD, gP;
+    Programs pg;           // level programs of the schedule's short path
 };
 
 // Decode pass for one candidate: checks its fields and the overflow guard,
@@ -108,7 +110,8 @@ struct EvalWith {
     struct One {
         // makespan of a decoded candidate (cuts packed by Decode<S>)
         static __device__ __forceinline__ void run(const Tab &t, const uint4 &rec,
-                                                   const uint4 &packed, int32_t &T) {
+                                                   const uint4 &packed, const Programs &pg,
+                                                   int32_t &T) {
             const uint32_t tcode = rec.z;
             const int M = (rec.w >> 8) & 0xff;
             const int tp = (rec.w >> 16) & 0xff;
@@ -122,17 +125,18 @@ struct EvalWith {
             cut[S] = t.L();
             StageW<S> w;
             stage_weights<S>(t, cut, cls, w);
-            T = makespan_1f1b<S, PATH>(w, M);
+            T = makespan_path<S, PATH>(w, M, pg);
         }
     };
 };
 
 template <int SLO, int SHI, int PATH>
 __device__ __forceinline__ void dispatch_range(int S, const Tab &t, const uint4 &rec,
-                                               const uint4 &packed, int32_t &T) {
+                                               const uint4 &packed, const Programs &pg,
+                                               int32_t &T) {
 #define POS_EV(n)                                                                            \
     if (n >= SLO && n <= SHI && S == n) {                                                    \
-        EvalWith<PATH>::template One<(n >= SLO && n <= SHI) ? n : SLO>::run(t, rec, packed, T); \
+        EvalWith<PATH>::template One<(n >= SLO && n <= SHI) ? n : SLO>::run(t, rec, packed, pg, T); \
         return;                                                                              \
     }
     POS_EV(1) POS_EV(2) POS_EV(3) POS_EV(4) POS_EV(5) POS_EV(6) POS_EV(7) POS_EV(8)
@@ -148,8 +152,9 @@ __global__ void __launch_bounds__(kEvalThreads, MINB) eval_kernel(EvalParams p) 
     stage_blob(sm, p.blob, p.lay.bytes);
     __syncthreads();
     const Tab t = tab_at(sm, p.lay);
-    const int key_lo = PATH == kPathFast ? fast_key_begin(SLO) : generic_key_begin(SLO);
-    const int key_hi = PATH == kPathFast ? fast_key_begin(SHI + 1) : generic_key_begin(SHI + 1);
+    constexpr bool kFast = PATH == kPathFast || PATH == kPathEager;
+    const int key_lo = kFast ? fast_key_begin(SLO) : generic_key_begin(SLO);
+    const int key_hi = kFast ? fast_key_begin(SHI + 1) : generic_key_begin(SHI + 1);
     const int64_t begin = p.offs[key_lo], end = p.offs[key_hi];
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     // whole warps iterate together (ballots below)
@@ -172,7 +177,7 @@ __global__ void __launch_bounds__(kEvalThreads, MINB) eval_kernel(EvalParams p) 
             const int Sg = __shfl_sync(0xffffffffu, S, leader);
             const bool mine = active && S == Sg;
             const unsigned grp = __ballot_sync(0xffffffffu, mine);
-            if (mine) dispatch_range<SLO, SHI, PATH>(Sg, t, rec, packed, T);
+            if (mine) dispatch_range<SLO, SHI, PATH>(Sg, t, rec, packed, p.pg, T);
             pending &= ~grp;
         }
         if (active) p.T[i] = T;
@@ -206,5 +211,12 @@ pos_status eval_generic_9_12(const EvalParams &p, cudaStream_t s);
 pos_status eval_generic_13_14(const EvalParams &p, cudaStream_t s);
 pos_status eval_generic_15_15(const EvalParams &p, cudaStream_t s);
 pos_status eval_generic_16_16(const EvalParams &p, cudaStream_t s);
+pos_status eval_eager_1_6(const EvalParams &p, cudaStream_t s);
+pos_status eval_eager_7_10(const EvalParams &p, cudaStream_t s);
+pos_status eval_eager_11_13(const EvalParams &p, cudaStream_t s);
+pos_status eval_eager_14_16(const EvalParams &p, cudaStream_t s);
+pos_status eval_eager_short_2_8(const EvalParams &p, cudaStream_t s);
+pos_status eval_eager_short_9_12(const EvalParams &p, cudaStream_t s);
+pos_status eval_eager_short_13_16(const EvalParams &p, cudaStream_t s);
 
 }  // namespace pos

@@ -902,13 +902,15 @@ struct Search {
     uint64_t launches_depth[POS_MAX_STAGES] = {};
     uint64_t n_expand = 0, n_complete = 0, n_leaf = 0, n_bound = 0, reruns = 0;
     int cur_nb = 0;    // slots of the batch being enumerated
+    Programs pg{};     // level programs of the schedule's short path
     size_t stage_off = 0;  // bytes of the staging area used by this search
     int n_vrows = 0;   // rows of the completion-bound tables (memory-feasible slices)
 };
 
 static pos_status validate_problem(const pos_problem *p) {
     if (!p) return fail(POS_EINVAL, "problem is NULL");
-    if (p->schedule != POS_SCHED_1F1B) return fail(POS_ENOTIMPL, "only 1F1B is implemented");
+    if (p->schedule != POS_SCHED_1F1B && p->schedule != POS_SCHED_EAGER_1F1B)
+        return fail(POS_ENOTIMPL, "schedule must be POS_SCHED_1F1B or POS_SCHED_EAGER_1F1B");
     if (p->S < 1 || p->S > POS_MAX_STAGES) return fail(POS_EINVAL, "S must be in 1..16");
     if (p->S > p->tables.L) return fail(POS_EINVAL, "S > L");
     if (p->n_M < 1 || !p->M_list) return fail(POS_EINVAL, "empty M_list");
@@ -1084,7 +1086,8 @@ static pos_status run_leaves(Search &s, const Leaf *leaves, unsigned long long *
     lp.blob = s.h->d_blob;
     lp.lay = s.h->lay;
     s.launches++;
-    return launch_leaf(s.S, M >= s.S, lp, s.grid_leaf, s.stream);
+    lp.pg = s.pg;
+    return launch_leaf(s.S, path_of(s.pb->schedule, s.S, M), lp, s.grid_leaf, s.stream);
 }
 
 template <bool COMPLETE, int X>
@@ -1217,13 +1220,15 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     if (n_slices64 > (1ull << 22)) return fail(POS_EINVAL, "more than 2^22 slices");
     const int n_slices = (int)n_slices64;
     if (s.n_map && n_slices64 > ~0ull / s.n_map) return fail(POS_EINVAL, "global index overflows");
+    if ((st = schedule_programs(p->schedule, &s.pg)) != POS_OK) return st;
     // pinned staging for this search's uploads (tables, slice records, lists)
     if ((st = reserve_stage(s, ((size_t)256 << 10) + (size_t)n_slices * 320 +
                                    (size_t)p->n_M * 16)) != POS_OK)
         return st;
     {
         std::vector<unsigned char> host;
-        st = build_blob(&p->tables, host, s.hd.lay, s.hd.guard_A, s.hd.guard_D, s.hd.guard_P);
+        st = build_blob(&p->tables, p->schedule, host, s.hd.lay, s.hd.guard_A, s.hd.guard_D,
+                        s.hd.guard_P);
         if (st != POS_OK) return st;
         POS_CUDA(cudaGetDevice(&s.hd.device));
         POS_CUDA(s.ws.blob.reserve(s.hd.lay.bytes));

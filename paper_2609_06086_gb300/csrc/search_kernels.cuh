@@ -141,6 +141,7 @@ struct LeafParams {
     unsigned long long *slice_best;  // optional per-slice minimum objective
     const void *blob;
     BlobLayout lay;
+    Programs pg;  // level programs of the schedule's short path
 };
 
 // leaf byte 4+s holds cut[s+1] (layers of stages 0..s)
@@ -154,9 +155,15 @@ __device__ __forceinline__ void leaf_cuts(const Vec32 &v, int (&cut)[S + 1]) {
     leaf_cuts_i<S>(v, cut, std::make_integer_sequence<int, S - 1>{});
 }
 
+// blocks per SM: the Eager paths keep three registers per stage, not two
+__host__ __device__ constexpr int leaf_min_blocks(int S, int path) {
+    return (path == kPathEager || path == kPathEagerShort)
+               ? (S <= 4 ? 4 : S <= 6 ? 3 : S <= 12 ? 2 : 1)
+               : (S <= 4 ? 4 : S <= 8 ? 3 : 2);
+}
+
 template <int S, int PATH>
-__global__ void __launch_bounds__(256, (S <= 4 ? 4 : (S <= 8 ? 3 : 2)))
-leaf_kernel(LeafParams p) {
+__global__ void __launch_bounds__(256, leaf_min_blocks(S, PATH)) leaf_kernel(LeafParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
     __shared__ uint64_t bar;
     const unsigned long long c0 = __ldcg(p.count);
@@ -195,7 +202,7 @@ leaf_kernel(LeafParams p) {
             const uint64_t rank = rank_cuts<S>(t, cut);
             StageW<S> w;
             stage_weights<S>(t, cut, cls, w);
-            const int32_t T = makespan_1f1b<S, PATH>(w, p.M);
+            const int32_t T = makespan_path<S, PATH>(w, p.M, p.pg);
             obj = (unsigned long long)T * scale;
             idx = ord * p.n_map + rank;
             ++evaluated;
@@ -231,21 +238,50 @@ pos_status launch_leaf_t(const LeafParams &p, int grid, cudaStream_t s) {
     return POS_OK;
 }
 
-// per-unit dispatchers (search_leaf_*.cu): S in the unit's range
-pos_status launch_leaf_1_6(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
-pos_status launch_leaf_7_10(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
-pos_status launch_leaf_11_12(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
-pos_status launch_leaf_13_14(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
-pos_status launch_leaf_15_15(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
-pos_status launch_leaf_16_16(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s);
+// Launch of leaf_kernel<S, path> for a runtime path of one schedule family
+// (instantiated by the search_leaf_*.cu units; S = 1 has only fast paths).
+template <int S, bool EAGER>
+pos_status launch_leaf_s(int path, const LeafParams &p, int grid, cudaStream_t s) {
+    if constexpr (EAGER) {
+        if (path == kPathEager) return launch_leaf_t<S, kPathEager>(p, grid, s);
+        if constexpr (S > 1)
+            if (path == kPathEagerShort) return launch_leaf_t<S, kPathEagerShort>(p, grid, s);
+    } else {
+        if (path == kPathFast) return launch_leaf_t<S, kPathFast>(p, grid, s);
+        if constexpr (S > 1)
+            if (path == kPathGeneric) return launch_leaf_t<S, kPathGeneric>(p, grid, s);
+    }
+    return fail(POS_EINVAL, "no such path for this stage count");
+}
 
-inline pos_status launch_leaf(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s) {
-    if (S <= 6) return launch_leaf_1_6(S, fast, p, grid, s);
-    if (S <= 10) return launch_leaf_7_10(S, fast, p, grid, s);
-    if (S <= 12) return launch_leaf_11_12(S, fast, p, grid, s);
-    if (S <= 14) return launch_leaf_13_14(S, fast, p, grid, s);
-    if (S == 15) return launch_leaf_15_15(S, fast, p, grid, s);
-    return launch_leaf_16_16(S, fast, p, grid, s);
+// per-unit dispatchers (search_leaf_*.cu): 1F1B or Eager paths, S in the
+// unit's range
+pos_status launch_leaf_1f1b_1_6(int S, int path, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_1f1b_7_10(int S, int path, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_1f1b_11_12(int S, int path, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_1f1b_13_14(int S, int path, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_1f1b_15_15(int S, int path, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_1f1b_16_16(int S, int path, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_eager_1_8(int S, int path, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_eager_9_12(int S, int path, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_eager_13_14(int S, int path, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_eager_15_15(int S, int path, const LeafParams &p, int grid, cudaStream_t s);
+pos_status launch_leaf_eager_16_16(int S, int path, const LeafParams &p, int grid, cudaStream_t s);
+
+inline pos_status launch_leaf(int S, int path, const LeafParams &p, int grid, cudaStream_t s) {
+    if (path == kPathEager || path == kPathEagerShort) {
+        if (S <= 8) return launch_leaf_eager_1_8(S, path, p, grid, s);
+        if (S <= 12) return launch_leaf_eager_9_12(S, path, p, grid, s);
+        if (S <= 14) return launch_leaf_eager_13_14(S, path, p, grid, s);
+        if (S == 15) return launch_leaf_eager_15_15(S, path, p, grid, s);
+        return launch_leaf_eager_16_16(S, path, p, grid, s);
+    }
+    if (S <= 6) return launch_leaf_1f1b_1_6(S, path, p, grid, s);
+    if (S <= 10) return launch_leaf_1f1b_7_10(S, path, p, grid, s);
+    if (S <= 12) return launch_leaf_1f1b_11_12(S, path, p, grid, s);
+    if (S <= 14) return launch_leaf_1f1b_13_14(S, path, p, grid, s);
+    if (S == 15) return launch_leaf_1f1b_15_15(S, path, p, grid, s);
+    return launch_leaf_1f1b_16_16(S, path, p, grid, s);
 }
 
 }  // namespace pos

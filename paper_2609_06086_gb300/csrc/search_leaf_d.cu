@@ -1,16 +1,16 @@
-// Instantiation unit of the search leaf kernel (see search_kernels.cuh).
+// Instantiation unit of the search leaf kernel (see search_kernels.cuh):
+// 1F1B (fast and short paths), S = 13..14.
 #include "search_kernels.cuh"
 
 namespace pos {
 
-pos_status launch_leaf_13_14(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s) {
+pos_status launch_leaf_1f1b_13_14(int S, int path, const LeafParams &p, int grid,
+                                   cudaStream_t s) {
     switch (S) {
         case 13:
-            return fast ? launch_leaf_t<13, kPathFast>(p, grid, s)
-                        : launch_leaf_t<13, kPathGeneric>(p, grid, s);
+            return launch_leaf_s<13, false>(path, p, grid, s);
         case 14:
-            return fast ? launch_leaf_t<14, kPathFast>(p, grid, s)
-                        : launch_leaf_t<14, kPathGeneric>(p, grid, s);
+            return launch_leaf_s<14, false>(path, p, grid, s);
         default:
             return fail(POS_EINVAL, "stage count outside this unit");
     }

@@ -1,13 +1,14 @@
-// Instantiation unit of the search leaf kernel (see search_kernels.cuh).
+// Instantiation unit of the search leaf kernel (see search_kernels.cuh):
+// 1F1B (fast and short paths), S = 15..15.
 #include "search_kernels.cuh"
 
 namespace pos {
 
-pos_status launch_leaf_15_15(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s) {
+pos_status launch_leaf_1f1b_15_15(int S, int path, const LeafParams &p, int grid,
+                                   cudaStream_t s) {
     switch (S) {
         case 15:
-            return fast ? launch_leaf_t<15, kPathFast>(p, grid, s)
-                        : launch_leaf_t<15, kPathGeneric>(p, grid, s);
+            return launch_leaf_s<15, false>(path, p, grid, s);
         default:
             return fail(POS_EINVAL, "stage count outside this unit");
     }

@@ -1,13 +1,14 @@
-// Instantiation unit of the search leaf kernel (see search_kernels.cuh).
+// Instantiation unit of the search leaf kernel (see search_kernels.cuh):
+// 1F1B (fast and short paths), S = 16..16.
 #include "search_kernels.cuh"
 
 namespace pos {
 
-pos_status launch_leaf_16_16(int S, bool fast, const LeafParams &p, int grid, cudaStream_t s) {
+pos_status launch_leaf_1f1b_16_16(int S, int path, const LeafParams &p, int grid,
+                                   cudaStream_t s) {
     switch (S) {
         case 16:
-            return fast ? launch_leaf_t<16, kPathFast>(p, grid, s)
-                        : launch_leaf_t<16, kPathGeneric>(p, grid, s);
+            return launch_leaf_s<16, false>(path, p, grid, s);
         default:
             return fail(POS_EINVAL, "stage count outside this unit");
     }

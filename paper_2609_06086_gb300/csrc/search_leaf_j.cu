@@ -1,0 +1,17 @@
+// Instantiation unit of the search leaf kernel (see search_kernels.cuh):
+// Eager 1F1B (fast path and level programs), S = 15..15.
+#include "search_kernels.cuh"
+
+namespace pos {
+
+pos_status launch_leaf_eager_15_15(int S, int path, const LeafParams &p, int grid,
+                                   cudaStream_t s) {
+    switch (S) {
+        case 15:
+            return launch_leaf_s<15, true>(path, p, grid, s);
+        default:
+            return fail(POS_EINVAL, "stage count outside this unit");
+    }
+}
+
+}  // namespace pos

@@ -57,6 +57,7 @@ BlobLayout make_layout(int L, int n_types, int n_tp) {
     ly.n_types = n_types;
     ly.n_tp = n_tp;
     ly.K = n_types * n_tp;
+    ly.sched = POS_SCHED_1F1B;
     const int K = ly.K, Lp1 = L + 1;
     int off = 0;
     ly.off_binom = off;
@@ -166,12 +167,13 @@ pos_status validate_tables(const pos_tables *t) {
     return POS_OK;
 }
 
-pos_status build_blob(const pos_tables *t, std::vector<unsigned char> &host, BlobLayout &ly,
-                      int64_t &guard_A, int64_t &guard_D, int64_t &guard_P) {
+pos_status build_blob(const pos_tables *t, int sched, std::vector<unsigned char> &host,
+                      BlobLayout &ly, int64_t &guard_A, int64_t &guard_D, int64_t &guard_P) {
     pos_status st = validate_tables(t);
     if (st != POS_OK) return st;
     const int L = t->L, K = t->n_types * t->n_tp, Lp1 = L + 1;
     ly = make_layout(L, t->n_types, t->n_tp);
+    ly.sched = sched;
     host.assign(ly.bytes, 0);
     // binomials by Pascal's rule (k <= 15 is exact in 64 bits for n <= 127)
     uint64_t *bn = reinterpret_cast<uint64_t *>(host.data() + ly.off_binom);  // [k][n]
@@ -224,11 +226,11 @@ pos_status launch_prefix_rows(void *d_blob, const BlobLayout &ly, cudaStream_t s
     return POS_OK;
 }
 
-pos_status create_handle(const pos_tables *t, Handle **out) {
+pos_status create_handle(const pos_tables *t, int sched, Handle **out) {
     std::vector<unsigned char> host;
     BlobLayout ly;
     int64_t A, D, P;
-    pos_status st = build_blob(t, host, ly, A, D, P);
+    pos_status st = build_blob(t, sched, host, ly, A, D, P);
     if (st != POS_OK) return st;
     Handle *h = new (std::nothrow) Handle();
     if (!h) return fail(POS_ENOMEM, "host allocation failed");
@@ -268,9 +270,10 @@ extern "C" {
 pos_status poseidon_tables_create(const pos_tables *tables, int32_t schedule, void **handle) {
     if (!handle) return pos::fail(POS_EINVAL, "handle out-pointer is NULL");
     *handle = nullptr;
-    if (schedule != POS_SCHED_1F1B) return pos::fail(POS_ENOTIMPL, "only 1F1B is implemented");
+    if (schedule != POS_SCHED_1F1B && schedule != POS_SCHED_EAGER_1F1B)
+        return pos::fail(POS_ENOTIMPL, "schedule must be POS_SCHED_1F1B or POS_SCHED_EAGER_1F1B");
     pos::Handle *h = nullptr;
-    const pos_status st = pos::create_handle(tables, &h);
+    const pos_status st = pos::create_handle(tables, schedule, &h);
     if (st == POS_OK) *handle = h;
     return st;
 }

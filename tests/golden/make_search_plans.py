@@ -1,9 +1,10 @@
 """Write tests/golden/search_plans.json: the oracle's exact search result for
-the four search workloads (configs 1-4 of gen/), so GPU tests and the bench
-can compare against the oracle without re-running its slowest search
-(config 4 takes minutes single-threaded).  Calls only oracle/ and gen/.
+the four search workloads (configs 1-4 of gen/), under 1F1B ("configN") and
+Eager 1F1B ("configN_eager"), so GPU tests and the bench can compare against
+the oracle without re-running its slowest search (config 4 takes minutes
+single-threaded).  Calls only oracle/ and gen/.
 
-    python tests/golden/make_search_plans.py [--configs 1 2 3 4]
+    python tests/golden/make_search_plans.py [--configs 1 2 3 4] [--schedules 0 1]
 """
 import argparse
 import json
@@ -23,15 +24,19 @@ OUT = os.path.join(os.path.dirname(os.path.abspath(__file__)), "search_plans.jso
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--configs", type=int, nargs="*", default=[1, 2, 3, 4])
+    ap.add_argument("--schedules", type=int, nargs="*", default=[0, 1],
+                    help="0 = 1F1B, 1 = Eager 1F1B")
     args = ap.parse_args()
     data = json.load(open(OUT)) if os.path.exists(OUT) else {}
-    for c in args.configs:
-        w = gen.get_config(c)
-        t0 = time.time()
-        plan, stats = oracle.search(w, prune=True, warmup=500, seed=0)
-        data[f"config{c}"] = dict(workload=w.name, seed=w.seed, plan=plan, oracle_stats=stats,
-                                  oracle_seconds=round(time.time() - t0, 2))
-        print(c, plan, flush=True)
+    for sched in args.schedules:
+        for c in args.configs:
+            w = gen.get_config(c)
+            t0 = time.time()
+            plan, stats = oracle.search(w, prune=True, warmup=500, seed=0, schedule=sched)
+            key = f"config{c}" + ("_eager" if sched == 1 else "")
+            data[key] = dict(workload=w.name, seed=w.seed, schedule=sched, plan=plan,
+                             oracle_stats=stats, oracle_seconds=round(time.time() - t0, 2))
+            print(key, plan, flush=True)
     with open(OUT, "w") as f:
         json.dump(data, f, indent=1, sort_keys=True)
 

@@ -82,7 +82,7 @@ def test_invalid_arguments_rejected_before_the_device(P):
     import gen
     w = gen.config1()
     t = P.Tables.from_workload(w)
-    assert L.poseidon_tables_create(C.byref(t.c), 1, C.byref(h)) == P.binding.POS_ENOTIMPL
+    assert L.poseidon_tables_create(C.byref(t.c), 2, C.byref(h)) == P.binding.POS_ENOTIMPL
     bad = P.Tables.from_workload(w)
     bad.arrays["fwd"][0, 0] = -5
     assert L.poseidon_tables_create(C.byref(bad.c), 0, C.byref(h)) == P.binding.POS_EINVAL
