@@ -130,7 +130,7 @@ def oracle_sample_rate(seconds: float, seed: int = 0):
     return n / dt, n, dt
 
 
-def eval_throughput(P, torch, n, reps, peak_alu):
+def eval_throughput(P, torch, n, reps, peak_alu, schedule=0):
     """poseidon_eval_batch on n config-5 candidates (L=64, S ~ U{2..16},
     M ~ U{8..128}, 2 device types), device-resident, timed with CUDA events
     on the launching stream; inputs (16 B x n) exceed L2 for n >= 1e7."""
@@ -140,7 +140,7 @@ def eval_throughput(P, torch, n, reps, peak_alu):
     M = c["M"].astype(np.int64)
     relax = int((2 * S * M).sum())
     ops = 3 * relax + 11 * int(S.sum())  # 6SM + 11S integer ops per candidate
-    h = P.Handle(P.Tables.from_workload(w))
+    h = P.Handle(P.Tables.from_workload(w), schedule=schedule)
     d_c = torch.from_numpy(c.view(np.uint8)).cuda()
     del c
     d_T = torch.empty(n, dtype=torch.int32, device="cuda")
@@ -163,6 +163,7 @@ def eval_throughput(P, torch, n, reps, peak_alu):
     h.close()
     ach = ops / sec / 1e12
     return {"workload": "config 5: L=64, S~U{2..16}, M~U{8..128}, 2 device types",
+            "schedule": "Eager 1F1B" if schedule == 1 else "1F1B",
             "batch": n, "ms_per_call": round(sec * 1e3, 4), "evals_per_s": n / sec,
             "relaxations_per_s": relax / sec, "bound": "alu", "achieved": round(ach, 3),
             "unit": "Tops/s", "peak": round(peak_alu, 3), "frac": round(ach / peak_alu, 4)}
@@ -326,6 +327,29 @@ def run_ours(args, rank, world, local_rank):
             "peak_note": (f"{n_sm} SMs x {SM_LANES} int32 lanes x {mhz:.0f} MHz (median SM "
                           "clock under load)" if b == "alu" else hbm_src)}
     evals = [eval_throughput(P, torch, int(n), 5, peak_alu) for n in args.eval_sizes]
+    evals_eager = [eval_throughput(P, torch, int(n), 5, peak_alu, schedule=1)
+                   for n in args.eval_sizes[:1]]
+    # the same search under Eager 1F1B (App. B schedule), for comparison
+    ref_e = _json.load(open(os.path.join(ROOT, "tests", "golden", "search_plans.json")))
+    ref_e = ref_e.get("config4_eager", {}).get("plan", {})
+    prob_e, keep_e = P.make_problem(w, warmup=WARMUP_SAMPLES, prune=args.prune, seed=0,
+                                    frontier_cap=args.frontier_cap, schedule=1)
+    P.poseidon_search(prob_e)
+    e_ms, e_ev, e_ok = [], 0, True
+    for _ in range(max(3, args.steps // 2)):
+        flush.zero_()
+        torch.cuda.synchronize()
+        ev0.record()
+        plan_e, st_e = P.poseidon_search(prob_e)
+        ev1.record()
+        torch.cuda.synchronize()
+        e_ms.append(ev0.elapsed_time(ev1))
+        e_ev += st_e["evaluated"]
+        e_ok &= plan_e["global_index"] == ref_e.get("global_index")
+    eager_search = {"schedule": "Eager 1F1B", "prune": PRUNE_NAMES[args.prune],
+                    "time_to_plan_s": sum(e_ms) / len(e_ms) / 1e3,
+                    "evaluations_per_step": e_ev / len(e_ms), "T_us": plan_e["T"],
+                    "matches_oracle": e_ok}
     # the other stage-level prune, same workload, for comparison (not the headline)
     other = PRUNE_NAMES[1 if args.prune == 2 else 2]
     other_mode = 1 if args.prune == 2 else 2
@@ -371,6 +395,8 @@ def run_ours(args, rank, world, local_rank):
         "roofline": roof,
         "other_prune": other_prune,
         "eval_throughput": evals,
+        "eval_throughput_eager": evals_eager,
+        "eager_search": eager_search,
         "cpu_baseline": {"value": cpu_rate, "unit": "evals/s", "cores": 1, "kind": "oracle",
                          "sample": f"{cpu_n} config-4 plan evaluations (S=8, M=32, L=80) in "
                                    f"{cpu_t:.1f} s, single-threaded oracle"},
