@@ -35,7 +35,8 @@ class Tables(C.Structure):
 
 class Problem(C.Structure):
     _fields_ = [("tab", Tables), ("S", C.c_int32), ("n_M", C.c_int32), ("M_list", C.c_void_p),
-                ("dp_list", C.c_void_p), ("placement", C.c_int32), ("type_counts", C.c_void_p)]
+                ("dp_list", C.c_void_p), ("placement", C.c_int32), ("type_counts", C.c_void_p),
+                ("ridge", C.c_int32)]
 
 
 class Plan(C.Structure):
@@ -48,7 +49,8 @@ class Plan(C.Structure):
 
 class Stats(C.Structure):
     _fields_ = [("leaves_evaluated", C.c_uint64), ("prefixes_pruned", C.c_uint64),
-                ("prefixes_memory", C.c_uint64), ("warmup_evaluated", C.c_uint64)]
+                ("prefixes_memory", C.c_uint64), ("warmup_evaluated", C.c_uint64),
+                ("prefixes_ridge", C.c_uint64)]
 
 
 class DagCounts(C.Structure):
@@ -204,14 +206,14 @@ def eval_batch(tab: OracleTables, cands: np.ndarray):
 
 
 def search(w, prune=True, warmup=0, seed=0, tab: OracleTables | None = None,
-           schedule=SCHED_1F1B):
+           schedule=SCHED_1F1B, ridge=False):
     """Exact search over a gen.Workload search problem.  Returns (plan dict, stats dict)."""
     tab = tab or OracleTables.from_workload(w, schedule)
     M_list = _i32(w.M_list)
     dp = _i32(w.dp_list)
     tc = _i32(w.type_counts if w.type_counts else [0] * w.n_types)
     p = Problem(tab.c, w.S, len(M_list), M_list.ctypes.data, dp.ctypes.data, w.placement,
-                tc.ctypes.data)
+                tc.ctypes.data, int(bool(ridge)))
     plan, st = Plan(), Stats()
     rc = lib().orc_search(C.byref(p), int(prune), int(warmup), C.c_uint64(seed), C.byref(plan),
                           C.byref(st))

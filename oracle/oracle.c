@@ -560,7 +560,7 @@ int orc_eval_batch(const orc_tables *t, const orc_candidate *c, int64_t n, int32
 /* ------------------------------------------------------------------ */
 typedef struct {
     const orc_problem *p;
-    int S, L, M, D, m_idx, tp_idx, prune;
+    int S, L, M, D, m_idx, tp_idx, prune, ridge;
     uint64_t place_rank, n_place, n_map;
     int32_t cls[ORC_MAX_S], types[ORC_MAX_S], layers[ORC_MAX_S];
     unsigned char *feas; /* feas[x*(L+1)+c]: layers [c, L) fit stages x..S-1 */
@@ -607,6 +607,23 @@ static void consider_leaf(search_ctx *cx) {
     }
 }
 
+/* Layer-level pruning (Theorem 2): among the stages 0..x (0-based) placed so
+ * far, the layer counts of the stages of each device type, in stage order,
+ * must never rise again after they have fallen (a ridge: non-decreasing,
+ * then non-increasing).  A prefix that breaks this has no ridge completion. */
+static int ridge_ok(const int32_t *types, const int32_t *layers, int n) {
+    for (int a = 0; a < n; ++a) {
+        int fallen = 0, prev = -1;
+        for (int s = 0; s < n; ++s) {
+            if (types[s] != types[a]) continue;
+            if (prev >= 0 && layers[s] < prev) fallen = 1;
+            if (prev >= 0 && layers[s] > prev && fallen) return 0;
+            prev = layers[s];
+        }
+    }
+    return 1;
+}
+
 /* Prefix S_x (stages 0..x-1 placed, 1-based x) is cut when its lower bound
  * exceeds the incumbent: g(S_x)/(D M) > T_inc/(D_inc M_inc), i.e. it is strictly worse. */
 static int pruned_by_bound(search_ctx *cx, int x) {
@@ -628,6 +645,10 @@ static void dfs(search_ctx *cx, int x, int used) {
         if (!stage_memory_ok(&cx->p->tab, S, cx->M, x, cx->cls[x], used, l) ||
             !cx->feas[(x + 1) * (L + 1) + used + l]) {
             cx->st->prefixes_memory++;
+            continue;
+        }
+        if (cx->ridge && !ridge_ok(cx->types, cx->layers, x + 1)) {
+            cx->st->prefixes_ridge++;
             continue;
         }
         /* the stage-x bound uses only stages 0..x, which are all fixed now */
@@ -728,6 +749,7 @@ int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_p
     cx.S = S;
     cx.L = L;
     cx.prune = prune;
+    cx.ridge = p->ridge;
     cx.best = plan;
     cx.st = stats;
     cx.n_map = n_comp(L, S);
@@ -766,7 +788,8 @@ int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_p
                     used += cx.layers[x];
                 }
                 stats->warmup_evaluated++;
-                consider_leaf(&cx);
+                /* with layer-level pruning only ridge-like plans can be the result */
+                if (!cx.ridge || ridge_ok(cx.types, cx.layers, cx.S)) consider_leaf(&cx);
             }
             free(places);
         }

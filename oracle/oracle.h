@@ -58,6 +58,9 @@ typedef struct {
     const int32_t *dp_list;     /* [n_tp] data-parallel degree D per TP index */
     int32_t placement;          /* 0 = any type per stage, 1 = exact per-type stage counts */
     const int32_t *type_counts; /* [n_types] (placement 1) */
+    int32_t ridge;              /* 1: layer-level pruning (Theorem 2): only plans whose
+                                   layer counts over the stages of each device type
+                                   rise, then fall ("ridge-like") */
 } orc_problem;
 
 typedef struct {
@@ -73,6 +76,7 @@ typedef struct {
     uint64_t prefixes_pruned;   /* partial configurations cut by g(S_x) > T_min */
     uint64_t prefixes_memory;   /* partial configurations cut by memory */
     uint64_t warmup_evaluated;
+    uint64_t prefixes_ridge;    /* partial configurations cut by the ridge rule */
 } orc_stats;
 
 typedef struct {
