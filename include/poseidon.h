@@ -222,6 +222,12 @@ typedef struct pos_problem {
                                    raised to at least 32*L */
     int32_t profile;            /* 1: device time per kernel kind in the stats (CUDA
                                    events around every launch); 0: those fields are 0 */
+    int32_t ridge;              /* 1: layer-level pruning (Theorem 2): only plans whose
+                                   layer counts over the stages of each device type rise,
+                                   then fall ("ridge-like") are enumerated or returned.
+                                   Theorem 2 guarantees a ridge-like optimum only under
+                                   its assumptions: the result may be worse than the
+                                   exact optimum (never better); 0: exact search */
 } pos_problem;
 
 typedef struct pos_plan {
@@ -263,6 +269,7 @@ typedef struct pos_search_stats {
     uint64_t launches_depth[POS_MAX_STAGES];
     uint64_t parents_depth[POS_MAX_STAGES];
     uint64_t children_depth[POS_MAX_STAGES];
+    uint64_t pruned_ridge;      /* children cut by the layer-level (ridge) rule */
 } pos_search_stats;
 
 /*

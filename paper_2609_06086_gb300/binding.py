@@ -42,7 +42,7 @@ class pos_problem(C.Structure):
                 ("M_list", C.c_void_p), ("tp_list", C.c_void_p), ("dp_list", C.c_void_p),
                 ("placement", C.c_int32), ("type_counts", C.c_void_p), ("warmup", C.c_int32),
                 ("prune", C.c_int32), ("seed", C.c_uint64), ("schedule", C.c_int32),
-                ("frontier_cap", C.c_int64), ("profile", C.c_int32)]
+                ("frontier_cap", C.c_int64), ("profile", C.c_int32), ("ridge", C.c_int32)]
 
 
 class pos_plan(C.Structure):
@@ -64,7 +64,8 @@ class pos_search_stats(C.Structure):
                                           "leaves")] + \
                [("ms_bound", C.c_double), ("bound_launches", C.c_uint64), ("reruns", C.c_uint64),
                 ("ms_depth", C.c_double * 16), ("launches_depth", C.c_uint64 * 16),
-                ("parents_depth", C.c_uint64 * 16), ("children_depth", C.c_uint64 * 16)]
+                ("parents_depth", C.c_uint64 * 16), ("children_depth", C.c_uint64 * 16),
+                ("pruned_ridge", C.c_uint64)]
 
 
 class PoseidonError(RuntimeError):
@@ -185,7 +186,7 @@ def _prune_mode(prune):
 
 
 def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0, profile=False,
-                 schedule=POS_SCHED_1F1B):
+                 schedule=POS_SCHED_1F1B, ridge=False):
     """pos_problem for a gen.Workload search; returns (problem, keep-alive list)."""
     tab = Tables.from_workload(w)
     keep = [tab]
@@ -198,7 +199,7 @@ def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0, profile=Fals
     p = pos_problem(tab.c, w.S, len(w.M_list), arr(w.M_list), arr(w.tp_list), arr(w.dp_list),
                     w.placement, arr(w.type_counts if w.type_counts else [0] * w.n_types),
                     int(warmup), _prune_mode(prune), int(seed), int(schedule), int(frontier_cap),
-                    int(bool(profile)))
+                    int(bool(profile)), int(bool(ridge)))
     return p, keep
 
 

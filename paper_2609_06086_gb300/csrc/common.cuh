@@ -700,6 +700,37 @@ __host__ __device__ __forceinline__ int path_of(int sched, int S, int M) {
                                          : (fast ? kPathFast : kPathGeneric);
 }
 
+// ---------------------------------------------------------------------------
+// Layer-level pruning (Theorem 2): for each device type the layer counts of
+// its stages, in stage order, rise and then fall ("ridge-like").  A partial
+// plan keeps one byte per type: bits 0-6 = layers of the type's last placed
+// stage (0 = none yet), bit 7 = its counts have fallen; a type whose counts
+// have fallen caps its next stage at its last count.
+// ---------------------------------------------------------------------------
+__host__ __device__ __forceinline__ int ridge_cap(uint32_t state, int type) {
+    const uint32_t b = (state >> (8 * type)) & 0xffu;
+    return (b & 0x80u) ? (int)(b & 0x7fu) : 127;
+}
+__host__ __device__ __forceinline__ uint32_t ridge_next(uint32_t state, int type, int l) {
+    const uint32_t b = (state >> (8 * type)) & 0xffu, last = b & 0x7fu;
+    const uint32_t fallen = (b & 0x80u) | ((last != 0u && (uint32_t)l < last) ? 0x80u : 0u);
+    return (state & ~(0xffu << (8 * type))) | ((fallen | (uint32_t)l) << (8 * type));
+}
+// Is a complete plan ridge-like?  cut[0..S], cls[s] = type * n_tp + tp.
+template <int S>
+__device__ __forceinline__ bool ridge_plan_ok(const int (&cut)[S + 1], const int (&cls)[S],
+                                              int n_tp) {
+    uint32_t st = 0;
+    bool ok = true;
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+        const int ty = cls[s] / n_tp, l = cut[s + 1] - cut[s];
+        ok &= l <= ridge_cap(st, ty);
+        st = ridge_next(st, ty, l);
+    }
+    return ok;
+}
+
 // Overflow guard U(S, M) >= 2^31 ?
 __host__ __device__ __forceinline__ bool guard_trips(int64_t A, int64_t D, int64_t P, int S,
                                                      int M) {

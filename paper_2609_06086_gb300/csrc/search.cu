@@ -314,6 +314,7 @@ struct ExpandParams {
     int x;                   // depth of the parents (stages 0..x-1 placed)
     int S, M;
     int prune;
+    int ridge;               // 1: layer-level (ridge) pruning
     int exact;               // 1: host-driven pass (lane-per-parent mode with deferral lists)
     const SliceRec *slices;
     const uint4 *feas;
@@ -354,7 +355,22 @@ struct ParentCtx {
     int c, k;
     int32_t f0, b0, d0;
     int32_t pf, pb;  // prune 2: F and B edge between the new stage and the next one
+    // ridge rule: state of the prefix, device types of the new and the next
+    // stage, most layers the new stage may take (127: no cap)
+    uint32_t rstate;
+    int rta, rtb, rcap;
 };
+
+// Ridge fields of a parent (when the rule is on): its state word, the types
+// of stages X and X+1, and the cap on stage X's layers.
+__device__ __forceinline__ void ridge_ctx(ParentCtx &q, bool on, uint32_t state, int ka, int kb,
+                                          int n_tp) {
+    if (!on) return;
+    q.rstate = state;
+    q.rta = ka / n_tp;
+    q.rtb = kb / n_tp;
+    q.rcap = ridge_cap(state, q.rta);
+}
 
 __device__ __forceinline__ ParentCtx parent_ctx(const Tab &t, int k, int c) {
     ParentCtx q;
@@ -365,6 +381,9 @@ __device__ __forceinline__ ParentCtx parent_ctx(const Tab &t, int k, int c) {
     q.d0 = Pd(t, k, c);
     q.pf = 0;
     q.pb = 0;
+    q.rstate = 0;
+    q.rta = q.rtb = 0;
+    q.rcap = 127;
     return q;
 }
 
@@ -378,10 +397,12 @@ __device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, i
                                           int64_t Bm, const ParentCtx &q, uint32_t gid,
                                           const int2 *vrow, uint64_t scale,
                                           uint64_t thr, Bits128 &acc, unsigned long long &cut_b,
-                                          unsigned long long &cut_m) {
+                                          unsigned long long &cut_m, unsigned long long &cut_r) {
     const int S = p.S, M = p.M, x = p.x, L = t.L();
     const int lmax = L - q.c - (S - x - 1);
-    const int hi_mem = min(lmax, (int)__ldg(p.lim + ((size_t)gid * S + x) * 128 + q.c));
+    const int hi_mem0 = min(lmax, (int)__ldg(p.lim + ((size_t)gid * S + x) * 128 + q.c));
+    const int hi_mem = min(hi_mem0, q.rcap);  // ridge rule: a cap on the layer count
+    cut_r += (unsigned long long)(hi_mem0 - hi_mem);
     int hi = hi_mem;
     if (p.prune) {  // g(S_{x+1}) grows with l: binary search for the last l within the bound
         int lo = 0;
@@ -400,7 +421,7 @@ __device__ __forceinline__ int expand_set(const ExpandParams &p, const Tab &t, i
     acc.w[2] = f.z & win.w[2];
     acc.w[3] = f.w & win.w[3];
     int n = popc128(acc);
-    cut_m += (unsigned long long)(lmax - hi_mem) + (unsigned long long)(hi - n);
+    cut_m += (unsigned long long)(lmax - hi_mem0) + (unsigned long long)(hi - n);
     cut_b += (unsigned long long)(hi_mem - hi);
     if (p.prune == 2 && n > 0) {
         // completion terms: the bound is not monotone in l, so every
@@ -448,11 +469,13 @@ __device__ __forceinline__ int complete_set(const ExpandParams &p, const Tab &t,
                                             int64_t Bm, const ParentCtx &q, int kb, uint32_t gid,
                                             uint64_t scale,
                                             uint64_t thr, Bits128 &acc, unsigned long long &cut_b,
-                                            unsigned long long &cut_m) {
+                                            unsigned long long &cut_m, unsigned long long &cut_r) {
     const int S = p.S, M = p.M, L = t.L(), a = S - 2, b = S - 1;
     const int c = q.c;
     const int lmax = L - c - 1;
-    const int hi_mem = min(lmax, (int)__ldg(p.lim + ((size_t)gid * S + a) * 128 + c));
+    const int hi_mem0 = min(lmax, (int)__ldg(p.lim + ((size_t)gid * S + a) * 128 + c));
+    const int hi_mem = min(hi_mem0, q.rcap);
+    cut_r += (unsigned long long)(hi_mem0 - hi_mem);
     int hi = hi_mem;
     if (p.prune) {  // g(S_{S-1}) grows with l
         int lo = 0;
@@ -478,6 +501,11 @@ __device__ __forceinline__ int complete_set(const ExpandParams &p, const Tab &t,
     const int32_t fbL = Pf(t, kb, L), bbL = Pb(t, kb, L), dbL = Pd(t, kb, L);
     for (int l = lo; l <= hi; ++l) {
         const int c2 = c + l;
+        // ridge rule for the last stage, after this one took l layers
+        if (p.ridge && L - c2 > ridge_cap(ridge_next(q.rstate, q.rta, l), q.rtb)) {
+            ++cut_r;
+            continue;
+        }
         if (p.prune) {
             const int64_t Fa = Pf(t, q.k, c2) - q.f0, Ba = Pb(t, q.k, c2) - q.b0;
             const int64_t da = Pd(t, q.k, c2) - q.d0;
@@ -494,7 +522,7 @@ __device__ __forceinline__ int complete_set(const ExpandParams &p, const Tab &t,
         for (int wd = 0; wd < 4; ++wd) acc.w[wd] |= (c2 >> 5) == wd ? 1u << (c2 & 31) : 0u;
         ++n;
     }
-    cut_m += (unsigned long long)(lmax - hi_mem) + (unsigned long long)(lo - 1 < hi ? lo - 1 : hi);
+    cut_m += (unsigned long long)(lmax - hi_mem0) + (unsigned long long)(lo - 1 < hi ? lo - 1 : hi);
     cut_b += (unsigned long long)(hi_mem - hi);
     return n;
 }
@@ -514,6 +542,7 @@ __device__ __forceinline__ void level_warp_mode(const ExpandParams &p, const Tab
                                                 const int2 *vdepth, uint64_t thr,
                                                 unsigned long long &emitted,
                                                 unsigned long long &cb, unsigned long long &cm,
+                                                unsigned long long &cr,
                                                 unsigned long long &written) {
     const int lane = threadIdx.x & 31;
     const unsigned lt_mask = (1u << lane) - 1u;
@@ -526,22 +555,24 @@ __device__ __forceinline__ void level_warp_mode(const ExpandParams &p, const Tab
         if (slice == kPrefixHole) continue;
         const SliceRec &sr = p.slices[slice];
         const int c = X > 0 ? (int)get_byte<(X > 0 ? X + 1 : 2)>(pv) : 0;
-        const ParentCtx q = parent_ctx(t, sr.cls[X], c);
+        ParentCtx q = parent_ctx(t, sr.cls[X], c);
         const int kb = sr.cls[X + 1];  // X + 1 <= S - 1
+        ridge_ctx(q, p.ridge != 0, pv.b.z, q.k, kb, t.n_tp());
         const int32_t pf = p.prune == 2 ? p2f(t, q.k, kb) : 0;
         const int32_t pb = p.prune == 2 ? p2b(t, kb, q.k) : 0;
         const uint64_t scale = sr.scale;
         const uint32_t gid = sr.gid;
         const int64_t A = (int32_t)pv.b.x, Bm = (int32_t)pv.b.y;
         const int lmax = COMPLETE ? L - c - 1 : L - c - (S - X - 1);
-        const int hi_mem = min(lmax, (int)__ldg(p.lim + ((size_t)gid * S + X) * 128 + c));
+        const int hi_mem0 = min(lmax, (int)__ldg(p.lim + ((size_t)gid * S + X) * 128 + c));
+        const int hi_mem = min(hi_mem0, q.rcap);  // ridge rule: a cap on the layer count
         // expansion: the next stage must fit from c + l (row X+1); completion:
         // stage S-1 must hold [c + l, L) (row S-1)
         const uint4 f = __ldg(p.feas + (size_t)gid * (S + 1) + (COMPLETE ? S - 1 : X + 1));
         const int2 *vrow = vsm ? vsm + (size_t)slice * 128
                                : (vdepth ? vdepth + (size_t)sr.vslot * 128 : nullptr);
         unsigned pass[4];
-        int n_bound = 0, n_win = 0, n_fail = 0;
+        int n_bound = 0, n_win = 0, n_fail = 0, n_ridge_b = 0;
 #pragma unroll
         for (int r = 0; r < 4; ++r) {
             const int l = 1 + lane + 32 * r;
@@ -556,6 +587,10 @@ __device__ __forceinline__ void level_warp_mode(const ExpandParams &p, const Tab
                 const uint32_t word2 = (c2 >> 5) == 0 ? f.x : (c2 >> 5) == 1 ? f.y
                                      : (c2 >> 5) == 2 ? f.z : f.w;
                 cand = g_ok && ((word2 >> (c2 & 31)) & 1u);
+                // ridge rule for the last stage, after this one took l layers
+                if (COMPLETE && cand && p.ridge &&
+                    L - c2 > ridge_cap(ridge_next(q.rstate, q.rta, l), q.rtb))
+                    cand = false, ++n_ridge_b;
                 ok = cand;
                 if (cand) {
                     const int64_t A2 = A + F + pf, Bm2 = max(Bm, d) + B + pb;
@@ -580,9 +615,14 @@ __device__ __forceinline__ void level_warp_mode(const ExpandParams &p, const Tab
             n_fail += __popc(__ballot_sync(0xffffffffu, cand && !ok));
         }
         const int total = __popc(pass[0]) + __popc(pass[1]) + __popc(pass[2]) + __popc(pass[3]);
+        // lanes cut by the last-stage ridge test, summed over the warp
+        int r_sum = n_ridge_b;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) r_sum += __shfl_xor_sync(0xffffffffu, r_sum, o);
         if (lane == 0) {
-            cm += (unsigned long long)(lmax - hi_mem) + (unsigned long long)(n_bound - n_win);
+            cm += (unsigned long long)(lmax - hi_mem0) + (unsigned long long)(n_bound - n_win - r_sum);
             cb += (unsigned long long)(hi_mem - n_bound) + (unsigned long long)n_fail;
+            cr += (unsigned long long)(hi_mem0 - hi_mem) + (unsigned long long)r_sum;
             written += 1;
         }
         if (total == 0) continue;
@@ -623,7 +663,8 @@ __device__ __forceinline__ void level_warp_mode(const ExpandParams &p, const Tab
                     const int32_t d = Pd(t, q.k, c2) - q.d0;
                     out.a = pv.a;
                     out.b = make_uint4((uint32_t)((int32_t)pv.b.x + F + pf),
-                                       (uint32_t)(max((int32_t)pv.b.y, d) + B + pb), 0u, 0u);
+                                       (uint32_t)(max((int32_t)pv.b.y, d) + B + pb),
+                                       p.ridge ? ridge_next(q.rstate, q.rta, c2 - c) : 0u, 0u);
                     set_byte<2 + (X < 14 ? X : 0)>(out, (uint32_t)c2);
                     store32(p.out + at, out);
                 }
@@ -639,7 +680,7 @@ __device__ __forceinline__ void level_warp_mode(const ExpandParams &p, const Tab
 // output slots with one atomic and writes them -- or, when the output is
 // full, marks its reserved slots as holes and defers the group.
 template <bool COMPLETE, int X>
-__global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(ExpandParams p) {
+__global__ void __launch_bounds__(kThreads, 3) level_kernel(ExpandParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
     long long n_in = p.n_in;
     if (p.n_in_dev) {
@@ -680,9 +721,9 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
     const uint64_t thr = p.prune ? __ldcg(&p.inc->obj) : ~0ull;
     const int lane = threadIdx.x & 31;
     const long long warp = (blockIdx.x * (long long)blockDim.x + threadIdx.x) >> 5;
-    unsigned long long emitted = 0, cb = 0, cm = 0, written_parents = 0;
+    unsigned long long emitted = 0, cb = 0, cm = 0, cr = 0, written_parents = 0;
     if (warp_mode)
-        level_warp_mode<COMPLETE, X>(p, t, n_in, vsm, vdepth, thr, emitted, cb, cm,
+        level_warp_mode<COMPLETE, X>(p, t, n_in, vsm, vdepth, thr, emitted, cb, cm, cr,
                                      written_parents);
     for (long long w = warp; !warp_mode && w < n_work; w += n_warps) {
         const long long g = p.groups ? (long long)p.groups[w] : w;
@@ -692,7 +733,7 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
         const uint32_t slice = pv.a.x & 0xffffu;
         const bool live = slice != kPrefixHole;
         Bits128 acc = {{0u, 0u, 0u, 0u}};
-        unsigned long long lb = 0, lm = 0;
+        unsigned long long lb = 0, lm = 0, lr = 0;
         int n = 0;
         ParentCtx q = {0, 0, 0, 0, 0};
         if (live) {
@@ -701,6 +742,7 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
             // parent byte 2+i holds cut[i]
             const int c = X > 0 ? (int)get_byte<(X > 0 ? X + 1 : 2)>(pv) : 0;
             q = parent_ctx(t, sr.cls[X], c);
+            ridge_ctx(q, p.ridge != 0, pv.b.z, sr.cls[X], sr.cls[X + 1], t.n_tp());
             if (p.prune == 2) {  // X + 1 <= S - 1: the next stage exists
                 q.pf = p2f(t, sr.cls[X], sr.cls[X + 1]);
                 q.pb = p2b(t, sr.cls[X + 1], sr.cls[X]);
@@ -708,12 +750,11 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
             const uint64_t scale = sr.scale;
             const int64_t A = (int32_t)pv.b.x, Bm = (int32_t)pv.b.y;
             n = COMPLETE ? complete_set(p, t, A, Bm, q, sr.cls[X + 1], sr.gid, scale, thr, acc, lb,
-                                        lm)
+                                        lm, lr)
                          : expand_set(p, t, A, Bm, q, sr.gid,
                                       vsm ? vsm + (size_t)slice * 128
                                           : (vdepth ? vdepth + (size_t)sr.vslot * 128 : nullptr),
-                                      scale, thr, acc,
-                                      lb, lm);
+                                      scale, thr, acc, lb, lm, lr);
         }
         int incl = n;
 #pragma unroll
@@ -728,6 +769,7 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
         if (total == 0) {
             cb += lb;
             cm += lm;
+            cr += lr;
             written_parents += live;
             continue;
         }
@@ -756,6 +798,7 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
                         ch.b.x = (uint32_t)((int32_t)pv.b.x + (Pf(t, q.k, c2) - q.f0) + q.pf);
                         ch.b.y = (uint32_t)(max((int32_t)pv.b.y, Pd(t, q.k, c2) - q.d0) +
                                             (Pb(t, q.k, c2) - q.b0) + q.pb);
+                        ch.b.z = p.ridge ? ridge_next(q.rstate, q.rta, c2 - q.c) : 0u;
                         store32(p.out + pos++, ch);
                     }
                 }
@@ -763,6 +806,7 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
             emitted += n;
             cb += lb;
             cm += lm;
+            cr += lr;
             written_parents += live;
         } else {
             // no room: mark this warp's reserved slots below cap as holes
@@ -783,9 +827,11 @@ __global__ void __launch_bounds__(kThreads, COMPLETE ? 3 : 4) level_kernel(Expan
         emitted += __shfl_xor_sync(0xffffffffu, emitted, o);
         cb += __shfl_xor_sync(0xffffffffu, cb, o);
         cm += __shfl_xor_sync(0xffffffffu, cm, o);
+        cr += __shfl_xor_sync(0xffffffffu, cr, o);
         written_parents += __shfl_xor_sync(0xffffffffu, written_parents, o);
     }
     if (lane == 0) {
+        if (cr) atomicAdd(p.stats + kStPrunedRidge, cr);
         if (emitted) atomicAdd(p.stats + (COMPLETE ? kStLeaves : kStPrefixes), emitted);
         if (cb) atomicAdd(p.stats + kStPrunedBound, cb);
         if (cm) atomicAdd(p.stats + kStPrunedMemory, cm);
@@ -932,6 +978,7 @@ static pos_status validate_problem(const pos_problem *p) {
     }
     if (p->warmup < 0) return fail(POS_EINVAL, "warmup < 0");
     if (p->prune < 0 || p->prune > 2) return fail(POS_EINVAL, "prune must be 0, 1 or 2");
+    if (p->ridge != 0 && p->ridge != 1) return fail(POS_EINVAL, "ridge must be 0 or 1");
     if (p->frontier_cap < 0) return fail(POS_EINVAL, "frontier_cap < 0");
     return POS_OK;
 }
@@ -1056,6 +1103,7 @@ static ExpandParams base_params(Search &s, const SliceRec *batch, int M) {
     p.S = s.S;
     p.M = M;
     p.prune = s.pb->prune;
+    p.ridge = s.pb->ridge;
     p.slices = batch;
     p.feas = static_cast<const uint4 *>(s.d_feas.p);
     p.lim = static_cast<const uint8_t *>(s.ws.d_lim.p);
@@ -1087,6 +1135,7 @@ static pos_status run_leaves(Search &s, const Leaf *leaves, unsigned long long *
     lp.lay = s.h->lay;
     s.launches++;
     lp.pg = s.pg;
+    lp.ridge = s.pb->ridge;
     return launch_leaf(s.S, path_of(s.pb->schedule, s.S, M), lp, s.grid_leaf, s.stream);
 }
 
@@ -1596,6 +1645,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         stats->prefixes = hs[kStPrefixes];
         stats->pruned_bound = hs[kStPrunedBound];
         stats->pruned_memory = hs[kStPrunedMemory];
+        stats->pruned_ridge = hs[kStPrunedRidge];
         stats->relaxations = hs[kStRelaxations];
         stats->slices = (uint64_t)n_slices;
         stats->slices_feasible = n_feasible;

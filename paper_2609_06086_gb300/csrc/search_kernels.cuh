@@ -96,6 +96,7 @@ enum {
     kStParentsExpand,
     kStParentsComplete,
     kStLeaves,
+    kStPrunedRidge,   // children cut by the layer-level (ridge) rule
     kStDepthParents,                                // + x: parents read at depth x
     kStDepthChildren = kStDepthParents + POS_MAX_STAGES,  // + x: children (plans) written
     kStCount = kStDepthChildren + POS_MAX_STAGES
@@ -142,6 +143,7 @@ struct LeafParams {
     const void *blob;
     BlobLayout lay;
     Programs pg;  // level programs of the schedule's short path
+    int ridge;    // 1: only ridge-like plans may lower the incumbent (warm-up plans)
 };
 
 // leaf byte 4+s holds cut[s+1] (layers of stages 0..s)
@@ -199,6 +201,8 @@ __global__ void __launch_bounds__(256, leaf_min_blocks(S, PATH)) leaf_kernel(Lea
             for (int s = 0; s < S; ++s) cls[s] = __ldg(&sr.cls[s]);
             const uint64_t scale = __ldg(&sr.scale);
             const uint64_t ord = __ldg(&sr.ordinal);
+            // enumerated plans are ridge-like already; warm-up plans may not be
+            const bool admissible = !p.ridge || ridge_plan_ok<S>(cut, cls, t.n_tp());
             const uint64_t rank = rank_cuts<S>(t, cut);
             StageW<S> w;
             stage_weights<S>(t, cut, cls, w);
@@ -206,7 +210,8 @@ __global__ void __launch_bounds__(256, leaf_min_blocks(S, PATH)) leaf_kernel(Lea
             obj = (unsigned long long)T * scale;
             idx = ord * p.n_map + rank;
             ++evaluated;
-            if (p.slice_best) atomicMin(p.slice_best + sl, obj);
+            if (p.slice_best) atomicMin(p.slice_best + sl, obj);  // ordering hint only
+            if (!admissible) obj = idx = ~0ull;
         }
         // warp minimum, then one CAS attempt per warp
 #pragma unroll

@@ -4,7 +4,10 @@ Eager 1F1B ("configN_eager"), so GPU tests and the bench can compare against
 the oracle without re-running its slowest search (config 4 takes minutes
 single-threaded).  Calls only oracle/ and gen/.
 
-    python tests/golden/make_search_plans.py [--configs 1 2 3 4] [--schedules 0 1]
+    python tests/golden/make_search_plans.py [--configs 1 2 3 4] [--schedules 0 1] [--ridge]
+
+With --ridge the searches use the layer-level (ridge) rule of Theorem 2 and
+are stored as "configN_ridge" / "configN_eager_ridge".
 """
 import argparse
 import json
@@ -26,15 +29,18 @@ def main():
     ap.add_argument("--configs", type=int, nargs="*", default=[1, 2, 3, 4])
     ap.add_argument("--schedules", type=int, nargs="*", default=[0, 1],
                     help="0 = 1F1B, 1 = Eager 1F1B")
+    ap.add_argument("--ridge", action="store_true", help="layer-level (ridge) pruning")
     args = ap.parse_args()
     data = json.load(open(OUT)) if os.path.exists(OUT) else {}
     for sched in args.schedules:
         for c in args.configs:
             w = gen.get_config(c)
             t0 = time.time()
-            plan, stats = oracle.search(w, prune=True, warmup=500, seed=0, schedule=sched)
-            key = f"config{c}" + ("_eager" if sched == 1 else "")
-            data[key] = dict(workload=w.name, seed=w.seed, schedule=sched, plan=plan,
+            plan, stats = oracle.search(w, prune=True, warmup=500, seed=0, schedule=sched,
+                                        ridge=args.ridge)
+            key = f"config{c}" + ("_eager" if sched == 1 else "") + ("_ridge" if args.ridge else "")
+            data[key] = dict(workload=w.name, seed=w.seed, schedule=sched, ridge=args.ridge,
+                             plan=plan,
                              oracle_stats=stats, oracle_seconds=round(time.time() - t0, 2))
             print(key, plan, flush=True)
     with open(OUT, "w") as f:
