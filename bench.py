@@ -346,6 +346,30 @@ def run_ours(args, rank, world, local_rank):
         e_ms.append(ev0.elapsed_time(ev1))
         e_ev += st_e["evaluated"]
         e_ok &= plan_e["global_index"] == ref_e.get("global_index")
+    # layer-level (ridge) pruning, Theorem 2: value against the exact optimum
+    ridge_lines = []
+    for sched, exact_ms, exact_T in ((0, t_dev / args.steps, plans[-1]["T"]),
+                                     (1, sum(e_ms) / len(e_ms), plan_e["T"])):
+        prob_r, keep_r = P.make_problem(w, warmup=WARMUP_SAMPLES, prune=args.prune, seed=0,
+                                        frontier_cap=args.frontier_cap, schedule=sched,
+                                        ridge=True)
+        P.poseidon_search(prob_r)
+        r_ms = []
+        for _ in range(max(3, args.steps // 2)):
+            flush.zero_()
+            torch.cuda.synchronize()
+            ev0.record()
+            plan_r, st_r = P.poseidon_search(prob_r)
+            ev1.record()
+            torch.cuda.synchronize()
+            r_ms.append(ev0.elapsed_time(ev1))
+        ridge_lines.append({"schedule": "Eager 1F1B" if sched else "1F1B",
+                            "time_to_plan_s": sum(r_ms) / len(r_ms) / 1e3,
+                            "speedup_vs_exact": exact_ms / (sum(r_ms) / len(r_ms)),
+                            "T_us": plan_r["T"], "exact_T_us": exact_T,
+                            "same_value": plan_r["T"] == exact_T,
+                            "evaluations_per_step": st_r["evaluated"],
+                            "pruned_by_ridge": st_r["pruned_ridge"]})
     eager_search = {"schedule": "Eager 1F1B", "prune": PRUNE_NAMES[args.prune],
                     "time_to_plan_s": sum(e_ms) / len(e_ms) / 1e3,
                     "evaluations_per_step": e_ev / len(e_ms), "T_us": plan_e["T"],
@@ -397,6 +421,7 @@ def run_ours(args, rank, world, local_rank):
         "eval_throughput": evals,
         "eval_throughput_eager": evals_eager,
         "eager_search": eager_search,
+        "ridge_search": ridge_lines,
         "cpu_baseline": {"value": cpu_rate, "unit": "evals/s", "cores": 1, "kind": "oracle",
                          "sample": f"{cpu_n} config-4 plan evaluations (S=8, M=32, L=80) in "
                                    f"{cpu_t:.1f} s, single-threaded oracle"},
