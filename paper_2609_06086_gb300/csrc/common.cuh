@@ -40,7 +40,7 @@ pos_status ensure_smem(const void *kernel, int smem);
 // ---------------------------------------------------------------------------
 // Table blob: one contiguous device buffer, staged whole into shared memory
 // by every kernel.  Offsets are bytes from the blob start, 16-byte aligned.
-//   binom  u64 [16][128]        C(n, k) at [k][n], k <= 15
+//   binom  u32 [16][128] twice  C(n, k) at [k][n], k <= 15: low halves, then high halves
 //   Pw, Pa i64 [K][L+1] each    exclusive prefix sums of mem_w, mem_a
 //   cap    i64 [K]
 //   Pf, Pb, Pd i32 [K][L+1]     exclusive prefix sums of fwd, bwd, dsync
@@ -134,10 +134,60 @@ __device__ __forceinline__ int32_t p2f(const Tab &t, int a, int b) {
 __device__ __forceinline__ int32_t p2b(const Tab &t, int a, int b) {
     return ld32(t.base, t.ly->off_p2b + 4u * (uint32_t)(a * t.ly->K + b));
 }
-// stored k-major ([k][n]) so that a warp reading C(n_lane, k) for one k
-// touches consecutive words (no shared-memory bank conflicts)
+// stored k-major ([k][n]) as 32-bit halves, so that a warp reading
+// C(n_lane, k) for one k touches consecutive 4-byte words
+__device__ __forceinline__ uint32_t binom_lo(const Tab &t, int n, int k) {
+    return (uint32_t)ld32(t.base, t.ly->off_binom + 4u * (uint32_t)(k * kBinomN + n));
+}
+__device__ __forceinline__ uint32_t binom_hi(const Tab &t, int n, int k) {
+    return (uint32_t)ld32(t.base,
+                          t.ly->off_binom + 4u * (uint32_t)(kBinomK * kBinomN + k * kBinomN + n));
+}
 __device__ __forceinline__ uint64_t binom(const Tab &t, int n, int k) {
-    return (uint64_t)ld64(t.base, t.ly->off_binom + 8u * (uint32_t)(k * kBinomN + n));
+    return ((uint64_t)binom_hi(t, n, k) << 32) | binom_lo(t, n, k);
+}
+
+// The stage of the combinatorial-number-system unranking: with rem layers
+// left for k+1 stages (k >= 1) and Y = C(rem-1, k) - rank >= 1, the smallest
+// j in [k, rem-1] with C(j, k) >= Y (the stage takes rem - j layers); returns
+// j and lowers rank to C(j, k) - Y.  C(j, k) grows with j.  Since
+// C(j, k) ~ (j - (k-1)/2)^k / k!, j is first estimated as
+// (Y k!)^(1/k) + (k-1)/2 with single-precision log2 / exp2, then moved by
+// exact comparisons to the answer (at most two steps either way over every
+// L <= 127, k <= 15, and exact whatever the estimate).  When
+// C(rem-1, k) < 2^32, every C(j, k) it reads is below 2^32 too and the
+// comparisons use the low halves.
+__device__ __constant__ static const float kLog2Fact[16] = {
+    0.000000000f, 0.000000000f, 1.000000000f, 2.584962501f, 4.584962501f, 6.906890596f,
+    9.491853096f, 12.299208018f, 15.299208018f, 18.469133020f, 21.791061115f, 25.250492733f,
+    28.835455234f, 32.535894952f, 36.343249874f, 40.250140470f};
+__device__ __constant__ static const float kInvK[16] = {
+    0.000000000f, 1.000000000f, 0.500000000f, 0.333333333f, 0.250000000f, 0.200000000f,
+    0.166666667f, 0.142857143f, 0.125000000f, 0.111111111f, 0.100000000f, 0.090909091f,
+    0.083333333f, 0.076923077f, 0.071428571f, 0.066666667f};
+
+__device__ __forceinline__ int unrank_guess(float Yf, int k, int rem) {
+    const float e = exp2f((__log2f(Yf) + kLog2Fact[k]) * kInvK[k]) + 0.5f * (float)(k - 1);
+    return min(max((int)e, k), rem - 1);
+}
+
+__device__ __forceinline__ int unrank_step(const Tab &t, int rem, int k, uint64_t &rank) {
+    const uint64_t total = binom(t, rem - 1, k);
+    int j;
+    if ((total >> 32) == 0) {
+        const uint32_t Y = (uint32_t)(total - rank);
+        j = unrank_guess(__uint2float_rn(Y), k, rem);
+        while (j > k && binom_lo(t, j - 1, k) >= Y) --j;
+        while (binom_lo(t, j, k) < Y) ++j;
+        rank = binom_lo(t, j, k) - Y;
+    } else {
+        const uint64_t Y = total - rank;
+        j = unrank_guess(__ull2float_rn(Y), k, rem);
+        while (j > k && binom(t, j - 1, k) >= Y) --j;
+        while (binom(t, j, k) < Y) ++j;
+        rank = binom(t, j, k) - Y;
+    }
+    return j;
 }
 
 // Cooperative 16-byte copy of the blob into shared memory, four loads in
@@ -227,17 +277,7 @@ __device__ __forceinline__ void unrank_cuts(const Tab &t, uint64_t rank, int (&c
     for (int s = 0; s < S - 1; ++s) {
         const int rem = L - cut[s];
         const int k = S - s - 1;  // p - 1 with p = S - s stages left
-        // Y = C(rem-1, k) - rank >= 1; the stage takes v = rem - j layers for
-        // the smallest j in [k, rem-1] with C(j, k) >= Y.
-        const uint64_t Y = binom(t, rem - 1, k) - rank;
-        int lo = k, hi = rem - 1;
-        while (lo < hi) {
-            const int mid = (lo + hi) >> 1;
-            if (binom(t, mid, k) >= Y) hi = mid;
-            else lo = mid + 1;
-        }
-        rank = binom(t, lo, k) - Y;
-        cut[s + 1] = cut[s] + (rem - lo);
+        cut[s + 1] = cut[s] + (rem - unrank_step(t, rem, k, rank));
     }
     cut[S] = L;
 }

@@ -66,15 +66,19 @@ __device__ __forceinline__ int eval_key(int sched, uint32_t w) {
 }
 
 // global key histogram; invalid records are answered right here
+// 2-byte key per candidate, written by the histogram pass and read by the
+// scatter pass (instead of the 16-byte record, twice)
+constexpr uint16_t kNoKey = 0xffff;
+
 __global__ void sort_hist_kernel(int sched, const uint4 *cands, int64_t n, uint32_t *hist,
-                                 int32_t *T,
-                                 uint8_t *F) {
+                                 uint16_t *keys, int32_t *T, uint8_t *F) {
     __shared__ uint32_t h[kKeys];
     for (int i = threadIdx.x; i < kKeys; i += blockDim.x) h[i] = 0;
     __syncthreads();
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
         const int k = eval_key(sched, __ldg(&cands[i].w));
+        keys[i] = k >= 0 ? (uint16_t)k : kNoKey;
         if (k >= 0) {
             atomicAdd(&h[k], 1u);
         } else {
@@ -118,7 +122,7 @@ __global__ void sort_scan_kernel(const uint32_t *hist, uint32_t *offs, uint32_t 
 // one range per key with a single atomic, then places the indices.
 constexpr int kChunk = 8192;
 
-__global__ void sort_scatter_kernel(int sched, const uint4 *cands, int64_t n, uint32_t *cursor,
+__global__ void sort_scatter_kernel(const uint16_t *keys, int64_t n, uint32_t *cursor,
                                     uint32_t *perm) {
     __shared__ uint32_t h[kKeys];
     for (int64_t c0 = blockIdx.x * (int64_t)kChunk; c0 < n; c0 += (int64_t)gridDim.x * kChunk) {
@@ -126,16 +130,16 @@ __global__ void sort_scatter_kernel(int sched, const uint4 *cands, int64_t n, ui
         for (int i = threadIdx.x; i < kKeys; i += blockDim.x) h[i] = 0;
         __syncthreads();
         for (int64_t i = c0 + threadIdx.x; i < c1; i += blockDim.x) {
-            const int k = eval_key(sched, __ldg(&cands[i].w));
-            if (k >= 0) atomicAdd(&h[k], 1u);
+            const uint16_t k = __ldg(keys + i);
+            if (k != kNoKey) atomicAdd(&h[k], 1u);
         }
         __syncthreads();
         for (int i = threadIdx.x; i < kKeys; i += blockDim.x)
             if (h[i]) h[i] = atomicAdd(&cursor[i], h[i]);
         __syncthreads();
         for (int64_t i = c0 + threadIdx.x; i < c1; i += blockDim.x) {
-            const int k = eval_key(sched, __ldg(&cands[i].w));
-            if (k >= 0) perm[atomicAdd(&h[k], 1u)] = (uint32_t)i;
+            const uint16_t k = __ldg(keys + i);
+            if (k != kNoKey) perm[atomicAdd(&h[k], 1u)] = (uint32_t)i;
         }
         __syncthreads();
     }
@@ -214,14 +218,16 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
     for (int64_t base = 0; base < n; base += chunk) {
         const int64_t m = std::min(chunk, n - base);
         void *scratch = nullptr;
-        // scratch: packed cuts (16 B per candidate), then the sort arrays
-        const size_t sbytes = 16 * (size_t)m + sizeof(uint32_t) * (3 * (size_t)kKeys + 1 + (size_t)m);
+        // scratch: packed cuts (16 B per candidate), the sort arrays, the keys
+        const size_t sbytes = 16 * (size_t)m + sizeof(uint32_t) * (3 * (size_t)kKeys + 1 + (size_t)m) +
+                              sizeof(uint16_t) * (size_t)m;
         POS_CUDA(cudaMallocFromPoolAsync(&scratch, sbytes, pool, stream));
         uint4 *cuts = static_cast<uint4 *>(scratch);
         uint32_t *hist = reinterpret_cast<uint32_t *>(static_cast<char *>(scratch) + 16 * (size_t)m);
         uint32_t *offs = hist + kKeys;
         uint32_t *cursor = offs + kKeys + 1;
         uint32_t *perm = cursor + kKeys;
+        uint16_t *keys = reinterpret_cast<uint16_t *>(perm + m);
         EvalParams p;
         p.cands = reinterpret_cast<const uint4 *>(d_cands) + base;
         p.n = m;
@@ -240,11 +246,12 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
             1, std::min<int64_t>((m + 255) / 256, 4LL * sm_count()));
         cudaError_t e = cudaMemsetAsync(hist, 0, sizeof(uint32_t) * kKeys, stream);
         if (e == cudaSuccess) {
-            sort_hist_kernel<<<grid, 256, 0, stream>>>(p.lay.sched, p.cands, m, hist, p.T, p.F);
+            sort_hist_kernel<<<grid, 256, 0, stream>>>(p.lay.sched, p.cands, m, hist, keys, p.T,
+                                                       p.F);
             sort_scan_kernel<<<1, 1024, 0, stream>>>(hist, offs, cursor);
             const int sgrid = (int)std::max<int64_t>(
                 1, std::min<int64_t>((m + kChunk - 1) / kChunk, 8LL * sm_count()));
-            sort_scatter_kernel<<<sgrid, 512, 0, stream>>>(p.lay.sched, p.cands, m, cursor, perm);
+            sort_scatter_kernel<<<sgrid, 512, 0, stream>>>(keys, m, cursor, perm);
             e = cudaGetLastError();
         }
         if (e == cudaSuccess) st = launch_decode(p, stream);

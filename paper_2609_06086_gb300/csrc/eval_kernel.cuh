@@ -83,15 +83,7 @@ __device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, cons
         int c2 = L;
         if (s < S - 1) {
             const int rem = L - c, k = S - s - 1;
-            const uint64_t Y = binom(t, rem - 1, k) - rank;
-            int lo = k, hi = rem - 1;
-            while (lo < hi) {
-                const int mid = (lo + hi) >> 1;
-                if (binom(t, mid, k) >= Y) hi = mid;
-                else lo = mid + 1;
-            }
-            rank = binom(t, lo, k) - Y;
-            c2 = c + (rem - lo);
+            c2 = c + (rem - unrank_step(t, rem, k, rank));
             if (s < 8) lo8 |= (uint64_t)c2 << (8 * s);
             else hi8 |= (uint64_t)c2 << (8 * (s - 8));
         }
