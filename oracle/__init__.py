@@ -22,7 +22,7 @@ _lib = None
 MAX_S = 16
 
 
-SCHED_1F1B, SCHED_EAGER_1F1B = 0, 1
+SCHED_1F1B, SCHED_EAGER_1F1B, SCHED_INTERLEAVED_1F1B = 0, 1, 2
 
 
 class Tables(C.Structure):
@@ -94,6 +94,10 @@ def lib():
         L.orc_lower_bound_tight.restype = C.c_int64
         L.orc_lower_bound_tight.argtypes = [C.POINTER(Tables), C.c_int, C.c_int, C.c_void_p,
                                             C.c_void_p, C.c_int]
+        L.orc_eval_interleaved.restype = C.c_int
+        L.orc_eval_interleaved.argtypes = [C.POINTER(Tables), C.c_int, C.c_int, C.c_int,
+                                           C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                           C.c_void_p]
         L.orc_eval_batch.restype = C.c_int
         L.orc_eval_batch.argtypes = [C.POINTER(Tables), C.c_void_p, C.c_int64, C.c_void_p,
                                      C.c_void_p]
@@ -179,6 +183,21 @@ def lower_bound(tab: OracleTables, S, M, cls, layers, x):
     if g < 0:
         raise ValueError("invalid configuration")
     return int(g)
+
+
+def evaluate_interleaved(tab: OracleTables, N, V, M, cls, layers, counts=False):
+    """Interleaved 1F1B: makespan and memory feasibility of N devices with
+    V chunks each; layers has N*V entries (virtual stages in model order)."""
+    c, l = _i32(cls, N), _i32(layers, N * V)
+    T, F = C.c_int32(), C.c_int32()
+    dc = DagCounts()
+    rc = lib().orc_eval_interleaved(C.byref(tab.c), N, V, M, c.ctypes.data, l.ctypes.data,
+                                    C.byref(T), C.byref(F), C.byref(dc))
+    if rc:
+        raise ValueError("invalid configuration")
+    if counts:
+        return T.value, bool(F.value), {n: getattr(dc, n) for n, _ in DagCounts._fields_}
+    return T.value, bool(F.value)
 
 
 def lower_bound_tight(tab: OracleTables, S, M, cls, layers, x):

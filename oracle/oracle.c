@@ -154,7 +154,8 @@ static int stage_memory_ok(const orc_tables *t, int S, int M, int s, int cls, in
         sw += mw[i];
         sa += ma[i];
     }
-    int64_t need = sw + (int64_t)warmup_count(t->schedule, S, M, s) * sa;
+    const int sched = t->schedule == ORC_SCHED_INTERLEAVED_1F1B ? ORC_SCHED_1F1B : t->schedule;
+    int64_t need = sw + (int64_t)warmup_count(sched, S, M, s) * sa;
     return need <= t->cap[cls];
 }
 
@@ -244,6 +245,37 @@ static void add_edge(dag *g, int a, int b, int64_t w) {
 #define NODE_B(s, m) (2 + 2 * ((s) * M + (m)))
 #define NODE_R(s) (1 + 2 * S * M + (s))
 
+/* Kahn topological order; longest path where a node finishes at its
+ * latest predecessor finish (+ edge weight) plus its own weight. */
+static int solve_longest(dag *g, int n_nodes, int node_E, int64_t *T_out) {
+    for (int i = 0; i < n_nodes; ++i) {
+        g->indeg[i] = 0;
+        g->head[i] = -1;
+        g->start[i] = 0;
+    }
+    for (int e = 0; e < g->n_edges; ++e) {
+        g->indeg[g->edst[e]]++;
+        g->next_e[e] = g->head[g->esrc[e]];
+        g->head[g->esrc[e]] = e;
+    }
+    int qh = 0, qt = 0;
+    for (int i = 0; i < n_nodes; ++i)
+        if (g->indeg[i] == 0) g->queue[qt++] = i;
+    while (qh < qt) {
+        int u = g->queue[qh++];
+        g->fin[u] = g->start[u] + g->w[u];
+        for (int e = g->head[u]; e >= 0; e = g->next_e[e]) {
+            int v = g->edst[e];
+            int64_t cand = g->fin[u] + g->ew[e];
+            if (cand > g->start[v]) g->start[v] = cand;
+            if (--g->indeg[v] == 0) g->queue[qt++] = v;
+        }
+    }
+    if (qt != n_nodes) return -1; /* not a DAG */
+    *T_out = g->fin[node_E];
+    return 0;
+}
+
 static int build_and_solve(dag *g, int sched, int S, int M, const stage_w *sw,
                            orc_dag_counts *counts, int64_t *T_out) {
     int n_nodes = 2 + 2 * S * M + S;
@@ -320,34 +352,7 @@ static int build_and_solve(dag *g, int sched, int S, int M, const stage_w *sw,
         counts->aux_edges = c_aux;
     }
 
-    /* Kahn topological order; longest path where a node finishes at its
-     * latest predecessor finish (+ edge weight) plus its own weight. */
-    for (int i = 0; i < n_nodes; ++i) {
-        g->indeg[i] = 0;
-        g->head[i] = -1;
-        g->start[i] = 0;
-    }
-    for (int e = 0; e < g->n_edges; ++e) {
-        g->indeg[g->edst[e]]++;
-        g->next_e[e] = g->head[g->esrc[e]];
-        g->head[g->esrc[e]] = e;
-    }
-    int qh = 0, qt = 0;
-    for (int i = 0; i < n_nodes; ++i)
-        if (g->indeg[i] == 0) g->queue[qt++] = i;
-    while (qh < qt) {
-        int u = g->queue[qh++];
-        g->fin[u] = g->start[u] + g->w[u];
-        for (int e = g->head[u]; e >= 0; e = g->next_e[e]) {
-            int v = g->edst[e];
-            int64_t cand = g->fin[u] + g->ew[e];
-            if (cand > g->start[v]) g->start[v] = cand;
-            if (--g->indeg[v] == 0) g->queue[qt++] = v;
-        }
-    }
-    if (qt != n_nodes) return -1; /* not a DAG */
-    *T_out = g->fin[node_E];
-    return 0;
+    return solve_longest(g, n_nodes, node_E, T_out);
 }
 
 static int check_inputs(const orc_tables *t, int S, int M, const int32_t *cls,
@@ -376,6 +381,184 @@ int orc_eval(const orc_tables *t, int S, int M, const int32_t *cls, const int32_
     if (T64 >= ((int64_t)1 << 31)) return -1;
     *T = (int32_t)T64;
     *feasible = config_memory_ok(t, S, M, cls, layers);
+    return 0;
+}
+
+/* ------------------------------------------------------------------ */
+/* Interleaved 1F1B (Sec. 4.1.4).                                      */
+/* ------------------------------------------------------------------ */
+/* N devices (physical stages) each hold V model chunks: virtual stage j
+ * (0-based, j < NV) is chunk j / N on device j % N, and the L layers are
+ * split over the NV virtual stages in order.  The paper fixes the node and
+ * edge counts (2VNM compute nodes, 2(NV-1)M inter-stage edges, N(2VM-1)
+ * intra-stage edges) but not the order of a device's 2VM ops; the order
+ * taken is the interleaved schedule the paper cites (Narayanan et al.
+ * 2021): forward number k (k = 0..VM-1) of a device runs chunk
+ * (k mod NV) div N on micro-batch (k div NV) N + k mod N, backward number k
+ * the chunk V-1-((k mod NV) div N) on the same micro-batch; the device runs
+ * w = min((N-d-1)*2 + (V-1)*N, VM) warm-up forwards (w = VM when M = N),
+ * then alternates one forward and one backward, then runs the remaining
+ * backwards.  M must be a multiple of N. */
+typedef struct {
+    int c, m, is_b;
+} il_op;
+
+static void interleaved_chain(int N, int V, int M, int d, il_op *ops) {
+    int total = M * V;
+    int warm = M == N ? total : (N - d - 1) * 2 + (V - 1) * N;
+    if (warm > total) warm = total;
+    /* forwards 0..warm-1, then (F, B) pairs, then the remaining backwards */
+    int f = 0, b = 0, n = 0;
+    while (f < warm) {
+        int p = f % (N * V);
+        ops[n].c = p / N;
+        ops[n].m = (f / (N * V)) * N + p % N;
+        ops[n].is_b = 0;
+        ++n;
+        ++f;
+    }
+    while (f < total) {
+        int p = f % (N * V);
+        ops[n].c = p / N;
+        ops[n].m = (f / (N * V)) * N + p % N;
+        ops[n].is_b = 0;
+        ++n;
+        ++f;
+        p = b % (N * V);
+        ops[n].c = V - 1 - p / N;
+        ops[n].m = (b / (N * V)) * N + p % N;
+        ops[n].is_b = 1;
+        ++n;
+        ++b;
+    }
+    while (b < total) {
+        int p = b % (N * V);
+        ops[n].c = V - 1 - p / N;
+        ops[n].m = (b / (N * V)) * N + p % N;
+        ops[n].is_b = 1;
+        ++n;
+        ++b;
+    }
+}
+
+int orc_eval_interleaved(const orc_tables *t, int N, int V, int M, const int32_t *cls,
+                         const int32_t *layers, int32_t *T, int32_t *feasible,
+                         orc_dag_counts *counts) {
+    const int J = N * V, L = t->L, K = t->n_types * t->n_tp;
+    if (N < 1 || V < 2 || J > ORC_MAX_S || M < 1 || M % N != 0) return -1;
+    int sum = 0;
+    for (int j = 0; j < J; ++j) {
+        if (layers[j] < 1) return -1;
+        sum += layers[j];
+    }
+    if (sum != L) return -1;
+    for (int d = 0; d < N; ++d)
+        if (cls[d] < 0 || cls[d] >= K) return -1;
+    /* virtual-stage weights (Sec. 4.1.3): F_j, B_j over chunk j's layers on
+       its device's class; all-reduce per device over all its chunks */
+    int64_t F[ORC_MAX_S], B[ORC_MAX_S], dsum[ORC_MAX_S], act[ORC_MAX_S], wsum[ORC_MAX_S];
+    for (int d = 0; d < N; ++d) dsum[d] = wsum[d] = 0;
+    int first = 0;
+    for (int j = 0; j < J; ++j) {
+        const int k = cls[j % N];
+        int64_t f = 0, b = 0, dd = 0, a = 0, w = 0;
+        for (int l = first; l < first + layers[j]; ++l) {
+            f += t->fwd[(int64_t)k * L + l];
+            b += t->bwd[(int64_t)k * L + l];
+            dd += t->dsync[(int64_t)k * L + l];
+            a += t->mem_a[(int64_t)k * L + l];
+            w += t->mem_w[(int64_t)k * L + l];
+        }
+        F[j] = f;
+        B[j] = b;
+        act[j] = a;
+        dsum[j % N] += dd;
+        wsum[j % N] += w;
+        first += layers[j];
+    }
+    /* nodes: S (0), F_{j,m} and B_{j,m}, R_d, E */
+    const int n_nodes = 2 + 2 * J * M + N, node_E = n_nodes - 1;
+    const int n_edges_max = 2 * (J - 1) * M + N * (2 * V * M - 1) + N + 1 + N + 1;
+    dag g;
+    memset(&g, 0, sizeof(g));
+    il_op *ops = malloc(sizeof(il_op) * 2 * V * M);
+    if (!ops || dag_reserve(&g, n_nodes, n_edges_max)) {
+        free(ops);
+        dag_free(&g);
+        return -1;
+    }
+#define IL_F(j, m) (1 + 2 * ((j) * M + (m)))
+#define IL_B(j, m) (2 + 2 * ((j) * M + (m)))
+#define IL_R(d) (1 + 2 * J * M + (d))
+    g.n_nodes = n_nodes;
+    g.n_edges = 0;
+    g.w[0] = 0;
+    g.w[node_E] = 0;
+    for (int j = 0; j < J; ++j)
+        for (int m = 0; m < M; ++m) {
+            g.w[IL_F(j, m)] = F[j];
+            g.w[IL_B(j, m)] = B[j];
+        }
+    for (int d = 0; d < N; ++d) g.w[IL_R(d)] = dsum[d];
+    int64_t c_inter = 0, c_intra = 0;
+    /* inter-stage edges between consecutive virtual stages (their devices) */
+    for (int m = 0; m < M; ++m)
+        for (int j = 0; j + 1 < J; ++j) {
+            const int ka = cls[j % N], kb = cls[(j + 1) % N];
+            add_edge(&g, IL_F(j, m), IL_F(j + 1, m), t->p2p_f[(int64_t)ka * K + kb]);
+            add_edge(&g, IL_B(j + 1, m), IL_B(j, m), t->p2p_b[(int64_t)kb * K + ka]);
+            c_inter += 2;
+        }
+    /* intra-device chains and the peak of the activations each device holds */
+    int ok = 1;
+    *feasible = 1;
+    for (int d = 0; d < N && ok; ++d) {
+        interleaved_chain(N, V, M, d, ops);
+        int64_t held = 0, peak = 0;
+        for (int i = 0; i < 2 * V * M; ++i) {
+            const int j = ops[i].c * N + d;
+            held += ops[i].is_b ? -act[j] : act[j];
+            if (held > peak) peak = held;
+            if (i > 0) {
+                const int a = ops[i - 1].c * N + d;
+                add_edge(&g, ops[i - 1].is_b ? IL_B(a, ops[i - 1].m) : IL_F(a, ops[i - 1].m),
+                         ops[i].is_b ? IL_B(j, ops[i].m) : IL_F(j, ops[i].m), 0);
+                c_intra += 1;
+            }
+        }
+        /* each forward precedes its backward on the device */
+        for (int i = 0; i < 2 * V * M && ok; ++i) {
+            if (!ops[i].is_b) continue;
+            int seen = 0;
+            for (int u = 0; u < i; ++u)
+                seen |= !ops[u].is_b && ops[u].c == ops[i].c && ops[u].m == ops[i].m;
+            ok = seen;
+        }
+        const int lc = ops[2 * V * M - 1].c * N + d;
+        add_edge(&g, IL_B(lc, ops[2 * V * M - 1].m), IL_R(d), 0);
+        add_edge(&g, IL_R(d), node_E, 0);
+        if (peak + wsum[d] > t->cap[cls[d]]) *feasible = 0;
+    }
+    add_edge(&g, 0, IL_F(0, 0), 0);
+    int64_t T64 = 0;
+    int rc = ok ? solve_longest(&g, n_nodes, node_E, &T64) : -1;
+    if (counts) {
+        counts->nodes = n_nodes;
+        counts->compute_nodes = 2 * (int64_t)J * M;
+        counts->allreduce_nodes = N;
+        counts->control_nodes = 2;
+        counts->inter_edges = c_inter;
+        counts->intra_edges = c_intra;
+        counts->allreduce_edges = N;
+        counts->aux_edges = N + 1;
+    }
+#undef IL_F
+#undef IL_B
+#undef IL_R
+    free(ops);
+    dag_free(&g);
+    if (rc || T64 >= ((int64_t)1 << 31)) return -1;
+    *T = (int32_t)T64;
     return 0;
 }
 
@@ -524,6 +707,36 @@ int orc_eval_batch(const orc_tables *t, const orc_candidate *c, int64_t n, int32
     for (int64_t i = 0; i < n; ++i) {
         int S = c[i].S, M = c[i].M;
         int32_t layers[ORC_MAX_S], cls[ORC_MAX_S];
+        /* Interleaved 1F1B: the pad byte is V, the model chunks per device;
+           the composition is over the S*V virtual stages */
+        const int V = t->schedule == ORC_SCHED_INTERLEAVED_1F1B && c[i].pad >= 2 ? c[i].pad : 1;
+        if (V >= 2) {
+            const int J = S * V;
+            int ok = S >= 1 && J <= ORC_MAX_S && J <= t->L && M >= 1 && M % S == 0 &&
+                     c[i].tp_idx < t->n_tp;
+            if (ok) ok = orc_unrank(t->L, J, c[i].map_rank, layers) == 0;
+            for (int s = 0; ok && s < S; ++s) {
+                int ty = (c[i].type_code >> (2 * s)) & 3;
+                if (ty >= t->n_types) ok = 0;
+                cls[s] = ty * t->n_tp + c[i].tp_idx;
+            }
+            if (!ok) {
+                T[i] = -1;
+                feasible[i] = 2;
+            } else if (overflow_bound(t, J, M) >= ((int64_t)1 << 31)) {
+                T[i] = -1;
+                feasible[i] = 3;
+            } else {
+                int32_t Ti, Fi;
+                if (orc_eval_interleaved(t, S, V, M, cls, layers, &Ti, &Fi, NULL)) {
+                    dag_free(&g);
+                    return -1;
+                }
+                T[i] = Ti;
+                feasible[i] = (uint8_t)Fi;
+            }
+            continue;
+        }
         int ok = S >= 1 && S <= ORC_MAX_S && S <= t->L && M >= 1 && c[i].tp_idx < t->n_tp;
         if (ok) ok = orc_unrank(t->L, S, c[i].map_rank, layers) == 0;
         for (int s = 0; ok && s < S; ++s) {
@@ -544,7 +757,8 @@ int orc_eval_batch(const orc_tables *t, const orc_candidate *c, int64_t n, int32
         stage_w sw;
         stage_weights(t, S, cls, layers, &sw);
         int64_t T64;
-        if (build_and_solve(&g, t->schedule, S, M, &sw, NULL, &T64)) {
+        const int sched = t->schedule == ORC_SCHED_INTERLEAVED_1F1B ? ORC_SCHED_1F1B : t->schedule;
+        if (build_and_solve(&g, sched, S, M, &sw, NULL, &T64)) {
             dag_free(&g);
             return -1;
         }

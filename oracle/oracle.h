@@ -42,6 +42,7 @@ typedef struct {
  *                forwards, steady B-F groups, cool-down backwards). */
 #define ORC_SCHED_1F1B 0
 #define ORC_SCHED_EAGER_1F1B 1
+#define ORC_SCHED_INTERLEAVED_1F1B 2  /* candidates carry V; V <= 1 runs 1F1B */
 
 /* 16-byte candidate record (same field meaning as the library's). */
 typedef struct {
@@ -116,6 +117,14 @@ int64_t orc_lower_bound(const orc_tables *t, int S, int M, const int32_t *cls,
  * invalid input and -2 when no completion fits in memory. */
 int64_t orc_lower_bound_tight(const orc_tables *t, int S, int M, const int32_t *cls,
                               const int32_t *layers, int x);
+/* Interleaved 1F1B (Sec. 4.1.4): N devices of classes cls[0..N-1], each
+ * holding V >= 2 model chunks; layers[0..NV-1] are the layer counts of the
+ * NV virtual stages in model order (virtual stage j is chunk j / N on
+ * device j % N).  Device order and memory: see oracle.c.  M must be a
+ * multiple of N.  Returns 0, or -1 on invalid input. */
+int orc_eval_interleaved(const orc_tables *t, int N, int V, int M, const int32_t *cls,
+                         const int32_t *layers, int32_t *T, int32_t *feasible,
+                         orc_dag_counts *counts);
 /* Decode and evaluate n candidate records.  feasible: 1 ok, 0 memory
  * infeasible, 2 invalid record, 3 overflow guard tripped. */
 int orc_eval_batch(const orc_tables *t, const orc_candidate *c, int64_t n, int32_t *T,
