@@ -6,6 +6,7 @@ no lower bound, no search.
 """
 from .workloads import (  # noqa: F401
     CANDIDATE_DTYPE, Workload, config1, config2, config3, config4, config5_tables,
-    config5_candidates, all_candidates, random_candidates, get_config, n_compositions,
+    config5_candidates, all_candidates, random_candidates, interleaved_candidates, get_config,
+    n_compositions,
     place_list,
 )

@@ -35,9 +35,10 @@ from itertools import permutations, product
 import numpy as np
 
 # pos_candidate layout (16 bytes): u64 map_rank, u32 type_code (2 bits per
-# stage, stage 1 in the low bits), u8 S, u8 M, u8 tp_idx, u8 pad.
+# stage, stage 1 in the low bits), u8 S, u8 M, u8 tp_idx, u8 V (model chunks
+# per device under Interleaved 1F1B; 0 otherwise).
 CANDIDATE_DTYPE = np.dtype([("map_rank", "<u8"), ("type_code", "<u4"), ("S", "u1"),
-                            ("M", "u1"), ("tp_idx", "u1"), ("pad", "u1")])
+                            ("M", "u1"), ("tp_idx", "u1"), ("V", "u1")])
 assert CANDIDATE_DTYPE.itemsize == 16
 
 PLACE_FREE = 0
@@ -243,7 +244,38 @@ def random_candidates(n: int, *, L: int, n_types: int, S_range=(2, 16), M_range=
         o["S"] = S.astype(np.uint8)
         o["M"] = M.astype(np.uint8)
         o["tp_idx"] = 0
-        o["pad"] = 0
+        o["V"] = 0
+    return out
+
+
+def interleaved_candidates(n: int, L: int = 64, n_types: int = 2, seed: int = 0,
+                           m_lo: int = 8, m_hi: int = 128) -> np.ndarray:
+    """Interleaved 1F1B batch (Sec. 4.1.4): per record, in this draw order,
+    N ~ U{1..8} devices, V ~ U{2..16//N} chunks per device, M ~ U{m_lo..m_hi}
+    rounded down to a multiple of N (at least N), the N device types i.i.d.
+    uniform, and the rank of the composition of L into the N*V virtual
+    stages uniform in [0, C(L-1, N*V-1)) from a 64-bit draw."""
+    rng = np.random.default_rng(seed)
+    N = rng.integers(1, 9, size=n)
+    V = 2 + (rng.random(n) * (16 // N - 1)).astype(np.int64)
+    M = rng.integers(m_lo, m_hi + 1, size=n)
+    M = np.maximum(N, (M // N) * N)
+    ty = rng.integers(0, n_types, size=(n, 8)).astype(np.uint32)
+    tc = np.zeros(n, np.uint32)
+    for s in range(8):
+        tc |= np.where(s < N, ty[:, s] << np.uint32(2 * s), 0).astype(np.uint32)
+    u = rng.integers(0, np.iinfo(np.uint64).max, size=n, dtype=np.uint64, endpoint=True)
+    J = N * V
+    highs = np.array([math.comb(L - 1, j - 1) if 1 <= j <= L else 1 for j in range(17)],
+                     dtype=object)
+    rank = np.array([int(x) % int(highs[j]) for x, j in zip(u.tolist(), J.tolist())],
+                    dtype=np.uint64)
+    out = np.zeros(n, dtype=CANDIDATE_DTYPE)
+    out["map_rank"] = rank
+    out["type_code"] = tc
+    out["S"] = N.astype(np.uint8)
+    out["M"] = M.astype(np.uint8)
+    out["V"] = V.astype(np.uint8)
     return out
 
 

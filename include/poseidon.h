@@ -42,9 +42,30 @@ typedef int32_t pos_status;
  * i = 1..M-W_s, then the remaining backwards, and holds the activations of
  * W_s micro-batches at once:
  *   POS_SCHED_1F1B        W_s = min(N-s+1, M)
- *   POS_SCHED_EAGER_1F1B  W_s = min(2(N-s)+1, M)   (Eager 1F1B, App. B) */
+ *   POS_SCHED_EAGER_1F1B  W_s = min(2(N-s)+1, M)   (Eager 1F1B, App. B)
+ *   POS_SCHED_INTERLEAVED_1F1B  Interleaved 1F1B (Sec. 4.1.4) for candidates
+ *       whose V field is >= 2, 1F1B for the others.  The S = N devices each
+ *       hold V model chunks; the L layers are split over the J = N*V
+ *       virtual stages in order, virtual stage j (0-based) being chunk j / N
+ *       on device j % N, so the DAG has 2VNM compute nodes, 2(NV-1)M
+ *       inter-stage and N(2VM-1) intra-stage edges.  M must be a multiple
+ *       of N.  Device d (0-based) runs the interleaved order of Narayanan et
+ *       al. (2021), which the paper cites: its k-th forward (k = 0..VM-1)
+ *       is chunk (k mod NV) / N of micro-batch (k / NV)*N + k mod N, its
+ *       k-th backward chunk V-1 - (k mod NV) / N of the same micro-batch;
+ *       it runs w_d = min(2(N-d-1) + (V-1)N, VM) forwards (all VM when
+ *       M = N), then alternates one forward and one backward, then runs
+ *       the remaining backwards.  Memory: the largest sum of activations
+ *       the device holds along that order (a forward of chunk c adds its
+ *       mem_a, the matching backward releases it) plus the mem_w of all its
+ *       chunks must fit cap of its class.  The edge between virtual stages
+ *       j and j+1 uses the classes of their devices (p2p_f[k_{j%N}][k_{(j+1)%N}],
+ *       p2p_b[k_{(j+1)%N}][k_{j%N}]); R_d sums dsync over the device's chunks
+ *       and follows its last op.  Evaluated by poseidon_eval_batch only;
+ *       poseidon_search returns POS_ENOTIMPL for it. */
 #define POS_SCHED_1F1B 0
 #define POS_SCHED_EAGER_1F1B 1
+#define POS_SCHED_INTERLEAVED_1F1B 2
 
 #define POS_PLACE_FREE 0    /* any device type on any stage */
 #define POS_PLACE_EXACT 1   /* exactly type_counts[t] stages of type t */
@@ -85,12 +106,17 @@ typedef struct pos_tables {
  *              all C(L-1, S-1) compositions of L into S non-empty stages;
  *              rank 0 = (1, ..., 1, L-S+1);
  *   type_code  device type of stage s (0-based) in bits [2s, 2s+2);
- *   S          stages (1..16), M micro-batches (1..255), tp_idx < n_tp.
+ *   S          stages (1..16), M micro-batches (1..255), tp_idx < n_tp;
+ *   V          model chunks per device under POS_SCHED_INTERLEAVED_1F1B
+ *              (V >= 2: S is the device count N, map_rank ranks the
+ *              composition of L into the J = S*V virtual stages among
+ *              C(L-1, J-1), J <= 16, and M must be a multiple of S);
+ *              ignored by the other schedules and when V < 2.
  */
 typedef struct pos_candidate {
     uint64_t map_rank;
     uint32_t type_code;
-    uint8_t S, M, tp_idx, pad;
+    uint8_t S, M, tp_idx, V;
 } pos_candidate;
 
 /* feasible[] codes written by poseidon_eval_batch */
@@ -110,8 +136,8 @@ typedef struct pos_candidate {
  * Copy the tables to the current CUDA device and build the per-class
  * exclusive prefix sums used by every kernel (hot-path step a1, Sec. 4.1.3).
  * *handle owns the device copies until poseidon_tables_destroy.  schedule
- * (POS_SCHED_1F1B or POS_SCHED_EAGER_1F1B) applies to every evaluation
- * through the handle.
+ * (POS_SCHED_1F1B, POS_SCHED_EAGER_1F1B or POS_SCHED_INTERLEAVED_1F1B)
+ * applies to every evaluation through the handle.
  * Errors: POS_EINVAL (null pointer, limits, negative cost or memory),
  * POS_EOVERFLOW (a class's summed costs reach 2^31), POS_ENOTIMPL (schedule),
  * POS_ENOMEM, POS_ECUDA.

@@ -21,6 +21,7 @@ STATUS_NAMES = ["POS_OK", "POS_EINVAL", "POS_EOVERFLOW", "POS_ENOMEM", "POS_ECUD
                 "POS_ETIMEOUT", "POS_EINFEASIBLE", "POS_ENOTIMPL"]
 POS_SCHED_1F1B = 0
 POS_SCHED_EAGER_1F1B = 1
+POS_SCHED_INTERLEAVED_1F1B = 2
 POS_PLACE_FREE, POS_PLACE_EXACT = 0, 1
 MAX_STAGES = 16
 

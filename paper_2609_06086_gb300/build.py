@@ -31,7 +31,8 @@ def nvcc() -> str:
 
 
 def _deps_mtime() -> float:
-    files = glob.glob(os.path.join(CSRC, "*.cuh")) + [os.path.join(ROOT, "include", "poseidon.h")]
+    files = (glob.glob(os.path.join(CSRC, "*.cuh")) + glob.glob(os.path.join(CSRC, "*.h")) +
+             [os.path.join(ROOT, "include", "poseidon.h")])
     return max(os.path.getmtime(f) for f in files)
 
 

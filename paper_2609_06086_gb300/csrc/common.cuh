@@ -51,7 +51,8 @@ constexpr int kBinomK = 16;
 
 struct BlobLayout {
     int L, K, n_types, n_tp;
-    int sched;  // POS_SCHED_1F1B or POS_SCHED_EAGER_1F1B (stage chains, in-flight counts)
+    int sched;  // POS_SCHED_* (stage chains, in-flight counts; Interleaved 1F1B
+                // evaluates records with V < 2 as 1F1B)
     int off_binom, off_Pw, off_Pa, off_cap, off_Pf, off_Pb, off_Pd, off_p2f, off_p2b;
     int bytes;  // multiple of 16
 };

@@ -4,7 +4,7 @@
 #include <mutex>
 #include <utility>
 
-#include "eval_kernel.cuh"
+#include "interleaved.cuh"
 
 namespace pos {
 
@@ -60,8 +60,13 @@ __global__ void argmin_final(const int32_t *part_t, const long long *part_i, int
 // counting sort of the candidates by (S, M) key
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ int eval_key(int sched, uint32_t w) {
-    const int S = w & 0xff, M = (w >> 8) & 0xff;
+    const int S = w & 0xff, M = (w >> 8) & 0xff, V = (int)(w >> 24);
     if (S < 1 || S > POS_MAX_STAGES || M < 1) return -1;
+    if (sched == POS_SCHED_INTERLEAVED_1F1B && V >= 2) {
+        // N = S devices, V chunks each: key block of (N, V), index q = M / N
+        if (S * V > POS_MAX_STAGES || M % S != 0) return -1;
+        return kKeys + kIlKeyOf[S - 1][V] + M / S;
+    }
     return M >= fast_min_m(sched, S) ? fast_key_begin(S) + M : generic_key_begin(S) + M;
 }
 
@@ -70,10 +75,11 @@ __device__ __forceinline__ int eval_key(int sched, uint32_t w) {
 // scatter pass (instead of the 16-byte record, twice)
 constexpr uint16_t kNoKey = 0xffff;
 
+template <int NK>
 __global__ void sort_hist_kernel(int sched, const uint4 *cands, int64_t n, uint32_t *hist,
                                  uint16_t *keys, int32_t *T, uint8_t *F) {
-    __shared__ uint32_t h[kKeys];
-    for (int i = threadIdx.x; i < kKeys; i += blockDim.x) h[i] = 0;
+    __shared__ uint32_t h[NK];
+    for (int i = threadIdx.x; i < NK; i += blockDim.x) h[i] = 0;
     __syncthreads();
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
@@ -87,15 +93,16 @@ __global__ void sort_hist_kernel(int sched, const uint4 *cands, int64_t n, uint3
         }
     }
     __syncthreads();
-    for (int i = threadIdx.x; i < kKeys; i += blockDim.x)
+    for (int i = threadIdx.x; i < NK; i += blockDim.x)
         if (h[i]) atomicAdd(&hist[i], h[i]);
 }
 
 // exclusive prefix sum of the histogram (one block); cursor = offs copy
+template <int NK>
 __global__ void sort_scan_kernel(const uint32_t *hist, uint32_t *offs, uint32_t *cursor) {
     __shared__ uint32_t part[1024];
-    const int per = (kKeys + blockDim.x - 1) / blockDim.x;
-    const int lo = threadIdx.x * per, hi = min(kKeys, lo + per);
+    const int per = (NK + blockDim.x - 1) / blockDim.x;
+    const int lo = threadIdx.x * per, hi = min(NK, lo + per);
     uint32_t sum = 0;
     for (int i = lo; i < hi; ++i) sum += hist[i];
     part[threadIdx.x] = sum;
@@ -107,7 +114,7 @@ __global__ void sort_scan_kernel(const uint32_t *hist, uint32_t *offs, uint32_t 
             part[i] = run;
             run += v;
         }
-        offs[kKeys] = run;
+        offs[NK] = run;
     }
     __syncthreads();
     uint32_t run = part[threadIdx.x];
@@ -122,19 +129,20 @@ __global__ void sort_scan_kernel(const uint32_t *hist, uint32_t *offs, uint32_t 
 // one range per key with a single atomic, then places the indices.
 constexpr int kChunk = 8192;
 
+template <int NK>
 __global__ void sort_scatter_kernel(const uint16_t *keys, int64_t n, uint32_t *cursor,
                                     uint32_t *perm) {
-    __shared__ uint32_t h[kKeys];
+    __shared__ uint32_t h[NK];
     for (int64_t c0 = blockIdx.x * (int64_t)kChunk; c0 < n; c0 += (int64_t)gridDim.x * kChunk) {
         const int64_t c1 = min(n, c0 + kChunk);
-        for (int i = threadIdx.x; i < kKeys; i += blockDim.x) h[i] = 0;
+        for (int i = threadIdx.x; i < NK; i += blockDim.x) h[i] = 0;
         __syncthreads();
         for (int64_t i = c0 + threadIdx.x; i < c1; i += blockDim.x) {
             const uint16_t k = __ldg(keys + i);
             if (k != kNoKey) atomicAdd(&h[k], 1u);
         }
         __syncthreads();
-        for (int i = threadIdx.x; i < kKeys; i += blockDim.x)
+        for (int i = threadIdx.x; i < NK; i += blockDim.x)
             if (h[i]) h[i] = atomicAdd(&cursor[i], h[i]);
         __syncthreads();
         for (int64_t i = c0 + threadIdx.x; i < c1; i += blockDim.x) {
@@ -145,13 +153,13 @@ __global__ void sort_scatter_kernel(const uint16_t *keys, int64_t n, uint32_t *c
     }
 }
 
-// Decode pass over the whole sorted range [0, offs[kKeys]).
+// Decode pass over the whole sorted range [0, offs[nkeys]).
 __global__ void __launch_bounds__(256, 4) decode_kernel(EvalParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
     stage_blob(sm, p.blob, p.lay.bytes);
     __syncthreads();
     const Tab t = tab_at(sm, p.lay);
-    const int64_t total = p.offs[kKeys];
+    const int64_t total = p.offs[p.nkeys];
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     const int64_t span = (total + 31) & ~(int64_t)31;
     for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < span; j += stride) {
@@ -218,15 +226,17 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
     for (int64_t base = 0; base < n; base += chunk) {
         const int64_t m = std::min(chunk, n - base);
         void *scratch = nullptr;
+        const bool il = h->lay.sched == POS_SCHED_INTERLEAVED_1F1B;
+        const int nk = il ? kKeysIl : kKeys;
         // scratch: packed cuts (16 B per candidate), the sort arrays, the keys
-        const size_t sbytes = 16 * (size_t)m + sizeof(uint32_t) * (3 * (size_t)kKeys + 1 + (size_t)m) +
+        const size_t sbytes = 16 * (size_t)m + sizeof(uint32_t) * (3 * (size_t)nk + 1 + (size_t)m) +
                               sizeof(uint16_t) * (size_t)m;
         POS_CUDA(cudaMallocFromPoolAsync(&scratch, sbytes, pool, stream));
         uint4 *cuts = static_cast<uint4 *>(scratch);
         uint32_t *hist = reinterpret_cast<uint32_t *>(static_cast<char *>(scratch) + 16 * (size_t)m);
-        uint32_t *offs = hist + kKeys;
-        uint32_t *cursor = offs + kKeys + 1;
-        uint32_t *perm = cursor + kKeys;
+        uint32_t *offs = hist + nk;
+        uint32_t *cursor = offs + nk + 1;
+        uint32_t *perm = cursor + nk;
         uint16_t *keys = reinterpret_cast<uint16_t *>(perm + m);
         EvalParams p;
         p.cands = reinterpret_cast<const uint4 *>(d_cands) + base;
@@ -242,16 +252,24 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
         p.gD = h->guard_D;
         p.gP = h->guard_P;
         p.pg = pg;
+        p.nkeys = nk;
         const int grid = (int)std::max<int64_t>(
             1, std::min<int64_t>((m + 255) / 256, 4LL * sm_count()));
-        cudaError_t e = cudaMemsetAsync(hist, 0, sizeof(uint32_t) * kKeys, stream);
+        cudaError_t e = cudaMemsetAsync(hist, 0, sizeof(uint32_t) * nk, stream);
         if (e == cudaSuccess) {
-            sort_hist_kernel<<<grid, 256, 0, stream>>>(p.lay.sched, p.cands, m, hist, keys, p.T,
-                                                       p.F);
-            sort_scan_kernel<<<1, 1024, 0, stream>>>(hist, offs, cursor);
             const int sgrid = (int)std::max<int64_t>(
                 1, std::min<int64_t>((m + kChunk - 1) / kChunk, 8LL * sm_count()));
-            sort_scatter_kernel<<<sgrid, 512, 0, stream>>>(keys, m, cursor, perm);
+            if (il) {
+                sort_hist_kernel<kKeysIl><<<grid, 256, 0, stream>>>(p.lay.sched, p.cands, m, hist,
+                                                                    keys, p.T, p.F);
+                sort_scan_kernel<kKeysIl><<<1, 1024, 0, stream>>>(hist, offs, cursor);
+                sort_scatter_kernel<kKeysIl><<<sgrid, 512, 0, stream>>>(keys, m, cursor, perm);
+            } else {
+                sort_hist_kernel<kKeys><<<grid, 256, 0, stream>>>(p.lay.sched, p.cands, m, hist,
+                                                                  keys, p.T, p.F);
+                sort_scan_kernel<kKeys><<<1, 1024, 0, stream>>>(hist, offs, cursor);
+                sort_scatter_kernel<kKeys><<<sgrid, 512, 0, stream>>>(keys, m, cursor, perm);
+            }
             e = cudaGetLastError();
         }
         if (e == cudaSuccess) st = launch_decode(p, stream);
@@ -274,6 +292,7 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
                        (st = eval_generic_15_15(p, stream)) == POS_OK) {
                 st = eval_generic_16_16(p, stream);
             }
+            if (st == POS_OK && il) st = eval_interleaved(p, stream);
         }
         const cudaError_t e2 = cudaFreeAsync(scratch, stream);
         if (e != cudaSuccess) return cuda_fail(e, "eval sort launch");

@@ -17,7 +17,8 @@
 //
 // Sort keys: fast path (M >= S for 1F1B, M >= 2S-1 for Eager 1F1B) ->
 // (S-1)*256 + M (the other slots of each S stay empty); short path ->
-// 4096 + (S-1)*32 + M; records with S outside 1..16 or M = 0 are flagged
+// 4096 + (S-1)*32 + M; Interleaved 1F1B records with V >= 2 get keys after
+// those (interleaved.cuh); records with S outside 1..16 or M = 0 are flagged
 // invalid by the sort pass and get no key.
 #pragma once
 #include <algorithm>
@@ -38,14 +39,56 @@ struct EvalParams {
     int32_t *T;
     uint8_t *F;
     const uint32_t *perm;  // sorted candidate indices
-    const uint32_t *offs;  // [kKeys + 1] start of every key in perm
+    const uint32_t *offs;  // [nkeys + 1] start of every key in perm
     uint4 *cuts;           // per sorted position: cut[1..S-1] in bytes 0..14,
                            // byte 15 = 1 when the result is already written
     const void *blob;
     BlobLayout lay;
     int64_t gA, gD, gP;
     Programs pg;           // level programs of the schedule's short path
+    int nkeys;             // kKeys, or kKeysIl under Interleaved 1F1B
 };
+
+// Decode pass for an Interleaved 1F1B record (pad byte V >= 2, S = N
+// devices): checks its fields (N*V <= 16 virtual stages, at most L, M a
+// multiple of N) and the overflow guard over the N*V virtual stages, and
+// unranks the composition of L layers into the virtual stages.  Memory is
+// checked by the makespan kernel (it needs the device chains).
+__device__ __forceinline__ uint4 decode_il(const Tab &t, const uint4 &rec, const EvalParams &p,
+                                           uint32_t i) {
+    uint64_t rank = (uint64_t)rec.x | ((uint64_t)rec.y << 32);
+    const uint32_t tcode = rec.z;
+    const int S = rec.w & 0xff;
+    const int M = (rec.w >> 8) & 0xff;
+    const int tp = (rec.w >> 16) & 0xff;
+    const int V = (int)(rec.w >> 24);
+    const int J = S * V, L = t.L();
+    bool ok = S >= 1 && J <= POS_MAX_STAGES && J <= L && M >= 1 && M % S == 0 &&
+              tp < t.n_tp() && rank < binom(t, L - 1, J - 1);
+    for (int s = 0; s < S && ok; ++s) ok = ((tcode >> (2 * s)) & 3) < (uint32_t)t.n_types();
+    const uint4 done = make_uint4(0, 0, 0, 1u << 24);
+    if (!ok) {
+        p.T[i] = -1;
+        p.F[i] = POS_FEAS_INVALID;
+        return done;
+    }
+    if (guard_trips(p.gA, p.gD, p.gP, J, M)) {
+        p.T[i] = -1;
+        p.F[i] = POS_FEAS_OVERFLOW;
+        return done;
+    }
+    uint64_t lo8 = 0, hi8 = 0;
+    int c = 0;
+#pragma unroll 1
+    for (int j = 0; j < J - 1; ++j) {
+        const int rem = L - c, k = J - j - 1;
+        c += rem - unrank_step(t, rem, k, rank);
+        if (j < 8) lo8 |= (uint64_t)c << (8 * j);
+        else hi8 |= (uint64_t)c << (8 * (j - 8));
+    }
+    return make_uint4((uint32_t)lo8, (uint32_t)(lo8 >> 32), (uint32_t)hi8,
+                      (uint32_t)(hi8 >> 32) & 0x00ffffffu);
+}
 
 // Decode pass for one candidate: checks its fields and the overflow guard,
 // unranks the composition stage by stage (the steps of unrank_cuts),
@@ -61,6 +104,8 @@ __device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, cons
     const int M = (rec.w >> 8) & 0xff;
     const int tp = (rec.w >> 16) & 0xff;
     const int L = t.L();
+    if (t.ly->sched == POS_SCHED_INTERLEAVED_1F1B && (rec.w >> 24) >= 2)
+        return decode_il(t, rec, p, i);
     bool ok = S >= 1 && S <= POS_MAX_STAGES && M >= 1 && S <= L && tp < t.n_tp() &&
               rank < binom(t, L - 1, S - 1);
     for (int s = 0; s < S && ok; ++s) ok = ((tcode >> (2 * s)) & 3) < (uint32_t)t.n_types();

@@ -1,0 +1,267 @@
+// Interleaved 1F1B evaluation (Sec. 4.1.4): N devices each hold V model
+// chunks, so the pipeline has J = N*V virtual stages (virtual stage j is
+// chunk j / N on device j % N) and the DAG 2VNM compute nodes.  One thread
+// evaluates one candidate with all state in registers:
+//   * weights: F_j, B_j of every virtual stage (prefix-sum differences on
+//     its device's class), the transfer times pf_d = p2p_f[k_d][k_{d+1}] and
+//     pb_d = p2p_b[k_{d+1}][k_d] (an edge j -> j+1 always joins device j % N
+//     to device (j+1) % N), and each device's all-reduce time summed over
+//     its chunks;
+//   * makespan: the ops in the static order of interleaved_order.h, where
+//     each op is one relaxation finish = max(device clock, finish of the
+//     latest op of its kind on the neighbouring virtual stage + edge) +
+//     weight, and T = max_d (clock_d + allreduce_d) (the last op of device d
+//     is B of chunk 0 on the last micro-batch, which feeds R_d);
+//   * memory: the largest activation footprint over device d's chain plus
+//     its resident bytes must fit its class's capacity.  The footprint after
+//     each op adds the chunk's activations on a forward and releases them on
+//     a backward; it is largest after a forward, and in the steady phase its
+//     values after the forwards repeat with period NV (every NV consecutive
+//     forwards, and backwards, cover each chunk N times), so the warm-up and
+//     at most one period are scanned.
+#pragma once
+#include "eval_kernel.cuh"
+#include "interleaved_order.h"
+
+namespace pos {
+
+// The interleaved key region follows the 1F1B keys: record (N, V, M) with
+// V >= 2, N*V <= 16 and M = q*N has key kKeys + kIlKeyOf[N-1][V] + q.
+constexpr int kKeysIl = kKeys + IlPair<kIlPairs>::key;
+
+template <int N, int V>
+struct IlState {
+    static constexpr int J = N * V;
+    int32_t Fo[J], Bo[J], clk[N];  // latest forward / backward finish per virtual stage
+    int32_t F[J], B[J], pf[N], pb[N];
+};
+
+template <int N, int V, int OP>
+__device__ __forceinline__ void il_relax(IlState<N, V> &s) {
+    constexpr int J = N * V, j = OP & 15, d = j % N;
+    if constexpr ((OP & 0x80) == 0) {
+        int32_t t = s.clk[d];
+        if constexpr (j > 0) t = max(t, s.Fo[j - 1] + s.pf[(j - 1) % N]);
+        s.Fo[j] = t + s.F[j];
+        s.clk[d] = s.Fo[j];
+    } else {
+        int32_t t = s.clk[d];
+        if constexpr (j + 1 < J) t = max(t, s.Bo[j + 1] + s.pb[d]);
+        s.Bo[j] = t + s.B[j];
+        s.clk[d] = s.Bo[j];
+    }
+}
+
+// part 0 = P, 1 = Body, 2 = E, 3 = Short
+template <int N, int V, int PART, int I>
+__device__ __forceinline__ constexpr int il_op() {
+    using O = IlOrder<N, V>;
+    if constexpr (PART == 0) return O::P[I];
+    else if constexpr (PART == 1) return O::Body[I];
+    else if constexpr (PART == 2) return O::E[I];
+    else return O::Short[I];
+}
+
+template <int N, int V, int PART, int... I>
+__device__ __forceinline__ void il_run(IlState<N, V> &s, std::integer_sequence<int, I...>) {
+    (il_relax<N, V, il_op<N, V, PART, I>()>(s), ...);
+}
+
+template <int N, int V>
+__device__ __forceinline__ void il_makespan_ops(IlState<N, V> &s, int q) {
+    using O = IlOrder<N, V>;
+#pragma unroll
+    for (int d = 0; d < N; ++d) s.clk[d] = 0;
+    if (q < O::q0) {
+        il_run<N, V, 3>(s, std::make_integer_sequence<int, O::nShort>{});
+        return;
+    }
+    il_run<N, V, 0>(s, std::make_integer_sequence<int, O::nP>{});
+#pragma unroll 1
+    for (int r = O::q0; r < q; ++r) il_run<N, V, 1>(s, std::make_integer_sequence<int, O::nBody>{});
+    il_run<N, V, 2>(s, std::make_integer_sequence<int, O::nE>{});
+}
+
+// Does device d (class k) fit?  act[c]: activations of its chunk c per
+// micro-batch; resident: its weights and optimizer state over all chunks.
+template <int N, int V, int d>
+__device__ __forceinline__ bool il_device_fits(const int64_t (&act)[V], int64_t resident,
+                                               int64_t cap, int q) {
+    constexpr int NV = N * V;
+    int64_t peak;
+    if (q == 1) {  // M = N: every forward runs before the first backward
+        int64_t all = 0;
+#pragma unroll
+        for (int c = 0; c < V; ++c) all += act[c];
+        peak = (int64_t)N * all;
+    } else {
+        constexpr int w = 2 * (N - d - 1) + (V - 1) * N;  // warm-up forwards (< VM for q >= 2)
+        int64_t held = 0;
+#pragma unroll
+        for (int k = 0; k < w; ++k) held += act[(k % NV) / N];
+        // steady pairs (F_{w+i}, B_i): all of one period for q >= 3, the
+        // 2NV - w pairs there are for q = 2 when fewer
+        constexpr int steady2 = 2 * NV - w;
+        const int steps = (q >= 3 || steady2 >= NV) ? NV : steady2;
+        peak = 0;
+#pragma unroll
+        for (int i = 0; i < NV; ++i) {
+            if (i < steps) {
+                held += act[((w + i) % NV) / N];
+                peak = max(peak, held);
+                held -= act[V - 1 - (i % NV) / N];
+            }
+        }
+    }
+    return peak + resident <= cap;
+}
+
+template <int N, int V, int... D>
+__device__ __forceinline__ bool il_fits_all(const Tab &t, const int (&cut)[N * V + 1],
+                                            const int (&cls)[N], int q,
+                                            std::integer_sequence<int, D...>) {
+    bool ok = true;
+    (
+        [&] {
+            constexpr int d = D;
+            const int k = cls[d];
+            int64_t act[V], resident = 0;
+#pragma unroll
+            for (int c = 0; c < V; ++c) {
+                const int j = c * N + d;
+                act[c] = Pa(t, k, cut[j + 1]) - Pa(t, k, cut[j]);
+                resident += Pw(t, k, cut[j + 1]) - Pw(t, k, cut[j]);
+            }
+            ok &= il_device_fits<N, V, d>(act, resident, cap_of(t, k), q);
+        }(),
+        ...);
+    return ok;
+}
+
+// Makespan and feasibility of one decoded interleaved candidate: S = N
+// devices, pad byte V, cut positions of the J virtual stages packed by the
+// decode pass.
+template <int N, int V>
+__device__ __forceinline__ void il_eval_one(const Tab &t, const uint4 &rec, const uint4 &packed,
+                                            int32_t &T, uint8_t &feasible) {
+    constexpr int J = N * V;
+    const uint32_t tcode = rec.z;
+    const int M = (rec.w >> 8) & 0xff;
+    const int tp = (rec.w >> 16) & 0xff;
+    const int q = M / N;
+    int cls[N], cut[J + 1];
+#pragma unroll
+    for (int d = 0; d < N; ++d) cls[d] = ((tcode >> (2 * d)) & 3) * t.n_tp() + tp;
+    const uint32_t pw[4] = {packed.x, packed.y, packed.z, packed.w};
+    cut[0] = 0;
+#pragma unroll
+    for (int j = 0; j < J - 1; ++j) cut[j + 1] = (pw[j / 4] >> (8 * (j % 4))) & 0xff;
+    cut[J] = t.L();
+    feasible = il_fits_all<N, V>(t, cut, cls, q, std::make_integer_sequence<int, N>{})
+                   ? POS_FEAS_YES
+                   : POS_FEAS_NO;
+    IlState<N, V> s;
+    int32_t dsum[N];
+#pragma unroll
+    for (int d = 0; d < N; ++d) {
+        dsum[d] = 0;
+        s.pf[d] = p2f(t, cls[d], cls[(d + 1) % N]);
+        s.pb[d] = p2b(t, cls[(d + 1) % N], cls[d]);
+    }
+#pragma unroll
+    for (int j = 0; j < J; ++j) {
+        const int k = cls[j % N];
+        s.F[j] = Pf(t, k, cut[j + 1]) - Pf(t, k, cut[j]);
+        s.B[j] = Pb(t, k, cut[j + 1]) - Pb(t, k, cut[j]);
+        dsum[j % N] += Pd(t, k, cut[j + 1]) - Pd(t, k, cut[j]);
+    }
+    il_makespan_ops<N, V>(s, q);
+    int32_t best = 0;
+#pragma unroll
+    for (int d = 0; d < N; ++d) best = max(best, s.clk[d] + dsum[d]);
+    T = best;
+}
+
+template <int PLO, int PHI>
+__device__ __forceinline__ void il_dispatch(int N, int V, const Tab &t, const uint4 &rec,
+                                            const uint4 &packed, int32_t &T, uint8_t &feasible) {
+    if constexpr (PLO <= PHI) {
+        if (N == IlPair<PLO>::N && V == IlPair<PLO>::V) {
+            il_eval_one<IlPair<PLO>::N, IlPair<PLO>::V>(t, rec, packed, T, feasible);
+            return;
+        }
+        il_dispatch<PLO + 1, PHI>(N, V, t, rec, packed, T, feasible);
+    }
+}
+
+// Evaluates the sorted range of pairs PLO..PHI (their key blocks are
+// contiguous); warps split by (N, V) like eval_kernel splits by S.
+template <int PLO, int PHI, int MINB>
+__global__ void __launch_bounds__(kEvalThreads, MINB) il_eval_kernel(EvalParams p) {
+    extern __shared__ __align__(16) unsigned char sm[];
+    stage_blob(sm, p.blob, p.lay.bytes);
+    __syncthreads();
+    const Tab t = tab_at(sm, p.lay);
+    const int64_t begin = p.offs[kKeys + IlPair<PLO>::key], end = p.offs[kKeys + IlPair<PHI + 1>::key];
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t span = ((end - begin) + 31) & ~(int64_t)31;
+    for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < span; j += stride) {
+        bool active = j < end - begin;
+        uint32_t i = 0;
+        uint4 rec = make_uint4(0, 0, 0, 0), packed = make_uint4(0, 0, 0, 0);
+        if (active) {
+            i = __ldg(p.perm + begin + j);
+            packed = __ldg(p.cuts + begin + j);
+            active = (packed.w >> 24) == 0;  // not answered by the decode pass
+            if (active) rec = __ldg(p.cands + i);
+        }
+        const int g = active ? (int)(rec.w & 0xff) * 32 + (int)(rec.w >> 24) : 0;  // N*32 + V
+        int32_t T = -1;
+        uint8_t feasible = POS_FEAS_INVALID;
+        unsigned pending = __ballot_sync(0xffffffffu, active);
+        while (pending) {
+            const int leader = __ffs(pending) - 1;
+            const int gg = __shfl_sync(0xffffffffu, g, leader);
+            const bool mine = active && g == gg;
+            const unsigned grp = __ballot_sync(0xffffffffu, mine);
+            if (mine) il_dispatch<PLO, PHI>(gg >> 5, gg & 31, t, rec, packed, T, feasible);
+            pending &= ~grp;
+        }
+        if (active) {
+            p.T[i] = T;
+            p.F[i] = feasible;
+        }
+    }
+}
+
+template <int PLO, int PHI, int MINB>
+pos_status launch_il_range(const EvalParams &p, cudaStream_t stream) {
+    auto kern = il_eval_kernel<PLO, PHI, MINB>;
+    const int smem = p.lay.bytes;
+    POS_TRY(ensure_smem(reinterpret_cast<const void *>(kern), smem));
+    int per_sm = 0;
+    POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kEvalThreads, smem));
+    if (per_sm < 1) return fail(POS_ECUDA, "interleaved eval kernel does not fit on an SM");
+    const int64_t blocks = (p.n + kEvalThreads - 1) / kEvalThreads;
+    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)per_sm * sm_count()));
+    kern<<<grid, kEvalThreads, smem, stream>>>(p);
+    POS_CUDA(cudaGetLastError());
+    return POS_OK;
+}
+
+// one launcher per instantiation unit (eval_il_*.cu), pairs by index
+pos_status eval_il_0_11(const EvalParams &p, cudaStream_t s);
+pos_status eval_il_12_22(const EvalParams &p, cudaStream_t s);
+pos_status eval_il_23_29(const EvalParams &p, cudaStream_t s);
+pos_status eval_il_30_31(const EvalParams &p, cudaStream_t s);
+pos_status eval_il_32_33(const EvalParams &p, cudaStream_t s);
+
+inline pos_status eval_interleaved(const EvalParams &p, cudaStream_t s) {
+    POS_TRY(eval_il_0_11(p, s));
+    POS_TRY(eval_il_12_22(p, s));
+    POS_TRY(eval_il_23_29(p, s));
+    POS_TRY(eval_il_30_31(p, s));
+    return eval_il_32_33(p, s);
+}
+
+}  // namespace pos

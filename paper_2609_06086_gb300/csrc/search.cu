@@ -956,7 +956,8 @@ struct Search {
 static pos_status validate_problem(const pos_problem *p) {
     if (!p) return fail(POS_EINVAL, "problem is NULL");
     if (p->schedule != POS_SCHED_1F1B && p->schedule != POS_SCHED_EAGER_1F1B)
-        return fail(POS_ENOTIMPL, "schedule must be POS_SCHED_1F1B or POS_SCHED_EAGER_1F1B");
+        return fail(POS_ENOTIMPL, "the search supports POS_SCHED_1F1B and POS_SCHED_EAGER_1F1B; "
+                                  "Interleaved 1F1B is evaluated by poseidon_eval_batch only");
     if (p->S < 1 || p->S > POS_MAX_STAGES) return fail(POS_EINVAL, "S must be in 1..16");
     if (p->S > p->tables.L) return fail(POS_EINVAL, "S > L");
     if (p->n_M < 1 || !p->M_list) return fail(POS_EINVAL, "empty M_list");

@@ -277,8 +277,10 @@ extern "C" {
 pos_status poseidon_tables_create(const pos_tables *tables, int32_t schedule, void **handle) {
     if (!handle) return pos::fail(POS_EINVAL, "handle out-pointer is NULL");
     *handle = nullptr;
-    if (schedule != POS_SCHED_1F1B && schedule != POS_SCHED_EAGER_1F1B)
-        return pos::fail(POS_ENOTIMPL, "schedule must be POS_SCHED_1F1B or POS_SCHED_EAGER_1F1B");
+    if (schedule != POS_SCHED_1F1B && schedule != POS_SCHED_EAGER_1F1B &&
+        schedule != POS_SCHED_INTERLEAVED_1F1B)
+        return pos::fail(POS_ENOTIMPL, "schedule must be POS_SCHED_1F1B, POS_SCHED_EAGER_1F1B "
+                                       "or POS_SCHED_INTERLEAVED_1F1B");
     pos::Handle *h = nullptr;
     const pos_status st = pos::create_handle(tables, schedule, &h);
     if (st == POS_OK) *handle = h;

@@ -45,7 +45,7 @@ def test_struct_layouts_match_the_header(P, tmp_path):
     prog = tmp_path / "layout.c"
     fields = {
         "pos_tables": [f[0] for f in P.binding.pos_tables._fields_],
-        "pos_candidate": ["map_rank", "type_code", "S", "M", "tp_idx", "pad"],
+        "pos_candidate": ["map_rank", "type_code", "S", "M", "tp_idx", "V"],
         "pos_problem": [f[0] for f in P.binding.pos_problem._fields_],
         "pos_plan": [f[0] for f in P.binding.pos_plan._fields_],
         "pos_search_stats": [f[0] for f in P.binding.pos_search_stats._fields_],
@@ -82,7 +82,7 @@ def test_invalid_arguments_rejected_before_the_device(P):
     import gen
     w = gen.config1()
     t = P.Tables.from_workload(w)
-    assert L.poseidon_tables_create(C.byref(t.c), 2, C.byref(h)) == P.binding.POS_ENOTIMPL
+    assert L.poseidon_tables_create(C.byref(t.c), 3, C.byref(h)) == P.binding.POS_ENOTIMPL
     bad = P.Tables.from_workload(w)
     bad.arrays["fwd"][0, 0] = -5
     assert L.poseidon_tables_create(C.byref(bad.c), 0, C.byref(h)) == P.binding.POS_EINVAL
@@ -99,6 +99,10 @@ def test_invalid_arguments_rejected_before_the_device(P):
     prob.warmup = -1
     assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
     prob.warmup = 0
+    prob.schedule = 2  # Interleaved 1F1B: evaluated by poseidon_eval_batch only
+    assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_ENOTIMPL
+    assert b"Interleaved" in L.poseidon_last_error()
+    prob.schedule = 0
     for mode in (-1, 3):
         prob.prune = mode
         assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
