@@ -133,10 +133,18 @@ def oracle_sample_rate(seconds: float, seed: int = 0):
 def eval_throughput(P, torch, n, reps, peak_alu, schedule=0):
     """poseidon_eval_batch on n config-5 candidates (L=64, S ~ U{2..16},
     M ~ U{8..128}, 2 device types), device-resident, timed with CUDA events
-    on the launching stream; inputs (16 B x n) exceed L2 for n >= 1e7."""
+    on the launching stream; inputs (16 B x n) exceed L2 for n >= 1e7.
+    Under Interleaved 1F1B (schedule 2) the records are the interleaved
+    sweep on the same tables: N ~ U{1..8} devices, V ~ U{2..16//N} chunks,
+    M ~ U{8..128} rounded down to a multiple of N; S counts the N*V virtual
+    stages below."""
     w = gen.config5_tables()
-    c = gen.config5_candidates(n, seed=0)
-    S = c["S"].astype(np.int64)
+    if schedule == 2:
+        c = gen.interleaved_candidates(n, L=w.L, seed=0)
+        S = c["S"].astype(np.int64) * c["V"].astype(np.int64)
+    else:
+        c = gen.config5_candidates(n, seed=0)
+        S = c["S"].astype(np.int64)
     M = c["M"].astype(np.int64)
     relax = int((2 * S * M).sum())
     ops = 3 * relax + 11 * int(S.sum())  # 6SM + 11S integer ops per candidate
@@ -162,8 +170,10 @@ def eval_throughput(P, torch, n, reps, peak_alu, schedule=0):
     sec = ms / 1e3 / reps
     h.close()
     ach = ops / sec / 1e12
-    return {"workload": "config 5: L=64, S~U{2..16}, M~U{8..128}, 2 device types",
-            "schedule": "Eager 1F1B" if schedule == 1 else "1F1B",
+    return {"workload": ("interleaved sweep: L=64, N~U{1..8}, V~U{2..16/N}, M~U{8..128} "
+                         "(multiple of N), 2 device types" if schedule == 2 else
+                         "config 5: L=64, S~U{2..16}, M~U{8..128}, 2 device types"),
+            "schedule": ["1F1B", "Eager 1F1B", "Interleaved 1F1B"][schedule],
             "batch": n, "ms_per_call": round(sec * 1e3, 4), "evals_per_s": n / sec,
             "relaxations_per_s": relax / sec, "bound": "alu", "achieved": round(ach, 3),
             "unit": "Tops/s", "peak": round(peak_alu, 3), "frac": round(ach / peak_alu, 4)}
@@ -329,6 +339,8 @@ def run_ours(args, rank, world, local_rank):
     evals = [eval_throughput(P, torch, int(n), 5, peak_alu) for n in args.eval_sizes]
     evals_eager = [eval_throughput(P, torch, int(n), 5, peak_alu, schedule=1)
                    for n in args.eval_sizes[:1]]
+    evals_il = [eval_throughput(P, torch, int(n), 5, peak_alu, schedule=2)
+                for n in args.eval_sizes[:1]]
     # the same search under Eager 1F1B (App. B schedule), for comparison
     ref_e = _json.load(open(os.path.join(ROOT, "tests", "golden", "search_plans.json")))
     ref_e = ref_e.get("config4_eager", {}).get("plan", {})
@@ -420,6 +432,7 @@ def run_ours(args, rank, world, local_rank):
         "other_prune": other_prune,
         "eval_throughput": evals,
         "eval_throughput_eager": evals_eager,
+        "eval_throughput_interleaved": evals_il,
         "eager_search": eager_search,
         "ridge_search": ridge_lines,
         "cpu_baseline": {"value": cpu_rate, "unit": "evals/s", "cores": 1, "kind": "oracle",
