@@ -152,8 +152,9 @@ pos_status poseidon_tables_destroy(void *handle);
  * are in input order; the call is asynchronous on `stream` (a cudaStream_t,
  * NULL = legacy default stream) and returns after the launches.  Infeasible
  * plans still get their makespan.  Scratch: the batch is counting-sorted by
- * (S, M) and decoded into a 22*n + 56 KB stream-ordered allocation (packed
- * cut positions 16 B, permutation 4 B and sort key 2 B per candidate, key
+ * (S, M) (and by (N, V, M/N) for interleaved records) and decoded into a
+ * 38*n + 56 KB (Interleaved 1F1B: 38*n + 121 KB) stream-ordered allocation
+ * (decoded record 32 B, permutation 4 B and sort key 2 B per candidate, key
  * histograms) from a library-owned memory pool (per device, kept between
  * calls); batches above 2^31 candidates go in chunks of 2^31.
  * Errors: POS_EINVAL (null handle or pointers, n < 0, misaligned

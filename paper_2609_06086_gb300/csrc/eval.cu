@@ -172,7 +172,10 @@ __global__ void __launch_bounds__(256, 4) decode_kernel(EvalParams p) {
         }
         uint4 out = make_uint4(0, 0, 0, 1u << 24);
         if (active) out = decode_one(t, rec, p, i);
-        if (active) p.cuts[j] = out;
+        if (active) {
+            p.cuts[2 * j] = out;
+            p.cuts[2 * j + 1] = make_uint4(i, rec.z, rec.w, 0u);
+        }
     }
 }
 
@@ -228,12 +231,12 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
         void *scratch = nullptr;
         const bool il = h->lay.sched == POS_SCHED_INTERLEAVED_1F1B;
         const int nk = il ? kKeysIl : kKeys;
-        // scratch: packed cuts (16 B per candidate), the sort arrays, the keys
-        const size_t sbytes = 16 * (size_t)m + sizeof(uint32_t) * (3 * (size_t)nk + 1 + (size_t)m) +
+        // scratch: decoded records (32 B per candidate), the sort arrays, the keys
+        const size_t sbytes = 32 * (size_t)m + sizeof(uint32_t) * (3 * (size_t)nk + 1 + (size_t)m) +
                               sizeof(uint16_t) * (size_t)m;
         POS_CUDA(cudaMallocFromPoolAsync(&scratch, sbytes, pool, stream));
         uint4 *cuts = static_cast<uint4 *>(scratch);
-        uint32_t *hist = reinterpret_cast<uint32_t *>(static_cast<char *>(scratch) + 16 * (size_t)m);
+        uint32_t *hist = reinterpret_cast<uint32_t *>(static_cast<char *>(scratch) + 32 * (size_t)m);
         uint32_t *offs = hist + nk;
         uint32_t *cursor = offs + nk + 1;
         uint32_t *perm = cursor + nk;

@@ -40,14 +40,32 @@ struct EvalParams {
     uint8_t *F;
     const uint32_t *perm;  // sorted candidate indices
     const uint32_t *offs;  // [nkeys + 1] start of every key in perm
-    uint4 *cuts;           // per sorted position: cut[1..S-1] in bytes 0..14,
-                           // byte 15 = 1 when the result is already written
+    uint4 *cuts;           // per sorted position j, two 16-byte words:
+                           // cuts[2j]: cut[1..S-1] in bytes 0..14, byte 15 = 1
+                           // when the result is already written;
+                           // cuts[2j+1]: (candidate index, type_code, the
+                           // record's S|M|tp|V word, 0), so the makespan
+                           // kernels read 32 contiguous bytes and no record
     const void *blob;
     BlobLayout lay;
     int64_t gA, gD, gP;
     Programs pg;           // level programs of the schedule's short path
     int nkeys;             // kKeys, or kKeysIl under Interleaved 1F1B
 };
+
+// Are the 2-bit type fields of stages 0..S-1 (1 <= S <= 16) all below
+// n_types (1..4)?  A field is >= n_types when its high bit is set
+// (n_types <= 2), when both bits are set (n_types = 3), or, for one type,
+// when it is not zero.
+__device__ __forceinline__ bool types_ok(uint32_t tcode, int S, int n_types) {
+    const uint32_t mask = S >= 16 ? 0xffffffffu : (1u << (2 * S)) - 1u;
+    const uint32_t f = tcode & mask;
+    const uint32_t bad = n_types >= 4   ? 0u
+                         : n_types == 3 ? (f & (f >> 1) & 0x55555555u)
+                         : n_types == 2 ? (f & 0xaaaaaaaau)
+                                        : f;
+    return bad == 0u;
+}
 
 // Decode pass for an Interleaved 1F1B record (pad byte V >= 2, S = N
 // devices): checks its fields (N*V <= 16 virtual stages, at most L, M a
@@ -65,7 +83,7 @@ __device__ __forceinline__ uint4 decode_il(const Tab &t, const uint4 &rec, const
     const int J = S * V, L = t.L();
     bool ok = S >= 1 && J <= POS_MAX_STAGES && J <= L && M >= 1 && M % S == 0 &&
               tp < t.n_tp() && rank < binom(t, L - 1, J - 1);
-    for (int s = 0; s < S && ok; ++s) ok = ((tcode >> (2 * s)) & 3) < (uint32_t)t.n_types();
+    ok = ok && types_ok(tcode, S, t.n_types());
     const uint4 done = make_uint4(0, 0, 0, 1u << 24);
     if (!ok) {
         p.T[i] = -1;
@@ -108,7 +126,7 @@ __device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, cons
         return decode_il(t, rec, p, i);
     bool ok = S >= 1 && S <= POS_MAX_STAGES && M >= 1 && S <= L && tp < t.n_tp() &&
               rank < binom(t, L - 1, S - 1);
-    for (int s = 0; s < S && ok; ++s) ok = ((tcode >> (2 * s)) & 3) < (uint32_t)t.n_types();
+    ok = ok && types_ok(tcode, S, t.n_types());
     const uint4 done = make_uint4(0, 0, 0, 1u << 24);  // byte 15 = 1: answered here
     if (!ok) {
         p.T[i] = -1;
@@ -201,10 +219,11 @@ __global__ void __launch_bounds__(kEvalThreads, MINB) eval_kernel(EvalParams p) 
         uint32_t i = 0;
         uint4 rec = make_uint4(0, 0, 0, 0), packed = make_uint4(0, 0, 0, 0);
         if (active) {
-            i = __ldg(p.perm + begin + j);
-            packed = __ldg(p.cuts + begin + j);
+            packed = __ldg(p.cuts + 2 * (begin + j));
+            const uint4 meta = __ldg(p.cuts + 2 * (begin + j) + 1);
             active = (packed.w >> 24) == 0;  // not answered by the decode pass
-            if (active) rec = __ldg(p.cands + i);
+            i = meta.x;
+            rec = make_uint4(0, 0, meta.y, meta.z);
         }
         const int S = active ? (int)(rec.w & 0xff) : 0;
         int32_t T = -1;

@@ -210,10 +210,11 @@ __global__ void __launch_bounds__(kEvalThreads, MINB) il_eval_kernel(EvalParams 
         uint32_t i = 0;
         uint4 rec = make_uint4(0, 0, 0, 0), packed = make_uint4(0, 0, 0, 0);
         if (active) {
-            i = __ldg(p.perm + begin + j);
-            packed = __ldg(p.cuts + begin + j);
+            packed = __ldg(p.cuts + 2 * (begin + j));
+            const uint4 meta = __ldg(p.cuts + 2 * (begin + j) + 1);
             active = (packed.w >> 24) == 0;  // not answered by the decode pass
-            if (active) rec = __ldg(p.cands + i);
+            i = meta.x;
+            rec = make_uint4(0, 0, meta.y, meta.z);
         }
         const int g = active ? (int)(rec.w & 0xff) * 32 + (int)(rec.w >> 24) : 0;  // N*32 + V
         int32_t T = -1;
