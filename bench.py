@@ -406,6 +406,40 @@ def run_ours(args, rank, world, local_rank):
     other_prune = {"prune": other, "time_to_plan_s": sum(o_ms) / len(o_ms) / 1e3,
                    "evaluations_per_step": o_ev / len(o_ms),
                    "evals_per_s": o_ev / (sum(o_ms) / 1e3), "matches_oracle": o_ok}
+    # config 3 (L=48, S=8, M=64, 4 A + 4 B stages): the exhaustive search
+    # (memory cut only, no stage-level prune) against the oracle's plan, and
+    # its leaf kernel's INT32 fraction from a profiled run
+    w3 = gen.config3()
+    ref3 = _json.load(open(os.path.join(ROOT, "tests", "golden", "search_plans.json")))
+    ref3 = ref3.get("config3", {}).get("plan", {})
+    prob3, keep3 = P.make_problem(w3, warmup=500, prune=0, seed=0,
+                                  frontier_cap=args.frontier_cap)
+    prob3p, keep3p = P.make_problem(w3, warmup=500, prune=0, seed=0,
+                                    frontier_cap=args.frontier_cap, profile=True)
+    P.poseidon_search(prob3)
+    c3_ms, c3_ok = [], True
+    for _ in range(max(3, args.steps // 2)):
+        flush.zero_()
+        torch.cuda.synchronize()
+        ev0.record()
+        plan3, st3 = P.poseidon_search(prob3)
+        ev1.record()
+        torch.cuda.synchronize()
+        c3_ms.append(ev0.elapsed_time(ev1))
+        c3_ok &= plan3["global_index"] == ref3.get("global_index")
+    _, st3p = P.poseidon_search(prob3p)
+    leaf3 = st3p["evaluated"] - st3p["warmup_evaluated"]
+    ops3 = (3 * 2 * w3.S * w3.M_list[0] + 9 * w3.S) * leaf3
+    ach3 = ops3 / max(st3p["ms_leaf"] / 1e3, 1e-12) / 1e12
+    exhaustive3 = {"workload": "config 3: L=48, h=5120, S=8, M=64, exactly 4 A + 4 B stages",
+                   "prune": "none (memory cut only)",
+                   "time_to_plan_s": sum(c3_ms) / len(c3_ms) / 1e3,
+                   "evaluations_per_step": st3["evaluated"], "T_us": plan3["T"],
+                   "matches_oracle": c3_ok,
+                   "leaf_kernel": {"ms": round(st3p["ms_leaf"], 4),
+                                   "launches": st3p["leaf_launches"], "bound": "alu",
+                                   "achieved": round(ach3, 3), "unit": "Tops/s",
+                                   "frac": round(ach3 / peak_alu, 4)}}
     cpu_rate, cpu_n, cpu_t = oracle_sample_rate(args.cpu_seconds)
     line = {
         "metric": METRIC, "value": value, "unit": "evals/s", "n_gpus": world,
@@ -434,6 +468,7 @@ def run_ours(args, rank, world, local_rank):
         "eval_throughput_eager": evals_eager,
         "eval_throughput_interleaved": evals_il,
         "eager_search": eager_search,
+        "config3_exhaustive": exhaustive3,
         "ridge_search": ridge_lines,
         "cpu_baseline": {"value": cpu_rate, "unit": "evals/s", "cores": 1, "kind": "oracle",
                          "sample": f"{cpu_n} config-4 plan evaluations (S=8, M=32, L=80) in "
