@@ -5,8 +5,7 @@ batches).  It holds none of the method's arithmetic: no DAG, no makespan,
 no lower bound, no search.
 """
 from .workloads import (  # noqa: F401
-    CANDIDATE_DTYPE, Workload, config1, config2, config3, config4, config5_tables,
-    config5_candidates, all_candidates, random_candidates, interleaved_candidates, get_config,
-    n_compositions,
-    place_list,
+    CANDIDATE_DTYPE, CANDIDATE_EX_DTYPE, Workload, config1, config2, config3, config4,
+    config5_tables, config5_candidates, all_candidates, random_candidates,
+    interleaved_candidates, per_stage_tp_candidates, get_config, n_compositions, place_list,
 )

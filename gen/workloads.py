@@ -41,6 +41,13 @@ CANDIDATE_DTYPE = np.dtype([("map_rank", "<u8"), ("type_code", "<u4"), ("S", "u1
                             ("M", "u1"), ("tp_idx", "u1"), ("V", "u1")])
 assert CANDIDATE_DTYPE.itemsize == 16
 
+# pos_candidate_ex layout (24 bytes): u64 map_rank, u32 type_code, u32 tp_code
+# (TP index of stage s in bits [2s, 2s+2)), u8 S, u8 M, u8 V, u8 pad, u32 pad.
+CANDIDATE_EX_DTYPE = np.dtype([("map_rank", "<u8"), ("type_code", "<u4"), ("tp_code", "<u4"),
+                               ("S", "u1"), ("M", "u1"), ("V", "u1"), ("pad0", "u1"),
+                               ("pad1", "<u4")])
+assert CANDIDATE_EX_DTYPE.itemsize == 24
+
 PLACE_FREE = 0
 PLACE_EXACT = 1
 
@@ -245,6 +252,36 @@ def random_candidates(n: int, *, L: int, n_types: int, S_range=(2, 16), M_range=
         o["M"] = M.astype(np.uint8)
         o["tp_idx"] = 0
         o["V"] = 0
+    return out
+
+
+def per_stage_tp_candidates(n: int, L: int, n_types: int, n_tp: int, seed: int = 0,
+                            S_range=(1, 16), M_range=(1, 64)) -> np.ndarray:
+    """Records with a TP index per stage, drawn in this order: S ~ U{S_range},
+    M ~ U{M_range}, 16 types and 16 TP indices i.i.d. uniform (fields beyond
+    S cleared), and the composition rank uniform in [0, C(L-1, S-1)) from a
+    64-bit draw."""
+    rng = np.random.default_rng(seed)
+    S = rng.integers(S_range[0], S_range[1] + 1, size=n)
+    S = np.minimum(S, L)
+    M = rng.integers(M_range[0], M_range[1] + 1, size=n)
+    ty = rng.integers(0, n_types, size=(n, 16)).astype(np.uint32)
+    tp = rng.integers(0, n_tp, size=(n, 16)).astype(np.uint32)
+    tc = np.zeros(n, np.uint32)
+    pc = np.zeros(n, np.uint32)
+    for s in range(16):
+        keep = s < S
+        tc |= np.where(keep, ty[:, s] << np.uint32(2 * s), 0).astype(np.uint32)
+        pc |= np.where(keep, tp[:, s] << np.uint32(2 * s), 0).astype(np.uint32)
+    u = rng.integers(0, np.iinfo(np.uint64).max, size=n, dtype=np.uint64, endpoint=True)
+    highs = [math.comb(L - 1, k - 1) if 1 <= k <= L else 1 for k in range(17)]
+    rank = np.array([int(x) % highs[k] for x, k in zip(u.tolist(), S.tolist())], dtype=np.uint64)
+    out = np.zeros(n, dtype=CANDIDATE_EX_DTYPE)
+    out["map_rank"] = rank
+    out["type_code"] = tc
+    out["tp_code"] = pc
+    out["S"] = S.astype(np.uint8)
+    out["M"] = M.astype(np.uint8)
     return out
 
 

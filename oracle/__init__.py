@@ -98,6 +98,9 @@ def lib():
         L.orc_eval_interleaved.argtypes = [C.POINTER(Tables), C.c_int, C.c_int, C.c_int,
                                            C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                            C.c_void_p]
+        L.orc_eval_batch_ex.restype = C.c_int
+        L.orc_eval_batch_ex.argtypes = [C.POINTER(Tables), C.c_void_p, C.c_int64, C.c_void_p,
+                                        C.c_void_p]
         L.orc_eval_batch.restype = C.c_int
         L.orc_eval_batch.argtypes = [C.POINTER(Tables), C.c_void_p, C.c_int64, C.c_void_p,
                                      C.c_void_p]
@@ -221,6 +224,20 @@ def eval_batch(tab: OracleTables, cands: np.ndarray):
     F = np.zeros(n, np.uint8)
     if lib().orc_eval_batch(C.byref(tab.c), cands.ctypes.data, n, T.ctypes.data, F.ctypes.data):
         raise RuntimeError("oracle eval_batch failed")
+    return T, F
+
+
+def eval_batch_ex(tab: OracleTables, cands: np.ndarray):
+    """Evaluate a structured array of 24-byte records with a TP index per
+    stage (bits [2s, 2s+2) of tp_code)."""
+    cands = np.ascontiguousarray(cands)
+    assert cands.dtype.itemsize == 24
+    n = len(cands)
+    T = np.zeros(n, np.int32)
+    F = np.zeros(n, np.uint8)
+    if lib().orc_eval_batch_ex(C.byref(tab.c), cands.ctypes.data, n, T.ctypes.data,
+                               F.ctypes.data):
+        raise RuntimeError("oracle eval_batch_ex failed (n_tp > 4?)")
     return T, F
 
 

@@ -698,72 +698,81 @@ int64_t orc_lower_bound_tight(const orc_tables *t, int S, int M, const int32_t *
     return lb;
 }
 
+/* Decode and evaluate one record: stage (device) s has type
+ * (tcode >> 2s) & 3 and TP index tp[s]; V >= 2 under the interleaved
+ * schedule makes it an interleaved record.  Returns -1 on an internal
+ * failure, else 0 with T and the flag written. */
+static int eval_record(const orc_tables *t, dag *g, uint64_t rank, uint32_t tcode,
+                       const int *tp, int S, int M, int Vbyte, int32_t *T, uint8_t *feasible) {
+    int32_t layers[ORC_MAX_S], cls[ORC_MAX_S];
+    /* Interleaved 1F1B: V model chunks per device; the composition is over
+       the S*V virtual stages */
+    const int V = t->schedule == ORC_SCHED_INTERLEAVED_1F1B && Vbyte >= 2 ? Vbyte : 1;
+    const int J = S * V;
+    int ok = S >= 1 && J <= ORC_MAX_S && J <= t->L && M >= 1 && (V == 1 || M % S == 0);
+    if (ok) ok = orc_unrank(t->L, J, rank, layers) == 0;
+    for (int s = 0; ok && s < S; ++s) {
+        const int ty = (tcode >> (2 * s)) & 3;
+        if (ty >= t->n_types || tp[s] < 0 || tp[s] >= t->n_tp) ok = 0;
+        cls[s] = ty * t->n_tp + tp[s];
+    }
+    if (!ok) {
+        *T = -1;
+        *feasible = 2;
+        return 0;
+    }
+    if (overflow_bound(t, J, M) >= ((int64_t)1 << 31)) {
+        *T = -1;
+        *feasible = 3;
+        return 0;
+    }
+    if (V >= 2) {
+        int32_t Ti, Fi;
+        if (orc_eval_interleaved(t, S, V, M, cls, layers, &Ti, &Fi, NULL)) return -1;
+        *T = Ti;
+        *feasible = (uint8_t)Fi;
+        return 0;
+    }
+    stage_w sw;
+    stage_weights(t, S, cls, layers, &sw);
+    int64_t T64;
+    const int sched = t->schedule == ORC_SCHED_INTERLEAVED_1F1B ? ORC_SCHED_1F1B : t->schedule;
+    if (build_and_solve(g, sched, S, M, &sw, NULL, &T64)) return -1;
+    *T = (int32_t)T64;
+    *feasible = (uint8_t)config_memory_ok(t, S, M, cls, layers);
+    return 0;
+}
+
 int orc_eval_batch(const orc_tables *t, const orc_candidate *c, int64_t n, int32_t *T,
                    uint8_t *feasible) {
-    int K = t->n_types * t->n_tp;
-    (void)K;
     dag g;
     memset(&g, 0, sizeof(g));
     for (int64_t i = 0; i < n; ++i) {
-        int S = c[i].S, M = c[i].M;
-        int32_t layers[ORC_MAX_S], cls[ORC_MAX_S];
-        /* Interleaved 1F1B: the pad byte is V, the model chunks per device;
-           the composition is over the S*V virtual stages */
-        const int V = t->schedule == ORC_SCHED_INTERLEAVED_1F1B && c[i].pad >= 2 ? c[i].pad : 1;
-        if (V >= 2) {
-            const int J = S * V;
-            int ok = S >= 1 && J <= ORC_MAX_S && J <= t->L && M >= 1 && M % S == 0 &&
-                     c[i].tp_idx < t->n_tp;
-            if (ok) ok = orc_unrank(t->L, J, c[i].map_rank, layers) == 0;
-            for (int s = 0; ok && s < S; ++s) {
-                int ty = (c[i].type_code >> (2 * s)) & 3;
-                if (ty >= t->n_types) ok = 0;
-                cls[s] = ty * t->n_tp + c[i].tp_idx;
-            }
-            if (!ok) {
-                T[i] = -1;
-                feasible[i] = 2;
-            } else if (overflow_bound(t, J, M) >= ((int64_t)1 << 31)) {
-                T[i] = -1;
-                feasible[i] = 3;
-            } else {
-                int32_t Ti, Fi;
-                if (orc_eval_interleaved(t, S, V, M, cls, layers, &Ti, &Fi, NULL)) {
-                    dag_free(&g);
-                    return -1;
-                }
-                T[i] = Ti;
-                feasible[i] = (uint8_t)Fi;
-            }
-            continue;
-        }
-        int ok = S >= 1 && S <= ORC_MAX_S && S <= t->L && M >= 1 && c[i].tp_idx < t->n_tp;
-        if (ok) ok = orc_unrank(t->L, S, c[i].map_rank, layers) == 0;
-        for (int s = 0; ok && s < S; ++s) {
-            int ty = (c[i].type_code >> (2 * s)) & 3;
-            if (ty >= t->n_types) ok = 0;
-            cls[s] = ty * t->n_tp + c[i].tp_idx;
-        }
-        if (!ok) {
-            T[i] = -1;
-            feasible[i] = 2;
-            continue;
-        }
-        if (overflow_bound(t, S, M) >= ((int64_t)1 << 31)) {
-            T[i] = -1;
-            feasible[i] = 3;
-            continue;
-        }
-        stage_w sw;
-        stage_weights(t, S, cls, layers, &sw);
-        int64_t T64;
-        const int sched = t->schedule == ORC_SCHED_INTERLEAVED_1F1B ? ORC_SCHED_1F1B : t->schedule;
-        if (build_and_solve(&g, sched, S, M, &sw, NULL, &T64)) {
+        int tp[ORC_MAX_S];
+        for (int s = 0; s < ORC_MAX_S; ++s) tp[s] = c[i].tp_idx;
+        if (eval_record(t, &g, c[i].map_rank, c[i].type_code, tp, c[i].S, c[i].M, c[i].pad,
+                        &T[i], &feasible[i])) {
             dag_free(&g);
             return -1;
         }
-        T[i] = (int32_t)T64;
-        feasible[i] = (uint8_t)config_memory_ok(t, S, M, cls, layers);
+    }
+    dag_free(&g);
+    return 0;
+}
+
+int orc_eval_batch_ex(const orc_tables *t, const orc_candidate_ex *c, int64_t n, int32_t *T,
+                      uint8_t *feasible) {
+    if (t->n_tp > 4) return -1;
+    dag g;
+    memset(&g, 0, sizeof(g));
+    for (int64_t i = 0; i < n; ++i) {
+        int tp[ORC_MAX_S];
+        for (int s = 0; s < ORC_MAX_S; ++s) tp[s] = (int)((c[i].tp_code >> (2 * s)) & 3);
+        if (eval_record(t, &g, c[i].map_rank, c[i].type_code, tp, c[i].S, c[i].M, c[i].V,
+                        &T[i], &feasible[i])) {
+            dag_free(&g);
+            return -1;
+        }
     }
     dag_free(&g);
     return 0;

@@ -51,6 +51,17 @@ typedef struct {
     uint8_t S, M, tp_idx, pad;
 } orc_candidate;
 
+/* 24-byte record with a TP index per stage (same field meaning as the
+ * library's pos_candidate_ex): TP index of stage s in bits [2s, 2s+2) of
+ * tp_code, so n_tp <= 4. */
+typedef struct {
+    uint64_t map_rank;
+    uint32_t type_code;
+    uint32_t tp_code;
+    uint8_t S, M, V, pad0;
+    uint32_t pad1;
+} orc_candidate_ex;
+
 typedef struct {
     orc_tables tab;
     int32_t S;
@@ -129,6 +140,10 @@ int orc_eval_interleaved(const orc_tables *t, int N, int V, int M, const int32_t
  * infeasible, 2 invalid record, 3 overflow guard tripped. */
 int orc_eval_batch(const orc_tables *t, const orc_candidate *c, int64_t n, int32_t *T,
                    uint8_t *feasible);
+/* Same with a TP index per stage (per device for interleaved records): the
+ * class of stage s is type_s * n_tp + tp_s.  Returns -1 when n_tp > 4. */
+int orc_eval_batch_ex(const orc_tables *t, const orc_candidate_ex *c, int64_t n, int32_t *T,
+                      uint8_t *feasible);
 /* Exact search of Sec. 4.2.3.  prune=0 disables the g(S_x) prune (memory
  * infeasible prefixes are still skipped).  warmup = number of random feasible
  * samples evaluated first (Sec. 4.2.3); it never changes the result.
