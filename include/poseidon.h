@@ -119,6 +119,26 @@ typedef struct pos_candidate {
     uint8_t S, M, tp_idx, V;
 } pos_candidate;
 
+/*
+ * A candidate whose stages may use different TP indices (the per-stage
+ * heterogeneous TP of the Metis and HexiScale plans in the paper's Table 1),
+ * 24 bytes:
+ *   map_rank, type_code, S, M, V   as in pos_candidate;
+ *   tp_code    TP index of stage s (0-based; of device s for interleaved
+ *              records) in bits [2s, 2s+2), so the class of stage s is
+ *              type_s * n_tp + tp_s; needs n_tp <= 4.
+ * The tables' TP axis may stand for any per-stage parallel setting (TP
+ * degree, and the data-parallel degree of the stage's all-reduce and
+ * memory); every stage still runs the pipeline's M micro-batches.
+ */
+typedef struct pos_candidate_ex {
+    uint64_t map_rank;
+    uint32_t type_code;
+    uint32_t tp_code;
+    uint8_t S, M, V, pad0;
+    uint32_t pad1;
+} pos_candidate_ex;
+
 /* feasible[] codes written by poseidon_eval_batch */
 #define POS_FEAS_NO 0        /* some stage exceeds its memory capacity */
 #define POS_FEAS_YES 1
@@ -162,6 +182,17 @@ pos_status poseidon_tables_destroy(void *handle);
  */
 pos_status poseidon_eval_batch(void *handle, const pos_candidate *d_cands, int64_t n,
                                int32_t *d_makespan, uint8_t *d_feasible, void *stream);
+
+/*
+ * poseidon_eval_batch for 24-byte pos_candidate_ex records (a TP index per
+ * stage): same outputs, flags, schedules, scratch and stream semantics;
+ * a record whose TP field of some stage s < S is >= n_tp is flagged
+ * POS_FEAS_INVALID.  d_cands must be 8-byte aligned.
+ * Errors: those of poseidon_eval_batch, and POS_EINVAL when the handle's
+ * tables have n_tp > 4.
+ */
+pos_status poseidon_eval_batch_ex(void *handle, const pos_candidate_ex *d_cands, int64_t n,
+                                  int32_t *d_makespan, uint8_t *d_feasible, void *stream);
 
 /*
  * Same as poseidon_eval_batch but with HOST buffers: copies the candidates

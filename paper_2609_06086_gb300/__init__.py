@@ -7,5 +7,5 @@ library and never computes anything itself.
 """
 from .binding import (  # noqa: F401
     EXPORTS, Handle, PoseidonError, Tables, lib, make_problem, poseidon_argmin,
-    poseidon_eval_batch, poseidon_eval_batch_host, poseidon_search,
+    poseidon_eval_batch, poseidon_eval_batch_ex, poseidon_eval_batch_host, poseidon_search,
 )

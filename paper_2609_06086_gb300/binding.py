@@ -27,8 +27,8 @@ MAX_STAGES = 16
 
 # the exported entry points, as declared in include/poseidon.h
 EXPORTS = ["poseidon_tables_create", "poseidon_tables_destroy", "poseidon_eval_batch",
-           "poseidon_eval_batch_host", "poseidon_argmin", "poseidon_argmin_noalloc",
-           "poseidon_search", "poseidon_last_error"]
+           "poseidon_eval_batch_ex", "poseidon_eval_batch_host", "poseidon_argmin",
+           "poseidon_argmin_noalloc", "poseidon_search", "poseidon_last_error"]
 
 
 class pos_tables(C.Structure):
@@ -89,6 +89,7 @@ def lib():
         L.poseidon_tables_create.argtypes = [C.POINTER(pos_tables), i32, C.POINTER(vp)]
         L.poseidon_tables_destroy.argtypes = [vp]
         L.poseidon_eval_batch.argtypes = [vp, vp, i64, vp, vp, vp]
+        L.poseidon_eval_batch_ex.argtypes = [vp, vp, i64, vp, vp, vp]
         L.poseidon_eval_batch_host.argtypes = [vp, vp, i64, vp, vp]
         L.poseidon_argmin.argtypes = [vp, vp, i64, vp, vp]
         L.poseidon_argmin_noalloc.argtypes = [vp, vp, i64, vp, vp]
@@ -152,6 +153,13 @@ def poseidon_eval_batch(handle: Handle, d_cands: int, n: int, d_makespan: int, d
                         stream: int = 0):
     """Device pointers in and out (asynchronous on `stream`)."""
     _check(lib().poseidon_eval_batch(handle.ptr, d_cands, n, d_makespan, d_feasible, stream))
+
+
+def poseidon_eval_batch_ex(handle: Handle, d_cands: int, n: int, d_makespan: int,
+                           d_feasible: int, stream: int = 0):
+    """24-byte records with a TP index per stage; device pointers in and out
+    (asynchronous on `stream`)."""
+    _check(lib().poseidon_eval_batch_ex(handle.ptr, d_cands, n, d_makespan, d_feasible, stream))
 
 
 def poseidon_eval_batch_host(handle: Handle, cands: np.ndarray):

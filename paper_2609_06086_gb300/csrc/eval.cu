@@ -75,15 +75,26 @@ __device__ __forceinline__ int eval_key(int sched, uint32_t w) {
 // scatter pass (instead of the 16-byte record, twice)
 constexpr uint16_t kNoKey = 0xffff;
 
+// The S | M << 8 | tp << 16 | V << 24 word of record i (24-byte records:
+// S, M, V at bytes 16..18, tp = 0).
+__device__ __forceinline__ uint32_t record_word(const EvalParams &p, int64_t i) {
+    if (p.per_stage_tp) {
+        const uint32_t w = __ldg(reinterpret_cast<const uint32_t *>(p.cands_ex) + 6 * i + 4);
+        return (w & 0xffffu) | ((w & 0xff0000u) << 8);
+    }
+    return __ldg(&p.cands[i].w);
+}
+
 template <int NK>
-__global__ void sort_hist_kernel(int sched, const uint4 *cands, int64_t n, uint32_t *hist,
-                                 uint16_t *keys, int32_t *T, uint8_t *F) {
+__global__ void sort_hist_kernel(EvalParams p, int64_t n, uint32_t *hist, uint16_t *keys,
+                                 int32_t *T, uint8_t *F) {
+    const int sched = p.lay.sched;
     __shared__ uint32_t h[NK];
     for (int i = threadIdx.x; i < NK; i += blockDim.x) h[i] = 0;
     __syncthreads();
     for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
          i += (int64_t)gridDim.x * blockDim.x) {
-        const int k = eval_key(sched, __ldg(&cands[i].w));
+        const int k = eval_key(sched, record_word(p, i));
         keys[i] = k >= 0 ? (uint16_t)k : kNoKey;
         if (k >= 0) {
             atomicAdd(&h[k], 1u);
@@ -165,16 +176,18 @@ __global__ void __launch_bounds__(256, 4) decode_kernel(EvalParams p) {
     for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < span; j += stride) {
         const bool active = j < total;
         uint32_t i = 0;
-        uint4 rec = make_uint4(0, 0, 0, 0);
+        RecView v;
+        v.rec = make_uint4(0, 0, 0, 0);
+        v.tpc = 0;
         if (active) {
             i = __ldg(p.perm + j);
-            rec = __ldg(p.cands + i);
+            v = load_record(p, i);
         }
         uint4 out = make_uint4(0, 0, 0, 1u << 24);
-        if (active) out = decode_one(t, rec, p, i);
+        if (active) out = decode_one(t, v.rec, v.tpc, p, i);
         if (active) {
             p.cuts[2 * j] = out;
-            p.cuts[2 * j + 1] = make_uint4(i, rec.z, rec.w, 0u);
+            p.cuts[2 * j + 1] = make_uint4(i, v.rec.z, v.rec.w, v.tpc);
         }
     }
 }
@@ -216,8 +229,9 @@ static pos_status scratch_pool(cudaMemPool_t *out) {
     return POS_OK;
 }
 
-pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32_t *d_T,
-                       uint8_t *d_F, cudaStream_t stream) {
+// d_cands: 16-byte records, or 24-byte records when per_stage_tp.
+pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_t n,
+                       int32_t *d_T, uint8_t *d_F, cudaStream_t stream) {
     if (n == 0) return POS_OK;
     cudaMemPool_t pool;
     pos_status st = scratch_pool(&pool);
@@ -242,7 +256,9 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
         uint32_t *perm = cursor + nk;
         uint16_t *keys = reinterpret_cast<uint16_t *>(perm + m);
         EvalParams p;
-        p.cands = reinterpret_cast<const uint4 *>(d_cands) + base;
+        p.per_stage_tp = per_stage_tp ? 1 : 0;
+        p.cands = per_stage_tp ? nullptr : static_cast<const uint4 *>(d_cands) + base;
+        p.cands_ex = per_stage_tp ? static_cast<const uint2 *>(d_cands) + 3 * base : nullptr;
         p.n = m;
         p.T = d_T + base;
         p.F = d_F + base;
@@ -263,13 +279,11 @@ pos_status launch_eval(Handle *h, const pos_candidate *d_cands, int64_t n, int32
             const int sgrid = (int)std::max<int64_t>(
                 1, std::min<int64_t>((m + kChunk - 1) / kChunk, 8LL * sm_count()));
             if (il) {
-                sort_hist_kernel<kKeysIl><<<grid, 256, 0, stream>>>(p.lay.sched, p.cands, m, hist,
-                                                                    keys, p.T, p.F);
+                sort_hist_kernel<kKeysIl><<<grid, 256, 0, stream>>>(p, m, hist, keys, p.T, p.F);
                 sort_scan_kernel<kKeysIl><<<1, 1024, 0, stream>>>(hist, offs, cursor);
                 sort_scatter_kernel<kKeysIl><<<sgrid, 512, 0, stream>>>(keys, m, cursor, perm);
             } else {
-                sort_hist_kernel<kKeys><<<grid, 256, 0, stream>>>(p.lay.sched, p.cands, m, hist,
-                                                                  keys, p.T, p.F);
+                sort_hist_kernel<kKeys><<<grid, 256, 0, stream>>>(p, m, hist, keys, p.T, p.F);
                 sort_scan_kernel<kKeys><<<1, 1024, 0, stream>>>(hist, offs, cursor);
                 sort_scatter_kernel<kKeys><<<sgrid, 512, 0, stream>>>(keys, m, cursor, perm);
             }
@@ -317,8 +331,23 @@ pos_status poseidon_eval_batch(void *handle, const pos_candidate *d_cands, int64
         return pos::fail(POS_EINVAL, "NULL buffer");
     if ((reinterpret_cast<uintptr_t>(d_cands) & 15) != 0)
         return pos::fail(POS_EINVAL, "candidates must be 16-byte aligned");
-    return pos::launch_eval(static_cast<pos::Handle *>(handle), d_cands, n, d_makespan,
+    return pos::launch_eval(static_cast<pos::Handle *>(handle), d_cands, false, n, d_makespan,
                             d_feasible, static_cast<cudaStream_t>(stream));
+}
+
+pos_status poseidon_eval_batch_ex(void *handle, const pos_candidate_ex *d_cands, int64_t n,
+                                  int32_t *d_makespan, uint8_t *d_feasible, void *stream) {
+    if (!handle) return pos::fail(POS_EINVAL, "handle is NULL");
+    if (n < 0) return pos::fail(POS_EINVAL, "n < 0");
+    if (n > 0 && (!d_cands || !d_makespan || !d_feasible))
+        return pos::fail(POS_EINVAL, "NULL buffer");
+    if ((reinterpret_cast<uintptr_t>(d_cands) & 7) != 0)
+        return pos::fail(POS_EINVAL, "candidates must be 8-byte aligned");
+    pos::Handle *h = static_cast<pos::Handle *>(handle);
+    if (h->lay.n_tp > 4)
+        return pos::fail(POS_EINVAL, "per-stage TP records need n_tp <= 4 (2-bit TP fields)");
+    return pos::launch_eval(h, d_cands, true, n, d_makespan, d_feasible,
+                            static_cast<cudaStream_t>(stream));
 }
 
 pos_status poseidon_eval_batch_host(void *handle, const pos_candidate *cands, int64_t n,
@@ -336,7 +365,7 @@ pos_status poseidon_eval_batch_host(void *handle, const pos_candidate *cands, in
     pos_status st = POS_OK;
     cudaError_t e = cudaMemcpy(dc, cands, bc, cudaMemcpyHostToDevice);
     if (e == cudaSuccess) {
-        st = pos::launch_eval(static_cast<pos::Handle *>(handle), dc, n, dt, df, 0);
+        st = pos::launch_eval(static_cast<pos::Handle *>(handle), dc, false, n, dt, df, 0);
         if (st == POS_OK) e = cudaMemcpy(makespan, dt, bt, cudaMemcpyDeviceToHost);
         if (st == POS_OK && e == cudaSuccess)
             e = cudaMemcpy(feasible, df, (size_t)n, cudaMemcpyDeviceToHost);

@@ -34,7 +34,9 @@ __host__ __device__ inline int fast_key_begin(int S) { return (S - 1) * 256; }
 __host__ __device__ inline int generic_key_begin(int S) { return 4096 + (S - 1) * 32; }
 
 struct EvalParams {
-    const uint4 *cands;
+    const uint4 *cands;    // 16-byte records (poseidon_eval_batch), or
+    const uint2 *cands_ex; // 24-byte records with a TP index per stage
+                           // (poseidon_eval_batch_ex; cands is then NULL)
     int64_t n;
     int32_t *T;
     uint8_t *F;
@@ -44,14 +46,45 @@ struct EvalParams {
                            // cuts[2j]: cut[1..S-1] in bytes 0..14, byte 15 = 1
                            // when the result is already written;
                            // cuts[2j+1]: (candidate index, type_code, the
-                           // record's S|M|tp|V word, 0), so the makespan
+                           // record's S|M|tp|V word, per-stage TP code), so the makespan
                            // kernels read 32 contiguous bytes and no record
     const void *blob;
     BlobLayout lay;
     int64_t gA, gD, gP;
     Programs pg;           // level programs of the schedule's short path
     int nkeys;             // kKeys, or kKeysIl under Interleaved 1F1B
+    int per_stage_tp;      // 1: records carry a TP index per stage (n_tp <= 4)
 };
+
+// The record fields every pass reads, in the 16-byte record's word layout:
+// x, y = composition rank, z = type code, w = S | M << 8 | tp << 16 | V << 24
+// (tp = 0 for a 24-byte record), plus the per-stage TP code of a 24-byte
+// record (TP index of stage s in bits [2s, 2s+2); 0 for 16-byte records).
+struct RecView {
+    uint4 rec;
+    uint32_t tpc;
+};
+__device__ __forceinline__ RecView load_record(const EvalParams &p, uint32_t i) {
+    RecView v;
+    if (p.per_stage_tp) {
+        // 24 bytes: u64 rank, u32 type code, u32 TP code, u8 S, M, V, pad, u32 pad
+        const uint2 a = __ldg(p.cands_ex + 3 * (size_t)i), b = __ldg(p.cands_ex + 3 * (size_t)i + 1),
+                    c = __ldg(p.cands_ex + 3 * (size_t)i + 2);
+        v.rec = make_uint4(a.x, a.y, b.x, (c.x & 0xffffu) | ((c.x & 0xff0000u) << 8));
+        v.tpc = b.y;
+    } else {
+        v.rec = __ldg(p.cands + i);
+        v.tpc = 0;
+    }
+    return v;
+}
+
+// Class of stage s: type_s * n_tp + its TP index, which is tp for a 16-byte
+// record (whose per-stage TP code reads 0) and the stage's field of the TP
+// code for a 24-byte record (whose tp reads 0), so no select is needed.
+__device__ __forceinline__ int stage_class(uint32_t tcode, uint32_t tpc, int tp, int n_tp, int s) {
+    return (int)((tcode >> (2 * s)) & 3u) * n_tp + tp + (int)((tpc >> (2 * s)) & 3u);
+}
 
 // Are the 2-bit type fields of stages 0..S-1 (1 <= S <= 16) all below
 // n_types (1..4)?  A field is >= n_types when its high bit is set
@@ -72,8 +105,8 @@ __device__ __forceinline__ bool types_ok(uint32_t tcode, int S, int n_types) {
 // multiple of N) and the overflow guard over the N*V virtual stages, and
 // unranks the composition of L layers into the virtual stages.  Memory is
 // checked by the makespan kernel (it needs the device chains).
-__device__ __forceinline__ uint4 decode_il(const Tab &t, const uint4 &rec, const EvalParams &p,
-                                           uint32_t i) {
+__device__ __forceinline__ uint4 decode_il(const Tab &t, const uint4 &rec, uint32_t tpc,
+                                           const EvalParams &p, uint32_t i) {
     uint64_t rank = (uint64_t)rec.x | ((uint64_t)rec.y << 32);
     const uint32_t tcode = rec.z;
     const int S = rec.w & 0xff;
@@ -83,7 +116,8 @@ __device__ __forceinline__ uint4 decode_il(const Tab &t, const uint4 &rec, const
     const int J = S * V, L = t.L();
     bool ok = S >= 1 && J <= POS_MAX_STAGES && J <= L && M >= 1 && M % S == 0 &&
               tp < t.n_tp() && rank < binom(t, L - 1, J - 1);
-    ok = ok && types_ok(tcode, S, t.n_types());
+    ok = ok && types_ok(tcode, S, t.n_types()) &&
+         types_ok(tpc, S, t.n_tp());  // tpc = 0 for 16-byte records
     const uint4 done = make_uint4(0, 0, 0, 1u << 24);
     if (!ok) {
         p.T[i] = -1;
@@ -114,8 +148,8 @@ __device__ __forceinline__ uint4 decode_il(const Tab &t, const uint4 &rec, const
 // positions.  Invalid and overflowing candidates are answered here.  S is a
 // runtime value and the stage loop is not unrolled, which keeps the kernel
 // small enough to run many warps per SM.
-__device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, const EvalParams &p,
-                                            uint32_t i) {
+__device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, uint32_t tpc,
+                                            const EvalParams &p, uint32_t i) {
     uint64_t rank = (uint64_t)rec.x | ((uint64_t)rec.y << 32);
     const uint32_t tcode = rec.z;
     const int S = rec.w & 0xff;
@@ -123,10 +157,11 @@ __device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, cons
     const int tp = (rec.w >> 16) & 0xff;
     const int L = t.L();
     if (t.ly->sched == POS_SCHED_INTERLEAVED_1F1B && (rec.w >> 24) >= 2)
-        return decode_il(t, rec, p, i);
+        return decode_il(t, rec, tpc, p, i);
     bool ok = S >= 1 && S <= POS_MAX_STAGES && M >= 1 && S <= L && tp < t.n_tp() &&
               rank < binom(t, L - 1, S - 1);
-    ok = ok && types_ok(tcode, S, t.n_types());
+    ok = ok && types_ok(tcode, S, t.n_types()) &&
+         types_ok(tpc, S, t.n_tp());  // tpc = 0 for 16-byte records
     const uint4 done = make_uint4(0, 0, 0, 1u << 24);  // byte 15 = 1: answered here
     if (!ok) {
         p.T[i] = -1;
@@ -150,7 +185,7 @@ __device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, cons
             if (s < 8) lo8 |= (uint64_t)c2 << (8 * s);
             else hi8 |= (uint64_t)c2 << (8 * (s - 8));
         }
-        const int cls = ((tcode >> (2 * s)) & 3) * t.n_tp() + tp;
+        const int cls = stage_class(tcode, tpc, tp, t.n_tp(), s);
         fits &= stage_fits(t, S, M, s, cls, c, c2);
         c = c2;
     }
@@ -167,12 +202,16 @@ struct EvalWith {
         static __device__ __forceinline__ void run(const Tab &t, const uint4 &rec,
                                                    const uint4 &packed, const Programs &pg,
                                                    int32_t &T) {
+            // rec: x = per-stage TP code (0 for 16-byte records), z = type
+            // code, w = S | M << 8 | tp << 16 | V << 24 (tp = 0 for 24-byte
+            // records)
             const uint32_t tcode = rec.z;
             const int M = (rec.w >> 8) & 0xff;
             const int tp = (rec.w >> 16) & 0xff;
             int cls[S], cut[S + 1];
 #pragma unroll
-            for (int s = 0; s < S; ++s) cls[s] = ((tcode >> (2 * s)) & 3) * t.n_tp() + tp;
+            for (int s = 0; s < S; ++s)
+                cls[s] = stage_class(tcode, rec.x, tp, t.n_tp(), s);
             const uint32_t pw[4] = {packed.x, packed.y, packed.z, packed.w};
             cut[0] = 0;
 #pragma unroll
@@ -223,7 +262,7 @@ __global__ void __launch_bounds__(kEvalThreads, MINB) eval_kernel(EvalParams p) 
             const uint4 meta = __ldg(p.cuts + 2 * (begin + j) + 1);
             active = (packed.w >> 24) == 0;  // not answered by the decode pass
             i = meta.x;
-            rec = make_uint4(0, 0, meta.y, meta.z);
+            rec = make_uint4(meta.w, 0u, meta.y, meta.z);
         }
         const int S = active ? (int)(rec.w & 0xff) : 0;
         int32_t T = -1;

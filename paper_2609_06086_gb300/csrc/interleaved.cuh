@@ -151,7 +151,7 @@ __device__ __forceinline__ void il_eval_one(const Tab &t, const uint4 &rec, cons
     const int q = M / N;
     int cls[N], cut[J + 1];
 #pragma unroll
-    for (int d = 0; d < N; ++d) cls[d] = ((tcode >> (2 * d)) & 3) * t.n_tp() + tp;
+    for (int d = 0; d < N; ++d) cls[d] = stage_class(tcode, rec.x, tp, t.n_tp(), d);
     const uint32_t pw[4] = {packed.x, packed.y, packed.z, packed.w};
     cut[0] = 0;
 #pragma unroll
@@ -214,7 +214,7 @@ __global__ void __launch_bounds__(kEvalThreads, MINB) il_eval_kernel(EvalParams 
             const uint4 meta = __ldg(p.cuts + 2 * (begin + j) + 1);
             active = (packed.w >> 24) == 0;  // not answered by the decode pass
             i = meta.x;
-            rec = make_uint4(0, 0, meta.y, meta.z);
+            rec = make_uint4(meta.w, 0u, meta.y, meta.z);
         }
         const int g = active ? (int)(rec.w & 0xff) * 32 + (int)(rec.w >> 24) : 0;  // N*32 + V
         int32_t T = -1;

@@ -46,6 +46,7 @@ def test_struct_layouts_match_the_header(P, tmp_path):
     fields = {
         "pos_tables": [f[0] for f in P.binding.pos_tables._fields_],
         "pos_candidate": ["map_rank", "type_code", "S", "M", "tp_idx", "V"],
+        "pos_candidate_ex": ["map_rank", "type_code", "tp_code", "S", "M", "V", "pad0", "pad1"],
         "pos_problem": [f[0] for f in P.binding.pos_problem._fields_],
         "pos_plan": [f[0] for f in P.binding.pos_plan._fields_],
         "pos_search_stats": [f[0] for f in P.binding.pos_search_stats._fields_],
@@ -72,6 +73,9 @@ def test_struct_layouts_match_the_header(P, tmp_path):
     assert int(got["pos_candidate"]) == gen.CANDIDATE_DTYPE.itemsize
     for f in fields["pos_candidate"]:
         assert int(got[f"pos_candidate.{f}"]) == gen.CANDIDATE_DTYPE.fields[f][1], f
+    assert int(got["pos_candidate_ex"]) == gen.CANDIDATE_EX_DTYPE.itemsize
+    for f in fields["pos_candidate_ex"]:
+        assert int(got[f"pos_candidate_ex.{f}"]) == gen.CANDIDATE_EX_DTYPE.fields[f][1], f
 
 
 def test_invalid_arguments_rejected_before_the_device(P):
