@@ -497,8 +497,20 @@ def main():
                     help="stage-level prune: 1 = Eq. 2 as printed, 2 = tightened bound")
     ap.add_argument("--frontier-cap", type=int, default=0,
                     help="frontier entries per depth (0 = library default)")
+    ap.add_argument("--eval-only", type=int, choices=[0, 1, 2], default=None,
+                    help="only the evaluator measurement, under this schedule (0 = 1F1B, "
+                         "1 = Eager 1F1B, 2 = Interleaved 1F1B), --steps calls per batch "
+                         "size, one JSON line per size (for profiling)")
     args = ap.parse_args()
     rank, world, local_rank = dist_env()
+    if args.eval_only is not None:
+        import torch
+        import paper_2609_06086_gb300 as P
+        peak = torch.cuda.get_device_properties(0).multi_processor_count * SM_LANES * 2070e6 / 1e12
+        for n in args.eval_sizes:
+            print(json.dumps(eval_throughput(P, torch, int(n), args.steps, peak,
+                                             schedule=args.eval_only)), flush=True)
+        return
     if args.impl == "reference":
         run_reference(args, rank, world)
     else:

@@ -243,13 +243,16 @@ __device__ __forceinline__ void dispatch_range(int S, const Tab &t, const uint4 
 template <int SLO, int SHI, int PATH, int MINB>
 __global__ void __launch_bounds__(kEvalThreads, MINB) eval_kernel(EvalParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
-    stage_blob(sm, p.blob, p.lay.bytes);
-    __syncthreads();
-    const Tab t = tab_at(sm, p.lay);
     constexpr bool kFast = PATH == kPathFast || PATH == kPathEager;
     const int key_lo = kFast ? fast_key_begin(SLO) : generic_key_begin(SLO);
     const int key_hi = kFast ? fast_key_begin(SHI + 1) : generic_key_begin(SHI + 1);
     const int64_t begin = p.offs[key_lo], end = p.offs[key_hi];
+    // blocks with no candidate (all of them when the range is empty) leave
+    // before staging the tables
+    if ((int64_t)blockIdx.x * blockDim.x >= end - begin) return;
+    stage_blob(sm, p.blob, p.lay.bytes);
+    __syncthreads();
+    const Tab t = tab_at(sm, p.lay);
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     // whole warps iterate together (ballots below)
     const int64_t span = ((end - begin) + 31) & ~(int64_t)31;

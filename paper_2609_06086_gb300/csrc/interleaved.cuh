@@ -199,10 +199,13 @@ __device__ __forceinline__ void il_dispatch(int N, int V, const Tab &t, const ui
 template <int PLO, int PHI, int MINB>
 __global__ void __launch_bounds__(kEvalThreads, MINB) il_eval_kernel(EvalParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
+    const int64_t begin = p.offs[kKeys + IlPair<PLO>::key], end = p.offs[kKeys + IlPair<PHI + 1>::key];
+    // blocks with no record (all of them when the range is empty) leave
+    // before staging the tables
+    if ((int64_t)blockIdx.x * blockDim.x >= end - begin) return;
     stage_blob(sm, p.blob, p.lay.bytes);
     __syncthreads();
     const Tab t = tab_at(sm, p.lay);
-    const int64_t begin = p.offs[kKeys + IlPair<PLO>::key], end = p.offs[kKeys + IlPair<PHI + 1>::key];
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     const int64_t span = ((end - begin) + 31) & ~(int64_t)31;
     for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < span; j += stride) {
