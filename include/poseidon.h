@@ -353,6 +353,17 @@ typedef struct pos_search_stats {
  */
 pos_status poseidon_search(const pos_problem *problem, pos_plan *out, pos_search_stats *stats);
 
+/*
+ * Measurement helper (no counterpart in the paper): runs a kernel made of
+ * the makespan kernels' relaxation, max(pred + edge, clock) + weight, in
+ * independent chains on every SM, twice, and reports the second run:
+ * *ops = int32 operations executed (3 per relaxation), *ms = its duration
+ * (CUDA events on `stream`).  ops / ms checks the INT32 roofline the
+ * ALU-bound kernels are measured against.  Synchronises the stream; uses a
+ * 4-byte stream-ordered allocation.  Errors: POS_EINVAL, POS_ECUDA.
+ */
+pos_status poseidon_int32_probe(void *stream, int64_t *ops, double *ms);
+
 /* Message describing the last error of the calling thread ("" if none). */
 const char *poseidon_last_error(void);
 

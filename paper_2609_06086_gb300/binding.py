@@ -28,7 +28,8 @@ MAX_STAGES = 16
 # the exported entry points, as declared in include/poseidon.h
 EXPORTS = ["poseidon_tables_create", "poseidon_tables_destroy", "poseidon_eval_batch",
            "poseidon_eval_batch_ex", "poseidon_eval_batch_host", "poseidon_argmin",
-           "poseidon_argmin_noalloc", "poseidon_search", "poseidon_last_error"]
+           "poseidon_argmin_noalloc", "poseidon_search", "poseidon_int32_probe",
+           "poseidon_last_error"]
 
 
 class pos_tables(C.Structure):
@@ -95,6 +96,7 @@ def lib():
         L.poseidon_argmin_noalloc.argtypes = [vp, vp, i64, vp, vp]
         L.poseidon_search.argtypes = [C.POINTER(pos_problem), C.POINTER(pos_plan),
                                       C.POINTER(pos_search_stats)]
+        L.poseidon_int32_probe.argtypes = [vp, C.POINTER(C.c_int64), C.POINTER(C.c_double)]
         L.poseidon_last_error.restype = C.c_char_p
         L.poseidon_last_error.argtypes = []
         for name in EXPORTS[:-1]:
@@ -160,6 +162,13 @@ def poseidon_eval_batch_ex(handle: Handle, d_cands: int, n: int, d_makespan: int
     """24-byte records with a TP index per stage; device pointers in and out
     (asynchronous on `stream`)."""
     _check(lib().poseidon_eval_batch_ex(handle.ptr, d_cands, n, d_makespan, d_feasible, stream))
+
+
+def poseidon_int32_probe(stream: int = 0):
+    """(int32 ops, ms) of the relaxation microbenchmark (see the header)."""
+    ops, ms = C.c_int64(), C.c_double()
+    _check(lib().poseidon_int32_probe(stream, C.byref(ops), C.byref(ms)))
+    return ops.value, ms.value
 
 
 def poseidon_eval_batch_host(handle: Handle, cands: np.ndarray):

@@ -186,3 +186,15 @@ def test_limits_L127_four_types_eight_tp(P, orc):
     Tr, Fr = orc.eval_batch(orc.OracleTables(**tab), c)
     assert np.array_equal(T, Tr) and np.array_equal(F, Fr)
     assert (F == 3).sum() > 0 and (F == 1).sum() > 0
+
+
+def test_int32_probe_runs_near_the_lane_count(P):
+    """The relaxation microbenchmark executes its stated op count; its rate
+    is within a plausible band of SMs x 128 lanes x the maximum clock."""
+    import torch
+    ops, ms = P.binding.poseidon_int32_probe(torch.cuda.current_stream().cuda_stream)
+    props = torch.cuda.get_device_properties(0)
+    nominal = props.multi_processor_count * 128 * 2.07e9
+    rate = ops / (ms / 1e3)
+    assert ops == props.multi_processor_count * 8 * 256 * 4096 * 8 * 6
+    assert 0.2 * nominal < rate < 1.5 * nominal, rate / nominal
