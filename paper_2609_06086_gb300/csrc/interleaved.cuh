@@ -208,13 +208,26 @@ __global__ void __launch_bounds__(kEvalThreads, MINB) il_eval_kernel(EvalParams 
     const Tab t = tab_at(sm, p.lay);
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     const int64_t span = ((end - begin) + 31) & ~(int64_t)31;
-    for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < span; j += stride) {
+    int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    // the next decoded record is loaded one iteration ahead, so its memory
+    // latency overlaps the current candidate's wavefront
+    const uint4 none = make_uint4(0, 0, 0, 1u << 24);
+    uint4 next_packed = none, next_meta = none;
+    if (j < end - begin) {
+        next_packed = __ldg(p.cuts + 2 * (begin + j));
+        next_meta = __ldg(p.cuts + 2 * (begin + j) + 1);
+    }
+    for (; j < span; j += stride) {
         bool active = j < end - begin;
         uint32_t i = 0;
-        uint4 rec = make_uint4(0, 0, 0, 0), packed = make_uint4(0, 0, 0, 0);
+        uint4 rec = make_uint4(0, 0, 0, 0);
+        const uint4 packed = next_packed, meta = next_meta;
+        next_packed = none;
+        if (j + stride < end - begin) {
+            next_packed = __ldg(p.cuts + 2 * (begin + j + stride));
+            next_meta = __ldg(p.cuts + 2 * (begin + j + stride) + 1);
+        }
         if (active) {
-            packed = __ldg(p.cuts + 2 * (begin + j));
-            const uint4 meta = __ldg(p.cuts + 2 * (begin + j) + 1);
             active = (packed.w >> 24) == 0;  // not answered by the decode pass
             i = meta.x;
             rec = make_uint4(meta.w, 0u, meta.y, meta.z);

@@ -182,15 +182,16 @@ __global__ void __launch_bounds__(256, leaf_min_blocks(S, PATH)) leaf_kernel(Lea
     const unsigned long long stride = (unsigned long long)gridDim.x * blockDim.x;
     // all lanes of a warp iterate together (the warp minimum uses shuffles)
     const unsigned long long n_round = (n + 31) & ~31ull;
-    for (unsigned long long i = blockIdx.x * (unsigned long long)blockDim.x + threadIdx.x;
-         i < n_round; i += stride) {
+    const Vec32 none = {make_uint4(kLeafHole, 0, 0, 0), make_uint4(0, 0, 0, 0)};
+    unsigned long long i = blockIdx.x * (unsigned long long)blockDim.x + threadIdx.x;
+    // the next plan's record is loaded one iteration ahead, so its memory
+    // latency overlaps the current plan's wavefront
+    Vec32 next = i < n ? load32(p.leaves + i) : none;
+    for (; i < n_round; i += stride) {
         unsigned long long obj = ~0ull, idx = ~0ull;
-        uint32_t sl = kLeafHole;
-        Vec32 lv = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};
-        if (i < n) {
-            lv = load32(p.leaves + i);
-            sl = lv.a.x;
-        }
+        const Vec32 lv = next;
+        next = i + stride < n ? load32(p.leaves + i + stride) : none;
+        const uint32_t sl = lv.a.x;
         if (sl != kLeafHole) {
             const SliceRec &sr = p.slices[sl];
             int cut[S + 1], cls[S];
