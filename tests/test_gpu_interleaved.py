@@ -157,3 +157,20 @@ def test_one_device_is_sequential(P, orc):
     for (rank, tc, N, M, _, V), t in zip(rows, T):
         k = tc & 3
         assert t == M * int(fwd[k].sum() + bwd[k].sum()) + int(ds[k].sum())
+
+
+def test_limits_L127_four_types_eight_tp(P, orc):
+    """The largest tables the ABI accepts under Interleaved 1F1B: L = 127,
+    4 types x 8 TP degrees, N*V up to 16 (ranks near C(126, 15)), M up to 255."""
+    from tests.test_gpu_eval import _max_tables
+    tab = _max_tables(127, 4, 8, 5)
+    h = P.Handle(P.Tables(**tab), IL)
+    c = gen.interleaved_candidates(20_000, L=127, n_types=4, seed=6, m_lo=1, m_hi=255)
+    c["tp_idx"] = np.random.default_rng(6).integers(0, 8, len(c))
+    J = c["S"].astype(np.int64) * c["V"].astype(np.int64)
+    top = np.nonzero(J == 16)[0][:40]
+    c["map_rank"][top] = math.comb(126, 15) - 1 - np.arange(len(top), dtype=np.uint64)
+    T, F = eval_device(P, h, c)
+    Tr, Fr = orc.eval_batch(orc.OracleTables(**tab, schedule=IL), c)
+    assert np.array_equal(T, Tr) and np.array_equal(F, Fr)
+    assert (F == 3).sum() > 0 and (F == 1).sum() > 0

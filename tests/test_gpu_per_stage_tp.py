@@ -101,3 +101,31 @@ def test_invalid_fields_and_too_many_tp_indices(P, orc):
     with pytest.raises(P.PoseidonError) as e:
         eval_device_ex(P, h, c)
     assert e.value.status == P.binding.POS_EINVAL
+
+
+@pytest.mark.parametrize("schedule", [0, 1, 2])
+def test_limits_L127_four_types_four_tp(P, orc, schedule):
+    """L = 127 with 4 types x 4 TP indices (every 2-bit TP field used), S up
+    to 16 and M up to 255 (guard permitting), under each schedule."""
+    from tests.test_gpu_eval import _max_tables
+    tab = _max_tables(127, 4, 4, 7 + schedule)
+    h = P.Handle(P.Tables(**tab), schedule)
+    if schedule == 2:
+        base = gen.interleaved_candidates(10_000, L=127, n_types=4, seed=8, m_lo=1, m_hi=255)
+        c = np.zeros(len(base), dtype=gen.CANDIDATE_EX_DTYPE)
+        for f in ("map_rank", "type_code", "S", "M", "V"):
+            c[f] = base[f]
+        pc = np.random.default_rng(8).integers(0, 1 << 16, len(c)).astype(np.uint32)
+        mask = ((np.uint64(1) << (2 * base["S"].astype(np.uint64))) - np.uint64(1))
+        c["tp_code"] = pc & mask.astype(np.uint32)
+    else:
+        c = gen.per_stage_tp_candidates(20_000, L=127, n_types=4, n_tp=4, seed=8,
+                                        M_range=(1, 255))
+        c["map_rank"][:30] = math.comb(126, 15) - 1 - np.arange(30, dtype=np.uint64)
+        c["S"][:30] = 16
+        c["type_code"][:30] = 0xffffffff
+        c["tp_code"][:30] = 0xffffffff
+    T, F = eval_device_ex(P, h, c)
+    Tr, Fr = orc.eval_batch_ex(orc.OracleTables(**tab, schedule=schedule), c)
+    assert np.array_equal(T, Tr) and np.array_equal(F, Fr)
+    assert (F == 1).sum() > 0
