@@ -891,6 +891,9 @@ struct Workspace {
     size_t h_stage_cap = 0;
     unsigned char *h_read = nullptr;           // pinned landing area for reads
     size_t h_read_cap = 0;
+    unsigned long long *h_lb = nullptr;        // pinned landing area of the root bounds
+    size_t h_lb_cap = 0;                       // (elements)
+    cudaEvent_t ev_lb = nullptr;               // recorded after their copy
     std::vector<cudaEvent_t> evs;              // timing events of the batch pipelines
 };
 
@@ -908,6 +911,7 @@ static pos_status get_workspace(Workspace **out) {
         if (!w) return fail(POS_ENOMEM, "host allocation failed");
         cudaError_t e = cudaStreamCreateWithFlags(&w->stream, cudaStreamNonBlocking);
         for (int i = 0; i < 3 && e == cudaSuccess; ++i) e = cudaEventCreate(&w->ev[i]);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&w->ev_lb, cudaEventDisableTiming);
         if (e == cudaSuccess) e = cudaMallocHost(&w->h_cnt, 64 * sizeof(unsigned long long));
         if (e != cudaSuccess) {
             delete w;
@@ -1400,6 +1404,20 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         if (p->profile) POS_CUDA(cudaEventRecord(s.ev[1], s.stream));
         s.launches++;
         s.n_bound++;
+        // the root bounds order the slices: their copy to the host is queued
+        // here and waited for alone, so the warm-up kernels queued next run
+        // while the host plans the batches
+        if ((size_t)n_slices > s.ws.h_lb_cap) {
+            POS_CUDA(cudaStreamSynchronize(s.stream));  // no copy into the old area in flight
+            if (s.ws.h_lb) cudaFreeHost(s.ws.h_lb);
+            s.ws.h_lb = nullptr;
+            s.ws.h_lb_cap = 0;
+            POS_CUDA(cudaMallocHost(&s.ws.h_lb, sizeof(unsigned long long) * n_slices));
+            s.ws.h_lb_cap = (size_t)n_slices;
+        }
+        POS_CUDA(cudaMemcpyAsync(s.ws.h_lb, s.ws.d_lb.p, sizeof(unsigned long long) * n_slices,
+                                 cudaMemcpyDeviceToHost, s.stream));
+        POS_CUDA(cudaEventRecord(s.ws.ev_lb, s.stream));
         // counts of the greedy plans per M index, then one leaf launch each
         std::vector<unsigned long long> gc(p->n_M);
         for (int mi = 0; mi < p->n_M; ++mi) gc[mi] = feas_by_m[mi].size();
@@ -1443,10 +1461,19 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
             warm_evals += (uint64_t)n_s;
         }
     }
-    std::vector<unsigned long long> best(n_slices);
-    if ((st = sync_read(s, best.data(), s.d_best.p, sizeof(unsigned long long) * n_slices)) !=
-        POS_OK)
+    // slice order: with the completion bounds, by each slice's root lower
+    // bound (the slice most likely to hold the optimum first), waiting for
+    // their copy only; otherwise by the best warm-up plan of the slice,
+    // after the warm-up
+    const bool by_bound = p->prune == 2 && n_feasible > 0;
+    std::vector<unsigned long long> key(n_slices);
+    if (by_bound) {
+        POS_CUDA(cudaEventSynchronize(s.ws.ev_lb));
+        std::memcpy(key.data(), s.ws.h_lb, sizeof(unsigned long long) * n_slices);
+    } else if ((st = sync_read(s, key.data(), s.d_best.p,
+                               sizeof(unsigned long long) * n_slices)) != POS_OK) {
         return st;
+    }
     if (p->profile && s.n_bound) {
         float ms_b = 0;
         POS_CUDA(cudaEventElapsedTime(&ms_b, s.ev[0], s.ev[1]));
@@ -1461,14 +1488,6 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         unsigned long long best;
     };
     std::vector<Group> groups;
-    // slice order: with the completion bounds, by each slice's root lower
-    // bound (the slice most likely to hold the optimum first); otherwise by
-    // the best warm-up plan of the slice
-    std::vector<unsigned long long> key = best;
-    if (p->prune == 2 && n_feasible > 0 &&
-        (st = sync_read(s, key.data(), s.ws.d_lb.p, sizeof(unsigned long long) * n_slices)) !=
-            POS_OK)
-        return st;
     for (int mi = 0; mi < p->n_M; ++mi) {
         if (feas_by_m[mi].empty()) continue;
         auto &fl = feas_by_m[mi];
