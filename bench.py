@@ -350,6 +350,12 @@ def run_ours(args, rank, world, local_rank):
     evals = [eval_throughput(P, torch, int(n), 5, peak_alu) for n in args.eval_sizes]
     for e in evals:
         e["frac_of_measured"] = round(e["achieved"] / probe["tops"], 4)
+    # batch-size sweep of the same evaluator (config 5)
+    sweep = []
+    for n in args.eval_sweep:
+        e = eval_throughput(P, torch, int(n), 5, peak_alu)
+        sweep.append({k: e[k] for k in ("batch", "ms_per_call", "evals_per_s",
+                                         "relaxations_per_s", "achieved", "frac")})
     evals_eager = [eval_throughput(P, torch, int(n), 5, peak_alu, schedule=1)
                    for n in args.eval_sizes[:1]]
     evals_il = [eval_throughput(P, torch, int(n), 5, peak_alu, schedule=2)
@@ -479,6 +485,7 @@ def run_ours(args, rank, world, local_rank):
         "int32_probe": probe,
         "other_prune": other_prune,
         "eval_throughput": evals,
+        "eval_sweep": sweep,
         "eval_throughput_eager": evals_eager,
         "eval_throughput_interleaved": evals_il,
         "eager_search": eager_search,
@@ -507,6 +514,8 @@ def main():
     ap.add_argument("--backend", choices=["nccl", "gloo"], default="nccl")
     ap.add_argument("--eval-sizes", type=float, nargs="*", default=[1e7],
                     help="config-5 batch sizes for the evaluator measurement")
+    ap.add_argument("--eval-sweep", type=float, nargs="*", default=[1e4, 1e5, 1e6, 1e8],
+                    help="further config-5 batch sizes (1F1B), reported as eval_sweep")
     ap.add_argument("--prune", type=int, choices=[1, 2], default=2,
                     help="stage-level prune: 1 = Eq. 2 as printed, 2 = tightened bound")
     ap.add_argument("--frontier-cap", type=int, default=0,

@@ -23,6 +23,10 @@ pos_status cuda_fail(cudaError_t e, const char *what);
 // device unless an earlier call already set at least that much (the
 // attribute call costs host time that a launch-bound pipeline feels).
 pos_status ensure_smem(const void *kernel, int smem);
+// Resident blocks per SM of `kernel` at (threads, smem), from the occupancy
+// calculator once per device and configuration, then from a cache (the
+// query costs host time on every launch otherwise).
+pos_status blocks_per_sm(const void *kernel, int threads, int smem, int *out);
 
 #define POS_CUDA(call)                                           \
     do {                                                         \

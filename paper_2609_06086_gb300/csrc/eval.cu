@@ -196,7 +196,7 @@ pos_status launch_decode(const EvalParams &p, cudaStream_t stream) {
     const int smem = p.lay.bytes;
     POS_TRY(ensure_smem(reinterpret_cast<const void *>(decode_kernel), smem));
     int per_sm = 0;
-    POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, decode_kernel, 256, smem));
+    POS_TRY(blocks_per_sm(reinterpret_cast<const void *>(decode_kernel), 256, smem, &per_sm));
     const int64_t blocks = (p.n + 255) / 256;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)std::max(per_sm, 1) * sm_count()));
     decode_kernel<<<grid, 256, smem, stream>>>(p);

@@ -288,7 +288,7 @@ pos_status launch_eval_range(const EvalParams &p, cudaStream_t stream) {
     const int smem = p.lay.bytes;
     POS_TRY(ensure_smem(reinterpret_cast<const void *>(kern), smem));
     int per_sm = 0;
-    POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kEvalThreads, smem));
+    POS_TRY(blocks_per_sm(reinterpret_cast<const void *>(kern), kEvalThreads, smem, &per_sm));
     if (per_sm < 1) return fail(POS_ECUDA, "eval kernel does not fit on an SM");
     const int64_t blocks = (p.n + kEvalThreads - 1) / kEvalThreads;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)per_sm * sm_count()));

@@ -1321,8 +1321,8 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     POS_TRY(ensure_smem(reinterpret_cast<const void *>(level_kernel<false, 0>), smem));
     POS_TRY(ensure_smem(reinterpret_cast<const void *>(feas_kernel), smem));
     POS_TRY(ensure_smem(reinterpret_cast<const void *>(bound_kernel), smem));
-    POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-        &per_sm, level_kernel<false, 0>, kThreads, timing_layout(s.h->lay).bytes));
+    POS_TRY(blocks_per_sm(reinterpret_cast<const void *>(level_kernel<false, 0>), kThreads,
+                          timing_layout(s.h->lay).bytes, &per_sm));
     s.grid_level = std::max(1, per_sm) * sm_count();
     s.grid_leaf = 2 * sm_count();
 

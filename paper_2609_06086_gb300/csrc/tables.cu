@@ -2,8 +2,10 @@
 // a1: per-class exclusive prefix sums of the Sec. 4.1.3 weights and the
 // Sec. 3.2 memory footprints).
 #include <algorithm>
+#include <atomic>
 #include <cstring>
 #include <map>
+#include <tuple>
 #include <mutex>
 #include <new>
 #include <string>
@@ -42,11 +44,35 @@ pos_status ensure_smem(const void *kernel, int smem) {
     return POS_OK;
 }
 
+pos_status blocks_per_sm(const void *kernel, int threads, int smem, int *out) {
+    static std::mutex mu;
+    // (device, kernel, threads, shared bytes) -> resident blocks per SM
+    static std::map<std::tuple<int, const void *, int, int>, int> known;
+    int dev = 0;
+    POS_CUDA(cudaGetDevice(&dev));
+    std::lock_guard<std::mutex> lock(mu);
+    const auto key = std::make_tuple(dev, kernel, threads, smem);
+    const auto it = known.find(key);
+    if (it != known.end()) {
+        *out = it->second;
+        return POS_OK;
+    }
+    int n = 0;
+    POS_CUDA(cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kernel, threads, smem));
+    known[key] = n;
+    *out = n;
+    return POS_OK;
+}
+
 int sm_count() {
+    static std::atomic<int> known[64];  // per device, 0 = not queried yet
     int dev = 0, n = 0;
     cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && (n = known[dev].load(std::memory_order_relaxed)) > 0) return n;
     cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-    return n > 0 ? n : 1;
+    if (n <= 0) return 1;
+    if (dev >= 0 && dev < 64) known[dev].store(n, std::memory_order_relaxed);
+    return n;
 }
 
 static int align16(int x) { return (x + 15) & ~15; }
