@@ -154,7 +154,10 @@ typedef struct pos_candidate_ex {
 
 /*
  * Copy the tables to the current CUDA device and build the per-class
- * exclusive prefix sums used by every kernel (hot-path step a1, Sec. 4.1.3).
+ * exclusive prefix sums used by every kernel (hot-path step a1, Sec. 4.1.3)
+ * and, when it takes at most 32 KB, a byte table of each class's largest
+ * memory-feasible stage end per start layer and in-flight count (the
+ * evaluator's memory check).
  * *handle owns the device copies until poseidon_tables_destroy.  schedule
  * (POS_SCHED_1F1B, POS_SCHED_EAGER_1F1B or POS_SCHED_INTERLEAVED_1F1B)
  * applies to every evaluation through the handle.

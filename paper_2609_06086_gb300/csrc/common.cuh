@@ -76,7 +76,14 @@ struct Handle {
     void *d_blob;  // device copy of the blob
     // overflow guard terms: sum_l max_k(fwd+bwd), sum_l max_k dsync, max p2p
     int64_t guard_A, guard_D, guard_P;
+    // memory-limit table of the evaluation's decode pass (after the blob in
+    // the same allocation, byte lim_off): lim[k][w-1][a] = the largest b with
+    // sum_{l in [a,b)} (mem_w + w mem_a) <= cap[k] (a when no layer fits), for
+    // w = 1..lim_w in-flight micro-batches; lim_bytes = 0 when the table
+    // would exceed kLimMaxBytes and the pass checks the sums directly
+    int lim_off, lim_w, lim_bytes;
 };
+constexpr int kLimMaxBytes = 32768;
 
 pos_status validate_tables(const pos_tables *t);
 pos_status create_handle(const pos_tables *t, int sched, Handle **out);

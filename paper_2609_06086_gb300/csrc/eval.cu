@@ -164,12 +164,22 @@ __global__ void sort_scatter_kernel(const uint16_t *keys, int64_t n, uint32_t *c
     }
 }
 
-// Decode pass over the whole sorted range [0, offs[nkeys]).
+// Decode pass over the whole sorted range [0, offs[nkeys]).  LIM: only the
+// binomials (the blob's first off_Pw bytes) and the memory-limit table are
+// staged, the table right after the binomials.
+template <bool LIM>
 __global__ void __launch_bounds__(256, 4) decode_kernel(EvalParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
-    stage_blob(sm, p.blob, p.lay.bytes);
+    if constexpr (LIM) {
+        stage_blob(sm, p.blob, p.lay.off_Pw);
+        stage_blob(sm + p.lay.off_Pw, static_cast<const unsigned char *>(p.blob) + p.lim_off,
+                   p.lim_bytes);
+    } else {
+        stage_blob(sm, p.blob, p.lay.bytes);
+    }
     __syncthreads();
     const Tab t = tab_at(sm, p.lay);
+    const uint8_t *lim = sm + p.lay.off_Pw;
     const int64_t total = p.offs[p.nkeys];
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     const int64_t span = (total + 31) & ~(int64_t)31;
@@ -184,7 +194,7 @@ __global__ void __launch_bounds__(256, 4) decode_kernel(EvalParams p) {
             v = load_record(p, i);
         }
         uint4 out = make_uint4(0, 0, 0, 1u << 24);
-        if (active) out = decode_one(t, v.rec, v.tpc, p, i);
+        if (active) out = decode_one<LIM>(t, v.rec, v.tpc, p, i, lim);
         if (active) {
             p.cuts[2 * j] = out;
             p.cuts[2 * j + 1] = make_uint4(i, v.rec.z, v.rec.w, v.tpc);
@@ -193,13 +203,17 @@ __global__ void __launch_bounds__(256, 4) decode_kernel(EvalParams p) {
 }
 
 pos_status launch_decode(const EvalParams &p, cudaStream_t stream) {
-    const int smem = p.lay.bytes;
-    POS_TRY(ensure_smem(reinterpret_cast<const void *>(decode_kernel), smem));
+    const bool lim = p.lim_bytes > 0;
+    const void *kern = lim ? reinterpret_cast<const void *>(decode_kernel<true>)
+                           : reinterpret_cast<const void *>(decode_kernel<false>);
+    const int smem = lim ? p.lay.off_Pw + p.lim_bytes : p.lay.bytes;
+    POS_TRY(ensure_smem(kern, smem));
     int per_sm = 0;
-    POS_TRY(blocks_per_sm(reinterpret_cast<const void *>(decode_kernel), 256, smem, &per_sm));
+    POS_TRY(blocks_per_sm(kern, 256, smem, &per_sm));
     const int64_t blocks = (p.n + 255) / 256;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)std::max(per_sm, 1) * sm_count()));
-    decode_kernel<<<grid, 256, smem, stream>>>(p);
+    if (lim) decode_kernel<true><<<grid, 256, smem, stream>>>(p);
+    else decode_kernel<false><<<grid, 256, smem, stream>>>(p);
     POS_CUDA(cudaGetLastError());
     return POS_OK;
 }
@@ -272,6 +286,9 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
         p.gP = h->guard_P;
         p.pg = pg;
         p.nkeys = nk;
+        p.lim_off = h->lim_off;
+        p.lim_w = h->lim_w;
+        p.lim_bytes = h->lim_bytes;
         const int grid = (int)std::max<int64_t>(
             1, std::min<int64_t>((m + 255) / 256, 4LL * sm_count()));
         cudaError_t e = cudaMemsetAsync(hist, 0, sizeof(uint32_t) * nk, stream);

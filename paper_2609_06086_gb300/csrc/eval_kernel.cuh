@@ -54,6 +54,9 @@ struct EvalParams {
     Programs pg;           // level programs of the schedule's short path
     int nkeys;             // kKeys, or kKeysIl under Interleaved 1F1B
     int per_stage_tp;      // 1: records carry a TP index per stage (n_tp <= 4)
+    // the handle's memory-limit table (Handle::lim_*): the decode pass stages
+    // the binomials and this table and checks memory with one byte per stage
+    int lim_off, lim_w, lim_bytes;
 };
 
 // The record fields every pass reads, in the 16-byte record's word layout:
@@ -144,12 +147,14 @@ __device__ __forceinline__ uint4 decode_il(const Tab &t, const uint4 &rec, uint3
 
 // Decode pass for one candidate: checks its fields and the overflow guard,
 // unranks the composition stage by stage (the steps of unrank_cuts),
-// checks each stage's memory as soon as its cut is known, and packs the cut
-// positions.  Invalid and overflowing candidates are answered here.  S is a
+// checks each stage's memory as soon as its cut is known (LIM: by the
+// memory-limit table staged at `lim`), and packs the cut positions.  Invalid and overflowing candidates are answered here.  S is a
 // runtime value and the stage loop is not unrolled, which keeps the kernel
 // small enough to run many warps per SM.
+template <bool LIM>
 __device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, uint32_t tpc,
-                                            const EvalParams &p, uint32_t i) {
+                                            const EvalParams &p, uint32_t i,
+                                            const uint8_t *lim) {
     uint64_t rank = (uint64_t)rec.x | ((uint64_t)rec.y << 32);
     const uint32_t tcode = rec.z;
     const int S = rec.w & 0xff;
@@ -186,7 +191,12 @@ __device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, uint
             else hi8 |= (uint64_t)c2 << (8 * (s - 8));
         }
         const int cls = stage_class(tcode, tpc, tp, t.n_tp(), s);
-        fits &= stage_fits(t, S, M, s, cls, c, c2);
+        if constexpr (LIM) {
+            const int w = inflight(t.ly->sched, S, M, s);
+            fits &= c2 <= (int)lim[(cls * p.lim_w + w - 1) * (L + 1) + c];
+        } else {
+            fits &= stage_fits(t, S, M, s, cls, c, c2);
+        }
         c = c2;
     }
     p.F[i] = fits ? POS_FEAS_YES : POS_FEAS_NO;

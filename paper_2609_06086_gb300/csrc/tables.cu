@@ -160,6 +160,27 @@ __global__ void prefix_rows_kernel(unsigned char *blob, BlobLayout ly) {
     }
 }
 
+// One block per (class, in-flight count w): lim[k][w-1][a] for every start
+// a, by binary search (the memory need grows with the layer count, the
+// tables being non-negative).
+__global__ void lim_kernel(unsigned char *blob, BlobLayout ly, int wmax, int lim_off) {
+    const int k = blockIdx.x / wmax, w = blockIdx.x % wmax + 1, L = ly.L;
+    const int64_t *Pw = reinterpret_cast<const int64_t *>(blob + ly.off_Pw) + (int64_t)k * (L + 1);
+    const int64_t *Pa = reinterpret_cast<const int64_t *>(blob + ly.off_Pa) + (int64_t)k * (L + 1);
+    const int64_t cap = reinterpret_cast<const int64_t *>(blob + ly.off_cap)[k];
+    uint8_t *out = blob + lim_off + (size_t)blockIdx.x * (L + 1);
+    for (int a = threadIdx.x; a <= L; a += blockDim.x) {
+        int lo = a, hi = L;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) / 2;
+            const int64_t need = (Pw[mid] - Pw[a]) + (int64_t)w * (Pa[mid] - Pa[a]);
+            if (need <= cap) lo = mid;
+            else hi = mid - 1;
+        }
+        out[a] = (uint8_t)lo;
+    }
+}
+
 pos_status validate_tables(const pos_tables *t) {
     if (!t) return fail(POS_EINVAL, "tables is NULL");
     if (t->L < 1 || t->L > POS_MAX_LAYERS) return fail(POS_EINVAL, "L must be in 1..127");
@@ -272,10 +293,20 @@ pos_status create_handle(const pos_tables *t, int sched, Handle **out) {
     h->guard_A = A;
     h->guard_D = D;
     h->guard_P = P;
+    // in-flight micro-batches of a stage: at most 16 (1F1B), 31 (Eager 1F1B)
+    h->lim_w = sched == POS_SCHED_EAGER_1F1B ? 2 * POS_MAX_STAGES - 1 : POS_MAX_STAGES;
+    h->lim_off = ly.bytes;
+    const long long lb = (long long)ly.K * h->lim_w * (ly.L + 1);
+    h->lim_bytes = lb <= kLimMaxBytes ? (int)((lb + 15) & ~15ll) : 0;
     cudaError_t e = cudaGetDevice(&h->device);
-    if (e == cudaSuccess) e = cudaMalloc(&h->d_blob, ly.bytes);
+    if (e == cudaSuccess) e = cudaMalloc(&h->d_blob, (size_t)ly.bytes + h->lim_bytes);
     if (e == cudaSuccess) e = cudaMemcpy(h->d_blob, host.data(), ly.bytes, cudaMemcpyHostToDevice);
     if (e == cudaSuccess && launch_prefix_rows(h->d_blob, ly, 0) != POS_OK) e = cudaErrorLaunchFailure;
+    if (e == cudaSuccess && h->lim_bytes > 0) {
+        lim_kernel<<<ly.K * h->lim_w, 128>>>(static_cast<unsigned char *>(h->d_blob), ly,
+                                            h->lim_w, h->lim_off);
+        e = cudaGetLastError();
+    }
     if (e == cudaSuccess) e = cudaStreamSynchronize(0);
     if (e != cudaSuccess) {
         if (h->d_blob) cudaFree(h->d_blob);
