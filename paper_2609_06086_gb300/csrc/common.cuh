@@ -692,9 +692,13 @@ __device__ __forceinline__ int32_t makespan_program(const StageW<S> &w, const ui
         Bo[s] = 0;
         clk[s] = 0;
     }
+    // the next level's word is loaded one level ahead, so the load latency
+    // overlaps the current level's relaxations
+    uint64_t next = n_levels > 0 ? __ldg(prog) : 0ull;
 #pragma unroll 1
     for (int l = 0; l < n_levels; ++l) {
-        const uint64_t word = __ldg(prog + l);
+        const uint64_t word = next;
+        if (l + 1 < n_levels) next = __ldg(prog + l + 1);
         const uint32_t fm = (uint32_t)word & 0xffffu, bm = (uint32_t)(word >> 16) & 0xffffu;
         const uint32_t lm = (uint32_t)(word >> 32) & 0xffffu;
 #pragma unroll
