@@ -274,8 +274,9 @@ def per_stage_tp_candidates(n: int, L: int, n_types: int, n_tp: int, seed: int =
         tc |= np.where(keep, ty[:, s] << np.uint32(2 * s), 0).astype(np.uint32)
         pc |= np.where(keep, tp[:, s] << np.uint32(2 * s), 0).astype(np.uint32)
     u = rng.integers(0, np.iinfo(np.uint64).max, size=n, dtype=np.uint64, endpoint=True)
-    highs = [math.comb(L - 1, k - 1) if 1 <= k <= L else 1 for k in range(17)]
-    rank = np.array([int(x) % highs[k] for x, k in zip(u.tolist(), S.tolist())], dtype=np.uint64)
+    highs = np.array([math.comb(L - 1, k - 1) if 1 <= k <= L else 1 for k in range(17)],
+                     dtype=np.uint64)  # C(126, 15) < 2^64
+    rank = u % highs[S]
     out = np.zeros(n, dtype=CANDIDATE_EX_DTYPE)
     out["map_rank"] = rank
     out["type_code"] = tc
@@ -304,9 +305,8 @@ def interleaved_candidates(n: int, L: int = 64, n_types: int = 2, seed: int = 0,
     u = rng.integers(0, np.iinfo(np.uint64).max, size=n, dtype=np.uint64, endpoint=True)
     J = N * V
     highs = np.array([math.comb(L - 1, j - 1) if 1 <= j <= L else 1 for j in range(17)],
-                     dtype=object)
-    rank = np.array([int(x) % int(highs[j]) for x, j in zip(u.tolist(), J.tolist())],
-                    dtype=np.uint64)
+                     dtype=np.uint64)  # C(126, 15) < 2^64
+    rank = u % highs[J]
     out = np.zeros(n, dtype=CANDIDATE_DTYPE)
     out["map_rank"] = rank
     out["type_code"] = tc

@@ -174,3 +174,25 @@ def test_limits_L127_four_types_eight_tp(P, orc):
     Tr, Fr = orc.eval_batch(orc.OracleTables(**tab, schedule=IL), c)
     assert np.array_equal(T, Tr) and np.array_equal(F, Fr)
     assert (F == 3).sum() > 0 and (F == 1).sum() > 0
+
+
+def test_bench_size_sampled(P, orc):
+    """The bench's interleaved batch (1e7 records, one call); 20,000 sampled
+    outputs checked against the oracle."""
+    import torch
+    w = gen.config5_tables()
+    n = 10_000_000
+    c = gen.interleaved_candidates(n, L=w.L, seed=0)
+    h = P.Handle(P.Tables.from_workload(w), IL)
+    d_c = torch.from_numpy(c.view(np.uint8)).cuda()
+    d_T = torch.empty(n, dtype=torch.int32, device="cuda")
+    d_F = torch.empty(n, dtype=torch.uint8, device="cuda")
+    P.poseidon_eval_batch(h, d_c.data_ptr(), n, d_T.data_ptr(), d_F.data_ptr(),
+                          torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+    idx = np.sort(np.random.default_rng(5).choice(n, 20_000, replace=False))
+    idx = np.concatenate([idx, [0, n - 1]])
+    Tr, Fr = orc.eval_batch(orc.OracleTables.from_workload(w, schedule=IL), c[idx])
+    ti = torch.from_numpy(idx).cuda()
+    assert np.array_equal(d_T[ti].cpu().numpy(), Tr)
+    assert np.array_equal(d_F[ti].cpu().numpy(), Fr)
