@@ -183,16 +183,23 @@ __global__ void __launch_bounds__(256, 4) decode_kernel(EvalParams p) {
     const int64_t total = p.offs[p.nkeys];
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     const int64_t span = (total + 31) & ~(int64_t)31;
-    for (int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; j < span; j += stride) {
+    // software pipeline over the grid-stride loop: the permutation entry is
+    // read two iterations ahead and the record it points to one iteration
+    // ahead, so neither load's latency stalls the decode of the current one
+    int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
+    RecView none;
+    none.rec = make_uint4(0, 0, 0, 0);
+    none.tpc = 0;
+    uint32_t i_next = j < total ? __ldg(p.perm + j) : 0u;
+    uint32_t i_after = j + stride < total ? __ldg(p.perm + j + stride) : 0u;
+    RecView v_next = j < total ? load_record(p, i_next) : none;
+    for (; j < span; j += stride) {
         const bool active = j < total;
-        uint32_t i = 0;
-        RecView v;
-        v.rec = make_uint4(0, 0, 0, 0);
-        v.tpc = 0;
-        if (active) {
-            i = __ldg(p.perm + j);
-            v = load_record(p, i);
-        }
+        const uint32_t i = i_next;
+        const RecView v = v_next;
+        i_next = i_after;
+        v_next = j + stride < total ? load_record(p, i_next) : none;
+        i_after = j + 2 * stride < total ? __ldg(p.perm + j + 2 * stride) : 0u;
         uint4 out = make_uint4(0, 0, 0, 1u << 24);
         if (active) out = decode_one<LIM>(t, v.rec, v.tpc, p, i, lim);
         if (active) {
