@@ -82,7 +82,7 @@ class Clocks:
         try:
             self.f = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(index), f"--query-gpu={q}",
-                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
                                          stdout=self.f, stderr=subprocess.DEVNULL)
         except (OSError, FileNotFoundError):
             self.proc = None
@@ -367,7 +367,7 @@ def run_ours(args, rank, world, local_rank):
                                     frontier_cap=args.frontier_cap, schedule=1)
     P.poseidon_search(prob_e)
     e_ms, e_ev, e_ok = [], 0, True
-    for _ in range(max(3, args.steps // 2)):
+    for _ in range(max(3, min(100, args.steps // 2))):
         flush.zero_()
         torch.cuda.synchronize()
         ev0.record()
@@ -386,7 +386,7 @@ def run_ours(args, rank, world, local_rank):
                                         ridge=True)
         P.poseidon_search(prob_r)
         r_ms = []
-        for _ in range(max(3, args.steps // 2)):
+        for _ in range(max(3, min(100, args.steps // 2))):
             flush.zero_()
             torch.cuda.synchronize()
             ev0.record()
@@ -412,7 +412,7 @@ def run_ours(args, rank, world, local_rank):
                                   frontier_cap=args.frontier_cap)
     P.poseidon_search(prob2)
     o_ms, o_ev, o_ok = [], 0, True
-    for _ in range(max(3, args.steps // 2)):
+    for _ in range(max(3, min(100, args.steps // 2))):
         flush.zero_()
         torch.cuda.synchronize()
         ev0.record()
@@ -437,7 +437,7 @@ def run_ours(args, rank, world, local_rank):
                                     frontier_cap=args.frontier_cap, profile=True)
     P.poseidon_search(prob3)
     c3_ms, c3_ok = [], True
-    for _ in range(max(3, args.steps // 2)):
+    for _ in range(max(3, min(100, args.steps // 2))):
         flush.zero_()
         torch.cuda.synchronize()
         ev0.record()
@@ -507,7 +507,8 @@ def run_ours(args, rank, world, local_rank):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=10)
+    # 1500 config-4 searches (~1 s) so that the clock sampler sees the timed region
+    ap.add_argument("--steps", type=int, default=1500)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
