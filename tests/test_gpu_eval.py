@@ -198,3 +198,23 @@ def test_int32_probe_runs_near_the_lane_count(P):
     rate = ops / (ms / 1e3)
     assert ops == props.multi_processor_count * 8 * 256 * 4096 * 8 * 6
     assert 0.2 * nominal < rate < 1.5 * nominal, rate / nominal
+
+
+@pytest.mark.parametrize("schedule", [0, 1])
+def test_memory_check_at_the_capacity_boundary(P, orc, schedule):
+    """Unit memory rows (mem_w = 1, mem_a = 1 per layer) make a stage's need
+    l + W*l exactly, so small integer capacities put many stages exactly on,
+    one above and one below the limit: the byte table of the decode pass
+    must agree with the oracle's direct check (need <= cap) everywhere."""
+    w = gen.config5_tables()
+    K = w.n_types * w.n_tp
+    w.mem_w = np.ones((K, w.L), np.int64)
+    w.mem_a = np.ones((K, w.L), np.int64)
+    w.cap = np.array([90, 150], np.int64)[:K]
+    c = gen.random_candidates(60_000, L=w.L, n_types=2, S_range=(2, 16), M_range=(1, 40),
+                              seed=17)
+    h = P.Handle(P.Tables.from_workload(w), schedule)
+    T, F = eval_device(P, h, c)
+    Tr, Fr = orc.eval_batch(orc.OracleTables.from_workload(w, schedule=schedule), c)
+    assert np.array_equal(T, Tr) and np.array_equal(F, Fr)
+    assert 0.05 < (F == 1).mean() < 0.95
