@@ -684,13 +684,17 @@ __device__ __forceinline__ int32_t makespan_eager(const StageW<S> &w, int M) {
 template <int S>
 __device__ __forceinline__ int32_t makespan_program(const StageW<S> &w, const uint64_t *prog,
                                                     int n_levels) {
-    int32_t Fo[S], Fp[S], Bo[S], clk[S];
+    // A stage's last op finished at max(Fo, Bo) (finishes grow along its
+    // chain), so no separate clock is kept.  The ops of one level are
+    // independent (at most one per stage, and an op's inter-stage
+    // predecessor lies on an earlier level), so a level's forwards run
+    // first and its backwards second, each phase skipped when empty.
+    int32_t Fo[S], Fp[S], Bo[S];
 #pragma unroll
     for (int s = 0; s < S; ++s) {
         Fo[s] = 0;
         Fp[s] = 0;
         Bo[s] = 0;
-        clk[s] = 0;
     }
     // the next level's word is loaded one level ahead, so the load latency
     // overlaps the current level's relaxations
@@ -701,19 +705,28 @@ __device__ __forceinline__ int32_t makespan_program(const StageW<S> &w, const ui
         if (l + 1 < n_levels) next = __ldg(prog + l + 1);
         const uint32_t fm = (uint32_t)word & 0xffffu, bm = (uint32_t)(word >> 16) & 0xffffu;
         const uint32_t lm = (uint32_t)(word >> 32) & 0xffffu;
+        if (fm) {
 #pragma unroll
-        for (int s = S - 1; s >= 0; --s) {
-            if ((fm >> s) & 1u) {
-                int32_t in = 0;
-                if (s > 0) in = (((lm >> s) & 1u) ? Fp[s - 1] : Fo[s - 1]) + w.pf[s > 0 ? s - 1 : 0];
-                Fp[s] = Fo[s];
-                Fo[s] = max(clk[s], in) + w.F[s];
-                clk[s] = Fo[s];
-            } else if ((bm >> s) & 1u) {
-                int32_t in = 0;
-                if (s + 1 < S) in = Bo[s + 1 < S ? s + 1 : s] + w.pb[s];
-                Bo[s] = max(clk[s], in) + w.B[s];
-                clk[s] = Bo[s];
+            for (int s = S - 1; s >= 0; --s) {
+                if ((fm >> s) & 1u) {
+                    int32_t start = max(Fo[s], Bo[s]);
+                    if (s > 0)
+                        start = max(start, (((lm >> s) & 1u) ? Fp[s > 0 ? s - 1 : 0]
+                                                             : Fo[s > 0 ? s - 1 : 0]) +
+                                               w.pf[s > 0 ? s - 1 : 0]);
+                    Fp[s] = Fo[s];
+                    Fo[s] = start + w.F[s];
+                }
+            }
+        }
+        if (bm) {
+#pragma unroll
+            for (int s = S - 1; s >= 0; --s) {
+                if ((bm >> s) & 1u) {
+                    int32_t start = max(Fo[s], Bo[s]);
+                    if (s + 1 < S) start = max(start, Bo[s + 1 < S ? s + 1 : s] + w.pb[s]);
+                    Bo[s] = start + w.B[s];
+                }
             }
         }
     }
