@@ -130,7 +130,7 @@ def oracle_sample_rate(seconds: float, seed: int = 0):
     return n / dt, n, dt
 
 
-def eval_throughput(P, torch, n, reps, peak_alu, schedule=0):
+def eval_throughput(P, torch, n, reps, peak_alu, schedule=0, space=None):
     """poseidon_eval_batch on n config-5 candidates (L=64, S ~ U{2..16},
     M ~ U{8..128}, 2 device types), device-resident, timed with CUDA events
     on the launching stream; inputs (16 B x n) exceed L2 for n >= 1e7.
@@ -138,8 +138,11 @@ def eval_throughput(P, torch, n, reps, peak_alu, schedule=0):
     sweep on the same tables: N ~ U{1..8} devices, V ~ U{2..16//N} chunks,
     M ~ U{8..128} rounded down to a multiple of N; S counts the N*V virtual
     stages below."""
-    w = gen.config5_tables()
-    if schedule == 2:
+    w = gen.config5_tables() if space is None else space
+    if space is not None:
+        c = gen.search_space_sample(space, n, seed=0)
+        S = c["S"].astype(np.int64)
+    elif schedule == 2:
         c = gen.interleaved_candidates(n, L=w.L, seed=0)
         S = c["S"].astype(np.int64) * c["V"].astype(np.int64)
     else:
@@ -170,7 +173,9 @@ def eval_throughput(P, torch, n, reps, peak_alu, schedule=0):
     sec = ms / 1e3 / reps
     h.close()
     ach = ops / sec / 1e12
-    return {"workload": ("interleaved sweep: L=64, N~U{1..8}, V~U{2..16/N}, M~U{8..128} "
+    return {"workload": (f"{space.name}: uniform sample of the whole search space "
+                         "(no memory cut, no prune)" if space is not None else
+                         "interleaved sweep: L=64, N~U{1..8}, V~U{2..16/N}, M~U{8..128} "
                          "(multiple of N), 2 device types" if schedule == 2 else
                          "config 5: L=64, S~U{2..16}, M~U{8..128}, 2 device types"),
             "schedule": ["1F1B", "Eager 1F1B", "Interleaved 1F1B"][schedule],
@@ -360,6 +365,10 @@ def run_ours(args, rank, world, local_rank):
                    for n in args.eval_sizes[:1]]
     evals_il = [eval_throughput(P, torch, int(n), 5, peak_alu, schedule=2)
                 for n in args.eval_sizes[:1]]
+    # config 3 unpruned: a uniform sample of its 4.4e9-plan space through the
+    # evaluator (S = 8, M = 64: 1024 relaxations per plan)
+    evals_c3 = [eval_throughput(P, torch, int(n), 5, peak_alu, space=gen.config3())
+                for n in args.eval_sizes[:1]]
     # the same search under Eager 1F1B (App. B schedule), for comparison
     ref_e = _json.load(open(os.path.join(ROOT, "tests", "golden", "search_plans.json")))
     ref_e = ref_e.get("config4_eager", {}).get("plan", {})
@@ -488,6 +497,7 @@ def run_ours(args, rank, world, local_rank):
         "eval_sweep": sweep,
         "eval_throughput_eager": evals_eager,
         "eval_throughput_interleaved": evals_il,
+        "eval_throughput_config3": evals_c3,
         "eager_search": eager_search,
         "config3_exhaustive": exhaustive3,
         "ridge_search": ridge_lines,

@@ -286,6 +286,26 @@ def per_stage_tp_candidates(n: int, L: int, n_types: int, n_tp: int, seed: int =
     return out
 
 
+def search_space_sample(w: Workload, n: int, seed: int = 0) -> np.ndarray:
+    """n plans drawn uniformly from a search workload's whole space (every
+    slice and composition, memory-feasible or not), in this order: the
+    M index, the TP index, the placement rank, then the composition rank
+    from a 64-bit draw."""
+    rng = np.random.default_rng(seed)
+    places = np.array([type_code_of(p) for p in place_list(w)], dtype=np.uint32)
+    mi = rng.integers(0, len(w.M_list), size=n)
+    ti = rng.integers(0, w.n_tp, size=n)
+    pi = rng.integers(0, len(places), size=n)
+    u = rng.integers(0, np.iinfo(np.uint64).max, size=n, dtype=np.uint64, endpoint=True)
+    out = np.zeros(n, dtype=CANDIDATE_DTYPE)
+    out["map_rank"] = u % np.uint64(math.comb(w.L - 1, w.S - 1))
+    out["type_code"] = places[pi]
+    out["S"] = w.S
+    out["M"] = np.asarray(w.M_list, np.uint8)[mi]
+    out["tp_idx"] = ti.astype(np.uint8)
+    return out
+
+
 def interleaved_candidates(n: int, L: int = 64, n_types: int = 2, seed: int = 0,
                            m_lo: int = 8, m_hi: int = 128) -> np.ndarray:
     """Interleaved 1F1B batch (Sec. 4.1.4): per record, in this draw order,

@@ -218,3 +218,12 @@ def test_memory_check_at_the_capacity_boundary(P, orc, schedule):
     Tr, Fr = orc.eval_batch(orc.OracleTables.from_workload(w, schedule=schedule), c)
     assert np.array_equal(T, Tr) and np.array_equal(F, Fr)
     assert 0.05 < (F == 1).mean() < 0.95
+
+
+def test_config3_whole_space_sample(P, orc):
+    """Plans drawn uniformly from config 3's whole space (the bench's
+    config-3 evaluator line), memory-feasible or not."""
+    w = gen.config3()
+    c = gen.search_space_sample(w, 50_000, seed=7)
+    T, F, Tr, Fr = _both(P, orc, w, c)
+    assert np.array_equal(T, Tr) and np.array_equal(F, Fr)
