@@ -1603,9 +1603,14 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
                 ep.nb = (int)b.nb;
                 ep.vb_smem = p->prune == 2 && !last && b.nb <= kVbSlotsSmem;
                 const int smem_l = ep.lay.bytes + (ep.vb_smem ? (int)b.nb * 128 * 8 : 0);
+                // depth 0: the batch's nb roots, one warp each (the kernel
+                // takes the warp-per-parent mapping when the grid has a warp
+                // per parent); deeper frontiers are sized on the device
                 const int grid = x == 0 ? (int)std::max<long long>(
-                                              1, std::min<long long>(((long long)b.nb + 255) / 256,
-                                                                     s.grid_level))
+                                              1, std::min<long long>(
+                                                     ((long long)b.nb + kThreads / 32 - 1) /
+                                                         (kThreads / 32),
+                                                     s.grid_level))
                                         : s.grid_level;
                 s.launches++;
                 if ((st = launch_level(last, x, ep, grid, smem_l, s.stream)) != POS_OK)
