@@ -82,6 +82,43 @@ __device__ __forceinline__ void il_makespan_ops(IlState<N, V> &s, int q) {
     il_run<N, V, 2>(s, std::make_integer_sequence<int, O::nE>{});
 }
 
+// Forwards of chunk c among a device's first k forwards: forward f runs
+// chunk (f mod NV) / N, so every NV consecutive forwards hold N of each
+// chunk.
+__host__ __device__ constexpr int il_fwd_count(int N, int V, int k, int c) {
+    const int part = k % (N * V) - c * N;
+    return (k / (N * V)) * N + (part < 0 ? 0 : part > N ? N : part);
+}
+
+// Largest footprint after a forward over the steady pairs (F_{W+i}, B_i),
+// i < STEPS, from `held` after the W warm-up forwards.  The forward's chunk
+// changes when (W + i) mod N = 0 and the backward's when i mod N = 0; in a
+// run between two changes both are fixed, the footprint after the run's
+// k-th forward is h0 + k (aF - aB), and its largest value is at the run's
+// first or last forward.
+template <int N, int V, int W, int STEPS>
+__device__ __forceinline__ int64_t il_steady_peak(const int64_t (&act)[V], int64_t held) {
+    constexpr int NV = N * V;
+    int64_t peak = 0, h0 = 0;
+    int first = 0;
+#pragma unroll
+    for (int i = 0; i < STEPS; ++i) {
+        const int64_t aF = act[((W + i) % NV) / N], aB = act[V - 1 - (i % NV) / N];
+        const bool start = i == 0 || (W + i) % N == 0 || i % N == 0;
+        const bool end = i == STEPS - 1 || (W + i + 1) % N == 0 || (i + 1) % N == 0;
+        if (start) {
+            h0 = held + aF;
+            first = i;
+        }
+        if (end) {
+            const int64_t span = (int64_t)(i - first) * (aF - aB);
+            peak = max(peak, max(h0, h0 + span));
+            held = h0 + span - aB;
+        }
+    }
+    return peak;
+}
+
 // Does device d (class k) fit?  act[c]: activations of its chunk c per
 // micro-batch; resident: its weights and optimizer state over all chunks.
 template <int N, int V, int d>
@@ -98,20 +135,12 @@ __device__ __forceinline__ bool il_device_fits(const int64_t (&act)[V], int64_t 
         constexpr int w = 2 * (N - d - 1) + (V - 1) * N;  // warm-up forwards (< VM for q >= 2)
         int64_t held = 0;
 #pragma unroll
-        for (int k = 0; k < w; ++k) held += act[(k % NV) / N];
+        for (int c = 0; c < V; ++c) held += (int64_t)il_fwd_count(N, V, w, c) * act[c];
         // steady pairs (F_{w+i}, B_i): all of one period for q >= 3, the
         // 2NV - w pairs there are for q = 2 when fewer
         constexpr int steady2 = 2 * NV - w;
-        const int steps = (q >= 3 || steady2 >= NV) ? NV : steady2;
-        peak = 0;
-#pragma unroll
-        for (int i = 0; i < NV; ++i) {
-            if (i < steps) {
-                held += act[((w + i) % NV) / N];
-                peak = max(peak, held);
-                held -= act[V - 1 - (i % NV) / N];
-            }
-        }
+        if (q >= 3 || steady2 >= NV) peak = il_steady_peak<N, V, w, NV>(act, held);
+        else peak = il_steady_peak<N, V, w, (steady2 < NV ? steady2 : NV)>(act, held);
     }
     return peak + resident <= cap;
 }

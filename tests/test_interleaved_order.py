@@ -97,6 +97,47 @@ def _peak_rule(N, V, q, act):
     return peaks
 
 
+def _peak_runs(N, V, q, act):
+    """The kernel's computation of the same peaks: the warm-up sum from
+    per-chunk forward counts, then the steady pairs in runs of a fixed
+    (forward chunk, backward chunk), each run's extreme at one of its ends."""
+    NV = N * V
+    peaks = []
+    for d in range(N):
+        a = [act[c * N + d] for c in range(V)]
+        if q == 1:
+            peaks.append(N * sum(a))
+            continue
+        w = 2 * (N - d - 1) + (V - 1) * N
+
+        def count(k, c):
+            part = k % NV - c * N
+            return (k // NV) * N + min(max(part, 0), N)
+        held = sum(count(w, c) * a[c] for c in range(V))
+        steps = NV if (q >= 3 or 2 * NV - w >= NV) else 2 * NV - w
+        peak, h0, first = 0, 0, 0
+        for i in range(steps):
+            aF, aB = a[((w + i) % NV) // N], a[V - 1 - (i % NV) // N]
+            if i == 0 or (w + i) % N == 0 or i % N == 0:
+                h0, first = held + aF, i
+            if i == steps - 1 or (w + i + 1) % N == 0 or (i + 1) % N == 0:
+                span = (i - first) * (aF - aB)
+                peak = max(peak, h0, h0 + span)
+                held = h0 + span - aB
+        peaks.append(peak)
+    return peaks
+
+
+@pytest.mark.parametrize("NV", sorted(ORDERS))
+def test_peak_runs_equal_the_step_rule(NV):
+    N, V = NV
+    rng = np.random.default_rng(7 * N + V)
+    for q in (1, 2, 3, 4):
+        for _ in range(20):
+            act = [int(x) for x in rng.integers(0, 10 ** 9, N * V)]
+            assert _peak_runs(N, V, q, act) == _peak_rule(N, V, q, act)
+
+
 @pytest.mark.parametrize("NV", sorted(ORDERS))
 def test_emulated_kernel_matches_oracle(orc, NV):
     N, V = NV
