@@ -19,6 +19,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -37,7 +38,7 @@ SM_LANES = 128  # INT32 lanes per SM (4 partitions x 32)
 ENTRY_BYTES = 32  # one frontier entry / one complete plan
 # DRAM bytes per evaluated plan of leaf_kernel, from one ncu capture of
 # dram__bytes_read.sum + dram__bytes_write.sum over a config-4 search's leaf
-# launches (profiles/leaf_kernel_config4.md), valid while the kernel's
+# launches (the leaf kernel's ncu summary), valid while the kernel's
 # sources hash to LEAF_SOURCES_SHA256 (else the traffic is reported as null)
 LEAF_DRAM_BYTES_PER_PLAN = 59694592 / 1925970
 LEAF_SOURCES = ("paper_2609_06086_gb300/csrc/search_kernels.cuh",
@@ -74,8 +75,7 @@ class Clocks:
 
     def __init__(self, index):
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
-        os.makedirs(os.path.dirname(self.path), exist_ok=True)
+        self.path = os.path.join(tempfile.gettempdir(), f"poseidon_clocks_{os.getpid()}.csv")
         q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
@@ -299,8 +299,7 @@ def run_ours(args, rank, world, local_rank):
     # Per kernel (device time from CUDA events around every launch on the
     # library's stream, profiled steps): the leaf kernel (makespans of the
     # complete plans) and the level kernel of each parent depth x (x = S-2
-    # completes the last two stages).  Algorithmic work (roofline
-    # section):
+    # completes the last two stages).  Algorithmic work per unit:
     #  leaf    : int32 ops, 3 per DAG node relaxation + 9 per stage
     #  level x : bytes, a 32-byte frontier entry read per parent and a 32-byte
     #            child (or complete plan) written per child
@@ -343,7 +342,7 @@ def run_ours(args, rank, world, local_rank):
             "achieved": per_kind[dom]["achieved"], "frac": per_kind[dom]["frac"],
             "work_per_launch": work[dom] / max(1, launches[dom]), "traffic": traffic,
             "traffic_note": ("DRAM bytes per launch: ncu dram__bytes_read.sum + "
-                             "dram__bytes_write.sum per plan (profiles/leaf_kernel_config4.md) "
+                             "dram__bytes_write.sum per plan (one ncu capture of a config-4 search) "
                              "x plans per launch" if traffic is not None else None),
             "peak_note": (f"{n_sm} SMs x {SM_LANES} int32 lanes x {mhz:.0f} MHz (median SM "
                           "clock under load)" if b == "alu" else hbm_src)}
