@@ -110,25 +110,37 @@ __global__ void sort_hist_kernel(EvalParams p, int64_t n, uint32_t *hist, uint16
 
 // exclusive prefix sum of the histogram (one block); cursor = offs copy
 template <int NK>
-__global__ void sort_scan_kernel(const uint32_t *hist, uint32_t *offs, uint32_t *cursor) {
-    __shared__ uint32_t part[1024];
+// (1024 threads: each sums a run of keys; the run totals are scanned within
+// each warp by shuffles, then across the 32 warp totals by the first warp)
+__global__ void __launch_bounds__(1024) sort_scan_kernel(const uint32_t *hist, uint32_t *offs,
+                                                        uint32_t *cursor) {
+    __shared__ uint32_t warp_total[32];
     const int per = (NK + blockDim.x - 1) / blockDim.x;
     const int lo = threadIdx.x * per, hi = min(NK, lo + per);
+    const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
     uint32_t sum = 0;
     for (int i = lo; i < hi; ++i) sum += hist[i];
-    part[threadIdx.x] = sum;
+    uint32_t incl = sum;  // inclusive scan over the warp's lanes
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t v = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += v;
+    }
+    if (lane == 31) warp_total[wid] = incl;
     __syncthreads();
-    if (threadIdx.x == 0) {
-        uint32_t run = 0;
-        for (int i = 0; i < (int)blockDim.x; ++i) {
-            const uint32_t v = part[i];
-            part[i] = run;
-            run += v;
+    if (wid == 0) {
+        const uint32_t t = lane < (int)(blockDim.x >> 5) ? warp_total[lane] : 0u;
+        uint32_t ti = t;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const uint32_t v = __shfl_up_sync(0xffffffffu, ti, o);
+            if (lane >= o) ti += v;
         }
-        offs[NK] = run;
+        warp_total[lane] = ti - t;  // exclusive prefix of the warp totals
+        if (lane == 31) offs[NK] = ti;
     }
     __syncthreads();
-    uint32_t run = part[threadIdx.x];
+    uint32_t run = warp_total[wid] + incl - sum;
     for (int i = lo; i < hi; ++i) {
         offs[i] = run;
         cursor[i] = run;
