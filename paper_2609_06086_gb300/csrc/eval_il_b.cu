@@ -5,7 +5,7 @@
 namespace pos {
 
 pos_status eval_il_12_22(const EvalParams &p, cudaStream_t s) {
-    return launch_il_range<12, 22, 5>(p, s);
+    return launch_il_range<12, 22, 4>(p, s);
 }
 
 }  // namespace pos

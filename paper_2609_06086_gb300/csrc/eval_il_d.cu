@@ -5,7 +5,7 @@
 namespace pos {
 
 pos_status eval_il_30_31(const EvalParams &p, cudaStream_t s) {
-    return launch_il_range<30, 31, 4>(p, s);
+    return launch_il_range<30, 31, 3>(p, s);
 }
 
 }  // namespace pos
