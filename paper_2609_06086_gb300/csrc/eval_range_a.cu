@@ -4,11 +4,11 @@
 namespace pos {
 
 pos_status eval_fast_1_4(const EvalParams &p, cudaStream_t s) {
-    return launch_eval_range<1, 4, kPathFast, 8>(p, s);
+    return launch_eval_range<1, 4, kPathFast, 6>(p, s);
 }
 
 pos_status eval_fast_5_8(const EvalParams &p, cudaStream_t s) {
-    return launch_eval_range<5, 8, kPathFast, 5>(p, s);
+    return launch_eval_range<5, 8, kPathFast, 4>(p, s);
 }
 
 }  // namespace pos

@@ -9,7 +9,7 @@ pos_status eval_eager_1_6(const EvalParams &p, cudaStream_t s) {
 }
 
 pos_status eval_eager_7_10(const EvalParams &p, cudaStream_t s) {
-    return launch_eval_range<7, 10, kPathEager, 4>(p, s);
+    return launch_eval_range<7, 10, kPathEager, 3>(p, s);
 }
 
 }  // namespace pos

@@ -4,7 +4,7 @@
 namespace pos {
 
 pos_status eval_generic_9_12(const EvalParams &p, cudaStream_t s) {
-    return launch_eval_range<9, 12, kPathGeneric, 4>(p, s);
+    return launch_eval_range<9, 12, kPathGeneric, 3>(p, s);
 }
 
 }  // namespace pos
