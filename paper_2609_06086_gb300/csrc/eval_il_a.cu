@@ -5,7 +5,7 @@
 namespace pos {
 
 pos_status eval_il_0_11(const EvalParams &p, cudaStream_t s) {
-    return launch_il_range<0, 11, 6>(p, s);
+    return launch_il_range<0, 11, 4>(p, s);
 }
 
 }  // namespace pos

@@ -4,7 +4,7 @@
 namespace pos {
 
 pos_status eval_generic_13_14(const EvalParams &p, cudaStream_t s) {
-    return launch_eval_range<13, 14, kPathGeneric, 4>(p, s);
+    return launch_eval_range<13, 14, kPathGeneric, 3>(p, s);
 }
 
 }  // namespace pos

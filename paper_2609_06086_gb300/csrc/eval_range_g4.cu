@@ -4,7 +4,7 @@
 namespace pos {
 
 pos_status eval_generic_15_15(const EvalParams &p, cudaStream_t s) {
-    return launch_eval_range<15, 15, kPathGeneric, 3>(p, s);
+    return launch_eval_range<15, 15, kPathGeneric, 2>(p, s);
 }
 
 }  // namespace pos
