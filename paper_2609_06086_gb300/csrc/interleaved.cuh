@@ -17,8 +17,9 @@
 //     each op adds the chunk's activations on a forward and releases them on
 //     a backward; it is largest after a forward, and in the steady phase its
 //     values after the forwards repeat with period NV (every NV consecutive
-//     forwards, and backwards, cover each chunk N times), so the warm-up and
-//     at most one period are scanned.
+//     forwards, and backwards, cover each chunk N times), so the warm-up
+//     footprint (from per-chunk forward counts) and at most one period,
+//     scanned in runs of fixed chunks, decide it.
 #pragma once
 #include "eval_kernel.cuh"
 #include "interleaved_order.h"
