@@ -79,6 +79,7 @@ class Clocks:
         q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        self.index, self.query = index, q
         try:
             self.f = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(index), f"--query-gpu={q}",
@@ -93,6 +94,16 @@ class Clocks:
         self.proc.terminate()
         self.proc.wait()
         self.f.close()
+        if not any(len(line.split(",")) >= 9 for line in open(self.path)):
+            # a timed region shorter than the sampling period: one reading
+            # taken as it ends
+            try:
+                with open(self.path, "a") as f:
+                    subprocess.run(["nvidia-smi", "-i", str(self.index),
+                                    f"--query-gpu={self.query}", "--format=csv,noheader,nounits"],
+                                   stdout=f, stderr=subprocess.DEVNULL, timeout=10)
+            except (OSError, subprocess.SubprocessError):
+                pass
         sm, mx, reasons = [], 0.0, set()
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
         for line in open(self.path):
