@@ -98,6 +98,9 @@ def lib():
         L.orc_eval_interleaved.argtypes = [C.POINTER(Tables), C.c_int, C.c_int, C.c_int,
                                            C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                            C.c_void_p]
+        L.orc_search_interleaved.restype = C.c_int
+        L.orc_search_interleaved.argtypes = [C.c_void_p, C.c_int, C.c_int, C.c_void_p,
+                                             C.c_void_p]
         L.orc_eval_batch_ex.restype = C.c_int
         L.orc_eval_batch_ex.argtypes = [C.POINTER(Tables), C.c_void_p, C.c_int64, C.c_void_p,
                                         C.c_void_p]
@@ -264,3 +267,28 @@ def search(w, prune=True, warmup=0, seed=0, tab: OracleTables | None = None,
                layers=list(plan.layers)[:S])
     stats = {n: getattr(st, n) for n, _ in Stats._fields_}
     return out, stats
+
+
+def search_interleaved(w, V, prune=True, tab: OracleTables | None = None):
+    """Search over Interleaved 1F1B plans with V chunks per device (w.S
+    devices).  Returns (plan dict, stats dict); layers has N*V entries."""
+    tab = tab or OracleTables.from_workload(w, SCHED_INTERLEAVED_1F1B)
+    M_list = _i32(w.M_list)
+    dp = _i32(w.dp_list)
+    tc = _i32(w.type_counts if w.type_counts else [0] * w.n_types)
+    p = Problem(tab.c, w.S, len(M_list), M_list.ctypes.data, dp.ctypes.data, w.placement,
+                tc.ctypes.data, 0)
+    plan, st = Plan(), Stats()
+    rc = lib().orc_search_interleaved(C.byref(p), int(V), int(prune), C.byref(plan),
+                                      C.byref(st))
+    if rc == -2:
+        raise OverflowError("overflow guard")
+    if rc:
+        raise RuntimeError("oracle interleaved search failed")
+    J = w.S * V
+    out = dict(found=bool(plan.found), m_idx=plan.m_idx, tp_idx=plan.tp_idx, M=plan.M, D=plan.D,
+               T=plan.T, place_rank=plan.place_rank, map_rank=plan.map_rank,
+               global_index=plan.global_index, types=list(plan.types)[:w.S],
+               layers=list(plan.layers)[:J])
+    return out, {n: getattr(st, n) for n, _ in Stats._fields_}
+

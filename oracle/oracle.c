@@ -1033,3 +1033,155 @@ int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_p
     dag_free(&cx.g);
     return cx.err ? -1 : 0;
 }
+
+/* ------------------------------------------------------------------ */
+/* Search over Interleaved 1F1B plans (Sec. 4.1.4 model, Sec. 4.2.3    */
+/* search order).                                                      */
+/* ------------------------------------------------------------------ */
+/* Slices (M, TP index, placement of types over the N = p->S devices) in
+ * the order of orc_search; per slice, every composition of the L layers
+ * into the J = N*V virtual stages in lexicographic order, evaluated by
+ * orc_eval_interleaved.  M values that are not multiples of N are skipped.
+ * Cuts (both only remove plans that cannot be feasible or better):
+ *   memory: the weights of a device's chunks placed so far already exceed
+ *     its capacity (activations only add to them);
+ *   bound (prune != 0): for a device d, the chain of its 2VM ops runs one
+ *     op at a time and R_d follows its last op, so
+ *       T >= M * sum over its chunks of (F + B) + its all-reduce time;
+ *     summed over the chunks placed so far this is a lower bound of every
+ *     completion; a prefix whose largest such bound is worse than the
+ *     incumbent (objective T/(D*M), strictly) is cut. */
+typedef struct {
+    const orc_problem *p;
+    int N, V, J, L, M, D, m_idx, tp_idx, prune;
+    uint64_t place_rank, n_place, n_map;
+    int32_t cls[ORC_MAX_S], types[ORC_MAX_S], layers[ORC_MAX_S];
+    int64_t wsum[ORC_MAX_S], work[ORC_MAX_S];
+    orc_plan *best;
+    orc_stats *st;
+    int err;
+} il_ctx;
+
+static void il_leaf(il_ctx *cx) {
+    int32_t T, F;
+    if (orc_eval_interleaved(&cx->p->tab, cx->N, cx->V, cx->M, cx->cls, cx->layers, &T, &F,
+                             NULL)) {
+        cx->err = 1;
+        return;
+    }
+    cx->st->leaves_evaluated++;
+    if (!F) return;
+    const int n_tp = cx->p->tab.n_tp;
+    const uint64_t map_rank = orc_rank(cx->L, cx->J, cx->layers);
+    const uint64_t idx =
+        (((uint64_t)cx->m_idx * n_tp + cx->tp_idx) * cx->n_place + cx->place_rank) * cx->n_map +
+        map_rank;
+    if (!better(T, cx->D, cx->M, idx, cx->best)) return;
+    orc_plan *b = cx->best;
+    b->found = 1;
+    b->m_idx = cx->m_idx;
+    b->tp_idx = cx->tp_idx;
+    b->M = cx->M;
+    b->D = cx->D;
+    b->T = T;
+    b->place_rank = cx->place_rank;
+    b->map_rank = map_rank;
+    b->global_index = idx;
+    for (int s = 0; s < ORC_MAX_S; ++s) {
+        b->types[s] = s < cx->N ? cx->types[s] : 0;
+        b->layers[s] = s < cx->J ? cx->layers[s] : 0;
+    }
+}
+
+static void il_dfs(il_ctx *cx, int j, int used) {
+    const orc_tables *t = &cx->p->tab;
+    const int L = cx->L, d = j % cx->N, k = cx->cls[d];
+    const int hi = L - used - (cx->J - j - 1), lo = j == cx->J - 1 ? hi : 1;
+    int64_t w = 0, work = 0;
+    for (int l = 1; l <= hi && !cx->err; ++l) {
+        const int at = used + l - 1;  /* the layer this step adds */
+        w += t->mem_w[(int64_t)k * L + at];
+        work += (int64_t)cx->M * (t->fwd[(int64_t)k * L + at] + t->bwd[(int64_t)k * L + at]) +
+                t->dsync[(int64_t)k * L + at];
+        if (l < lo) continue;
+        if (cx->wsum[d] + w > t->cap[k]) {  /* more layers only add weights */
+            cx->st->prefixes_memory++;
+            break;
+        }
+        cx->wsum[d] += w;
+        cx->work[d] += work;
+        cx->layers[j] = l;
+        int cut = 0;
+        if (cx->prune && cx->best->found) {
+            int64_t lb = 0;
+            for (int e = 0; e < cx->N; ++e)
+                if (cx->work[e] > lb) lb = cx->work[e];
+            /* lb / (D M) > T_min / (D_min M_min) */
+            cut = lb * (int64_t)cx->best->D * cx->best->M >
+                  (int64_t)cx->best->T * cx->D * cx->M;
+        }
+        if (cut) {
+            cx->st->prefixes_pruned++;
+        } else if (j == cx->J - 1) {
+            il_leaf(cx);
+        } else {
+            il_dfs(cx, j + 1, used + l);
+        }
+        cx->wsum[d] -= w;
+        cx->work[d] -= work;
+        if (cut) break;  /* the bound only grows with the stage's layers */
+    }
+}
+
+int orc_search_interleaved(const orc_problem *p, int V, int prune, orc_plan *plan,
+                           orc_stats *stats) {
+    const int N = p->S, L = p->tab.L, J = N * V;
+    if (N < 1 || V < 2 || J > ORC_MAX_S || J > L || L > 127 || p->n_M < 1 ||
+        p->tab.n_types < 1 || p->tab.n_types > 4 || p->tab.n_tp < 1)
+        return -1;
+    for (int i = 0; i < p->n_M; ++i)
+        if (p->M_list[i] < 1 || p->M_list[i] > 255) return -1;
+    for (int i = 0; i < p->tab.n_tp; ++i)
+        if (p->dp_list[i] < 1) return -1;
+    for (int i = 0; i < p->n_M; ++i)
+        if (p->M_list[i] % N == 0 && overflow_bound(&p->tab, J, p->M_list[i]) >= ((int64_t)1 << 31))
+            return -2;
+    memset(plan, 0, sizeof(*plan));
+    memset(stats, 0, sizeof(*stats));
+    il_ctx cx;
+    memset(&cx, 0, sizeof(cx));
+    cx.p = p;
+    cx.N = N;
+    cx.V = V;
+    cx.J = J;
+    cx.L = L;
+    cx.prune = prune;
+    cx.best = plan;
+    cx.st = stats;
+    cx.n_map = n_comp(L, J);
+    int32_t seq[ORC_MAX_S];
+    cx.n_place = 0;
+    for (int f = 1; next_placement(p, seq, f); f = 0) cx.n_place++;
+    for (int mi = 0; mi < p->n_M && !cx.err; ++mi) {
+        if (p->M_list[mi] % N != 0) continue;
+        for (int tp = 0; tp < p->tab.n_tp && !cx.err; ++tp) {
+            uint64_t pr = 0;
+            for (int f = 1; next_placement(p, seq, f) && !cx.err; f = 0, ++pr) {
+                cx.m_idx = mi;
+                cx.tp_idx = tp;
+                cx.M = p->M_list[mi];
+                cx.D = p->dp_list[tp];
+                cx.place_rank = pr;
+                for (int s = 0; s < N; ++s) {
+                    cx.types[s] = seq[s];
+                    cx.cls[s] = seq[s] * p->tab.n_tp + tp;
+                    cx.wsum[s] = 0;
+                    cx.work[s] = 0;
+                }
+                il_dfs(&cx, 0, 0);
+            }
+        }
+    }
+    return cx.err ? -1 : 0;
+}
+

@@ -151,6 +151,17 @@ int orc_eval_batch_ex(const orc_tables *t, const orc_candidate_ex *c, int64_t n,
 int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_plan *plan,
                orc_stats *stats);
 
+/* Search over Interleaved 1F1B plans with V chunks per device: the slices
+ * of orc_search over the N = p->S devices (M values that are not multiples
+ * of N skipped), every composition of L into the N*V virtual stages,
+ * evaluated by orc_eval_interleaved; objective, global index (with
+ * C(L-1, N*V-1) compositions per slice) and ties as in orc_search.  Cuts:
+ * memory (a device's placed chunk weights exceed its capacity) and, when
+ * prune != 0, the per-device serial-work bound (see oracle.c).  Returns 0,
+ * -1 on invalid input, -2 when the overflow guard trips. */
+int orc_search_interleaved(const orc_problem *p, int V, int prune, orc_plan *plan,
+                           orc_stats *stats);
+
 #ifdef __cplusplus
 }
 #endif
