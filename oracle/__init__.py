@@ -98,6 +98,10 @@ def lib():
         L.orc_eval_interleaved.argtypes = [C.POINTER(Tables), C.c_int, C.c_int, C.c_int,
                                            C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                            C.c_void_p]
+        L.orc_eval_interleaved_detail.restype = C.c_int
+        L.orc_eval_interleaved_detail.argtypes = [C.POINTER(Tables), C.c_int, C.c_int, C.c_int,
+                                                  C.c_void_p, C.c_void_p, C.c_void_p,
+                                                  C.c_void_p, C.c_void_p, C.c_void_p]
         L.orc_search_interleaved.restype = C.c_int
         L.orc_search_interleaved.argtypes = [C.c_void_p, C.c_int, C.c_int, C.c_void_p,
                                              C.c_void_p]
@@ -204,6 +208,24 @@ def evaluate_interleaved(tab: OracleTables, N, V, M, cls, layers, counts=False):
     if counts:
         return T.value, bool(F.value), {n: getattr(dc, n) for n, _ in DagCounts._fields_}
     return T.value, bool(F.value)
+
+
+def interleaved_detail(tab: OracleTables, N, V, M, cls, layers):
+    """Interleaved 1F1B with every compute node's finish time and each
+    device's activation peak: (T, feasible, F finish [NV][M], B finish
+    [NV][M], peak [N])."""
+    J = N * V
+    c, l = _i32(cls, N), _i32(layers, J)
+    T, F = C.c_int32(), C.c_int32()
+    fin = np.zeros(2 * J * M, np.int32)
+    peak = np.zeros(N, np.int64)
+    rc = lib().orc_eval_interleaved_detail(C.byref(tab.c), N, V, M, c.ctypes.data, l.ctypes.data,
+                                           C.byref(T), C.byref(F), fin.ctypes.data,
+                                           peak.ctypes.data)
+    if rc:
+        raise ValueError("invalid configuration")
+    return (T.value, bool(F.value), fin[:J * M].reshape(J, M), fin[J * M:].reshape(J, M),
+            peak.tolist())
 
 
 def lower_bound_tight(tab: OracleTables, S, M, cls, layers, x):

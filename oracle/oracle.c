@@ -441,9 +441,12 @@ static void interleaved_chain(int N, int V, int M, int d, il_op *ops) {
     }
 }
 
-int orc_eval_interleaved(const orc_tables *t, int N, int V, int M, const int32_t *cls,
-                         const int32_t *layers, int32_t *T, int32_t *feasible,
-                         orc_dag_counts *counts) {
+/* The interleaved DAG of one plan and its longest path; optionally the
+ * finish time of every compute node (finish[j*M + m] for F_{j,m},
+ * finish[J*M + j*M + m] for B_{j,m}) and each device's activation peak. */
+static int il_eval(const orc_tables *t, int N, int V, int M, const int32_t *cls,
+                   const int32_t *layers, int32_t *T, int32_t *feasible, orc_dag_counts *counts,
+                   int32_t *finish, int64_t *peak_out) {
     const int J = N * V, L = t->L, K = t->n_types * t->n_tp;
     if (N < 1 || V < 2 || J > ORC_MAX_S || M < 1 || M % N != 0) return -1;
     int sum = 0;
@@ -537,6 +540,7 @@ int orc_eval_interleaved(const orc_tables *t, int N, int V, int M, const int32_t
         const int lc = ops[2 * V * M - 1].c * N + d;
         add_edge(&g, IL_B(lc, ops[2 * V * M - 1].m), IL_R(d), 0);
         add_edge(&g, IL_R(d), node_E, 0);
+        if (peak_out) peak_out[d] = peak;
         if (peak + wsum[d] > t->cap[cls[d]]) *feasible = 0;
     }
     add_edge(&g, 0, IL_F(0, 0), 0);
@@ -552,6 +556,12 @@ int orc_eval_interleaved(const orc_tables *t, int N, int V, int M, const int32_t
         counts->allreduce_edges = N;
         counts->aux_edges = N + 1;
     }
+    if (!rc && finish)
+        for (int j = 0; j < J; ++j)
+            for (int m = 0; m < M; ++m) {
+                finish[j * M + m] = (int32_t)g.fin[IL_F(j, m)];
+                finish[J * M + j * M + m] = (int32_t)g.fin[IL_B(j, m)];
+            }
 #undef IL_F
 #undef IL_B
 #undef IL_R
@@ -560,6 +570,18 @@ int orc_eval_interleaved(const orc_tables *t, int N, int V, int M, const int32_t
     if (rc || T64 >= ((int64_t)1 << 31)) return -1;
     *T = (int32_t)T64;
     return 0;
+}
+
+int orc_eval_interleaved(const orc_tables *t, int N, int V, int M, const int32_t *cls,
+                         const int32_t *layers, int32_t *T, int32_t *feasible,
+                         orc_dag_counts *counts) {
+    return il_eval(t, N, V, M, cls, layers, T, feasible, counts, NULL, NULL);
+}
+
+int orc_eval_interleaved_detail(const orc_tables *t, int N, int V, int M, const int32_t *cls,
+                                const int32_t *layers, int32_t *T, int32_t *feasible,
+                                int32_t *finish, int64_t *peak) {
+    return il_eval(t, N, V, M, cls, layers, T, feasible, NULL, finish, peak);
 }
 
 int orc_eval_finish(const orc_tables *t, int S, int M, const int32_t *cls, const int32_t *layers,
@@ -793,6 +815,22 @@ typedef struct {
     int err;
 } search_ctx;
 
+/* The searches' cuts assume non-negative weights: a lower bound from a
+ * partial plan (Theorem 1, the per-device serial work) only grows as
+ * stages are added, and so does the memory of a stage as it takes more
+ * layers.  Tables with a negative cost, transfer or memory entry are
+ * rejected by both searches. */
+static int tables_nonnegative(const orc_tables *t) {
+    const int64_t K = (int64_t)t->n_types * t->n_tp, L = t->L;
+    for (int64_t i = 0; i < K * L; ++i)
+        if (t->fwd[i] < 0 || t->bwd[i] < 0 || t->dsync[i] < 0 || t->mem_w[i] < 0 ||
+            t->mem_a[i] < 0)
+            return 0;
+    for (int64_t i = 0; i < K * K; ++i)
+        if (t->p2p_f[i] < 0 || t->p2p_b[i] < 0) return 0;
+    return 1;
+}
+
 /* a strictly better than the incumbent: smaller T/(D*M), then smaller index */
 static int better(int64_t T, int D, int M, uint64_t idx, const orc_plan *b) {
     if (!b->found) return 1;
@@ -955,7 +993,7 @@ int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_p
                orc_stats *stats) {
     int S = p->S, L = p->tab.L;
     if (S < 1 || S > ORC_MAX_S || S > L || L > 127 || p->n_M < 1 || p->tab.n_types < 1 ||
-        p->tab.n_types > 4 || p->tab.n_tp < 1)
+        p->tab.n_types > 4 || p->tab.n_tp < 1 || !tables_nonnegative(&p->tab))
         return -1;
     for (int i = 0; i < p->n_M; ++i)
         if (p->M_list[i] < 1 || p->M_list[i] > 255) return -1;
@@ -1137,7 +1175,8 @@ int orc_search_interleaved(const orc_problem *p, int V, int prune, orc_plan *pla
                            orc_stats *stats) {
     const int N = p->S, L = p->tab.L, J = N * V;
     if (N < 1 || V < 2 || J > ORC_MAX_S || J > L || L > 127 || p->n_M < 1 ||
-        p->tab.n_types < 1 || p->tab.n_types > 4 || p->tab.n_tp < 1)
+        p->tab.n_types < 1 || p->tab.n_types > 4 || p->tab.n_tp < 1 ||
+        !tables_nonnegative(&p->tab))
         return -1;
     for (int i = 0; i < p->n_M; ++i)
         if (p->M_list[i] < 1 || p->M_list[i] > 255) return -1;

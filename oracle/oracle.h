@@ -136,6 +136,13 @@ int64_t orc_lower_bound_tight(const orc_tables *t, int S, int M, const int32_t *
 int orc_eval_interleaved(const orc_tables *t, int N, int V, int M, const int32_t *cls,
                          const int32_t *layers, int32_t *T, int32_t *feasible,
                          orc_dag_counts *counts);
+/* orc_eval_interleaved with the finish time of every compute node
+ * (finish[j*M + m] for F_{j,m}, finish[NV*M + j*M + m] for B_{j,m}; 2NVM
+ * entries) and each device's largest activation footprint along its order
+ * (peak[0..N-1], bytes, without its weights). */
+int orc_eval_interleaved_detail(const orc_tables *t, int N, int V, int M, const int32_t *cls,
+                                const int32_t *layers, int32_t *T, int32_t *feasible,
+                                int32_t *finish, int64_t *peak);
 /* Decode and evaluate n candidate records.  feasible: 1 ok, 0 memory
  * infeasible, 2 invalid record, 3 overflow guard tripped. */
 int orc_eval_batch(const orc_tables *t, const orc_candidate *c, int64_t n, int32_t *T,

@@ -1,8 +1,12 @@
-"""Pins for the oracle's Interleaved 1F1B (Sec. 4.1.4): the node and edge
-counts the paper gives, the V-fold smaller pipeline bubble of uniform
-stages, an event-driven simulator with its own derivation of the device
-order, the serial-work bound, the memory rule on a hand-sized case, and the
-batch decoding of interleaved candidates."""
+"""Pins for the oracle's Interleaved 1F1B (Sec. 4.1.4): a hand-worked
+pipeline (every finish time, the makespan and two activation peaks, one of
+them reached in the steady phase, in tests/golden/interleaved_n2_v2_m4.txt),
+the node and edge counts the paper gives, the V-fold smaller pipeline
+bubble of uniform stages, an event-driven simulator (same device order,
+written in the test from the schedule's description; it checks the DAG
+arithmetic, not the order), the serial-work bound, the memory rule at
+M = N, and the batch decoding of interleaved candidates."""
+import os
 import random
 
 import numpy as np
@@ -46,6 +50,79 @@ def chunk_tables(orc, N, V, F, B, d=None, pf=None, pb=None, act=None, wts=None, 
                             cap=np.full(N, 1 << 40) if cap is None else cap, schedule=IL)
 
 
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "interleaved_n2_v2_m4.txt")
+
+
+def _golden():
+    rows = {}
+    mem = []
+    with open(GOLDEN) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith("#"):
+                continue
+            key, rest = line.split(None, 1)
+            if key == "mem":
+                mem.append([[int(v) for v in part.split()] for part in rest.split("|")])
+            else:
+                rows.setdefault(key, []).append([int(v) for v in rest.split()])
+    return rows, mem
+
+
+def _golden_tables(orc, rows, act=(0, 0, 0, 0), wts=(0, 0, 0, 0), cap=(1 << 40, 1 << 40)):
+    """L = 4 layers, one per virtual stage; device d has class d (two types,
+    one TP index); layer j is read on the class of its device j mod 2."""
+    F, B = rows["F"][0], rows["B"][0]
+    pf, pb = rows["pf"][0], rows["pb"][0]
+    fwd = np.zeros((2, 4), np.int32)
+    bwd = np.zeros((2, 4), np.int32)
+    ma = np.zeros((2, 4), np.int64)
+    mw = np.zeros((2, 4), np.int64)
+    for j in range(4):
+        fwd[j % 2, j], bwd[j % 2, j] = F[j], B[j]
+        ma[j % 2, j], mw[j % 2, j] = act[j], wts[j]
+    ds = np.zeros((2, 4), np.int32)
+    ds[0, 0], ds[0, 2], ds[1, 1] = 1, 2, 4  # device all-reduce 3 and 4
+    # F edge j -> j+1 reads p2p_f[class of j][class of j+1]; B edge j+1 -> j
+    # reads p2p_b[class of j+1][class of j]; both pairs (0,1) and (1,0) occur
+    p2f = np.array([[0, pf[0]], [pf[1], 0]], np.int32)
+    p2b = np.array([[0, pb[1]], [pb[0], 0]], np.int32)
+    assert pf[2] == pf[0] and pb[2] == pb[0]  # the 2->3 crossing reuses the 0->1 entries
+    return orc.OracleTables(L=4, n_types=2, n_tp=1, fwd=fwd, bwd=bwd, dsync=ds, p2p_f=p2f,
+                            p2p_b=p2b, mem_w=mw, mem_a=ma, cap=np.array(cap, np.int64),
+                            schedule=IL)
+
+
+def test_hand_worked_pipeline(orc):
+    """Every finish time and the makespan of the hand-worked N = 2, V = 2,
+    M = 4 pipeline (distinct chunk weights, transfers in both directions,
+    different all-reduce times)."""
+    rows, _ = _golden()
+    tab = _golden_tables(orc, rows)
+    T, fits, f_fin, b_fin, _ = orc.interleaved_detail(tab, 2, 2, 4, [0, 1], [1, 1, 1, 1])
+    assert f_fin.tolist() == rows["Ffin"]
+    assert b_fin.tolist() == rows["Bfin"]
+    assert T == rows["T"][0][0] and fits
+    assert rows["d"][0] == [3, 4]
+
+
+def test_hand_worked_memory_peaks(orc):
+    """The activation peak of each device along its order, and the capacity
+    boundary: a device fits at exactly peak + weights and not one byte
+    below.  The second case peaks in the steady phase (M = 2N)."""
+    rows, mem = _golden()
+    for act, wts, peaks, need in mem:
+        tab = _golden_tables(orc, rows, act=act, wts=wts)
+        _, fits, _, _, peak = orc.interleaved_detail(tab, 2, 2, 4, [0, 1], [1, 1, 1, 1])
+        assert peak == peaks and fits
+        for dev in range(2):
+            for slack, ok in ((0, True), (-1, False)):
+                cap = list(need)
+                cap[dev] += slack
+                tab = _golden_tables(orc, rows, act=act, wts=wts, cap=cap)
+                assert orc.evaluate_interleaved(tab, 2, 2, 4, [0, 1], [1, 1, 1, 1])[1] is ok
+
+
 @pytest.mark.parametrize("N,V,M", [(2, 2, 2), (2, 3, 6), (4, 2, 8), (4, 4, 4), (8, 2, 16)])
 def test_node_and_edge_counts(orc, N, V, M):
     """Sec. 4.1.4: 2VNM compute nodes, 2(NV-1)M inter-stage edges and
@@ -70,11 +147,14 @@ def test_uniform_bubble_shrinks_by_V(orc):
 
 
 def device_order(N, V, M, d):
-    """The interleaved schedule, derived from its description: forward
-    number k of a device is chunk (k mod NV) div N of micro-batch
-    (k div NV) N + k mod N (backwards take the chunks in reverse); the
-    device first runs (N-d-1)*2 + (V-1)*N forwards (all of them if M = N),
-    then a forward and a backward at a time, then the rest."""
+    """The interleaved schedule's device order, written from its
+    description: forward number k of a device is chunk (k mod NV) div N of
+    micro-batch (k div NV) N + k mod N (backwards take the chunks in
+    reverse); the device first runs (N-d-1)*2 + (V-1)*N forwards (all of
+    them if M = N), then a forward and a backward at a time, then the rest.
+    This restates the order the oracle builds, so the simulator below pins
+    the DAG arithmetic (edges, weights, longest path), not the order; the
+    hand-worked pipeline and the uniform-bubble closed form pin the order."""
     total = V * M
     group = N * V
 

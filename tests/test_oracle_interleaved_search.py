@@ -10,6 +10,7 @@ import random
 from fractions import Fraction
 
 import numpy as np
+import pytest
 
 import gen
 
@@ -112,3 +113,19 @@ def test_bound_is_below_every_makespan(orc):
                            int(ds[k, b[j]:b[j + 1]].sum()) for j in range(d, J, N))
                 lb = max(lb, work)
             assert lb <= T, seed
+
+
+@pytest.mark.parametrize("field", ["fwd", "bwd", "dsync", "mem_w", "mem_a", "p2p_f", "p2p_b"])
+def test_negative_tables_are_rejected(orc, field):
+    """The cuts assume non-negative weights (a partial plan's bound and a
+    stage's memory only grow as layers are added), so both searches refuse
+    a table with a negative entry instead of silently cutting plans."""
+    w, V = _problem(random.Random(7), 0)
+    arr = np.array(getattr(w, field))
+    arr.flat[0] = -1
+    setattr(w, field, arr)
+    with pytest.raises(RuntimeError):
+        orc.search_interleaved(w, V, prune=True)
+    w.S = 2 if w.L >= 2 else 1
+    with pytest.raises(RuntimeError):
+        orc.search(w, prune=True)
