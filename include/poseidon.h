@@ -227,6 +227,9 @@ pos_status poseidon_argmin(const int32_t *d_makespan, const uint8_t *d_feasible,
  * loading the library holds until the process exits.  The first call on a
  * device looks up that array's device address (cudaGetSymbolAddress) with
  * the device current; make that first call before any stream capture.
+ * That address is kept for the life of the process: do not use the
+ * library across a cudaDeviceReset (the array may move when the module is
+ * loaded again).
  * All calls on a device share the array and it keeps the last call's
  * contents (every slot a call reads is written earlier in the same call, so
  * nothing needs clearing); calls that overlap on the GPU, e.g. on two
@@ -291,6 +294,12 @@ typedef struct pos_problem {
                                    Theorem 2 guarantees a ridge-like optimum only under
                                    its assumptions: the result may be worse than the
                                    exact optimum (never better); 0: exact search */
+    int32_t V;                  /* POS_SCHED_INTERLEAVED_1F1B: model chunks per device
+                                   (>= 2, S*V <= 16); ignored by the other schedules */
+    int32_t cas_limit;          /* rounds of the incumbent's compare-and-swap loop before
+                                   the search gives up with POS_ETIMEOUT: 0 = default
+                                   (2^20); < 0 = no round, so every update that would
+                                   lower the incumbent gives up (tests the time-out path) */
 } pos_problem;
 
 typedef struct pos_plan {
@@ -344,8 +353,11 @@ typedef struct pos_search_stats {
  * Errors: POS_EINVAL, POS_EOVERFLOW (guard fails for some M), POS_ENOMEM,
  * POS_ECUDA, POS_ETIMEOUT, POS_EINFEASIBLE (no memory-feasible plan; *out
  * has found = 0).
- * Limits: at most 65535 slices with a feasible root per M value; the global
- * index must fit in 64 bits; lcm of all D*M below 2^32.
+ * Limits (checked on the host before the device is touched; POS_EINVAL):
+ * at most 2^22 slices (M values x TP indices x placements) and 2^22
+ * placements; the global index (slices x compositions) must fit in 64
+ * bits; the lcm of all D*M must be below 2^32.  Memory-feasible slices are
+ * enumerated in batches of at most 65535 slices, one after another.
  * Memory: the work buffers (one frontier of frontier_cap 32-byte entries per
  * depth, a leaf buffer of the same length, slice and feasibility tables,
  * and with POS_PRUNE_TIGHT 1 KB of bound tables per stage and slice of a
@@ -355,17 +367,6 @@ typedef struct pos_search_stats {
  * are serialised.
  */
 pos_status poseidon_search(const pos_problem *problem, pos_plan *out, pos_search_stats *stats);
-
-/*
- * Measurement helper (no counterpart in the paper): runs a kernel made of
- * the makespan kernels' relaxation, max(pred + edge, clock) + weight, in
- * independent chains on every SM, twice, and reports the second run:
- * *ops = int32 operations executed (3 per relaxation), *ms = its duration
- * (CUDA events on `stream`).  ops / ms checks the INT32 roofline the
- * ALU-bound kernels are measured against.  Synchronises the stream; uses a
- * 4-byte stream-ordered allocation.  Errors: POS_EINVAL, POS_ECUDA.
- */
-pos_status poseidon_int32_probe(void *stream, int64_t *ops, double *ms);
 
 /* Message describing the last error of the calling thread ("" if none). */
 const char *poseidon_last_error(void);

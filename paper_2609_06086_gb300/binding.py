@@ -28,8 +28,7 @@ MAX_STAGES = 16
 # the exported entry points, as declared in include/poseidon.h
 EXPORTS = ["poseidon_tables_create", "poseidon_tables_destroy", "poseidon_eval_batch",
            "poseidon_eval_batch_ex", "poseidon_eval_batch_host", "poseidon_argmin",
-           "poseidon_argmin_noalloc", "poseidon_search", "poseidon_int32_probe",
-           "poseidon_last_error"]
+           "poseidon_argmin_noalloc", "poseidon_search", "poseidon_last_error"]
 
 
 class pos_tables(C.Structure):
@@ -44,7 +43,8 @@ class pos_problem(C.Structure):
                 ("M_list", C.c_void_p), ("tp_list", C.c_void_p), ("dp_list", C.c_void_p),
                 ("placement", C.c_int32), ("type_counts", C.c_void_p), ("warmup", C.c_int32),
                 ("prune", C.c_int32), ("seed", C.c_uint64), ("schedule", C.c_int32),
-                ("frontier_cap", C.c_int64), ("profile", C.c_int32), ("ridge", C.c_int32)]
+                ("frontier_cap", C.c_int64), ("profile", C.c_int32), ("ridge", C.c_int32),
+                ("V", C.c_int32), ("cas_limit", C.c_int32)]
 
 
 class pos_plan(C.Structure):
@@ -96,7 +96,6 @@ def lib():
         L.poseidon_argmin_noalloc.argtypes = [vp, vp, i64, vp, vp]
         L.poseidon_search.argtypes = [C.POINTER(pos_problem), C.POINTER(pos_plan),
                                       C.POINTER(pos_search_stats)]
-        L.poseidon_int32_probe.argtypes = [vp, C.POINTER(C.c_int64), C.POINTER(C.c_double)]
         L.poseidon_last_error.restype = C.c_char_p
         L.poseidon_last_error.argtypes = []
         for name in EXPORTS[:-1]:
@@ -164,10 +163,26 @@ def poseidon_eval_batch_ex(handle: Handle, d_cands: int, n: int, d_makespan: int
     _check(lib().poseidon_eval_batch_ex(handle.ptr, d_cands, n, d_makespan, d_feasible, stream))
 
 
+_probe = None
+
+
 def poseidon_int32_probe(stream: int = 0):
-    """(int32 ops, ms) of the relaxation microbenchmark (see the header)."""
+    """(int32 ops, ms) of the relaxation microbenchmark in the measurement
+    library libposeidon_probe.so (include/poseidon_probe.h)."""
+    global _probe
+    if _probe is None:
+        path = os.path.join(os.path.dirname(LIB_PATH), "libposeidon_probe.so")
+        if not os.path.exists(path):
+            raise ImportError(f"{path} is missing: run __graft_entry__.build() first")
+        P = C.CDLL(path)
+        P.poseidon_probe_int32.restype = C.c_int
+        P.poseidon_probe_int32.argtypes = [C.c_void_p, C.POINTER(C.c_int64),
+                                           C.POINTER(C.c_double)]
+        _probe = P
     ops, ms = C.c_int64(), C.c_double()
-    _check(lib().poseidon_int32_probe(stream, C.byref(ops), C.byref(ms)))
+    rc = _probe.poseidon_probe_int32(stream, C.byref(ops), C.byref(ms))
+    if rc != 0:
+        raise RuntimeError(f"INT32 probe failed: cudaError {rc}")
     return ops.value, ms.value
 
 
@@ -204,8 +219,11 @@ def _prune_mode(prune):
 
 
 def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0, profile=False,
-                 schedule=POS_SCHED_1F1B, ridge=False):
-    """pos_problem for a gen.Workload search; returns (problem, keep-alive list)."""
+                 schedule=POS_SCHED_1F1B, ridge=False, V=0, cas_limit=0):
+    """pos_problem for a gen.Workload search; returns (problem, keep-alive list).
+    V: model chunks per device under POS_SCHED_INTERLEAVED_1F1B; cas_limit:
+    rounds of the incumbent's compare-and-swap loop (0 = the library's
+    default, < 0 = none)."""
     tab = Tables.from_workload(w)
     keep = [tab]
 
@@ -217,7 +235,7 @@ def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0, profile=Fals
     p = pos_problem(tab.c, w.S, len(w.M_list), arr(w.M_list), arr(w.tp_list), arr(w.dp_list),
                     w.placement, arr(w.type_counts if w.type_counts else [0] * w.n_types),
                     int(warmup), _prune_mode(prune), int(seed), int(schedule), int(frontier_cap),
-                    int(bool(profile)), int(bool(ridge)))
+                    int(bool(profile)), int(bool(ridge)), int(V), int(cas_limit))
     return p, keep
 
 
@@ -227,10 +245,11 @@ def poseidon_search(problem: pos_problem):
     plan, st = pos_plan(), pos_search_stats()
     _check(lib().poseidon_search(C.byref(problem), C.byref(plan), C.byref(st)))
     S = problem.S
+    J = S * problem.V if problem.schedule == POS_SCHED_INTERLEAVED_1F1B else S
     out = dict(found=bool(plan.found), m_idx=plan.m_idx, tp_idx=plan.tp_idx, M=plan.M,
                tp=plan.tp, D=plan.D, T=plan.makespan, place_rank=plan.place_rank,
                map_rank=plan.map_rank, global_index=plan.global_index,
-               types=list(plan.type)[:S], layers=list(plan.layers)[:S])
+               types=list(plan.type)[:S], layers=list(plan.layers)[:J])
     stats = {n: (list(getattr(st, n)) if n.endswith("_depth") else getattr(st, n))
              for n, _ in pos_search_stats._fields_}
     return out, stats

@@ -19,6 +19,9 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libposeidon.so")
+# measurement tooling (the INT32 rate probe), kept out of the library's ABI
+PROBE_SRC = os.path.join(PKG, "probe", "int32_probe.cu")
+PROBE_LIB = os.path.join(PKG, "libposeidon_probe.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC"]
 
@@ -53,15 +56,31 @@ def _compile(src: str, verbose: bool, force: bool) -> str:
     return obj
 
 
+def _build_probe(force: bool) -> str:
+    hdr = os.path.join(ROOT, "include", "poseidon_probe.h")
+    if (force or not os.path.exists(PROBE_LIB) or
+            os.path.getmtime(PROBE_LIB) < max(os.path.getmtime(PROBE_SRC), os.path.getmtime(hdr))):
+        tmp = PROBE_LIB + f".tmp{os.getpid()}"
+        r = subprocess.run([nvcc(), *ARCH, *FLAGS, "-shared", PROBE_SRC, "-o", tmp],
+                           capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"nvcc failed for {PROBE_SRC}:\n{r.stdout}\n{r.stderr}")
+        os.replace(tmp, PROBE_LIB)
+    return PROBE_LIB
+
+
 def build(force: bool = False, verbose: bool = False, jobs: int | None = None) -> str:
-    """Compile every csrc/*.cu and link libposeidon.so; returns its path."""
+    """Compile every csrc/*.cu and link libposeidon.so (and the measurement
+    probe, libposeidon_probe.so); returns the library's path."""
     os.makedirs(BUILD, exist_ok=True)
     srcs = sorted(glob.glob(os.path.join(CSRC, "*.cu")))
-    jobs = jobs or max(1, min(len(srcs), os.cpu_count() or 1))
+    jobs = jobs or max(1, min(len(srcs) + 1, os.cpu_count() or 1))
     # the heaviest units (many unrolled instantiations) first
     srcs.sort(key=lambda s: (0 if "range" in s or "leaf" in s else 1, s))
     with ThreadPoolExecutor(jobs) as ex:
+        probe = ex.submit(_build_probe, force)
         objs = list(ex.map(lambda s: _compile(s, verbose, force), srcs))
+        probe.result()
     if (force or not os.path.exists(LIB) or
             os.path.getmtime(LIB) < max(os.path.getmtime(o) for o in objs)):
         tmp = LIB + f".tmp{os.getpid()}"

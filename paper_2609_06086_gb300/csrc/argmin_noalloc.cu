@@ -20,7 +20,6 @@ __global__ void argmin_final(const int32_t *part_t, const long long *part_i, int
                              int64_t *out);
 
 constexpr int kNoAllocParts = 4096;  // partial results the fixed scratch holds
-constexpr int kNoAllocThreads = 256;
 
 // 4096 x (int32 makespan, padded to 8 bytes) + 4096 x int64 index = 64 KB
 static __device__ __align__(256) unsigned char g_argmin_scratch[kNoAllocParts * 16];
@@ -31,7 +30,9 @@ static void *g_scratch_addr[kMaxDevices];  // device address of the array, per d
 
 // The name g_argmin_scratch in host code is only a host-side stand-in for
 // the array; its device address comes from cudaGetSymbolAddress, taken once
-// per device with that device current.
+// per device with that device current and kept for the life of the
+// process.  After cudaDeviceReset the module is loaded again and the array
+// may move, so the library must not be used across a device reset.
 static pos_status scratch_address(void **out) {
     int dev = 0;
     POS_CUDA(cudaGetDevice(&dev));
@@ -54,7 +55,7 @@ extern "C" pos_status poseidon_argmin_noalloc(const int32_t *d_makespan,
     if (n < 0 || !d_out || (n > 0 && (!d_makespan || !d_feasible)))
         return pos::fail(POS_EINVAL, "bad argmin arguments");
     const int64_t parts = std::max<int64_t>(
-        1, std::min<int64_t>((n + pos::kNoAllocThreads - 1) / pos::kNoAllocThreads,
+        1, std::min<int64_t>((n + pos::kArgminThreads - 1) / pos::kArgminThreads,
                              4LL * pos::sm_count()));
     if (parts > pos::kNoAllocParts)
         return pos::fail(POS_EINVAL,
@@ -69,7 +70,7 @@ extern "C" pos_status poseidon_argmin_noalloc(const int32_t *d_makespan,
         reinterpret_cast<long long *>(static_cast<char *>(scratch) + pos::kNoAllocParts * 8);
     // every slot the final kernel reads is written by the partial kernel of
     // the same call, so nothing has to be cleared between calls
-    pos::argmin_partial<<<(int)parts, pos::kNoAllocThreads, 0, s>>>(d_makespan, d_feasible, n, pt,
+    pos::argmin_partial<<<(int)parts, pos::kArgminThreads, 0, s>>>(d_makespan, d_feasible, n, pt,
                                                                      pi);
     pos::argmin_final<<<1, 32, 0, s>>>(pt, pi, (int)parts, d_out);
     const cudaError_t e = cudaGetLastError();

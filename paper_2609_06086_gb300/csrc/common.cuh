@@ -84,6 +84,10 @@ struct Handle {
     int lim_off, lim_w, lim_bytes;
 };
 constexpr int kLimMaxBytes = 32768;
+// Threads per block of the argmin partial kernel (poseidon_argmin and
+// poseidon_argmin_noalloc): its shared arrays hold one entry per warp of a
+// block of this size, so every launch must use exactly this many threads.
+constexpr int kArgminThreads = 256;
 
 pos_status validate_tables(const pos_tables *t);
 pos_status create_handle(const pos_tables *t, int sched, Handle **out);

@@ -11,8 +11,6 @@ namespace pos {
 // ---------------------------------------------------------------------------
 // argmin over (makespan, index) among feasible entries, ties -> lowest index
 // ---------------------------------------------------------------------------
-constexpr int kArgThreads = 256;
-
 __device__ __forceinline__ void better_of(int32_t &bt, long long &bi, int32_t t, long long i) {
     if (i >= 0 && (bi < 0 || t < bt || (t == bt && i < bi))) {
         bt = t;
@@ -33,8 +31,8 @@ __global__ void argmin_partial(const int32_t *T, const uint8_t *F, int64_t n, in
         const long long oi = __shfl_down_sync(0xffffffffu, bi, o);
         better_of(bt, bi, ot, oi);
     }
-    __shared__ int32_t st[kArgThreads / 32];
-    __shared__ long long si[kArgThreads / 32];
+    __shared__ int32_t st[kArgminThreads / 32];
+    __shared__ long long si[kArgminThreads / 32];
     if ((threadIdx.x & 31) == 0) {
         st[threadIdx.x >> 5] = bt;
         si[threadIdx.x >> 5] = bi;
@@ -417,13 +415,13 @@ pos_status poseidon_argmin(const int32_t *d_makespan, const uint8_t *d_feasible,
         return pos::fail(POS_EINVAL, "bad argmin arguments");
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const int parts = (int)std::max<int64_t>(
-        1, std::min<int64_t>((n + pos::kArgThreads - 1) / pos::kArgThreads,
+        1, std::min<int64_t>((n + pos::kArgminThreads - 1) / pos::kArgminThreads,
                              4LL * pos::sm_count()));
     void *scratch = nullptr;
     POS_CUDA(cudaMallocAsync(&scratch, (size_t)parts * 16, s));
     int32_t *pt = static_cast<int32_t *>(scratch);
     long long *pi = reinterpret_cast<long long *>(static_cast<char *>(scratch) + parts * 8);
-    pos::argmin_partial<<<parts, pos::kArgThreads, 0, s>>>(d_makespan, d_feasible, n, pt, pi);
+    pos::argmin_partial<<<parts, pos::kArgminThreads, 0, s>>>(d_makespan, d_feasible, n, pt, pi);
     pos::argmin_final<<<1, 32, 0, s>>>(pt, pi, parts, d_out);
     const cudaError_t e = cudaGetLastError();
     const cudaError_t e2 = cudaFreeAsync(scratch, s);

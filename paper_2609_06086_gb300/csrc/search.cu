@@ -61,7 +61,7 @@ __global__ void feas_kernel(const SliceRec *slices, int n_slices, int S, uint4 *
     __shared__ uint32_t prev[4], cur[4];
     __shared__ uint64_t bar;
     if (!stage_blob_bulk(sm, blob, lay.bytes, &bar)) {
-        if (threadIdx.x == 0) atomicAdd(stats + kStTimeout, 1ull);
+        if (threadIdx.x == 0) atomicAdd(stats + kStBulkTimeout, 1ull);
         return;
     }
     const Tab t = tab_at(sm, lay);
@@ -154,7 +154,7 @@ __global__ void __launch_bounds__(kBoundThreads) bound_kernel(
     __shared__ uint8_t arg[POS_MAX_STAGES][128];
     __shared__ uint64_t bar;
     if (!stage_blob_bulk(sm, blob, lay.bytes, &bar)) {
-        if (threadIdx.x == 0) atomicAdd(stats + kStTimeout, 1ull);
+        if (threadIdx.x == 0) atomicAdd(stats + kStBulkTimeout, 1ull);
         return;
     }
     const Tab t = tab_at(sm, lay);
@@ -713,7 +713,7 @@ __global__ void __launch_bounds__(kThreads, 3) level_kernel(ExpandParams p) {
                           vdepth + (size_t)__ldg(&p.slices[slot].vslot) * 128, 1024u, &bar);
     }
     if (!bulk_wait(&bar)) {
-        if (threadIdx.x == 0) atomicAdd(p.stats + kStTimeout, 1ull);
+        if (threadIdx.x == 0) atomicAdd(p.stats + kStBulkTimeout, 1ull);
         return;
     }
     const int2 *vsm = stage_v ? reinterpret_cast<const int2 *>(sm + p.lay.bytes) : nullptr;
@@ -985,6 +985,8 @@ static pos_status validate_problem(const pos_problem *p) {
     if (p->prune < 0 || p->prune > 2) return fail(POS_EINVAL, "prune must be 0, 1 or 2");
     if (p->ridge != 0 && p->ridge != 1) return fail(POS_EINVAL, "ridge must be 0 or 1");
     if (p->frontier_cap < 0) return fail(POS_EINVAL, "frontier_cap < 0");
+    if (p->schedule == POS_SCHED_INTERLEAVED_1F1B && (p->V < 2 || p->S * p->V > POS_MAX_STAGES))
+        return fail(POS_EINVAL, "Interleaved 1F1B needs V >= 2 and S*V <= 16");
     return POS_OK;
 }
 
@@ -1024,6 +1026,43 @@ static uint64_t host_binom(int n, int k) {
     uint64_t r = 1;
     for (int i = 1; i <= k; ++i) r = r * (uint64_t)(n - k + i) / (uint64_t)i;
     return r;
+}
+
+// Size limits of the search space, checked on the host before the device
+// is touched: at most 2^22 placements and 2^22 slices, a global index
+// (slices x compositions) below 2^64 and an objective scale (lcm of every
+// D*M) below 2^32.
+static pos_status validate_space(const pos_problem *p) {
+    const int S = p->S, T = p->tables.n_types, n_tp = p->tables.n_tp;
+    const uint64_t limit = 1ull << 22;
+    uint64_t n_place = 1;
+    if (p->placement == POS_PLACE_EXACT) {
+        // distinct orders of the multiset: S! / prod counts!, by binomials
+        int left = S;
+        for (int ty = 0; ty < T; ++ty) {
+            n_place *= host_binom(left, p->type_counts[ty]);  // <= C(16, 8) each step
+            left -= p->type_counts[ty];
+            if (n_place > limit) return fail(POS_EINVAL, "too many placements (above 2^22)");
+        }
+    } else {
+        for (int x = 0; x < S; ++x) {
+            n_place *= (uint64_t)T;
+            if (n_place > limit) return fail(POS_EINVAL, "too many placements (above 2^22)");
+        }
+    }
+    const uint64_t n_slices = (uint64_t)p->n_M * n_tp * n_place;
+    if (n_slices > limit) return fail(POS_EINVAL, "more than 2^22 slices");
+    const int J = p->schedule == POS_SCHED_INTERLEAVED_1F1B ? S * p->V : S;
+    const uint64_t n_map = host_binom(p->tables.L - 1, J - 1);
+    if (n_map && n_slices > ~0ull / n_map) return fail(POS_EINVAL, "global index overflows");
+    uint64_t Q = 1;
+    for (int i = 0; i < p->n_M; ++i)
+        for (int j = 0; j < n_tp; ++j) {
+            const uint64_t dm = (uint64_t)p->dp_list[j] * p->M_list[i];
+            Q = Q / gcd64(Q, dm) * dm;
+            if (Q >= (1ull << 32)) return fail(POS_EINVAL, "lcm of D*M reaches 2^32");
+        }
+    return POS_OK;
 }
 
 static void host_unrank(int L, int S, uint64_t rank, int32_t *layers) {
@@ -1141,6 +1180,7 @@ static pos_status run_leaves(Search &s, const Leaf *leaves, unsigned long long *
     s.launches++;
     lp.pg = s.pg;
     lp.ridge = s.pb->ridge;
+    lp.cas_limit = s.pb->cas_limit == 0 ? kCasLimit : std::max(0, s.pb->cas_limit);
     return launch_leaf(s.S, path_of(s.pb->schedule, s.S, M), lp, s.grid_leaf, s.stream);
 }
 
@@ -1660,7 +1700,12 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     if ((st = sync_read(s, &inc, s.d_inc.p, sizeof(inc))) != POS_OK) return st;
     unsigned long long hs[kStCount];
     if ((st = sync_read(s, hs, s.stats, sizeof(hs))) != POS_OK) return st;
-    if (hs[kStTimeout]) return fail(POS_ETIMEOUT, "incumbent update hit its iteration limit");
+    if (hs[kStTimeout])
+        return fail(POS_ETIMEOUT, "the incumbent's compare-and-swap loop hit its iteration "
+                                  "limit (pos_problem.cas_limit rounds)");
+    if (hs[kStBulkTimeout])
+        return fail(POS_ETIMEOUT, "a block's cost-table staging (TMA bulk copy) did not "
+                                  "complete within its poll limit");
 
     std::memset(out, 0, sizeof(*out));
     if (stats) {
@@ -1731,6 +1776,7 @@ extern "C" pos_status poseidon_search(const pos_problem *problem, pos_plan *out,
     pos::set_error("");
     pos_status st = pos::validate_problem(problem);  // before touching the device
     if (st == POS_OK) st = pos::validate_tables(&problem->tables);
+    if (st == POS_OK) st = pos::validate_space(problem);
     if (st != POS_OK) return st;
     pos::Workspace *ws = nullptr;
     st = pos::get_workspace(&ws);

@@ -97,12 +97,13 @@ enum {
     kStParentsComplete,
     kStLeaves,
     kStPrunedRidge,   // children cut by the layer-level (ridge) rule
+    kStBulkTimeout,   // blocks whose table staging (TMA bulk copy) wait ran out
     kStDepthParents,                                // + x: parents read at depth x
     kStDepthChildren = kStDepthParents + POS_MAX_STAGES,  // + x: children (plans) written
     kStCount = kStDepthChildren + POS_MAX_STAGES
 };
 
-constexpr int kCasLimit = 1 << 20;
+constexpr int kCasLimit = 1 << 20;  // default rounds of the incumbent's CAS loop
 
 __device__ __forceinline__ bool key_less(unsigned long long ao, unsigned long long ai,
                                          unsigned long long bo, unsigned long long bi) {
@@ -110,15 +111,16 @@ __device__ __forceinline__ bool key_less(unsigned long long ao, unsigned long lo
 }
 
 // Lower the incumbent to (obj, idx) if that is smaller.  Bounded loop: every
-// failed CAS means another thread lowered the key; after kCasLimit rounds
-// the timeout counter is raised and the update is abandoned.
+// failed CAS means another thread lowered the key; after `limit` rounds
+// (kCasLimit unless the problem sets another) the timeout counter is raised
+// and the update is abandoned.
 __device__ __forceinline__ void incumbent_update(Key128 *inc, unsigned long long obj,
                                                  unsigned long long idx,
-                                                 unsigned long long *stats) {
+                                                 unsigned long long *stats, int limit) {
     Key128 cur;
     cur.obj = __ldcg(&inc->obj);
     cur.idx = __ldcg(&inc->idx);
-    for (int it = 0; it < kCasLimit; ++it) {
+    for (int it = 0; it < limit; ++it) {
         if (!key_less(obj, idx, cur.obj, cur.idx)) return;
         Key128 want;
         want.obj = obj;
@@ -144,6 +146,7 @@ struct LeafParams {
     BlobLayout lay;
     Programs pg;  // level programs of the schedule's short path
     int ridge;    // 1: only ridge-like plans may lower the incumbent (warm-up plans)
+    int cas_limit;  // rounds of the incumbent's CAS loop
 };
 
 // leaf byte 4+s holds cut[s+1] (layers of stages 0..s)
@@ -173,7 +176,7 @@ __global__ void __launch_bounds__(256, leaf_min_blocks(S, PATH)) leaf_kernel(Lea
     // blocks without a plan leave before staging the tables
     if ((unsigned long long)blockIdx.x * blockDim.x >= n) return;
     if (!stage_blob_bulk(sm, p.blob, p.lay.bytes, &bar)) {
-        if (threadIdx.x == 0) atomicAdd(p.stats + kStTimeout, 1ull);
+        if (threadIdx.x == 0) atomicAdd(p.stats + kStBulkTimeout, 1ull);
         return;
     }
     const Tab t = tab_at(sm, p.lay);
@@ -224,7 +227,7 @@ __global__ void __launch_bounds__(256, leaf_min_blocks(S, PATH)) leaf_kernel(Lea
                 idx = oi;
             }
         }
-        if ((threadIdx.x & 31) == 0 && obj != ~0ull) incumbent_update(p.inc, obj, idx, p.stats);
+        if ((threadIdx.x & 31) == 0 && obj != ~0ull) incumbent_update(p.inc, obj, idx, p.stats, p.cas_limit);
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) evaluated += __shfl_xor_sync(0xffffffffu, evaluated, o);

@@ -1,12 +1,15 @@
-// poseidon_int32_probe: the rate at which this GPU runs the relaxation the
-// makespan kernels are built from, finish = max(pred + edge, clock) + weight
-// (one add, one max, one add: 3 int32 ops), with enough independent chains
-// per thread and threads per SM that no dependency or latency limits it.
-// The result checks the roofline denominator used for the ALU-bound kernels
-// (SMs x 128 int32 lanes x clock).
-#include "common.cuh"
+// Measurement tooling, not part of libposeidon: poseidon_probe_int32 times
+// the relaxation the makespan kernels are built from,
+// finish = max(pred + edge, clock) + weight (one add, one max, one add:
+// 3 int32 ops), with enough independent chains per thread and threads per
+// SM that no dependency or latency limits it.  The result checks the
+// roofline denominator the benchmark uses for the ALU-bound kernels
+// (SMs x 128 int32 lanes x clock).  Built into libposeidon_probe.so.
+#include <cuda_runtime.h>
 
-namespace pos {
+#include "../../include/poseidon_probe.h"
+
+namespace {
 
 constexpr int kProbeChains = 8;    // independent relaxation chains per thread
 constexpr int kProbeThreads = 256;
@@ -38,24 +41,29 @@ __global__ void __launch_bounds__(kProbeThreads) int32_probe_kernel(int iters, i
     if (acc == seed) out[0] = acc;  // keeps the chains live; practically never taken
 }
 
-}  // namespace pos
+}  // namespace
 
-extern "C" pos_status poseidon_int32_probe(void *stream, int64_t *ops, double *ms) {
-    if (!ops || !ms) return pos::fail(POS_EINVAL, "NULL output");
+extern "C" int poseidon_probe_int32(void *stream, int64_t *ops, double *ms) {
+    if (!ops || !ms) return (int)cudaErrorInvalidValue;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    const int blocks = pos::sm_count() * pos::kProbeBlocksPerSm;
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return (int)e;
+    const int blocks = sms * kProbeBlocksPerSm;
     const int iters = 4096;
     int32_t *d_out = nullptr;
-    POS_CUDA(cudaMallocAsync(reinterpret_cast<void **>(&d_out), sizeof(int32_t), s));
+    e = cudaMallocAsync(reinterpret_cast<void **>(&d_out), sizeof(int32_t), s);
+    if (e != cudaSuccess) return (int)e;
     cudaEvent_t e0 = nullptr, e1 = nullptr;
-    cudaError_t e = cudaEventCreate(&e0);
+    e = cudaEventCreate(&e0);
     if (e == cudaSuccess) e = cudaEventCreate(&e1);
     if (e == cudaSuccess) {
-        pos::int32_probe_kernel<<<blocks, pos::kProbeThreads, 0, s>>>(iters, 0x2f6e2b1, d_out);
+        int32_probe_kernel<<<blocks, kProbeThreads, 0, s>>>(iters, 0x2f6e2b1, d_out);
         e = cudaEventRecord(e0, s);
     }
     if (e == cudaSuccess) {
-        pos::int32_probe_kernel<<<blocks, pos::kProbeThreads, 0, s>>>(iters, 0x1b873593, d_out);
+        int32_probe_kernel<<<blocks, kProbeThreads, 0, s>>>(iters, 0x1b873593, d_out);
         e = cudaEventRecord(e1, s);
     }
     if (e == cudaSuccess) e = cudaGetLastError();
@@ -65,9 +73,9 @@ extern "C" pos_status poseidon_int32_probe(void *stream, int64_t *ops, double *m
     if (e0) cudaEventDestroy(e0);
     if (e1) cudaEventDestroy(e1);
     const cudaError_t e2 = cudaFreeAsync(d_out, s);
-    if (e != cudaSuccess) return pos::cuda_fail(e, "int32 probe");
-    if (e2 != cudaSuccess) return pos::cuda_fail(e2, "int32 probe free");
-    *ops = (int64_t)blocks * pos::kProbeThreads * iters * pos::kProbeChains * 6;
+    if (e != cudaSuccess) return (int)e;
+    if (e2 != cudaSuccess) return (int)e2;
+    *ops = (int64_t)blocks * kProbeThreads * iters * kProbeChains * 6;
     *ms = t;
-    return POS_OK;
+    return 0;
 }

@@ -115,6 +115,37 @@ def test_invalid_arguments_rejected_before_the_device(P):
         P.Handle(bad)
 
 
+def test_search_space_limits_rejected_before_the_device(P):
+    """poseidon_search checks its documented limits on the host: more than
+    2^22 slices (here 4 types free over 12 stages: 4^12 placements), and an
+    lcm of the D*M values reaching 2^32."""
+    import gen
+    L = P.lib()
+    plan = P.binding.pos_plan()
+    rng = np.random.default_rng(5)
+    K, Lw = 4, 16
+    w = gen.Workload(name="wide", L=Lw, n_types=4, n_tp=1,
+                     fwd=rng.integers(1, 9, (K, Lw)).astype(np.int32),
+                     bwd=rng.integers(1, 9, (K, Lw)).astype(np.int32),
+                     dsync=np.zeros((K, Lw), np.int32), p2p_f=np.zeros((K, K), np.int32),
+                     p2p_b=np.zeros((K, K), np.int32), mem_w=np.zeros((K, Lw), np.int64),
+                     mem_a=np.zeros((K, Lw), np.int64), cap=np.full(K, 10, np.int64),
+                     S=12, M_list=[4], tp_list=[1], dp_list=[1], seed=0)
+    prob, keep = P.make_problem(w)
+    assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
+    assert b"placements" in L.poseidon_last_error()
+    w.S = 11  # 4^11 = 2^22 placements pass; with two M values there are 2^23 slices
+    w.M_list = [4, 8]
+    prob, keep = P.make_problem(w)
+    assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
+    assert b"2^22 slices" in L.poseidon_last_error()
+    w.S = 2
+    w.M_list = [229, 233, 239, 241, 251]  # pairwise coprime: lcm = product > 2^32
+    prob, keep = P.make_problem(w)
+    assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
+    assert b"lcm" in L.poseidon_last_error()
+
+
 def test_binding_refuses_to_run_without_the_library(tmp_path, monkeypatch):
     import paper_2609_06086_gb300.binding as b
     monkeypatch.setattr(b, "LIB_PATH", str(tmp_path / "missing.so"))

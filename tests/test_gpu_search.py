@@ -164,3 +164,20 @@ def test_search_at_the_limits(P, orc, S, L, types, placement, counts, M_list):
             assert e.status == P.binding.POS_EINFEASIBLE and not ref["found"]
             continue
         assert same_plan(plan, ref), (prune, plan, ref)
+
+
+def test_incumbent_cas_limit_times_out_and_the_next_search_recovers(P, orc):
+    """The incumbent's compare-and-swap loop is bounded.  With no round
+    allowed (cas_limit < 0) every update that would lower the incumbent
+    gives up, the search returns POS_ETIMEOUT with a message naming that
+    loop, and the device stays usable: the next search on the same
+    workspace returns the oracle's plan."""
+    w = gen.config2()
+    prob, keep = P.make_problem(w, warmup=64, prune=2, cas_limit=-1)
+    with pytest.raises(P.PoseidonError) as err:
+        P.poseidon_search(prob)
+    assert err.value.status == P.binding.POS_ETIMEOUT
+    assert "compare-and-swap" in str(err.value)
+    plan, _ = gpu_search(P, w, warmup=64, prune=2)
+    ref, _ = orc.search(w, prune=True)
+    assert plan["global_index"] == ref["global_index"] and plan["T"] == ref["T"]
