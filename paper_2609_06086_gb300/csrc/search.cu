@@ -21,7 +21,7 @@
 #include <numeric>
 #include <vector>
 
-#include "search_kernels.cuh"
+#include "search_host.h"
 
 namespace pos {
 
@@ -846,62 +846,11 @@ __global__ void __launch_bounds__(kThreads, 3) level_kernel(ExpandParams p) {
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
-static uint64_t gcd64(uint64_t a, uint64_t b) {
-    while (b) {
-        const uint64_t r = a % b;
-        a = b;
-        b = r;
-    }
-    return a;
-}
-
-struct DevBuf {
-    void *p = nullptr;
-    size_t bytes = 0;
-    DevBuf() = default;
-    DevBuf(const DevBuf &) = delete;
-    DevBuf &operator=(const DevBuf &) = delete;
-    ~DevBuf() {
-        if (p) cudaFree(p);
-    }
-    cudaError_t reserve(size_t b) {
-        if (b <= bytes) return cudaSuccess;
-        if (p) cudaFree(p);
-        p = nullptr;
-        bytes = 0;
-        const cudaError_t e = cudaMalloc(&p, b);
-        if (e == cudaSuccess) bytes = b;
-        return e;
-    }
-};
-
-// Device work buffers, stream and events of one GPU, kept between calls
-// (grown on demand) so that a search allocates and frees nothing in the
-// steady state.  Searches on the same device are serialised by `mu`.
-struct Workspace {
-    std::mutex mu;
-    cudaStream_t stream = nullptr;
-    cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
-    DevBuf blob, d_lim, d_vb, d_bctr, d_rows, d_greedy, d_wcnt, d_lb, d_slices, d_feas, d_batch, d_inc, d_ctr, d_best, d_feasible, d_leaves, d_roots,
-        d_root;
-    DevBuf d_front[POS_MAX_STAGES + 1];        // per depth: Prefix buffers
-    DevBuf d_defer[2 * (POS_MAX_STAGES + 1)];  // per depth: two deferred group lists
-    unsigned long long *h_cnt = nullptr;       // pinned host counters
-    unsigned char *h_stage = nullptr;          // pinned staging area for uploads
-    size_t h_stage_cap = 0;
-    unsigned char *h_read = nullptr;           // pinned landing area for reads
-    size_t h_read_cap = 0;
-    unsigned long long *h_lb = nullptr;        // pinned landing area of the root bounds
-    size_t h_lb_cap = 0;                       // (elements)
-    cudaEvent_t ev_lb = nullptr;               // recorded after their copy
-    std::vector<cudaEvent_t> evs;              // timing events of the batch pipelines
-};
-
 constexpr int kMaxDevices = 64;
 static std::mutex g_ws_mutex;
 static Workspace *g_ws[kMaxDevices];
 
-static pos_status get_workspace(Workspace **out) {
+pos_status get_workspace(Workspace **out) {
     int dev = 0;
     POS_CUDA(cudaGetDevice(&dev));
     if (dev < 0 || dev >= kMaxDevices) return fail(POS_EINVAL, "device index above 63");
@@ -959,9 +908,12 @@ struct Search {
 
 static pos_status validate_problem(const pos_problem *p) {
     if (!p) return fail(POS_EINVAL, "problem is NULL");
-    if (p->schedule != POS_SCHED_1F1B && p->schedule != POS_SCHED_EAGER_1F1B)
-        return fail(POS_ENOTIMPL, "the search supports POS_SCHED_1F1B and POS_SCHED_EAGER_1F1B; "
-                                  "Interleaved 1F1B is evaluated by poseidon_eval_batch only");
+    if (p->schedule != POS_SCHED_1F1B && p->schedule != POS_SCHED_EAGER_1F1B &&
+        p->schedule != POS_SCHED_INTERLEAVED_1F1B)
+        return fail(POS_ENOTIMPL, "unknown schedule");
+    if (p->schedule == POS_SCHED_INTERLEAVED_1F1B && p->ridge)
+        return fail(POS_EINVAL, "layer-level (ridge) pruning is defined for 1F1B and Eager 1F1B "
+                                "plans only");
     if (p->S < 1 || p->S > POS_MAX_STAGES) return fail(POS_EINVAL, "S must be in 1..16");
     if (p->S > p->tables.L) return fail(POS_EINVAL, "S > L");
     if (p->n_M < 1 || !p->M_list) return fail(POS_EINVAL, "empty M_list");
@@ -1021,13 +973,6 @@ static pos_status enumerate_places(Search &s) {
     return POS_OK;
 }
 
-static uint64_t host_binom(int n, int k) {
-    if (k < 0 || k > n) return 0;
-    uint64_t r = 1;
-    for (int i = 1; i <= k; ++i) r = r * (uint64_t)(n - k + i) / (uint64_t)i;
-    return r;
-}
-
 // Size limits of the search space, checked on the host before the device
 // is touched: at most 2^22 placements and 2^22 slices, a global index
 // (slices x compositions) below 2^64 and an objective scale (lcm of every
@@ -1063,22 +1008,6 @@ static pos_status validate_space(const pos_problem *p) {
             if (Q >= (1ull << 32)) return fail(POS_EINVAL, "lcm of D*M reaches 2^32");
         }
     return POS_OK;
-}
-
-static void host_unrank(int L, int S, uint64_t rank, int32_t *layers) {
-    int rem = L;
-    for (int s = 0; s < S - 1; ++s) {
-        const int after = S - s - 1;
-        int v = 1;
-        for (; v <= rem - after; ++v) {
-            const uint64_t cnt = host_binom(rem - v - 1, after - 1);
-            if (rank < cnt) break;
-            rank -= cnt;
-        }
-        layers[s] = v;
-        rem -= v;
-    }
-    layers[S - 1] = rem;
 }
 
 static pos_status sync_read(Search &s, void *dst, const void *src, size_t bytes) {
@@ -1783,6 +1712,8 @@ extern "C" pos_status poseidon_search(const pos_problem *problem, pos_plan *out,
     if (st != POS_OK) return st;
     std::lock_guard<std::mutex> lock(ws->mu);
     try {
+        if (problem->schedule == POS_SCHED_INTERLEAVED_1F1B)
+            return pos::search_interleaved(*ws, problem, out, stats);
         pos::Search s(*ws);
         s.pb = problem;
         return pos::search_impl(s, out, stats);

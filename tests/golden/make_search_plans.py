@@ -7,7 +7,9 @@ single-threaded).  Calls only oracle/ and gen/.
     python tests/golden/make_search_plans.py [--configs 1 2 3 4] [--schedules 0 1] [--ridge]
 
 With --ridge the searches use the layer-level (ridge) rule of Theorem 2 and
-are stored as "configN_ridge" / "configN_eager_ridge".
+are stored as "configN_ridge" / "configN_eager_ridge".  With
+--interleaved V [V ...] the oracle's Interleaved 1F1B search (V chunks per
+device over the config's S devices) is stored as "configN_il_vV" instead.
 """
 import argparse
 import json
@@ -30,8 +32,23 @@ def main():
     ap.add_argument("--schedules", type=int, nargs="*", default=[0, 1],
                     help="0 = 1F1B, 1 = Eager 1F1B")
     ap.add_argument("--ridge", action="store_true", help="layer-level (ridge) pruning")
+    ap.add_argument("--interleaved", type=int, nargs="*", default=None,
+                    help="V values: Interleaved 1F1B searches instead")
     args = ap.parse_args()
     data = json.load(open(OUT)) if os.path.exists(OUT) else {}
+    if args.interleaved:
+        for c in args.configs:
+            for V in args.interleaved:
+                w = gen.get_config(c)
+                t0 = time.time()
+                plan, stats = oracle.search_interleaved(w, V, prune=True)
+                key = f"config{c}_il_v{V}"
+                data[key] = dict(workload=w.name, seed=w.seed, schedule=2, V=V, plan=plan,
+                                 oracle_stats=stats, oracle_seconds=round(time.time() - t0, 2))
+                print(key, plan, flush=True)
+                with open(OUT, "w") as f:
+                    json.dump(data, f, indent=1, sort_keys=True)
+        return
     for sched in args.schedules:
         for c in args.configs:
             w = gen.get_config(c)

@@ -103,9 +103,17 @@ def test_invalid_arguments_rejected_before_the_device(P):
     prob.warmup = -1
     assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
     prob.warmup = 0
-    prob.schedule = 2  # Interleaved 1F1B: evaluated by poseidon_eval_batch only
+    prob.schedule = 2  # Interleaved 1F1B needs V >= 2 and S*V <= 16 (S = 2 here)
+    for V in (0, 1, 9):
+        prob.V = V
+        assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
+        assert b"Interleaved" in L.poseidon_last_error()
+    prob.V = 2
+    prob.ridge = 1  # the ridge rule is defined for 1F1B and Eager 1F1B plans
+    assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
+    prob.ridge = 0
+    prob.schedule = 7
     assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_ENOTIMPL
-    assert b"Interleaved" in L.poseidon_last_error()
     prob.schedule = 0
     for mode in (-1, 3):
         prob.prune = mode
