@@ -61,8 +61,8 @@ typedef int32_t pos_status;
  *       chunks must fit cap of its class.  The edge between virtual stages
  *       j and j+1 uses the classes of their devices (p2p_f[k_{j%N}][k_{(j+1)%N}],
  *       p2p_b[k_{(j+1)%N}][k_{j%N}]); R_d sums dsync over the device's chunks
- *       and follows its last op.  Evaluated by poseidon_eval_batch only;
- *       poseidon_search returns POS_ENOTIMPL for it. */
+ *       and follows its last op.  poseidon_eval_batch evaluates such
+ *       records; poseidon_search searches over them (pos_problem.V). */
 #define POS_SCHED_1F1B 0
 #define POS_SCHED_EAGER_1F1B 1
 #define POS_SCHED_INTERLEAVED_1F1B 2
@@ -283,7 +283,8 @@ typedef struct pos_problem {
     int32_t warmup;             /* random feasible samples seeding T_min (paper: 500) */
     int32_t prune;              /* POS_PRUNE_NONE, POS_PRUNE_EQ2 or POS_PRUNE_TIGHT */
     uint64_t seed;              /* warm-up sampling seed */
-    int32_t schedule;           /* POS_SCHED_1F1B or POS_SCHED_EAGER_1F1B */
+    int32_t schedule;           /* POS_SCHED_1F1B, POS_SCHED_EAGER_1F1B or
+                                   POS_SCHED_INTERLEAVED_1F1B (with V below) */
     int64_t frontier_cap;       /* entries per frontier buffer; 0 = default 2^24;
                                    raised to at least 32*L */
     int32_t profile;            /* 1: device time per kernel kind in the stats (CUDA
@@ -350,6 +351,16 @@ typedef struct pos_search_stats {
  * and the stage-level prune chosen by problem->prune (Eq. 2 / Theorem 1, or
  * the tighter bound); the result equals the exhaustive optimum.  Host pointers in, host plan out;
  * synchronous.  stats may be NULL.
+ * Under POS_SCHED_INTERLEAVED_1F1B the S = N devices hold problem->V chunks
+ * each: a plan is a slice (M, TP index, type placement over the N devices)
+ * and a composition of L into the N*V virtual stages (C(L-1, NV-1) per
+ * slice in the global index); M values that are not multiples of N are
+ * skipped (their indices still count).  Prune modes there: POS_PRUNE_EQ2
+ * cuts a prefix when some device's serial work over its placed chunks,
+ * M * sum (F + B) + sum dsync, is already worse than the incumbent;
+ * POS_PRUNE_TIGHT adds, per device whose first chunk is placed, the path
+ * through the fill forwards, its chain and the drain backwards.  Layer-level
+ * (ridge) pruning is not defined there (POS_EINVAL).
  * Errors: POS_EINVAL, POS_EOVERFLOW (guard fails for some M), POS_ENOMEM,
  * POS_ECUDA, POS_ETIMEOUT, POS_EINFEASIBLE (no memory-feasible plan; *out
  * has found = 0).

@@ -65,13 +65,12 @@ def test_config2_v2_matches_oracle_live(P, orc):
         assert st["evaluated"] > 0 and st["relaxations"] > 0
 
 
-@pytest.mark.parametrize("V", [2, 3, 4])
+@pytest.mark.parametrize("V", [2, 3])
 def test_config2_matches_stored_oracle_plan(P, V):
+    """Stored oracle plans (V = 4 would make the oracle enumerate 16 virtual
+    stages over 32 layers, C(31, 15) compositions per slice: not stored)."""
     data = json.load(open(GOLDEN))
-    key = f"config2_il_v{V}"
-    if key not in data:
-        pytest.skip(f"{key} not stored")
-    ref = data[key]["plan"]
+    ref = data[f"config2_il_v{V}"]["plan"]
     for prune in (1, 2):
         check(P, gen.config2(), V, ref, prune=prune)
 
