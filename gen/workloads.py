@@ -50,6 +50,7 @@ assert CANDIDATE_EX_DTYPE.itemsize == 24
 
 PLACE_FREE = 0
 PLACE_EXACT = 1
+PLACE_DEVICES = 2  # a (type, TP index) per stage; type_counts = devices per type
 
 
 @dataclass
@@ -72,7 +73,8 @@ class Workload:
     tp_list: list = field(default_factory=list)
     dp_list: list = field(default_factory=list)
     placement: int = PLACE_FREE
-    type_counts: list = field(default_factory=list)
+    type_counts: list = field(default_factory=list)   # stages (EXACT) / devices (DEVICES) per type
+    D_list: list = field(default_factory=list)        # data-parallel degrees (DEVICES)
     seed: int = 0
 
     @property

@@ -36,7 +36,8 @@ class Tables(C.Structure):
 class Problem(C.Structure):
     _fields_ = [("tab", Tables), ("S", C.c_int32), ("n_M", C.c_int32), ("M_list", C.c_void_p),
                 ("dp_list", C.c_void_p), ("placement", C.c_int32), ("type_counts", C.c_void_p),
-                ("ridge", C.c_int32)]
+                ("ridge", C.c_int32), ("tp_list", C.c_void_p), ("n_D", C.c_int32),
+                ("D_list", C.c_void_p)]
 
 
 class Plan(C.Structure):
@@ -44,7 +45,8 @@ class Plan(C.Structure):
                 ("M", C.c_int32), ("D", C.c_int32), ("T", C.c_int32),
                 ("place_rank", C.c_uint64), ("map_rank", C.c_uint64),
                 ("global_index", C.c_uint64),
-                ("types", C.c_int32 * MAX_S), ("layers", C.c_int32 * MAX_S)]
+                ("types", C.c_int32 * MAX_S), ("layers", C.c_int32 * MAX_S),
+                ("tps", C.c_int32 * MAX_S), ("d_idx", C.c_int32)]
 
 
 class Stats(C.Structure):
@@ -266,15 +268,31 @@ def eval_batch_ex(tab: OracleTables, cands: np.ndarray):
     return T, F
 
 
+def _problem(w, tab, ridge):
+    """Problem struct for a gen.Workload and the arrays it points into."""
+    keep = [_i32(w.M_list), _i32(w.dp_list if w.dp_list else [1] * w.n_tp),
+            _i32(w.type_counts if w.type_counts else [0] * w.n_types),
+            _i32(w.tp_list if w.tp_list else [1] * w.n_tp),
+            _i32(w.D_list if w.D_list else [1])]
+    M_list, dp, tc, tpl, Dl = keep
+    p = Problem(tab.c, w.S, len(M_list), M_list.ctypes.data, dp.ctypes.data, w.placement,
+                tc.ctypes.data, int(bool(ridge)), tpl.ctypes.data, len(Dl), Dl.ctypes.data)
+    return p, keep
+
+
+def _plan_dict(plan, n_units, n_layers):
+    return dict(found=bool(plan.found), m_idx=plan.m_idx, tp_idx=plan.tp_idx,
+                d_idx=plan.d_idx, M=plan.M, D=plan.D, T=plan.T, place_rank=plan.place_rank,
+                map_rank=plan.map_rank, global_index=plan.global_index,
+                types=list(plan.types)[:n_units], tps=list(plan.tps)[:n_units],
+                layers=list(plan.layers)[:n_layers])
+
+
 def search(w, prune=True, warmup=0, seed=0, tab: OracleTables | None = None,
            schedule=SCHED_1F1B, ridge=False):
     """Exact search over a gen.Workload search problem.  Returns (plan dict, stats dict)."""
     tab = tab or OracleTables.from_workload(w, schedule)
-    M_list = _i32(w.M_list)
-    dp = _i32(w.dp_list)
-    tc = _i32(w.type_counts if w.type_counts else [0] * w.n_types)
-    p = Problem(tab.c, w.S, len(M_list), M_list.ctypes.data, dp.ctypes.data, w.placement,
-                tc.ctypes.data, int(bool(ridge)))
+    p, keep = _problem(w, tab, ridge)
     plan, st = Plan(), Stats()
     rc = lib().orc_search(C.byref(p), int(prune), int(warmup), C.c_uint64(seed), C.byref(plan),
                           C.byref(st))
@@ -282,11 +300,7 @@ def search(w, prune=True, warmup=0, seed=0, tab: OracleTables | None = None,
         raise OverflowError("overflow guard")
     if rc:
         raise RuntimeError("oracle search failed")
-    S = w.S
-    out = dict(found=bool(plan.found), m_idx=plan.m_idx, tp_idx=plan.tp_idx, M=plan.M, D=plan.D,
-               T=plan.T, place_rank=plan.place_rank, map_rank=plan.map_rank,
-               global_index=plan.global_index, types=list(plan.types)[:S],
-               layers=list(plan.layers)[:S])
+    out = _plan_dict(plan, w.S, w.S)
     stats = {n: getattr(st, n) for n, _ in Stats._fields_}
     return out, stats
 
@@ -295,11 +309,7 @@ def search_interleaved(w, V, prune=True, tab: OracleTables | None = None):
     """Search over Interleaved 1F1B plans with V chunks per device (w.S
     devices).  Returns (plan dict, stats dict); layers has N*V entries."""
     tab = tab or OracleTables.from_workload(w, SCHED_INTERLEAVED_1F1B)
-    M_list = _i32(w.M_list)
-    dp = _i32(w.dp_list)
-    tc = _i32(w.type_counts if w.type_counts else [0] * w.n_types)
-    p = Problem(tab.c, w.S, len(M_list), M_list.ctypes.data, dp.ctypes.data, w.placement,
-                tc.ctypes.data, 0)
+    p, keep = _problem(w, tab, False)
     plan, st = Plan(), Stats()
     rc = lib().orc_search_interleaved(C.byref(p), int(V), int(prune), C.byref(plan),
                                       C.byref(st))
@@ -307,10 +317,6 @@ def search_interleaved(w, V, prune=True, tab: OracleTables | None = None):
         raise OverflowError("overflow guard")
     if rc:
         raise RuntimeError("oracle interleaved search failed")
-    J = w.S * V
-    out = dict(found=bool(plan.found), m_idx=plan.m_idx, tp_idx=plan.tp_idx, M=plan.M, D=plan.D,
-               T=plan.T, place_rank=plan.place_rank, map_rank=plan.map_rank,
-               global_index=plan.global_index, types=list(plan.types)[:w.S],
-               layers=list(plan.layers)[:J])
+    out = _plan_dict(plan, w.S, w.S * V)
     return out, {n: getattr(st, n) for n, _ in Stats._fields_}
 

@@ -805,9 +805,9 @@ int orc_eval_batch_ex(const orc_tables *t, const orc_candidate_ex *c, int64_t n,
 /* ------------------------------------------------------------------ */
 typedef struct {
     const orc_problem *p;
-    int S, L, M, D, m_idx, tp_idx, prune, ridge;
-    uint64_t place_rank, n_place, n_map;
-    int32_t cls[ORC_MAX_S], types[ORC_MAX_S], layers[ORC_MAX_S];
+    int S, L, M, D, m_idx, tp_idx, d_idx, prune, ridge;
+    uint64_t place_rank, ordinal, n_map;
+    int32_t cls[ORC_MAX_S], types[ORC_MAX_S], tps[ORC_MAX_S], layers[ORC_MAX_S];
     unsigned char *feas; /* feas[x*(L+1)+c]: layers [c, L) fit stages x..S-1 */
     orc_plan *best;
     orc_stats *st;
@@ -848,13 +848,13 @@ static void consider_leaf(search_ctx *cx) {
         return;
     }
     uint64_t map_rank = orc_rank(cx->L, cx->S, cx->layers);
-    uint64_t idx = ((((uint64_t)cx->m_idx * cx->p->tab.n_tp + cx->tp_idx) * cx->n_place +
-                     cx->place_rank) * cx->n_map) + map_rank;
+    uint64_t idx = cx->ordinal * cx->n_map + map_rank;
     if (better(T64, cx->D, cx->M, idx, cx->best)) {
         orc_plan *b = cx->best;
         b->found = 1;
         b->m_idx = cx->m_idx;
         b->tp_idx = cx->tp_idx;
+        b->d_idx = cx->d_idx;
         b->M = cx->M;
         b->D = cx->D;
         b->T = (int32_t)T64;
@@ -863,6 +863,7 @@ static void consider_leaf(search_ctx *cx) {
         b->global_index = idx;
         for (int s = 0; s < ORC_MAX_S; ++s) {
             b->types[s] = s < cx->S ? cx->types[s] : -1;
+            b->tps[s] = s < cx->S ? cx->tps[s] : -1;
             b->layers[s] = s < cx->S ? cx->layers[s] : 0;
         }
     }
@@ -942,28 +943,125 @@ static void suffix_feasibility(search_ctx *cx) {
                 }
 }
 
-/* next type sequence in lexicographic order among the allowed placements */
-static int next_placement(const orc_problem *p, int32_t *seq, int first) {
-    int S = p->S, T = p->tab.n_types;
-    for (;;) {
-        if (first) {
-            for (int s = 0; s < S; ++s) seq[s] = 0;
-            first = 0;
-        } else {
+/* ------------------------------------------------------------------ */
+/* Slices of the search space in global-index order (Sec. 4.2.3): the  */
+/* M value, then the TP index (placements 0, 1) or the data-parallel   */
+/* degree (placement 2), then the allowed stage sequences in           */
+/* lexicographic order.                                                */
+/* ------------------------------------------------------------------ */
+typedef struct {
+    int m_idx, grp;          /* grp: TP index (placements 0, 1), D index (placement 2) */
+    int M, D;
+    uint64_t place_rank;     /* rank among the allowed sequences of this grp */
+    uint64_t ordinal;        /* global index = ordinal * n_map + map_rank */
+    int32_t cls[ORC_MAX_S], types[ORC_MAX_S], tps[ORC_MAX_S];
+} orc_slice;
+
+/* Is the sequence seq[0..S-1] allowed?  Placements 0 and 1: seq holds
+ * device types (1: exactly type_counts[t] stages of type t).  Placement 2:
+ * seq holds classes k = type * n_tp + tp_idx, and the stages of each type
+ * use D * tp_list[tp_idx] devices each, type_counts[type] in total. */
+static int sequence_allowed(const orc_problem *p, const int32_t *seq, int S, int D) {
+    int T = p->tab.n_types, n_tp = p->tab.n_tp;
+    if (p->placement == 0) return 1;
+    for (int ty = 0; ty < T; ++ty) {
+        int64_t cnt = 0;
+        for (int s = 0; s < S; ++s) {
+            if (p->placement == 1) cnt += seq[s] == ty;
+            else if (seq[s] / n_tp == ty) cnt += (int64_t)D * p->tp_list[seq[s] % n_tp];
+        }
+        if (cnt != p->type_counts[ty]) return 0;
+    }
+    return 1;
+}
+
+/* Every slice of p for S stages (devices), in order; NULL on failure. */
+static orc_slice *list_slices(const orc_problem *p, int S, uint64_t *count) {
+    const int n_tp = p->tab.n_tp, per_stage = p->placement == 2;
+    const int alpha = per_stage ? p->tab.n_types * n_tp : p->tab.n_types;
+    const int n_grp = per_stage ? p->n_D : n_tp;
+    /* allowed sequences per group (one list shared by every TP index when
+       the rule does not depend on it), each in lexicographic order */
+    int32_t **seqs = calloc((size_t)n_grp, sizeof(int32_t *));
+    uint64_t *n_seq = calloc((size_t)n_grp, sizeof(uint64_t));
+    orc_slice *out = NULL;
+    *count = 0;
+    if (!seqs || !n_seq) goto done;
+    for (int g = 0; g < n_grp; ++g) {
+        if (!per_stage && g > 0) break;
+        const int D = per_stage ? p->D_list[g] : 1;
+        uint64_t cap = 0;
+        int32_t seq[ORC_MAX_S];
+        for (int s = 0; s < S; ++s) seq[s] = 0;
+        for (;;) {  /* odometer over alpha^S, last stage fastest */
+            if (sequence_allowed(p, seq, S, D)) {
+                if (n_seq[g] == cap) {
+                    cap = cap ? 2 * cap : 64;
+                    int32_t *grown = realloc(seqs[g], sizeof(int32_t) * S * cap);
+                    if (!grown) goto done;
+                    seqs[g] = grown;
+                }
+                memcpy(seqs[g] + n_seq[g] * S, seq, sizeof(int32_t) * S);
+                n_seq[g]++;
+            }
             int s = S - 1;
-            while (s >= 0 && seq[s] == T - 1) seq[s--] = 0;
-            if (s < 0) return 0;
+            while (s >= 0 && seq[s] == alpha - 1) seq[s--] = 0;
+            if (s < 0) break;
             seq[s]++;
         }
-        if (p->placement == 0) return 1;
-        int ok = 1;
-        for (int ty = 0; ty < T && ok; ++ty) {
-            int cnt = 0;
-            for (int s = 0; s < S; ++s) cnt += seq[s] == ty;
-            ok = cnt == p->type_counts[ty];
-        }
-        if (ok) return 1;
     }
+    uint64_t per_m = 0;
+    for (int g = 0; g < n_grp; ++g) per_m += n_seq[per_stage ? g : 0];
+    out = malloc(sizeof(orc_slice) * (per_m * p->n_M > 0 ? per_m * p->n_M : 1));
+    if (!out) goto done;
+    uint64_t o = 0;
+    for (int mi = 0; mi < p->n_M; ++mi)
+        for (int g = 0; g < n_grp; ++g) {
+            const int q = per_stage ? g : 0;
+            for (uint64_t pr = 0; pr < n_seq[q]; ++pr, ++o) {
+                orc_slice *sl = &out[o];
+                const int32_t *seq = seqs[q] + pr * S;
+                sl->m_idx = mi;
+                sl->grp = g;
+                sl->M = p->M_list[mi];
+                sl->D = per_stage ? p->D_list[g] : p->dp_list[g];
+                sl->place_rank = pr;
+                sl->ordinal = o;
+                for (int s = 0; s < ORC_MAX_S; ++s) {
+                    const int k = s < S ? (per_stage ? seq[s] : seq[s] * n_tp + g) : 0;
+                    sl->cls[s] = k;
+                    sl->types[s] = k / n_tp;
+                    sl->tps[s] = k % n_tp;
+                }
+            }
+        }
+    *count = o;
+done:
+    if (seqs)
+        for (int g = 0; g < n_grp; ++g) free(seqs[g]);
+    free(seqs);
+    free(n_seq);
+    return out;
+}
+
+/* Checks shared by both searches on the slice-space fields of p. */
+static int slice_space_valid(const orc_problem *p) {
+    if (p->placement < 0 || p->placement > 2) return 0;
+    if (p->placement >= 1 && !p->type_counts) return 0;
+    if (p->placement == 2) {
+        if (p->ridge || !p->tp_list || !p->D_list || p->n_D < 1) return 0;
+        for (int i = 0; i < p->tab.n_tp; ++i)
+            if (p->tp_list[i] < 1) return 0;
+        for (int i = 0; i < p->n_D; ++i)
+            if (p->D_list[i] < 1) return 0;
+        for (int ty = 0; ty < p->tab.n_types; ++ty)
+            if (p->type_counts[ty] < 0) return 0;
+    } else {
+        if (!p->dp_list) return 0;
+        for (int i = 0; i < p->tab.n_tp; ++i)
+            if (p->dp_list[i] < 1) return 0;
+    }
+    return 1;
 }
 
 /* splitmix64 (Steele, Lea & Flood, OOPSLA 2014) for warm-up sampling */
@@ -974,17 +1072,18 @@ static uint64_t splitmix64(uint64_t *state) {
     return z ^ (z >> 31);
 }
 
-static void set_slice(search_ctx *cx, int m_idx, int tp_idx, uint64_t place_rank,
-                      const int32_t *seq) {
-    const orc_problem *p = cx->p;
-    cx->m_idx = m_idx;
-    cx->tp_idx = tp_idx;
-    cx->M = p->M_list[m_idx];
-    cx->D = p->dp_list[tp_idx];
-    cx->place_rank = place_rank;
+static void set_slice(search_ctx *cx, const orc_slice *sl) {
+    cx->m_idx = sl->m_idx;
+    cx->tp_idx = cx->p->placement == 2 ? -1 : sl->grp;
+    cx->d_idx = cx->p->placement == 2 ? sl->grp : -1;
+    cx->M = sl->M;
+    cx->D = sl->D;
+    cx->place_rank = sl->place_rank;
+    cx->ordinal = sl->ordinal;
     for (int s = 0; s < cx->S; ++s) {
-        cx->types[s] = seq[s];
-        cx->cls[s] = seq[s] * p->tab.n_tp + tp_idx;
+        cx->types[s] = sl->types[s];
+        cx->tps[s] = sl->tps[s];
+        cx->cls[s] = sl->cls[s];
     }
     suffix_feasibility(cx);
 }
@@ -993,12 +1092,11 @@ int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_p
                orc_stats *stats) {
     int S = p->S, L = p->tab.L;
     if (S < 1 || S > ORC_MAX_S || S > L || L > 127 || p->n_M < 1 || p->tab.n_types < 1 ||
-        p->tab.n_types > 4 || p->tab.n_tp < 1 || !tables_nonnegative(&p->tab))
+        p->tab.n_types > 4 || p->tab.n_tp < 1 || !tables_nonnegative(&p->tab) ||
+        !slice_space_valid(p))
         return -1;
     for (int i = 0; i < p->n_M; ++i)
         if (p->M_list[i] < 1 || p->M_list[i] > 255) return -1;
-    for (int i = 0; i < p->tab.n_tp; ++i)
-        if (p->dp_list[i] < 1) return -1;
     for (int i = 0; i < p->n_M; ++i)
         if (overflow_bound(&p->tab, S, p->M_list[i]) >= ((int64_t)1 << 31)) return -2;
 
@@ -1015,58 +1113,44 @@ int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_p
     cx.st = stats;
     cx.n_map = n_comp(L, S);
     cx.feas = malloc((size_t)(S + 1) * (L + 1));
-    if (!cx.feas) return -1;
-
-    int32_t seq[ORC_MAX_S];
-    cx.n_place = 0;
-    for (int f = 1; next_placement(p, seq, f); f = 0) cx.n_place++;
+    uint64_t n_slices = 0;
+    orc_slice *slices = list_slices(p, S, &n_slices);
+    if (!cx.feas || !slices) {
+        free(cx.feas);
+        free(slices);
+        return -1;
+    }
 
     /* warm-up: random feasible configurations seed T_min (Sec. 4.2.3) */
-    if (warmup > 0 && cx.n_place > 0 && cx.n_place <= (1u << 20)) {
-        int32_t *places = malloc(sizeof(int32_t) * S * cx.n_place);
-        if (places) {
-            uint64_t i = 0;
-            for (int f = 1; next_placement(p, seq, f); f = 0, ++i)
-                memcpy(places + i * S, seq, sizeof(int32_t) * S);
-            uint64_t rs = seed;
-            uint64_t n_slices = (uint64_t)p->n_M * p->tab.n_tp * cx.n_place;
-            for (int w = 0; w < warmup; ++w) {
-                uint64_t sl = splitmix64(&rs) % n_slices;
-                uint64_t pr = sl % cx.n_place;
-                int tp = (int)((sl / cx.n_place) % p->tab.n_tp);
-                int mi = (int)(sl / cx.n_place / p->tab.n_tp);
-                set_slice(&cx, mi, tp, pr, places + pr * S);
-                if (!cx.feas[0]) continue;
-                int used = 0;
-                for (int x = 0; x < S; ++x) {
-                    int opts[128], n = 0;
-                    int hi = L - used - (S - x - 1), lo = x == S - 1 ? hi : 1;
-                    for (int l = lo; l <= hi; ++l)
-                        if (stage_memory_ok(&p->tab, S, cx.M, x, cx.cls[x], used, l) &&
-                            cx.feas[(x + 1) * (L + 1) + used + l])
-                            opts[n++] = l;
-                    cx.layers[x] = opts[splitmix64(&rs) % (uint64_t)n];
-                    used += cx.layers[x];
-                }
-                stats->warmup_evaluated++;
-                /* with layer-level pruning only ridge-like plans can be the result */
-                if (!cx.ridge || ridge_ok(cx.types, cx.layers, cx.S)) consider_leaf(&cx);
+    if (warmup > 0 && n_slices > 0) {
+        uint64_t rs = seed;
+        for (int w = 0; w < warmup; ++w) {
+            set_slice(&cx, &slices[splitmix64(&rs) % n_slices]);
+            if (!cx.feas[0]) continue;
+            int used = 0;
+            for (int x = 0; x < S; ++x) {
+                int opts[128], n = 0;
+                int hi = L - used - (S - x - 1), lo = x == S - 1 ? hi : 1;
+                for (int l = lo; l <= hi; ++l)
+                    if (stage_memory_ok(&p->tab, S, cx.M, x, cx.cls[x], used, l) &&
+                        cx.feas[(x + 1) * (L + 1) + used + l])
+                        opts[n++] = l;
+                cx.layers[x] = opts[splitmix64(&rs) % (uint64_t)n];
+                used += cx.layers[x];
             }
-            free(places);
+            stats->warmup_evaluated++;
+            /* with layer-level pruning only ridge-like plans can be the result */
+            if (!cx.ridge || ridge_ok(cx.types, cx.layers, cx.S)) consider_leaf(&cx);
         }
     }
 
     /* exhaustive enumeration in global-index order with the two cuts */
-    for (int mi = 0; mi < p->n_M && !cx.err; ++mi) {
-        for (int tp = 0; tp < p->tab.n_tp && !cx.err; ++tp) {
-            uint64_t pr = 0;
-            for (int f = 1; next_placement(p, seq, f) && !cx.err; f = 0, ++pr) {
-                set_slice(&cx, mi, tp, pr, seq);
-                if (!cx.feas[0]) continue;
-                dfs(&cx, 0, 0);
-            }
-        }
+    for (uint64_t i = 0; i < n_slices && !cx.err; ++i) {
+        set_slice(&cx, &slices[i]);
+        if (!cx.feas[0]) continue;
+        dfs(&cx, 0, 0);
     }
+    free(slices);
     free(cx.feas);
     dag_free(&cx.g);
     return cx.err ? -1 : 0;
@@ -1091,9 +1175,9 @@ int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_p
  *     incumbent (objective T/(D*M), strictly) is cut. */
 typedef struct {
     const orc_problem *p;
-    int N, V, J, L, M, D, m_idx, tp_idx, prune;
-    uint64_t place_rank, n_place, n_map;
-    int32_t cls[ORC_MAX_S], types[ORC_MAX_S], layers[ORC_MAX_S];
+    int N, V, J, L, M, D, m_idx, tp_idx, d_idx, prune;
+    uint64_t place_rank, ordinal, n_map;
+    int32_t cls[ORC_MAX_S], types[ORC_MAX_S], tps[ORC_MAX_S], layers[ORC_MAX_S];
     int64_t wsum[ORC_MAX_S], work[ORC_MAX_S];
     orc_plan *best;
     orc_stats *st;
@@ -1109,16 +1193,14 @@ static void il_leaf(il_ctx *cx) {
     }
     cx->st->leaves_evaluated++;
     if (!F) return;
-    const int n_tp = cx->p->tab.n_tp;
     const uint64_t map_rank = orc_rank(cx->L, cx->J, cx->layers);
-    const uint64_t idx =
-        (((uint64_t)cx->m_idx * n_tp + cx->tp_idx) * cx->n_place + cx->place_rank) * cx->n_map +
-        map_rank;
+    const uint64_t idx = cx->ordinal * cx->n_map + map_rank;
     if (!better(T, cx->D, cx->M, idx, cx->best)) return;
     orc_plan *b = cx->best;
     b->found = 1;
     b->m_idx = cx->m_idx;
     b->tp_idx = cx->tp_idx;
+    b->d_idx = cx->d_idx;
     b->M = cx->M;
     b->D = cx->D;
     b->T = T;
@@ -1127,6 +1209,7 @@ static void il_leaf(il_ctx *cx) {
     b->global_index = idx;
     for (int s = 0; s < ORC_MAX_S; ++s) {
         b->types[s] = s < cx->N ? cx->types[s] : 0;
+        b->tps[s] = s < cx->N ? cx->tps[s] : -1;
         b->layers[s] = s < cx->J ? cx->layers[s] : 0;
     }
 }
@@ -1176,12 +1259,10 @@ int orc_search_interleaved(const orc_problem *p, int V, int prune, orc_plan *pla
     const int N = p->S, L = p->tab.L, J = N * V;
     if (N < 1 || V < 2 || J > ORC_MAX_S || J > L || L > 127 || p->n_M < 1 ||
         p->tab.n_types < 1 || p->tab.n_types > 4 || p->tab.n_tp < 1 ||
-        !tables_nonnegative(&p->tab))
+        !tables_nonnegative(&p->tab) || !slice_space_valid(p) || p->ridge)
         return -1;
     for (int i = 0; i < p->n_M; ++i)
         if (p->M_list[i] < 1 || p->M_list[i] > 255) return -1;
-    for (int i = 0; i < p->tab.n_tp; ++i)
-        if (p->dp_list[i] < 1) return -1;
     for (int i = 0; i < p->n_M; ++i)
         if (p->M_list[i] % N == 0 && overflow_bound(&p->tab, J, p->M_list[i]) >= ((int64_t)1 << 31))
             return -2;
@@ -1198,29 +1279,28 @@ int orc_search_interleaved(const orc_problem *p, int V, int prune, orc_plan *pla
     cx.best = plan;
     cx.st = stats;
     cx.n_map = n_comp(L, J);
-    int32_t seq[ORC_MAX_S];
-    cx.n_place = 0;
-    for (int f = 1; next_placement(p, seq, f); f = 0) cx.n_place++;
-    for (int mi = 0; mi < p->n_M && !cx.err; ++mi) {
-        if (p->M_list[mi] % N != 0) continue;
-        for (int tp = 0; tp < p->tab.n_tp && !cx.err; ++tp) {
-            uint64_t pr = 0;
-            for (int f = 1; next_placement(p, seq, f) && !cx.err; f = 0, ++pr) {
-                cx.m_idx = mi;
-                cx.tp_idx = tp;
-                cx.M = p->M_list[mi];
-                cx.D = p->dp_list[tp];
-                cx.place_rank = pr;
-                for (int s = 0; s < N; ++s) {
-                    cx.types[s] = seq[s];
-                    cx.cls[s] = seq[s] * p->tab.n_tp + tp;
-                    cx.wsum[s] = 0;
-                    cx.work[s] = 0;
-                }
-                il_dfs(&cx, 0, 0);
-            }
+    uint64_t n_slices = 0;
+    orc_slice *slices = list_slices(p, N, &n_slices);
+    if (!slices) return -1;
+    for (uint64_t i = 0; i < n_slices && !cx.err; ++i) {
+        const orc_slice *sl = &slices[i];
+        if (sl->M % N != 0) continue;  /* no interleaved schedule; its indices still count */
+        cx.m_idx = sl->m_idx;
+        cx.tp_idx = p->placement == 2 ? -1 : sl->grp;
+        cx.d_idx = p->placement == 2 ? sl->grp : -1;
+        cx.M = sl->M;
+        cx.D = sl->D;
+        cx.place_rank = sl->place_rank;
+        cx.ordinal = sl->ordinal;
+        for (int s = 0; s < N; ++s) {
+            cx.types[s] = sl->types[s];
+            cx.tps[s] = sl->tps[s];
+            cx.cls[s] = sl->cls[s];
+            cx.wsum[s] = 0;
+            cx.work[s] = 0;
         }
+        il_dfs(&cx, 0, 0);
     }
+    free(slices);
     return cx.err ? -1 : 0;
 }
-

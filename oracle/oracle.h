@@ -68,11 +68,21 @@ typedef struct {
     int32_t n_M;
     const int32_t *M_list;      /* [n_M] ascending */
     const int32_t *dp_list;     /* [n_tp] data-parallel degree D per TP index */
-    int32_t placement;          /* 0 = any type per stage, 1 = exact per-type stage counts */
-    const int32_t *type_counts; /* [n_types] (placement 1) */
+    int32_t placement;          /* 0 = any type per stage, 1 = exact per-type stage counts,
+                                   2 = a (type, TP index) per stage using exactly the
+                                   devices of each type (per-stage TP, see below) */
+    const int32_t *type_counts; /* [n_types] stages per type (placement 1), devices per
+                                   type (placement 2) */
     int32_t ridge;              /* 1: layer-level pruning (Theorem 2): only plans whose
                                    layer counts over the stages of each device type
-                                   rise, then fall ("ridge-like") */
+                                   rise, then fall ("ridge-like"); placements 0 and 1 */
+    /* placement 2 only: slices are (M, D, class sequence k_1..k_S) with
+     * k = type * n_tp + tp_idx chosen per stage, allowed when for every type
+     * sum over its stages of D * tp_list[tp_idx] == type_counts[type]; the
+     * class sequences of one D in lexicographic order. */
+    const int32_t *tp_list;     /* [n_tp] TP degree of each TP index */
+    int32_t n_D;                /* data-parallel degrees tried */
+    const int32_t *D_list;      /* [n_D] */
 } orc_problem;
 
 typedef struct {
@@ -81,6 +91,8 @@ typedef struct {
     int32_t T;                  /* makespan (us) */
     uint64_t place_rank, map_rank, global_index;
     int32_t types[ORC_MAX_S], layers[ORC_MAX_S];
+    int32_t tps[ORC_MAX_S];     /* TP index of each stage (device, interleaved) */
+    int32_t d_idx;              /* placement 2: index into D_list (tp_idx is -1) */
 } orc_plan;
 
 typedef struct {
@@ -154,6 +166,11 @@ int orc_eval_batch_ex(const orc_tables *t, const orc_candidate_ex *c, int64_t n,
 /* Exact search of Sec. 4.2.3.  prune=0 disables the g(S_x) prune (memory
  * infeasible prefixes are still skipped).  warmup = number of random feasible
  * samples evaluated first (Sec. 4.2.3); it never changes the result.
+ * Slice order and global index: placements 0 and 1 take (m_idx, tp_idx,
+ * type sequence), ordinal (m_idx * n_tp + tp_idx) * n_place + place_rank;
+ * placement 2 takes (m_idx, d_idx, class sequence), ordinal
+ * m_idx * P + (sequences of D_list[0..d_idx-1]) + place_rank, P = the
+ * sequences of all D; global index = ordinal * C(L-1, S-1) + map_rank.
  * Returns 0 (plan->found tells whether a feasible plan exists) or -1. */
 int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_plan *plan,
                orc_stats *stats);

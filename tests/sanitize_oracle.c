@@ -132,6 +132,17 @@ int main(void) {
         orc_plan plan;
         orc_stats ss;
         if (orc_search(&p, 1, 20, (uint64_t)iter, &plan, &ss) < -1) return 10;
+        /* per-stage TP: a (type, TP index) per stage under per-type device counts */
+        int32_t tps[4] = {1, 2, 4, 8}, Ds[2] = {1, 2}, devs[2] = {uniform(0, 6), uniform(1, 6)};
+        p.placement = 2;
+        p.ridge = 0;
+        p.tp_list = tps;
+        p.n_D = 2;
+        p.D_list = Ds;
+        p.type_counts = devs;
+        if (orc_search(&p, 1, 20, (uint64_t)iter, &plan, &ss) < -1) return 12;
+        p.placement = 0;
+        p.type_counts = counts;
         p.S = N;
         p.ridge = 0;
         p.tab.schedule = 2;
