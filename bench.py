@@ -157,6 +157,67 @@ def oracle_all_cores_rate(seconds: float):
     return sum(r[0] for r in res), n, sum(r[1] for r in res)
 
 
+def _oracle_search_part(args):
+    cfg, part, n_parts = args
+    import oracle
+    w = gen.get_config(cfg)
+    plan, st = oracle.search(w, prune=True, warmup=500, seed=0, part=part, n_parts=n_parts)
+    return plan, st["leaves_evaluated"] + st["warmup_evaluated"]
+
+
+def oracle_time_to_plan(configs_procs):
+    """The CPU oracle's search (Eq. 2 prune as printed, 500 warm-up samples,
+    the paper's method) on each (config, processes): the slices are dealt
+    round-robin to `processes` spawned single-threaded oracle processes
+    (orc_search_part), the best plan of the parts by (T/(D*M), global index)
+    is the result; wall time from the first part's start to the last part's
+    end (the process pool is started before the clock)."""
+    import multiprocessing as mp
+    from fractions import Fraction
+    n_max = max(n for _, n in configs_procs)
+    out = []
+    with mp.get_context("spawn").Pool(n_max) as pool:
+        pool.map(_oracle_worker, [(0.01, i) for i in range(n_max)])  # workers up, oracle loaded
+        for cfg, n in configs_procs:
+            t0 = time.perf_counter()
+            res = pool.map(_oracle_search_part, [(cfg, i, n) for i in range(n)])
+            wall = time.perf_counter() - t0
+            best = None
+            for plan, _ in res:
+                if plan["found"]:
+                    key = (Fraction(plan["T"], plan["D"] * plan["M"]), plan["global_index"])
+                    if best is None or key < best[0]:
+                        best = (key, plan)
+            out.append({"config": cfg, "seconds": round(wall, 3), "processes": n,
+                        "evaluations": sum(e for _, e in res),
+                        "T_us": best[1]["T"] if best else None,
+                        "global_index": best[1]["global_index"] if best else None})
+    return out
+
+
+def _oracle_eval_chunk(args):
+    lo, hi = args
+    import oracle
+    w = gen.config5_tables()
+    tab = oracle.OracleTables.from_workload(w)
+    c = gen.config5_candidates(hi, seed=0)[lo:hi]
+    t0 = time.perf_counter()
+    oracle.eval_batch(tab, c)
+    return hi - lo, time.perf_counter() - t0
+
+
+def oracle_config5_rate(n, procs):
+    """The CPU oracle evaluating the first n candidates of the config-5 batch
+    (L=64, S~U{2..16}, M~U{8..128}), split into `procs` spawned
+    single-threaded processes; evals/s = n / the slowest process's time."""
+    import multiprocessing as mp
+    step = (n + procs - 1) // procs
+    with mp.get_context("spawn").Pool(procs) as pool:
+        res = pool.map(_oracle_eval_chunk, [(i * step, min(n, (i + 1) * step))
+                                            for i in range(procs) if i * step < n])
+    return n / max(t for _, t in res), max(t for _, t in res)
+
+
 def eval_throughput(P, torch, n, reps, peak_alu, schedule=0, space=None):
     """poseidon_eval_batch on n config-5 candidates (L=64, S ~ U{2..16},
     M ~ U{8..128}, 2 device types), device-resident, timed with CUDA events
@@ -441,6 +502,48 @@ def run_ours(args, rank, world, local_rank):
                     "time_to_plan_s": sum(e_ms) / len(e_ms) / 1e3,
                     "evaluations_per_step": e_ev / len(e_ms), "T_us": plan_e["T"],
                     "matches_oracle": e_ok}
+    # the search with a TP degree chosen per stage (POS_PLACE_DEVICES): config
+    # 4's tables and cluster, D in {2, 4, 8, 16}, each type's devices used up
+    def timed_search(wl, ref_plan, **kw):
+        pr, kp = P.make_problem(wl, warmup=WARMUP_SAMPLES, seed=0,
+                                frontier_cap=args.frontier_cap, **kw)
+        P.poseidon_search(pr)
+        ms, ok, st_sum = [], True, 0
+        for _ in range(max(3, min(100, args.steps // 2))):
+            flush.zero_()
+            torch.cuda.synchronize()
+            ev0.record()
+            pl, st_ = P.poseidon_search(pr)
+            ev1.record()
+            torch.cuda.synchronize()
+            ms.append(ev0.elapsed_time(ev1))
+            st_sum += st_["evaluated"]
+            ok &= ref_plan is not None and all(pl[k] == ref_plan.get(k) for k in
+                                               ("global_index", "T", "layers"))
+        return pl, st_, sum(ms) / len(ms), st_sum / len(ms), ok
+
+    stored = _json.load(open(os.path.join(ROOT, "tests", "golden", "search_plans.json")))
+    w_ps = gen.config4_per_stage_tp()
+    ref_ps = stored.get("config4_per_stage_tp", {}).get("plan")
+    pl_ps, st_ps, ms_ps, ev_ps, ok_ps = timed_search(w_ps, ref_ps, prune=args.prune)
+    per_stage_tp = {"workload": w_ps.name, "prune": PRUNE_NAMES[args.prune],
+                    "time_to_plan_s": ms_ps / 1e3, "evaluations_per_step": ev_ps,
+                    "slices": st_ps["slices"], "slices_feasible": st_ps["slices_feasible"],
+                    "plan": {"T_us": pl_ps["T"], "D": pl_ps["D"], "tp_per_stage":
+                             [w_ps.tp_list[i] for i in pl_ps["tps"]], "types": pl_ps["types"],
+                             "layers": pl_ps["layers"]},
+                    "matches_oracle": ok_ps}
+    # the search over Interleaved 1F1B plans (config 2 tables, V = 2 and 3
+    # chunks per device), against the oracle's stored plans
+    il_lines = []
+    for V in (2, 3):
+        ref_il = stored.get(f"config2_il_v{V}", {}).get("plan")
+        pl_il, st_il, ms_il, ev_il, ok_il = timed_search(gen.config2(), ref_il,
+                                                          prune=args.prune, schedule=2, V=V)
+        il_lines.append({"workload": "config 2 (L=32, S=4, M in {8,16,32}), V = %d" % V,
+                         "prune": PRUNE_NAMES[args.prune], "time_to_plan_s": ms_il / 1e3,
+                         "evaluations_per_step": ev_il, "T_us": pl_il["T"],
+                         "matches_oracle": ok_il})
     # the other stage-level prune, same workload, for comparison (not the headline)
     other = PRUNE_NAMES[1 if args.prune == 2 else 2]
     other_mode = 1 if args.prune == 2 else 2
@@ -496,6 +599,28 @@ def run_ours(args, rank, world, local_rank):
                                    "achieved": round(ach3, 3), "unit": "Tops/s",
                                    "frac": round(ach3 / peak_alu, 4)}}
     cpu_rate, cpu_n, cpu_t = oracle_sample_rate(args.cpu_seconds)
+    # the oracle's time to the plan on this host: configs 1-3 on one core,
+    # config 4 on every core (slices dealt round-robin), beside the GPU's
+    cpu_ttp = None
+    if args.cpu_time_to_plan:
+        procs = max(1, os.cpu_count() or 1)
+        gpu_plans = {4: (plans[-1]["T"], plans[-1]["global_index"], t_dev / args.steps / 1e3)}
+        gpu_plans[3] = (plan3["T"], plan3["global_index"], sum(c3_ms) / len(c3_ms) / 1e3)
+        cpu_ttp = oracle_time_to_plan([(1, 1), (2, 1), (3, 1), (4, procs)])
+        for e in cpu_ttp:
+            ref_c = _json.load(open(os.path.join(ROOT, "tests", "golden",
+                                                 "search_plans.json")))[f"config{e['config']}"]
+            e["matches_stored_oracle_plan"] = (e["T_us"] == ref_c["plan"]["T"] and
+                                               e["global_index"] == ref_c["plan"]["global_index"])
+            if e["config"] in gpu_plans:
+                T, gi, sec = gpu_plans[e["config"]]
+                e["gpu_time_to_plan_s"] = sec
+                e["gpu_prune"] = PRUNE_NAMES[args.prune] if e["config"] == 4 else "none"
+                e["same_plan_as_gpu"] = e["T_us"] == T and e["global_index"] == gi
+        c5_rate, c5_t = oracle_config5_rate(int(args.cpu_config5), procs)
+        cpu_ttp.append({"config": 5, "evals_per_s": c5_rate, "processes": procs,
+                        "sample": f"first {int(args.cpu_config5)} config-5 candidates",
+                        "seconds": round(c5_t, 3)})
     cpu_all = None
     if args.cpu_seconds >= 1.0:
         rate_all, procs, n_all = oracle_all_cores_rate(min(5.0, args.cpu_seconds))
@@ -534,10 +659,13 @@ def run_ours(args, rank, world, local_rank):
         "eager_search": eager_search,
         "config3_exhaustive": exhaustive3,
         "ridge_search": ridge_lines,
+        "per_stage_tp_search": per_stage_tp,
+        "interleaved_search": il_lines,
         "cpu_baseline": {"value": cpu_rate, "unit": "evals/s", "cores": 1, "kind": "oracle",
                          "sample": f"{cpu_n} config-4 plan evaluations (S=8, M=32, L=80) in "
                                    f"{cpu_t:.1f} s, single-threaded oracle"},
         "cpu_baseline_all_cores": cpu_all,
+        "cpu_time_to_plan": cpu_ttp,
         "e2e": {"value": e2e, "unit": "evals/s", "h2d_bytes_per_step": int(tab_bytes),
                 "d2h_bytes_per_step": int(P.binding.C.sizeof(P.binding.pos_plan))},
         "gpu_launches": int(agg["launches"]),
@@ -556,6 +684,10 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--cpu-time-to-plan", type=int, choices=[0, 1], default=1,
+                    help="time the oracle's search on configs 1-4 on this host's cores")
+    ap.add_argument("--cpu-config5", type=float, default=1e6,
+                    help="config-5 candidates the oracle evaluates on all cores")
     ap.add_argument("--backend", choices=["nccl", "gloo"], default="nccl")
     ap.add_argument("--eval-sizes", type=float, nargs="*", default=[1e7],
                     help="config-5 batch sizes for the evaluator measurement")

@@ -6,6 +6,7 @@ no lower bound, no search.
 """
 from .workloads import (  # noqa: F401
     CANDIDATE_DTYPE, CANDIDATE_EX_DTYPE, Workload, config1, config2, config3, config4,
+    config4_per_stage_tp,
     config5_tables, config5_candidates, all_candidates, random_candidates,
     interleaved_candidates, per_stage_tp_candidates, search_space_sample, get_config,
     n_compositions, place_list,

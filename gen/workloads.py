@@ -205,6 +205,16 @@ def config4(seed: int = 0) -> Workload:
     return w
 
 
+def config4_per_stage_tp(seed: int = 0) -> Workload:
+    """Config 4's tables and cluster with a TP degree chosen per stage:
+    D in {2, 4, 8, 16}, and the stages of each type use exactly its devices
+    (32/32/64): sum over its stages of D * t = devices (PLACE_DEVICES)."""
+    w = config4(seed)
+    w.name = "70B-like L=80 S=8 M=32 (3 types, per-stage t in {1,2,4,8}, D in {2,4,8,16})"
+    w.placement, w.type_counts, w.D_list = PLACE_DEVICES, [32, 32, 64], [2, 4, 8, 16]
+    return w
+
+
 def config5_tables(seed: int = 0) -> Workload:
     """Evaluator sweep tables: L=64, 7B-like costs (h=4096), 2 types, t=1."""
     rng = np.random.default_rng(seed)

@@ -69,6 +69,9 @@ typedef int32_t pos_status;
 
 #define POS_PLACE_FREE 0    /* any device type on any stage */
 #define POS_PLACE_EXACT 1   /* exactly type_counts[t] stages of type t */
+#define POS_PLACE_DEVICES 2 /* a (device type, TP index) per stage; the stages of
+                               type t use exactly type_counts[t] devices: the sum
+                               over them of D * tp_list[tp index] (per-stage TP) */
 
 #define POS_MAX_STAGES 16
 #define POS_MAX_LAYERS 127
@@ -248,6 +251,17 @@ pos_status poseidon_argmin_noalloc(const int32_t *d_makespan, const uint8_t *d_f
  * plan = (((m_idx*n_tp + tp_idx)*n_place + place_rank)*n_map + map_rank),
  * n_map = C(L-1, S-1).  Objective: time per sample T/(D*M), compared exactly;
  * ties go to the lowest global index.
+ * POS_PLACE_DEVICES (per-stage TP, as in the mixed-TP plans of the paper's
+ * Table 1): slices are (m_idx, d_idx, class sequence), the classes
+ * k_s = type_s * n_tp + tp_s of the S stages chosen freely among those whose
+ * stages of every type t use exactly type_counts[t] devices (sum of
+ * D_list[d_idx] * tp_list[tp_s]); the sequences of one D in lexicographic
+ * order of (k_1, ..., k_S); slice ordinal = m_idx * P + (sequences of
+ * D_list[0..d_idx-1]) + place_rank, P = the sequences of every D; global
+ * index = ordinal * n_map + map_rank.  The tables must hold every class's
+ * costs for each D tried; ridge pruning is not available (POS_EINVAL);
+ * under POS_SCHED_INTERLEAVED_1F1B the sequence is over the S devices and
+ * needs n_tp <= 4 (POS_EINVAL).
  */
 /* Stage-level pruning (Sec. 4.2.1).  Every mode returns the same plan.
  *   POS_PRUNE_NONE   exhaustive enumeration (memory cut only).
@@ -301,15 +315,19 @@ typedef struct pos_problem {
                                    the search gives up with POS_ETIMEOUT: 0 = default
                                    (2^20); < 0 = no round, so every update that would
                                    lower the incumbent gives up (tests the time-out path) */
+    int32_t n_D;                /* POS_PLACE_DEVICES: data-parallel degrees tried */
+    const int32_t *D_list;      /* [n_D] (>= 1); dp_list is not read there */
 } pos_problem;
 
 typedef struct pos_plan {
     int32_t found;
-    int32_t m_idx, tp_idx, M, tp, D, S;
+    int32_t m_idx, tp_idx, M, tp, D, S;  /* tp_idx, tp: -1 under POS_PLACE_DEVICES */
     int32_t makespan;           /* T in us */
-    int32_t type[POS_MAX_STAGES];
-    int32_t layers[POS_MAX_STAGES];
+    int32_t type[POS_MAX_STAGES];    /* device type per stage (per device, interleaved) */
+    int32_t layers[POS_MAX_STAGES];  /* layers per stage (per virtual stage, interleaved) */
     uint64_t place_rank, map_rank, global_index;
+    int32_t tp_stage[POS_MAX_STAGES];  /* TP index per stage (per device); -1 past S */
+    int32_t d_idx;              /* POS_PLACE_DEVICES: index of D in D_list; else -1 */
 } pos_plan;
 
 typedef struct pos_search_stats {
@@ -365,9 +383,11 @@ typedef struct pos_search_stats {
  * POS_ECUDA, POS_ETIMEOUT, POS_EINFEASIBLE (no memory-feasible plan; *out
  * has found = 0).
  * Limits (checked on the host before the device is touched; POS_EINVAL):
- * at most 2^22 slices (M values x TP indices x placements) and 2^22
- * placements; the global index (slices x compositions) must fit in 64
- * bits; the lcm of all D*M must be below 2^32.  Memory-feasible slices are
+ * at most 2^22 slices (M values x TP indices x placements; M values x
+ * class sequences of every D under POS_PLACE_DEVICES) and 2^22 placements;
+ * under POS_PLACE_DEVICES at most 65536 devices per type; the global index
+ * (slices x compositions) must fit in 64 bits; the lcm of all D*M must be
+ * below 2^32.  Memory-feasible slices are
  * enumerated in batches of at most 65535 slices, one after another.
  * Memory: the work buffers (one frontier of frontier_cap 32-byte entries per
  * depth, a leaf buffer of the same length, slice and feasibility tables,

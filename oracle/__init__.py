@@ -116,6 +116,9 @@ def lib():
         L.orc_search.restype = C.c_int
         L.orc_search.argtypes = [C.POINTER(Problem), C.c_int, C.c_int, C.c_uint64,
                                  C.POINTER(Plan), C.POINTER(Stats)]
+        L.orc_search_part.restype = C.c_int
+        L.orc_search_part.argtypes = [C.POINTER(Problem), C.c_int, C.c_int, C.c_uint64,
+                                      C.c_int, C.c_int, C.POINTER(Plan), C.POINTER(Stats)]
         _lib = L
     return _lib
 
@@ -289,13 +292,15 @@ def _plan_dict(plan, n_units, n_layers):
 
 
 def search(w, prune=True, warmup=0, seed=0, tab: OracleTables | None = None,
-           schedule=SCHED_1F1B, ridge=False):
-    """Exact search over a gen.Workload search problem.  Returns (plan dict, stats dict)."""
+           schedule=SCHED_1F1B, ridge=False, part=0, n_parts=1):
+    """Exact search over a gen.Workload search problem.  Returns (plan dict, stats dict).
+    With n_parts > 1 only the slices whose global-order index is part
+    (mod n_parts) are searched (orc_search_part)."""
     tab = tab or OracleTables.from_workload(w, schedule)
     p, keep = _problem(w, tab, ridge)
     plan, st = Plan(), Stats()
-    rc = lib().orc_search(C.byref(p), int(prune), int(warmup), C.c_uint64(seed), C.byref(plan),
-                          C.byref(st))
+    rc = lib().orc_search_part(C.byref(p), int(prune), int(warmup), C.c_uint64(seed), int(part),
+                               int(n_parts), C.byref(plan), C.byref(st))
     if rc == -2:
         raise OverflowError("overflow guard")
     if rc:

@@ -1090,7 +1090,13 @@ static void set_slice(search_ctx *cx, const orc_slice *sl) {
 
 int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_plan *plan,
                orc_stats *stats) {
+    return orc_search_part(p, prune, warmup, seed, 0, 1, plan, stats);
+}
+
+int orc_search_part(const orc_problem *p, int prune, int warmup, uint64_t seed, int part,
+                    int n_parts, orc_plan *plan, orc_stats *stats) {
     int S = p->S, L = p->tab.L;
+    if (n_parts < 1 || part < 0 || part >= n_parts) return -1;
     if (S < 1 || S > ORC_MAX_S || S > L || L > 127 || p->n_M < 1 || p->tab.n_types < 1 ||
         p->tab.n_types > 4 || p->tab.n_tp < 1 || !tables_nonnegative(&p->tab) ||
         !slice_space_valid(p))
@@ -1125,7 +1131,14 @@ int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_p
     if (warmup > 0 && n_slices > 0) {
         uint64_t rs = seed;
         for (int w = 0; w < warmup; ++w) {
-            set_slice(&cx, &slices[splitmix64(&rs) % n_slices]);
+            uint64_t pick = splitmix64(&rs) % n_slices;
+            if (n_parts > 1) {  /* a slice of this part */
+                uint64_t in_part = (uint64_t)part < n_slices
+                                       ? (n_slices - (uint64_t)part + n_parts - 1) / n_parts : 0;
+                if (in_part == 0) break;
+                pick = (pick % in_part) * n_parts + part;
+            }
+            set_slice(&cx, &slices[pick]);
             if (!cx.feas[0]) continue;
             int used = 0;
             for (int x = 0; x < S; ++x) {
@@ -1145,7 +1158,7 @@ int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_p
     }
 
     /* exhaustive enumeration in global-index order with the two cuts */
-    for (uint64_t i = 0; i < n_slices && !cx.err; ++i) {
+    for (uint64_t i = (uint64_t)part; i < n_slices && !cx.err; i += (uint64_t)n_parts) {
         set_slice(&cx, &slices[i]);
         if (!cx.feas[0]) continue;
         dfs(&cx, 0, 0);

@@ -174,6 +174,12 @@ int orc_eval_batch_ex(const orc_tables *t, const orc_candidate_ex *c, int64_t n,
  * Returns 0 (plan->found tells whether a feasible plan exists) or -1. */
 int orc_search(const orc_problem *p, int prune, int warmup, uint64_t seed, orc_plan *plan,
                orc_stats *stats);
+/* orc_search over the slices whose index in the global order is
+ * part (mod n_parts) only (warm-up samples too): a driver that runs the
+ * parts in separate processes and keeps the best plan by (T/(D*M), global
+ * index) obtains orc_search's plan. */
+int orc_search_part(const orc_problem *p, int prune, int warmup, uint64_t seed, int part,
+                    int n_parts, orc_plan *plan, orc_stats *stats);
 
 /* Search over Interleaved 1F1B plans with V chunks per device: the slices
  * of orc_search over the N = p->S devices (M values that are not multiples

@@ -22,7 +22,7 @@ STATUS_NAMES = ["POS_OK", "POS_EINVAL", "POS_EOVERFLOW", "POS_ENOMEM", "POS_ECUD
 POS_SCHED_1F1B = 0
 POS_SCHED_EAGER_1F1B = 1
 POS_SCHED_INTERLEAVED_1F1B = 2
-POS_PLACE_FREE, POS_PLACE_EXACT = 0, 1
+POS_PLACE_FREE, POS_PLACE_EXACT, POS_PLACE_DEVICES = 0, 1, 2
 MAX_STAGES = 16
 
 # the exported entry points, as declared in include/poseidon.h
@@ -44,7 +44,8 @@ class pos_problem(C.Structure):
                 ("placement", C.c_int32), ("type_counts", C.c_void_p), ("warmup", C.c_int32),
                 ("prune", C.c_int32), ("seed", C.c_uint64), ("schedule", C.c_int32),
                 ("frontier_cap", C.c_int64), ("profile", C.c_int32), ("ridge", C.c_int32),
-                ("V", C.c_int32), ("cas_limit", C.c_int32)]
+                ("V", C.c_int32), ("cas_limit", C.c_int32), ("n_D", C.c_int32),
+                ("D_list", C.c_void_p)]
 
 
 class pos_plan(C.Structure):
@@ -52,7 +53,8 @@ class pos_plan(C.Structure):
                 ("M", C.c_int32), ("tp", C.c_int32), ("D", C.c_int32), ("S", C.c_int32),
                 ("makespan", C.c_int32), ("type", C.c_int32 * MAX_STAGES),
                 ("layers", C.c_int32 * MAX_STAGES), ("place_rank", C.c_uint64),
-                ("map_rank", C.c_uint64), ("global_index", C.c_uint64)]
+                ("map_rank", C.c_uint64), ("global_index", C.c_uint64),
+                ("tp_stage", C.c_int32 * MAX_STAGES), ("d_idx", C.c_int32)]
 
 
 class pos_search_stats(C.Structure):
@@ -232,10 +234,13 @@ def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0, profile=Fals
         keep.append(a)
         return a.ctypes.data
 
-    p = pos_problem(tab.c, w.S, len(w.M_list), arr(w.M_list), arr(w.tp_list), arr(w.dp_list),
+    D_list = list(getattr(w, "D_list", None) or [])
+    p = pos_problem(tab.c, w.S, len(w.M_list), arr(w.M_list), arr(w.tp_list),
+                    arr(w.dp_list if w.dp_list else [1] * w.n_tp),
                     w.placement, arr(w.type_counts if w.type_counts else [0] * w.n_types),
                     int(warmup), _prune_mode(prune), int(seed), int(schedule), int(frontier_cap),
-                    int(bool(profile)), int(bool(ridge)), int(V), int(cas_limit))
+                    int(bool(profile)), int(bool(ridge)), int(V), int(cas_limit), len(D_list),
+                    arr(D_list if D_list else [1]))
     return p, keep
 
 
@@ -247,9 +252,10 @@ def poseidon_search(problem: pos_problem):
     S = problem.S
     J = S * problem.V if problem.schedule == POS_SCHED_INTERLEAVED_1F1B else S
     out = dict(found=bool(plan.found), m_idx=plan.m_idx, tp_idx=plan.tp_idx, M=plan.M,
-               tp=plan.tp, D=plan.D, T=plan.makespan, place_rank=plan.place_rank,
-               map_rank=plan.map_rank, global_index=plan.global_index,
-               types=list(plan.type)[:S], layers=list(plan.layers)[:J])
+               tp=plan.tp, D=plan.D, d_idx=plan.d_idx, T=plan.makespan,
+               place_rank=plan.place_rank, map_rank=plan.map_rank,
+               global_index=plan.global_index, types=list(plan.type)[:S],
+               tps=list(plan.tp_stage)[:S], layers=list(plan.layers)[:J])
     stats = {n: (list(getattr(st, n)) if n.endswith("_depth") else getattr(st, n))
              for n, _ in pos_search_stats._fields_}
     return out, stats

@@ -28,6 +28,38 @@ pos_status ensure_smem(const void *kernel, int smem);
 // query costs host time on every launch otherwise).
 pos_status blocks_per_sm(const void *kernel, int threads, int smem, int *out);
 
+// Programmatic dependent launch (sm_90 and later).  A kernel launched by
+// launch_dependent may be scheduled while the kernel queued before it on
+// the stream is still running; before it reads anything that kernel wrote
+// it executes grid_dep_wait(), which returns once that grid has completed
+// and its memory is visible.  It then calls grid_dep_trigger(), which lets
+// the next such kernel be scheduled: a kernel's pre-wait part can therefore
+// only overlap the post-wait part of its predecessor, so it may read
+// whatever was written two or more kernels earlier (the cost tables, slice
+// records and bound tables of a search).  Without the launch attribute the
+// two instructions do nothing.
+__device__ __forceinline__ void grid_dep_wait() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+__device__ __forceinline__ void grid_dep_trigger() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_dependent(void (*kern)(KArgs...), int grid, int block, int smem,
+                                    cudaStream_t stream, Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3((unsigned)block);
+    cfg.dynamicSmemBytes = (size_t)smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
+
 #define POS_CUDA(call)                                           \
     do {                                                         \
         cudaError_t e_ = (call);                                 \

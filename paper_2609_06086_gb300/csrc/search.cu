@@ -682,19 +682,9 @@ __device__ __forceinline__ void level_warp_mode(const ExpandParams &p, const Tab
 template <bool COMPLETE, int X>
 __global__ void __launch_bounds__(kThreads, 3) level_kernel(ExpandParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
-    long long n_in = p.n_in;
-    if (p.n_in_dev) {
-        const unsigned long long c0 = __ldcg(p.n_in_dev);
-        n_in = (long long)(c0 < p.cap ? c0 : p.cap);
-    }
-    const long long n_work = p.groups ? p.n_groups : (n_in + 31) / 32;
-    const long long n_warps = ((long long)gridDim.x * blockDim.x) >> 5;
-    // small frontier in the pipelined pass: one warp per parent
-    const bool warp_mode = !p.exact && !p.groups && n_in <= n_warps;
-    // blocks without work leave before staging anything
-    if ((long long)blockIdx.x * (kThreads / 32) >= (warp_mode ? n_in : n_work)) return;
     // timing tables and, when expanding under prune mode 2, the
-    // completion-bound rows of depth X+1 of every slot (contiguous), by TMA
+    // completion-bound rows of depth X+1 of every slot (contiguous), by TMA;
+    // all written before the previous kernel, so staged while it finishes
     __shared__ uint64_t bar;
     const bool use_v = !COMPLETE && p.prune == 2;
     const bool stage_v = use_v && p.vb_smem;
@@ -716,6 +706,20 @@ __global__ void __launch_bounds__(kThreads, 3) level_kernel(ExpandParams p) {
         if (threadIdx.x == 0) atomicAdd(p.stats + kStBulkTimeout, 1ull);
         return;
     }
+    // the frontier, its count and the incumbent only after the previous
+    // kernel has completed
+    grid_dep_wait();
+    grid_dep_trigger();
+    long long n_in = p.n_in;
+    if (p.n_in_dev) {
+        const unsigned long long c0 = __ldcg(p.n_in_dev);
+        n_in = (long long)(c0 < p.cap ? c0 : p.cap);
+    }
+    const long long n_work = p.groups ? p.n_groups : (n_in + 31) / 32;
+    const long long n_warps = ((long long)gridDim.x * blockDim.x) >> 5;
+    // small frontier in the pipelined pass: one warp per parent
+    const bool warp_mode = !p.exact && !p.groups && n_in <= n_warps;
+    if ((long long)blockIdx.x * (kThreads / 32) >= (warp_mode ? n_in : n_work)) return;
     const int2 *vsm = stage_v ? reinterpret_cast<const int2 *>(sm + p.lay.bytes) : nullptr;
     const Tab t = tab_at(sm, p.lay);
     const uint64_t thr = p.prune ? __ldcg(&p.inc->obj) : ~0ull;
@@ -884,10 +888,10 @@ struct Search {
     cudaStream_t stream;
     cudaEvent_t (&ev)[3];
     int S = 0, L = 0, n_tp = 0;
-    uint64_t n_map = 0, n_place = 0;
+    uint64_t n_map = 0;
     long long cap = 0;
-    int grid_level = 0, grid_leaf = 0;
-    std::vector<uint8_t> places;  // n_place x S stage types, placement-rank order
+    int grid_level = 0;
+    const SliceSpace *sp = nullptr;  // the slices' identities, global-index order
     std::vector<SliceRec> slices;
     DevBuf &d_slices, &d_feas, &d_batch, &d_inc, &d_ctr, &d_best, &d_feasible, &d_leaves,
         &d_roots, &d_root;
@@ -919,11 +923,29 @@ static pos_status validate_problem(const pos_problem *p) {
     if (p->n_M < 1 || !p->M_list) return fail(POS_EINVAL, "empty M_list");
     for (int i = 0; i < p->n_M; ++i)
         if (p->M_list[i] < 1 || p->M_list[i] > 255) return fail(POS_EINVAL, "M out of 1..255");
-    if (!p->dp_list || !p->tp_list) return fail(POS_EINVAL, "tp_list/dp_list is NULL");
-    for (int i = 0; i < p->tables.n_tp; ++i)
-        if (p->dp_list[i] < 1) return fail(POS_EINVAL, "D must be >= 1");
-    if (p->placement != POS_PLACE_FREE && p->placement != POS_PLACE_EXACT)
+    if (!p->tp_list) return fail(POS_EINVAL, "tp_list is NULL");
+    if (p->placement != POS_PLACE_FREE && p->placement != POS_PLACE_EXACT &&
+        p->placement != POS_PLACE_DEVICES)
         return fail(POS_EINVAL, "unknown placement rule");
+    if (p->placement == POS_PLACE_DEVICES) {
+        if (!p->D_list || p->n_D < 1) return fail(POS_EINVAL, "D_list is empty");
+        for (int i = 0; i < p->n_D; ++i)
+            if (p->D_list[i] < 1) return fail(POS_EINVAL, "D must be >= 1");
+        for (int i = 0; i < p->tables.n_tp; ++i)
+            if (p->tp_list[i] < 1) return fail(POS_EINVAL, "TP degrees must be >= 1");
+        if (!p->type_counts) return fail(POS_EINVAL, "type_counts is NULL");
+        for (int i = 0; i < p->tables.n_types; ++i)
+            if (p->type_counts[i] < 0 || p->type_counts[i] > 65536)
+                return fail(POS_EINVAL, "device counts must be in 0..65536");
+        if (p->ridge)
+            return fail(POS_EINVAL, "layer-level (ridge) pruning is not defined for per-stage TP");
+        if (p->schedule == POS_SCHED_INTERLEAVED_1F1B && p->tables.n_tp > 4)
+            return fail(POS_EINVAL, "Interleaved 1F1B with a TP index per device needs n_tp <= 4");
+    } else {
+        if (!p->dp_list) return fail(POS_EINVAL, "dp_list is NULL");
+        for (int i = 0; i < p->tables.n_tp; ++i)
+            if (p->dp_list[i] < 1) return fail(POS_EINVAL, "D must be >= 1");
+    }
     if (p->placement == POS_PLACE_EXACT) {
         if (!p->type_counts) return fail(POS_EINVAL, "type_counts is NULL");
         int sum = 0;
@@ -942,72 +964,175 @@ static pos_status validate_problem(const pos_problem *p) {
     return POS_OK;
 }
 
-// allowed stage-type sequences in lexicographic order
-static pos_status enumerate_places(Search &s) {
-    const pos_problem *p = s.pb;
-    const int S = p->S, T = p->tables.n_types;
+// POS_PLACE_DEVICES: the class sequences of one D in lexicographic order,
+// by a depth-first walk that keeps only prefixes with a completion: the
+// remaining r stages can use up every type's remaining devices iff there
+// are counts n_t (sum r) such that each remainder, in units of D, is a sum
+// of exactly n_t TP degrees (reach[n][v]).
+static pos_status device_sequences(const pos_problem *p, int units, int D,
+                                   std::vector<uint8_t> &out, uint64_t *total) {
+    const int T = p->tables.n_types, n_tp = p->tables.n_tp, K = T * n_tp;
     const uint64_t limit = 1ull << 22;
-    std::vector<uint8_t> seq;
-    if (p->placement == POS_PLACE_EXACT) {
-        // the distinct permutations of the multiset, in lexicographic order
-        for (int ty = 0; ty < T; ++ty) seq.insert(seq.end(), p->type_counts[ty], (uint8_t)ty);
-        do {
-            s.places.insert(s.places.end(), seq.begin(), seq.end());
-            if (s.places.size() > limit * S) return fail(POS_EINVAL, "too many placements");
-        } while (std::next_permutation(seq.begin(), seq.end()));
-    } else {
-        // every sequence in T^S, as an odometer (last stage fastest)
-        double total = 1;
-        for (int x = 0; x < S; ++x) total *= T;
-        if (total > (double)limit) return fail(POS_EINVAL, "too many placements");
-        seq.assign(S, 0);
-        for (;;) {
-            s.places.insert(s.places.end(), seq.begin(), seq.end());
-            int x = S - 1;
-            while (x >= 0 && seq[x] == T - 1) seq[x--] = 0;
-            if (x < 0) break;
-            seq[x]++;
+    int bud[POS_MAX_TYPES];
+    int vmax = 0;
+    for (int t = 0; t < T; ++t) {
+        if (p->type_counts[t] % D != 0) return POS_OK;  // no stage split uses them up
+        bud[t] = p->type_counts[t] / D;
+        vmax = std::max(vmax, bud[t]);
+    }
+    // reach[n * (vmax + 1) + v]: v is a sum of exactly n TP degrees
+    std::vector<uint8_t> reach((size_t)(units + 1) * (vmax + 1), 0);
+    reach[0] = 1;
+    for (int n = 1; n <= units; ++n)
+        for (int v = 0; v <= vmax; ++v)
+            for (int j = 0; j < n_tp; ++j) {
+                const int d = p->tp_list[j];
+                if (d <= v && reach[(size_t)(n - 1) * (vmax + 1) + v - d]) {
+                    reach[(size_t)n * (vmax + 1) + v] = 1;
+                    break;
+                }
+            }
+    auto completes = [&](int r) {
+        uint32_t mask = 1u;  // bit n: n stages used by the types seen so far
+        for (int t = 0; t < T; ++t) {
+            uint32_t next = 0;
+            for (int n = 0; n <= r; ++n)
+                if (reach[(size_t)n * (vmax + 1) + bud[t]]) next |= mask << n;
+            mask = next & ((2u << r) - 1u);
+        }
+        return (mask >> r) & 1u;
+    };
+    if (!completes(units)) return POS_OK;
+    uint8_t seq[POS_MAX_STAGES];
+    int k_at[POS_MAX_STAGES];
+    int u = 0;
+    k_at[0] = -1;
+    while (u >= 0) {  // iterative depth-first walk, classes in ascending order
+        int k = k_at[u] + 1;
+        if (k_at[u] >= 0) bud[k_at[u] / n_tp] += p->tp_list[k_at[u] % n_tp];  // undo
+        for (; k < K; ++k) {
+            const int t = k / n_tp, d = p->tp_list[k % n_tp];
+            if (bud[t] < d) continue;
+            bud[t] -= d;
+            if (completes(units - u - 1)) break;
+            bud[t] += d;
+        }
+        if (k == K) {  // no further class at this position: back up
+            k_at[u] = -1;
+            --u;
+            continue;
+        }
+        k_at[u] = k;
+        seq[u] = (uint8_t)k;
+        if (u == units - 1) {
+            out.insert(out.end(), seq, seq + units);
+            if (++*total > limit) return fail(POS_EINVAL, "more than 2^22 class sequences");
+        } else {
+            k_at[++u] = -1;
         }
     }
-    s.n_place = s.places.size() / S;
     return POS_OK;
 }
 
-// Size limits of the search space, checked on the host before the device
-// is touched: at most 2^22 placements and 2^22 slices, a global index
-// (slices x compositions) below 2^64 and an objective scale (lcm of every
-// D*M) below 2^32.
-static pos_status validate_space(const pos_problem *p) {
-    const int S = p->S, T = p->tables.n_types, n_tp = p->tables.n_tp;
+pos_status build_slice_space(const pos_problem *p, int units, SliceSpace &sp) {
+    const int T = p->tables.n_types, n_tp = p->tables.n_tp;
     const uint64_t limit = 1ull << 22;
-    uint64_t n_place = 1;
-    if (p->placement == POS_PLACE_EXACT) {
-        // distinct orders of the multiset: S! / prod counts!, by binomials
-        int left = S;
-        for (int ty = 0; ty < T; ++ty) {
-            n_place *= host_binom(left, p->type_counts[ty]);  // <= C(16, 8) each step
-            left -= p->type_counts[ty];
-            if (n_place > limit) return fail(POS_EINVAL, "too many placements (above 2^22)");
+    sp = SliceSpace();
+    sp.units = units;
+    sp.per_stage = p->placement == POS_PLACE_DEVICES;
+    sp.n_grp = sp.per_stage ? p->n_D : n_tp;
+    if (sp.per_stage) {
+        uint64_t total = 0;
+        sp.seqs.resize(p->n_D);
+        for (int g = 0; g < p->n_D; ++g) {
+            POS_TRY(device_sequences(p, units, p->D_list[g], sp.seqs[g], &total));
+            sp.D.push_back(p->D_list[g]);
         }
     } else {
-        for (int x = 0; x < S; ++x) {
-            n_place *= (uint64_t)T;
-            if (n_place > limit) return fail(POS_EINVAL, "too many placements (above 2^22)");
+        sp.seqs.resize(1);
+        std::vector<uint8_t> &places = sp.seqs[0];
+        std::vector<uint8_t> seq;
+        if (p->placement == POS_PLACE_EXACT) {
+            // the distinct permutations of the multiset, in lexicographic order
+            int sum = 0;
+            for (int ty = 0; ty < T; ++ty) sum += p->type_counts[ty];
+            if (sum != units) return fail(POS_EINVAL, "type_counts must sum to S");
+            for (int ty = 0; ty < T; ++ty) seq.insert(seq.end(), p->type_counts[ty], (uint8_t)ty);
+            do {
+                places.insert(places.end(), seq.begin(), seq.end());
+                if (places.size() > limit * units) return fail(POS_EINVAL, "too many placements");
+            } while (std::next_permutation(seq.begin(), seq.end()));
+        } else {
+            // every sequence in T^S, as an odometer (last stage fastest)
+            double total = 1;
+            for (int x = 0; x < units; ++x) total *= T;
+            if (total > (double)limit) return fail(POS_EINVAL, "too many placements");
+            seq.assign(units, 0);
+            for (;;) {
+                places.insert(places.end(), seq.begin(), seq.end());
+                int x = units - 1;
+                while (x >= 0 && seq[x] == T - 1) seq[x--] = 0;
+                if (x < 0) break;
+                seq[x]++;
+            }
         }
+        for (int g = 0; g < n_tp; ++g) sp.D.push_back(p->dp_list[g]);
     }
-    const uint64_t n_slices = (uint64_t)p->n_M * n_tp * n_place;
-    if (n_slices > limit) return fail(POS_EINVAL, "more than 2^22 slices");
+    sp.grp_off.assign(sp.n_grp + 1, 0);
+    for (int g = 0; g < sp.n_grp; ++g) sp.grp_off[g + 1] = sp.grp_off[g] + sp.n_seq(g);
+    sp.per_m = sp.grp_off[sp.n_grp];
+    if ((uint64_t)p->n_M * sp.per_m > limit) return fail(POS_EINVAL, "more than 2^22 slices");
+    return POS_OK;
+}
+
+void plan_slice_fields(const pos_problem *p, const SliceSpace &sp, uint64_t ord, pos_plan *out) {
+    int mi = 0, g = 0;
+    uint64_t pr = 0;
+    sp.decode(ord, &mi, &g, &pr);
+    const int n_tp = p->tables.n_tp;
+    out->m_idx = mi;
+    out->M = p->M_list[mi];
+    out->D = sp.D[g];
+    out->place_rank = pr;
+    out->tp_idx = sp.per_stage ? -1 : g;
+    out->tp = sp.per_stage ? -1 : p->tp_list[g];
+    out->d_idx = sp.per_stage ? g : -1;
+    for (int x = 0; x < POS_MAX_STAGES; ++x) {
+        const int k = x < sp.units ? sp.cls(g, pr, x, n_tp) : -1;
+        out->type[x] = k < 0 ? -1 : k / n_tp;
+        out->tp_stage[x] = k < 0 ? -1 : k % n_tp;
+    }
+}
+
+// Size limits of the search space that do not need the slices, checked on
+// the host before the device is touched: the global index (slices x
+// compositions) below 2^64 and the objective scale (lcm of every D*M) below
+// 2^32.
+static pos_status validate_space(const pos_problem *p, const SliceSpace &sp) {
+    const int S = p->S;
+    const uint64_t n_slices = (uint64_t)p->n_M * sp.per_m;
     const int J = p->schedule == POS_SCHED_INTERLEAVED_1F1B ? S * p->V : S;
     const uint64_t n_map = host_binom(p->tables.L - 1, J - 1);
     if (n_map && n_slices > ~0ull / n_map) return fail(POS_EINVAL, "global index overflows");
     uint64_t Q = 1;
     for (int i = 0; i < p->n_M; ++i)
-        for (int j = 0; j < n_tp; ++j) {
-            const uint64_t dm = (uint64_t)p->dp_list[j] * p->M_list[i];
+        for (int32_t D : sp.D) {
+            const uint64_t dm = (uint64_t)D * p->M_list[i];
             Q = Q / gcd64(Q, dm) * dm;
             if (Q >= (1ull << 32)) return fail(POS_EINVAL, "lcm of D*M reaches 2^32");
         }
     return POS_OK;
+}
+
+// Q = lcm of every D*M: T * Q / (D*M) orders plans by time per sample
+static uint64_t objective_scale(const pos_problem *p, const SliceSpace &sp) {
+    uint64_t Q = 1;
+    for (int i = 0; i < p->n_M; ++i)
+        for (int32_t D : sp.D) {
+            const uint64_t dm = (uint64_t)D * p->M_list[i];
+            Q = Q / gcd64(Q, dm) * dm;
+        }
+    return Q;
 }
 
 static pos_status sync_read(Search &s, void *dst, const void *src, size_t bytes) {
@@ -1110,15 +1235,16 @@ static pos_status run_leaves(Search &s, const Leaf *leaves, unsigned long long *
     lp.pg = s.pg;
     lp.ridge = s.pb->ridge;
     lp.cas_limit = s.pb->cas_limit == 0 ? kCasLimit : std::max(0, s.pb->cas_limit);
-    return launch_leaf(s.S, path_of(s.pb->schedule, s.S, M), lp, s.grid_leaf, s.stream);
+    // as many blocks as the launch bounds keep resident on every SM
+    const int path = path_of(s.pb->schedule, s.S, M);
+    return launch_leaf(s.S, path, lp, leaf_min_blocks(s.S, path) * sm_count(), s.stream);
 }
 
 template <bool COMPLETE, int X>
 static pos_status launch_level_t(const ExpandParams &p, int grid, int smem, cudaStream_t st) {
     auto kern = level_kernel<COMPLETE, X>;
     POS_TRY(ensure_smem(reinterpret_cast<const void *>(kern), smem));
-    kern<<<grid, kThreads, smem, st>>>(p);
-    POS_CUDA(cudaGetLastError());
+    POS_CUDA(launch_dependent(kern, grid, kThreads, smem, st, p));
     return POS_OK;
 }
 
@@ -1238,8 +1364,8 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     // deferral pass makes progress
     s.cap = p->frontier_cap > 0 ? p->frontier_cap : (1ll << 24);
     s.cap = std::max<long long>(s.cap, 32LL * s.L);
-    if ((st = enumerate_places(s)) != POS_OK) return st;
-    const uint64_t n_slices64 = (uint64_t)p->n_M * s.n_tp * s.n_place;
+    const SliceSpace &sp = *s.sp;
+    const uint64_t n_slices64 = (uint64_t)p->n_M * sp.per_m;
     if (n_slices64 > (1ull << 22)) return fail(POS_EINVAL, "more than 2^22 slices");
     const int n_slices = (int)n_slices64;
     if (s.n_map && n_slices64 > ~0ull / s.n_map) return fail(POS_EINVAL, "global index overflows");
@@ -1264,27 +1390,22 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         if (guard_trips(s.h->guard_A, s.h->guard_D, s.h->guard_P, s.S, p->M_list[i]))
             return fail(POS_EOVERFLOW, "makespan bound reaches 2^31 for some M");
     // objective scale: Q = lcm(D*M); T*Q/(D*M) orders plans by time per sample
-    uint64_t Q = 1;
-    for (int i = 0; i < p->n_M; ++i)
-        for (int j = 0; j < s.n_tp; ++j) {
-            const uint64_t dm = (uint64_t)p->dp_list[j] * p->M_list[i];
-            Q = Q / gcd64(Q, dm) * dm;
-            if (Q >= (1ull << 32)) return fail(POS_EINVAL, "lcm of D*M reaches 2^32");
-        }
+    const uint64_t Q = objective_scale(p, sp);
     s.slices.resize(n_slices);
-    for (int mi = 0; mi < p->n_M; ++mi)
-        for (int tp = 0; tp < s.n_tp; ++tp)
-            for (uint64_t pr = 0; pr < s.n_place; ++pr) {
-                const uint64_t ord = ((uint64_t)mi * s.n_tp + tp) * s.n_place + pr;
-                SliceRec &r = s.slices[ord];
-                std::memset(&r, 0, sizeof(r));
-                r.ordinal = ord;
-                r.M = p->M_list[mi];
-                r.scale = Q / ((uint64_t)p->dp_list[tp] * p->M_list[mi]);
-                r.gid = (uint32_t)ord;
-                for (int x = 0; x < s.S; ++x)
-                    r.cls[x] = (uint8_t)(s.places[pr * s.S + x] * s.n_tp + tp);
-            }
+    {
+        uint64_t ord = 0;
+        for (int mi = 0; mi < p->n_M; ++mi)
+            for (int g = 0; g < sp.n_grp; ++g)
+                for (uint64_t pr = 0; pr < sp.n_seq(g); ++pr, ++ord) {
+                    SliceRec &r = s.slices[ord];
+                    std::memset(&r, 0, sizeof(r));
+                    r.ordinal = ord;
+                    r.M = p->M_list[mi];
+                    r.scale = Q / ((uint64_t)sp.D[g] * p->M_list[mi]);
+                    r.gid = (uint32_t)ord;
+                    for (int x = 0; x < s.S; ++x) r.cls[x] = (uint8_t)sp.cls(g, pr, x, s.n_tp);
+                }
+    }
     const int smem = s.h->lay.bytes;
     int per_sm = 0;
     POS_TRY(ensure_smem(reinterpret_cast<const void *>(level_kernel<false, 0>), smem));
@@ -1293,7 +1414,6 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     POS_TRY(blocks_per_sm(reinterpret_cast<const void *>(level_kernel<false, 0>), kThreads,
                           timing_layout(s.h->lay).bytes, &per_sm));
     s.grid_level = std::max(1, per_sm) * sm_count();
-    s.grid_leaf = 2 * sm_count();
 
     POS_CUDA(s.d_slices.reserve(sizeof(SliceRec) * n_slices));
     POS_CUDA(s.d_feas.reserve(sizeof(uint4) * (size_t)n_slices * (s.S + 1)));
@@ -1334,7 +1454,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     uint64_t n_feasible = 0;
     for (int i = 0; i < n_slices; ++i)
         if (root[i]) {
-            feas_by_m[i / (s.n_tp * s.n_place)].push_back((uint32_t)i);
+            feas_by_m[i / sp.per_m].push_back((uint32_t)i);
             ++n_feasible;
         }
     const double ms_setup = ms_since(t_start);
@@ -1679,19 +1799,11 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     const SliceRec &sr = s.slices[ord];
     out->found = 1;
     out->map_rank = inc.idx % s.n_map;
-    out->place_rank = ord % s.n_place;
-    out->tp_idx = (int32_t)((ord / s.n_place) % s.n_tp);
-    out->m_idx = (int32_t)(ord / s.n_place / s.n_tp);
-    out->M = p->M_list[out->m_idx];
-    out->tp = p->tp_list[out->tp_idx];
-    out->D = p->dp_list[out->tp_idx];
+    plan_slice_fields(p, sp, ord, out);
     out->S = s.S;
     out->makespan = (int32_t)(inc.obj / sr.scale);
     out->global_index = inc.idx;
-    for (int x = 0; x < POS_MAX_STAGES; ++x) {
-        out->type[x] = x < s.S ? s.places[out->place_rank * s.S + x] : -1;
-        out->layers[x] = 0;
-    }
+    for (int x = 0; x < POS_MAX_STAGES; ++x) out->layers[x] = 0;
     host_unrank(s.L, s.S, out->map_rank, out->layers);
     if (stats) stats->ms_total = ms_since(t_start);
     return POS_OK;
@@ -1705,7 +1817,14 @@ extern "C" pos_status poseidon_search(const pos_problem *problem, pos_plan *out,
     pos::set_error("");
     pos_status st = pos::validate_problem(problem);  // before touching the device
     if (st == POS_OK) st = pos::validate_tables(&problem->tables);
-    if (st == POS_OK) st = pos::validate_space(problem);
+    if (st != POS_OK) return st;
+    pos::SliceSpace sp;
+    try {
+        st = pos::build_slice_space(problem, problem->S, sp);
+    } catch (...) {
+        return pos::fail(POS_ENOMEM, "host exception (allocation failure)");
+    }
+    if (st == POS_OK) st = pos::validate_space(problem, sp);
     if (st != POS_OK) return st;
     pos::Workspace *ws = nullptr;
     st = pos::get_workspace(&ws);
@@ -1713,9 +1832,10 @@ extern "C" pos_status poseidon_search(const pos_problem *problem, pos_plan *out,
     std::lock_guard<std::mutex> lock(ws->mu);
     try {
         if (problem->schedule == POS_SCHED_INTERLEAVED_1F1B)
-            return pos::search_interleaved(*ws, problem, out, stats);
+            return pos::search_interleaved(*ws, problem, sp, out, stats);
         pos::Search s(*ws);
         s.pb = problem;
+        s.sp = &sp;
         return pos::search_impl(s, out, stats);
     } catch (...) {
         return pos::fail(POS_ENOMEM, "host exception (allocation failure)");

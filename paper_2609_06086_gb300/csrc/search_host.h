@@ -88,12 +88,56 @@ inline void host_unrank(int L, int S, uint64_t rank, int32_t *layers) {
     layers[S - 1] = rem;
 }
 
+// The slices of a search in global-index order (Sec. 4.2.3): the M value,
+// then a group -- the TP index under POS_PLACE_FREE / POS_PLACE_EXACT
+// (every stage on it), the data-parallel degree under POS_PLACE_DEVICES (a
+// class per stage) -- then the group's allowed sequences in lexicographic
+// order.  Built on the host before the device is touched.
+struct SliceSpace {
+    int units = 0;          // stages (devices under Interleaved 1F1B)
+    bool per_stage = false; // POS_PLACE_DEVICES
+    int n_grp = 0;          // TP indices, or D values
+    // FREE / EXACT: one list of type sequences shared by the TP indices;
+    // DEVICES: one list of class sequences per D value (units bytes each)
+    std::vector<std::vector<uint8_t>> seqs;
+    std::vector<uint64_t> grp_off;  // first slice of each group within one M value
+    uint64_t per_m = 0;             // slices per M value
+    std::vector<int32_t> D;         // data-parallel degree of each group
+
+    uint64_t n_seq(int g) const { return seqs[per_stage ? g : 0].size() / units; }
+    const uint8_t *seq(int g, uint64_t place_rank) const {
+        return seqs[per_stage ? g : 0].data() + place_rank * units;
+    }
+    // (m_idx, group, place_rank) of a slice ordinal
+    void decode(uint64_t ord, int *m_idx, int *grp, uint64_t *place_rank) const {
+        *m_idx = (int)(ord / per_m);
+        const uint64_t r = ord % per_m;
+        int g = 0;
+        while (g + 1 < n_grp && grp_off[g + 1] <= r) ++g;
+        *grp = g;
+        *place_rank = r - grp_off[g];
+    }
+    // class of unit u of the slice (group g, rank pr)
+    int cls(int g, uint64_t pr, int u, int n_tp) const {
+        const uint8_t v = seq(g, pr)[u];
+        return per_stage ? v : v * n_tp + g;
+    }
+};
+
+// Validates the placement fields of p and enumerates its slices for
+// `units` stages: POS_EINVAL beyond 2^22 placements or slices.
+pos_status build_slice_space(const pos_problem *p, int units, SliceSpace &sp);
+
+// Writes the slice-identity fields of a found plan (m_idx, tp_idx, M, tp,
+// D, d_idx, place_rank, type[], tp_stage[]) for slice ordinal `ord`.
+void plan_slice_fields(const pos_problem *p, const SliceSpace &sp, uint64_t ord, pos_plan *out);
+
 // The workspace of the current device, created on first use.
 pos_status get_workspace(Workspace **out);
 
 // poseidon_search under POS_SCHED_INTERLEAVED_1F1B (search_il.cu), for a
 // validated problem; the caller holds the workspace's lock.
-pos_status search_interleaved(Workspace &ws, const pos_problem *p, pos_plan *out,
-                              pos_search_stats *stats);
+pos_status search_interleaved(Workspace &ws, const pos_problem *p, const SliceSpace &sp,
+                              pos_plan *out, pos_search_stats *stats);
 
 }  // namespace pos

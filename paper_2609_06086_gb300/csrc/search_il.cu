@@ -183,17 +183,39 @@ __device__ __forceinline__ int il_last_true(int hi, Pred pred) {
     return lo;
 }
 
-// The 16-byte record word of a slice's plans (S = N | M | tp | V) and its
-// type code (2 bits per device), as the interleaved makespan kernels read them.
+// The decoded record's second word of a slice's plans, as the interleaved
+// makespan kernels read it: (slot, type code with 2 bits per device,
+// S = N | M << 8 | tp << 16 | V << 24, per-device TP code).  The class of
+// device d is type_d * n_tp + tp + its field of the TP code: with at most
+// four TP indices each device's index goes in the TP code (tp = 0), which
+// holds a TP index per device (POS_PLACE_DEVICES); above four every device
+// shares one index (checked on the host), carried by tp.
+__device__ __forceinline__ uint4 il_meta_pack(uint32_t tcode, uint32_t tpc, int cls0, int N,
+                                              int n_tp, int M, int V, uint32_t slot) {
+    const uint32_t tp = n_tp <= 4 ? 0u : (uint32_t)(cls0 % n_tp);
+    const uint32_t word = (uint32_t)N | ((uint32_t)M << 8) | (tp << 16) | ((uint32_t)V << 24);
+    return make_uint4(slot, tcode, word, n_tp <= 4 ? tpc : 0u);
+}
 template <int N>
 __device__ __forceinline__ uint4 il_meta(const int (&cls)[N], int n_tp, int M, int V,
                                          uint32_t slot) {
-    uint32_t tcode = 0;
+    uint32_t tcode = 0, tpc = 0;
 #pragma unroll
-    for (int d = 0; d < N; ++d) tcode |= (uint32_t)(cls[d] / n_tp) << (2 * d);
-    const uint32_t word = (uint32_t)N | ((uint32_t)M << 8) | ((uint32_t)(cls[0] % n_tp) << 16) |
-                          ((uint32_t)V << 24);
-    return make_uint4(slot, tcode, word, 0u);
+    for (int d = 0; d < N; ++d) {
+        tcode |= (uint32_t)(cls[d] / n_tp) << (2 * d);
+        tpc |= (uint32_t)(cls[d] % n_tp) << (2 * d);
+    }
+    return il_meta_pack(tcode, tpc, cls[0], N, n_tp, M, V, slot);
+}
+// the same from a slice record (runtime N)
+__device__ __forceinline__ uint4 il_meta_rt(const uint8_t *cls, int N, int n_tp, int M, int V,
+                                            uint32_t slot) {
+    uint32_t tcode = 0, tpc = 0;
+    for (int d = 0; d < N; ++d) {
+        tcode |= (uint32_t)(cls[d] / n_tp) << (2 * d);
+        tpc |= (uint32_t)(cls[d] % n_tp) << (2 * d);
+    }
+    return il_meta_pack(tcode, tpc, cls[0], N, n_tp, M, V, slot);
 }
 
 template <int N>
@@ -517,12 +539,8 @@ __global__ void __launch_bounds__(32 * kSeedWarps) il_seed_kernel(
                 c += arg[j * (L + 1) + c];
                 put_cut(lf, j, c);
             }
-            uint32_t tcode = 0;
-            for (int d = 0; d < N; ++d) tcode |= (uint32_t)(sr.cls[d] / t.n_tp()) << (2 * d);
-            const uint32_t word = (uint32_t)N | ((uint32_t)M << 8) |
-                                  ((uint32_t)(sr.cls[0] % t.n_tp()) << 16) | ((uint32_t)V << 24);
             rec[2 * sl] = make_uint4(lf.a.y, lf.a.z, lf.a.w, lf.b.x & 0x00ffffffu);
-            rec[2 * sl + 1] = make_uint4((uint32_t)sl, tcode, word, 0u);
+            rec[2 * sl + 1] = il_meta_rt(sr.cls, N, t.n_tp(), M, V, (uint32_t)sl);
             leaf_slice[sl] = (uint32_t)sl;
         }
         __syncwarp();
@@ -713,8 +731,8 @@ double il_ms_since(std::chrono::steady_clock::time_point t0) {
 
 // Exact search over Interleaved 1F1B plans (poseidon_search with
 // POS_SCHED_INTERLEAVED_1F1B); the problem has been validated.
-pos_status search_interleaved(Workspace &ws, const pos_problem *p, pos_plan *out,
-                              pos_search_stats *stats) {
+pos_status search_interleaved(Workspace &ws, const pos_problem *p, const SliceSpace &sp,
+                              pos_plan *out, pos_search_stats *stats) {
     const auto t_start = std::chrono::steady_clock::now();
     IlRun r(ws);
     r.p = p;
@@ -727,24 +745,7 @@ pos_status search_interleaved(Workspace &ws, const pos_problem *p, pos_plan *out
     r.pair_key = il_pair_key(r.N, r.V);
     if (r.pair_key < 0) return fail(POS_EINVAL, "Interleaved 1F1B needs V >= 2 and S*V <= 16");
     r.n_map = host_binom(r.L - 1, r.J - 1);
-    // placements over the N devices, lexicographic
-    std::vector<uint8_t> places, seq;
-    const int T = p->tables.n_types, N = r.N;
-    if (p->placement == POS_PLACE_EXACT) {
-        for (int ty = 0; ty < T; ++ty) seq.insert(seq.end(), p->type_counts[ty], (uint8_t)ty);
-        do places.insert(places.end(), seq.begin(), seq.end());
-        while (std::next_permutation(seq.begin(), seq.end()));
-    } else {
-        seq.assign(N, 0);
-        for (;;) {
-            places.insert(places.end(), seq.begin(), seq.end());
-            int x = N - 1;
-            while (x >= 0 && seq[x] == T - 1) seq[x--] = 0;
-            if (x < 0) break;
-            seq[x]++;
-        }
-    }
-    const uint64_t n_place = places.size() / N;
+    const int N = r.N;  // the slices (sp) are over the N devices
     // tables: raw rows uploaded, prefix sums built on the device
     std::vector<unsigned char> host;
     int64_t gA = 0, gD = 0, gP = 0;
@@ -756,25 +757,27 @@ pos_status search_interleaved(Workspace &ws, const pos_problem *p, pos_plan *out
     r.blob = ws.blob.p;
     POS_CUDA(cudaMemcpyAsync(r.blob, host.data(), r.lay.bytes, cudaMemcpyHostToDevice, r.st));
     POS_TRY(launch_prefix_rows(r.blob, r.lay, r.st));
-    // slices: M values that are multiples of N, TP indices, placements
+    // slices: M values that are multiples of N, then the groups (TP index or
+    // D) and their sequences in global-index order
     uint64_t Q = 1;
     for (int i = 0; i < p->n_M; ++i)
-        for (int j = 0; j < r.n_tp; ++j) {
-            const uint64_t dm = (uint64_t)p->dp_list[j] * p->M_list[i];
+        for (int32_t D : sp.D) {
+            const uint64_t dm = (uint64_t)D * p->M_list[i];
             Q = Q / gcd64(Q, dm) * dm;
         }
     std::vector<SliceRec> slices;
     for (int mi = 0; mi < p->n_M; ++mi) {
         if (p->M_list[mi] % N != 0) continue;
-        for (int tp = 0; tp < r.n_tp; ++tp)
-            for (uint64_t pr = 0; pr < n_place; ++pr) {
+        uint64_t ord = (uint64_t)mi * sp.per_m;
+        for (int g = 0; g < sp.n_grp; ++g)
+            for (uint64_t pr = 0; pr < sp.n_seq(g); ++pr, ++ord) {
                 SliceRec sr;
                 std::memset(&sr, 0, sizeof(sr));
-                sr.ordinal = ((uint64_t)mi * r.n_tp + tp) * n_place + pr;
+                sr.ordinal = ord;
                 sr.M = p->M_list[mi];
-                sr.scale = Q / ((uint64_t)p->dp_list[tp] * p->M_list[mi]);
+                sr.scale = Q / ((uint64_t)sp.D[g] * p->M_list[mi]);
                 sr.gid = (uint32_t)slices.size();
-                for (int d = 0; d < N; ++d) sr.cls[d] = (uint8_t)(places[pr * N + d] * r.n_tp + tp);
+                for (int d = 0; d < N; ++d) sr.cls[d] = (uint8_t)sp.cls(g, pr, d, r.n_tp);
                 slices.push_back(sr);
             }
     }
@@ -904,19 +907,11 @@ pos_status search_interleaved(Workspace &ws, const pos_problem *p, pos_plan *out
     const uint64_t ord = inc.idx / r.n_map;
     out->found = 1;
     out->map_rank = inc.idx % r.n_map;
-    out->place_rank = ord % n_place;
-    out->tp_idx = (int32_t)((ord / n_place) % r.n_tp);
-    out->m_idx = (int32_t)(ord / n_place / r.n_tp);
-    out->M = p->M_list[out->m_idx];
-    out->tp = p->tp_list[out->tp_idx];
-    out->D = p->dp_list[out->tp_idx];
+    plan_slice_fields(p, sp, ord, out);
     out->S = N;
     out->makespan = (int32_t)(inc.obj / (Q / ((uint64_t)out->D * out->M)));
     out->global_index = inc.idx;
-    for (int x = 0; x < POS_MAX_STAGES; ++x) {
-        out->type[x] = x < N ? places[out->place_rank * N + x] : -1;
-        out->layers[x] = 0;
-    }
+    for (int x = 0; x < POS_MAX_STAGES; ++x) out->layers[x] = 0;
     host_unrank(r.L, r.J, out->map_rank, out->layers);
     if (stats) stats->ms_total = il_ms_since(t_start);
     return POS_OK;

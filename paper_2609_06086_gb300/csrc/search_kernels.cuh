@@ -171,14 +171,17 @@ template <int S, int PATH>
 __global__ void __launch_bounds__(256, leaf_min_blocks(S, PATH)) leaf_kernel(LeafParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
     __shared__ uint64_t bar;
-    const unsigned long long c0 = __ldcg(p.count);
-    const unsigned long long n = c0 < p.cap ? c0 : p.cap;
-    // blocks without a plan leave before staging the tables
-    if ((unsigned long long)blockIdx.x * blockDim.x >= n) return;
+    // the tables were written before the previous kernel: staged while it
+    // finishes; the plans and their count only after it has completed
     if (!stage_blob_bulk(sm, p.blob, p.lay.bytes, &bar)) {
         if (threadIdx.x == 0) atomicAdd(p.stats + kStBulkTimeout, 1ull);
         return;
     }
+    grid_dep_wait();
+    grid_dep_trigger();
+    const unsigned long long c0 = __ldcg(p.count);
+    const unsigned long long n = c0 < p.cap ? c0 : p.cap;
+    if ((unsigned long long)blockIdx.x * blockDim.x >= n) return;  // no plan for this block
     const Tab t = tab_at(sm, p.lay);
     const int L = p.lay.L;
     unsigned long long evaluated = 0;
@@ -242,8 +245,7 @@ pos_status launch_leaf_t(const LeafParams &p, int grid, cudaStream_t s) {
     auto kern = leaf_kernel<S, PATH>;
     const int smem = p.lay.bytes;
     POS_TRY(ensure_smem(reinterpret_cast<const void *>(kern), smem));
-    kern<<<grid, 256, smem, s>>>(p);
-    POS_CUDA(cudaGetLastError());
+    POS_CUDA(launch_dependent(kern, grid, 256, smem, s, p));
     return POS_OK;
 }
 

@@ -10,6 +10,9 @@ With --ridge the searches use the layer-level (ridge) rule of Theorem 2 and
 are stored as "configN_ridge" / "configN_eager_ridge".  With
 --interleaved V [V ...] the oracle's Interleaved 1F1B search (V chunks per
 device over the config's S devices) is stored as "configN_il_vV" instead.
+With --per-stage-tp the search over config 4's tables with a TP degree per
+stage (gen.config4_per_stage_tp, POS_PLACE_DEVICES) is stored as
+"config4_per_stage_tp" instead.
 """
 import argparse
 import json
@@ -34,8 +37,21 @@ def main():
     ap.add_argument("--ridge", action="store_true", help="layer-level (ridge) pruning")
     ap.add_argument("--interleaved", type=int, nargs="*", default=None,
                     help="V values: Interleaved 1F1B searches instead")
+    ap.add_argument("--per-stage-tp", action="store_true",
+                    help="config 4 with a TP degree per stage instead")
     args = ap.parse_args()
     data = json.load(open(OUT)) if os.path.exists(OUT) else {}
+    if args.per_stage_tp:
+        w = gen.config4_per_stage_tp()
+        t0 = time.time()
+        plan, stats = oracle.search(w, prune=True, warmup=500, seed=0)
+        data["config4_per_stage_tp"] = dict(workload=w.name, seed=w.seed, schedule=0,
+                                            plan=plan, oracle_stats=stats,
+                                            oracle_seconds=round(time.time() - t0, 2))
+        print("config4_per_stage_tp", plan, flush=True)
+        with open(OUT, "w") as f:
+            json.dump(data, f, indent=1, sort_keys=True)
+        return
     if args.interleaved:
         for c in args.configs:
             for V in args.interleaved:

@@ -154,6 +154,55 @@ def test_search_space_limits_rejected_before_the_device(P):
     assert b"lcm" in L.poseidon_last_error()
 
 
+def test_per_stage_tp_problems_checked_before_the_device(P):
+    """POS_PLACE_DEVICES: the device counts, D values, the ridge option and
+    the 2^22 limit on class sequences are checked on the host."""
+    import gen
+    L = P.lib()
+    plan = P.binding.pos_plan()
+    rng = np.random.default_rng(6)
+    T_, n_tp, Lw = 4, 4, 16
+    K = T_ * n_tp
+    w = gen.Workload(name="wide-tp", L=Lw, n_types=T_, n_tp=n_tp,
+                     fwd=rng.integers(1, 9, (K, Lw)).astype(np.int32),
+                     bwd=rng.integers(1, 9, (K, Lw)).astype(np.int32),
+                     dsync=np.zeros((K, Lw), np.int32), p2p_f=np.zeros((K, K), np.int32),
+                     p2p_b=np.zeros((K, K), np.int32), mem_w=np.zeros((K, Lw), np.int64),
+                     mem_a=np.zeros((K, Lw), np.int64), cap=np.full(K, 10, np.int64),
+                     S=12, M_list=[4], tp_list=[1, 1, 1, 1], dp_list=[1] * n_tp,
+                     placement=gen.workloads.PLACE_DEVICES, type_counts=[3, 3, 3, 3],
+                     D_list=[1], seed=0)
+    # 12!/(3!)^4 type orders x 4^12 TP choices: far above 2^22 sequences
+    prob, keep = P.make_problem(w)
+    assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
+    assert b"2^22 class sequences" in L.poseidon_last_error()
+    for field, value, msg in (("type_counts", [3, 3, 3, 70000], b"device counts"),
+                              ("D_list", [0], b"D must be"), ("tp_list", [1, 0, 1, 1], b"TP")):
+        w2 = gen.Workload(**{**w.__dict__, field: value})
+        prob, keep = P.make_problem(w2)
+        assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
+        assert msg in L.poseidon_last_error(), field
+    prob, keep = P.make_problem(w, ridge=True)
+    assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
+    assert b"ridge" in L.poseidon_last_error()
+    w5 = gen.Workload(**{**w.__dict__, "n_tp": 5, "n_types": 3, "S": 2,
+                         "tp_list": [1] * 5, "dp_list": [1] * 5,
+                         "type_counts": [1, 1, 0]})
+    K5 = 15
+    for f in ("fwd", "bwd", "dsync", "mem_w", "mem_a"):
+        setattr(w5, f, np.resize(getattr(w, f), (K5, Lw)))
+    for f in ("p2p_f", "p2p_b"):
+        setattr(w5, f, np.zeros((K5, K5), getattr(w, f).dtype))
+    w5.cap = np.full(K5, 10, np.int64)
+    prob, keep = P.make_problem(w5, schedule=2, V=2)
+    assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
+    assert b"n_tp <= 4" in L.poseidon_last_error()
+    prob, keep = P.make_problem(w)
+    prob.n_D = 0
+    assert L.poseidon_search(C.byref(prob), C.byref(plan), None) == P.binding.POS_EINVAL
+    assert b"D_list" in L.poseidon_last_error()
+
+
 def test_binding_refuses_to_run_without_the_library(tmp_path, monkeypatch):
     import paper_2609_06086_gb300.binding as b
     monkeypatch.setattr(b, "LIB_PATH", str(tmp_path / "missing.so"))

@@ -209,3 +209,26 @@ def test_empty_D_list_is_rejected(orc):
     plan, st = orc.Plan(), orc.Stats()
     assert orc.lib().orc_search(orc.C.byref(p), 1, 0, orc.C.c_uint64(0), orc.C.byref(plan),
                                 orc.C.byref(st)) == -1
+
+
+def test_partitioned_search_keeps_the_plan(orc):
+    """orc_search_part over slice index classes mod n, best of the parts by
+    (T/(D*M), global index) = the whole search's plan (config 2, and random
+    per-stage-TP problems); a part index outside 0..n-1 is rejected."""
+    cases = [gen.config2()] + [_problem(random.Random(71), s) for s in range(30)]
+    for w in cases:
+        ref, _ = orc.search(w, prune=True, warmup=20, seed=1)
+        for n in (2, 3, 7):
+            best = None
+            for part in range(n):
+                plan, _ = orc.search(w, prune=True, warmup=20, seed=1, part=part, n_parts=n)
+                if plan["found"]:
+                    key = (Fraction(plan["T"], plan["D"] * plan["M"]), plan["global_index"])
+                    if best is None or key < best[0]:
+                        best = (key, plan)
+            if not ref["found"]:
+                assert best is None
+            else:
+                assert best[1] == ref
+    with pytest.raises(RuntimeError):
+        orc.search(cases[0], part=3, n_parts=3)
