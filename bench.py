@@ -40,10 +40,10 @@ ENTRY_BYTES = 32  # one frontier entry / one complete plan
 # dram__bytes_read.sum + dram__bytes_write.sum over a config-4 search's leaf
 # launches (the leaf kernel's ncu summary), valid while the kernel's
 # sources hash to LEAF_SOURCES_SHA256 (else the traffic is reported as null)
-LEAF_DRAM_BYTES_PER_PLAN = 59694592 / 1925970
+LEAF_DRAM_BYTES_PER_PLAN = 59695616 / 1925970
 LEAF_SOURCES = ("paper_2609_06086_gb300/csrc/search_kernels.cuh",
                 "paper_2609_06086_gb300/csrc/common.cuh")
-LEAF_SOURCES_SHA256 = "dd2bc510df85d299"
+LEAF_SOURCES_SHA256 = "811e2f2a4ea5f047"
 PRUNE_NAMES = {1: "stage-level, Eq. 2 as printed (Theorem 1)",
                2: "stage-level, tightened: Eq. 2 with P2P edges + completion bounds"}
 
@@ -529,6 +529,8 @@ def run_ours(args, rank, world, local_rank):
     per_stage_tp = {"workload": w_ps.name, "prune": PRUNE_NAMES[args.prune],
                     "time_to_plan_s": ms_ps / 1e3, "evaluations_per_step": ev_ps,
                     "slices": st_ps["slices"], "slices_feasible": st_ps["slices_feasible"],
+                    "host_ms": {k: round(st_ps[k], 3) for k in ("ms_setup", "ms_warmup",
+                                                                 "ms_search")},
                     "plan": {"T_us": pl_ps["T"], "D": pl_ps["D"], "tp_per_stage":
                              [w_ps.tp_list[i] for i in pl_ps["tps"]], "types": pl_ps["types"],
                              "layers": pl_ps["layers"]},

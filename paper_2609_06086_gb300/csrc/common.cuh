@@ -347,6 +347,12 @@ __device__ __forceinline__ uint64_t rank_cuts(const Tab &t, const int (&cut)[S +
 // ---------------------------------------------------------------------------
 // Stage weights (Sec. 4.1.3) from prefix-sum differences; memory (Sec. 3.2).
 // ---------------------------------------------------------------------------
+// max(a + b, c) as one fused integer add-max (the CUDA intrinsic
+// __viaddmax_s32); the makespan relaxations are built from it.
+__device__ __forceinline__ int32_t add_max(int32_t a, int32_t b, int32_t c) {
+    return __viaddmax_s32(a, b, c);
+}
+
 template <int S>
 struct StageW {
     int32_t F[S], B[S], d[S];
@@ -448,18 +454,20 @@ __host__ __device__ constexpr bool down_last_is_b(int S, int s1, int tau) {
     return (s1 & 1) == 0;
 }
 
-// One relaxation of stage s (0-based) on the forward or backward side.
+// One relaxation of stage s (0-based) on the forward or backward side:
+// finish = max(stage clock, predecessor's finish + edge) + node weight, the
+// add-max fused into one integer instruction (add_max).  Every time is >= 0
+// (non-negative weights from time 0), so a stage without an inter-stage
+// predecessor takes its clock alone.
 template <int S, int s>
 __device__ __forceinline__ void relax_f(int32_t (&Fo)[S], const StageW<S> &w, int32_t clock) {
-    int32_t in = 0;
-    if constexpr (s > 0) in = Fo[s - 1] + w.pf[s - 1];
-    Fo[s] = max(clock, in) + w.F[s];
+    if constexpr (s > 0) Fo[s] = add_max(Fo[s - 1], w.pf[s - 1], clock) + w.F[s];
+    else Fo[s] = clock + w.F[s];
 }
 template <int S, int s>
 __device__ __forceinline__ void relax_b(int32_t (&Bo)[S], const StageW<S> &w, int32_t clock) {
-    int32_t in = 0;
-    if constexpr (s + 1 < S) in = Bo[s + 1] + w.pb[s];
-    Bo[s] = max(clock, in) + w.B[s];
+    if constexpr (s + 1 < S) Bo[s] = add_max(Bo[s + 1], w.pb[s], clock) + w.B[s];
+    else Bo[s] = clock + w.B[s];
 }
 
 // Ramp op of 1-based stage s1 at level t (UP) or at level 2M + t (DOWN);
@@ -641,13 +649,13 @@ __host__ __device__ constexpr int eager_down_lag(int S, int s1, int tau) {
 template <int S, int s, int LAG>
 __device__ __forceinline__ void relax_f_lag(int32_t (&Fo)[S], int32_t (&Fp)[S],
                                             const StageW<S> &w, int32_t clock) {
-    int32_t in = 0;
+    Fp[s] = Fo[s];
     if constexpr (s > 0) {
         static_assert(LAG == 1 || LAG == 2, "forward lag");
-        in = (LAG == 2 ? Fp[s - 1] : Fo[s - 1]) + w.pf[s - 1];
+        Fo[s] = add_max(LAG == 2 ? Fp[s - 1] : Fo[s - 1], w.pf[s - 1], clock) + w.F[s];
+    } else {
+        Fo[s] = clock + w.F[s];
     }
-    Fp[s] = Fo[s];
-    Fo[s] = max(clock, in) + w.F[s];
 }
 
 template <int S, bool UP, int t, int s1>

@@ -42,12 +42,12 @@ __device__ __forceinline__ void il_relax(IlState<N, V> &s) {
     constexpr int J = N * V, j = OP & 15, d = j % N;
     if constexpr ((OP & 0x80) == 0) {
         int32_t t = s.clk[d];
-        if constexpr (j > 0) t = max(t, s.Fo[j - 1] + s.pf[(j - 1) % N]);
+        if constexpr (j > 0) t = add_max(s.Fo[j - 1], s.pf[(j - 1) % N], t);
         s.Fo[j] = t + s.F[j];
         s.clk[d] = s.Fo[j];
     } else {
         int32_t t = s.clk[d];
-        if constexpr (j + 1 < J) t = max(t, s.Bo[j + 1] + s.pb[d]);
+        if constexpr (j + 1 < J) t = add_max(s.Bo[j + 1], s.pb[d], t);
         s.Bo[j] = t + s.B[j];
         s.clk[d] = s.Bo[j];
     }

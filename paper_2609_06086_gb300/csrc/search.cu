@@ -980,27 +980,43 @@ static pos_status device_sequences(const pos_problem *p, int units, int D,
         bud[t] = p->type_counts[t] / D;
         vmax = std::max(vmax, bud[t]);
     }
-    // reach[n * (vmax + 1) + v]: v is a sum of exactly n TP degrees
-    std::vector<uint8_t> reach((size_t)(units + 1) * (vmax + 1), 0);
-    reach[0] = 1;
-    for (int n = 1; n <= units; ++n)
-        for (int v = 0; v <= vmax; ++v)
-            for (int j = 0; j < n_tp; ++j) {
-                const int d = p->tp_list[j];
-                if (d <= v && reach[(size_t)(n - 1) * (vmax + 1) + v - d]) {
-                    reach[(size_t)n * (vmax + 1) + v] = 1;
-                    break;
-                }
-            }
-    auto completes = [&](int r) {
+    // reach[v], bit n: v is a sum of exactly n TP degrees (n <= units)
+    std::vector<uint32_t> reach((size_t)vmax + 1, 0u);
+    reach[0] = 1u;
+    for (int v = 1; v <= vmax; ++v)
+        for (int j = 0; j < n_tp; ++j) {
+            const int d = p->tp_list[j];
+            if (d <= v) reach[v] |= (reach[v - d] << 1) & ((2u << units) - 1u);
+        }
+    // completes(r): the remaining budgets bud[] split over exactly r stages;
+    // memoised over (r, budgets) when that table is small
+    size_t states = (size_t)units + 1;
+    int radix[POS_MAX_TYPES];
+    for (int t = 0; t < T; ++t) {
+        radix[t] = bud[t] + 1;
+        states = states <= ((size_t)1 << 24) / (size_t)radix[t] ? states * radix[t] : 0;
+        if (states == 0) break;
+    }
+    std::vector<uint8_t> memo(states, 0);  // 0 unknown, 1 no, 2 yes
+    auto completes = [&](int r) -> bool {
+        size_t key = 0;
+        if (!memo.empty()) {
+            for (int t = T - 1; t >= 0; --t) key = key * radix[t] + bud[t];
+            key = key * (units + 1) + r;
+            if (memo[key]) return memo[key] == 2;
+        }
         uint32_t mask = 1u;  // bit n: n stages used by the types seen so far
-        for (int t = 0; t < T; ++t) {
-            uint32_t next = 0;
-            for (int n = 0; n <= r; ++n)
-                if (reach[(size_t)n * (vmax + 1) + bud[t]]) next |= mask << n;
+        for (int t = 0; t < T && mask; ++t) {
+            uint32_t next = 0, m = reach[bud[t]] & ((2u << r) - 1u);
+            while (m) {
+                next |= mask << __builtin_ctz(m);
+                m &= m - 1u;
+            }
             mask = next & ((2u << r) - 1u);
         }
-        return (mask >> r) & 1u;
+        const bool ok = (mask >> r) & 1u;
+        if (!memo.empty()) memo[key] = ok ? 2 : 1;
+        return ok;
     };
     if (!completes(units)) return POS_OK;
     uint8_t seq[POS_MAX_STAGES];
@@ -1008,6 +1024,21 @@ static pos_status device_sequences(const pos_problem *p, int units, int D,
     int u = 0;
     k_at[0] = -1;
     while (u >= 0) {  // iterative depth-first walk, classes in ascending order
+        if (u == units - 1) {
+            // the last stage takes what is left: one type with a budget equal
+            // to a TP degree (the prefix was kept only if such a class exists)
+            for (int k = 0; k < K; ++k) {
+                const int t = k / n_tp;
+                bool only = bud[t] == p->tp_list[k % n_tp];
+                for (int o = 0; o < T && only; ++o) only = o == t || bud[o] == 0;
+                if (!only) continue;
+                seq[u] = (uint8_t)k;
+                out.insert(out.end(), seq, seq + units);
+                if (++*total > limit) return fail(POS_EINVAL, "more than 2^22 class sequences");
+            }
+            --u;  // the parent's class is undone on its next step
+            continue;
+        }
         int k = k_at[u] + 1;
         if (k_at[u] >= 0) bud[k_at[u] / n_tp] += p->tp_list[k_at[u] % n_tp];  // undo
         for (; k < K; ++k) {
@@ -1024,12 +1055,7 @@ static pos_status device_sequences(const pos_problem *p, int units, int D,
         }
         k_at[u] = k;
         seq[u] = (uint8_t)k;
-        if (u == units - 1) {
-            out.insert(out.end(), seq, seq + units);
-            if (++*total > limit) return fail(POS_EINVAL, "more than 2^22 class sequences");
-        } else {
-            k_at[++u] = -1;
-        }
+        k_at[++u] = -1;
     }
     return POS_OK;
 }

@@ -198,6 +198,7 @@ __global__ void __launch_bounds__(256, leaf_min_blocks(S, PATH)) leaf_kernel(Lea
         const Vec32 lv = next;
         next = i + stride < n ? load32(p.leaves + i + stride) : none;
         const uint32_t sl = lv.a.x;
+        bool cand = false;
         if (sl != kLeafHole) {
             const SliceRec &sr = p.slices[sl];
             int cut[S + 1], cls[S];
@@ -207,18 +208,30 @@ __global__ void __launch_bounds__(256, leaf_min_blocks(S, PATH)) leaf_kernel(Lea
 #pragma unroll
             for (int s = 0; s < S; ++s) cls[s] = __ldg(&sr.cls[s]);
             const uint64_t scale = __ldg(&sr.scale);
-            const uint64_t ord = __ldg(&sr.ordinal);
             // enumerated plans are ridge-like already; warm-up plans may not be
-            const bool admissible = !p.ridge || ridge_plan_ok<S>(cut, cls, t.n_tp());
-            const uint64_t rank = rank_cuts<S>(t, cut);
+            cand = !p.ridge || ridge_plan_ok<S>(cut, cls, t.n_tp());
             StageW<S> w;
             stage_weights<S>(t, cut, cls, w);
             const int32_t T = makespan_path<S, PATH>(w, p.M, p.pg);
             obj = (unsigned long long)T * scale;
-            idx = ord * p.n_map + rank;
             ++evaluated;
             if (p.slice_best) atomicMin(p.slice_best + sl, obj);  // ordering hint only
-            if (!admissible) obj = idx = ~0ull;
+        }
+        // A plan whose objective is above the incumbent's cannot lower it
+        // (the incumbent only decreases, so a stale read lets more through,
+        // never fewer): most warps stop here, and only the candidates pay
+        // for their global index (the composition's rank) and the warp
+        // minimum.
+        cand = cand && obj <= __ldcg(&p.inc->obj);
+        if (!__any_sync(0xffffffffu, cand)) continue;
+        if (cand) {
+            int cut[S + 1];
+            cut[0] = 0;
+            leaf_cuts<S>(lv, cut);
+            cut[S] = L;
+            idx = __ldg(&p.slices[sl].ordinal) * p.n_map + rank_cuts<S>(t, cut);
+        } else {
+            obj = ~0ull;
         }
         // warp minimum, then one CAS attempt per warp
 #pragma unroll

@@ -1,7 +1,7 @@
 // Measurement tooling, not part of libposeidon: poseidon_probe_int32 times
 // the relaxation the makespan kernels are built from,
 // finish = max(pred + edge, clock) + weight (one add, one max, one add:
-// 3 int32 ops), with enough independent chains per thread and threads per
+// 3 int32 ops; the add-max fused into one instruction as the kernels do), with enough independent chains per thread and threads per
 // SM that no dependency or latency limits it.  The result checks the
 // roofline denominator the benchmark uses for the ALU-bound kernels
 // (SMs x 128 int32 lanes x clock).  Built into libposeidon_probe.so.
@@ -30,9 +30,10 @@ __global__ void __launch_bounds__(kProbeThreads) int32_probe_kernel(int iters, i
     for (int i = 0; i < iters; ++i) {
 #pragma unroll
         for (int k = 0; k < kProbeChains; ++k) {
-            // two chained relaxations per chain and iteration (6 int32 ops)
-            x[k] = max(y[k] + e[k], x[k]) + w[k];
-            y[k] = max(x[k] + w[k], y[k]) + e[k];
+            // two chained relaxations per chain and iteration (6 int32 ops),
+            // the add-max fused as in the makespan kernels (__viaddmax_s32)
+            x[k] = __viaddmax_s32(y[k], e[k], x[k]) + w[k];
+            y[k] = __viaddmax_s32(x[k], w[k], y[k]) + e[k];
         }
     }
     int32_t acc = 0;
