@@ -53,9 +53,10 @@ __device__ __forceinline__ int popc128(const Bits128 &b) {
 // suffix feasibility: one block per slice, thread c
 // ---------------------------------------------------------------------------
 // Also fills lim[(gid*S + x)*128 + c] = the largest l such that stage x
-// holds layers [c, c+l) within memory (0 if none), capped at L - c.
+// holds layers [c, c+l) within memory (0 if none), capped at L - c, and
+// root[gid] = 1 when the slice has a memory-feasible plan.
 __global__ void feas_kernel(const SliceRec *slices, int n_slices, int S, uint4 *feas,
-                            uint8_t *lim, const void *blob, BlobLayout lay,
+                            uint8_t *lim, uint8_t *root, const void *blob, BlobLayout lay,
                             unsigned long long *stats) {
     extern __shared__ __align__(16) unsigned char sm[];
     __shared__ uint32_t prev[4], cur[4];
@@ -100,20 +101,12 @@ __global__ void feas_kernel(const SliceRec *slices, int n_slices, int S, uint4 *
             __syncthreads();
             if (c == 0) row[x] = make_uint4(prev[0], prev[1], prev[2], prev[3]);
         }
+        // root[gid] = the whole model fits the slice's stages (bit c = 0 of row 0)
+        if (c == 0) root[sr.gid] = (uint8_t)(prev[0] & 1u);
         __syncthreads();
     }
 }
 
-__device__ __forceinline__ bool feas_bit(const uint4 *feas, int S, uint32_t gid, int x, int c) {
-    const uint4 w = __ldg(feas + (size_t)gid * (S + 1) + x);
-    const uint32_t word = (c >> 5) == 0 ? w.x : (c >> 5) == 1 ? w.y : (c >> 5) == 2 ? w.z : w.w;
-    return (word >> (c & 31)) & 1u;
-}
-
-__global__ void root_bits_kernel(const uint4 *feas, int n_slices, int S, uint8_t *out) {
-    const int i = blockIdx.x * blockDim.x + threadIdx.x;
-    if (i < n_slices) out[i] = feas_bit(feas, S, i, 0, 0);
-}
 
 // ---------------------------------------------------------------------------
 // completion bounds (prune mode 2).  For a complete plan and 0-based stages
@@ -1181,6 +1174,38 @@ static pos_status sync_read(Search &s, void *dst, const void *src, size_t bytes)
     return POS_OK;
 }
 
+// Several device-to-host copies behind one synchronisation (each
+// synchronisation leaves the device idle for a host round trip).
+struct ReadPart {
+    void *dst;
+    const void *src;
+    size_t bytes;
+};
+static pos_status sync_read_many(Search &s, const ReadPart *parts, int n) {
+    size_t total = 0;
+    for (int i = 0; i < n; ++i) total += (parts[i].bytes + 15) & ~(size_t)15;
+    if (total > s.ws.h_read_cap) {  // no copy is in flight: the old area can go
+        if (s.ws.h_read) cudaFreeHost(s.ws.h_read);
+        s.ws.h_read = nullptr;
+        s.ws.h_read_cap = 0;
+        POS_CUDA(cudaMallocHost(&s.ws.h_read, total + total / 2));
+        s.ws.h_read_cap = total + total / 2;
+    }
+    size_t off = 0;
+    for (int i = 0; i < n; ++i) {
+        POS_CUDA(cudaMemcpyAsync(s.ws.h_read + off, parts[i].src, parts[i].bytes,
+                                 cudaMemcpyDeviceToHost, s.stream));
+        off += (parts[i].bytes + 15) & ~(size_t)15;
+    }
+    POS_CUDA(cudaStreamSynchronize(s.stream));
+    off = 0;
+    for (int i = 0; i < n; ++i) {
+        std::memcpy(parts[i].dst, s.ws.h_read + off, parts[i].bytes);
+        off += (parts[i].bytes + 15) & ~(size_t)15;
+    }
+    return POS_OK;
+}
+
 // Enqueues an upload through the workspace's pinned staging area (an
 // upload straight from pageable memory makes the host wait while the
 // driver stages it).  The area is sized at the start of a search and only
@@ -1456,21 +1481,17 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     POS_CUDA(cudaMemsetAsync(s.d_ctr.p, 0, sizeof(unsigned long long) * 128, s.stream));
     POS_CUDA(cudaMemsetAsync(s.d_best.p, 0xff, sizeof(unsigned long long) * n_slices, s.stream));
     const SliceRec *d_all = static_cast<const SliceRec *>(s.d_slices.p);
+    DevBuf &d_root = s.d_root;
+    POS_CUDA(d_root.reserve(n_slices));
     {
         // the memory tables alone (Pw, Pa, cap) are staged per block
         const BlobLayout ml = memory_layout(s.h->lay);
         POS_TRY(ensure_smem(reinterpret_cast<const void *>(feas_kernel), ml.bytes));
         feas_kernel<<<std::min(n_slices, 16 * sm_count()), 128, ml.bytes, s.stream>>>(
             d_all, n_slices, s.S, static_cast<uint4 *>(s.d_feas.p),
-            static_cast<uint8_t *>(s.ws.d_lim.p),
+            static_cast<uint8_t *>(s.ws.d_lim.p), static_cast<uint8_t *>(d_root.p),
             static_cast<const unsigned char *>(s.h->d_blob) + s.h->lay.off_Pw, ml, s.stats);
     }
-    POS_CUDA(cudaGetLastError());
-    s.launches++;
-    DevBuf &d_root = s.d_root;
-    POS_CUDA(d_root.reserve(n_slices));
-    root_bits_kernel<<<(n_slices + 255) / 256, 256, 0, s.stream>>>(
-        static_cast<const uint4 *>(s.d_feas.p), n_slices, s.S, static_cast<uint8_t *>(d_root.p));
     POS_CUDA(cudaGetLastError());
     s.launches++;
     std::vector<uint8_t> root(n_slices);
@@ -1656,6 +1677,9 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     const SliceRec *d_ordered = static_cast<const SliceRec *>(s.d_batch.p);
     const Prefix *d_rootp = static_cast<const Prefix *>(s.d_roots.p);
 
+    Key128 inc;
+    unsigned long long hs[kStCount];
+    bool have_results = false;  // inc and hs read after the last launch
     if (s.S == 1) {
         // the single stage takes every layer: each feasible slice is one plan
         for (const Batch &b : batches) {
@@ -1740,9 +1764,15 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
             s.n_leaf++;
             if (prof) POS_CUDA(cudaEventRecord(ev[S], s.stream));
         }
+        // the passes' counters, the incumbent and the statistics in one read
         std::vector<unsigned long long> hb(32 * n_b);
-        if ((st = sync_read(s, hb.data(), bctr, sizeof(unsigned long long) * hb.size())) != POS_OK)
-            return st;
+        {
+            const ReadPart parts[3] = {{hb.data(), bctr, sizeof(unsigned long long) * hb.size()},
+                                       {&inc, s.d_inc.p, sizeof(inc)},
+                                       {hs, s.stats, sizeof(hs)}};
+            if ((st = sync_read_many(s, parts, 3)) != POS_OK) return st;
+            have_results = true;
+        }
         for (size_t bi = 0; bi < n_b && prof; ++bi) {
             cudaEvent_t *ev = s.ws.evs.data() + bi * (S + 1);
             for (int x = 0; x <= S - 1; ++x) {
@@ -1762,19 +1792,19 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
             for (int x = 0; x <= S - 2; ++x) overflow |= hb[32 * bi + 2 * x + 1] != 0;
             if (!overflow) continue;
             s.reruns++;
+            have_results = false;
             const Batch &b = batches[bi];
             s.cur_nb = (int)b.nb;
             st = process(s, d_ordered + b.off, b.M, 0, d_rootp, (long long)b.nb);
             if (st != POS_OK) return st;
         }
     }
-    POS_CUDA(cudaStreamSynchronize(s.stream));
+    if (!have_results) {
+        const ReadPart parts[2] = {{&inc, s.d_inc.p, sizeof(inc)}, {hs, s.stats, sizeof(hs)}};
+        if ((st = sync_read_many(s, parts, 2)) != POS_OK) return st;
+    }
     const double ms_search = ms_since(t_search);
 
-    Key128 inc;
-    if ((st = sync_read(s, &inc, s.d_inc.p, sizeof(inc))) != POS_OK) return st;
-    unsigned long long hs[kStCount];
-    if ((st = sync_read(s, hs, s.stats, sizeof(hs))) != POS_OK) return st;
     if (hs[kStTimeout])
         return fail(POS_ETIMEOUT, "the incumbent's compare-and-swap loop hit its iteration "
                                   "limit (pos_problem.cas_limit rounds)");
