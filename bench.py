@@ -332,19 +332,46 @@ def run_ours(args, rank, world, local_rank):
                ms_leaf=0.0, expand_launches=0, complete_launches=0, leaf_launches=0,
                parents_expand=0, parents_complete=0, leaves=0, prefixes=0,
                ms_setup=0.0, ms_warmup=0.0, ms_search=0.0)
+    # the device time brackets the library call alone (the binding's plan and
+    # statistics dicts are built after ev1); e2e times the public Python call
+    Lib, Cb = P.lib(), P.binding.C
+    plan_c, st_c = P.binding.pos_plan(), P.binding.pos_search_stats()
+
+    def timed_search_call(pr):
+        """One search with L2 flushed before it; the CUDA events bracket the
+        library call alone.  Returns (ms, plan dict, stats dict)."""
+        pc, sc = P.binding.pos_plan(), P.binding.pos_search_stats()
+        flush.zero_()
+        torch.cuda.synchronize()
+        ev0.record()
+        rc_ = Lib.poseidon_search(Cb.byref(pr), Cb.byref(pc), Cb.byref(sc))
+        ev1.record()
+        torch.cuda.synchronize()
+        if rc_ != P.binding.POS_OK:
+            raise P.PoseidonError(rc_, Lib.poseidon_last_error().decode())
+        return ev0.elapsed_time(ev1), P.binding.plan_dict(pr, pc), P.binding.stats_dict(sc)
+
     for _ in range(args.steps):
         flush.zero_()  # evict L2 (129 MB) between steps
         torch.cuda.synchronize()
-        t0 = time.perf_counter()
         ev0.record()
-        plan, st = P.poseidon_search(prob)
+        rc = Lib.poseidon_search(Cb.byref(prob), Cb.byref(plan_c), Cb.byref(st_c))
         ev1.record()
         torch.cuda.synchronize()
-        wall_ms.append(1e3 * (time.perf_counter() - t0))
+        if rc != P.binding.POS_OK:
+            raise P.PoseidonError(rc, Lib.poseidon_last_error().decode())
         dev_ms.append(ev0.elapsed_time(ev1))
-        plans.append(plan)
+        plans.append(P.binding.plan_dict(prob, plan_c))
+        st = P.binding.stats_dict(st_c)
         for k in agg:
             agg[k] += st[k]
+    for _ in range(args.steps):
+        flush.zero_()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        P.poseidon_search(prob)
+        torch.cuda.synchronize()
+        wall_ms.append(1e3 * (time.perf_counter() - t0))
     clk = clocks.stop() if clocks else None
     # per-kernel breakdown: the same number of steps again, with CUDA events
     # around every launch on the library's stream (profile=1)
@@ -353,13 +380,8 @@ def run_ours(args, rank, world, local_rank):
     for k in ("ms_depth", "launches_depth", "parents_depth", "children_depth"):
         kagg[k] = [0] * 16
     for _ in range(args.steps):
-        flush.zero_()
-        torch.cuda.synchronize()
-        ev0.record()
-        plan_p, st_p = P.poseidon_search(prob_prof)
-        ev1.record()
-        torch.cuda.synchronize()
-        prof_ms.append(ev0.elapsed_time(ev1))
+        ms_, plan_p, st_p = timed_search_call(prob_prof)
+        prof_ms.append(ms_)
         for k in kagg:
             if isinstance(kagg[k], list):
                 kagg[k] = [u + v for u, v in zip(kagg[k], st_p[k])]
@@ -465,13 +487,8 @@ def run_ours(args, rank, world, local_rank):
     P.poseidon_search(prob_e)
     e_ms, e_ev, e_ok = [], 0, True
     for _ in range(max(3, min(100, args.steps // 2))):
-        flush.zero_()
-        torch.cuda.synchronize()
-        ev0.record()
-        plan_e, st_e = P.poseidon_search(prob_e)
-        ev1.record()
-        torch.cuda.synchronize()
-        e_ms.append(ev0.elapsed_time(ev1))
+        ms_, plan_e, st_e = timed_search_call(prob_e)
+        e_ms.append(ms_)
         e_ev += st_e["evaluated"]
         e_ok &= plan_e["global_index"] == ref_e.get("global_index")
     # layer-level (ridge) pruning, Theorem 2: value against the exact optimum
@@ -484,13 +501,8 @@ def run_ours(args, rank, world, local_rank):
         P.poseidon_search(prob_r)
         r_ms = []
         for _ in range(max(3, min(100, args.steps // 2))):
-            flush.zero_()
-            torch.cuda.synchronize()
-            ev0.record()
-            plan_r, st_r = P.poseidon_search(prob_r)
-            ev1.record()
-            torch.cuda.synchronize()
-            r_ms.append(ev0.elapsed_time(ev1))
+            ms_, plan_r, st_r = timed_search_call(prob_r)
+            r_ms.append(ms_)
         ridge_lines.append({"schedule": "Eager 1F1B" if sched else "1F1B",
                             "time_to_plan_s": sum(r_ms) / len(r_ms) / 1e3,
                             "speedup_vs_exact": exact_ms / (sum(r_ms) / len(r_ms)),
@@ -510,13 +522,8 @@ def run_ours(args, rank, world, local_rank):
         P.poseidon_search(pr)
         ms, ok, st_sum = [], True, 0
         for _ in range(max(3, min(100, args.steps // 2))):
-            flush.zero_()
-            torch.cuda.synchronize()
-            ev0.record()
-            pl, st_ = P.poseidon_search(pr)
-            ev1.record()
-            torch.cuda.synchronize()
-            ms.append(ev0.elapsed_time(ev1))
+            ms_, pl, st_ = timed_search_call(pr)
+            ms.append(ms_)
             st_sum += st_["evaluated"]
             ok &= ref_plan is not None and all(pl[k] == ref_plan.get(k) for k in
                                                ("global_index", "T", "layers"))
@@ -554,13 +561,8 @@ def run_ours(args, rank, world, local_rank):
     P.poseidon_search(prob2)
     o_ms, o_ev, o_ok = [], 0, True
     for _ in range(max(3, min(100, args.steps // 2))):
-        flush.zero_()
-        torch.cuda.synchronize()
-        ev0.record()
-        plan2, st2 = P.poseidon_search(prob2)
-        ev1.record()
-        torch.cuda.synchronize()
-        o_ms.append(ev0.elapsed_time(ev1))
+        ms_, plan2, st2 = timed_search_call(prob2)
+        o_ms.append(ms_)
         o_ev += st2["evaluated"]
         o_ok &= plan2["global_index"] == ref["plan"]["global_index"]
     other_prune = {"prune": other, "time_to_plan_s": sum(o_ms) / len(o_ms) / 1e3,
@@ -579,13 +581,8 @@ def run_ours(args, rank, world, local_rank):
     P.poseidon_search(prob3)
     c3_ms, c3_ok = [], True
     for _ in range(max(3, min(100, args.steps // 2))):
-        flush.zero_()
-        torch.cuda.synchronize()
-        ev0.record()
-        plan3, st3 = P.poseidon_search(prob3)
-        ev1.record()
-        torch.cuda.synchronize()
-        c3_ms.append(ev0.elapsed_time(ev1))
+        ms_, plan3, st3 = timed_search_call(prob3)
+        c3_ms.append(ms_)
         c3_ok &= plan3["global_index"] == ref3.get("global_index")
     _, st3p = P.poseidon_search(prob3p)
     leaf3 = st3p["evaluated"] - st3p["warmup_evaluated"]

@@ -244,18 +244,26 @@ def make_problem(w, warmup=500, prune=True, seed=0, frontier_cap=0, profile=Fals
     return p, keep
 
 
+def plan_dict(problem: pos_problem, plan: pos_plan):
+    """The fields of a pos_plan as a dict (layers of the S stages, or of the
+    S*V virtual stages under Interleaved 1F1B)."""
+    S = problem.S
+    J = S * problem.V if problem.schedule == POS_SCHED_INTERLEAVED_1F1B else S
+    return dict(found=bool(plan.found), m_idx=plan.m_idx, tp_idx=plan.tp_idx, M=plan.M,
+                tp=plan.tp, D=plan.D, d_idx=plan.d_idx, T=plan.makespan,
+                place_rank=plan.place_rank, map_rank=plan.map_rank,
+                global_index=plan.global_index, types=list(plan.type)[:S],
+                tps=list(plan.tp_stage)[:S], layers=list(plan.layers)[:J])
+
+
+def stats_dict(st: pos_search_stats):
+    return {n: (list(getattr(st, n)) if n.endswith("_depth") else getattr(st, n))
+            for n, _ in pos_search_stats._fields_}
+
+
 def poseidon_search(problem: pos_problem):
     """Returns (plan dict, stats dict); raises PoseidonError on failure
     (POS_EINFEASIBLE included)."""
     plan, st = pos_plan(), pos_search_stats()
     _check(lib().poseidon_search(C.byref(problem), C.byref(plan), C.byref(st)))
-    S = problem.S
-    J = S * problem.V if problem.schedule == POS_SCHED_INTERLEAVED_1F1B else S
-    out = dict(found=bool(plan.found), m_idx=plan.m_idx, tp_idx=plan.tp_idx, M=plan.M,
-               tp=plan.tp, D=plan.D, d_idx=plan.d_idx, T=plan.makespan,
-               place_rank=plan.place_rank, map_rank=plan.map_rank,
-               global_index=plan.global_index, types=list(plan.type)[:S],
-               tps=list(plan.tp_stage)[:S], layers=list(plan.layers)[:J])
-    stats = {n: (list(getattr(st, n)) if n.endswith("_depth") else getattr(st, n))
-             for n, _ in pos_search_stats._fields_}
-    return out, stats
+    return plan_dict(problem, plan), stats_dict(st)

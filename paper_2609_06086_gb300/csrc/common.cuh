@@ -36,8 +36,11 @@ pos_status blocks_per_sm(const void *kernel, int threads, int smem, int *out);
 // the next such kernel be scheduled: a kernel's pre-wait part can therefore
 // only overlap the post-wait part of its predecessor, so it may read
 // whatever was written two or more kernels earlier (the cost tables, slice
-// records and bound tables of a search).  Without the launch attribute the
-// two instructions do nothing.
+// records and bound tables of a search).  Every block of such a kernel
+// executes grid_dep_wait() before it exits, even when it has no work: a grid
+// completes only after its predecessor has, which keeps the chain's order
+// transitive for the kernels after it.  Without the launch attribute the two
+// instructions do nothing.
 __device__ __forceinline__ void grid_dep_wait() {
     asm volatile("griddepcontrol.wait;" ::: "memory");
 }

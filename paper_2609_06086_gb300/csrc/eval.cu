@@ -113,6 +113,8 @@ template <int NK>
 __global__ void __launch_bounds__(1024) sort_scan_kernel(const uint32_t *hist, uint32_t *offs,
                                                         uint32_t *cursor) {
     __shared__ uint32_t warp_total[32];
+    grid_dep_wait();  // the histogram
+    grid_dep_trigger();
     const int per = (NK + blockDim.x - 1) / blockDim.x;
     const int lo = threadIdx.x * per, hi = min(NK, lo + per);
     const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
@@ -146,16 +148,23 @@ __global__ void __launch_bounds__(1024) sort_scan_kernel(const uint32_t *hist, u
     }
 }
 
-// Each block takes chunks of kChunk candidates: counts their keys, reserves
-// one range per key with a single atomic, then places the indices.
-constexpr int kChunk = 8192;
+// Each block takes chunks of `chunk` candidates: counts their keys, reserves
+// one range per key with a single atomic, then places the indices.  The
+// chunk grows with the batch (about two chunks per SM, 2048 to 65536), so
+// that large batches reserve fewer ranges.
+__host__ inline int64_t scatter_chunk(int64_t n, int sms) {
+    int64_t c = (n / (2 * (int64_t)sms) + 511) & ~(int64_t)511;
+    return c < 2048 ? 2048 : (c > 65536 ? 65536 : c);
+}
 
 template <int NK>
-__global__ void sort_scatter_kernel(const uint16_t *keys, int64_t n, uint32_t *cursor,
-                                    uint32_t *perm) {
+__global__ void sort_scatter_kernel(const uint16_t *keys, int64_t n, int64_t chunk,
+                                    uint32_t *cursor, uint32_t *perm) {
     __shared__ uint32_t h[NK];
-    for (int64_t c0 = blockIdx.x * (int64_t)kChunk; c0 < n; c0 += (int64_t)gridDim.x * kChunk) {
-        const int64_t c1 = min(n, c0 + kChunk);
+    grid_dep_wait();  // the keys (histogram pass) and the cursors (scan)
+    grid_dep_trigger();
+    for (int64_t c0 = blockIdx.x * chunk; c0 < n; c0 += (int64_t)gridDim.x * chunk) {
+        const int64_t c1 = min(n, c0 + chunk);
         for (int i = threadIdx.x; i < NK; i += blockDim.x) h[i] = 0;
         __syncthreads();
         for (int64_t i = c0 + threadIdx.x; i < c1; i += blockDim.x) {
@@ -188,6 +197,8 @@ __global__ void __launch_bounds__(256, 4) decode_kernel(EvalParams p) {
         stage_blob(sm, p.blob, p.lay.bytes);
     }
     __syncthreads();
+    grid_dep_wait();  // the permutation (scatter pass)
+    grid_dep_trigger();
     const Tab t = tab_at(sm, p.lay);
     const uint8_t *lim = sm + p.lay.off_Pw;
     const int64_t total = p.offs[p.nkeys];
@@ -229,9 +240,8 @@ pos_status launch_decode(const EvalParams &p, cudaStream_t stream) {
     POS_TRY(blocks_per_sm(kern, 256, smem, &per_sm));
     const int64_t blocks = (p.n + 255) / 256;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)std::max(per_sm, 1) * sm_count()));
-    if (lim) decode_kernel<true><<<grid, 256, smem, stream>>>(p);
-    else decode_kernel<false><<<grid, 256, smem, stream>>>(p);
-    POS_CUDA(cudaGetLastError());
+    if (lim) POS_CUDA(launch_dependent(decode_kernel<true>, grid, 256, smem, stream, p));
+    else POS_CUDA(launch_dependent(decode_kernel<false>, grid, 256, smem, stream, p));
     return POS_OK;
 }
 
@@ -310,18 +320,30 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
             1, std::min<int64_t>((m + 255) / 256, 4LL * sm_count()));
         cudaError_t e = cudaMemsetAsync(hist, 0, sizeof(uint32_t) * nk, stream);
         if (e == cudaSuccess) {
+            const int64_t chunk = scatter_chunk(m, sm_count());
             const int sgrid = (int)std::max<int64_t>(
-                1, std::min<int64_t>((m + kChunk - 1) / kChunk, 8LL * sm_count()));
+                1, std::min<int64_t>((m + chunk - 1) / chunk, 8LL * sm_count()));
+            // the histogram follows a memset; the kernels after it are chained
+            // by programmatic dependent launch
             if (il) {
                 sort_hist_kernel<kKeysIl><<<grid, 256, 0, stream>>>(p, m, hist, keys, p.T, p.F);
-                sort_scan_kernel<kKeysIl><<<1, 1024, 0, stream>>>(hist, offs, cursor);
-                sort_scatter_kernel<kKeysIl><<<sgrid, 512, 0, stream>>>(keys, m, cursor, perm);
+                e = cudaGetLastError();
+                if (e == cudaSuccess)
+                    e = launch_dependent(sort_scan_kernel<kKeysIl>, 1, 1024, 0, stream, hist, offs,
+                                         cursor);
+                if (e == cudaSuccess)
+                    e = launch_dependent(sort_scatter_kernel<kKeysIl>, sgrid, 512, 0, stream, keys,
+                                         m, chunk, cursor, perm);
             } else {
                 sort_hist_kernel<kKeys><<<grid, 256, 0, stream>>>(p, m, hist, keys, p.T, p.F);
-                sort_scan_kernel<kKeys><<<1, 1024, 0, stream>>>(hist, offs, cursor);
-                sort_scatter_kernel<kKeys><<<sgrid, 512, 0, stream>>>(keys, m, cursor, perm);
+                e = cudaGetLastError();
+                if (e == cudaSuccess)
+                    e = launch_dependent(sort_scan_kernel<kKeys>, 1, 1024, 0, stream, hist, offs,
+                                         cursor);
+                if (e == cudaSuccess)
+                    e = launch_dependent(sort_scatter_kernel<kKeys>, sgrid, 512, 0, stream, keys, m,
+                                         chunk, cursor, perm);
             }
-            e = cudaGetLastError();
         }
         if (e == cudaSuccess) st = launch_decode(p, stream);
         if (e == cudaSuccess && st == POS_OK) {

@@ -256,12 +256,18 @@ __global__ void __launch_bounds__(kEvalThreads, MINB) eval_kernel(EvalParams p) 
     constexpr bool kFast = PATH == kPathFast || PATH == kPathEager;
     const int key_lo = kFast ? fast_key_begin(SLO) : generic_key_begin(SLO);
     const int key_hi = kFast ? fast_key_begin(SHI + 1) : generic_key_begin(SHI + 1);
+    // the key offsets come from the sort's scan, two or more kernels back
     const int64_t begin = p.offs[key_lo], end = p.offs[key_hi];
     // blocks with no candidate (all of them when the range is empty) leave
-    // before staging the tables
-    if ((int64_t)blockIdx.x * blockDim.x >= end - begin) return;
+    // without staging the tables, after the decode pass has completed
+    if ((int64_t)blockIdx.x * blockDim.x >= end - begin) {
+        grid_dep_wait();
+        return;
+    }
     stage_blob(sm, p.blob, p.lay.bytes);
     __syncthreads();
+    grid_dep_wait();  // the decoded records
+    grid_dep_trigger();
     const Tab t = tab_at(sm, p.lay);
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     // whole warps iterate together (ballots below)
@@ -302,8 +308,7 @@ pos_status launch_eval_range(const EvalParams &p, cudaStream_t stream) {
     if (per_sm < 1) return fail(POS_ECUDA, "eval kernel does not fit on an SM");
     const int64_t blocks = (p.n + kEvalThreads - 1) / kEvalThreads;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)per_sm * sm_count()));
-    kern<<<grid, kEvalThreads, smem, stream>>>(p);
-    POS_CUDA(cudaGetLastError());
+    POS_CUDA(launch_dependent(kern, grid, kEvalThreads, smem, stream, p));
     return POS_OK;
 }
 

@@ -229,12 +229,18 @@ __device__ __forceinline__ void il_dispatch(int N, int V, const Tab &t, const ui
 template <int PLO, int PHI, int MINB>
 __global__ void __launch_bounds__(kEvalThreads, MINB) il_eval_kernel(EvalParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
+    // the key offsets come from the sort's scan, two or more kernels back
     const int64_t begin = p.offs[kKeys + IlPair<PLO>::key], end = p.offs[kKeys + IlPair<PHI + 1>::key];
     // blocks with no record (all of them when the range is empty) leave
-    // before staging the tables
-    if ((int64_t)blockIdx.x * blockDim.x >= end - begin) return;
+    // without staging the tables, after the decode pass has completed
+    if ((int64_t)blockIdx.x * blockDim.x >= end - begin) {
+        grid_dep_wait();
+        return;
+    }
     stage_blob(sm, p.blob, p.lay.bytes);
     __syncthreads();
+    grid_dep_wait();  // the decoded records
+    grid_dep_trigger();
     const Tab t = tab_at(sm, p.lay);
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     const int64_t span = ((end - begin) + 31) & ~(int64_t)31;
@@ -291,8 +297,7 @@ pos_status launch_il_range(const EvalParams &p, cudaStream_t stream) {
     if (per_sm < 1) return fail(POS_ECUDA, "interleaved eval kernel does not fit on an SM");
     const int64_t blocks = (p.n + kEvalThreads - 1) / kEvalThreads;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)per_sm * sm_count()));
-    kern<<<grid, kEvalThreads, smem, stream>>>(p);
-    POS_CUDA(cudaGetLastError());
+    POS_CUDA(launch_dependent(kern, grid, kEvalThreads, smem, stream, p));
     return POS_OK;
 }
 

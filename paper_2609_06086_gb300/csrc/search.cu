@@ -697,6 +697,7 @@ __global__ void __launch_bounds__(kThreads, 3) level_kernel(ExpandParams p) {
     }
     if (!bulk_wait(&bar)) {
         if (threadIdx.x == 0) atomicAdd(p.stats + kStBulkTimeout, 1ull);
+        grid_dep_wait();  // a block never leaves before its predecessor has completed
         return;
     }
     // the frontier, its count and the incumbent only after the previous

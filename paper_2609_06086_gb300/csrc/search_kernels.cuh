@@ -175,6 +175,7 @@ __global__ void __launch_bounds__(256, leaf_min_blocks(S, PATH)) leaf_kernel(Lea
     // finishes; the plans and their count only after it has completed
     if (!stage_blob_bulk(sm, p.blob, p.lay.bytes, &bar)) {
         if (threadIdx.x == 0) atomicAdd(p.stats + kStBulkTimeout, 1ull);
+        grid_dep_wait();  // a block never leaves before its predecessor has completed
         return;
     }
     grid_dep_wait();
