@@ -182,7 +182,8 @@ pos_status poseidon_tables_destroy(void *handle);
  * 38*n + 56 KB (Interleaved 1F1B: 38*n + 121 KB) stream-ordered allocation
  * (decoded record 32 B, permutation 4 B and sort key 2 B per candidate, key
  * histograms) from a library-owned memory pool (per device, kept between
- * calls); batches above 2^31 candidates go in chunks of 2^31.
+ * calls); batches above 2^24 candidates go in chunks of 2^24, one after
+ * another.
  * Errors: POS_EINVAL (null handle or pointers, n < 0, misaligned
  * candidates), POS_ENOMEM, POS_ECUDA (launch failure).
  */

@@ -279,8 +279,11 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
     if (st != POS_OK) return st;
     Programs pg;  // the schedule's level programs (Eager 1F1B, few micro-batches)
     if ((st = schedule_programs(h->lay.sched, &pg)) != POS_OK) return st;
-    // permutation indices are 32-bit: batches above 2^31 go in chunks
-    const int64_t chunk = (int64_t)1 << 31;
+    // batches above 2^24 candidates go in chunks of 2^24: a chunk's outputs
+    // (5 bytes per candidate, 80 MB), written in sorted order and so
+    // scattered over the output arrays, stay in L2 until whole sectors are
+    // written back (the permutation's 32-bit indices would allow 2^31)
+    const int64_t chunk = (int64_t)1 << 24;
     for (int64_t base = 0; base < n; base += chunk) {
         const int64_t m = std::min(chunk, n - base);
         void *scratch = nullptr;

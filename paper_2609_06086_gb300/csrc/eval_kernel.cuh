@@ -42,7 +42,9 @@ struct EvalParams {
     uint8_t *F;
     const uint32_t *perm;  // sorted candidate indices
     const uint32_t *offs;  // [nkeys + 1] start of every key in perm
-    uint4 *cuts;           // per sorted position j, two 16-byte words:
+    uint4 *cuts;           // per sorted position j, two 16-byte words (read once,
+                           // with evict-first loads, so that the outputs'
+                           // sectors stay in L2):
                            // cuts[2j]: cut[1..S-1] in bytes 0..14, byte 15 = 1
                            // when the result is already written;
                            // cuts[2j+1]: (candidate index, type_code, the
@@ -277,8 +279,8 @@ __global__ void __launch_bounds__(kEvalThreads, MINB) eval_kernel(EvalParams p) 
         uint32_t i = 0;
         uint4 rec = make_uint4(0, 0, 0, 0), packed = make_uint4(0, 0, 0, 0);
         if (active) {
-            packed = __ldg(p.cuts + 2 * (begin + j));
-            const uint4 meta = __ldg(p.cuts + 2 * (begin + j) + 1);
+            packed = __ldcs(p.cuts + 2 * (begin + j));
+            const uint4 meta = __ldcs(p.cuts + 2 * (begin + j) + 1);
             active = (packed.w >> 24) == 0;  // not answered by the decode pass
             i = meta.x;
             rec = make_uint4(meta.w, 0u, meta.y, meta.z);

@@ -250,8 +250,8 @@ __global__ void __launch_bounds__(kEvalThreads, MINB) il_eval_kernel(EvalParams 
     const uint4 none = make_uint4(0, 0, 0, 1u << 24);
     uint4 next_packed = none, next_meta = none;
     if (j < end - begin) {
-        next_packed = __ldg(p.cuts + 2 * (begin + j));
-        next_meta = __ldg(p.cuts + 2 * (begin + j) + 1);
+        next_packed = __ldcs(p.cuts + 2 * (begin + j));
+        next_meta = __ldcs(p.cuts + 2 * (begin + j) + 1);
     }
     for (; j < span; j += stride) {
         bool active = j < end - begin;
@@ -260,8 +260,8 @@ __global__ void __launch_bounds__(kEvalThreads, MINB) il_eval_kernel(EvalParams 
         const uint4 packed = next_packed, meta = next_meta;
         next_packed = none;
         if (j + stride < end - begin) {
-            next_packed = __ldg(p.cuts + 2 * (begin + j + stride));
-            next_meta = __ldg(p.cuts + 2 * (begin + j + stride) + 1);
+            next_packed = __ldcs(p.cuts + 2 * (begin + j + stride));
+            next_meta = __ldcs(p.cuts + 2 * (begin + j + stride) + 1);
         }
         if (active) {
             active = (packed.w >> 24) == 0;  // not answered by the decode pass
