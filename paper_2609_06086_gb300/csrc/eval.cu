@@ -149,12 +149,13 @@ __global__ void __launch_bounds__(1024) sort_scan_kernel(const uint32_t *hist, u
 }
 
 // Each block takes chunks of `chunk` candidates: counts their keys, reserves
-// one range per key with a single atomic, then places the indices.  The
-// chunk grows with the batch (about two chunks per SM, 2048 to 65536), so
-// that large batches reserve fewer ranges.
+// one range per key with a single atomic, then places the indices.  Chunks
+// of 8192 for large batches (measured: 65536-candidate chunks, with fewer
+// reservations but fewer blocks, took 112 instead of 89 us at 1e7), smaller
+// ones (down to 1024) so that small batches still spread over the SMs.
 __host__ inline int64_t scatter_chunk(int64_t n, int sms) {
-    int64_t c = (n / (2 * (int64_t)sms) + 511) & ~(int64_t)511;
-    return c < 2048 ? 2048 : (c > 65536 ? 65536 : c);
+    int64_t c = (n / (8 * (int64_t)sms) + 511) & ~(int64_t)511;
+    return c < 1024 ? 1024 : (c > 8192 ? 8192 : c);
 }
 
 template <int NK>
