@@ -203,9 +203,9 @@ __device__ __forceinline__ uint64_t binom(const Tab &t, int n, int k) {
 // j in [k, rem-1] with C(j, k) >= Y (the stage takes rem - j layers); returns
 // j and lowers rank to C(j, k) - Y.  C(j, k) grows with j.  Since
 // C(j, k) ~ (j - (k-1)/2)^k / k!, j is first estimated as
-// (Y k!)^(1/k) + (k-1)/2 with single-precision log2 / exp2, then moved by
-// exact comparisons to the answer (at most two steps either way over every
-// L <= 127, k <= 15, and exact whatever the estimate).  When
+// (Y k!)^(1/k) + (k-1)/2 with the hardware's approximate log2 / exp2, then
+// moved by exact comparisons to the answer (a step or two either way in
+// practice, and exact whatever the estimate).  When
 // C(rem-1, k) < 2^32, every C(j, k) it reads is below 2^32 too and the
 // comparisons use the low halves.
 __device__ __constant__ static const float kLog2Fact[16] = {
@@ -218,7 +218,11 @@ __device__ __constant__ static const float kInvK[16] = {
     0.083333333f, 0.076923077f, 0.071428571f, 0.066666667f};
 
 __device__ __forceinline__ int unrank_guess(float Yf, int k, int rem) {
-    const float e = exp2f((__log2f(Yf) + kLog2Fact[k]) * kInvK[k]) + 0.5f * (float)(k - 1);
+    // an estimate only (the exact comparisons that follow fix any error), so
+    // the hardware approximations of log2 and exp2 serve
+    // 2^x as the intrinsic __expf(x ln 2)
+    const float e = __expf((__log2f(Yf) + kLog2Fact[k]) * kInvK[k] * 0.693147181f) +
+                    0.5f * (float)(k - 1);
     return min(max((int)e, k), rem - 1);
 }
 

@@ -1019,15 +1019,17 @@ static pos_status device_sequences(const pos_problem *p, int units, int D,
     k_at[0] = -1;
     while (u >= 0) {  // iterative depth-first walk, classes in ascending order
         if (u == units - 1) {
-            // the last stage takes what is left: one type with a budget equal
-            // to a TP degree (the prefix was kept only if such a class exists)
-            for (int k = 0; k < K; ++k) {
-                const int t = k / n_tp;
-                bool only = bud[t] == p->tp_list[k % n_tp];
-                for (int o = 0; o < T && only; ++o) only = o == t || bud[o] == 0;
-                if (!only) continue;
-                seq[u] = (uint8_t)k;
-                out.insert(out.end(), seq, seq + units);
+            // the last stage takes what is left: the one type with a budget
+            // left, with a TP degree equal to it (the prefix was kept only if
+            // such a class exists)
+            int t = 0;
+            while (t < T && bud[t] == 0) ++t;
+            for (int j = 0; t < T && j < n_tp; ++j) {
+                if (p->tp_list[j] != bud[t]) continue;
+                seq[u] = (uint8_t)(t * n_tp + j);
+                const size_t at = out.size();
+                out.resize(at + units);
+                std::memcpy(out.data() + at, seq, units);
                 if (++*total > limit) return fail(POS_EINVAL, "more than 2^22 class sequences");
             }
             --u;  // the parent's class is undone on its next step
