@@ -138,22 +138,36 @@ __global__ void feas_kernel(const SliceRec *slices, int n_slices, int S, uint4 *
 // root_lb[slice] = V1[0][0] * scale, a lower bound on the slice's objective.
 constexpr int kBoundThreads = 512;
 
+// rows = NULL: row r is slice r, for every slice (n_rows = the slice count);
+// a slice whose root is infeasible (root[r] == 0) then gets a hole for its
+// greedy plan and an infinite root bound, and no table rows.
 __global__ void __launch_bounds__(kBoundThreads) bound_kernel(
-    const SliceRec *slices, const uint32_t *rows, int n_rows, int S, const uint8_t *lim,
-    int2 *vb, Leaf *greedy, unsigned long long *root_lb, const void *blob, BlobLayout lay,
-    unsigned long long *stats) {
+    const SliceRec *slices, const uint32_t *rows, const uint8_t *root, int n_rows, int S,
+    const uint8_t *lim, int2 *vb, Leaf *greedy, unsigned long long *root_lb, const void *blob,
+    BlobLayout lay, unsigned long long *stats) {
     extern __shared__ __align__(16) unsigned char sm[];
     __shared__ int2 nxt[128];
     __shared__ uint8_t arg[POS_MAX_STAGES][128];
     __shared__ uint64_t bar;
     if (!stage_blob_bulk(sm, blob, lay.bytes, &bar)) {
         if (threadIdx.x == 0) atomicAdd(stats + kStBulkTimeout, 1ull);
+        grid_dep_wait();  // a block never leaves before its predecessor has completed
         return;
     }
+    grid_dep_wait();  // the memory-limit rows and root bits (feasibility kernel)
+    grid_dep_trigger();
     const Tab t = tab_at(sm, lay);
     const int L = lay.L, c = threadIdx.x >> 2, part = threadIdx.x & 3;
     for (int r = blockIdx.x; r < n_rows; r += gridDim.x) {
-        const uint32_t sl = rows[r];
+        const uint32_t sl = rows ? rows[r] : (uint32_t)r;
+        if (!rows && !root[sl]) {  // the same for the whole block
+            if (threadIdx.x == 0) {
+                const Vec32 hole = {make_uint4(kLeafHole, 0, 0, 0), make_uint4(0, 0, 0, 0)};
+                store32(greedy + r, hole);
+                root_lb[sl] = ~0ull;
+            }
+            continue;
+        }
         const SliceRec &sr = slices[sl];
         const int M = sr.M;
         const uint32_t vslot = sr.vslot;
@@ -1457,6 +1471,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
                     r.M = p->M_list[mi];
                     r.scale = Q / ((uint64_t)sp.D[g] * p->M_list[mi]);
                     r.gid = (uint32_t)ord;
+                    r.vslot = (uint32_t)ord;  // bound-table row when every slice has one
                     for (int x = 0; x < s.S; ++x) r.cls[x] = (uint8_t)sp.cls(g, pr, x, s.n_tp);
                 }
     }
@@ -1498,24 +1513,76 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     POS_CUDA(cudaGetLastError());
     s.launches++;
     std::vector<uint8_t> root(n_slices);
-    if ((st = sync_read(s, root.data(), d_root.p, n_slices)) != POS_OK) return st;
-    // feasible slices, grouped by M index
-    std::vector<std::vector<uint32_t>> feas_by_m(p->n_M);
+    std::vector<std::vector<uint32_t>> feas_by_m(p->n_M);  // feasible slices per M index
     uint64_t n_feasible = 0;
-    for (int i = 0; i < n_slices; ++i)
-        if (root[i]) {
-            feas_by_m[i / sp.per_m].push_back((uint32_t)i);
-            ++n_feasible;
+    auto list_feasible = [&]() {
+        for (int i = 0; i < n_slices; ++i)
+            if (root[i]) {
+                feas_by_m[i / sp.per_m].push_back((uint32_t)i);
+                ++n_feasible;
+            }
+    };
+    uint64_t warm_evals = 0;
+    // prune mode 2 with tables for every slice small enough (up to 256 MB):
+    // the completion bounds of all slices right after the feasibility kernel
+    // (the infeasible ones skip out), no host round trip in between; the
+    // root bits come back with the root bounds
+    const bool bound_all = p->prune == 2 && (uint64_t)n_slices * s.S * 1024 <= (256ull << 20);
+    if (bound_all) {
+        s.n_vrows = n_slices;  // table row = slice index (vslot = gid)
+        POS_CUDA(s.ws.d_vb.reserve(sizeof(int2) * 128 * (size_t)s.S * n_slices));
+        POS_CUDA(s.ws.d_greedy.reserve(sizeof(Leaf) * n_slices));
+        POS_CUDA(s.ws.d_lb.reserve(sizeof(unsigned long long) * n_slices));
+        const BlobLayout tl = timing_layout(s.h->lay);
+        POS_TRY(ensure_smem(reinterpret_cast<const void *>(bound_kernel), tl.bytes));
+        if (p->profile) POS_CUDA(cudaEventRecord(s.ev[0], s.stream));
+        POS_CUDA(launch_dependent(
+            bound_kernel, std::min(n_slices, 8 * sm_count()), kBoundThreads, tl.bytes, s.stream,
+            d_all, static_cast<const uint32_t *>(nullptr),
+            static_cast<const uint8_t *>(d_root.p), n_slices, s.S,
+            static_cast<const uint8_t *>(s.ws.d_lim.p), static_cast<int2 *>(s.ws.d_vb.p),
+            static_cast<Leaf *>(s.ws.d_greedy.p), static_cast<unsigned long long *>(s.ws.d_lb.p),
+            static_cast<const void *>(static_cast<const unsigned char *>(s.h->d_blob) +
+                                      s.h->lay.off_Pf),
+            tl, s.stats));
+        if (p->profile) POS_CUDA(cudaEventRecord(s.ev[1], s.stream));
+        s.launches++;
+        s.n_bound++;
+        // the greedy plans of each M index (holes for the infeasible slices)
+        std::vector<unsigned long long> gc(p->n_M, (unsigned long long)sp.per_m);
+        POS_CUDA(s.ws.d_wcnt.reserve(sizeof(unsigned long long) * p->n_M));
+        POS_TRY(upload(s, s.ws.d_wcnt.p, gc.data(), sizeof(unsigned long long) * p->n_M));
+        for (int mi = 0; mi < p->n_M; ++mi)
+            if ((st = run_leaves(s, static_cast<const Leaf *>(s.ws.d_greedy.p) + mi * sp.per_m,
+                                 static_cast<unsigned long long *>(s.ws.d_wcnt.p) + mi, d_all,
+                                 p->M_list[mi], static_cast<unsigned long long *>(s.d_best.p))) !=
+                POS_OK)
+                return st;
+        if ((size_t)n_slices > s.ws.h_lb_cap) {
+            POS_CUDA(cudaStreamSynchronize(s.stream));  // no copy into the old area in flight
+            if (s.ws.h_lb) cudaFreeHost(s.ws.h_lb);
+            s.ws.h_lb = nullptr;
+            s.ws.h_lb_cap = 0;
+            POS_CUDA(cudaMallocHost(&s.ws.h_lb, sizeof(unsigned long long) * n_slices));
+            s.ws.h_lb_cap = (size_t)n_slices;
         }
+        const ReadPart parts[2] = {{root.data(), d_root.p, (size_t)n_slices},
+                                   {s.ws.h_lb, s.ws.d_lb.p, sizeof(unsigned long long) * n_slices}};
+        if ((st = sync_read_many(s, parts, 2)) != POS_OK) return st;
+        list_feasible();
+        for (int mi = 0; mi < p->n_M; ++mi) warm_evals += feas_by_m[mi].size();
+    } else {
+        if ((st = sync_read(s, root.data(), d_root.p, n_slices)) != POS_OK) return st;
+        list_feasible();
+    }
     const double ms_setup = ms_since(t_start);
 
     // prune mode 2: completion-bound tables of every memory-feasible slice
     // (one launch), and each slice's argmin completion as a warm-up plan
     const auto t_warm = std::chrono::steady_clock::now();
-    uint64_t warm_evals = 0;
     std::vector<size_t> feas_off(p->n_M + 1, 0);  // first row of each M index
     for (int mi = 0; mi < p->n_M; ++mi) feas_off[mi + 1] = feas_off[mi] + feas_by_m[mi].size();
-    if (p->prune == 2 && n_feasible > 0) {
+    if (p->prune == 2 && n_feasible > 0 && !bound_all) {
         std::vector<uint32_t> rows;
         rows.reserve(n_feasible);
         for (int mi = 0; mi < p->n_M; ++mi)
@@ -1535,7 +1602,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         if (p->profile) POS_CUDA(cudaEventRecord(s.ev[0], s.stream));
         bound_kernel<<<(int)std::min<size_t>(rows.size(), 8 * sm_count()), kBoundThreads, tl.bytes,
                        s.stream>>>(
-            d_all, static_cast<const uint32_t *>(s.ws.d_rows.p), (int)rows.size(), s.S,
+            d_all, static_cast<const uint32_t *>(s.ws.d_rows.p), nullptr, (int)rows.size(), s.S,
             static_cast<const uint8_t *>(s.ws.d_lim.p), static_cast<int2 *>(s.ws.d_vb.p),
             static_cast<Leaf *>(s.ws.d_greedy.p), static_cast<unsigned long long *>(s.ws.d_lb.p),
             static_cast<const unsigned char *>(s.h->d_blob) + s.h->lay.off_Pf, tl, s.stats);
@@ -1607,7 +1674,7 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     const bool by_bound = p->prune == 2 && n_feasible > 0;
     std::vector<unsigned long long> key(n_slices);
     if (by_bound) {
-        POS_CUDA(cudaEventSynchronize(s.ws.ev_lb));
+        if (!bound_all) POS_CUDA(cudaEventSynchronize(s.ws.ev_lb));  // else read already
         std::memcpy(key.data(), s.ws.h_lb, sizeof(unsigned long long) * n_slices);
     } else if ((st = sync_read(s, key.data(), s.d_best.p,
                                sizeof(unsigned long long) * n_slices)) != POS_OK) {
