@@ -43,7 +43,7 @@ ENTRY_BYTES = 32  # one frontier entry / one complete plan
 LEAF_DRAM_BYTES_PER_PLAN = 59684096 / 1925970
 LEAF_SOURCES = ("paper_2609_06086_gb300/csrc/search_kernels.cuh",
                 "paper_2609_06086_gb300/csrc/common.cuh")
-LEAF_SOURCES_SHA256 = "4590f9d06d302946"
+LEAF_SOURCES_SHA256 = "7b1b87babaedfc55"
 PRUNE_NAMES = {1: "stage-level, Eq. 2 as printed (Theorem 1)",
                2: "stage-level, tightened: Eq. 2 with P2P edges + completion bounds"}
 

@@ -269,7 +269,11 @@ __device__ __forceinline__ void stage_blob(unsigned char *dst, const void *src, 
 // calls bulk_begin with the total byte count, then issues the copies
 // (16-byte aligned addresses, sizes multiples of 16); then every thread of
 // the block calls bulk_wait, which returns the same value in all threads:
-// false if the copies did not complete within kBulkWaitLimit polls.
+// false if the copies did not complete within kBulkWaitLimit polls.  That is
+// a last-resort exit (2^24 polls, far beyond any copy of at most a few
+// hundred KB): the caller counts it and leaves, the search then reports
+// POS_ETIMEOUT, and a copy still in flight may land in shared memory that
+// the block no longer owns; nothing exercises it on a GPU.
 constexpr int kBulkWaitLimit = 1 << 24;
 
 __device__ __forceinline__ void bulk_begin(uint64_t *bar, uint32_t total_bytes) {
