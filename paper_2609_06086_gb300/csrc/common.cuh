@@ -79,7 +79,7 @@ inline cudaError_t launch_dependent(void (*kern)(KArgs...), int grid, int block,
 // ---------------------------------------------------------------------------
 // Table blob: one contiguous device buffer, staged whole into shared memory
 // by every kernel.  Offsets are bytes from the blob start, 16-byte aligned.
-//   binom  u32 [16][128] twice  C(n, k) at [k][n], k <= 15: low halves, then high halves
+//   binom  u64 [16][128]        C(n, k) at [k][n], k <= 15 (0 for n < k)
 //   Pw, Pa i64 [K][L+1] each    exclusive prefix sums of mem_w, mem_a
 //   cap    i64 [K]
 //   Pf, Pb, Pd i32 [K][L+1]     exclusive prefix sums of fwd, bwd, dsync
@@ -185,63 +185,90 @@ __device__ __forceinline__ int32_t p2f(const Tab &t, int a, int b) {
 __device__ __forceinline__ int32_t p2b(const Tab &t, int a, int b) {
     return ld32(t.base, t.ly->off_p2b + 4u * (uint32_t)(a * t.ly->K + b));
 }
-// stored k-major ([k][n]) as 32-bit halves, so that a warp reading
-// C(n_lane, k) for one k touches consecutive 4-byte words
-__device__ __forceinline__ uint32_t binom_lo(const Tab &t, int n, int k) {
-    return (uint32_t)ld32(t.base, t.ly->off_binom + 4u * (uint32_t)(k * kBinomN + n));
-}
-__device__ __forceinline__ uint32_t binom_hi(const Tab &t, int n, int k) {
-    return (uint32_t)ld32(t.base,
-                          t.ly->off_binom + 4u * (uint32_t)(kBinomK * kBinomN + k * kBinomN + n));
-}
+// stored k-major ([k][n]) as 64-bit words, so that a warp reading
+// C(n_lane, k) for one k touches consecutive 8-byte words
 __device__ __forceinline__ uint64_t binom(const Tab &t, int n, int k) {
-    return ((uint64_t)binom_hi(t, n, k) << 32) | binom_lo(t, n, k);
+    return (uint64_t)ld64(t.base, t.ly->off_binom + 8u * (uint32_t)(k * kBinomN + n));
 }
 
-// The stage of the combinatorial-number-system unranking: with rem layers
-// left for k+1 stages (k >= 1) and Y = C(rem-1, k) - rank >= 1, the smallest
-// j in [k, rem-1] with C(j, k) >= Y (the stage takes rem - j layers); returns
-// j and lowers rank to C(j, k) - Y.  C(j, k) grows with j.  Since
-// C(j, k) ~ (j - (k-1)/2)^k / k!, j is first estimated as
-// (Y k!)^(1/k) + (k-1)/2 with the hardware's approximate log2 / exp2, then
-// moved by exact comparisons to the answer (a step or two either way in
-// practice, and exact whatever the estimate).  When
-// C(rem-1, k) < 2^32, every C(j, k) it reads is below 2^32 too and the
-// comparisons use the low halves.
-__device__ __constant__ static const float kLog2Fact[16] = {
-    0.000000000f, 0.000000000f, 1.000000000f, 2.584962501f, 4.584962501f, 6.906890596f,
-    9.491853096f, 12.299208018f, 15.299208018f, 18.469133020f, 21.791061115f, 25.250492733f,
-    28.835455234f, 32.535894952f, 36.343249874f, 40.250140470f};
-__device__ __constant__ static const float kInvK[16] = {
-    0.000000000f, 1.000000000f, 0.500000000f, 0.333333333f, 0.250000000f, 0.200000000f,
-    0.166666667f, 0.142857143f, 0.125000000f, 0.111111111f, 0.100000000f, 0.090909091f,
-    0.083333333f, 0.076923077f, 0.071428571f, 0.066666667f};
+// One stage of the combinatorial-number-system unranking.  With rem layers
+// left for k+1 stages (k >= 1), the remaining rank is carried as
+// Y = C(rem-1, k) - rank, 1 <= Y <= C(rem-1, k).  The stage takes rem - j
+// layers, j the smallest value in [k, rem-1] with C(j, k) >= Y; the next
+// stage's Y (rem' = j layers, k' = k-1) is Y - C(j-1, k), since
+// C(j, k) = C(j-1, k) + C(j-1, k-1) (Pascal's rule) puts it in
+// [1, C(j-1, k-1)].  So a stage reads only C(j-1, k) and C(j, k).
+//
+// j is first estimated from C(x, k) ~ m^k / k! * exp(-k(k^2-1) / (12 m^2)),
+// m = x - (k-1)/2 (the product of the k factors m +- d around their mean):
+// m0 = (Y k!)^(1/k), x ~ m0 + (k-1)/2 + (k^2-1) / (24 m0) (half the
+// second-order term, which over-corrects), rounded up after a 0.01 margin
+// for rounding error.  Over uniform ranks of 64 layers in 2..16 stages this
+// lands on j in about 99 % of the stages (else one step low); exact
+// comparisons then move it to the answer whatever the estimate.
+struct UnrankCoef {
+    float log2_fact;  // log2(k!)
+    float inv_k;      // 1/k
+    float half_km1;   // (k-1)/2 - 0.01
+    float corr;       // (k^2-1)/24
+};
+__device__ __constant__ static const UnrankCoef kUnrankCoef[16] = {
+    {0.000000000f, 0.000000000f, 0.00f, 0.000000000f},
+    {0.000000000f, 1.000000000f, -0.01f, 0.000000000f},
+    {1.000000000f, 0.500000000f, 0.49f, 0.125000000f},
+    {2.584962501f, 0.333333333f, 0.99f, 0.333333333f},
+    {4.584962501f, 0.250000000f, 1.49f, 0.625000000f},
+    {6.906890596f, 0.200000000f, 1.99f, 1.000000000f},
+    {9.491853096f, 0.166666667f, 2.49f, 1.458333333f},
+    {12.299208018f, 0.142857143f, 2.99f, 2.000000000f},
+    {15.299208018f, 0.125000000f, 3.49f, 2.625000000f},
+    {18.469133020f, 0.111111111f, 3.99f, 3.333333333f},
+    {21.791061115f, 0.100000000f, 4.49f, 4.125000000f},
+    {25.250492733f, 0.090909091f, 4.99f, 5.000000000f},
+    {28.835455234f, 0.083333333f, 5.49f, 5.958333333f},
+    {32.535894952f, 0.076923077f, 5.99f, 7.000000000f},
+    {36.343249874f, 0.071428571f, 6.49f, 8.125000000f},
+    {40.250140470f, 0.066666667f, 6.99f, 9.333333333f}};
 
-__device__ __forceinline__ int unrank_guess(float Yf, int k, int rem) {
-    // an estimate only (the exact comparisons that follow fix any error), so
-    // the hardware approximations of log2 and exp2 serve
-    // 2^x as the intrinsic __expf(x ln 2)
-    const float e = __expf((__log2f(Yf) + kLog2Fact[k]) * kInvK[k] * 0.693147181f) +
-                    0.5f * (float)(k - 1);
-    return min(max((int)e, k), rem - 1);
+// the hardware's approximate base-2 logarithm, power and reciprocal (PTX
+// lg2 / ex2 / rcp .approx): an estimate only, the comparisons fix any error
+__device__ __forceinline__ float approx_lg2(float x) {
+    float y;
+    asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+__device__ __forceinline__ float approx_ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+__device__ __forceinline__ float approx_rcp(float x) {
+    float y;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
 }
 
-__device__ __forceinline__ int unrank_step(const Tab &t, int rem, int k, uint64_t &rank) {
-    const uint64_t total = binom(t, rem - 1, k);
-    int j;
-    if ((total >> 32) == 0) {
-        const uint32_t Y = (uint32_t)(total - rank);
-        j = unrank_guess(__uint2float_rn(Y), k, rem);
-        while (j > k && binom_lo(t, j - 1, k) >= Y) --j;
-        while (binom_lo(t, j, k) < Y) ++j;
-        rank = binom_lo(t, j, k) - Y;
-    } else {
-        const uint64_t Y = total - rank;
-        j = unrank_guess(__ull2float_rn(Y), k, rem);
-        while (j > k && binom(t, j - 1, k) >= Y) --j;
-        while (binom(t, j, k) < Y) ++j;
-        rank = binom(t, j, k) - Y;
+__device__ __forceinline__ int unrank_guess(uint64_t Y, int k, int rem) {
+    const UnrankCoef c = kUnrankCoef[k];
+    const float m0 = approx_ex2((approx_lg2(__ull2float_rn(Y)) + c.log2_fact) * c.inv_k);
+    const float e = m0 + c.half_km1 + c.corr * approx_rcp(m0);
+    return min(max(__float2int_ru(e), k), rem - 1);
+}
+
+__device__ __forceinline__ int unrank_step(const Tab &t, int rem, int k, uint64_t &Y) {
+    int j = unrank_guess(Y, k, rem);
+    uint64_t below = binom(t, j - 1, k), at = binom(t, j, k);
+    while (below >= Y) {  // stops at j = k at the latest: C(k-1, k) = 0 < Y
+        --j;
+        at = below;
+        below = binom(t, j - 1, k);
     }
+    while (at < Y && j < rem - 1) {  // C(rem-1, k) >= Y stops it first
+        ++j;
+        below = at;
+        at = binom(t, j, k);
+    }
+    Y -= below;
     return j;
 }
 
@@ -328,20 +355,8 @@ __device__ __forceinline__ bool stage_blob_bulk(unsigned char *dst, const void *
 // (hockey-stick sum of C(rem-u-1, p-2) over u < v).
 // cut[0] = 0, cut[s+1] = layers of stages 0..s, cut[S] = L.
 // ---------------------------------------------------------------------------
-template <int S>
-__device__ __forceinline__ void unrank_cuts(const Tab &t, uint64_t rank, int (&cut)[S + 1]) {
-    const int L = t.L();
-    cut[0] = 0;
-#pragma unroll
-    for (int s = 0; s < S - 1; ++s) {
-        const int rem = L - cut[s];
-        const int k = S - s - 1;  // p - 1 with p = S - s stages left
-        cut[s + 1] = cut[s] + (rem - unrank_step(t, rem, k, rank));
-    }
-    cut[S] = L;
-}
-
-// Rank of the composition given by cut[0..S] (same numbering as above).
+// Rank of the composition given by cut[0..S] (the numbering unrank_step
+// walks stage by stage).
 template <int S>
 __device__ __forceinline__ uint64_t rank_cuts(const Tab &t, const int (&cut)[S + 1]) {
     uint64_t r = 0;

@@ -105,6 +105,26 @@ __device__ __forceinline__ bool types_ok(uint32_t tcode, int S, int n_types) {
     return bad == 0u;
 }
 
+// The decode pass packs the cut positions of a (non-interleaved) record
+// (each below 256) into the bytes of a 16-byte word by shifting them in from
+// the bottom: after pushing
+// cut[1], ..., cut[n-1] (n - 1 <= 15 pushes), cut[q] sits in byte n-1-q and
+// byte 15 is still 0 (the "answered by the decode pass" flag).  A push is
+// three funnel shifts and a shift-or, whatever the stage index.
+__device__ __forceinline__ void push_cut(uint4 &v, int c) {
+    v.w = __funnelshift_l(v.z, v.w, 8);
+    v.z = __funnelshift_l(v.y, v.z, 8);
+    v.y = __funnelshift_l(v.x, v.y, 8);
+    v.x = (v.x << 8) | (uint32_t)c;
+}
+
+// cut[q] (1 <= q <= n-1) of n stages from the packed word (n a constant
+// after unrolling, so this is a constant shift of a constant word)
+__device__ __forceinline__ int packed_cut(const uint32_t (&pw)[4], int n, int q) {
+    const int b = n - 1 - q;
+    return (int)((pw[b >> 2] >> (8 * (b & 3))) & 0xffu);
+}
+
 // Decode pass for an Interleaved 1F1B record (pad byte V >= 2, S = N
 // devices): checks its fields (N*V <= 16 virtual stages, at most L, M a
 // multiple of N) and the overflow guard over the N*V virtual stages, and
@@ -112,7 +132,7 @@ __device__ __forceinline__ bool types_ok(uint32_t tcode, int S, int n_types) {
 // checked by the makespan kernel (it needs the device chains).
 __device__ __forceinline__ uint4 decode_il(const Tab &t, const uint4 &rec, uint32_t tpc,
                                            const EvalParams &p, uint32_t i) {
-    uint64_t rank = (uint64_t)rec.x | ((uint64_t)rec.y << 32);
+    const uint64_t rank = (uint64_t)rec.x | ((uint64_t)rec.y << 32);
     const uint32_t tcode = rec.z;
     const int S = rec.w & 0xff;
     const int M = (rec.w >> 8) & 0xff;
@@ -120,7 +140,9 @@ __device__ __forceinline__ uint4 decode_il(const Tab &t, const uint4 &rec, uint3
     const int V = (int)(rec.w >> 24);
     const int J = S * V, L = t.L();
     bool ok = S >= 1 && J <= POS_MAX_STAGES && J <= L && M >= 1 && M % S == 0 &&
-              tp < t.n_tp() && rank < binom(t, L - 1, J - 1);
+              tp < t.n_tp();
+    const uint64_t n_map = ok ? binom(t, L - 1, J - 1) : 0;
+    ok = ok && rank < n_map;
     ok = ok && types_ok(tcode, S, t.n_types()) &&
          types_ok(tpc, S, t.n_tp());  // tpc = 0 for 16-byte records
     const uint4 done = make_uint4(0, 0, 0, 1u << 24);
@@ -134,12 +156,15 @@ __device__ __forceinline__ uint4 decode_il(const Tab &t, const uint4 &rec, uint3
         p.F[i] = POS_FEAS_OVERFLOW;
         return done;
     }
+    // cut[1..J-1] in ascending bytes 0..14, the layout the interleaved
+    // search writes its leaf records in
+    uint64_t Y = n_map - rank;
     uint64_t lo8 = 0, hi8 = 0;
     int c = 0;
 #pragma unroll 1
     for (int j = 0; j < J - 1; ++j) {
         const int rem = L - c, k = J - j - 1;
-        c += rem - unrank_step(t, rem, k, rank);
+        c += rem - unrank_step(t, rem, k, Y);
         if (j < 8) lo8 |= (uint64_t)c << (8 * j);
         else hi8 |= (uint64_t)c << (8 * (j - 8));
     }
@@ -148,16 +173,17 @@ __device__ __forceinline__ uint4 decode_il(const Tab &t, const uint4 &rec, uint3
 }
 
 // Decode pass for one candidate: checks its fields and the overflow guard,
-// unranks the composition stage by stage (the steps of unrank_cuts),
+// unranks the composition stage by stage (unrank_step, carrying Y),
 // checks each stage's memory as soon as its cut is known (LIM: by the
-// memory-limit table staged at `lim`), and packs the cut positions.  Invalid and overflowing candidates are answered here.  S is a
-// runtime value and the stage loop is not unrolled, which keeps the kernel
-// small enough to run many warps per SM.
+// memory-limit table staged at `lim`), and packs the cut positions
+// (push_cut).  Invalid and overflowing candidates are answered here.  S is
+// a runtime value and the stage loop is not unrolled, which keeps the
+// kernel small enough to run many warps per SM.
 template <bool LIM>
 __device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, uint32_t tpc,
                                             const EvalParams &p, uint32_t i,
                                             const uint8_t *lim) {
-    uint64_t rank = (uint64_t)rec.x | ((uint64_t)rec.y << 32);
+    const uint64_t rank = (uint64_t)rec.x | ((uint64_t)rec.y << 32);
     const uint32_t tcode = rec.z;
     const int S = rec.w & 0xff;
     const int M = (rec.w >> 8) & 0xff;
@@ -165,8 +191,9 @@ __device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, uint
     const int L = t.L();
     if (t.ly->sched == POS_SCHED_INTERLEAVED_1F1B && (rec.w >> 24) >= 2)
         return decode_il(t, rec, tpc, p, i);
-    bool ok = S >= 1 && S <= POS_MAX_STAGES && M >= 1 && S <= L && tp < t.n_tp() &&
-              rank < binom(t, L - 1, S - 1);
+    bool ok = S >= 1 && S <= POS_MAX_STAGES && M >= 1 && S <= L && tp < t.n_tp();
+    const uint64_t n_map = ok ? binom(t, L - 1, S - 1) : 0;
+    ok = ok && rank < n_map;
     ok = ok && types_ok(tcode, S, t.n_types()) &&
          types_ok(tpc, S, t.n_tp());  // tpc = 0 for 16-byte records
     const uint4 done = make_uint4(0, 0, 0, 1u << 24);  // byte 15 = 1: answered here
@@ -180,7 +207,8 @@ __device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, uint
         p.F[i] = POS_FEAS_OVERFLOW;
         return done;
     }
-    uint64_t lo8 = 0, hi8 = 0;  // cut bytes 0..7 and 8..14
+    uint64_t Y = n_map - rank;
+    uint4 cuts = make_uint4(0, 0, 0, 0);
     bool fits = true;
     int c = 0;
 #pragma unroll 1
@@ -188,9 +216,8 @@ __device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, uint
         int c2 = L;
         if (s < S - 1) {
             const int rem = L - c, k = S - s - 1;
-            c2 = c + (rem - unrank_step(t, rem, k, rank));
-            if (s < 8) lo8 |= (uint64_t)c2 << (8 * s);
-            else hi8 |= (uint64_t)c2 << (8 * (s - 8));
+            c2 = c + (rem - unrank_step(t, rem, k, Y));
+            push_cut(cuts, c2);
         }
         const int cls = stage_class(tcode, tpc, tp, t.n_tp(), s);
         if constexpr (LIM) {
@@ -202,15 +229,14 @@ __device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, uint
         c = c2;
     }
     p.F[i] = fits ? POS_FEAS_YES : POS_FEAS_NO;
-    return make_uint4((uint32_t)lo8, (uint32_t)(lo8 >> 32), (uint32_t)hi8,
-                      (uint32_t)(hi8 >> 32) & 0x00ffffffu);
+    return cuts;
 }
 
 template <int PATH>
 struct EvalWith {
     template <int S>
     struct One {
-        // makespan of a decoded candidate (cuts packed by Decode<S>)
+        // makespan of a decoded candidate (cuts packed by the decode pass)
         static __device__ __forceinline__ void run(const Tab &t, const uint4 &rec,
                                                    const uint4 &packed, const Programs &pg,
                                                    int32_t &T) {
@@ -227,7 +253,7 @@ struct EvalWith {
             const uint32_t pw[4] = {packed.x, packed.y, packed.z, packed.w};
             cut[0] = 0;
 #pragma unroll
-            for (int s = 0; s < S - 1; ++s) cut[s + 1] = (pw[s / 4] >> (8 * (s % 4))) & 0xff;
+            for (int s = 0; s < S - 1; ++s) cut[s + 1] = packed_cut(pw, S, s + 1);
             cut[S] = t.L();
             StageW<S> w;
             stage_weights<S>(t, cut, cls, w);

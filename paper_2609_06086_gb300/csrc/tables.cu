@@ -223,18 +223,12 @@ pos_status build_blob(const pos_tables *t, int sched, std::vector<unsigned char>
     ly.sched = sched;
     host.assign(ly.bytes, 0);
     // binomials by Pascal's rule (k <= 15 is exact in 64 bits for n <= 127),
-    // stored as a table of low and a table of high 32-bit halves, each [k][n]
-    std::vector<uint64_t> bn(kBinomN * kBinomK);
+    // one 64-bit word each, [k][n]
+    uint64_t *bn = reinterpret_cast<uint64_t *>(host.data() + ly.off_binom);
     for (int n = 0; n < kBinomN; ++n)
         for (int k = 0; k < kBinomK; ++k)
             bn[k * kBinomN + n] =
                 k == 0 ? 1 : (n == 0 ? 0 : bn[(k - 1) * kBinomN + n - 1] + bn[k * kBinomN + n - 1]);
-    uint32_t *blo = reinterpret_cast<uint32_t *>(host.data() + ly.off_binom);
-    uint32_t *bhi = blo + kBinomN * kBinomK;
-    for (int i = 0; i < kBinomN * kBinomK; ++i) {
-        blo[i] = (uint32_t)bn[i];
-        bhi[i] = (uint32_t)(bn[i] >> 32);
-    }
     // raw rows at entries 1..L; prefix_rows_kernel turns them into sums
     int64_t *Pw_ = reinterpret_cast<int64_t *>(host.data() + ly.off_Pw);
     int64_t *Pa_ = reinterpret_cast<int64_t *>(host.data() + ly.off_Pa);
