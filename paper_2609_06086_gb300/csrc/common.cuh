@@ -202,33 +202,34 @@ __device__ __forceinline__ uint64_t binom(const Tab &t, int n, int k) {
 // j is first estimated from C(x, k) ~ m^k / k! * exp(-k(k^2-1) / (12 m^2)),
 // m = x - (k-1)/2 (the product of the k factors m +- d around their mean):
 // m0 = (Y k!)^(1/k), x ~ m0 + (k-1)/2 + (k^2-1) / (24 m0) (half the
-// second-order term, which over-corrects), rounded up after a 0.01 margin
-// for rounding error.  Over uniform ranks of 64 layers in 2..16 stages this
-// lands on j in about 99 % of the stages (else one step low); exact
-// comparisons then move it to the answer whatever the estimate.
+// second-order term, which over-corrects), and j = ceil(x - 0.01) (a margin
+// for rounding error), taken as the nearest integer to x + 0.49.  Over
+// uniform ranks of 64 layers in 2..16 stages this lands on j in about 99 %
+// of the stages (else one step low); exact comparisons then move it to the
+// answer whatever the estimate.
 struct UnrankCoef {
     float log2_fact;  // log2(k!)
     float inv_k;      // 1/k
-    float half_km1;   // (k-1)/2 - 0.01
+    float shift;      // (k-1)/2 + 0.49
     float corr;       // (k^2-1)/24
 };
 __device__ __constant__ static const UnrankCoef kUnrankCoef[16] = {
     {0.000000000f, 0.000000000f, 0.00f, 0.000000000f},
-    {0.000000000f, 1.000000000f, -0.01f, 0.000000000f},
-    {1.000000000f, 0.500000000f, 0.49f, 0.125000000f},
-    {2.584962501f, 0.333333333f, 0.99f, 0.333333333f},
-    {4.584962501f, 0.250000000f, 1.49f, 0.625000000f},
-    {6.906890596f, 0.200000000f, 1.99f, 1.000000000f},
-    {9.491853096f, 0.166666667f, 2.49f, 1.458333333f},
-    {12.299208018f, 0.142857143f, 2.99f, 2.000000000f},
-    {15.299208018f, 0.125000000f, 3.49f, 2.625000000f},
-    {18.469133020f, 0.111111111f, 3.99f, 3.333333333f},
-    {21.791061115f, 0.100000000f, 4.49f, 4.125000000f},
-    {25.250492733f, 0.090909091f, 4.99f, 5.000000000f},
-    {28.835455234f, 0.083333333f, 5.49f, 5.958333333f},
-    {32.535894952f, 0.076923077f, 5.99f, 7.000000000f},
-    {36.343249874f, 0.071428571f, 6.49f, 8.125000000f},
-    {40.250140470f, 0.066666667f, 6.99f, 9.333333333f}};
+    {0.000000000f, 1.000000000f, 0.49f, 0.000000000f},
+    {1.000000000f, 0.500000000f, 0.99f, 0.125000000f},
+    {2.584962501f, 0.333333333f, 1.49f, 0.333333333f},
+    {4.584962501f, 0.250000000f, 1.99f, 0.625000000f},
+    {6.906890596f, 0.200000000f, 2.49f, 1.000000000f},
+    {9.491853096f, 0.166666667f, 2.99f, 1.458333333f},
+    {12.299208018f, 0.142857143f, 3.49f, 2.000000000f},
+    {15.299208018f, 0.125000000f, 3.99f, 2.625000000f},
+    {18.469133020f, 0.111111111f, 4.49f, 3.333333333f},
+    {21.791061115f, 0.100000000f, 4.99f, 4.125000000f},
+    {25.250492733f, 0.090909091f, 5.49f, 5.000000000f},
+    {28.835455234f, 0.083333333f, 5.99f, 5.958333333f},
+    {32.535894952f, 0.076923077f, 6.49f, 7.000000000f},
+    {36.343249874f, 0.071428571f, 6.99f, 8.125000000f},
+    {40.250140470f, 0.066666667f, 7.49f, 9.333333333f}};
 
 // the hardware's approximate base-2 logarithm, power and reciprocal (PTX
 // lg2 / ex2 / rcp .approx): an estimate only, the comparisons fix any error
@@ -250,9 +251,17 @@ __device__ __forceinline__ float approx_rcp(float x) {
 
 __device__ __forceinline__ int unrank_guess(uint64_t Y, int k, int rem) {
     const UnrankCoef c = kUnrankCoef[k];
-    const float m0 = approx_ex2((approx_lg2(__ull2float_rn(Y)) + c.log2_fact) * c.inv_k);
-    const float e = m0 + c.half_km1 + c.corr * approx_rcp(m0);
-    return min(max(__float2int_ru(e), k), rem - 1);
+    // Y as a float from its two 32-bit words: a 64-bit integer conversion
+    // issues to the FP64 pipe, a small fraction of the FP32 rate here
+    const float yf = __fmaf_rz(__uint2float_rz((uint32_t)(Y >> 32)), 4294967296.0f,
+                               __uint2float_rz((uint32_t)Y));
+    const float lg = approx_lg2(yf);
+    const float m0 = approx_ex2((lg + c.log2_fact) * c.inv_k);
+    const float x = m0 + c.shift + c.corr * approx_rcp(m0);
+    // nearest integer by the float adder: 1.5 * 2^23 + x (0 <= x < 2^22)
+    // has unit spacing, so its low bits are round(x)
+    const int j = __float_as_int(x + 12582912.0f) - 0x4B400000;
+    return min(max(j, k), rem - 1);
 }
 
 __device__ __forceinline__ int unrank_step(const Tab &t, int rem, int k, uint64_t &Y) {
