@@ -403,11 +403,14 @@ __host__ __device__ __forceinline__ int inflight(int sched, int S, int M, int s)
 }
 
 // Does 0-based stage s of an S-stage pipeline on class k fit layers [a, b)?
+// ... with w micro-batches in flight
+__device__ __forceinline__ bool stage_fits_w(const Tab &t, int w, int k, int a, int b) {
+    const int64_t need = (Pw(t, k, b) - Pw(t, k, a)) + (int64_t)w * (Pa(t, k, b) - Pa(t, k, a));
+    return need <= cap_of(t, k);
+}
 __device__ __forceinline__ bool stage_fits(const Tab &t, int S, int M, int s, int k, int a,
                                            int b) {
-    const int64_t need = (Pw(t, k, b) - Pw(t, k, a)) +
-                         (int64_t)inflight(t.ly->sched, S, M, s) * (Pa(t, k, b) - Pa(t, k, a));
-    return need <= cap_of(t, k);
+    return stage_fits_w(t, inflight(t.ly->sched, S, M, s), k, a, b);
 }
 
 template <int S>

@@ -209,25 +209,36 @@ __device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, uint
     }
     uint64_t Y = n_map - rank;
     uint4 cuts = make_uint4(0, 0, 0, 0);
+    const int n_tp = t.n_tp();
+    // in-flight micro-batches of stage s before the cap at M: S - s under
+    // 1F1B, 2(S-1-s)+1 under Eager 1F1B (inflight()), stepped per stage
+    const bool eager = t.ly->sched == POS_SCHED_EAGER_1F1B;
+    const int dw = eager ? 2 : 1;
+    int wl = eager ? 2 * S - 1 : S;
+    // the stage's memory check, with the type and TP fields shifted down as
+    // the stages go
+    uint32_t tc = tcode, tq = tpc;
+    auto fits_stage = [&](int a, int b) {
+        const int cls = (int)(tc & 3u) * n_tp + tp + (int)(tq & 3u);  // stage_class
+        const int w = min(wl, M);
+        tc >>= 2;
+        tq >>= 2;
+        wl -= dw;
+        if constexpr (LIM) return b <= (int)lim[(cls * p.lim_w + w - 1) * (L + 1) + a];
+        else return stage_fits_w(t, w, cls, a, b);
+    };
     bool fits = true;
     int c = 0;
+    // stages 0..S-2 (k stages after each), then the last one up to L
 #pragma unroll 1
-    for (int s = 0; s < S; ++s) {
-        int c2 = L;
-        if (s < S - 1) {
-            const int rem = L - c, k = S - s - 1;
-            c2 = c + (rem - unrank_step(t, rem, k, Y));
-            push_cut(cuts, c2);
-        }
-        const int cls = stage_class(tcode, tpc, tp, t.n_tp(), s);
-        if constexpr (LIM) {
-            const int w = inflight(t.ly->sched, S, M, s);
-            fits &= c2 <= (int)lim[(cls * p.lim_w + w - 1) * (L + 1) + c];
-        } else {
-            fits &= stage_fits(t, S, M, s, cls, c, c2);
-        }
+    for (int k = S - 1; k >= 1; --k) {
+        const int rem = L - c;
+        const int c2 = c + (rem - unrank_step(t, rem, k, Y));
+        push_cut(cuts, c2);
+        fits &= fits_stage(c, c2);
         c = c2;
     }
+    fits &= fits_stage(c, L);
     p.F[i] = fits ? POS_FEAS_YES : POS_FEAS_NO;
     return cuts;
 }
