@@ -149,18 +149,23 @@ __global__ void __launch_bounds__(1024) sort_scan_kernel(const uint32_t *hist, u
 }
 
 // Each block takes chunks of `chunk` candidates: counts their keys, reserves
-// one range per key with a single atomic, then places the indices.  Chunks
-// of 8192 for large batches (measured: 65536-candidate chunks, with fewer
+// one range per key with a single atomic, then gives every candidate its
+// sorted position (written in input order, so coalesced).  Chunks of 8192
+// for large batches (measured: 65536-candidate chunks, with fewer
 // reservations but fewer blocks, took 112 instead of 89 us at 1e7), smaller
 // ones (down to 1024) so that small batches still spread over the SMs.
+// Within a chunk the candidates of one key get consecutive positions, so
+// the decode pass's scattered record writes come in short runs.
 __host__ inline int64_t scatter_chunk(int64_t n, int sms) {
     int64_t c = (n / (8 * (int64_t)sms) + 511) & ~(int64_t)511;
     return c < 1024 ? 1024 : (c > 8192 ? 8192 : c);
 }
 
+constexpr uint32_t kNoDest = 0xffffffffu;
+
 template <int NK>
 __global__ void sort_scatter_kernel(const uint16_t *keys, int64_t n, int64_t chunk,
-                                    uint32_t *cursor, uint32_t *perm) {
+                                    uint32_t *cursor, uint32_t *dest) {
     __shared__ uint32_t h[NK];
     grid_dep_wait();  // the keys (histogram pass) and the cursors (scan)
     grid_dep_trigger();
@@ -178,18 +183,52 @@ __global__ void sort_scatter_kernel(const uint16_t *keys, int64_t n, int64_t chu
         __syncthreads();
         for (int64_t i = c0 + threadIdx.x; i < c1; i += blockDim.x) {
             const uint16_t k = __ldg(keys + i);
-            if (k != kNoKey) perm[atomicAdd(&h[k], 1u)] = (uint32_t)i;
+            dest[i] = k != kNoKey ? atomicAdd(&h[k], 1u) : kNoDest;
         }
         __syncthreads();
     }
 }
 
-// Decode pass over the whole sorted range [0, offs[nkeys]).  LIM: only the
-// binomials (the blob's first off_Pw bytes) and the memory-limit table are
-// staged, the table right after the binomials.
+// Decode pass.  Blocks take windows of `window` consecutive candidates:
+// their records and sorted positions are read coalesced into shared memory,
+// and each decoded 32-byte record is written to its sorted position.  The
+// decode's cost grows with the number of unranking stages (S, or N*V for an
+// interleaved record) and a window mixes them, so the block orders the
+// window's candidates by that count (a counting sort over 16 buckets) and
+// its warps then decode 32 consecutive entries of that order at a time:
+// the lanes of a warp loop over (nearly) the same number of stages.
+// LIM: only the binomials (the blob's first off_Pw bytes) and the
+// memory-limit table are staged, the table right after the binomials.
+constexpr int kDecodeThreads = 256;
+constexpr int kDecodeWindowMax = 1024;
+constexpr int kDecodeBuckets = POS_MAX_STAGES + 1;  // stage counts 1..16 (0 unused)
+
+__device__ __forceinline__ int decode_bucket(int sched, uint32_t w) {
+    const int S = w & 0xff, V = (int)(w >> 24);
+    const int J = (sched == POS_SCHED_INTERLEAVED_1F1B && V >= 2) ? S * V : S;
+    return min(max(J, 1), POS_MAX_STAGES);  // records beyond are answered at once
+}
+
+// the two 16-byte words of a decoded record in one 32-byte store
+__device__ __forceinline__ void store_decoded(uint4 *dst, const uint4 &a, const uint4 &b) {
+    asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(dst),
+                 "r"(a.x), "r"(a.y), "r"(a.z), "r"(a.w), "r"(b.x), "r"(b.y), "r"(b.z), "r"(b.w)
+                 : "memory");
+}
+
+struct DecodeWindow {
+    uint4 rec[kDecodeWindowMax];       // RecView::rec of each candidate
+    uint32_t tpc[kDecodeWindowMax];    // RecView::tpc
+    uint32_t dest[kDecodeWindowMax];   // sorted position (kNoDest: no key)
+    uint16_t order[kDecodeWindowMax];  // window offsets in bucket order
+    uint32_t slot[kDecodeBuckets + 1]; // bucket counts, then next free slots
+    uint32_t n_valid;
+};
+
 template <bool LIM>
-__global__ void __launch_bounds__(256, 4) decode_kernel(EvalParams p) {
+__global__ void __launch_bounds__(kDecodeThreads, 4) decode_kernel(EvalParams p, int window) {
     extern __shared__ __align__(16) unsigned char sm[];
+    __shared__ DecodeWindow win;
     if constexpr (LIM) {
         stage_blob(sm, p.blob, p.lay.off_Pw);
         stage_blob(sm + p.lay.off_Pw, static_cast<const unsigned char *>(p.blob) + p.lim_off,
@@ -198,36 +237,59 @@ __global__ void __launch_bounds__(256, 4) decode_kernel(EvalParams p) {
         stage_blob(sm, p.blob, p.lay.bytes);
     }
     __syncthreads();
-    grid_dep_wait();  // the permutation (scatter pass)
+    grid_dep_wait();  // the sorted positions (scatter pass)
     grid_dep_trigger();
     const Tab t = tab_at(sm, p.lay);
     const uint8_t *lim = sm + p.lay.off_Pw;
-    const int64_t total = p.offs[p.nkeys];
-    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    const int64_t span = (total + 31) & ~(int64_t)31;
-    // software pipeline over the grid-stride loop: the permutation entry is
-    // read two iterations ahead and the record it points to one iteration
-    // ahead, so neither load's latency stalls the decode of the current one
-    int64_t j = blockIdx.x * (int64_t)blockDim.x + threadIdx.x;
-    RecView none;
-    none.rec = make_uint4(0, 0, 0, 0);
-    none.tpc = 0;
-    uint32_t i_next = j < total ? __ldg(p.perm + j) : 0u;
-    uint32_t i_after = j + stride < total ? __ldg(p.perm + j + stride) : 0u;
-    RecView v_next = j < total ? load_record(p, i_next) : none;
-    for (; j < span; j += stride) {
-        const bool active = j < total;
-        const uint32_t i = i_next;
-        const RecView v = v_next;
-        i_next = i_after;
-        v_next = j + stride < total ? load_record(p, i_next) : none;
-        i_after = j + 2 * stride < total ? __ldg(p.perm + j + 2 * stride) : 0u;
-        uint4 out = make_uint4(0, 0, 0, 1u << 24);
-        if (active) out = decode_one<LIM>(t, v.rec, v.tpc, p, i, lim);
-        if (active) {
-            p.cuts[2 * j] = out;
-            p.cuts[2 * j + 1] = make_uint4(i, v.rec.z, v.rec.w, v.tpc);
+    const int sched = p.lay.sched;
+    const int lane = threadIdx.x & 31;
+    for (int64_t w0 = blockIdx.x * (int64_t)window; w0 < p.n; w0 += (int64_t)gridDim.x * window) {
+        const int wn = (int)min((int64_t)window, p.n - w0);
+        // 1. the window's records and positions, and the candidates per
+        // bucket (those without a key are already answered)
+        if (threadIdx.x <= kDecodeBuckets) win.slot[threadIdx.x] = 0;
+        __syncthreads();
+#pragma unroll 4
+        for (int li = threadIdx.x; li < wn; li += kDecodeThreads) {
+            const uint32_t i = (uint32_t)(w0 + li);
+            const RecView v = load_record(p, i);
+            const uint32_t d = __ldg(p.dest + i);
+            win.rec[li] = v.rec;
+            win.tpc[li] = v.tpc;
+            win.dest[li] = d;
+            if (d != kNoDest) atomicAdd(&win.slot[decode_bucket(sched, v.rec.w)], 1u);
         }
+        __syncthreads();
+        // 2. exclusive prefix over the buckets (first warp)
+        if (threadIdx.x < 32) {
+            const uint32_t c = lane <= kDecodeBuckets ? win.slot[lane] : 0u;
+            uint32_t incl = c;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t v = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += v;
+            }
+            if (lane <= kDecodeBuckets) win.slot[lane] = incl - c;
+            if (lane == 31) win.n_valid = incl;
+        }
+        __syncthreads();
+        // 3. the window's offsets in bucket order
+        for (int li = threadIdx.x; li < wn; li += kDecodeThreads)
+            if (win.dest[li] != kNoDest)
+                win.order[atomicAdd(&win.slot[decode_bucket(sched, win.rec[li].w)], 1u)] =
+                    (uint16_t)li;
+        __syncthreads();
+        // 4. decode: each warp takes 32 consecutive entries of the order
+        const int nv = (int)win.n_valid;
+        for (int k = threadIdx.x; k < nv; k += kDecodeThreads) {
+            const int li = win.order[k];
+            const uint32_t i = (uint32_t)(w0 + li);
+            const uint4 rec = win.rec[li];
+            const uint32_t tpc = win.tpc[li];
+            const uint4 out = decode_one<LIM>(t, rec, tpc, p, i, lim);
+            store_decoded(p.cuts + 2 * (size_t)win.dest[li], out, make_uint4(i, rec.z, rec.w, tpc));
+        }
+        __syncthreads();  // the window's arrays are rewritten for the next one
     }
 }
 
@@ -238,11 +300,15 @@ pos_status launch_decode(const EvalParams &p, cudaStream_t stream) {
     const int smem = lim ? p.lay.off_Pw + p.lim_bytes : p.lay.bytes;
     POS_TRY(ensure_smem(kern, smem));
     int per_sm = 0;
-    POS_TRY(blocks_per_sm(kern, 256, smem, &per_sm));
-    const int64_t blocks = (p.n + 255) / 256;
-    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)std::max(per_sm, 1) * sm_count()));
-    if (lim) POS_CUDA(launch_dependent(decode_kernel<true>, grid, 256, smem, stream, p));
-    else POS_CUDA(launch_dependent(decode_kernel<false>, grid, 256, smem, stream, p));
+    POS_TRY(blocks_per_sm(kern, kDecodeThreads, smem, &per_sm));
+    // blocks of at least 1024 candidates; the same number of windows for
+    // every block (up to one), so that the blocks finish together
+    const int64_t blocks = std::max<int64_t>(
+        1, std::min<int64_t>((p.n + 1023) / 1024, (int64_t)std::max(per_sm, 1) * sm_count()));
+    const int64_t rounds = (p.n + blocks * kDecodeWindowMax - 1) / (blocks * kDecodeWindowMax);
+    const int window = (int)((p.n + blocks * rounds - 1) / (blocks * rounds));
+    if (lim) POS_CUDA(launch_dependent(decode_kernel<true>, (int)blocks, kDecodeThreads, smem, stream, p, window));
+    else POS_CUDA(launch_dependent(decode_kernel<false>, (int)blocks, kDecodeThreads, smem, stream, p, window));
     return POS_OK;
 }
 
@@ -283,7 +349,7 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
     // batches above 2^24 candidates go in chunks of 2^24: a chunk's outputs
     // (5 bytes per candidate, 80 MB), written in sorted order and so
     // scattered over the output arrays, stay in L2 until whole sectors are
-    // written back (the permutation's 32-bit indices would allow 2^31)
+    // written back (the 32-bit sorted positions would allow 2^31)
     const int64_t chunk = (int64_t)1 << 24;
     for (int64_t base = 0; base < n; base += chunk) {
         const int64_t m = std::min(chunk, n - base);
@@ -298,8 +364,8 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
         uint32_t *hist = reinterpret_cast<uint32_t *>(static_cast<char *>(scratch) + 32 * (size_t)m);
         uint32_t *offs = hist + nk;
         uint32_t *cursor = offs + nk + 1;
-        uint32_t *perm = cursor + nk;
-        uint16_t *keys = reinterpret_cast<uint16_t *>(perm + m);
+        uint32_t *dest = cursor + nk;
+        uint16_t *keys = reinterpret_cast<uint16_t *>(dest + m);
         EvalParams p;
         p.per_stage_tp = per_stage_tp ? 1 : 0;
         p.cands = per_stage_tp ? nullptr : static_cast<const uint4 *>(d_cands) + base;
@@ -307,7 +373,7 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
         p.n = m;
         p.T = d_T + base;
         p.F = d_F + base;
-        p.perm = perm;
+        p.dest = dest;
         p.offs = offs;
         p.cuts = cuts;
         p.blob = h->d_blob;
@@ -337,7 +403,7 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
                                          cursor);
                 if (e == cudaSuccess)
                     e = launch_dependent(sort_scatter_kernel<kKeysIl>, sgrid, 512, 0, stream, keys,
-                                         m, chunk, cursor, perm);
+                                         m, chunk, cursor, dest);
             } else {
                 sort_hist_kernel<kKeys><<<grid, 256, 0, stream>>>(p, m, hist, keys, p.T, p.F);
                 e = cudaGetLastError();
@@ -346,7 +412,7 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
                                          cursor);
                 if (e == cudaSuccess)
                     e = launch_dependent(sort_scatter_kernel<kKeys>, sgrid, 512, 0, stream, keys, m,
-                                         chunk, cursor, perm);
+                                         chunk, cursor, dest);
             }
         }
         if (e == cudaSuccess) st = launch_decode(p, stream);

@@ -1,19 +1,19 @@
 // Evaluation kernels of poseidon_eval_batch (hot-path steps a2-a5).
 //
-// One thread evaluates one candidate, in two passes over the (S, M)-sorted
-// batch: a decode pass (field checks, overflow guard, unranking, memory
-// check; few registers, so the latency of its dependent shared-memory
-// lookups is hidden by many warps) writes the cut positions in sorted order,
-// and the makespan pass reads them coalesced.  The makespan loop costs ~6*S*M
-// integer ops and its live registers grow with S (about 7*S), so the batch
-// is first counting-sorted by exact (S, M) into a permutation (stream-ordered
-// scratch), and then a family of kernels, each owning the candidates of one
-// S range and either M >= S (ramps unrolled, steady loop) or M < S (the
-// whole schedule unrolled per (S, M)), walks its contiguous range of the
-// permutation with launch bounds
-// matched to its register need.  Warps therefore see one (S, M) except at
-// bucket boundaries, and no kernel waits at a block barrier after staging the
-// cost tables.
+// One thread evaluates one candidate, in two passes: a decode pass (field
+// checks, overflow guard, unranking, memory check; few registers, so the
+// latency of its dependent shared-memory lookups is hidden by many warps)
+// writes every candidate's cut positions to its place in the (S, M)-sorted
+// order, and the makespan pass reads them coalesced.  The makespan loop
+// costs ~6*S*M integer ops and its live registers grow with S (about 7*S),
+// so the batch is first counting-sorted by exact (S, M) (stream-ordered
+// scratch: every candidate's sorted position), and then a family of
+// kernels, each owning the candidates of one S range and either M >= S
+// (ramps unrolled, steady loop) or M < S (the whole schedule unrolled per
+// (S, M)), walks its contiguous range of the sorted records with launch
+// bounds matched to its register need.  Warps therefore see one (S, M)
+// except at bucket boundaries, and no kernel waits at a block barrier after
+// staging the cost tables.
 //
 // Sort keys: fast path (M >= S for 1F1B, M >= 2S-1 for Eager 1F1B) ->
 // (S-1)*256 + M (the other slots of each S stay empty); short path ->
@@ -40,13 +40,15 @@ struct EvalParams {
     int64_t n;
     int32_t *T;
     uint8_t *F;
-    const uint32_t *perm;  // sorted candidate indices
-    const uint32_t *offs;  // [nkeys + 1] start of every key in perm
+    const uint32_t *dest;  // sorted position of every candidate (kNoDest:
+                           // no key, answered by the histogram pass)
+    const uint32_t *offs;  // [nkeys + 1] start of every key in sorted order
     uint4 *cuts;           // per sorted position j, two 16-byte words (read once,
                            // with evict-first loads, so that the outputs'
                            // sectors stay in L2):
-                           // cuts[2j]: cut[1..S-1] in bytes 0..14, byte 15 = 1
-                           // when the result is already written;
+                           // cuts[2j]: the cut positions (push_cut's layout;
+                           // ascending bytes 0..14 for interleaved records),
+                           // byte 15 = 1 when the result is already written;
                            // cuts[2j+1]: (candidate index, type_code, the
                            // record's S|M|tp|V word, per-stage TP code), so the makespan
                            // kernels read 32 contiguous bytes and no record
@@ -287,8 +289,8 @@ __device__ __forceinline__ void dispatch_range(int S, const Tab &t, const uint4 
 #undef POS_EV
 }
 
-// Evaluates perm[offs[key_lo] .. offs[key_hi]) -- all candidates with S in
-// [SLO, SHI] on path PATH.
+// Evaluates the sorted positions [offs[key_lo], offs[key_hi]): all
+// candidates with S in [SLO, SHI] on path PATH.
 template <int SLO, int SHI, int PATH, int MINB>
 __global__ void __launch_bounds__(kEvalThreads, MINB) eval_kernel(EvalParams p) {
     extern __shared__ __align__(16) unsigned char sm[];
