@@ -461,8 +461,9 @@ __device__ __forceinline__ bool plan_fits(const Tab &t, int M, const int (&cut)[
 // ---------------------------------------------------------------------------
 // Paths: 1F1B with M >= S (ramps + steady loop), 1F1B with M < S (unrolled
 // per M), Eager 1F1B with M >= 2S-1 (ramps + steady loop), Eager 1F1B with
-// M < 2S-1 (level program).
-enum { kPathFast = 0, kPathGeneric = 1, kPathEager = 2, kPathEagerShort = 3 };
+// M < 2S-1 as a level program (the search's leaf kernel) or unrolled per M
+// (the evaluator).
+enum { kPathFast = 0, kPathGeneric = 1, kPathEager = 2, kPathEagerShort = 3, kPathEagerUnrolled = 4 };
 
 // Op of 1-based stage s1 at ramp-up level t (1 <= t <= 2S-1) and at
 // ramp-down level 2M + tau (0 <= tau <= 2S-2), for M >= S: 0 none, 1 F, 2 B.
@@ -758,6 +759,153 @@ __device__ __forceinline__ int32_t makespan_eager(const StageW<S> &w, int M) {
     return T;
 }
 
+// Eager 1F1B with M < 2S-1: the unit-weight ASAP level order has no closed
+// form, so it is computed at compile time for each (S, M) and unrolled like
+// the ramps.  Stage s (0-based) runs W = min(2(S-1-s)+1, M) forwards, then
+// (B_i, F_{W+i}) pairs, then the remaining backwards; an op's level is one
+// more than the later of its stage's previous op and its inter-stage
+// predecessor (F_{s-1,m} for F_{s,m}, B_{s+1,m} for B_{s,m}).  Within a
+// level the stages are visited in descending order, as in the ramps, and
+// while the program is built every op is checked to read the finish it
+// depends on: F_{s-1,m} from stage s-1's latest forward (lag 1) or the one
+// before (lag 2), B_{s+1,m} from stage s+1's latest backward.
+struct EagerShortOp {
+    int kind;      // 0 none, 1 forward, 2 backward
+    int lag;       // forward of a stage s > 0: 1 or 2
+    bool clock_b;  // the stage's previous op is a backward (else a forward)
+};
+template <int S, int M>
+struct EagerShortProgram {
+    static constexpr int kMaxLevels = 2 * (M + S) + 2;
+    EagerShortOp op[kMaxLevels][S];
+    int n_levels;
+    bool ok;
+    __host__ __device__ constexpr EagerShortProgram() : op{}, n_levels(0), ok(true) {
+        int kind[S][2 * M] = {}, mb[S][2 * M] = {};  // chains: op kind and micro-batch
+        for (int s = 0; s < S; ++s) {
+            const int W = 2 * (S - 1 - s) + 1 < M ? 2 * (S - 1 - s) + 1 : M;
+            int n = 0;
+            for (int m = 0; m < W; ++m) kind[s][n] = 1, mb[s][n++] = m;
+            for (int i = 0; i < M - W; ++i) {
+                kind[s][n] = 2, mb[s][n++] = i;
+                kind[s][n] = 1, mb[s][n++] = W + i;
+            }
+            for (int m = M - W; m < M; ++m) kind[s][n] = 2, mb[s][n++] = m;
+        }
+        int lf[S][M] = {}, lb[S][M] = {};  // ASAP levels (1-based)
+        for (bool changed = true; changed;) {
+            changed = false;
+            for (int s = 0; s < S; ++s) {
+                int prev = 0;
+                for (int n = 0; n < 2 * M; ++n) {
+                    const int m = mb[s][n];
+                    int p = prev;
+                    if (kind[s][n] == 2 && s + 1 < S && lb[s + 1][m] > p) p = lb[s + 1][m];
+                    if (kind[s][n] == 1 && s > 0 && lf[s - 1][m] > p) p = lf[s - 1][m];
+                    int &v = kind[s][n] == 2 ? lb[s][m] : lf[s][m];
+                    if (v != p + 1) {
+                        v = p + 1;
+                        changed = true;
+                    }
+                    prev = p + 1;
+                }
+            }
+        }
+        for (int s = 0; s < S; ++s)
+            for (int m = 0; m < M; ++m) {
+                if (lf[s][m] > n_levels) n_levels = lf[s][m];
+                if (lb[s][m] > n_levels) n_levels = lb[s][m];
+            }
+        if (n_levels > kMaxLevels) {
+            ok = false;
+            n_levels = kMaxLevels;
+        }
+        // registers: the micro-batch whose finish Fo / Fp / Bo of a stage
+        // holds (-1: none yet) and whether its last op was a backward
+        int fo[S] = {}, fp[S] = {}, bo[S] = {};
+        bool last_b[S] = {};
+        for (int s = 0; s < S; ++s) fo[s] = fp[s] = bo[s] = -1;
+        for (int l = 1; l <= n_levels; ++l)
+            for (int s = S - 1; s >= 0; --s) {
+                int k = 0, m = -1;
+                for (int u = 0; u < M; ++u) {
+                    if (lf[s][u] == l) k = k ? 3 : 1, m = u;
+                    if (lb[s][u] == l) k = k ? 3 : 2, m = u;
+                }
+                if (k == 3) ok = false;  // two ops of one stage in a level
+                if (k == 1) {
+                    int lag = 1;
+                    if (s > 0) {
+                        if (fo[s - 1] == m) lag = 1;
+                        else if (fp[s - 1] == m) lag = 2;
+                        else ok = false;
+                    }
+                    op[l - 1][s] = EagerShortOp{1, lag, last_b[s]};
+                    fp[s] = fo[s];
+                    fo[s] = m;
+                    last_b[s] = false;
+                } else if (k == 2) {
+                    if (s + 1 < S && bo[s + 1] != m) ok = false;
+                    op[l - 1][s] = EagerShortOp{2, 0, last_b[s]};
+                    bo[s] = m;
+                    last_b[s] = true;
+                }
+            }
+    }
+};
+template <int S, int M>
+struct EagerShortTab {
+    static constexpr EagerShortProgram<S, M> value{};
+    static_assert(value.ok, "Eager 1F1B short level order: an op would read the wrong finish");
+};
+
+template <int S, int M, int l, int i>
+__device__ __forceinline__ void eager_short_op(int32_t (&Fo)[S], int32_t (&Fp)[S],
+                                               int32_t (&Bo)[S], const StageW<S> &w) {
+    constexpr int s = S - 1 - i;
+    constexpr EagerShortOp o = EagerShortTab<S, M>::value.op[l][s];
+    if constexpr (o.kind == 1)
+        relax_f_lag<S, s, (s > 0 ? o.lag : 1)>(Fo, Fp, w, o.clock_b ? Bo[s] : Fo[s]);
+    else if constexpr (o.kind == 2)
+        relax_b<S, s>(Bo, w, o.clock_b ? Bo[s] : Fo[s]);
+}
+template <int S, int M, int l, int... i>
+__device__ __forceinline__ void eager_short_level(int32_t (&Fo)[S], int32_t (&Fp)[S],
+                                                  int32_t (&Bo)[S], const StageW<S> &w,
+                                                  std::integer_sequence<int, i...>) {
+    (eager_short_op<S, M, l, i>(Fo, Fp, Bo, w), ...);
+}
+template <int S, int M, int... l>
+__device__ __forceinline__ void eager_short_all(int32_t (&Fo)[S], int32_t (&Fp)[S],
+                                                int32_t (&Bo)[S], const StageW<S> &w,
+                                                std::integer_sequence<int, l...>) {
+    (eager_short_level<S, M, l>(Fo, Fp, Bo, w, std::make_integer_sequence<int, S>{}), ...);
+}
+template <int S, int M>
+__device__ __forceinline__ int32_t makespan_eager_short(const StageW<S> &w) {
+    int32_t Fo[S], Fp[S], Bo[S];
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+        Fo[s] = 0;
+        Fp[s] = 0;
+        Bo[s] = 0;
+    }
+    eager_short_all<S, M>(Fo, Fp, Bo, w,
+                          std::make_integer_sequence<int, EagerShortTab<S, M>::value.n_levels>{});
+    int32_t T = 0;
+#pragma unroll
+    for (int s = 0; s < S; ++s) T = max(T, Bo[s] + w.d[s]);
+    return T;
+}
+// runtime M in 1..2S-2 -> its unrolled instance
+template <int S, int... m>
+__device__ __forceinline__ int32_t makespan_eager_short_dispatch(const StageW<S> &w, int M,
+                                                                 std::integer_sequence<int, m...>) {
+    int32_t T = -1;
+    ((M == m + 1 ? (T = makespan_eager_short<S, m + 1>(w), 0) : 0), ...);
+    return T;
+}
+
 // Level program of one (schedule, S, M): per level one 64-bit word, bit s of
 // bits 0-15 = stage s runs a forward, bits 16-31 = a backward, bits 32-47 =
 // that forward's predecessor is the previous forward of stage s-1 (lag 2).
@@ -836,6 +984,11 @@ __device__ __forceinline__ int32_t makespan_path(const StageW<S> &w, int M, cons
     } else if constexpr (PATH == kPathEagerShort) {
         const uint2 ix = __ldg(pg.index + (S - 1) * 32 + M);
         return makespan_program<S>(w, pg.words + ix.x, (int)ix.y);
+    } else if constexpr (PATH == kPathEagerUnrolled) {
+        if constexpr (S > 1)
+            return makespan_eager_short_dispatch<S>(w, M, std::make_integer_sequence<int, 2 * S - 2>{});
+        else
+            return -1;  // S = 1 has no short case
     } else {
         return makespan_1f1b<S, PATH>(w, M);
     }

@@ -423,8 +423,12 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
                     (st = eval_eager_11_13(p, stream)) == POS_OK &&
                     (st = eval_eager_14_16(p, stream)) == POS_OK &&
                     (st = eval_eager_short_2_8(p, stream)) == POS_OK &&
-                    (st = eval_eager_short_9_12(p, stream)) == POS_OK)
-                    st = eval_eager_short_13_16(p, stream);
+                    (st = eval_eager_short_9_10(p, stream)) == POS_OK &&
+                    (st = eval_eager_short_11_12(p, stream)) == POS_OK &&
+                    (st = eval_eager_short_13_13(p, stream)) == POS_OK &&
+                    (st = eval_eager_short_14_14(p, stream)) == POS_OK &&
+                    (st = eval_eager_short_15_15(p, stream)) == POS_OK)
+                    st = eval_eager_short_16_16(p, stream);
             } else if ((st = eval_fast_1_4(p, stream)) == POS_OK &&
                        (st = eval_fast_5_8(p, stream)) == POS_OK &&
                        (st = eval_fast_9_12(p, stream)) == POS_OK &&

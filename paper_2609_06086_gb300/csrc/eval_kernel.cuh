@@ -370,7 +370,11 @@ pos_status eval_eager_7_10(const EvalParams &p, cudaStream_t s);
 pos_status eval_eager_11_13(const EvalParams &p, cudaStream_t s);
 pos_status eval_eager_14_16(const EvalParams &p, cudaStream_t s);
 pos_status eval_eager_short_2_8(const EvalParams &p, cudaStream_t s);
-pos_status eval_eager_short_9_12(const EvalParams &p, cudaStream_t s);
-pos_status eval_eager_short_13_16(const EvalParams &p, cudaStream_t s);
+pos_status eval_eager_short_9_10(const EvalParams &p, cudaStream_t s);
+pos_status eval_eager_short_11_12(const EvalParams &p, cudaStream_t s);
+pos_status eval_eager_short_13_13(const EvalParams &p, cudaStream_t s);
+pos_status eval_eager_short_14_14(const EvalParams &p, cudaStream_t s);
+pos_status eval_eager_short_15_15(const EvalParams &p, cudaStream_t s);
+pos_status eval_eager_short_16_16(const EvalParams &p, cudaStream_t s);
 
 }  // namespace pos

@@ -1,0 +1,11 @@
+// Instantiation unit of the eval kernel family (see eval_kernel.cuh):
+// Eager 1F1B with M < 2S-1 (unrolled per (S, M)), S = 16.
+#include "eval_kernel.cuh"
+
+namespace pos {
+
+pos_status eval_eager_short_16_16(const EvalParams &p, cudaStream_t s) {
+    return launch_eval_range<16, 16, kPathEagerUnrolled, 2>(p, s);
+}
+
+}  // namespace pos
