@@ -90,15 +90,25 @@ __global__ void sort_hist_kernel(EvalParams p, int64_t n, uint32_t *hist, uint16
     __shared__ uint32_t h[NK];
     for (int i = threadIdx.x; i < NK; i += blockDim.x) h[i] = 0;
     __syncthreads();
-    for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n;
-         i += (int64_t)gridDim.x * blockDim.x) {
-        const int k = eval_key(sched, record_word(p, i));
-        keys[i] = k >= 0 ? (uint16_t)k : kNoKey;
-        if (k >= 0) {
-            atomicAdd(&h[k], 1u);
-        } else {
-            T[i] = -1;
-            F[i] = POS_FEAS_INVALID;
+    // four record words in flight per thread (the pass is bound by HBM
+    // latency: one load per thread and iteration kept too few bytes in flight)
+    const int64_t bd = blockDim.x;
+    for (int64_t i0 = blockIdx.x * 4 * bd + threadIdx.x; i0 < n; i0 += (int64_t)gridDim.x * 4 * bd) {
+        uint32_t wv[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) wv[u] = i0 + u * bd < n ? record_word(p, i0 + u * bd) : 0u;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int64_t i = i0 + u * bd;
+            if (i >= n) break;
+            const int k = eval_key(sched, wv[u]);
+            keys[i] = k >= 0 ? (uint16_t)k : kNoKey;
+            if (k >= 0) {
+                atomicAdd(&h[k], 1u);
+            } else {
+                T[i] = -1;
+                F[i] = POS_FEAS_INVALID;
+            }
         }
     }
     __syncthreads();
@@ -386,8 +396,9 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
         p.lim_off = h->lim_off;
         p.lim_w = h->lim_w;
         p.lim_bytes = h->lim_bytes;
+        // histogram pass: 256 threads, four candidates per thread and round
         const int grid = (int)std::max<int64_t>(
-            1, std::min<int64_t>((m + 255) / 256, 4LL * sm_count()));
+            1, std::min<int64_t>((m + 1023) / 1024, 4LL * sm_count()));
         cudaError_t e = cudaMemsetAsync(hist, 0, sizeof(uint32_t) * nk, stream);
         if (e == cudaSuccess) {
             const int64_t chunk = scatter_chunk(m, sm_count());
