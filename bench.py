@@ -40,10 +40,10 @@ ENTRY_BYTES = 32  # one frontier entry / one complete plan
 # dram__bytes_read.sum + dram__bytes_write.sum over a config-4 search's leaf
 # launches (the leaf kernel's ncu summary), valid while the kernel's
 # sources hash to LEAF_SOURCES_SHA256 (else the traffic is reported as null)
-LEAF_DRAM_BYTES_PER_PLAN = 59689984 / 1925970
+LEAF_DRAM_BYTES_PER_PLAN = 59682816 / 1925970
 LEAF_SOURCES = ("paper_2609_06086_gb300/csrc/search_kernels.cuh",
                 "paper_2609_06086_gb300/csrc/common.cuh")
-LEAF_SOURCES_SHA256 = "366abc3efae9b375"
+LEAF_SOURCES_SHA256 = "c701e85b0c1184ee"
 PRUNE_NAMES = {1: "stage-level, Eq. 2 as printed (Theorem 1)",
                2: "stage-level, tightened: Eq. 2 with P2P edges + completion bounds"}
 
