@@ -231,6 +231,7 @@ struct DecodeWindow {
     uint32_t tpc[kDecodeWindowMax];    // RecView::tpc
     uint32_t dest[kDecodeWindowMax];   // sorted position (kNoDest: no key)
     uint16_t order[kDecodeWindowMax];  // window offsets in bucket order
+    uint8_t bucket[kDecodeWindowMax];  // bucket of each candidate (0: no key)
     uint32_t slot[kDecodeBuckets + 1]; // bucket counts, then next free slots
     uint32_t n_valid;
 };
@@ -267,7 +268,9 @@ __global__ void __launch_bounds__(kDecodeThreads, 4) decode_kernel(EvalParams p,
             win.rec[li] = v.rec;
             win.tpc[li] = v.tpc;
             win.dest[li] = d;
-            if (d != kNoDest) atomicAdd(&win.slot[decode_bucket(sched, v.rec.w)], 1u);
+            const int b = d != kNoDest ? decode_bucket(sched, v.rec.w) : 0;
+            win.bucket[li] = (uint8_t)b;
+            if (b) atomicAdd(&win.slot[b], 1u);
         }
         __syncthreads();
         // 2. exclusive prefix over the buckets (first warp)
@@ -284,10 +287,10 @@ __global__ void __launch_bounds__(kDecodeThreads, 4) decode_kernel(EvalParams p,
         }
         __syncthreads();
         // 3. the window's offsets in bucket order
-        for (int li = threadIdx.x; li < wn; li += kDecodeThreads)
-            if (win.dest[li] != kNoDest)
-                win.order[atomicAdd(&win.slot[decode_bucket(sched, win.rec[li].w)], 1u)] =
-                    (uint16_t)li;
+        for (int li = threadIdx.x; li < wn; li += kDecodeThreads) {
+            const int b = win.bucket[li];
+            if (b) win.order[atomicAdd(&win.slot[b], 1u)] = (uint16_t)li;
+        }
         __syncthreads();
         // 4. decode: each warp takes 32 consecutive entries of the order
         const int nv = (int)win.n_valid;
@@ -388,9 +391,16 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
         p.cuts = cuts;
         p.blob = h->d_blob;
         p.lay = h->lay;
-        p.gA = h->guard_A;
-        p.gD = h->guard_D;
-        p.gP = h->guard_P;
+        for (int J = 1; J <= POS_MAX_STAGES; ++J) {  // smallest tripping M, by bisection
+            int lo = 1, hi = 256;
+            while (lo < hi) {
+                const int mid = (lo + hi) / 2;
+                if (guard_trips(h->guard_A, h->guard_D, h->guard_P, J, mid)) hi = mid;
+                else lo = mid + 1;
+            }
+            p.guard_m[J] = (uint16_t)lo;
+        }
+        p.guard_m[0] = 0;
         p.pg = pg;
         p.nkeys = nk;
         p.lim_off = h->lim_off;

@@ -54,7 +54,10 @@ struct EvalParams {
                            // kernels read 32 contiguous bytes and no record
     const void *blob;
     BlobLayout lay;
-    int64_t gA, gD, gP;
+    // guard_m[J]: the smallest M (1..255; 256 for none) at which the
+    // overflow guard (guard_trips) trips for J (virtual) stages: U(J, M)
+    // grows with M since every cost is non-negative
+    uint16_t guard_m[POS_MAX_STAGES + 1];
     Programs pg;           // level programs of the schedule's short path
     int nkeys;             // kKeys, or kKeysIl under Interleaved 1F1B
     int per_stage_tp;      // 1: records carry a TP index per stage (n_tp <= 4)
@@ -153,7 +156,7 @@ __device__ __forceinline__ uint4 decode_il(const Tab &t, const uint4 &rec, uint3
         p.F[i] = POS_FEAS_INVALID;
         return done;
     }
-    if (guard_trips(p.gA, p.gD, p.gP, J, M)) {
+    if (M >= (int)p.guard_m[J]) {  // the overflow guard
         p.T[i] = -1;
         p.F[i] = POS_FEAS_OVERFLOW;
         return done;
@@ -197,14 +200,14 @@ __device__ __forceinline__ uint4 decode_one(const Tab &t, const uint4 &rec, uint
     const uint64_t n_map = ok ? binom(t, L - 1, S - 1) : 0;
     ok = ok && rank < n_map;
     ok = ok && types_ok(tcode, S, t.n_types()) &&
-         types_ok(tpc, S, t.n_tp());  // tpc = 0 for 16-byte records
+         (!p.per_stage_tp || types_ok(tpc, S, t.n_tp()));  // tpc = 0 for 16-byte records
     const uint4 done = make_uint4(0, 0, 0, 1u << 24);  // byte 15 = 1: answered here
     if (!ok) {
         p.T[i] = -1;
         p.F[i] = POS_FEAS_INVALID;
         return done;
     }
-    if (guard_trips(p.gA, p.gD, p.gP, S, M)) {
+    if (M >= (int)p.guard_m[S]) {  // the overflow guard
         p.T[i] = -1;
         p.F[i] = POS_FEAS_OVERFLOW;
         return done;

@@ -89,6 +89,36 @@ def test_invalid_records_flagged(P, orc):
     assert F[:6].tolist() == [2] * 6 and (T[:6] == -1).all()
 
 
+def test_invalid_records_scattered(P, orc):
+    """Invalid records spread over a batch that takes several decode windows
+    per block: records without a sort key (S = 0, S = 17, M = 0) and records
+    the decode pass rejects (rank, type or TP index out of range) sit
+    between valid ones, in every window."""
+    w = gen.config5_tables()
+    n = 200_000
+    c = gen.config5_candidates(n, seed=11)
+    rng = np.random.default_rng(11)
+    bad = rng.choice(n, n // 7, replace=False)
+    kinds = rng.integers(0, 6, len(bad))
+    for i, k in zip(bad, kinds):
+        if k == 0:
+            c[i]["S"] = 0
+        elif k == 1:
+            c[i]["S"] = 17
+        elif k == 2:
+            c[i]["M"] = 0
+        elif k == 3:
+            c[i]["map_rank"] = math.comb(63, int(c[i]["S"]) - 1)
+        elif k == 4:
+            c[i]["type_code"] |= 2 << (2 * int(rng.integers(0, int(c[i]["S"]))))
+        else:
+            c[i]["tp_idx"] = 1
+    T, F, Tr, Fr = _both(P, orc, w, c)
+    assert np.array_equal(T, Tr) and np.array_equal(F, Fr)
+    assert (F[bad] == 2).all() and (T[bad] == -1).all()
+    assert (F != 2).sum() == n - len(bad)
+
+
 def test_overflow_guard_flagged(P, orc):
     big = dict(L=4, n_types=1, n_tp=1, fwd=[[2 ** 26] * 4], bwd=[[2 ** 26] * 4],
                dsync=[[0] * 4], p2p_f=[[0]], p2p_b=[[0]], mem_w=[[0] * 4], mem_a=[[0] * 4],
