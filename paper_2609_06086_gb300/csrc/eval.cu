@@ -350,6 +350,36 @@ static pos_status scratch_pool(cudaMemPool_t *out) {
     return POS_OK;
 }
 
+// A second stream per device for the short-path kernels (M < S under 1F1B,
+// M < 2S-1 under Eager 1F1B): they depend only on the decode pass, like the
+// fast-path kernels, and are bound by instruction fetch rather than by the
+// ALU, so they run beside the fast-path kernels instead of after them.  The
+// fork and join events are shared per device, so a call holds the device's
+// side mutex from the fork to the join (two calls from different host
+// threads must not interleave their record / wait pairs).
+struct SideStream {
+    cudaStream_t s = nullptr;
+    cudaEvent_t fork = nullptr, join = nullptr;
+    std::mutex mu;
+};
+static std::mutex g_side_mutex;
+static SideStream g_side[64];
+
+static pos_status side_stream(SideStream **out) {
+    int dev = 0;
+    POS_CUDA(cudaGetDevice(&dev));
+    if (dev < 0 || dev >= 64) return fail(POS_EINVAL, "device index above 63");
+    std::lock_guard<std::mutex> lock(g_side_mutex);
+    SideStream &ss = g_side[dev];
+    if (!ss.s) {
+        POS_CUDA(cudaEventCreateWithFlags(&ss.fork, cudaEventDisableTiming));
+        POS_CUDA(cudaEventCreateWithFlags(&ss.join, cudaEventDisableTiming));
+        POS_CUDA(cudaStreamCreateWithFlags(&ss.s, cudaStreamNonBlocking));
+    }
+    *out = &ss;
+    return POS_OK;
+}
+
 // d_cands: 16-byte records, or 24-byte records when per_stage_tp.
 pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_t n,
                        int32_t *d_T, uint8_t *d_F, cudaStream_t stream) {
@@ -438,29 +468,45 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
         }
         if (e == cudaSuccess) st = launch_decode(p, stream);
         if (e == cudaSuccess && st == POS_OK) {
-            if (p.lay.sched == POS_SCHED_EAGER_1F1B) {
-                if ((st = eval_eager_1_6(p, stream)) == POS_OK &&
-                    (st = eval_eager_7_10(p, stream)) == POS_OK &&
-                    (st = eval_eager_11_13(p, stream)) == POS_OK &&
-                    (st = eval_eager_14_16(p, stream)) == POS_OK &&
-                    (st = eval_eager_short_2_8(p, stream)) == POS_OK &&
-                    (st = eval_eager_short_9_10(p, stream)) == POS_OK &&
-                    (st = eval_eager_short_11_12(p, stream)) == POS_OK &&
-                    (st = eval_eager_short_13_13(p, stream)) == POS_OK &&
-                    (st = eval_eager_short_14_14(p, stream)) == POS_OK &&
-                    (st = eval_eager_short_15_15(p, stream)) == POS_OK)
-                    st = eval_eager_short_16_16(p, stream);
-            } else if ((st = eval_fast_1_4(p, stream)) == POS_OK &&
-                       (st = eval_fast_5_8(p, stream)) == POS_OK &&
-                       (st = eval_fast_9_12(p, stream)) == POS_OK &&
-                       (st = eval_fast_13_16(p, stream)) == POS_OK &&
-                       (st = eval_generic_2_8(p, stream)) == POS_OK &&
-                       (st = eval_generic_9_12(p, stream)) == POS_OK &&
-                       (st = eval_generic_13_14(p, stream)) == POS_OK &&
-                       (st = eval_generic_15_15(p, stream)) == POS_OK) {
-                st = eval_generic_16_16(p, stream);
+            SideStream *ss = nullptr;
+            st = side_stream(&ss);
+            if (st == POS_OK) {
+                std::lock_guard<std::mutex> lock(ss->mu);
+                // fork: the short-path kernels on the side stream, after the decode pass
+                e = cudaEventRecord(ss->fork, stream);
+                if (e == cudaSuccess) e = cudaStreamWaitEvent(ss->s, ss->fork, 0);
+                if (e == cudaSuccess) {
+                    const cudaStream_t side = ss->s;
+                    if (p.lay.sched == POS_SCHED_EAGER_1F1B) {
+                        if ((st = eval_eager_short_2_8(p, side)) == POS_OK &&
+                            (st = eval_eager_short_9_10(p, side)) == POS_OK &&
+                            (st = eval_eager_short_11_12(p, side)) == POS_OK &&
+                            (st = eval_eager_short_13_13(p, side)) == POS_OK &&
+                            (st = eval_eager_short_14_14(p, side)) == POS_OK &&
+                            (st = eval_eager_short_15_15(p, side)) == POS_OK &&
+                            (st = eval_eager_short_16_16(p, side)) == POS_OK &&
+                            (st = eval_eager_1_6(p, stream)) == POS_OK &&
+                            (st = eval_eager_7_10(p, stream)) == POS_OK &&
+                            (st = eval_eager_11_13(p, stream)) == POS_OK)
+                            st = eval_eager_14_16(p, stream);
+                    } else if ((st = eval_generic_2_8(p, side)) == POS_OK &&
+                               (st = eval_generic_9_12(p, side)) == POS_OK &&
+                               (st = eval_generic_13_14(p, side)) == POS_OK &&
+                               (st = eval_generic_15_15(p, side)) == POS_OK &&
+                               (st = eval_generic_16_16(p, side)) == POS_OK &&
+                               (st = eval_fast_1_4(p, stream)) == POS_OK &&
+                               (st = eval_fast_5_8(p, stream)) == POS_OK &&
+                               (st = eval_fast_9_12(p, stream)) == POS_OK) {
+                        st = eval_fast_13_16(p, stream);
+                    }
+                    // join, also after a failed launch (the side stream's
+                    // queued work stays ordered before the scratch is freed)
+                    cudaError_t ej = cudaEventRecord(ss->join, side);
+                    if (ej == cudaSuccess) ej = cudaStreamWaitEvent(stream, ss->join, 0);
+                    if (e == cudaSuccess) e = ej;
+                }
             }
-            if (st == POS_OK && il) st = eval_interleaved(p, stream);
+            if (e == cudaSuccess && st == POS_OK && il) st = eval_interleaved(p, stream);
         }
         const cudaError_t e2 = cudaFreeAsync(scratch, stream);
         if (e != cudaSuccess) return cuda_fail(e, "eval sort launch");
