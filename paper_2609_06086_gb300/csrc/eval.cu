@@ -351,9 +351,12 @@ static pos_status scratch_pool(cudaMemPool_t *out) {
 }
 
 // A second stream per device for the short-path kernels (M < S under 1F1B,
-// M < 2S-1 under Eager 1F1B): they depend only on the decode pass, like the
-// fast-path kernels, and are bound by instruction fetch rather than by the
-// ALU, so they run beside the fast-path kernels instead of after them.  The
+// M < 2S-1 under Eager 1F1B) and then the smallest fast-path range: every
+// evaluation kernel depends only on the decode pass, and the short paths are
+// bound by instruction fetch rather than by the ALU, so they run beside the
+// other fast-path kernels instead of after them (measured: the side chain
+// with the smallest fast range was faster than the short paths alone, two
+// chains splitting the fast ranges slower).  The
 // fork and join events are shared per device, so a call holds the device's
 // side mutex from the fork to the join (two calls from different host
 // threads must not interleave their record / wait pairs).
@@ -472,7 +475,7 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
             st = side_stream(&ss);
             if (st == POS_OK) {
                 std::lock_guard<std::mutex> lock(ss->mu);
-                // fork: the short-path kernels on the side stream, after the decode pass
+                // fork: the side chain starts after the decode pass
                 e = cudaEventRecord(ss->fork, stream);
                 if (e == cudaSuccess) e = cudaStreamWaitEvent(ss->s, ss->fork, 0);
                 if (e == cudaSuccess) {
@@ -485,7 +488,7 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
                             (st = eval_eager_short_14_14(p, side)) == POS_OK &&
                             (st = eval_eager_short_15_15(p, side)) == POS_OK &&
                             (st = eval_eager_short_16_16(p, side)) == POS_OK &&
-                            (st = eval_eager_1_6(p, stream)) == POS_OK &&
+                            (st = eval_eager_1_6(p, side)) == POS_OK &&
                             (st = eval_eager_7_10(p, stream)) == POS_OK &&
                             (st = eval_eager_11_13(p, stream)) == POS_OK)
                             st = eval_eager_14_16(p, stream);
@@ -494,7 +497,7 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
                                (st = eval_generic_13_14(p, side)) == POS_OK &&
                                (st = eval_generic_15_15(p, side)) == POS_OK &&
                                (st = eval_generic_16_16(p, side)) == POS_OK &&
-                               (st = eval_fast_1_4(p, stream)) == POS_OK &&
+                               (st = eval_fast_1_4(p, side)) == POS_OK &&
                                (st = eval_fast_5_8(p, stream)) == POS_OK &&
                                (st = eval_fast_9_12(p, stream)) == POS_OK) {
                         st = eval_fast_13_16(p, stream);
