@@ -176,14 +176,18 @@ pos_status poseidon_tables_destroy(void *handle);
  * (Sec. 3.2).  d_cands (16-byte aligned), d_makespan (int32[n]) and
  * d_feasible (uint8[n]) are DEVICE pointers on the handle's device; outputs
  * are in input order; the call is asynchronous on `stream` (a cudaStream_t,
- * NULL = legacy default stream) and returns after the launches.  Infeasible
+ * NULL = legacy default stream) and returns after the launches.  Part of the
+ * work runs on a library-owned second stream of the device, forked from
+ * `stream` after the sort and joined back into it before the call's last
+ * operation, so every effect is still ordered after earlier work on
+ * `stream` and before later work on it.  Infeasible
  * plans still get their makespan.  Scratch: the batch is counting-sorted by
  * (S, M) (and by (N, V, M/N) for interleaved records) and decoded into a
  * 38*n + 56 KB (Interleaved 1F1B: 38*n + 121 KB) stream-ordered allocation
- * (decoded record 32 B, permutation 4 B and sort key 2 B per candidate, key
- * histograms) from a library-owned memory pool (per device, kept between
- * calls); batches above 2^24 candidates go in chunks of 2^24, one after
- * another.
+ * (decoded record 32 B, sorted position 4 B and sort key 2 B per candidate,
+ * key histograms) from a library-owned memory pool (per device, kept
+ * between calls); batches above 2^24 candidates go in chunks of 2^24, one
+ * after another.
  * Errors: POS_EINVAL (null handle or pointers, n < 0, misaligned
  * candidates), POS_ENOMEM, POS_ECUDA (launch failure).
  */
