@@ -351,12 +351,13 @@ static pos_status scratch_pool(cudaMemPool_t *out) {
 }
 
 // A second stream per device for the short-path kernels (M < S under 1F1B,
-// M < 2S-1 under Eager 1F1B) and then the smallest fast-path range: every
-// evaluation kernel depends only on the decode pass, and the short paths are
-// bound by instruction fetch rather than by the ALU, so they run beside the
-// other fast-path kernels instead of after them (measured: the side chain
-// with the smallest fast range was faster than the short paths alone, two
-// chains splitting the fast ranges slower).  The
+// M < 2S-1 under Eager 1F1B) and then the smallest fast-path range (under
+// Interleaved 1F1B: every 1F1B range, then the smallest interleaved range):
+// every evaluation kernel depends only on the decode pass, and the short
+// paths are bound by instruction fetch rather than by the ALU, so they run
+// beside the other fast-path kernels instead of after them (measured: the
+// side chain with the smallest fast range was faster than the short paths
+// alone, two chains splitting the fast ranges slower).  The
 // fork and join events are shared per device, so a call holds the device's
 // side mutex from the fork to the join (two calls from different host
 // threads must not interleave their record / wait pairs).
@@ -492,6 +493,24 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
                             (st = eval_eager_7_10(p, stream)) == POS_OK &&
                             (st = eval_eager_11_13(p, stream)) == POS_OK)
                             st = eval_eager_14_16(p, stream);
+                    } else if (il) {
+                        // interleaved handle: the 1F1B ranges (records with
+                        // V < 2, usually none) and the smallest interleaved
+                        // range on the side, the other interleaved ranges here
+                        if ((st = eval_generic_2_8(p, side)) == POS_OK &&
+                            (st = eval_generic_9_12(p, side)) == POS_OK &&
+                            (st = eval_generic_13_14(p, side)) == POS_OK &&
+                            (st = eval_generic_15_15(p, side)) == POS_OK &&
+                            (st = eval_generic_16_16(p, side)) == POS_OK &&
+                            (st = eval_fast_1_4(p, side)) == POS_OK &&
+                            (st = eval_fast_5_8(p, side)) == POS_OK &&
+                            (st = eval_fast_9_12(p, side)) == POS_OK &&
+                            (st = eval_fast_13_16(p, side)) == POS_OK &&
+                            (st = eval_il_30_31(p, side)) == POS_OK &&
+                            (st = eval_il_0_11(p, stream)) == POS_OK &&
+                            (st = eval_il_12_22(p, stream)) == POS_OK &&
+                            (st = eval_il_23_29(p, stream)) == POS_OK)
+                            st = eval_il_32_33(p, stream);
                     } else if ((st = eval_generic_2_8(p, side)) == POS_OK &&
                                (st = eval_generic_9_12(p, side)) == POS_OK &&
                                (st = eval_generic_13_14(p, side)) == POS_OK &&
@@ -509,7 +528,6 @@ pos_status launch_eval(Handle *h, const void *d_cands, bool per_stage_tp, int64_
                     if (e == cudaSuccess) e = ej;
                 }
             }
-            if (e == cudaSuccess && st == POS_OK && il) st = eval_interleaved(p, stream);
         }
         const cudaError_t e2 = cudaFreeAsync(scratch, stream);
         if (e != cudaSuccess) return cuda_fail(e, "eval sort launch");
