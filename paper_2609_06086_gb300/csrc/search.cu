@@ -873,6 +873,9 @@ pos_status get_workspace(Workspace **out) {
         cudaError_t e = cudaStreamCreateWithFlags(&w->stream, cudaStreamNonBlocking);
         for (int i = 0; i < 3 && e == cudaSuccess; ++i) e = cudaEventCreate(&w->ev[i]);
         if (e == cudaSuccess) e = cudaEventCreateWithFlags(&w->ev_lb, cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&w->side, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&w->ev_fork, cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&w->ev_join, cudaEventDisableTiming);
         if (e == cudaSuccess) e = cudaMallocHost(&w->h_cnt, 64 * sizeof(unsigned long long));
         if (e != cudaSuccess) {
             delete w;
@@ -1286,7 +1289,8 @@ static ExpandParams base_params(Search &s, const SliceRec *batch, int M) {
 }
 
 static pos_status run_leaves(Search &s, const Leaf *leaves, unsigned long long *count,
-                             const SliceRec *table, int M, unsigned long long *slice_best) {
+                             const SliceRec *table, int M, unsigned long long *slice_best,
+                             cudaStream_t stream = nullptr) {
     LeafParams lp;
     lp.leaves = leaves;
     lp.count = count;
@@ -1305,7 +1309,8 @@ static pos_status run_leaves(Search &s, const Leaf *leaves, unsigned long long *
     lp.cas_limit = s.pb->cas_limit == 0 ? kCasLimit : std::max(0, s.pb->cas_limit);
     // as many blocks as the launch bounds keep resident on every SM
     const int path = path_of(s.pb->schedule, s.S, M);
-    return launch_leaf(s.S, path, lp, leaf_min_blocks(s.S, path) * sm_count(), s.stream);
+    return launch_leaf(s.S, path, lp, leaf_min_blocks(s.S, path) * sm_count(),
+                       stream ? stream : s.stream);
 }
 
 template <bool COMPLETE, int X>
@@ -1438,6 +1443,9 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
     const int n_slices = (int)n_slices64;
     if (s.n_map && n_slices64 > ~0ull / s.n_map) return fail(POS_EINVAL, "global index overflows");
     if ((st = schedule_programs(p->schedule, &s.pg)) != POS_OK) return st;
+    // after the side-stream work of an earlier search (which may have
+    // returned early), since this one reuses its buffers
+    POS_CUDA(cudaStreamWaitEvent(s.stream, s.ws.ev_join, 0));
     // pinned staging for this search's uploads (tables, slice records, lists)
     if ((st = reserve_stage(s, ((size_t)256 << 10) + (size_t)n_slices * 320 +
                                    (size_t)p->n_M * 16)) != POS_OK)
@@ -1548,16 +1556,21 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         if (p->profile) POS_CUDA(cudaEventRecord(s.ev[1], s.stream));
         s.launches++;
         s.n_bound++;
-        // the greedy plans of each M index (holes for the infeasible slices)
+        // the greedy plans of each M index (holes for the infeasible slices),
+        // on the side stream: they only lower the incumbent, which the
+        // enumeration reads after the join below
         std::vector<unsigned long long> gc(p->n_M, (unsigned long long)sp.per_m);
         POS_CUDA(s.ws.d_wcnt.reserve(sizeof(unsigned long long) * p->n_M));
         POS_TRY(upload(s, s.ws.d_wcnt.p, gc.data(), sizeof(unsigned long long) * p->n_M));
+        POS_CUDA(cudaEventRecord(s.ws.ev_fork, s.stream));
+        POS_CUDA(cudaStreamWaitEvent(s.ws.side, s.ws.ev_fork, 0));
         for (int mi = 0; mi < p->n_M; ++mi)
             if ((st = run_leaves(s, static_cast<const Leaf *>(s.ws.d_greedy.p) + mi * sp.per_m,
                                  static_cast<unsigned long long *>(s.ws.d_wcnt.p) + mi, d_all,
-                                 p->M_list[mi], static_cast<unsigned long long *>(s.d_best.p))) !=
-                POS_OK)
+                                 p->M_list[mi], static_cast<unsigned long long *>(s.d_best.p),
+                                 s.ws.side)) != POS_OK)
                 return st;
+        POS_CUDA(cudaEventRecord(s.ws.ev_join, s.ws.side));
         if ((size_t)n_slices > s.ws.h_lb_cap) {
             POS_CUDA(cudaStreamSynchronize(s.stream));  // no copy into the old area in flight
             if (s.ws.h_lb) cudaFreeHost(s.ws.h_lb);
@@ -1667,6 +1680,9 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
             warm_evals += (uint64_t)n_s;
         }
     }
+    // the greedy plans' makespans (side stream) before anything that reads
+    // the incumbent or the per-slice bests
+    POS_CUDA(cudaStreamWaitEvent(s.stream, s.ws.ev_join, 0));
     // slice order: with the completion bounds, by each slice's root lower
     // bound (the slice most likely to hold the optimum first), waiting for
     // their copy only; otherwise by the best warm-up plan of the slice,

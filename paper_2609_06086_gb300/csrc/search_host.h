@@ -62,6 +62,11 @@ struct Workspace {
     unsigned long long *h_lb = nullptr;        // pinned landing area of the root bounds
     size_t h_lb_cap = 0;                       // (elements)
     cudaEvent_t ev_lb = nullptr;               // recorded after their copy
+    // second stream for the greedy plans' makespans (forked after the bound
+    // kernel, joined before the enumeration), so that they run while the
+    // host reads the root bounds and plans the batches
+    cudaStream_t side = nullptr;
+    cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
     std::vector<cudaEvent_t> evs;              // timing events of the batch pipelines
 };
 

@@ -753,6 +753,9 @@ pos_status search_interleaved(Workspace &ws, const pos_problem *p, const SliceSp
     for (int i = 0; i < p->n_M; ++i)
         if (p->M_list[i] % N == 0 && guard_trips(gA, gD, gP, r.J, p->M_list[i]))
             return fail(POS_EOVERFLOW, "makespan bound reaches 2^31 for some M");
+    // after the side-stream work of an earlier search, whose buffers this
+    // one reuses
+    POS_CUDA(cudaStreamWaitEvent(r.st, ws.ev_join, 0));
     POS_CUDA(ws.blob.reserve(r.lay.bytes));
     r.blob = ws.blob.p;
     POS_CUDA(cudaMemcpyAsync(r.blob, host.data(), r.lay.bytes, cudaMemcpyHostToDevice, r.st));
