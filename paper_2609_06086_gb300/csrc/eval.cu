@@ -57,13 +57,15 @@ __global__ void argmin_final(const int32_t *part_t, const long long *part_i, int
 // ---------------------------------------------------------------------------
 // counting sort of the candidates by (S, M) key
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ int eval_key(int sched, uint32_t w) {
+// il_key: kIlKeyOf staged in shared memory (a __constant__ read whose index
+// differs between the lanes of a warp is served one address at a time)
+__device__ __forceinline__ int eval_key(int sched, uint32_t w, const int16_t *il_key) {
     const int S = w & 0xff, M = (w >> 8) & 0xff, V = (int)(w >> 24);
     if (S < 1 || S > POS_MAX_STAGES || M < 1) return -1;
     if (sched == POS_SCHED_INTERLEAVED_1F1B && V >= 2) {
         // N = S devices, V chunks each: key block of (N, V), index q = M / N
         if (S * V > POS_MAX_STAGES || M % S != 0) return -1;
-        return kKeys + kIlKeyOf[S - 1][V] + M / S;
+        return kKeys + il_key[(S - 1) * 17 + V] + M / S;
     }
     return M >= fast_min_m(sched, S) ? fast_key_begin(S) + M : generic_key_begin(S) + M;
 }
@@ -88,7 +90,10 @@ __global__ void sort_hist_kernel(EvalParams p, int64_t n, uint32_t *hist, uint16
                                  int32_t *T, uint8_t *F) {
     const int sched = p.lay.sched;
     __shared__ uint32_t h[NK];
+    __shared__ int16_t il_key[8 * 17];
     for (int i = threadIdx.x; i < NK; i += blockDim.x) h[i] = 0;
+    if (sched == POS_SCHED_INTERLEAVED_1F1B)
+        for (int i = threadIdx.x; i < 8 * 17; i += blockDim.x) il_key[i] = kIlKeyOf[i / 17][i % 17];
     __syncthreads();
     // four record words in flight per thread (the pass is bound by HBM
     // latency: one load per thread and iteration kept too few bytes in flight)
@@ -101,7 +106,7 @@ __global__ void sort_hist_kernel(EvalParams p, int64_t n, uint32_t *hist, uint16
         for (int u = 0; u < 4; ++u) {
             const int64_t i = i0 + u * bd;
             if (i >= n) break;
-            const int k = eval_key(sched, wv[u]);
+            const int k = eval_key(sched, wv[u], il_key);
             keys[i] = k >= 0 ? (uint16_t)k : kNoKey;
             if (k >= 0) {
                 atomicAdd(&h[k], 1u);
