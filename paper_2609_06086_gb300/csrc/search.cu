@@ -1564,13 +1564,14 @@ static pos_status search_impl(Search &s, pos_plan *out, pos_search_stats *stats)
         POS_TRY(upload(s, s.ws.d_wcnt.p, gc.data(), sizeof(unsigned long long) * p->n_M));
         POS_CUDA(cudaEventRecord(s.ws.ev_fork, s.stream));
         POS_CUDA(cudaStreamWaitEvent(s.ws.side, s.ws.ev_fork, 0));
-        for (int mi = 0; mi < p->n_M; ++mi)
-            if ((st = run_leaves(s, static_cast<const Leaf *>(s.ws.d_greedy.p) + mi * sp.per_m,
-                                 static_cast<unsigned long long *>(s.ws.d_wcnt.p) + mi, d_all,
-                                 p->M_list[mi], static_cast<unsigned long long *>(s.d_best.p),
-                                 s.ws.side)) != POS_OK)
-                return st;
+        for (int mi = 0; mi < p->n_M && st == POS_OK; ++mi)
+            st = run_leaves(s, static_cast<const Leaf *>(s.ws.d_greedy.p) + mi * sp.per_m,
+                            static_cast<unsigned long long *>(s.ws.d_wcnt.p) + mi, d_all,
+                            p->M_list[mi], static_cast<unsigned long long *>(s.d_best.p),
+                            s.ws.side);
+        // recorded also after a failed launch: the next search waits on it
         POS_CUDA(cudaEventRecord(s.ws.ev_join, s.ws.side));
+        if (st != POS_OK) return st;
         if ((size_t)n_slices > s.ws.h_lb_cap) {
             POS_CUDA(cudaStreamSynchronize(s.stream));  // no copy into the old area in flight
             if (s.ws.h_lb) cudaFreeHost(s.ws.h_lb);
